@@ -1,0 +1,393 @@
+#!/usr/bin/env python3
+"""Benchmark of the CompressKV prefill KV-compression step on GB300.
+
+One step = ckv_compress_layer (score + pool + top-k + gather) for every layer of the
+Llama-3.1-8B-shaped workload (32 layers, 32 query / 8 KV heads, d = 128, one sequence of 8192
+prefix tokens, w = 32, 2 selected heads per group, max-pool 7, layer budgets summing to
+32 x 256), on synthetic seeded inputs already resident in HBM.  Each layer has its own K/V/Q
+buffers, so one step streams 1.07 GB (far more than the 129 MB L2); the step is replayed from a
+CUDA graph.
+
+Prints one JSON line (rank 0).  `--impl reference` times the fp64 CPU oracle instead (the
+reference arm of this build), on bounded samples of the same workload.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "KV-compress prefix tokens/s per layer (score+topk+gather); % of HBM peak"
+UNIT = "prefix tokens/s per layer"
+WORKLOAD = "llama8b_l8192"
+HBM_FALLBACK_GBS = 6800.0
+
+# dram__bytes_read.sum + dram__bytes_write.sum per launch pair of the scoring stage, from the
+# ncu capture summarised in profiles/, keyed by the sha256 of the kernel source it was taken on.
+SCORE_TRAFFIC = {}
+
+
+def _args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--workload", default=WORKLOAD)
+    ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    return ap.parse_args()
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return HBM_FALLBACK_GBS, "fallback"
+
+
+def _dist():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+# ----------------------------------------------------------------------------- clocks
+_REASONS = {0x1: "gpu_idle", 0x2: "applications_clocks_setting", 0x4: "sw_power_cap",
+            0x8: "hw_slowdown", 0x10: "sync_boost", 0x20: "sw_thermal_slowdown",
+            0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown",
+            0x100: "display_clock_setting"}
+
+
+class ClockSampler:
+    def __init__(self, device_index: int):
+        self.path = tempfile.mktemp(prefix="ckv_clocks_", suffix=".csv")
+        self.dev = device_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.dev),
+                 "--query-gpu=clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active",
+                 "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=self.f, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            time.sleep(0.1)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+            self.f.close()
+
+    def summary(self):
+        rows = []
+        try:
+            for line in open(self.path):
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 4:
+                    continue
+                try:
+                    rows.append((float(parts[0]), float(parts[1]), float(parts[2]), int(parts[3], 16)))
+                except ValueError:
+                    continue
+        finally:
+            try:
+                os.unlink(self.path)
+            except OSError:
+                pass
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        busy = [r for r in rows if not (r[3] & 0x1)] or rows
+        reasons = sorted({name for r in busy for bit, name in _REASONS.items()
+                          if r[3] & bit and bit != 0x1})
+        return {"sm_mhz": statistics.median(r[0] for r in busy), "sm_max_mhz": max(r[1] for r in rows),
+                "power_w_max": max(r[2] for r in rows), "reasons": reasons, "samples": len(busy)}
+
+
+# ----------------------------------------------------------------------------- our arm
+def run_ours(args):
+    import numpy as np
+    import torch
+
+    import ckv_synth as cs
+    import __graft_entry__ as entry
+
+    rank, world, local = _dist()
+    torch.cuda.set_device(local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    entry.build()
+    import paper_2508_02401_gb300 as ckv
+
+    wl = cs.workload(args.workload)
+    cfg = ckv.Config.from_workload(wl)
+    batch = ckv.Batch(wl.cu_seqlens(), device=f"cuda:{local}")
+    T, Hkv, nl = wl.total_tokens, wl.num_kv_heads, wl.num_layers
+
+    def dev(bits):
+        return torch.from_numpy(bits.view(np.int16)).cuda().view(torch.bfloat16)
+
+    layers = []
+    host_layers = []
+    for l in range(nl):
+        li = wl.layer(l)
+        host_layers.append(li)
+        idx, cu_keep_dev, k_out, v_out, cu_keep = ckv.new_outputs(cfg, l, batch)
+        layers.append(dict(q=dev(li.q_win), k=dev(li.k), v=dev(li.v), idx=idx, cu_keep_dev=cu_keep_dev,
+                           k_out=k_out, v_out=v_out, t_keep=int(cu_keep[-1])))
+    ws_bytes = max(ckv.ckv_workspace_size(cfg, l, batch) for l in range(nl))
+    ws = torch.zeros(ws_bytes, dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.Stream()
+
+    def step():
+        for l, d in enumerate(layers):
+            ckv.ckv_compress_layer(cfg, l, batch, d["q"], d["k"], d["v"], d["idx"], d["cu_keep_dev"],
+                                   d["k_out"], d["v_out"], ws, stream=stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(max(1, args.warmup)):
+            step()
+    torch.cuda.synchronize()
+    code, detail = ckv.ckv_read_device_status(ws, stream=stream)
+    if code != 0:
+        raise RuntimeError(f"device status {code} ({detail}) after warm-up")
+
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        step()
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            graph.replay()
+    torch.cuda.synchronize()
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        barrier()
+        torch.cuda.synchronize()
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(args.steps):
+                graph.replay()
+            e1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+    ms = e0.elapsed_time(e1)
+    clocks = clk.summary()
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    code, detail = ckv.ckv_read_device_status(ws, stream=stream)
+    if code != 0:
+        raise RuntimeError(f"device status {code} ({detail}) after the timed region")
+    ms_per_step = ms / args.steps
+    value = world * nl * T / (ms_per_step / 1e3)
+
+    launches_per_step = 0
+    for l, d in enumerate(layers):
+        launches_per_step += 4 + (1 if d["t_keep"] > 0 else 0)
+
+    # --- scoring stage (the dominant kernels): per-layer event timing on its stream
+    hbm_peak, peak_kind = _peaks()
+    score_rows = torch.empty((int(cfg.head_mask[0].sum()), T), dtype=torch.float32, device="cuda")
+    reps = 5
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(reps * nl)]
+    with torch.cuda.stream(stream):
+        for l, d in enumerate(layers):  # warm
+            ckv.ckv_score_window(cfg, l, batch, d["q"], d["k"], score_rows, ws, stream=stream)
+        for r in range(reps):
+            for l, d in enumerate(layers):
+                a, b = ev[r * nl + l]
+                a.record(stream)
+                ckv.ckv_score_window(cfg, l, batch, d["q"], d["k"], score_rows, ws, stream=stream)
+                b.record(stream)
+    torch.cuda.synchronize()
+    score_ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
+    k_bytes = T * Hkv * 256
+    score_gbs = k_bytes / (score_ms / 1e3) / 1e9
+    src = open(os.path.join(ROOT, "paper_2508_02401_gb300", "csrc", "score_kernel.cu"), "rb").read()
+    traffic = SCORE_TRAFFIC.get(hashlib.sha256(src).hexdigest())
+    roofline = {"bound": "hbm", "kernel": "score_window (pass 1 + pass 2, one layer)",
+                "achieved": round(score_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
+                "frac": round(score_gbs / hbm_peak, 4), "peak_kind": peak_kind,
+                "traffic": traffic, "algorithmic_bytes_per_launch": k_bytes,
+                "avg_launch_us": round(score_ms * 1e3, 2)}
+    keep_bytes = sum(4 * 256 * Hkv * d["t_keep"] for d in layers) / nl
+    layer_bytes = k_bytes + keep_bytes
+    layer_gbs = layer_bytes / (ms_per_step / nl / 1e3) / 1e9
+
+    # --- end to end through the public API from pinned host memory
+    e2e = None
+    if args.e2e_steps > 0:
+        hq = [torch.from_numpy(h.q_win.view(np.int16)).view(torch.bfloat16).pin_memory() for h in host_layers]
+        hk = [torch.from_numpy(h.k.view(np.int16)).view(torch.bfloat16).pin_memory() for h in host_layers]
+        hv = [torch.from_numpy(h.v.view(np.int16)).view(torch.bfloat16).pin_memory() for h in host_layers]
+        oi = [torch.empty(d["idx"].shape, dtype=torch.int32, pin_memory=True) for d in layers]
+        ok = [torch.empty(d["k_out"].shape, dtype=torch.bfloat16, pin_memory=True) for d in layers]
+        ov = [torch.empty(d["v_out"].shape, dtype=torch.bfloat16, pin_memory=True) for d in layers]
+        h2d = sum(x.numel() * 2 for x in hq + hk + hv)
+        d2h = sum(x.numel() * x.element_size() for x in oi + ok + ov)
+
+        def e2e_step():
+            for l, d in enumerate(layers):
+                d["q"].copy_(hq[l], non_blocking=True)
+                d["k"].copy_(hk[l], non_blocking=True)
+                d["v"].copy_(hv[l], non_blocking=True)
+                ckv.ckv_compress_layer(cfg, l, batch, d["q"], d["k"], d["v"], d["idx"],
+                                       d["cu_keep_dev"], d["k_out"], d["v_out"], ws, stream=stream)
+                oi[l].copy_(d["idx"], non_blocking=True)
+                ok[l].copy_(d["k_out"], non_blocking=True)
+                ov[l].copy_(d["v_out"], non_blocking=True)
+
+        with torch.cuda.stream(stream):
+            for _ in range(2):
+                e2e_step()
+            torch.cuda.synchronize()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            for _ in range(args.e2e_steps):
+                e2e_step()
+            b.record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = a.elapsed_time(b) / args.e2e_steps
+        e2e = {"value": world * nl * T / (e2e_ms / 1e3), "unit": UNIT, "ms_per_step": round(e2e_ms, 4),
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+
+    cpu = None
+    if rank == 0 and world == 1 and args.cpu_seconds > 0:
+        cpu = _cpu_baseline(wl, host_layers, args.cpu_seconds)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 5),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic",
+            "config": {"workload": wl.name, "layers": nl, "seq_len": T, "q_heads": wl.num_q_heads,
+                       "kv_heads": Hkv, "head_dim": 128, "window": wl.window,
+                       "heads_per_group": wl.heads_per_group, "pool": f"{wl.pool_type}{wl.pool_kernel}",
+                       "budget_total": int(wl.budgets().sum()), "parallelism": f"replicas{world}",
+                       "l2": "inputs larger than L2 (distinct per-layer buffers, 1.07 GB per step)",
+                       "graph": "one CUDA graph per step"},
+            "roofline": roofline,
+            "layer_roofline": {"bound": "hbm", "achieved": round(layer_gbs, 1), "peak": hbm_peak,
+                               "unit": "GB/s", "frac": round(layer_gbs / hbm_peak, 4),
+                               "frac_of_8TBs": round(layer_gbs / 8000.0, 4),
+                               "algorithmic_bytes_per_layer": int(layer_bytes)},
+            "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks,
+            "gpu_launches": launches_per_step * args.steps,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+# ----------------------------------------------------------------------------- the oracle
+def _cpu_baseline(wl, host_layers, seconds):
+    """The fp64 oracle as it stands, whole layers in order until `seconds` have passed."""
+    import oracle
+    oracle.build()
+    cores = oracle.threads(0)
+    t0 = time.perf_counter()
+    done = 0
+    for l, li in enumerate(host_layers):
+        oracle.compress_layer(li.q_win, li.k, li.v, wl.cu_seqlens(), wl.head_mask()[l],
+                              int(wl.budgets()[l]), wl.window, wl.pool_kernel,
+                              0 if wl.pool_type == "max" else 1,
+                              0 if wl.head_order == "pool_then_sum" else 1)
+        done += 1
+        if time.perf_counter() - t0 >= seconds:
+            break
+    dt = time.perf_counter() - t0
+    return {"value": round(done * wl.total_tokens / dt, 2), "unit": UNIT, "cores": cores,
+            "kind": "oracle", "sample": f"{done} of {wl.num_layers} layers, whole layers, "
+                                        f"{dt:.1f} s, OpenMP over (sequence, KV head)"}
+
+
+def run_reference(args):
+    rank, world, local = _dist()
+    if rank != 0:
+        return
+    import ckv_synth as cs
+    import oracle
+    oracle.build()
+    wl = cs.workload(args.workload)
+    cores = oracle.threads(0)
+    li_cache = {}
+
+    def sample(i):
+        l = i % wl.num_layers
+        if l not in li_cache:
+            li_cache.clear()
+            li_cache[l] = wl.layer(l)
+        li = li_cache[l]
+        g = (i // wl.num_layers) % wl.num_kv_heads
+        oracle.compress_layer(li.q_win, li.k, li.v, wl.cu_seqlens(), wl.head_mask()[l],
+                              int(wl.budgets()[l]), wl.window, wl.pool_kernel,
+                              0 if wl.pool_type == "max" else 1,
+                              0 if wl.head_order == "pool_then_sum" else 1, groups=[g])
+
+    for i in range(args.warmup):
+        sample(i)
+    times = []
+    for i in range(args.steps):
+        t = time.perf_counter()
+        sample(args.warmup + i)
+        times.append(time.perf_counter() - t)
+    per_unit = statistics.mean(times)
+    value = wl.total_tokens / (per_unit * wl.num_kv_heads)  # a layer = H_kv (seq, head) units
+    line = {"impl": "reference", "metric": METRIC, "value": round(value, 2), "unit": UNIT,
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(per_unit * 1e3, 3), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": wl.name, "layers": wl.num_layers, "seq_len": wl.total_tokens,
+                       "parallelism": "host cores"},
+            "cpu_baseline": {"value": round(value, 2), "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": "one (layer, KV head) unit of the workload per step"},
+            "e2e": {"value": round(value, 2), "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = _args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,175 @@
+/*
+ * ckv.h -- C ABI of libckv, a GB300 (sm_103a) implementation of CompressKV's prefill-time
+ * KV-cache compression step (arxiv 2508.02401, Sec. 3.3 and Fig. 3, token selection by the
+ * semantic retrieval heads; attention as in Eq. 2; pooling hyper-parameters from App. A).
+ *
+ * For one transformer layer and every GQA KV head g, the step
+ *   1. scores every prefix token j by the attention that the observation window (the last w
+ *      query rows) of the layer's selected heads in group g pays to it:
+ *        a_h[j] = sum_r softmax_j(scale * q_{h,r} . k_{g,j}),  row r sees keys j <= L - w + r;
+ *   2. smooths a_h along the token axis with a 1-D pool and combines the selected heads;
+ *   3. keeps the top (B_l - w) candidate positions j < L - w (B_l = the layer's budget) plus
+ *      the w window positions, in ascending order (every position when L <= B_l);
+ *   4. gathers the kept K/V rows into a compacted, position-ordered cache.
+ *
+ * Conventions shared by every entry point
+ *   - Pointers named *_dev and all tensor arguments are DEVICE memory of the current CUDA
+ *     device; pointers named *_host and the config's head mask / budgets are HOST memory.
+ *   - Tensors are bfloat16 unless stated; head_dim is 128.  Layouts, row-major:
+ *       q_win  [S, w, H_q, 128]       the last w query rows of every sequence (packed)
+ *       k, v   [T, H_kv, 128]         varlen-packed by cu_seqlens; element (t, g, c) lives at
+ *                                     t*tok_stride + g*head_stride + c (strides in elements,
+ *                                     0 = packed: tok_stride = H_kv*128, head_stride = 128)
+ *       scores [n_sel, T]   fp32      one row per selected head of the layer, in ascending
+ *                                     query-head order (so grouped by KV head)
+ *       pooled [H_kv, T]    fp32      combined, pooled scores on candidate positions; 0 at the
+ *                                     window positions
+ *       idx    [H_kv, T_keep] int32   kept sequence-local positions; the positions of sequence
+ *                                     s for head g are idx[g*T_keep + cu_keep[s] ...]
+ *       k_out, v_out [T_keep, H_kv, 128]  packed
+ *     with T = cu_seqlens[S], T_keep = sum_s min(B_l, L_s).
+ *   - The caller owns every buffer.  The library allocates no device or host memory during a
+ *     call and keeps no per-call state; all work is enqueued asynchronously on `stream`
+ *     (NULL = the legacy default stream).  Only ckv_read_device_status synchronises.
+ *   - Argument errors are detected on the host before anything is enqueued and leave every
+ *     output untouched.  No entry point aborts, exits or throws.  Errors that only the device
+ *     can see (cu_seqlens_dev disagreeing with cu_seqlens_host, a kernel wait that timed out)
+ *     are recorded in the workspace's status word and reported by ckv_read_device_status.
+ *   - Device pointers must be 16-byte aligned, the workspace 256-byte aligned.
+ *   - A workspace may be reused by calls that are ordered on one stream; calls that may run
+ *     concurrently need separate workspaces.  Zero it once (cudaMemset) before its first use.
+ */
+#ifndef CKV_H
+#define CKV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define CKV_ABI_VERSION 1
+
+#if defined(__GNUC__)
+#define CKV_API __attribute__((visibility("default")))
+#else
+#define CKV_API
+#endif
+
+typedef struct CUstream_st* ckv_stream; /* the same type as cudaStream_t */
+
+typedef enum ckv_status {
+    CKV_OK = 0,
+    CKV_ERR_INVALID_ARG = 1, /* a pointer, size, layout or config field is invalid */
+    CKV_ERR_UNSUPPORTED = 2, /* valid, but outside what this build supports (e.g. head_dim) */
+    CKV_ERR_WORKSPACE = 3,   /* workspace missing, misaligned or smaller than required */
+    CKV_ERR_CUDA = 4,        /* a CUDA runtime call failed; see ckv_last_error_message() */
+    CKV_ERR_DEVICE = 5       /* a kernel recorded an error in the workspace status word */
+} ckv_status;
+
+typedef enum ckv_pool_type { CKV_POOL_MAX = 0, CKV_POOL_AVG = 1 } ckv_pool_type;
+
+/* How the selected heads of a KV group are combined (Sec. 3.3 pools each head's window sum
+ * and then averages the vectors; averaging is replaced by summing, which ranks identically). */
+typedef enum ckv_head_order {
+    CKV_POOL_THEN_SUM = 0, /* c_g = sum_h pool(a_h)  -- the order of Sec. 3.3 */
+    CKV_SUM_THEN_POOL = 1  /* c_g = pool(sum_h a_h) */
+} ckv_head_order;
+
+/* Per-model settings.  head_mask and budgets are the paper's per-layer head-selection mask
+ * (Sec. 3.3, top Semantic Retrieval Heads per layer, Eq. 5) and per-layer budgets (Sec. 3.4,
+ * Algorithm 1); both stay in host memory and are read during each call. */
+typedef struct ckv_config {
+    int32_t num_layers;
+    int32_t num_q_heads;   /* H_q, a multiple of num_kv_heads; at most 256 */
+    int32_t num_kv_heads;  /* H_kv; query head h belongs to KV head h / (H_q / H_kv) */
+    int32_t head_dim;      /* must be 128 */
+    int32_t window;        /* w, observation window rows, 1..64 */
+    int32_t pool_kernel;   /* odd, 1..63; 1 = no pooling */
+    int32_t pool_type;     /* ckv_pool_type: max ignores padding; avg counts zero padding and
+                              divides by pool_kernel */
+    int32_t head_order;    /* ckv_head_order */
+    float softmax_scale;   /* scale of q.k; 0 selects 1/sqrt(head_dim) */
+    const uint8_t* head_mask; /* host [num_layers * num_q_heads]; non-zero = selected.  Every
+                                 KV group of a layer needs at least one selected head. */
+    const int32_t* budgets;   /* host [num_layers]; kept tokens per KV head, window included,
+                                 >= window */
+} ckv_config;
+
+/* A varlen batch: sequence s occupies tokens [cu_seqlens[s], cu_seqlens[s+1]). */
+typedef struct ckv_batch {
+    int32_t num_seqs;               /* S >= 1 */
+    const int32_t* cu_seqlens_host; /* host   [S+1], cu[0] = 0, non-decreasing */
+    const int32_t* cu_seqlens_dev;  /* device [S+1], the same values */
+} ckv_batch;
+
+/* Version of this ABI (CKV_ABI_VERSION of the built library). */
+CKV_API int32_t ckv_abi_version(void);
+
+/* Human-readable name of a status code (static storage). */
+CKV_API const char* ckv_status_string(ckv_status status);
+
+/* Detail of the last failing call on this host thread (static thread-local storage). */
+CKV_API const char* ckv_last_error_message(void);
+
+/* Workspace bytes that every entry point below needs for (cfg, layer, batch).  Host only. */
+CKV_API ckv_status ckv_workspace_size(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
+                              size_t* bytes);
+
+/* Host only: cu_keep_host[S+1] = prefix sums of min(B_layer, L_s), and the number of score
+ * rows n_sel of the layer (may be NULL). */
+CKV_API ckv_status ckv_keep_lengths(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
+                            int32_t* cu_keep_host, int32_t* n_sel);
+
+/* Step 1 (Sec. 3.3, with the attention of Eq. 2; the window rows' probabilities are added):
+ * scores[i, t] = a_h[j] for the i-th selected head h of the layer and every token t = cu[s]+j,
+ * including window positions (there a_h[j] sums only the rows that see key j).  The softmax of
+ * window row r runs over keys 0..L-w+r (causal).  Computed for every sequence of the batch. */
+CKV_API ckv_status ckv_score_window(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
+                            const void* q_win, const void* k, int64_t tok_stride,
+                            int64_t head_stride, float* scores, void* workspace,
+                            size_t workspace_bytes, ckv_stream stream);
+
+/* Step 2 (Sec. 3.3 token-axis smoothing; App. A sizes): pooled[g, cu[s]+j] for
+ * j < L_s - w from the scores of group g's selected heads, in cfg->head_order; 0 at window
+ * positions.  Pooling runs over the candidate range only (window scores never enter it). */
+CKV_API ckv_status ckv_pool(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
+                    const float* scores, float* pooled, ckv_stream stream);
+
+/* Step 3 (Sec. 3.3, top-N selection):
+ * per (sequence, KV head), the B_l - w largest pooled candidates (ties: lower position first)
+ * followed by the window positions, ascending; every position when L_s <= B_l.  Writes idx
+ * and cu_keep_dev[S+1] (device copy of ckv_keep_lengths). */
+CKV_API ckv_status ckv_select_topk(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
+                           const float* pooled, int32_t* idx, int32_t* cu_keep_dev,
+                           void* workspace, size_t workspace_bytes, ckv_stream stream);
+
+/* Step 4 (Sec. 3.3, the kept tokens' K/V pairs form the new cache): k_out / v_out rows
+ * = the k / v rows at idx.  t_keep = cu_keep[S].  Bit copy. */
+CKV_API ckv_status ckv_gather_compact(const ckv_config* cfg, const ckv_batch* batch, int32_t t_keep,
+                              const void* k, const void* v, int64_t tok_stride,
+                              int64_t head_stride, const int32_t* idx,
+                              const int32_t* cu_keep_dev, void* k_out, void* v_out,
+                              void* workspace, size_t workspace_bytes, ckv_stream stream);
+
+/* Steps 1-4 for one layer.  Sequences with L_s <= B_l are copied whole without being scored.
+ * pooled_out may be NULL (then the pooled scores stay in the workspace). */
+CKV_API ckv_status ckv_compress_layer(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
+                              const void* q_win, const void* k, const void* v,
+                              int64_t tok_stride, int64_t head_stride, int32_t* idx,
+                              int32_t* cu_keep_dev, void* k_out, void* v_out, float* pooled_out,
+                              void* workspace, size_t workspace_bytes, ckv_stream stream);
+
+/* Synchronises `stream`, then returns the workspace's device status: *code = 0 if no kernel
+ * recorded an error since the last reset, else the first error (1 = cu_seqlens_dev disagrees
+ * with the host copy, 2 = a wait timed out, 3 = an index out of range); *detail says where.
+ * With reset != 0 the status word is cleared afterwards. */
+CKV_API ckv_status ckv_read_device_status(void* workspace, ckv_stream stream, int32_t reset,
+                                  int32_t* code, int32_t* detail);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CKV_H */

@@ -2,11 +2,11 @@
  * ckv_oracle.c -- TEST INFRASTRUCTURE ONLY.
  *
  * A plain, slow, fp64 CPU statement of what CompressKV's prefill-time KV-cache compression step
- * computes (arxiv 2508.02401, Sec. 3.3 "Token Selection Driven by Semantic Retrieval Heads",
- * with the attention of Eq. 2 and the pooling hyper-parameters of App. A "More Implementation
- * Details").  It exists to check the CUDA library and is only ever loaded by the tests, by the
- * package's smoke check and by the benchmark's CPU-baseline leg.  It shares no code, header,
- * table or helper with the CUDA library.
+ * computes (arxiv 2508.02401, Sec. 3.3, token selection by the semantic retrieval heads,
+ * with the attention of Eq. 2 and the pooling hyper-parameters of App. A).  It exists to
+ * check the CUDA library and is only ever loaded by the tests, by the package's smoke check
+ * and by the benchmark's CPU-baseline leg.  It shares no code, header, table or helper with
+ * the CUDA library.
  *
  * Everything is written out the obvious way: explicit loops, one value at a time, fp64
  * accumulation, a library sort for the selection.  Inputs are bfloat16 bit patterns (uint16),
@@ -50,8 +50,8 @@ static double widen_bf16(uint16_t bits) {
 }
 
 /*
- * Window attention of one query head over one sequence (Eq. 2; Sec. 3.3: "summing over the
- * observation window").
+ * Window attention of one query head over one sequence (Eq. 2; Sec. 3.3 adds up the
+ * window rows' attention per key).
  *
  *   q: w rows of d values, row r is the query at sequence position P + r, P = L - w;
  *      consecutive rows are q_row_stride elements apart.
@@ -103,9 +103,8 @@ int ckv_oracle_window_scores(int L, int w, int d, double scale,
 }
 
 /*
- * 1-D pooling along the token axis (Sec. 3.3 "pooling across the token dimension"; App. A:
- * kernel 5, average pooling in the paper's runs).  Stride 1, output length n, window
- * [j - kernel/2, j + kernel/2] clipped to [0, n).
+ * 1-D pooling along the token axis (Sec. 3.3; App. A uses kernel 5 with average pooling).
+ * Stride 1, output length n, window [j - kernel/2, j + kernel/2] clipped to [0, n).
  *   type 0 (max): maximum over the clipped window (padded cells ignored);
  *   type 1 (avg): sum over the clipped window divided by kernel (zero padding counted).
  */
@@ -148,9 +147,8 @@ static int by_int_asc(const void* pa, const void* pb) {
 }
 
 /*
- * Top-N selection (Sec. 3.3: "the tokens with the top N highest attention scores will be
- * selected"): the k positions of c[0..P) with the largest values, ties to the lower position,
- * written to out[0..k) in ascending order.
+ * Top-N selection (Sec. 3.3): the k positions of c[0..P) with the largest values, ties to the
+ * lower position, written to out[0..k) in ascending order.
  */
 int ckv_oracle_topk(const double* c, int P, int k, int32_t* out) {
     if (P < 0 || k < 0 || k > P) return ORACLE_BAD_ARG;

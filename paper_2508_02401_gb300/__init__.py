@@ -1,0 +1,251 @@
+"""Python binding of libckv (include/ckv.h): CompressKV's prefill-time KV-cache compression
+step on GB300.
+
+The functions here carry the C names and only marshal arguments (torch tensors -> device
+pointers, numpy arrays -> host pointers, the current torch stream -> cudaStream_t).  Every step
+of the computation runs in the library's CUDA kernels; there is no other implementation behind
+these calls.  Loading fails loudly if the library has not been built.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+from dataclasses import dataclass
+
+import numpy as np
+
+__all__ = [
+    "CkvError", "Config", "Batch", "lib_path", "load",
+    "ckv_workspace_size", "ckv_keep_lengths", "ckv_score_window", "ckv_pool", "ckv_select_topk",
+    "ckv_gather_compact", "ckv_compress_layer", "ckv_read_device_status", "ckv_status_string",
+    "ckv_abi_version", "POOL_MAX", "POOL_AVG", "POOL_THEN_SUM", "SUM_THEN_POOL",
+]
+
+POOL_MAX, POOL_AVG = 0, 1
+POOL_THEN_SUM, SUM_THEN_POOL = 0, 1
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_lib = None
+
+
+def lib_path() -> str:
+    return os.path.join(_HERE, "libckv.so")
+
+
+class CkvError(RuntimeError):
+    def __init__(self, status: int, where: str, message: str):
+        self.status = status
+        super().__init__(f"{where}: {_STATUS.get(status, status)}: {message}")
+
+
+_STATUS = {0: "CKV_OK", 1: "CKV_ERR_INVALID_ARG", 2: "CKV_ERR_UNSUPPORTED", 3: "CKV_ERR_WORKSPACE",
+           4: "CKV_ERR_CUDA", 5: "CKV_ERR_DEVICE"}
+
+
+class _Config(C.Structure):
+    _fields_ = [("num_layers", C.c_int32), ("num_q_heads", C.c_int32), ("num_kv_heads", C.c_int32),
+                ("head_dim", C.c_int32), ("window", C.c_int32), ("pool_kernel", C.c_int32),
+                ("pool_type", C.c_int32), ("head_order", C.c_int32), ("softmax_scale", C.c_float),
+                ("head_mask", C.c_void_p), ("budgets", C.c_void_p)]
+
+
+class _Batch(C.Structure):
+    _fields_ = [("num_seqs", C.c_int32), ("cu_seqlens_host", C.c_void_p),
+                ("cu_seqlens_dev", C.c_void_p)]
+
+
+def load():
+    """Loads libckv.so (built by ``paper_2508_02401_gb300.build``)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = lib_path()
+    if not os.path.exists(path):
+        raise ImportError(f"libckv.so is not built ({path}); run "
+                          "`python -c 'import __graft_entry__ as g; g.build()'`")
+    lib = C.CDLL(path)
+    P, I32, I64, SZ = C.c_void_p, C.c_int32, C.c_int64, C.c_size_t
+    cfg, bat = C.POINTER(_Config), C.POINTER(_Batch)
+    sigs = {
+        "ckv_abi_version": ([], I32),
+        "ckv_status_string": ([C.c_int], C.c_char_p),
+        "ckv_last_error_message": ([], C.c_char_p),
+        "ckv_workspace_size": ([cfg, I32, bat, C.POINTER(SZ)], C.c_int),
+        "ckv_keep_lengths": ([cfg, I32, bat, P, C.POINTER(I32)], C.c_int),
+        "ckv_score_window": ([cfg, I32, bat, P, P, I64, I64, P, P, SZ, P], C.c_int),
+        "ckv_pool": ([cfg, I32, bat, P, P, P], C.c_int),
+        "ckv_select_topk": ([cfg, I32, bat, P, P, P, P, SZ, P], C.c_int),
+        "ckv_gather_compact": ([cfg, bat, I32, P, P, I64, I64, P, P, P, P, P, SZ, P], C.c_int),
+        "ckv_compress_layer": ([cfg, I32, bat, P, P, P, I64, I64, P, P, P, P, P, P, SZ, P], C.c_int),
+        "ckv_read_device_status": ([P, P, I32, C.POINTER(I32), C.POINTER(I32)], C.c_int),
+    }
+    for name, (args, res) in sigs.items():
+        fn = getattr(lib, name)
+        fn.argtypes = args
+        fn.restype = res
+    _lib = lib
+    return lib
+
+
+def _check(rc: int, where: str):
+    if rc != 0:
+        raise CkvError(rc, where, load().ckv_last_error_message().decode())
+
+
+@dataclass
+class Config:
+    """Per-model settings: the paper's per-layer head mask and per-layer budgets."""
+    num_layers: int
+    num_q_heads: int
+    num_kv_heads: int
+    window: int
+    pool_kernel: int
+    pool_type: int
+    head_order: int
+    head_mask: np.ndarray   # uint8 [num_layers, num_q_heads]
+    budgets: np.ndarray     # int32 [num_layers]
+    softmax_scale: float = 0.0
+    head_dim: int = 128
+
+    def __post_init__(self):
+        self.head_mask = np.ascontiguousarray(self.head_mask, dtype=np.uint8)
+        self.budgets = np.ascontiguousarray(self.budgets, dtype=np.int32)
+        self._c = _Config(self.num_layers, self.num_q_heads, self.num_kv_heads, self.head_dim,
+                          self.window, self.pool_kernel, self.pool_type, self.head_order,
+                          self.softmax_scale, self.head_mask.ctypes.data, self.budgets.ctypes.data)
+
+    @classmethod
+    def from_workload(cls, wl, **overrides):
+        kw = dict(num_layers=wl.num_layers, num_q_heads=wl.num_q_heads,
+                  num_kv_heads=wl.num_kv_heads, window=wl.window, pool_kernel=wl.pool_kernel,
+                  pool_type=POOL_MAX if wl.pool_type == "max" else POOL_AVG,
+                  head_order=POOL_THEN_SUM if wl.head_order == "pool_then_sum" else SUM_THEN_POOL,
+                  head_mask=wl.head_mask(), budgets=wl.budgets(), head_dim=wl.head_dim)
+        kw.update(overrides)
+        return cls(**kw)
+
+    @property
+    def ref(self):
+        return C.byref(self._c)
+
+
+class Batch:
+    """A varlen batch: host and device copies of cu_seqlens [S+1]."""
+
+    def __init__(self, cu_seqlens, device=None, cu_seqlens_dev=None):
+        import torch
+        self.cu_host = np.ascontiguousarray(cu_seqlens, dtype=np.int32)
+        if cu_seqlens_dev is None:
+            cu_seqlens_dev = torch.from_numpy(self.cu_host.copy()).to(device or "cuda")
+        self.cu_dev = cu_seqlens_dev
+        self._c = _Batch(len(self.cu_host) - 1, self.cu_host.ctypes.data, self.cu_dev.data_ptr())
+
+    @property
+    def num_seqs(self) -> int:
+        return len(self.cu_host) - 1
+
+    @property
+    def total_tokens(self) -> int:
+        return int(self.cu_host[-1])
+
+    @property
+    def ref(self):
+        return C.byref(self._c)
+
+
+def _ptr(t):
+    return None if t is None else C.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        stream = torch.cuda.current_stream()
+    return C.c_void_p(stream if isinstance(stream, int) else stream.cuda_stream)
+
+
+def ckv_abi_version() -> int:
+    return load().ckv_abi_version()
+
+
+def ckv_status_string(status: int) -> str:
+    return load().ckv_status_string(status).decode()
+
+
+def ckv_workspace_size(cfg: Config, layer: int, batch: Batch) -> int:
+    n = C.c_size_t(0)
+    _check(load().ckv_workspace_size(cfg.ref, layer, batch.ref, C.byref(n)), "ckv_workspace_size")
+    return n.value
+
+
+def ckv_keep_lengths(cfg: Config, layer: int, batch: Batch):
+    """Returns (cu_keep [S+1] int32 numpy, n_sel)."""
+    out = np.zeros(batch.num_seqs + 1, np.int32)
+    n_sel = C.c_int32(0)
+    _check(load().ckv_keep_lengths(cfg.ref, layer, batch.ref, out.ctypes.data, C.byref(n_sel)),
+           "ckv_keep_lengths")
+    return out, n_sel.value
+
+
+def ckv_score_window(cfg, layer, batch, q_win, k, scores, workspace, stream=None,
+                     tok_stride=0, head_stride=0):
+    _check(load().ckv_score_window(cfg.ref, layer, batch.ref, _ptr(q_win), _ptr(k), tok_stride,
+                                   head_stride, _ptr(scores), _ptr(workspace),
+                                   workspace.numel() * workspace.element_size(), _stream(stream)),
+           "ckv_score_window")
+
+
+def ckv_pool(cfg, layer, batch, scores, pooled, stream=None):
+    _check(load().ckv_pool(cfg.ref, layer, batch.ref, _ptr(scores), _ptr(pooled), _stream(stream)),
+           "ckv_pool")
+
+
+def ckv_select_topk(cfg, layer, batch, pooled, idx, cu_keep_dev, workspace, stream=None):
+    _check(load().ckv_select_topk(cfg.ref, layer, batch.ref, _ptr(pooled), _ptr(idx),
+                                  _ptr(cu_keep_dev), _ptr(workspace),
+                                  workspace.numel() * workspace.element_size(), _stream(stream)),
+           "ckv_select_topk")
+
+
+def ckv_gather_compact(cfg, batch, t_keep, k, v, idx, cu_keep_dev, k_out, v_out, workspace,
+                       stream=None, tok_stride=0, head_stride=0):
+    _check(load().ckv_gather_compact(cfg.ref, batch.ref, t_keep, _ptr(k), _ptr(v), tok_stride,
+                                     head_stride, _ptr(idx), _ptr(cu_keep_dev), _ptr(k_out),
+                                     _ptr(v_out), _ptr(workspace),
+                                     workspace.numel() * workspace.element_size(), _stream(stream)),
+           "ckv_gather_compact")
+
+
+def ckv_compress_layer(cfg, layer, batch, q_win, k, v, idx, cu_keep_dev, k_out, v_out, workspace,
+                       pooled_out=None, stream=None, tok_stride=0, head_stride=0):
+    _check(load().ckv_compress_layer(cfg.ref, layer, batch.ref, _ptr(q_win), _ptr(k), _ptr(v),
+                                     tok_stride, head_stride, _ptr(idx), _ptr(cu_keep_dev),
+                                     _ptr(k_out), _ptr(v_out), _ptr(pooled_out), _ptr(workspace),
+                                     workspace.numel() * workspace.element_size(), _stream(stream)),
+           "ckv_compress_layer")
+
+
+def ckv_read_device_status(workspace, stream=None, reset=True):
+    """Synchronises the stream; returns (code, detail) of the workspace status word."""
+    code, detail = C.c_int32(0), C.c_int32(0)
+    _check(load().ckv_read_device_status(_ptr(workspace), _stream(stream), 1 if reset else 0,
+                                         C.byref(code), C.byref(detail)), "ckv_read_device_status")
+    return code.value, detail.value
+
+
+def new_workspace(cfg, layer, batch, device="cuda"):
+    """A zeroed workspace of ckv_workspace_size bytes (uint8 tensor, 256-byte aligned)."""
+    import torch
+    n = ckv_workspace_size(cfg, layer, batch)
+    return torch.zeros(n, dtype=torch.uint8, device=device)
+
+
+def new_outputs(cfg, layer, batch, device="cuda"):
+    """Allocates (idx, cu_keep_dev, k_out, v_out) for one layer; returns them with cu_keep_host."""
+    import torch
+    cu_keep, _ = ckv_keep_lengths(cfg, layer, batch)
+    tk = int(cu_keep[-1])
+    idx = torch.empty((cfg.num_kv_heads, tk), dtype=torch.int32, device=device)
+    cu_keep_dev = torch.empty(batch.num_seqs + 1, dtype=torch.int32, device=device)
+    k_out = torch.empty((tk, cfg.num_kv_heads, cfg.head_dim), dtype=torch.bfloat16, device=device)
+    v_out = torch.empty_like(k_out)
+    return idx, cu_keep_dev, k_out, v_out, cu_keep

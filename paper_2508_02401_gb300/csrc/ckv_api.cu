@@ -1,0 +1,558 @@
+// The C ABI declared in include/ckv.h: argument validation (all on the host, before anything
+// is enqueued), per-layer planning of the head batches and key chunks, the workspace layout,
+// TMA descriptor set-up and kernel dispatch.
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <algorithm>
+#include <vector>
+
+#include "ckv.h"
+#include "ckv_device.cuh"
+#include "ckv_internal.h"
+
+namespace ckv {
+namespace {
+
+thread_local char g_msg[512] = "";
+
+ckv_status fail(ckv_status st, const char* fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_msg, sizeof g_msg, fmt, ap);
+    va_end(ap);
+    return st;
+}
+
+ckv_status cuda_fail(cudaError_t e, const char* what) {
+    return fail(CKV_ERR_CUDA, "%s: %s (%s)", what, cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+constexpr size_t kWsAlign = 256;
+constexpr int kPartialCapacityItems = 1024;  // >= the SM count of any supported GPU
+
+size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Everything a call needs to know about one layer of the config.
+struct Plan {
+    int Hq = 0, Hkv = 0, G = 0, w = 0, w_pad = 0, n_cols = 0, hpb = 0, budget = 0;
+    int n_sel = 0, nb = 0;
+    float scale = 0.f;
+    std::vector<int> sel_heads, batch_group, batch_first, batch_nheads, group_first;
+};
+
+ckv_status check_config(const ckv_config* cfg) {
+    if (!cfg) return fail(CKV_ERR_INVALID_ARG, "cfg is NULL");
+    if (cfg->num_layers < 1) return fail(CKV_ERR_INVALID_ARG, "num_layers %d < 1", cfg->num_layers);
+    if (cfg->num_kv_heads < 1 || cfg->num_q_heads < 1)
+        return fail(CKV_ERR_INVALID_ARG, "head counts must be positive");
+    if (cfg->num_q_heads % cfg->num_kv_heads != 0)
+        return fail(CKV_ERR_INVALID_ARG, "num_q_heads %d is not a multiple of num_kv_heads %d",
+                    cfg->num_q_heads, cfg->num_kv_heads);
+    if (cfg->num_q_heads > kMaxQHeads)
+        return fail(CKV_ERR_UNSUPPORTED, "num_q_heads %d > %d", cfg->num_q_heads, kMaxQHeads);
+    if (cfg->head_dim <= 0) return fail(CKV_ERR_INVALID_ARG, "head_dim %d", cfg->head_dim);
+    if (cfg->head_dim != kHeadDim)
+        return fail(CKV_ERR_UNSUPPORTED, "head_dim %d (only 128 is supported)", cfg->head_dim);
+    if (cfg->window < 1) return fail(CKV_ERR_INVALID_ARG, "window %d < 1", cfg->window);
+    if (cfg->window > kMaxWindow)
+        return fail(CKV_ERR_UNSUPPORTED, "window %d > %d", cfg->window, kMaxWindow);
+    if (cfg->pool_kernel < 1 || cfg->pool_kernel % 2 == 0)
+        return fail(CKV_ERR_INVALID_ARG, "pool_kernel %d must be odd and >= 1", cfg->pool_kernel);
+    if (cfg->pool_kernel > kMaxPoolKernel)
+        return fail(CKV_ERR_UNSUPPORTED, "pool_kernel %d > %d", cfg->pool_kernel, kMaxPoolKernel);
+    if (cfg->pool_type != CKV_POOL_MAX && cfg->pool_type != CKV_POOL_AVG)
+        return fail(CKV_ERR_INVALID_ARG, "pool_type %d", cfg->pool_type);
+    if (cfg->head_order != CKV_POOL_THEN_SUM && cfg->head_order != CKV_SUM_THEN_POOL)
+        return fail(CKV_ERR_INVALID_ARG, "head_order %d", cfg->head_order);
+    if (!(cfg->softmax_scale >= 0.f) || !isfinite(cfg->softmax_scale))
+        return fail(CKV_ERR_INVALID_ARG, "softmax_scale must be finite and >= 0");
+    if (!cfg->head_mask || !cfg->budgets)
+        return fail(CKV_ERR_INVALID_ARG, "head_mask and budgets must be host pointers");
+    return CKV_OK;
+}
+
+ckv_status make_plan(const ckv_config* cfg, int32_t layer, Plan& pl) {
+    ckv_status st = check_config(cfg);
+    if (st) return st;
+    if (layer < 0 || layer >= cfg->num_layers)
+        return fail(CKV_ERR_INVALID_ARG, "layer %d outside [0, %d)", layer, cfg->num_layers);
+    pl.Hq = cfg->num_q_heads;
+    pl.Hkv = cfg->num_kv_heads;
+    pl.G = pl.Hq / pl.Hkv;
+    pl.w = cfg->window;
+    pl.budget = cfg->budgets[layer];
+    if (pl.budget < pl.w)
+        return fail(CKV_ERR_INVALID_ARG, "budget %d of layer %d is below the window %d", pl.budget,
+                    layer, pl.w);
+    pl.scale = cfg->softmax_scale > 0.f ? cfg->softmax_scale : 1.0f / sqrtf(static_cast<float>(kHeadDim));
+    pl.w_pad = 8;
+    while (pl.w_pad < pl.w) pl.w_pad *= 2;
+    pl.hpb = kMaxCols / pl.w_pad;
+    const uint8_t* mask = cfg->head_mask + static_cast<size_t>(layer) * pl.Hq;
+    pl.group_first.assign(pl.Hkv + 1, 0);
+    int max_heads = 0;
+    for (int g = 0; g < pl.Hkv; ++g) {
+        pl.group_first[g] = pl.n_sel;
+        std::vector<int> heads;
+        for (int h = g * pl.G; h < (g + 1) * pl.G; ++h)
+            if (mask[h]) heads.push_back(h);
+        if (heads.empty())
+            return fail(CKV_ERR_INVALID_ARG, "KV group %d of layer %d has no selected head", g, layer);
+        for (size_t i = 0; i < heads.size(); i += pl.hpb) {
+            const int n = std::min<int>(pl.hpb, static_cast<int>(heads.size() - i));
+            pl.batch_group.push_back(g);
+            pl.batch_first.push_back(pl.n_sel + static_cast<int>(i));
+            pl.batch_nheads.push_back(n);
+            max_heads = std::max(max_heads, n);
+        }
+        for (int h : heads) pl.sel_heads.push_back(h);
+        pl.n_sel += static_cast<int>(heads.size());
+    }
+    pl.group_first[pl.Hkv] = pl.n_sel;
+    pl.nb = static_cast<int>(pl.batch_group.size());
+    if (pl.nb > kMaxBatches) return fail(CKV_ERR_UNSUPPORTED, "too many head batches (%d)", pl.nb);
+    pl.n_cols = (max_heads * pl.w_pad <= 32) ? 32 : 64;
+    return CKV_OK;
+}
+
+ckv_status check_batch(const ckv_batch* b, int* T_out) {
+    if (!b) return fail(CKV_ERR_INVALID_ARG, "batch is NULL");
+    if (b->num_seqs < 1) return fail(CKV_ERR_INVALID_ARG, "num_seqs %d < 1", b->num_seqs);
+    if (!b->cu_seqlens_host || !b->cu_seqlens_dev)
+        return fail(CKV_ERR_INVALID_ARG, "cu_seqlens_host and cu_seqlens_dev are required");
+    if (b->cu_seqlens_host[0] != 0) return fail(CKV_ERR_INVALID_ARG, "cu_seqlens[0] != 0");
+    for (int s = 0; s < b->num_seqs; ++s)
+        if (b->cu_seqlens_host[s + 1] < b->cu_seqlens_host[s])
+            return fail(CKV_ERR_INVALID_ARG, "cu_seqlens decreases at %d", s);
+    *T_out = b->cu_seqlens_host[b->num_seqs];
+    return CKV_OK;
+}
+
+int64_t keep_total(const ckv_batch* b, int budget) {
+    int64_t t = 0;
+    for (int s = 0; s < b->num_seqs; ++s)
+        t += std::min(budget, b->cu_seqlens_host[s + 1] - b->cu_seqlens_host[s]);
+    return t;
+}
+
+int count_units(const Plan& pl, const ckv_batch* b, int skip_le) {
+    int n = 0;
+    for (int s = 0; s < b->num_seqs; ++s) {
+        const int L = b->cu_seqlens_host[s + 1] - b->cu_seqlens_host[s];
+        if (L > skip_le && L > 0) n += pl.nb;
+    }
+    return n;
+}
+
+// Smallest chunk (in key tiles) that yields at most `ctas` work items.
+void choose_chunks(const Plan& pl, const ckv_batch* b, int skip_le, int ctas, int* chunk_tiles,
+                   int* n_items) {
+    std::vector<int> tiles;
+    for (int s = 0; s < b->num_seqs; ++s) {
+        const int L = b->cu_seqlens_host[s + 1] - b->cu_seqlens_host[s];
+        if (L > skip_le && L > 0) tiles.push_back((L + kTileKeys - 1) / kTileKeys);
+    }
+    if (tiles.empty()) {
+        *chunk_tiles = 1;
+        *n_items = 0;
+        return;
+    }
+    auto count = [&](int C) {
+        long long n = 0;
+        for (int t : tiles) n += (t + C - 1) / C;
+        return n * pl.nb;
+    };
+    int lo = 1, hi = *std::max_element(tiles.begin(), tiles.end());
+    while (lo < hi) {
+        const int mid = (lo + hi) / 2;
+        if (count(mid) <= ctas) hi = mid;
+        else lo = mid + 1;
+    }
+    *chunk_tiles = lo;
+    *n_items = static_cast<int>(count(lo));
+}
+
+struct WsLayout {
+    size_t header = 0, partials = 0, scores = 0, pooled = 0, total = 0;
+};
+
+WsLayout ws_layout(const Plan& pl, const ckv_batch* b, int T) {
+    WsLayout l;
+    size_t off = round_up(sizeof(WsHeader), kWsAlign);
+    const size_t items = std::max(kPartialCapacityItems, count_units(pl, b, -1));
+    l.partials = off;
+    off = round_up(off + items * kMaxCols * sizeof(float2), kWsAlign);
+    l.scores = off;
+    off = round_up(off + static_cast<size_t>(pl.n_sel) * T * sizeof(float), kWsAlign);
+    l.pooled = off;
+    off = round_up(off + static_cast<size_t>(pl.Hkv) * T * sizeof(float), kWsAlign);
+    l.total = off;
+    return l;
+}
+
+ckv_status check_ws(const Plan& pl, const ckv_batch* b, int T, void* ws, size_t bytes, WsLayout* l) {
+    *l = ws_layout(pl, b, T);
+    if (!ws) return fail(CKV_ERR_WORKSPACE, "workspace is NULL");
+    if (!aligned(ws, kWsAlign)) return fail(CKV_ERR_WORKSPACE, "workspace not 256-byte aligned");
+    if (bytes < l->total)
+        return fail(CKV_ERR_WORKSPACE, "workspace %zu bytes < required %zu", bytes, l->total);
+    return CKV_OK;
+}
+
+ckv_status check_kv(const void* p, const char* name, int T) {
+    if (T == 0) return CKV_OK;
+    if (!p) return fail(CKV_ERR_INVALID_ARG, "%s is NULL", name);
+    if (!aligned(p, 16)) return fail(CKV_ERR_INVALID_ARG, "%s is not 16-byte aligned", name);
+    return CKV_OK;
+}
+
+ckv_status resolve_strides(const Plan& pl, int64_t* tok, int64_t* head) {
+    if (*tok == 0) *tok = static_cast<int64_t>(pl.Hkv) * kHeadDim;
+    if (*head == 0) *head = kHeadDim;
+    if (*tok < 0 || *head < 0 || *tok % 8 || *head % 8)
+        return fail(CKV_ERR_INVALID_ARG, "strides must be non-negative multiples of 8 elements");
+    if (*tok >= (static_cast<int64_t>(1) << 38) || *head >= (static_cast<int64_t>(1) << 38))
+        return fail(CKV_ERR_UNSUPPORTED, "stride too large");
+    return CKV_OK;
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        void* ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(ptr);
+    }
+    return fn;
+}
+
+// K viewed as {128 (dim), H_kv, T} with a {64, 1, 128} box and the 128-byte swizzle.
+ckv_status make_k_map(CUtensorMap* map, const void* k, int Hkv, int T, int64_t tok, int64_t head) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return fail(CKV_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
+    const cuuint64_t dims[3] = {static_cast<cuuint64_t>(kHeadDim), static_cast<cuuint64_t>(Hkv),
+                                static_cast<cuuint64_t>(T)};
+    const cuuint64_t strides[2] = {static_cast<cuuint64_t>(head) * 2, static_cast<cuuint64_t>(tok) * 2};
+    const cuuint32_t box[3] = {64, 1, static_cast<cuuint32_t>(kTileKeys)};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    const CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(k), dims,
+                          strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                          CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(CKV_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", static_cast<int>(r));
+    return CKV_OK;
+}
+
+}  // namespace
+
+int device_sm_count() {
+    static int cached[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 0;
+    if (dev < 64 && cached[dev]) return cached[dev];
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    if (dev < 64) cached[dev] = n;
+    return n;
+}
+
+namespace {
+
+ckv_status enqueue_score(const Plan& pl, const ckv_batch* b, int T, const void* q_win,
+                         const void* k, int64_t tok, int64_t head, float* scores, void* ws,
+                         const WsLayout& l, int skip_le, cudaStream_t stream) {
+    int ctas = device_sm_count();
+    if (ctas <= 0) return cuda_fail(cudaGetLastError(), "querying the SM count");
+    ctas = std::min(ctas, kPartialCapacityItems);
+    ScoreLaunch L;
+    memset(&L, 0, sizeof L);
+    choose_chunks(pl, b, skip_le, ctas, &L.chunk_tiles, &L.n_items);
+    if (L.n_items == 0) return CKV_OK;
+    ckv_status st = make_k_map(&L.tmap_k, k, pl.Hkv, T, tok, head);
+    if (st) return st;
+    uint8_t* w8 = static_cast<uint8_t*>(ws);
+    L.q_win = q_win;
+    L.cu_seqlens_dev = b->cu_seqlens_dev;
+    L.partials = w8 + l.partials;
+    L.scores = scores;
+    L.status = reinterpret_cast<int*>(w8);
+    L.S = b->num_seqs;
+    L.T = T;
+    L.Hq = pl.Hq;
+    L.w = pl.w;
+    L.w_pad = pl.w_pad;
+    L.n_cols = pl.n_cols;
+    L.nb = pl.nb;
+    L.grid = ctas;
+    L.skip_le = skip_le;
+    L.cu_hash = seqlens_hash(b->cu_seqlens_host, b->num_seqs);
+    L.softmax_scale = pl.scale;
+    L.n_sel = pl.n_sel;
+    L.batch_group = pl.batch_group.data();
+    L.batch_first = pl.batch_first.data();
+    L.batch_nheads = pl.batch_nheads.data();
+    L.sel_heads = pl.sel_heads.data();
+    const cudaError_t e = launch_score(L, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "launching the scoring kernels");
+    return CKV_OK;
+}
+
+SelectLaunch select_launch(const Plan& pl, const ckv_batch* b, int T, int T_keep, int skip_le,
+                           const ckv_config* cfg, void* ws) {
+    SelectLaunch L;
+    memset(&L, 0, sizeof L);
+    L.cu_seqlens_dev = b->cu_seqlens_dev;
+    L.status = static_cast<int*>(ws);
+    L.S = b->num_seqs;
+    L.T = T;
+    L.Hkv = pl.Hkv;
+    L.w = pl.w;
+    L.budget = pl.budget;
+    L.T_keep = T_keep;
+    L.pool_kernel = cfg->pool_kernel;
+    L.pool_type = cfg->pool_type;
+    L.head_order = cfg->head_order;
+    L.skip_le = skip_le;
+    L.cu_hash = seqlens_hash(b->cu_seqlens_host, b->num_seqs);
+    L.group_first = pl.group_first.data();
+    return L;
+}
+
+}  // namespace
+}  // namespace ckv
+
+using namespace ckv;
+
+extern "C" {
+
+int32_t ckv_abi_version(void) { return CKV_ABI_VERSION; }
+
+const char* ckv_status_string(ckv_status s) {
+    switch (s) {
+        case CKV_OK: return "CKV_OK";
+        case CKV_ERR_INVALID_ARG: return "CKV_ERR_INVALID_ARG";
+        case CKV_ERR_UNSUPPORTED: return "CKV_ERR_UNSUPPORTED";
+        case CKV_ERR_WORKSPACE: return "CKV_ERR_WORKSPACE";
+        case CKV_ERR_CUDA: return "CKV_ERR_CUDA";
+        case CKV_ERR_DEVICE: return "CKV_ERR_DEVICE";
+    }
+    return "unknown ckv_status";
+}
+
+const char* ckv_last_error_message(void) { return g_msg; }
+
+ckv_status ckv_workspace_size(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
+                              size_t* bytes) {
+    Plan pl;
+    ckv_status st = make_plan(cfg, layer, pl);
+    if (st) return st;
+    int T = 0;
+    if ((st = check_batch(batch, &T))) return st;
+    if (!bytes) return fail(CKV_ERR_INVALID_ARG, "bytes is NULL");
+    *bytes = ws_layout(pl, batch, T).total;
+    return CKV_OK;
+}
+
+ckv_status ckv_keep_lengths(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
+                            int32_t* cu_keep_host, int32_t* n_sel) {
+    Plan pl;
+    ckv_status st = make_plan(cfg, layer, pl);
+    if (st) return st;
+    int T = 0;
+    if ((st = check_batch(batch, &T))) return st;
+    if (!cu_keep_host) return fail(CKV_ERR_INVALID_ARG, "cu_keep_host is NULL");
+    cu_keep_host[0] = 0;
+    for (int s = 0; s < batch->num_seqs; ++s)
+        cu_keep_host[s + 1] = cu_keep_host[s] +
+                              std::min(pl.budget, batch->cu_seqlens_host[s + 1] - batch->cu_seqlens_host[s]);
+    if (n_sel) *n_sel = pl.n_sel;
+    return CKV_OK;
+}
+
+ckv_status ckv_score_window(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
+                            const void* q_win, const void* k, int64_t tok_stride,
+                            int64_t head_stride, float* scores, void* workspace,
+                            size_t workspace_bytes, ckv_stream stream) {
+    Plan pl;
+    ckv_status st = make_plan(cfg, layer, pl);
+    if (st) return st;
+    int T = 0;
+    WsLayout l;
+    if ((st = check_batch(batch, &T)) || (st = resolve_strides(pl, &tok_stride, &head_stride)) ||
+        (st = check_kv(q_win, "q_win", T)) || (st = check_kv(k, "k", T)) ||
+        (st = check_kv(scores, "scores", T)) ||
+        (st = check_ws(pl, batch, T, workspace, workspace_bytes, &l)))
+        return st;
+    return enqueue_score(pl, batch, T, q_win, k, tok_stride, head_stride, scores, workspace, l, -1,
+                         reinterpret_cast<cudaStream_t>(stream));
+}
+
+ckv_status ckv_pool(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
+                    const float* scores, float* pooled, ckv_stream stream) {
+    Plan pl;
+    ckv_status st = make_plan(cfg, layer, pl);
+    if (st) return st;
+    int T = 0;
+    if ((st = check_batch(batch, &T)) || (st = check_kv(scores, "scores", T)) ||
+        (st = check_kv(pooled, "pooled", T)))
+        return st;
+    SelectLaunch L = select_launch(pl, batch, T, 0, -1, cfg, nullptr);
+    L.scores = scores;
+    L.pooled = pooled;
+    const cudaError_t e = launch_pool(L, reinterpret_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? CKV_OK : cuda_fail(e, "launching the pooling kernel");
+}
+
+ckv_status ckv_select_topk(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
+                           const float* pooled, int32_t* idx, int32_t* cu_keep_dev,
+                           void* workspace, size_t workspace_bytes, ckv_stream stream) {
+    Plan pl;
+    ckv_status st = make_plan(cfg, layer, pl);
+    if (st) return st;
+    int T = 0;
+    WsLayout l;
+    if ((st = check_batch(batch, &T)) || (st = check_kv(pooled, "pooled", T)) ||
+        (st = check_ws(pl, batch, T, workspace, workspace_bytes, &l)))
+        return st;
+    const int64_t tk = keep_total(batch, pl.budget);
+    if (tk > 0 && !idx) return fail(CKV_ERR_INVALID_ARG, "idx is NULL");
+    if (!cu_keep_dev) return fail(CKV_ERR_INVALID_ARG, "cu_keep_dev is NULL");
+    SelectLaunch L = select_launch(pl, batch, T, static_cast<int>(tk), -1, cfg, workspace);
+    L.pooled = const_cast<float*>(pooled);
+    L.idx = idx;
+    L.cu_keep_dev = cu_keep_dev;
+    const cudaError_t e = launch_select(L, reinterpret_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? CKV_OK : cuda_fail(e, "launching the selection kernel");
+}
+
+ckv_status ckv_gather_compact(const ckv_config* cfg, const ckv_batch* batch, int32_t t_keep,
+                              const void* k, const void* v, int64_t tok_stride,
+                              int64_t head_stride, const int32_t* idx,
+                              const int32_t* cu_keep_dev, void* k_out, void* v_out,
+                              void* workspace, size_t workspace_bytes, ckv_stream stream) {
+    ckv_status st = check_config(cfg);
+    if (st) return st;
+    Plan pl;
+    pl.Hkv = cfg->num_kv_heads;
+    int T = 0;
+    if ((st = check_batch(batch, &T)) || (st = resolve_strides(pl, &tok_stride, &head_stride)))
+        return st;
+    if (!workspace || !aligned(workspace, kWsAlign) || workspace_bytes < sizeof(WsHeader))
+        return fail(CKV_ERR_WORKSPACE, "workspace missing, misaligned or too small");
+    if (t_keep < 0) return fail(CKV_ERR_INVALID_ARG, "t_keep %d < 0", t_keep);
+    if (t_keep == 0) return CKV_OK;
+    if ((st = check_kv(k, "k", T)) || (st = check_kv(v, "v", T)) ||
+        (st = check_kv(k_out, "k_out", t_keep)) || (st = check_kv(v_out, "v_out", t_keep)))
+        return st;
+    if (!idx || !cu_keep_dev) return fail(CKV_ERR_INVALID_ARG, "idx and cu_keep_dev are required");
+    GatherLaunch L;
+    L.k = k;
+    L.v = v;
+    L.tok_stride = tok_stride;
+    L.head_stride = head_stride;
+    L.idx = idx;
+    L.cu_keep_dev = cu_keep_dev;
+    L.cu_seqlens_dev = batch->cu_seqlens_dev;
+    L.k_out = k_out;
+    L.v_out = v_out;
+    L.status = static_cast<int*>(workspace);
+    L.S = batch->num_seqs;
+    L.T = T;
+    L.Hkv = pl.Hkv;
+    L.T_keep = t_keep;
+    L.cu_hash = seqlens_hash(batch->cu_seqlens_host, batch->num_seqs);
+    const cudaError_t e = launch_gather(L, reinterpret_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? CKV_OK : cuda_fail(e, "launching the gather kernel");
+}
+
+ckv_status ckv_compress_layer(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
+                              const void* q_win, const void* k, const void* v,
+                              int64_t tok_stride, int64_t head_stride, int32_t* idx,
+                              int32_t* cu_keep_dev, void* k_out, void* v_out, float* pooled_out,
+                              void* workspace, size_t workspace_bytes, ckv_stream stream) {
+    Plan pl;
+    ckv_status st = make_plan(cfg, layer, pl);
+    if (st) return st;
+    int T = 0;
+    WsLayout l;
+    if ((st = check_batch(batch, &T)) || (st = resolve_strides(pl, &tok_stride, &head_stride)) ||
+        (st = check_kv(q_win, "q_win", T)) || (st = check_kv(k, "k", T)) ||
+        (st = check_kv(v, "v", T)) || (st = check_ws(pl, batch, T, workspace, workspace_bytes, &l)))
+        return st;
+    if (pooled_out && !aligned(pooled_out, 16))
+        return fail(CKV_ERR_INVALID_ARG, "pooled_out is not 16-byte aligned");
+    const int64_t tk = keep_total(batch, pl.budget);
+    if (tk > INT32_MAX) return fail(CKV_ERR_UNSUPPORTED, "too many kept tokens");
+    if (!cu_keep_dev) return fail(CKV_ERR_INVALID_ARG, "cu_keep_dev is NULL");
+    if (tk > 0 && (st = check_kv(idx, "idx", 1))) return st;
+    if (tk > 0 && ((st = check_kv(k_out, "k_out", 1)) || (st = check_kv(v_out, "v_out", 1))))
+        return st;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    uint8_t* w8 = static_cast<uint8_t*>(workspace);
+    float* scores = reinterpret_cast<float*>(w8 + l.scores);
+    float* pooled = pooled_out ? pooled_out : reinterpret_cast<float*>(w8 + l.pooled);
+    const int skip_le = pl.budget;  // sequences that fit the budget are kept whole
+    if ((st = enqueue_score(pl, batch, T, q_win, k, tok_stride, head_stride, scores, workspace, l,
+                            skip_le, s)))
+        return st;
+    SelectLaunch L = select_launch(pl, batch, T, static_cast<int>(tk), skip_le, cfg, workspace);
+    L.scores = scores;
+    L.pooled = pooled;
+    L.idx = idx;
+    L.cu_keep_dev = cu_keep_dev;
+    cudaError_t e = launch_pool(L, s);
+    if (e != cudaSuccess) return cuda_fail(e, "launching the pooling kernel");
+    e = launch_select(L, s);
+    if (e != cudaSuccess) return cuda_fail(e, "launching the selection kernel");
+    if (tk == 0) return CKV_OK;
+    GatherLaunch G;
+    G.k = k;
+    G.v = v;
+    G.tok_stride = tok_stride;
+    G.head_stride = head_stride;
+    G.idx = idx;
+    G.cu_keep_dev = cu_keep_dev;
+    G.cu_seqlens_dev = batch->cu_seqlens_dev;
+    G.k_out = k_out;
+    G.v_out = v_out;
+    G.status = static_cast<int*>(workspace);
+    G.S = batch->num_seqs;
+    G.T = T;
+    G.Hkv = pl.Hkv;
+    G.T_keep = static_cast<int>(tk);
+    G.cu_hash = seqlens_hash(batch->cu_seqlens_host, batch->num_seqs);
+    e = launch_gather(G, s);
+    return e == cudaSuccess ? CKV_OK : cuda_fail(e, "launching the gather kernel");
+}
+
+ckv_status ckv_read_device_status(void* workspace, ckv_stream stream, int32_t reset,
+                                  int32_t* code, int32_t* detail) {
+    if (!workspace || !code) return fail(CKV_ERR_INVALID_ARG, "workspace and code are required");
+    cudaError_t e = cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "synchronising the stream");
+    int32_t hdr[2] = {0, 0};
+    e = cudaMemcpy(hdr, workspace, sizeof hdr, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(e, "reading the status word");
+    *code = hdr[0];
+    if (detail) *detail = hdr[1];
+    if (reset) {
+        e = cudaMemset(workspace, 0, sizeof hdr);
+        if (e != cudaSuccess) return cuda_fail(e, "clearing the status word");
+    }
+    return CKV_OK;
+}
+
+}  // extern "C"

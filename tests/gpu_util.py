@@ -1,0 +1,132 @@
+"""Helpers for the GPU parity tests: run the CUDA path through the C ABI and compare with the
+oracle under the tolerances of the parity contract.
+
+Tolerances (the GPU accumulates in fp32, the oracle in fp64):
+  * scores, pooled:  |gpu - oracle| <= 1e-3 * |oracle| + 1e-12 * max(oracle of that row)
+    (the floor absorbs fp32 underflow of probabilities that are negligible in the row);
+  * pooling of the GPU's own scores: 1e-5 relative (a handful of fp32 roundings);
+  * selection on the GPU's own pooled scores: bit-exact (same fp32 values, same decision);
+  * selection against the oracle's scores: exact unless the k-th and (k+1)-th oracle scores
+    are within 1e-3 of each other, otherwise every token clearly above / below the threshold
+    band must be in / out;
+  * gathered K/V: bit-exact against the input rows at the GPU's indices.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import oracle
+import paper_2508_02401_gb300 as ckv
+
+SCORE_RTOL = 1e-3
+SCORE_FLOOR = 1e-12
+
+
+def to_dev(bits: np.ndarray) -> torch.Tensor:
+    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).cuda().view(torch.bfloat16)
+
+
+def to_host(t: torch.Tensor) -> np.ndarray:
+    return t.view(torch.int16).cpu().numpy().view(np.uint16)
+
+
+def run_gpu(wl, layer, li, cfg=None, scores=True, stream=None, check_status=True):
+    """compress_layer (+ score_window when asked) for one layer; numpy outputs."""
+    cfg = cfg or ckv.Config.from_workload(wl)
+    batch = ckv.Batch(wl.cu_seqlens())
+    q, k, v = to_dev(li.q_win), to_dev(li.k), to_dev(li.v)
+    ws = ckv.new_workspace(cfg, layer, batch)
+    idx, cu_keep_dev, k_out, v_out, cu_keep = ckv.new_outputs(cfg, layer, batch)
+    T = batch.total_tokens
+    pooled = torch.full((cfg.num_kv_heads, T), float("nan"), dtype=torch.float32, device="cuda")
+    ckv.ckv_compress_layer(cfg, layer, batch, q, k, v, idx, cu_keep_dev, k_out, v_out, ws,
+                           pooled_out=pooled, stream=stream)
+    out = dict(cfg=cfg, cu_keep=cu_keep)
+    if scores:
+        _, n_sel = ckv.ckv_keep_lengths(cfg, layer, batch)
+        sc = torch.full((n_sel, T), float("nan"), dtype=torch.float32, device="cuda")
+        ckv.ckv_score_window(cfg, layer, batch, q, k, sc, ws, stream=stream)
+        out["scores"] = sc.cpu().numpy()
+    code, detail = ckv.ckv_read_device_status(ws, stream=stream)
+    if check_status:
+        assert code == 0, f"device status {code} ({detail})"
+    out.update(status=(code, detail), pooled=pooled.cpu().numpy(), idx=idx.cpu().numpy(),
+               cu_keep_dev=cu_keep_dev.cpu().numpy(), k_out=to_host(k_out), v_out=to_host(v_out))
+    return out
+
+
+def run_oracle(wl, layer, li, mask=None, groups=None, want_kv=True):
+    m = wl.head_mask()[layer] if mask is None else mask
+    return oracle.compress_layer(li.q_win, li.k, li.v, wl.cu_seqlens(), m,
+                                 int(wl.budgets()[layer]), wl.window, wl.pool_kernel,
+                                 0 if wl.pool_type == "max" else 1,
+                                 0 if wl.head_order == "pool_then_sum" else 1,
+                                 want_kv=want_kv, groups=groups)
+
+
+def assert_close_rows(gpu, orc, rtol=SCORE_RTOL, floor=SCORE_FLOOR, what="scores"):
+    gpu = np.asarray(gpu, np.float64)
+    orc = np.asarray(orc, np.float64)
+    assert gpu.shape == orc.shape
+    if orc.size == 0:
+        return
+    tol = rtol * np.abs(orc) + floor * np.max(np.abs(orc))
+    bad = ~(np.abs(gpu - orc) <= tol)
+    if bad.any():
+        i = np.argmax(np.where(bad, np.abs(gpu - orc) / (np.abs(orc) + 1e-300), 0))
+        raise AssertionError(f"{what}: {bad.sum()} of {bad.size} outside tolerance; worst at {i}: "
+                             f"gpu={gpu.flat[i]!r} oracle={orc.flat[i]!r}")
+
+
+def check_layer(wl, layer, li, g, o, groups=None, exact_select=True):
+    """All parity checks of one layer: g = run_gpu output, o = run_oracle output."""
+    cu = wl.cu_seqlens()
+    B = int(wl.budgets()[layer])
+    w = wl.window
+    np.testing.assert_array_equal(g["cu_keep"], o["cu_keep"])
+    np.testing.assert_array_equal(g["cu_keep_dev"], o["cu_keep"])
+    ck = o["cu_keep"]
+    groups = range(wl.num_kv_heads) if groups is None else groups
+    sel_rows = np.nonzero(wl.head_mask()[layer])[0]
+    G = wl.group_size
+    for s in range(wl.num_seqs):
+        t0, t1 = int(cu[s]), int(cu[s + 1])
+        L = t1 - t0
+        P = L - w
+        for gi in groups:
+            # scores of the group's selected heads, every position
+            if "scores" in g and L > 0:
+                rows = [i for i, h in enumerate(sel_rows) if h // G == gi]
+                assert_close_rows(g["scores"][rows, t0:t1], o["scores"][rows, t0:t1])
+            ix = g["idx"][gi, ck[s]:ck[s + 1]]
+            if L <= B:
+                np.testing.assert_array_equal(ix, np.arange(L))
+                continue
+            k = B - w
+            assert_close_rows(g["pooled"][gi, t0:t0 + P], o["pooled"][gi, t0:t0 + P], what="pooled")
+            np.testing.assert_array_equal(ix[k:], np.arange(P, L))
+            cand = ix[:k]
+            assert np.all(np.diff(cand) > 0) and (k == 0 or (cand[0] >= 0 and cand[-1] < P))
+            if exact_select:
+                # the selection, decided on the GPU's own fp32 pooled scores, is exact
+                np.testing.assert_array_equal(
+                    cand, oracle.topk(g["pooled"][gi, t0:t0 + P].astype(np.float64), k))
+            # against the oracle's fp64 scores: exact unless the k-th / (k+1)-th are too close
+            c = o["pooled"][gi, t0:t0 + P]
+            if k == 0:
+                continue
+            order = np.lexsort((np.arange(P), -c))
+            ck_, floor = c[order[k - 1]], SCORE_FLOOR * c.max()
+            band = SCORE_RTOL * ck_ + floor
+            cs = set(cand.tolist())
+            assert set(np.nonzero(c > ck_ + band)[0].tolist()) <= cs
+            assert not (set(np.nonzero(c < ck_ - band)[0].tolist()) & cs)
+            if k < P and c[order[k - 1]] - c[order[k]] >= band:
+                assert cs == set(order[:k].tolist())
+    # gathered rows are the input rows at the GPU's indices, bit for bit
+    for s in range(wl.num_seqs):
+        for gi in groups:
+            rows = cu[s] + g["idx"][gi, ck[s]:ck[s + 1]]
+            np.testing.assert_array_equal(g["k_out"][ck[s]:ck[s + 1], gi], li.k[rows, gi])
+            np.testing.assert_array_equal(g["v_out"][ck[s]:ck[s + 1], gi], li.v[rows, gi])

@@ -1,0 +1,195 @@
+"""Parity of the CUDA path (through the C ABI) with the fp64 oracle on seeded inputs.
+
+Sizes span several key tiles, several chunks per (sequence, KV head), ragged tails, short and
+empty sequences, every head-row padding width and both pooling orders; the five workloads are
+run at full size on sampled layers (and sampled KV heads where the oracle would be slow).
+"""
+import numpy as np
+import pytest
+import torch
+
+import ckv_synth as cs
+import oracle
+import paper_2508_02401_gb300 as ckv
+from tests import gpu_util as gu
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a GPU")
+    ckv.load()
+    oracle.build()
+
+
+def _wl(**kw):
+    base = dict(name="fuzz", num_layers=2, num_q_heads=8, num_kv_heads=2, seqlens=(300,),
+                window=32, heads_per_group=2, budget_mean=48, budget_uniform=True, pool_kernel=7,
+                seed=11)
+    base.update(kw)
+    return cs.Workload(**base)
+
+
+FUZZ = [
+    dict(),
+    dict(seqlens=(1, 5, 31, 32, 33, 127, 128, 129, 300, 0, 2000), budget_mean=40),
+    dict(seqlens=(700, 129), budget_mean=32),                        # k = 0: the window only
+    dict(window=8, pool_kernel=5, pool_type="avg", heads_per_group=4, seqlens=(1000,)),
+    dict(window=8, pool_kernel=5, pool_type="avg", heads_per_group=4, seqlens=(1000, 77),
+         head_order="sum_then_pool"),
+    dict(window=17, heads_per_group=3, seqlens=(900, 450)),          # padded rows, 2 batches
+    dict(window=64, heads_per_group=1, seqlens=(1500,), budget_mean=100),
+    dict(window=64, heads_per_group=2, seqlens=(1500,), budget_mean=100),  # 2 batches of 1 head
+    dict(window=1, heads_per_group=1, pool_kernel=1, seqlens=(513,), budget_mean=20),
+    dict(window=16, heads_per_group=4, seqlens=(4096, 333), head_order="sum_then_pool"),
+    dict(num_q_heads=28, num_kv_heads=4, heads_per_group=3, seqlens=(3000, 1200)),
+    dict(num_q_heads=28, num_kv_heads=4, heads_per_group=7, window=8, seqlens=(2500,)),
+    dict(num_q_heads=32, num_kv_heads=8, heads_per_group=2, seqlens=(8192,), budget_mean=256,
+         outlier_channels=8),
+    dict(seqlens=(5000,), plant="span", plant_count=32, plant_beta=4.0, plant_noise=True,
+         budget_mean=64, pool_type="avg"),
+    dict(seqlens=(20000,), budget_mean=600, heads_per_group=1, pool_kernel=9),
+]
+
+
+@pytest.mark.parametrize("case", range(len(FUZZ)))
+def test_fuzz_shapes(case):
+    wl = _wl(**FUZZ[case])
+    for layer in range(wl.num_layers):
+        li = wl.layer(layer)
+        g = gu.run_gpu(wl, layer, li)
+        o = gu.run_oracle(wl, layer, li)
+        gu.check_layer(wl, layer, li, g, o)
+
+
+def test_single_layer_workload_full():
+    wl = cs.workload("single_layer_l2048")
+    li = wl.layer(0)
+    g = gu.run_gpu(wl, 0, li)
+    o = gu.run_oracle(wl, 0, li)
+    gu.check_layer(wl, 0, li, g, o)
+    ck = o["cu_keep"]
+    for gi in range(wl.num_kv_heads):  # the planted keys survive
+        assert set(li.planted[0].tolist()) <= set(g["idx"][gi, ck[0]:ck[1]].tolist())
+
+
+@pytest.mark.parametrize("name,layers,groups", [
+    ("llama8b_l8192", (0, 13, 31), None),
+    ("llama8b_l32768", (0, 5), None),
+    ("needle_l131072", (7,), (0, 5)),
+    ("ragged_qwen7b", (0, 27), None),
+])
+def test_full_size_workloads(name, layers, groups):
+    wl = cs.workload(name)
+    for layer in layers:
+        li = wl.layer(layer)
+        g = gu.run_gpu(wl, layer, li, scores=groups is None)
+        o = gu.run_oracle(wl, layer, li, groups=groups, want_kv=False)
+        if groups is not None:
+            g["scores"] = None
+            g.pop("scores")
+        gu.check_layer(wl, layer, li, g, o, groups=groups)
+        if wl.plant == "span":  # the needle span is kept by every KV head
+            ck = o["cu_keep"]
+            for gi in range(wl.num_kv_heads):
+                assert set(li.planted[0].tolist()) <= set(g["idx"][gi, ck[0]:ck[1]].tolist())
+
+
+def test_unselected_heads_are_ignored():
+    wl = _wl(seqlens=(3000, 400))
+    li = wl.layer(0)
+    a = gu.run_gpu(wl, 0, li)
+    m = wl.head_mask()[0]
+    li.q_win[:, :, m == 0, :] = 0x7FC0  # NaN in every unselected head
+    b = gu.run_gpu(wl, 0, li)
+    for key in ("scores", "pooled", "idx", "k_out", "v_out"):
+        np.testing.assert_array_equal(np.nan_to_num(a[key]), np.nan_to_num(b[key]))
+
+
+def test_deterministic():
+    wl = _wl(seqlens=(6000, 300), num_q_heads=32, num_kv_heads=8)
+    li = wl.layer(1)
+    a = gu.run_gpu(wl, 1, li)
+    b = gu.run_gpu(wl, 1, li)
+    for key in ("scores", "pooled", "idx", "k_out", "v_out"):
+        assert np.array_equal(a[key], b[key], equal_nan=True)
+
+
+def test_standalone_entry_points_match_the_fused_call():
+    wl = _wl(seqlens=(4000, 1000, 20), num_q_heads=32, num_kv_heads=8, pool_type="avg")
+    layer = 0
+    li = wl.layer(layer)
+    cfg = ckv.Config.from_workload(wl)
+    batch = ckv.Batch(wl.cu_seqlens())
+    q, k, v = gu.to_dev(li.q_win), gu.to_dev(li.k), gu.to_dev(li.v)
+    ws = ckv.new_workspace(cfg, layer, batch)
+    cu_keep, n_sel = ckv.ckv_keep_lengths(cfg, layer, batch)
+    T, tk = batch.total_tokens, int(cu_keep[-1])
+    scores = torch.empty((n_sel, T), dtype=torch.float32, device="cuda")
+    pooled = torch.empty((8, T), dtype=torch.float32, device="cuda")
+    idx = torch.empty((8, tk), dtype=torch.int32, device="cuda")
+    cu_keep_dev = torch.empty(4, dtype=torch.int32, device="cuda")
+    k_out = torch.empty((tk, 8, 128), dtype=torch.bfloat16, device="cuda")
+    v_out = torch.empty_like(k_out)
+    ckv.ckv_score_window(cfg, layer, batch, q, k, scores, ws)
+    ckv.ckv_pool(cfg, layer, batch, scores, pooled)
+    ckv.ckv_select_topk(cfg, layer, batch, pooled, idx, cu_keep_dev, ws)
+    ckv.ckv_gather_compact(cfg, batch, tk, k, v, idx, cu_keep_dev, k_out, v_out, ws)
+    assert ckv.ckv_read_device_status(ws) == (0, 0)
+    fused = gu.run_gpu(wl, layer, li)
+    np.testing.assert_array_equal(scores.cpu().numpy(), fused["scores"])
+    np.testing.assert_array_equal(idx.cpu().numpy(), fused["idx"])
+    np.testing.assert_array_equal(gu.to_host(k_out), fused["k_out"])
+    np.testing.assert_array_equal(gu.to_host(v_out), fused["v_out"])
+    # pooling: the GPU's pooled scores equal the oracle's pooling of the GPU's own scores
+    sc = scores.cpu().numpy().astype(np.float64)
+    pl = pooled.cpu().numpy()
+    cu = wl.cu_seqlens()
+    sel = np.nonzero(wl.head_mask()[layer])[0]
+    for s in range(wl.num_seqs):
+        t0, P = int(cu[s]), wl.seqlens[s] - wl.window
+        if P <= 0:
+            continue
+        for gi in range(8):
+            rows = [i for i, h in enumerate(sel) if h // 4 == gi]
+            ref = sum(oracle.pool(sc[r, t0:t0 + P], wl.pool_kernel, 1) for r in rows)
+            np.testing.assert_allclose(pl[gi, t0:t0 + P], ref, rtol=1e-5, atol=1e-30)
+
+
+def test_strided_kv_layout():
+    """K and V interleaved in one [T, 2, H_kv, 128] buffer: strides select each half."""
+    wl = _wl(seqlens=(2500, 700), num_q_heads=32, num_kv_heads=8)
+    layer = 1
+    li = wl.layer(layer)
+    ref = gu.run_gpu(wl, layer, li)
+    cfg = ref["cfg"]
+    batch = ckv.Batch(wl.cu_seqlens())
+    kv = torch.stack([gu.to_dev(li.k), gu.to_dev(li.v)], dim=1).contiguous()  # [T, 2, 8, 128]
+    k_view, v_view = kv[:, 0], kv[:, 1]
+    ws = ckv.new_workspace(cfg, layer, batch)
+    idx, cu_keep_dev, k_out, v_out, _ = ckv.new_outputs(cfg, layer, batch)
+    ckv.ckv_compress_layer(cfg, layer, batch, gu.to_dev(li.q_win), k_view, v_view, idx, cu_keep_dev,
+                           k_out, v_out, ws, tok_stride=2 * 8 * 128, head_stride=128)
+    assert ckv.ckv_read_device_status(ws) == (0, 0)
+    np.testing.assert_array_equal(idx.cpu().numpy(), ref["idx"])
+    np.testing.assert_array_equal(gu.to_host(k_out), ref["k_out"])
+    np.testing.assert_array_equal(gu.to_host(v_out), ref["v_out"])
+
+
+def test_device_lengths_that_disagree_are_reported():
+    """cu_seqlens_dev splitting the same tokens differently from the host copy: the kernels
+    stay in bounds and the status word says so."""
+    wl = _wl(seqlens=(2000, 1000))
+    li = wl.layer(0)
+    cfg = ckv.Config.from_workload(wl)
+    batch = ckv.Batch(wl.cu_seqlens(),
+                      cu_seqlens_dev=torch.tensor([0, 1500, 3000], dtype=torch.int32, device="cuda"))
+    ws = ckv.new_workspace(cfg, 0, batch)
+    idx, cu_keep_dev, k_out, v_out, _ = ckv.new_outputs(cfg, 0, batch)
+    ckv.ckv_compress_layer(cfg, 0, batch, gu.to_dev(li.q_win), gu.to_dev(li.k), gu.to_dev(li.v),
+                           idx, cu_keep_dev, k_out, v_out, ws)
+    code, _ = ckv.ckv_read_device_status(ws)
+    assert code == 1
+    assert ckv.ckv_read_device_status(ws) == (0, 0)  # the read reset it
