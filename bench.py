@@ -47,6 +47,8 @@ def _args():
     ap.add_argument("--workload", default=WORKLOAD)
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--layers", type=int, default=0, help="use only the first N layers (0 = all)")
+    ap.add_argument("--breakdown", action="store_true", help="per-stage times on stderr")
     return ap.parse_args()
 
 
@@ -144,6 +146,8 @@ def run_ours(args):
     import paper_2508_02401_gb300 as ckv
 
     wl = cs.workload(args.workload)
+    if args.layers:
+        wl = wl.with_(num_layers=args.layers)
     cfg = ckv.Config.from_workload(wl)
     batch = ckv.Batch(wl.cu_seqlens(), device=f"cuda:{local}")
     T, Hkv, nl = wl.total_tokens, wl.num_kv_heads, wl.num_layers
@@ -217,23 +221,55 @@ def run_ours(args):
     for l, d in enumerate(layers):
         launches_per_step += 4 + (1 if d["t_keep"] > 0 else 0)
 
-    # --- scoring stage (the dominant kernels): per-layer event timing on its stream
+    # --- scoring stage (the dominant kernels): a graph of every layer's ckv_score_window,
+    # timed with events on its stream; the average per layer is one pass-1 + pass-2 pair.
     hbm_peak, peak_kind = _peaks()
-    score_rows = torch.empty((int(cfg.head_mask[0].sum()), T), dtype=torch.float32, device="cuda")
-    reps = 5
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-          for _ in range(reps * nl)]
-    with torch.cuda.stream(stream):
-        for l, d in enumerate(layers):  # warm
-            ckv.ckv_score_window(cfg, l, batch, d["q"], d["k"], score_rows, ws, stream=stream)
-        for r in range(reps):
+    n_sel = int(cfg.head_mask[0].sum())
+    score_rows = [torch.empty((int(cfg.head_mask[l].sum()), T), dtype=torch.float32, device="cuda")
+                  for l in range(nl)]
+    pooled_rows = [torch.empty((Hkv, T), dtype=torch.float32, device="cuda") for _ in range(nl)]
+
+    def stage(fn):
+        with torch.cuda.stream(stream):
+            fn()
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            fn()
+        reps = 20
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            g.replay()
+            a.record(stream)
+            for _ in range(reps):
+                g.replay()
+            b.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / reps / nl  # ms per layer
+
+    def score_all():
+        for l, d in enumerate(layers):
+            ckv.ckv_score_window(cfg, l, batch, d["q"], d["k"], score_rows[l], ws, stream=stream)
+
+    score_ms = stage(score_all)
+    if args.breakdown:
+        def pool_all():
+            for l in range(nl):
+                ckv.ckv_pool(cfg, l, batch, score_rows[l], pooled_rows[l], stream=stream)
+
+        def select_all():
             for l, d in enumerate(layers):
-                a, b = ev[r * nl + l]
-                a.record(stream)
-                ckv.ckv_score_window(cfg, l, batch, d["q"], d["k"], score_rows, ws, stream=stream)
-                b.record(stream)
-    torch.cuda.synchronize()
-    score_ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
+                ckv.ckv_select_topk(cfg, l, batch, pooled_rows[l], d["idx"], d["cu_keep_dev"], ws,
+                                    stream=stream)
+
+        def gather_all():
+            for l, d in enumerate(layers):
+                ckv.ckv_gather_compact(cfg, batch, d["t_keep"], d["k"], d["v"], d["idx"],
+                                       d["cu_keep_dev"], d["k_out"], d["v_out"], ws, stream=stream)
+        parts = {"score": score_ms, "pool": stage(pool_all), "select": stage(select_all),
+                 "gather": stage(gather_all), "step": ms_per_step / nl}
+        print("per-layer stage times (us): " + ", ".join(f"{k}={v * 1e3:.2f}" for k, v in parts.items()),
+              file=sys.stderr, flush=True)
     k_bytes = T * Hkv * 256
     score_gbs = k_bytes / (score_ms / 1e3) / 1e9
     src = open(os.path.join(ROOT, "paper_2508_02401_gb300", "csrc", "score_kernel.cu"), "rb").read()

@@ -306,7 +306,7 @@ _W = [
              description="Llama-3.1-8B-shaped 32 layers, L=32768, w=32, maxpool 7, mean budget 1024"),
     Workload(name="needle_l131072", num_layers=32, num_q_heads=32, num_kv_heads=8,
              seqlens=(131072,), window=32, heads_per_group=2, budget_mean=128, budget_uniform=True,
-             outlier_channels=8, plant="span", plant_count=64, plant_beta=4.0, plant_noise=True,
+             outlier_channels=8, plant="span", plant_count=64, plant_beta=6.0, plant_noise=True,
              seed=20250802 + 3,
              description="needle-style L=131072, planted 64-token span, budget 128"),
     Workload(name="ragged_qwen7b", num_layers=28, num_q_heads=28, num_kv_heads=4,
