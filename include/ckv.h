@@ -168,6 +168,32 @@ CKV_API ckv_status ckv_compress_layer(const ckv_config* cfg, int32_t layer, cons
 CKV_API ckv_status ckv_read_device_status(void* workspace, ckv_stream stream, int32_t reset,
                                   int32_t* code, int32_t* detail);
 
+/* ckv_score_window for callers that cannot allocate device memory (no counterpart in the
+ * paper).  Some callers have no allocator to hand: code running inside a host-side engine
+ * whose memory pool is owned elsewhere, or code that must not grow the process's device
+ * footprint after start-up.  This variant takes no workspace.  Its scratch (the per-chunk
+ * softmax partials and a status word) is a fixed, file-scope device array of
+ * CKV_STATIC_SCRATCH_BYTES that every GPU loading the library holds until the process exits.
+ *   - Same arguments, results and layouts as ckv_score_window, minus the workspace.
+ *   - The first call on a device looks up the array's device address (once per device, with
+ *     that device current); make that first call before any stream capture.
+ *   - Calls whose work needs more scratch than the array holds (more than
+ *     CKV_STATIC_SCRATCH_ITEMS work items) return CKV_ERR_UNSUPPORTED before enqueuing
+ *     anything; ckv_score_window has no such limit.
+ *   - Every call shares the one array: calls that may overlap on the GPU (other streams,
+ *     other host threads) race and must be serialised by the caller.
+ *   - Each call clears the status word first.  If status_out (device, 2 x int32) is not NULL,
+ *     the call's device status (code, detail as in ckv_read_device_status) is copied there at
+ *     the end of the call, in stream order.
+ *   - Allocates nothing: no cudaMalloc, cudaFree or allocating library call. */
+#define CKV_STATIC_SCRATCH_ITEMS 1024
+#define CKV_STATIC_SCRATCH_BYTES (256 + CKV_STATIC_SCRATCH_ITEMS * 64 * 8)
+CKV_API ckv_status ckv_score_window_static(const ckv_config* cfg, int32_t layer,
+                                           const ckv_batch* batch, const void* q_win,
+                                           const void* k, int64_t tok_stride,
+                                           int64_t head_stride, float* scores,
+                                           int32_t* status_out, ckv_stream stream);
+
 #ifdef __cplusplus
 }
 #endif

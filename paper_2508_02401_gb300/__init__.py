@@ -18,7 +18,7 @@ __all__ = [
     "CkvError", "Config", "Batch", "lib_path", "load",
     "ckv_workspace_size", "ckv_keep_lengths", "ckv_score_window", "ckv_pool", "ckv_select_topk",
     "ckv_gather_compact", "ckv_compress_layer", "ckv_read_device_status", "ckv_status_string",
-    "ckv_abi_version", "POOL_MAX", "POOL_AVG", "POOL_THEN_SUM", "SUM_THEN_POOL",
+    "ckv_abi_version", "ckv_score_window_static", "POOL_MAX", "POOL_AVG", "POOL_THEN_SUM", "SUM_THEN_POOL",
 ]
 
 POOL_MAX, POOL_AVG = 0, 1
@@ -77,6 +77,7 @@ def load():
         "ckv_gather_compact": ([cfg, bat, I32, P, P, I64, I64, P, P, P, P, P, SZ, P], C.c_int),
         "ckv_compress_layer": ([cfg, I32, bat, P, P, P, I64, I64, P, P, P, P, P, P, SZ, P], C.c_int),
         "ckv_read_device_status": ([P, P, I32, C.POINTER(I32), C.POINTER(I32)], C.c_int),
+        "ckv_score_window_static": ([cfg, I32, bat, P, P, I64, I64, P, P, P], C.c_int),
     }
     for name, (args, res) in sigs.items():
         fn = getattr(lib, name)
@@ -222,6 +223,14 @@ def ckv_compress_layer(cfg, layer, batch, q_win, k, v, idx, cu_keep_dev, k_out, 
                                      _ptr(k_out), _ptr(v_out), _ptr(pooled_out), _ptr(workspace),
                                      workspace.numel() * workspace.element_size(), _stream(stream)),
            "ckv_compress_layer")
+
+
+def ckv_score_window_static(cfg, layer, batch, q_win, k, scores, status_out=None, stream=None,
+                            tok_stride=0, head_stride=0):
+    """ckv_score_window without a workspace: the library's fixed static scratch is used."""
+    _check(load().ckv_score_window_static(cfg.ref, layer, batch.ref, _ptr(q_win), _ptr(k),
+                                          tok_stride, head_stride, _ptr(scores), _ptr(status_out),
+                                          _stream(stream)), "ckv_score_window_static")
 
 
 def ckv_read_device_status(workspace, stream=None, reset=True):

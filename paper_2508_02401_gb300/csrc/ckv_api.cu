@@ -7,6 +7,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <mutex>
 #include <vector>
 
 #include "ckv.h"
@@ -551,6 +552,71 @@ ckv_status ckv_read_device_status(void* workspace, ckv_stream stream, int32_t re
     if (reset) {
         e = cudaMemset(workspace, 0, sizeof hdr);
         if (e != cudaSuccess) return cuda_fail(e, "clearing the status word");
+    }
+    return CKV_OK;
+}
+
+// ---------------------------------------------------------------------- no-allocation variant
+// The scratch of ckv_score_window_static: a status header followed by the per-chunk softmax
+// partials (float2 per window-row column, kMaxCols columns per work item).
+static __device__ __align__(256) unsigned char g_score_scratch[CKV_STATIC_SCRATCH_BYTES];
+
+namespace {
+constexpr int kMaxDevices = 64;
+std::once_flag g_scratch_once[kMaxDevices];
+void* g_scratch_addr[kMaxDevices] = {};
+cudaError_t g_scratch_err[kMaxDevices] = {};
+}  // namespace
+
+ckv_status ckv_score_window_static(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
+                                   const void* q_win, const void* k, int64_t tok_stride,
+                                   int64_t head_stride, float* scores, int32_t* status_out,
+                                   ckv_stream stream) {
+    static_assert(sizeof(WsHeader) == 256, "header");
+    Plan pl;
+    ckv_status st = make_plan(cfg, layer, pl);
+    if (st) return st;
+    int T = 0;
+    if ((st = check_batch(batch, &T)) || (st = resolve_strides(pl, &tok_stride, &head_stride)) ||
+        (st = check_kv(q_win, "q_win", T)) || (st = check_kv(k, "k", T)) ||
+        (st = check_kv(scores, "scores", T)))
+        return st;
+    if (status_out && !aligned(status_out, 4))
+        return fail(CKV_ERR_INVALID_ARG, "status_out is not 4-byte aligned");
+    int dev = -1;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (dev < 0 || dev >= kMaxDevices) return fail(CKV_ERR_UNSUPPORTED, "device index %d", dev);
+    int ctas = device_sm_count();
+    if (ctas <= 0) return cuda_fail(cudaGetLastError(), "querying the SM count");
+    ctas = std::min(ctas, kPartialCapacityItems);
+    int chunk_tiles = 0, n_items = 0;
+    choose_chunks(pl, batch, -1, ctas, &chunk_tiles, &n_items);
+    if (n_items > CKV_STATIC_SCRATCH_ITEMS)
+        return fail(CKV_ERR_UNSUPPORTED,
+                    "this batch needs %d scratch work items; the static scratch holds %d "
+                    "(use ckv_score_window with a workspace)", n_items, CKV_STATIC_SCRATCH_ITEMS);
+    // Once per device, with that device current: the device address of the scratch array.
+    std::call_once(g_scratch_once[dev], [dev] {
+        void* ptr = nullptr;
+        g_scratch_err[dev] = cudaGetSymbolAddress(&ptr, g_score_scratch);
+        g_scratch_addr[dev] = ptr;
+    });
+    if (g_scratch_err[dev] != cudaSuccess || !g_scratch_addr[dev])
+        return cuda_fail(g_scratch_err[dev], "cudaGetSymbolAddress of the static scratch");
+    void* scratch = g_scratch_addr[dev];
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    e = cudaMemsetAsync(scratch, 0, 2 * sizeof(int32_t), s);  // the status word starts at zero
+    if (e != cudaSuccess) return cuda_fail(e, "clearing the static status word");
+    WsLayout l;
+    l.header = 0;
+    l.partials = sizeof(WsHeader);
+    l.total = CKV_STATIC_SCRATCH_BYTES;
+    if ((st = enqueue_score(pl, batch, T, q_win, k, tok_stride, head_stride, scores, scratch, l, -1, s)))
+        return st;
+    if (status_out) {
+        e = cudaMemcpyAsync(status_out, scratch, 2 * sizeof(int32_t), cudaMemcpyDeviceToDevice, s);
+        if (e != cudaSuccess) return cuda_fail(e, "copying the static status word");
     }
     return CKV_OK;
 }
