@@ -435,6 +435,8 @@ ckv_status ckv_select_topk(const ckv_config* cfg, int32_t layer, const ckv_batch
     L.pooled = const_cast<float*>(pooled);
     L.idx = idx;
     L.cu_keep_dev = cu_keep_dev;
+    L.from_scores = 0;
+    L.write_pooled = 0;
     const cudaError_t e = launch_select(L, reinterpret_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? CKV_OK : cuda_fail(e, "launching the selection kernel");
 }
@@ -514,10 +516,10 @@ ckv_status ckv_compress_layer(const ckv_config* cfg, int32_t layer, const ckv_ba
     L.pooled = pooled;
     L.idx = idx;
     L.cu_keep_dev = cu_keep_dev;
-    cudaError_t e = launch_pool(L, s);
-    if (e != cudaSuccess) return cuda_fail(e, "launching the pooling kernel");
-    e = launch_select(L, s);
-    if (e != cudaSuccess) return cuda_fail(e, "launching the selection kernel");
+    L.from_scores = 1;                      // pooling is fused into the selection kernel
+    L.write_pooled = pooled_out != nullptr;
+    cudaError_t e = launch_select(L, s);
+    if (e != cudaSuccess) return cuda_fail(e, "launching the pool + selection kernel");
     if (tk == 0) return CKV_OK;
     GatherLaunch G;
     G.k = k;

@@ -41,6 +41,8 @@ struct SelectLaunch {
     int S, T, Hkv, w, budget, T_keep;
     int pool_kernel, pool_type, head_order;
     int skip_le;                // pooled is produced only for sequences with L > skip_le
+    int from_scores;            // select: pool the scores on the fly (else read pooled)
+    int write_pooled;           // select with from_scores: also store the pooled scores
     uint32_t cu_hash;
     const int* group_first;     // [H_kv+1] first score row of each group
 };

@@ -262,19 +262,29 @@ __global__ void __launch_bounds__(256, 1) score_kernel(const __grid_constant__ S
                 record_error(p.status, kDevTimeout, 10 * PASS + 2);
                 break;
             }
-            for (int e = tid; e < N * 16; e += 64) {
-                const int r = e >> 4, c = e & 15;
+            // Each thread owns one 16-byte column chunk c of rows r0, r0+4, ...: all of its
+            // loads are issued before any store, so their latencies overlap.
+            constexpr int kPer = N * 16 / 64;
+            const int c = tid & 15, r0 = tid >> 4;
+            uint4 vals[kPer];
+#pragma unroll
+            for (int i = 0; i < kPer; ++i) {
+                const int r = r0 + 4 * i;
                 const int slot = r / W_PAD, rr = r % W_PAD;
-                uint4 val = make_uint4(0u, 0u, 0u, 0u);
+                vals[i] = make_uint4(0u, 0u, 0u, 0u);
                 if (slot < I.nheads && rr < p.w) {
                     const int h = p.sel_heads[I.first + slot];
                     const uint4* src = reinterpret_cast<const uint4*>(
                         p.q_win + ((static_cast<size_t>(I.s) * p.w + rr) * p.Hq + h) * kHeadDim);
-                    val = __ldg(src + c);
+                    vals[i] = __ldg(src + c);
                 }
+            }
+#pragma unroll
+            for (int i = 0; i < kPer; ++i) {
+                const int r = r0 + 4 * i;
                 const int half = c >> 3, cc = c & 7;
                 *reinterpret_cast<uint4*>(qbuf + half * SL::kQHalf + r * 128 +
-                                          ((cc ^ (r & 7)) << 4)) = val;
+                                          ((cc ^ (r & 7)) << 4)) = vals[i];
             }
             fence_proxy_async_smem();
             mbar_arrive(q_full);
@@ -307,8 +317,22 @@ __global__ void __launch_bounds__(256, 1) score_kernel(const __grid_constant__ S
                 named_bar_sync(1, 128);  // previous item's readers of lse_s are done
                 if (tid < N) {
                     float M = -INFINITY, S = 0.f;
-                    for (int k = 0; k < I.nchunks && I.unit_base + k < p.n_items; ++k) {
-                        const float2 pr = p.partials[static_cast<size_t>(I.unit_base + k) * N + tid];
+                    const int n = min(I.nchunks, p.n_items - I.unit_base);
+                    const float2* src = p.partials + static_cast<size_t>(I.unit_base) * N + tid;
+                    int k = 0;
+                    for (; k + 4 <= n; k += 4) {  // four independent loads in flight
+                        float2 pr[4];
+#pragma unroll
+                        for (int u = 0; u < 4; ++u) pr[u] = src[static_cast<size_t>(k + u) * N];
+#pragma unroll
+                        for (int u = 0; u < 4; ++u) {
+                            const float Mn = fmaxf(M, pr[u].x);
+                            S = S * ex2_approx(M - Mn) + pr[u].y * ex2_approx(pr[u].x - Mn);
+                            M = Mn;
+                        }
+                    }
+                    for (; k < n; ++k) {
+                        const float2 pr = src[static_cast<size_t>(k) * N];
                         const float Mn = fmaxf(M, pr.x);
                         S = S * ex2_approx(M - Mn) + pr.y * ex2_approx(pr.x - Mn);
                         M = Mn;
@@ -415,11 +439,30 @@ __global__ void __launch_bounds__(256, 1) score_kernel(const __grid_constant__ S
 
             if constexpr (PASS == 1) {
                 // Combine the 128 threads' (max, sum) per column and write the chunk partial.
+                // Level-major butterflies over 32 columns at a time, so the shuffles of
+                // different columns overlap instead of forming one long dependent chain.
 #pragma unroll
-                for (int c = 0; c < N; ++c) {
-                    const float M = warp_max(st_a[c]);
-                    const float Ls = warp_sum(st_b[c] * ex2_approx(st_a[c] - M));
-                    if (lane == 0) red[eq * N + c] = make_float2(M, Ls);
+                for (int hc = 0; hc < N / 32; ++hc) {
+                    float M[32];
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) M[i] = st_a[hc * 32 + i];
+#pragma unroll
+                    for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+                        for (int i = 0; i < 32; ++i)
+                            M[i] = fmaxf(M[i], __shfl_xor_sync(0xffffffffu, M[i], o));
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) st_b[hc * 32 + i] *= ex2_approx(st_a[hc * 32 + i] - M[i]);
+#pragma unroll
+                    for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+                        for (int i = 0; i < 32; ++i)
+                            st_b[hc * 32 + i] += __shfl_xor_sync(0xffffffffu, st_b[hc * 32 + i], o);
+                    if (lane == 0) {
+#pragma unroll
+                        for (int i = 0; i < 32; ++i)
+                            red[eq * N + hc * 32 + i] = make_float2(M[i], st_b[hc * 32 + i]);
+                    }
                 }
                 named_bar_sync(1, 128);
                 if (tid < N) {

@@ -67,16 +67,24 @@ __global__ void __launch_bounds__(256) pool_kernel(const __grid_constant__ PoolP
 }
 
 struct SelectParams {
-    const float* pooled;
+    const float* scores;   // [n_sel, T]: pooled on the fly when from_scores != 0
+    float* pooled;         // [H_kv, T]: read when from_scores == 0, else written if write_pooled
     int32_t* idx;
     int32_t* cu_keep;
     const int32_t* cu_seqlens;
     int* status;
     int S, T, Hkv, w, budget, T_keep;
+    int pool_kernel, pool_type, head_order, from_scores, write_pooled;
     uint32_t cu_hash;
+    int16_t group_first[kMaxQHeads + 1];
 };
 
 constexpr int kSelThreads = 1024;
+constexpr int kSelWarps = kSelThreads / 32;
+constexpr int kPoolTile = 8192;                         // candidate positions pooled per round
+constexpr int kMaxHalo = kMaxPoolKernel / 2;
+constexpr int kResidentKeys = 40960;                    // candidates kept in shared memory
+constexpr int kSelSmemBytes = (kResidentKeys + kPoolTile + 2 * kMaxHalo) * 4;
 
 // Order-preserving key of a non-negative float (-0 maps to +0).
 __device__ __forceinline__ uint32_t rank_key(float f) {
@@ -84,37 +92,48 @@ __device__ __forceinline__ uint32_t rank_key(float f) {
     return u == 0x80000000u ? 0u : u;
 }
 
-// Block-wide exclusive count of `flag` in thread order; returns the rank, *total the sum.
-__device__ __forceinline__ int block_rank(bool flag, int* warp_tot, int* total) {
+// Block-wide exclusive prefix sum of v in thread order; *total gets the block's sum.
+__device__ __forceinline__ int block_excl_scan(int v, int* scratch, int* total) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const unsigned bal = __ballot_sync(0xffffffffu, flag);
-    const int in_warp = __popc(bal & ((1u << lane) - 1u));
-    if (lane == 0) warp_tot[warp] = __popc(bal);
+    int incl = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+    }
+    if (lane == 31) scratch[warp] = incl;
     __syncthreads();
     if (warp == 0) {
-        const int x = warp_tot[lane];
-        int incl = x;
+        const int x = lane < kSelWarps ? scratch[lane] : 0;
+        int wincl = x;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
-            const int y = __shfl_up_sync(0xffffffffu, incl, o);
-            if (lane >= o) incl += y;
+            const int y = __shfl_up_sync(0xffffffffu, wincl, o);
+            if (lane >= o) wincl += y;
         }
-        warp_tot[lane] = incl - x;                    // exclusive warp offsets
-        if (lane == 31) warp_tot[32] = incl;          // block total
+        if (lane < kSelWarps) scratch[lane] = wincl - x;
+        if (lane == 31) scratch[32] = wincl;
     }
     __syncthreads();
-    const int r = warp_tot[warp] + in_warp;
-    *total = warp_tot[32];
+    const int r = scratch[warp] + incl - v;
+    *total = scratch[32];
     __syncthreads();
     return r;
 }
 
-// One block per (sequence, KV head): radix select of the k-th largest pooled score (8-bit
-// digits, most significant first), then a stable, position-ordered compaction that takes
-// every score above the threshold and the lowest-positioned ties, then the window.
-__global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_constant__ SelectParams p) {
+// One block per (sequence, KV head):
+//   1. pooling of the selected heads' window scores along the candidate positions (max or avg,
+//      zero padding outside [0, P)), in either head order, staged through shared memory;
+//   2. radix select of the k-th largest pooled score (8-bit digits, most significant first)
+//      over shared-memory keys;
+//   3. a stable, position-ordered compaction: every candidate above the threshold and the
+//      lowest-positioned ties, then the window positions.
+__global__ void __launch_bounds__(kSelThreads, 1) pool_select_kernel(const __grid_constant__ SelectParams p) {
+    extern __shared__ uint32_t sel_smem[];
+    uint32_t* keys = sel_smem;                                               // [kResidentKeys]
+    float* stage = reinterpret_cast<float*>(sel_smem + kResidentKeys);       // [kPoolTile + 2*halo]
     __shared__ int hist[256];
-    __shared__ int warp_tot[33];
+    __shared__ int scratch[33];
     __shared__ int s_digit, s_above;
 
     const int s = blockIdx.x / p.Hkv, g = blockIdx.x % p.Hkv;
@@ -126,7 +145,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
     int keep_off = 0;
     for (int u = 0; u < s; ++u) keep_off += min(p.budget, p.cu_seqlens[u + 1] - p.cu_seqlens[u]);
     const int n_keep = min(p.budget, L);
-    if (L < 0 || keep_off + n_keep > p.T_keep || t0 + L > p.T) {
+    if (L < 0 || t0 < 0 || keep_off < 0 || keep_off + n_keep > p.T_keep || t0 + L > p.T) {
         if (tid == 0) record_error(p.status, kDevBadSeqlens, 200 + s);
         return;
     }
@@ -135,21 +154,92 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
         if (s == 0) p.cu_keep[0] = 0;
     }
     int32_t* out = p.idx + static_cast<size_t>(g) * p.T_keep + keep_off;
+    float* pooled = p.pooled ? p.pooled + static_cast<size_t>(g) * p.T + t0 : nullptr;
     if (L <= p.budget) {
-        for (int i = tid; i < L; i += kSelThreads) out[i] = i;
+        for (int i = tid; i < L; i += kSelThreads) {
+            out[i] = i;
+            if (p.from_scores && p.write_pooled) pooled[i] = 0.f;
+        }
         return;
     }
     const int P = L - p.w, k = p.budget - p.w;
-    const float* c = p.pooled + static_cast<size_t>(g) * p.T + t0;
+    const bool resident = P <= kResidentKeys;
+
+    // ---------------------------------------------------------------- 1. pooling
+    if (p.from_scores) {
+        const int half = p.pool_kernel >> 1;
+        const bool is_max = p.pool_type == 0;
+        const float kf = static_cast<float>(p.pool_kernel);
+        const int r0 = p.group_first[g], r1 = p.group_first[g + 1];
+        const float* base = p.scores + t0;
+        for (int tile0 = 0; tile0 < P; tile0 += kPoolTile) {
+            const int n = min(kPoolTile, P - tile0);
+            constexpr int kPer = kPoolTile / kSelThreads;
+            float acc[kPer];
+#pragma unroll
+            for (int i = 0; i < kPer; ++i) acc[i] = 0.f;
+            const int passes = p.head_order == 0 ? r1 - r0 : 1;
+            for (int ps = 0; ps < passes; ++ps) {
+                // stage positions tile0-half .. tile0+n+half (zeros outside [0, P))
+                for (int e = tid; e < n + 2 * half; e += kSelThreads) {
+                    const int u = tile0 - half + e;
+                    float x = 0.f;
+                    if (u >= 0 && u < P) {
+                        if (p.head_order == 0) {
+                            x = __ldg(base + static_cast<size_t>(r0 + ps) * p.T + u);
+                        } else {
+                            for (int r = r0; r < r1; ++r) x += __ldg(base + static_cast<size_t>(r) * p.T + u);
+                        }
+                    }
+                    stage[e] = x;
+                }
+                __syncthreads();
+#pragma unroll
+                for (int i = 0; i < kPer; ++i) {
+                    const int jl = tid + i * kSelThreads;  // window is stage[jl .. jl + 2*half]
+                    if (jl < n) {
+                        float m = stage[jl];
+                        if (is_max) {
+                            for (int t = 1; t <= 2 * half; ++t) m = fmaxf(m, stage[jl + t]);
+                            acc[i] += m;
+                        } else {
+                            for (int t = 1; t <= 2 * half; ++t) m += stage[jl + t];
+                            acc[i] += m / kf;  // IEEE division, as in pool_kernel
+                        }
+                    }
+                }
+                __syncthreads();
+            }
+#pragma unroll
+            for (int i = 0; i < kPer; ++i) {
+                const int jl = tid + i * kSelThreads;
+                if (jl < n) {
+                    if (resident) keys[tile0 + jl] = rank_key(acc[i]);
+                    if (p.write_pooled || !resident) pooled[tile0 + jl] = acc[i];
+                }
+            }
+        }
+        if (p.write_pooled)
+            for (int j = P + tid; j < L; j += kSelThreads) pooled[j] = 0.f;
+    } else if (resident) {
+        for (int j = tid; j < P; j += kSelThreads) keys[j] = rank_key(__ldg(pooled + j));
+    }
+    __syncthreads();
+    // keys are either resident in shared memory or re-read from the pooled scores in global
+    // memory (written above, visible to the block after the barrier)
+    auto key_at = [&](int j) -> uint32_t {
+        return resident ? keys[j] : rank_key(pooled[j]);
+    };
 
     if (k > 0) {
+        // ------------------------------------------------------------ 2. radix select
         uint32_t prefix = 0, mask = 0;
         int remaining = k;
         for (int shift = 24; shift >= 0; shift -= 8) {
             if (tid < 256) hist[tid] = 0;
             __syncthreads();
             for (int j = tid; j < P; j += kSelThreads) {
-                const uint32_t u = rank_key(__ldg(c + j));
+                const uint32_t u = key_at(j);
                 if ((u & mask) == prefix) atomicAdd(&hist[(u >> shift) & 255u], 1);
             }
             __syncthreads();
@@ -165,9 +255,8 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
                     const int y = __shfl_down_sync(0xffffffffu, above, o);
                     if (tid + o < 32) above += y;
                 }
-                const int strictly_above = above - local;  // bins of higher lanes
-                const bool here = strictly_above < remaining && above >= remaining;
-                if (here) {
+                const int strictly_above = above - local;
+                if (strictly_above < remaining && above >= remaining) {
                     int acc = strictly_above;
                     for (int b = 7; b >= 0; --b) {
                         const int h = hist[tid * 8 + b];
@@ -186,24 +275,29 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
             remaining -= s_above;
             __syncthreads();
         }
-        const uint32_t thr = prefix;  // the k-th largest key
+        const uint32_t thr = prefix;    // the k-th largest key
         const int need_eq = remaining;  // ties at the threshold that are kept
-        int written = 0, eq_seen = 0;
-        for (int j0 = 0; j0 < P; j0 += kSelThreads) {
-            const int j = j0 + tid;
-            const uint32_t u = j < P ? rank_key(__ldg(c + j)) : 0u;
-            const bool gt = j < P && u > thr;
-            const bool eq = j < P && u == thr;
-            int eq_tot;
-            const int eq_rank = block_rank(eq, warp_tot, &eq_tot);
-            const bool take = gt || (eq && eq_seen + eq_rank < need_eq);
-            int take_tot;
-            const int out_rank = block_rank(take, warp_tot, &take_tot);
-            if (take && written + out_rank < k) out[written + out_rank] = j;
-            written += take_tot;
-            eq_seen += eq_tot;
+
+        // ------------------------------------------------------------ 3. compaction
+        const int seg = (P + kSelThreads - 1) / kSelThreads;
+        const int j0 = min(P, tid * seg), j1 = min(P, j0 + seg);
+        int n_gt = 0, n_eq = 0;
+        for (int j = j0; j < j1; ++j) {
+            const uint32_t u = key_at(j);
+            n_gt += u > thr;
+            n_eq += u == thr;
         }
-        if (tid == 0 && written != k) record_error(p.status, kDevBadIndex, 300 + blockIdx.x);
+        int tot;
+        const int eq_before = block_excl_scan(n_eq, scratch, &tot);
+        const int eq_take = max(0, min(n_eq, need_eq - eq_before));
+        const int out_before = block_excl_scan(n_gt + eq_take, scratch, &tot);
+        if (tid == 0 && tot != k) record_error(p.status, kDevBadIndex, 300 + blockIdx.x);
+        int o = out_before, eq_seen = 0;
+        for (int j = j0; j < j1; ++j) {
+            const uint32_t u = key_at(j);
+            const bool take = u > thr || (u == thr && eq_seen++ < eq_take);
+            if (take && o < k) out[o++] = j;
+        }
     }
     for (int i = tid; i < p.w; i += kSelThreads) out[k + i] = P + i;
 }
@@ -268,6 +362,7 @@ cudaError_t launch_pool(const SelectLaunch& L, cudaStream_t stream) {
 
 cudaError_t launch_select(const SelectLaunch& L, cudaStream_t stream) {
     SelectParams p;
+    p.scores = L.scores;
     p.pooled = L.pooled;
     p.idx = L.idx;
     p.cu_keep = L.cu_keep_dev;
@@ -279,8 +374,21 @@ cudaError_t launch_select(const SelectLaunch& L, cudaStream_t stream) {
     p.w = L.w;
     p.budget = L.budget;
     p.T_keep = L.T_keep;
+    p.pool_kernel = L.pool_kernel;
+    p.pool_type = L.pool_type;
+    p.head_order = L.head_order;
+    p.from_scores = L.from_scores;
+    p.write_pooled = L.write_pooled;
     p.cu_hash = L.cu_hash;
-    select_kernel<<<L.S * L.Hkv, kSelThreads, 0, stream>>>(p);
+    for (int g = 0; g <= L.Hkv; ++g) p.group_first[g] = static_cast<int16_t>(L.group_first[g]);
+    static bool configured = false;
+    if (!configured) {
+        cudaError_t e = cudaFuncSetAttribute(pool_select_kernel,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, kSelSmemBytes);
+        if (e != cudaSuccess) return e;
+        configured = true;
+    }
+    pool_select_kernel<<<L.S * L.Hkv, kSelThreads, kSelSmemBytes, stream>>>(p);
     return cudaGetLastError();
 }
 
