@@ -172,7 +172,8 @@ CKV_API ckv_status ckv_read_device_status(void* workspace, ckv_stream stream, in
  * paper).  Some callers have no allocator to hand: code running inside a host-side engine
  * whose memory pool is owned elsewhere, or code that must not grow the process's device
  * footprint after start-up.  This variant takes no workspace.  Its scratch (the per-chunk
- * softmax partials and a status word) is a fixed, file-scope device array of
+ * softmax partials, per-unit arrival counters and a status word) is a fixed, file-scope
+ * device array of
  * CKV_STATIC_SCRATCH_BYTES that every GPU loading the library holds until the process exits.
  *   - Same arguments, results and layouts as ckv_score_window, minus the workspace.
  *   - The first call on a device looks up the array's device address (once per device, with
@@ -187,7 +188,7 @@ CKV_API ckv_status ckv_read_device_status(void* workspace, ckv_stream stream, in
  *     the end of the call, in stream order.
  *   - Allocates nothing: no cudaMalloc, cudaFree or allocating library call. */
 #define CKV_STATIC_SCRATCH_ITEMS 1024
-#define CKV_STATIC_SCRATCH_BYTES (256 + CKV_STATIC_SCRATCH_ITEMS * 64 * 8)
+#define CKV_STATIC_SCRATCH_BYTES (256 + CKV_STATIC_SCRATCH_ITEMS * 64 * 8 + 2048)
 CKV_API ckv_status ckv_score_window_static(const ckv_config* cfg, int32_t layer,
                                            const ckv_batch* batch, const void* q_win,
                                            const void* k, int64_t tok_stride,

@@ -34,7 +34,6 @@ ckv_status cuda_fail(cudaError_t e, const char* what) {
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
 constexpr size_t kWsAlign = 256;
-constexpr int kPartialCapacityItems = 1024;  // >= the SM count of any supported GPU
 
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
@@ -141,53 +140,124 @@ int64_t keep_total(const ckv_batch* b, int budget) {
     return t;
 }
 
-int count_units(const Plan& pl, const ckv_batch* b, int skip_le) {
-    int n = 0;
-    for (int s = 0; s < b->num_seqs; ++s) {
-        const int L = b->cu_seqlens_host[s + 1] - b->cu_seqlens_host[s];
-        if (L > skip_le && L > 0) n += pl.nb;
-    }
-    return n;
-}
-
-// Smallest chunk (in key tiles) that yields at most `ctas` work items.
-void choose_chunks(const Plan& pl, const ckv_batch* b, int skip_le, int ctas, int* chunk_tiles,
-                   int* n_items) {
-    std::vector<int> tiles;
-    for (int s = 0; s < b->num_seqs; ++s) {
-        const int L = b->cu_seqlens_host[s + 1] - b->cu_seqlens_host[s];
-        if (L > skip_le && L > 0) tiles.push_back((L + kTileKeys - 1) / kTileKeys);
-    }
-    if (tiles.empty()) {
-        *chunk_tiles = 1;
-        *n_items = 0;
-        return;
-    }
-    auto count = [&](int C) {
-        long long n = 0;
-        for (int t : tiles) n += (t + C - 1) / C;
-        return n * pl.nb;
+// Splits every (sequence, head batch) unit's key tiles into items of at most `c` tiles and
+// packs units whole into rounds of at most `ctas` items; `c` minimises an estimate of the
+// launch's time: per round, the longest item, plus the tiles of it that do not stay resident
+// in the kernel's shared-memory slots (they are loaded a second time), plus a fixed cost.
+ckv_status plan_score(const Plan& pl, const ckv_batch* b, int skip_le, int ctas, ScoreLaunch& L,
+                      int max_items_per_launch) {
+    struct RawUnit {
+        int seq, start, len, batch, tiles;
     };
-    int lo = 1, hi = *std::max_element(tiles.begin(), tiles.end());
-    while (lo < hi) {
-        const int mid = (lo + hi) / 2;
-        if (count(mid) <= ctas) hi = mid;
-        else lo = mid + 1;
+    std::vector<RawUnit> raw;
+    int max_tiles = 0;
+    for (int s = 0; s < b->num_seqs; ++s) {
+        const int t0 = b->cu_seqlens_host[s];
+        const int len = b->cu_seqlens_host[s + 1] - t0;
+        if (len <= skip_le || len <= 0) continue;
+        const int tiles = (len + kTileKeys - 1) / kTileKeys;
+        max_tiles = std::max(max_tiles, tiles);
+        for (int bt = 0; bt < pl.nb; ++bt) raw.push_back({s, t0, len, bt, tiles});
     }
-    *chunk_tiles = lo;
-    *n_items = static_cast<int>(count(lo));
+    L.items.clear();
+    L.units.clear();
+    L.slices.clear();
+    if (raw.empty()) return CKV_OK;
+    if (b->num_seqs > 65535) return fail(CKV_ERR_UNSUPPORTED, "more than 65535 sequences");
+    constexpr int kResident = 6, kFixed = 3;
+    int best_c = -1;
+    long long best_cost = 0;
+    for (int c = 1; c <= max_tiles; ++c) {
+        long long rounds = 0;
+        int cur = 0;
+        bool feasible = c <= 65535;
+        for (const RawUnit& u : raw) {
+            const int n = (u.tiles + c - 1) / c;
+            if (n > ctas) {
+                feasible = false;
+                break;
+            }
+            if (cur + n > ctas) {
+                ++rounds;
+                cur = 0;
+            }
+            cur += n;
+        }
+        if (!feasible) continue;
+        rounds += cur > 0;
+        const long long cost = rounds * (c + std::max(0, c - kResident) + kFixed);
+        if (best_c < 0 || cost < best_cost) {
+            best_c = c;
+            best_cost = cost;
+        }
+    }
+    if (best_c < 0) return fail(CKV_ERR_UNSUPPORTED, "cannot partition the scoring work");
+    // Rounds of units; the grid is the largest round.
+    std::vector<std::vector<int>> rounds(1);
+    std::vector<int> round_items(1, 0);
+    for (int ui = 0; ui < static_cast<int>(raw.size()); ++ui) {
+        const int n = (raw[ui].tiles + best_c - 1) / best_c;
+        if (round_items.back() + n > ctas) {
+            rounds.emplace_back();
+            round_items.push_back(0);
+        }
+        rounds.back().push_back(ui);
+        round_items.back() += n;
+    }
+    const int grid = *std::max_element(round_items.begin(), round_items.end());
+    if (grid > max_items_per_launch) return fail(CKV_ERR_UNSUPPORTED, "scoring grid too large");
+    L.grid = grid;
+    // Slices of consecutive rounds that fit one launch's item and unit tables.
+    ScoreSlice cur{0, 0, 0, 0};
+    for (size_t r = 0; r < rounds.size(); ++r) {
+        const int nu = static_cast<int>(rounds[r].size());
+        if (cur.n_rounds > 0 && ((cur.n_rounds + 1) * grid > max_items_per_launch ||
+                                 cur.n_units + nu > kMaxScoreUnits)) {
+            L.slices.push_back(cur);
+            cur = ScoreSlice{static_cast<int>(L.items.size()), 0, static_cast<int>(L.units.size()), 0};
+        }
+        if (nu > kMaxScoreUnits) return fail(CKV_ERR_UNSUPPORTED, "too many scoring units in a round");
+        int slot = 0;
+        for (int ui : rounds[r]) {
+            const RawUnit& u = raw[ui];
+            const int n = (u.tiles + best_c - 1) / best_c;
+            ScoreUnit su;
+            su.seq_start = u.start;
+            su.len = u.len;
+            su.seq = static_cast<uint16_t>(u.seq);
+            su.batch = static_cast<uint16_t>(u.batch);
+            su.first_item = static_cast<uint16_t>(cur.n_rounds * grid + slot);
+            su.nitems = static_cast<uint16_t>(n);
+            const int uidx = cur.n_units;
+            L.units.push_back(su);
+            ++cur.n_units;
+            for (int k = 0; k < n; ++k, ++slot) {
+                ScoreItem it;
+                it.unit = static_cast<uint16_t>(uidx);
+                it.tile0 = static_cast<uint32_t>(k * best_c);
+                it.ntiles = static_cast<uint16_t>(std::min(best_c, u.tiles - k * best_c));
+                L.items.push_back(it);
+            }
+        }
+        for (; slot < grid; ++slot) L.items.push_back(ScoreItem{0, 0, 0});
+        ++cur.n_rounds;
+    }
+    L.slices.push_back(cur);
+    return CKV_OK;
 }
 
 struct WsLayout {
-    size_t header = 0, partials = 0, scores = 0, pooled = 0, total = 0;
+    size_t header = 0, partials = 0, counters = 0, scores = 0, pooled = 0, total = 0;
 };
 
 WsLayout ws_layout(const Plan& pl, const ckv_batch* b, int T) {
+    (void)b;
     WsLayout l;
     size_t off = round_up(sizeof(WsHeader), kWsAlign);
-    const size_t items = std::max(kPartialCapacityItems, count_units(pl, b, -1));
     l.partials = off;
-    off = round_up(off + items * kMaxCols * sizeof(float2), kWsAlign);
+    off = round_up(off + static_cast<size_t>(kMaxScoreItems) * kMaxCols * sizeof(float2), kWsAlign);
+    l.counters = off;
+    off = round_up(off + kMaxScoreUnits * sizeof(int), kWsAlign);
     l.scores = off;
     off = round_up(off + static_cast<size_t>(pl.n_sel) * T * sizeof(float), kWsAlign);
     l.pooled = off;
@@ -274,20 +344,21 @@ namespace {
 
 ckv_status enqueue_score(const Plan& pl, const ckv_batch* b, int T, const void* q_win,
                          const void* k, int64_t tok, int64_t head, float* scores, void* ws,
-                         const WsLayout& l, int skip_le, cudaStream_t stream) {
+                         const WsLayout& l, int skip_le, cudaStream_t stream,
+                         int max_items_per_launch = kMaxScoreItems) {
     int ctas = device_sm_count();
     if (ctas <= 0) return cuda_fail(cudaGetLastError(), "querying the SM count");
-    ctas = std::min(ctas, kPartialCapacityItems);
-    ScoreLaunch L;
-    memset(&L, 0, sizeof L);
-    choose_chunks(pl, b, skip_le, ctas, &L.chunk_tiles, &L.n_items);
-    if (L.n_items == 0) return CKV_OK;
-    ckv_status st = make_k_map(&L.tmap_k, k, pl.Hkv, T, tok, head);
+    static thread_local ScoreLaunch L;  // reused: keeps the plan's vectors allocated
+    ckv_status st = plan_score(pl, b, skip_le, std::min(ctas, max_items_per_launch), L,
+                               max_items_per_launch);
     if (st) return st;
+    if (L.slices.empty()) return CKV_OK;
+    if ((st = make_k_map(&L.tmap_k, k, pl.Hkv, T, tok, head))) return st;
     uint8_t* w8 = static_cast<uint8_t*>(ws);
     L.q_win = q_win;
     L.cu_seqlens_dev = b->cu_seqlens_dev;
     L.partials = w8 + l.partials;
+    L.counters = reinterpret_cast<int*>(w8 + l.counters);
     L.scores = scores;
     L.status = reinterpret_cast<int*>(w8);
     L.S = b->num_seqs;
@@ -297,8 +368,6 @@ ckv_status enqueue_score(const Plan& pl, const ckv_batch* b, int T, const void* 
     L.w_pad = pl.w_pad;
     L.n_cols = pl.n_cols;
     L.nb = pl.nb;
-    L.grid = ctas;
-    L.skip_le = skip_le;
     L.cu_hash = seqlens_hash(b->cu_seqlens_host, b->num_seqs);
     L.softmax_scale = pl.scale;
     L.n_sel = pl.n_sel;
@@ -307,7 +376,7 @@ ckv_status enqueue_score(const Plan& pl, const ckv_batch* b, int T, const void* 
     L.batch_nheads = pl.batch_nheads.data();
     L.sel_heads = pl.sel_heads.data();
     const cudaError_t e = launch_score(L, stream);
-    if (e != cudaSuccess) return cuda_fail(e, "launching the scoring kernels");
+    if (e != cudaSuccess) return cuda_fail(e, "launching the scoring kernel");
     return CKV_OK;
 }
 
@@ -591,13 +660,17 @@ ckv_status ckv_score_window_static(const ckv_config* cfg, int32_t layer, const c
     if (dev < 0 || dev >= kMaxDevices) return fail(CKV_ERR_UNSUPPORTED, "device index %d", dev);
     int ctas = device_sm_count();
     if (ctas <= 0) return cuda_fail(cudaGetLastError(), "querying the SM count");
-    ctas = std::min(ctas, kPartialCapacityItems);
-    int chunk_tiles = 0, n_items = 0;
-    choose_chunks(pl, batch, -1, ctas, &chunk_tiles, &n_items);
-    if (n_items > CKV_STATIC_SCRATCH_ITEMS)
-        return fail(CKV_ERR_UNSUPPORTED,
-                    "this batch needs %d scratch work items; the static scratch holds %d "
-                    "(use ckv_score_window with a workspace)", n_items, CKV_STATIC_SCRATCH_ITEMS);
+    {
+        static thread_local ScoreLaunch probe;
+        if ((st = plan_score(pl, batch, -1, std::min(ctas, CKV_STATIC_SCRATCH_ITEMS), probe,
+                             CKV_STATIC_SCRATCH_ITEMS)))
+            return st;
+        const int n_items = static_cast<int>(probe.items.size());
+        if (n_items > CKV_STATIC_SCRATCH_ITEMS)
+            return fail(CKV_ERR_UNSUPPORTED,
+                        "this batch needs %d scratch work items; the static scratch holds %d "
+                        "(use ckv_score_window with a workspace)", n_items, CKV_STATIC_SCRATCH_ITEMS);
+    }
     // Once per device, with that device current: the device address of the scratch array.
     std::call_once(g_scratch_once[dev], [dev] {
         void* ptr = nullptr;
@@ -613,8 +686,10 @@ ckv_status ckv_score_window_static(const ckv_config* cfg, int32_t layer, const c
     WsLayout l;
     l.header = 0;
     l.partials = sizeof(WsHeader);
+    l.counters = l.partials + static_cast<size_t>(CKV_STATIC_SCRATCH_ITEMS) * kMaxCols * sizeof(float2);
     l.total = CKV_STATIC_SCRATCH_BYTES;
-    if ((st = enqueue_score(pl, batch, T, q_win, k, tok_stride, head_stride, scores, scratch, l, -1, s)))
+    if ((st = enqueue_score(pl, batch, T, q_win, k, tok_stride, head_stride, scores, scratch, l, -1, s,
+                            CKV_STATIC_SCRATCH_ITEMS)))
         return st;
     if (status_out) {
         e = cudaMemcpyAsync(status_out, scratch, 2 * sizeof(int32_t), cudaMemcpyDeviceToDevice, s);

@@ -6,21 +6,46 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#include <vector>
+
 namespace ckv {
 
-// One scoring launch pair (pass 1 -> partials, pass 2 -> scores).
+// A scoring work item: `ntiles` key tiles (128 keys each) of one unit, from tile `tile0`.
+struct ScoreItem {
+    uint16_t unit;     // index into the launch's unit table
+    uint16_t ntiles;   // 0 = no work (round padding)
+    uint32_t tile0;
+};
+// A scoring unit: one sequence x one batch of selected heads of a KV group.  Its items are
+// contiguous in the item table and all belong to the same round.
+struct ScoreUnit {
+    int32_t seq_start;
+    int32_t len;
+    uint16_t seq;
+    uint16_t batch;
+    uint16_t first_item;  // relative to the launch
+    uint16_t nitems;
+};
+constexpr int kMaxScoreItems = 2048;  // per launch (kernel-parameter table)
+constexpr int kMaxScoreUnits = 384;
+
+// A contiguous run of rounds that is launched together.
+struct ScoreSlice {
+    int item0, n_rounds, unit0, n_units;
+};
+
 struct ScoreLaunch {
     CUtensorMap tmap_k;
     const void* q_win;
     const int32_t* cu_seqlens_dev;
-    void* partials;        // float2 [n_items, n_cols]
+    void* partials;        // float2 [items per launch, n_cols]
+    int* counters;         // [units per launch]
     float* scores;         // [n_sel, T]
     int* status;
     int S, T, Hq, w;
     int w_pad, n_cols;     // rows per head in the MMA (8/16/32/64), MMA N (32/64)
     int nb;                // head batches
-    int n_items, chunk_tiles, grid;
-    int skip_le;           // sequences with L <= skip_le are skipped (-1: none)
+    int grid;              // CTAs (= items per round)
     uint32_t cu_hash;      // seqlens_hash of the host copy of cu_seqlens
     float softmax_scale;
     int n_sel;
@@ -28,6 +53,9 @@ struct ScoreLaunch {
     const int* batch_first;
     const int* batch_nheads;
     const int* sel_heads;
+    std::vector<ScoreItem> items;   // rounds x grid, units' items contiguous
+    std::vector<ScoreUnit> units;   // first_item relative to the unit's slice
+    std::vector<ScoreSlice> slices;
 };
 cudaError_t launch_score(const ScoreLaunch& L, cudaStream_t stream);
 

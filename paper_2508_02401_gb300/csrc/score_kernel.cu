@@ -3,145 +3,178 @@
 //   a_h[j] = sum_{r < w, j <= P+r} exp(s_{h,r,j} - lse_{h,r}),   s_{h,r,j} = scale * q_{h,r}.k_j
 //
 // for every selected head h of a KV group, every window row r and every key j of a sequence
-// (P = L - w).  The row normalisers lse need all keys before any probability can be summed
-// over rows, so the work runs as two launches over the same decomposition:
+// (P = L - w).  A row's normaliser lse needs every key before any probability can be summed
+// over rows, so each key tile is used twice -- once for the row statistics, once for the
+// probabilities -- and kept in shared memory in between.
 //
-//   pass 1: per chunk of keys, per window row: running (max, sum of 2^(x - max)) -> partials
-//   pass 2: per chunk: combine the unit's partials into lse, recompute the logits and write
-//           the window-summed probabilities a_h (the chunk's keys are usually still in L2).
+// One cooperative launch; one CTA per SM, 384 threads, warp-specialised:
+//   warp 0      TMA producer: 128-key x 128-dim bf16 tiles of K (two 128-byte-swizzled boxes of
+//               64 dims) into kSlots shared-memory slots; tile i of an item lives in slot
+//               i % kSlots;
+//   warp 1      allocates TMEM and issues tcgen05.mma (M = 128 keys, N = the window rows of a
+//               batch of heads, K = 128) into two TMEM accumulators;
+//   warps 2-3   stage the unit's window query rows (the MMA's B operand);
+//   warps 4-11  two epilogue warpgroups, each owning half of the window-row columns; every
+//               thread owns one key (one TMEM lane), so per-row running statistics (pass 1)
+//               and per-key sums over rows (pass 2) are thread-local.
 //
-// One CTA per SM, 256 threads, warp-specialised:
-//   warp 0      TMA producer: streams 128-key x 128-dim bf16 tiles of K (two 128-byte-swizzled
-//               64-column boxes) into a 6-stage shared-memory ring;
-//   warp 1      allocates TMEM and issues tcgen05.mma (M = 128 keys, N = window rows of the
-//               batch's heads, K = 128) into one of two TMEM accumulators;
-//   warps 2-3   stage the unit's window query rows (the MMA's B operand) in shared memory;
-//   warps 4-7   epilogue: each thread owns one key (one TMEM lane) and reads all of its
-//               window-row logits, so both the per-row online softmax state (pass 1) and the
-//               per-key sum over rows (pass 2) are thread-local.
-//
-// Work unit = (sequence, KV head, batch of up to 64/W_PAD selected heads); each unit's key
-// tiles are split into chunks of `chunk_tiles` tiles (one chunk = one work item).
+// Work: a unit is (sequence, batch of selected heads of one KV group); its key tiles are cut
+// into items (chunks).  Per item:
+//   pass 1  tiles in increasing order: per-thread running (max, sum of 2^(x - max)) per row,
+//           rescaled only when a logit exceeds the running max by more than 2^8; then the
+//           CTA's per-row partial goes to global memory and the unit's arrival counter is
+//           incremented;
+//   wait    until every item of the unit has published its partial (a bounded spin; all CTAs
+//           of a launch are co-resident, and a unit's items all belong to one round);
+//   pass 2  tiles in decreasing order, so the last kSlots tiles are still resident and only
+//           older ones are loaded again: exp2(x - lse) summed over each head's rows.
+// Items are dealt out in rounds of gridDim.x; CTA b takes item (round * gridDim.x + b).
 #include "ckv_device.cuh"
 #include "ckv_internal.h"
 
+#include <string.h>
+
+#include <mutex>
+
 namespace ckv {
+
+constexpr int kSlots = 6;
+constexpr int kTileBytes = kTileKeys * kHeadDim * 2;  // 32 KiB
+constexpr int kHalfBytes = kTileBytes / 2;            // 64 dims x 128 keys
+constexpr float kLazyTau = 8.0f;                      // rescale only when 2^(x-m) > 2^8
+constexpr int kThreads = 384;
+constexpr int kEpiThreads = 256;
 
 struct alignas(128) ScoreParams {
     CUtensorMap tmap_k;            // K as {128 (dim), H_kv, T}, box {64, 1, 128}, 128B swizzle
     const __nv_bfloat16* q_win;    // [S, w, H_q, 128] packed
-    const int32_t* cu_seqlens;     // device [S+1]
+    const int32_t* cu_seqlens;     // device [S+1] (checked against cu_hash)
     float2* partials;              // [n_items, N]: (max, sum) per window-row column
+    int* counters;                 // [n_units] arrivals, zero at launch
     float* scores;                 // [n_sel, T]
     int* status;
-    int S, T, Hq, w, nb, n_items, chunk_tiles, skip_le;
+    int S, T, Hq, w, n_rounds, n_items, n_units;
     uint32_t cu_hash;
     float sl2;                     // softmax scale * log2(e)
     int16_t batch_group[kMaxBatches];   // KV head of each head batch
     int16_t batch_first[kMaxBatches];   // score row of the batch's first head
     int16_t batch_nheads[kMaxBatches];  // heads in the batch
     int16_t sel_heads[kMaxQHeads];      // query head of each score row
+    ScoreItem items[kMaxScoreItems];    // [n_rounds * gridDim.x]
+    ScoreUnit units[kMaxScoreUnits];
 };
-
-struct Item {
-    int s, seq_start, L, P, b, g, first, nheads, chunk, nchunks, tile0, tile1, unit_base;
-};
-
-constexpr int kStages = 6;
-constexpr int kTileBytes = kTileKeys * kHeadDim * 2;  // 32 KiB
-constexpr int kHalfBytes = kTileBytes / 2;            // 64 columns x 128 keys
-constexpr float kLazyTau = 8.0f;                      // rescale only when 2^(x-m) > 2^8
-
-// Maps a work item to its sequence, head batch and key-tile range by walking cu_seqlens.
-// Returns false (and records an error) if the device lengths do not produce this item.
-__device__ __forceinline__ bool decode_item(const ScoreParams& p, int item, Item& it) {
-    int base = 0;
-    for (int s = 0; s < p.S; ++s) {
-        const int t0 = p.cu_seqlens[s], t1 = p.cu_seqlens[s + 1];
-        const int L = t1 - t0;
-        if (L < 0 || t0 < 0 || t1 > p.T) return false;
-        const int tiles = (L + kTileKeys - 1) / kTileKeys;
-        const int nch = (L > p.skip_le && L > 0) ? (tiles + p.chunk_tiles - 1) / p.chunk_tiles : 0;
-        const int cnt = nch * p.nb;
-        if (item < base + cnt) {
-            const int rem = item - base;
-            it.s = s;
-            it.seq_start = t0;
-            it.L = L;
-            it.P = L - p.w;
-            it.b = rem / nch;
-            it.chunk = rem % nch;
-            it.nchunks = nch;
-            it.g = p.batch_group[it.b];
-            it.first = p.batch_first[it.b];
-            it.nheads = p.batch_nheads[it.b];
-            it.tile0 = it.chunk * p.chunk_tiles;
-            it.tile1 = min(tiles, it.tile0 + p.chunk_tiles);
-            it.unit_base = item - it.chunk;
-            return true;
-        }
-        base += cnt;
-    }
-    return false;
-}
 
 template <int N>
 struct SmemLayout {
-    static constexpr int kRing = 0;
-    static constexpr int kQ = kRing + kStages * kTileBytes;
+    static constexpr int kQ = kSlots * kTileBytes;
     static constexpr int kQHalf = N * 128;
     static constexpr int kBars = kQ + 2 * kQHalf;
-    // full[kStages], empty[kStages], acc_full[2], acc_empty[2], q_full, q_empty, done
-    static constexpr int kNumBars = 2 * kStages + 7;
-    static constexpr int kRed = kBars + 8 * kNumBars;   // float2 [4][N]
+    // full[kSlots], freed[kSlots], acc_full[2], acc_empty[2], q_full, q_empty, done
+    static constexpr int kNumBars = 2 * kSlots + 7;
+    static constexpr int kRed = kBars + 8 * kNumBars;   // float2 [2 wg][4 quarters][N/2]
     static constexpr int kLse = kRed + 8 * 4 * N;       // float [N]
-    static constexpr int kTmemSlot = kLse + 4 * N;
+    static constexpr int kXsum = kLse + 4 * N + 16;     // float [2][128] (lse: N + flag)
+    static constexpr int kFills = kXsum + 4 * 256;      // int [2][kSlots]: producer, MMA
+    static constexpr int kTmemSlot = kFills + 4 * 2 * kSlots;
     static constexpr int kAbort = kTmemSlot + 4;
     static constexpr int kBytes = kAbort + 4;
     static constexpr int kDynamic = kBytes + 1024;      // slack to align the base to 1024 B
 };
 
-template <int PASS, int N, int W_PAD>
-__global__ void __launch_bounds__(256, 1) score_kernel(const __grid_constant__ ScoreParams p) {
+__device__ __forceinline__ float redux_max(float v) {
+    float r;
+    asm volatile("redux.sync.max.f32 %0, %1, 0xffffffff;" : "=f"(r) : "f"(v));
+    return r;
+}
+
+__device__ __forceinline__ int ld_acquire(const int* p) {
+    int v;
+    asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+template <int CPW>
+__device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, float (&v)[CPW]) {
+    if constexpr (CPW == 32) {
+        tmem_ld32(taddr, v);
+    } else {
+        static_assert(CPW == 16, "CPW");
+        uint32_t r[16];
+        asm volatile(
+            "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+            "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n\t"
+            "tcgen05.wait::ld.sync.aligned;"
+            : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]),
+              "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]),
+              "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+            : "r"(taddr)
+            : "memory");
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+    }
+}
+
+// Valid-column mask of one thread for a tile: columns holding a real window row that sees
+// key j.  Row r of a head sees key j iff r >= j - P (causal window); keys >= L are padding.
+template <int CPW, int W_PAD>
+__device__ __forceinline__ uint32_t tile_mask(uint32_t colmask, int col0, int t, int j, int P, int L) {
+    const bool edge = (t * kTileKeys + kTileKeys - 1 >= P) || (t * kTileKeys + kTileKeys > L);
+    if (!edge) return colmask;
+    if (j >= L) return 0u;
+    const int jr = j - P;
+    uint32_t cm = 0;
+#pragma unroll
+    for (int i = 0; i < CPW; ++i) cm |= (((col0 + i) % W_PAD) >= jr ? 1u : 0u) << i;
+    return colmask & cm;
+}
+
+template <int N, int W_PAD>
+__global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constant__ ScoreParams p) {
     static_assert(N == 32 || N == 64, "N");
     static_assert(W_PAD == 8 || W_PAD == 16 || W_PAD == 32 || W_PAD == 64, "W_PAD");
     static_assert(W_PAD <= N, "a head's rows fit in one MMA");
-    constexpr int HPB = N / W_PAD;  // heads per batch
+    constexpr int CPW = N / 2;                         // columns per epilogue warpgroup
+    constexpr bool kSplitHead = W_PAD > CPW;           // one head spans both warpgroups
+    constexpr int HPW = kSplitHead ? 1 : CPW / W_PAD;  // heads (or half a head) per warpgroup
     using SL = SmemLayout<N>;
     constexpr uint32_t kIdesc = idesc_bf16_f32(kTileKeys, N);
+    constexpr uint32_t kFullMask = CPW == 32 ? 0xffffffffu : 0xffffu;
 
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-    uint8_t* ring = sm + SL::kRing;
+    uint8_t* slots = sm;
     uint8_t* qbuf = sm + SL::kQ;
     uint64_t* bars = reinterpret_cast<uint64_t*>(sm + SL::kBars);
     uint64_t* full = bars;
-    uint64_t* empty = bars + kStages;
-    uint64_t* acc_full = bars + 2 * kStages;
+    uint64_t* freed = bars + kSlots;
+    uint64_t* acc_full = bars + 2 * kSlots;
     uint64_t* acc_empty = acc_full + 2;
     uint64_t* q_full = acc_empty + 2;
     uint64_t* q_empty = q_full + 1;
     uint64_t* done = q_empty + 1;
     float2* red = reinterpret_cast<float2*>(sm + SL::kRed);
     float* lse_s = reinterpret_cast<float*>(sm + SL::kLse);
+    float* xsum = reinterpret_cast<float*>(sm + SL::kXsum);
+    int* fills = reinterpret_cast<int*>(sm + SL::kFills);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + SL::kTmemSlot);
     volatile int* abort = reinterpret_cast<volatile int*>(sm + SL::kAbort);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     if (threadIdx.x == 0) {
-        for (int i = 0; i < kStages; ++i) {
+        for (int i = 0; i < kSlots; ++i) {
             mbar_init(&full[i], 1);
-            mbar_init(&empty[i], 1);
+            mbar_init(&freed[i], 1);
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&acc_full[i], 1);
-            mbar_init(&acc_empty[i], 128);
+            mbar_init(&acc_empty[i], kEpiThreads);
         }
         mbar_init(q_full, 64);
         mbar_init(q_empty, 1);
         mbar_init(done, 1);
+        for (int i = 0; i < 2 * kSlots; ++i) fills[i] = 0;
         *abort = 0;
         fence_mbar_init();
         tma_prefetch_desc(&p.tmap_k);
@@ -150,20 +183,8 @@ __global__ void __launch_bounds__(256, 1) score_kernel(const __grid_constant__ S
         tmem_alloc(tmem_slot, 2 * N);
         tmem_relinquish();
     }
-    // Work items as the host counted them must match what the device lengths produce.
-    if (blockIdx.x == 0 && threadIdx.x == 32 * 2) {
-        int total = 0;
-        bool ok = true;
-        for (int s = 0; s < p.S; ++s) {
-            const int L = p.cu_seqlens[s + 1] - p.cu_seqlens[s];
-            if (L < 0 || p.cu_seqlens[s + 1] > p.T) ok = false;
-            const int tiles = (L + kTileKeys - 1) / kTileKeys;
-            total += (L > p.skip_le && L > 0) ? (tiles + p.chunk_tiles - 1) / p.chunk_tiles * p.nb : 0;
-        }
-        if (!ok || total != p.n_items || p.cu_seqlens[p.S] != p.T ||
-            seqlens_hash(p.cu_seqlens, p.S) != p.cu_hash)
-            record_error(p.status, kDevBadSeqlens, 100 + PASS);
-    }
+    if (blockIdx.x == 0 && threadIdx.x == 64 && seqlens_hash(p.cu_seqlens, p.S) != p.cu_hash)
+        record_error(p.status, kDevBadSeqlens, 100);
     tc_fence_before_sync();
     __syncthreads();
     tc_fence_after_sync();
@@ -172,78 +193,87 @@ __global__ void __launch_bounds__(256, 1) score_kernel(const __grid_constant__ S
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
-            int it = 0;
+            int* pf = fills;  // fills issued per slot
             bool ok = true;
-            for (int item = blockIdx.x; ok && item < p.n_items; item += gridDim.x) {
-                Item I;
-                if (!decode_item(p, item, I)) continue;
-                for (int t = I.tile0; t < I.tile1; ++t, ++it) {
-                    const int stage = it % kStages;
-                    const uint32_t ph = (it / kStages) & 1;
-                    if (!mbar_wait(&empty[stage], ph ^ 1, abort)) {
-                        ok = false;
-                        break;
-                    }
-                    mbar_arrive_expect_tx(&full[stage], kTileBytes);
-                    uint8_t* dst = ring + stage * kTileBytes;
-                    const int tok = I.seq_start + t * kTileKeys;
-                    tma_load_3d(dst, &p.tmap_k, &full[stage], 0, I.g, tok);
-                    tma_load_3d(dst + kHalfBytes, &p.tmap_k, &full[stage], 64, I.g, tok);
-                }
+            auto load = [&](const ScoreUnit& U, int tile0, int jt) {
+                const int s = jt % kSlots;
+                if (!mbar_wait(&freed[s], (pf[s] & 1) ^ 1, abort)) return false;
+                ++pf[s];
+                mbar_arrive_expect_tx(&full[s], kTileBytes);
+                uint8_t* dst = slots + s * kTileBytes;
+                const int tok = U.seq_start + (tile0 + jt) * kTileKeys;
+                const int g = p.batch_group[U.batch];
+                tma_load_3d(dst, &p.tmap_k, &full[s], 0, g, tok);
+                tma_load_3d(dst + kHalfBytes, &p.tmap_k, &full[s], 64, g, tok);
+                return true;
+            };
+            for (int r = 0; ok && r < p.n_rounds; ++r) {
+                const ScoreItem& I = p.items[r * gridDim.x + blockIdx.x];
+                const int n = I.ntiles;
+                if (n == 0) continue;
+                const ScoreUnit& U = p.units[I.unit];
+                for (int jt = 0; ok && jt < n; ++jt) ok = load(U, I.tile0, jt);               // pass 1
+                for (int jt = n - kSlots - 1; ok && jt >= 0; --jt) ok = load(U, I.tile0, jt);  // pass 2
             }
             if (!ok) {
                 *abort = 1;
-                record_error(p.status, kDevTimeout, 10 * PASS + 0);
+                record_error(p.status, kDevTimeout, 10);
             }
             // Let every issued copy land before the block may exit.
-            const int n_issued = it;
-            for (int k = n_issued - 1; k >= 0 && k >= n_issued - kStages; --k) {
+            for (int s = 0; s < kSlots; ++s) {
                 volatile int never = 0;
-                mbar_wait(&full[k % kStages], (k / kStages) & 1, &never);
+                if (pf[s] > 0) mbar_wait(&full[s], (pf[s] - 1) & 1, &never);
             }
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
-            int it = 0, acc_it = 0, item_it = 0;
+            int* mf = fills + kSlots;  // fills consumed per slot
+            int acc_it = 0, item_it = 0;
             bool ok = true;
-            for (int item = blockIdx.x; ok && item < p.n_items; item += gridDim.x) {
-                Item I;
-                if (!decode_item(p, item, I)) continue;
+            auto mma_tile = [&](int s, bool wait_fill, bool release) {
+                if (wait_fill) {
+                    if (!mbar_wait(&full[s], mf[s] & 1, abort)) return false;
+                    ++mf[s];
+                }
+                const int acc = acc_it & 1;
+                if (!mbar_wait(&acc_empty[acc], ((acc_it >> 1) & 1) ^ 1, abort)) return false;
+                tc_fence_after_sync();
+                const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * N);
+                const uint32_t a0 = smem_u32(slots + s * kTileBytes);
+                const uint32_t b0 = smem_u32(qbuf);
+#pragma unroll
+                for (int kk = 0; kk < kHeadDim / 16; ++kk) {
+                    const uint32_t koff = (kk & 3) * 32;
+                    const uint64_t ad = sdesc_k_major_sw128(a0 + (kk >> 2) * kHalfBytes + koff);
+                    const uint64_t bd = sdesc_k_major_sw128(b0 + (kk >> 2) * SL::kQHalf + koff);
+                    umma_bf16(d_tmem, ad, bd, kIdesc, kk > 0 ? 1u : 0u);
+                }
+                umma_commit(&acc_full[acc]);
+                if (release) umma_commit(&freed[s]);
+                ++acc_it;
+                return true;
+            };
+            for (int r = 0; ok && r < p.n_rounds; ++r) {
+                const ScoreItem& I = p.items[r * gridDim.x + blockIdx.x];
+                const int n = I.ntiles;
+                if (n == 0) continue;
                 if (!mbar_wait(q_full, item_it & 1, abort)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after_sync();
-                for (int t = I.tile0; t < I.tile1; ++t, ++it, ++acc_it) {
-                    const int stage = it % kStages;
-                    const int acc = acc_it & 1;
-                    if (!mbar_wait(&full[stage], (it / kStages) & 1, abort) ||
-                        !mbar_wait(&acc_empty[acc], ((acc_it >> 1) & 1) ^ 1, abort)) {
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after_sync();
-                    const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * N);
-                    const uint32_t a0 = smem_u32(ring + stage * kTileBytes);
-                    const uint32_t b0 = smem_u32(qbuf);
-#pragma unroll
-                    for (int kk = 0; kk < kHeadDim / 16; ++kk) {
-                        const uint32_t koff = (kk & 3) * 32;
-                        const uint64_t ad = sdesc_k_major_sw128(a0 + (kk >> 2) * kHalfBytes + koff);
-                        const uint64_t bd = sdesc_k_major_sw128(b0 + (kk >> 2) * SL::kQHalf + koff);
-                        umma_bf16(d_tmem, ad, bd, kIdesc, kk > 0 ? 1u : 0u);
-                    }
-                    umma_commit(&empty[stage]);
-                    umma_commit(&acc_full[acc]);
-                }
+                // pass 1: a tile that is evicted before pass 2 frees its slot right away
+                for (int jt = 0; ok && jt < n; ++jt) ok = mma_tile(jt % kSlots, true, jt < n - kSlots);
+                // pass 2: resident tiles need no new fill; every tile frees its slot after use
+                for (int jt = n - 1; ok && jt >= 0; --jt) ok = mma_tile(jt % kSlots, jt < n - kSlots, true);
                 if (!ok) break;
                 umma_commit(q_empty);
                 ++item_it;
             }
             if (!ok) {
                 *abort = 1;
-                record_error(p.status, kDevTimeout, 10 * PASS + 1);
+                record_error(p.status, kDevTimeout, 11);
             }
             umma_commit(done);
             volatile int never = 0;
@@ -254,37 +284,39 @@ __global__ void __launch_bounds__(256, 1) score_kernel(const __grid_constant__ S
         // ------------------------------------------------------------ query-row staging
         const int tid = threadIdx.x - 64;
         int item_it = 0;
-        for (int item = blockIdx.x; item < p.n_items; item += gridDim.x) {
-            Item I;
-            if (!decode_item(p, item, I)) continue;
+        for (int r = 0; r < p.n_rounds; ++r) {
+            const ScoreItem& I = p.items[r * gridDim.x + blockIdx.x];
+            if (I.ntiles == 0) continue;
+            const ScoreUnit& U = p.units[I.unit];
             if (!mbar_wait(q_empty, (item_it & 1) ^ 1, abort)) {
                 *abort = 1;
-                record_error(p.status, kDevTimeout, 10 * PASS + 2);
+                record_error(p.status, kDevTimeout, 12);
                 break;
             }
-            // Each thread owns one 16-byte column chunk c of rows r0, r0+4, ...: all of its
-            // loads are issued before any store, so their latencies overlap.
+            const int first = p.batch_first[U.batch], nheads = p.batch_nheads[U.batch];
+            // Each thread owns one 16-byte chunk c of rows r0, r0+4, ...; every load is issued
+            // before any store.
             constexpr int kPer = N * 16 / 64;
             const int c = tid & 15, r0 = tid >> 4;
             uint4 vals[kPer];
 #pragma unroll
             for (int i = 0; i < kPer; ++i) {
-                const int r = r0 + 4 * i;
-                const int slot = r / W_PAD, rr = r % W_PAD;
+                const int row = r0 + 4 * i;
+                const int slot = row / W_PAD, rr = row % W_PAD;
                 vals[i] = make_uint4(0u, 0u, 0u, 0u);
-                if (slot < I.nheads && rr < p.w) {
-                    const int h = p.sel_heads[I.first + slot];
+                if (slot < nheads && rr < p.w) {
+                    const int h = p.sel_heads[first + slot];
                     const uint4* src = reinterpret_cast<const uint4*>(
-                        p.q_win + ((static_cast<size_t>(I.s) * p.w + rr) * p.Hq + h) * kHeadDim);
+                        p.q_win + ((static_cast<size_t>(U.seq) * p.w + rr) * p.Hq + h) * kHeadDim);
                     vals[i] = __ldg(src + c);
                 }
             }
 #pragma unroll
             for (int i = 0; i < kPer; ++i) {
-                const int r = r0 + 4 * i;
+                const int row = r0 + 4 * i;
                 const int half = c >> 3, cc = c & 7;
-                *reinterpret_cast<uint4*>(qbuf + half * SL::kQHalf + r * 128 +
-                                          ((cc ^ (r & 7)) << 4)) = vals[i];
+                *reinterpret_cast<uint4*>(qbuf + half * SL::kQHalf + row * 128 +
+                                          ((cc ^ (row & 7)) << 4)) = vals[i];
             }
             fence_proxy_async_smem();
             mbar_arrive(q_full);
@@ -292,194 +324,216 @@ __global__ void __launch_bounds__(256, 1) score_kernel(const __grid_constant__ S
         }
     } else {
         // ------------------------------------------------------------ epilogue
-        const int eq = warp - 4;           // TMEM lane quarter
-        const int tid = threadIdx.x - 128;
+        const int wg = (warp - 4) >> 2;      // warpgroup: columns [wg*CPW, wg*CPW+CPW)
+        const int eq = warp & 3;             // TMEM lane quarter
+        const int etid = threadIdx.x - 128;  // 0..255 over both warpgroups
+        const int col0 = wg * CPW;
+        const uint32_t lane_base = static_cast<uint32_t>(eq * 32) << 16;
         int acc_it = 0;
         bool ok = true;
-        for (int item = blockIdx.x; ok && item < p.n_items; item += gridDim.x) {
-            Item I;
-            if (!decode_item(p, item, I)) continue;
-            uint64_t colmask = 0;
+        for (int r = 0; ok && r < p.n_rounds; ++r) {
+            const int item = r * gridDim.x + blockIdx.x;
+            const ScoreItem& I = p.items[item];
+            const int n = I.ntiles;
+            if (n == 0) continue;
+            const ScoreUnit& U = p.units[I.unit];
+            const int L = U.len, P = L - p.w;
+            const int first = p.batch_first[U.batch], nheads = p.batch_nheads[U.batch];
+            uint32_t colmask = 0;  // this warpgroup's columns that hold a real window row
 #pragma unroll
-            for (int c = 0; c < N; ++c)
-                if ((c % W_PAD) < p.w && (c / W_PAD) < I.nheads) colmask |= 1ull << c;
-            const bool all_cols = colmask == (N == 64 ? ~0ull : ((1ull << N) - 1));
-
-            float st_a[N];  // pass 1: running max (log2 units); pass 2: lse (log2 units)
-            float st_b[N];  // pass 1: running sum relative to st_a
-            if constexpr (PASS == 1) {
-#pragma unroll
-                for (int c = 0; c < N; ++c) {  // set from the first tile below
-                    st_a[c] = -1e30f;
-                    st_b[c] = 0.f;
-                }
-            } else {
-                named_bar_sync(1, 128);  // previous item's readers of lse_s are done
-                if (tid < N) {
-                    float M = -INFINITY, S = 0.f;
-                    const int n = min(I.nchunks, p.n_items - I.unit_base);
-                    const float2* src = p.partials + static_cast<size_t>(I.unit_base) * N + tid;
-                    int k = 0;
-                    for (; k + 4 <= n; k += 4) {  // four independent loads in flight
-                        float2 pr[4];
-#pragma unroll
-                        for (int u = 0; u < 4; ++u) pr[u] = src[static_cast<size_t>(k + u) * N];
-#pragma unroll
-                        for (int u = 0; u < 4; ++u) {
-                            const float Mn = fmaxf(M, pr[u].x);
-                            S = S * ex2_approx(M - Mn) + pr[u].y * ex2_approx(pr[u].x - Mn);
-                            M = Mn;
-                        }
-                    }
-                    for (; k < n; ++k) {
-                        const float2 pr = src[static_cast<size_t>(k) * N];
-                        const float Mn = fmaxf(M, pr.x);
-                        S = S * ex2_approx(M - Mn) + pr.y * ex2_approx(pr.x - Mn);
-                        M = Mn;
-                    }
-                    lse_s[tid] = M + log2f(S);
-                }
-                named_bar_sync(1, 128);
-#pragma unroll
-                for (int c = 0; c < N; ++c) st_a[c] = lse_s[c];
+            for (int i = 0; i < CPW; ++i) {
+                const int c = col0 + i;
+                if ((c % W_PAD) < p.w && (c / W_PAD) < nheads) colmask |= 1u << i;
             }
+            float st_a[CPW];  // pass 1: running max (log2 units); pass 2: lse (log2 units)
+            float st_b[CPW];  // pass 1: running sum relative to st_a
 
-            for (int t = I.tile0; t < I.tile1; ++t, ++acc_it) {
+            // ---------------------------------------------------- pass 1
+            for (int jt = 0; jt < n; ++jt, ++acc_it) {
                 const int acc = acc_it & 1;
                 if (!mbar_wait(&acc_full[acc], (acc_it >> 1) & 1, abort)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after_sync();
-                const uint32_t taddr = tmem_base + (static_cast<uint32_t>(eq * 32) << 16) +
-                                       static_cast<uint32_t>(acc * N);
-                const int j = t * kTileKeys + eq * 32 + lane;  // sequence-local key position
-                const bool edge = (t * kTileKeys + kTileKeys - 1 >= I.P) ||
-                                  (t * kTileKeys + kTileKeys > I.L);
-                const bool simple = all_cols && !edge;
-                const bool key_ok = j < I.L;
-                const int jr = j - I.P;  // row r sees key j iff r >= jr
-                const bool first = t == I.tile0;
-                float accum[HPB];
+                float v[CPW];
+                tmem_ld_cols<CPW>(tmem_base + lane_base + static_cast<uint32_t>(acc * N + col0), v);
+                tc_fence_before_sync();
+                mbar_arrive(&acc_empty[acc]);
+                const int t = I.tile0 + jt;
+                const int j = t * kTileKeys + eq * 32 + lane;  // sequence-local key
+                const uint32_t vm = tile_mask<CPW, W_PAD>(colmask, col0, t, j, P, L);
+                if (jt == 0) {
+                    // The thread's first key of the item seeds each row's running maximum.  A
+                    // row that cannot see this key cannot see the thread's later keys either.
 #pragma unroll
-                for (int h = 0; h < HPB; ++h) accum[h] = 0.f;
-
-#pragma unroll
-                for (int cc = 0; cc < N / 32; ++cc) {
-                    float v[32];
-                    tmem_ld32(taddr + cc * 32, v);
-                    if (cc == N / 32 - 1) {  // the accumulator is free for the next tile
-                        tc_fence_before_sync();
-                        mbar_arrive(&acc_empty[acc]);
+                    for (int i = 0; i < CPW; ++i) {
+                        const bool valid = (vm >> i) & 1u;
+                        st_a[i] = valid ? v[i] * p.sl2 : -1e30f;
+                        st_b[i] = valid ? 1.f : 0.f;
                     }
-                    if constexpr (PASS == 1) {
-                        if (first) {
-                            // The thread's first key of the item seeds each row's running
-                            // maximum.  A row that cannot see this key cannot see the thread's
-                            // later keys either (they lie further right), so it stays empty.
+                    continue;
+                }
+                float dmax = -INFINITY;
+                if (vm == kFullMask) {
 #pragma unroll
-                            for (int i = 0; i < 32; ++i) {
-                                const int c = cc * 32 + i;
-                                const bool valid = simple || (((colmask >> c) & 1ull) && key_ok &&
-                                                              (c % W_PAD) >= jr);
-                                st_a[c] = valid ? v[i] * p.sl2 : -1e30f;
-                                st_b[c] = valid ? 1.f : 0.f;
-                            }
-                            continue;
-                        }
-                        float dmax = -INFINITY;
+                    for (int i = 0; i < CPW; ++i) {
+                        v[i] = fmaf(v[i], p.sl2, -st_a[i]);
+                        dmax = fmaxf(dmax, v[i]);
+                    }
+                } else {
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) {
-                            const int c = cc * 32 + i;
-                            float d = fmaf(v[i], p.sl2, -st_a[c]);
-                            if (!simple) {
-                                const bool valid = ((colmask >> c) & 1ull) && key_ok && (c % W_PAD) >= jr;
-                                d = valid ? d : -INFINITY;
-                            }
-                            v[i] = d;
-                            dmax = fmaxf(dmax, d);
-                        }
-                        if (dmax > kLazyTau) {  // a new running maximum well above the old one
+                    for (int i = 0; i < CPW; ++i) {
+                        const float d = fmaf(v[i], p.sl2, -st_a[i]);
+                        v[i] = ((vm >> i) & 1u) ? d : -INFINITY;
+                        dmax = fmaxf(dmax, v[i]);
+                    }
+                }
+                if (dmax > kLazyTau) {  // a new running maximum well above the old one
 #pragma unroll
-                            for (int i = 0; i < 32; ++i) {
-                                const int c = cc * 32 + i;
-                                if (v[i] > kLazyTau) {
-                                    st_b[c] *= ex2_approx(-v[i]);
-                                    st_a[c] += v[i];
-                                    v[i] = 0.f;
-                                }
-                            }
-                        }
-#pragma unroll
-                        for (int i = 0; i < 32; ++i) st_b[cc * 32 + i] += ex2_approx(v[i]);
-                    } else {
-#pragma unroll
-                        for (int i = 0; i < 32; ++i) {
-                            const int c = cc * 32 + i;
-                            float e = ex2_approx(fmaf(v[i], p.sl2, -st_a[c]));
-                            if (!simple) {
-                                const bool valid = ((colmask >> c) & 1ull) && key_ok && (c % W_PAD) >= jr;
-                                e = valid ? e : 0.f;
-                            }
-                            accum[c / W_PAD] += e;
+                    for (int i = 0; i < CPW; ++i) {
+                        if (v[i] > kLazyTau) {
+                            st_b[i] *= ex2_approx(-v[i]);
+                            st_a[i] += v[i];
+                            v[i] = 0.f;
                         }
                     }
                 }
-                if constexpr (PASS == 2) {
-                    if (key_ok) {
-                        const size_t col = static_cast<size_t>(I.seq_start) + j;
 #pragma unroll
-                        for (int h = 0; h < HPB; ++h)
-                            if (h < I.nheads)
-                                p.scores[static_cast<size_t>(I.first + h) * p.T + col] = accum[h];
-                    }
-                }
+                for (int i = 0; i < CPW; ++i) st_b[i] += ex2_approx(v[i]);
             }
             if (!ok) break;
 
-            if constexpr (PASS == 1) {
-                // Combine the 128 threads' (max, sum) per column and write the chunk partial.
-                // Level-major butterflies over 32 columns at a time, so the shuffles of
-                // different columns overlap instead of forming one long dependent chain.
+            // The warpgroup's 128 threads per column: warp max by redux, rescale, level-major
+            // butterfly sums; then the 4 warps of each warpgroup through shared memory.
 #pragma unroll
-                for (int hc = 0; hc < N / 32; ++hc) {
-                    float M[32];
+            for (int i = 0; i < CPW; ++i) {
+                const float M = redux_max(st_a[i]);
+                st_b[i] *= ex2_approx(st_a[i] - M);
+                st_a[i] = M;
+            }
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) M[i] = st_a[hc * 32 + i];
+            for (int o = 16; o > 0; o >>= 1)
 #pragma unroll
-                    for (int o = 16; o > 0; o >>= 1)
+                for (int i = 0; i < CPW; ++i) st_b[i] += __shfl_xor_sync(0xffffffffu, st_b[i], o);
+            if (lane == 0) {
 #pragma unroll
-                        for (int i = 0; i < 32; ++i)
-                            M[i] = fmaxf(M[i], __shfl_xor_sync(0xffffffffu, M[i], o));
+                for (int i = 0; i < CPW; ++i) red[(wg * 4 + eq) * CPW + i] = make_float2(st_a[i], st_b[i]);
+            }
+            named_bar_sync(1, kEpiThreads);
+            if (etid < N) {
+                const int cw = etid / CPW, ci = etid % CPW;
+                float M = red[(cw * 4) * CPW + ci].x;
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) st_b[hc * 32 + i] *= ex2_approx(st_a[hc * 32 + i] - M[i]);
+                for (int q = 1; q < 4; ++q) M = fmaxf(M, red[(cw * 4 + q) * CPW + ci].x);
+                float S = 0.f;
 #pragma unroll
-                    for (int o = 16; o > 0; o >>= 1)
-#pragma unroll
-                        for (int i = 0; i < 32; ++i)
-                            st_b[hc * 32 + i] += __shfl_xor_sync(0xffffffffu, st_b[hc * 32 + i], o);
-                    if (lane == 0) {
-#pragma unroll
-                        for (int i = 0; i < 32; ++i)
-                            red[eq * N + hc * 32 + i] = make_float2(M[i], st_b[hc * 32 + i]);
+                for (int q = 0; q < 4; ++q) {
+                    const float2 x = red[(cw * 4 + q) * CPW + ci];
+                    S += x.y * ex2_approx(x.x - M);
+                }
+                p.partials[static_cast<size_t>(item) * N + etid] = make_float2(M, S);
+                __threadfence();
+            }
+            named_bar_sync(1, kEpiThreads);
+
+            // ---------------------------------------------------- exchange with the unit
+            if (etid == 0) {
+                atomicAdd(p.counters + I.unit, 1);
+                const uint64_t t0 = globaltimer_ns();
+                bool got = true;
+                while (ld_acquire(p.counters + I.unit) < U.nitems) {
+                    if (*abort || globaltimer_ns() - t0 > kWaitTimeoutNs) {
+                        *abort = 1;
+                        record_error(p.status, kDevTimeout, 13);
+                        got = false;
+                        break;
                     }
                 }
-                named_bar_sync(1, 128);
-                if (tid < N) {
-                    float M = red[tid].x;
+                __threadfence();
+                lse_s[N] = got ? 1.f : 0.f;  // one verdict for the whole epilogue
+            }
+            named_bar_sync(1, kEpiThreads);
+            if (lse_s[N] == 0.f) {
+                ok = false;
+                break;
+            }
+            if (etid < N) {
+                float M = -INFINITY, S = 0.f;
+                const float2* src = p.partials + static_cast<size_t>(U.first_item) * N + etid;
+                int k = 0;
+                for (; k + 4 <= U.nitems; k += 4) {  // four independent loads in flight
+                    float2 pr[4];
 #pragma unroll
-                    for (int q = 1; q < 4; ++q) M = fmaxf(M, red[q * N + tid].x);
-                    float S = 0.f;
+                    for (int u = 0; u < 4; ++u) pr[u] = __ldcg(src + static_cast<size_t>(k + u) * N);
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) S += red[q * N + tid].y * ex2_approx(red[q * N + tid].x - M);
-                    p.partials[static_cast<size_t>(item) * N + tid] = make_float2(M, S);
+                    for (int u = 0; u < 4; ++u) {
+                        const float Mn = fmaxf(M, pr[u].x);
+                        S = S * ex2_approx(M - Mn) + pr[u].y * ex2_approx(pr[u].x - Mn);
+                        M = Mn;
+                    }
                 }
-                named_bar_sync(1, 128);
+                for (; k < U.nitems; ++k) {
+                    const float2 pr = __ldcg(src + static_cast<size_t>(k) * N);
+                    const float Mn = fmaxf(M, pr.x);
+                    S = S * ex2_approx(M - Mn) + pr.y * ex2_approx(pr.x - Mn);
+                    M = Mn;
+                }
+                lse_s[etid] = M + log2f(S);
+            }
+            named_bar_sync(1, kEpiThreads);
+#pragma unroll
+            for (int i = 0; i < CPW; ++i) st_a[i] = lse_s[col0 + i];
+
+            // ---------------------------------------------------- pass 2 (tiles in reverse)
+            for (int jt = n - 1; jt >= 0; --jt, ++acc_it) {
+                const int acc = acc_it & 1;
+                if (!mbar_wait(&acc_full[acc], (acc_it >> 1) & 1, abort)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after_sync();
+                float v[CPW];
+                tmem_ld_cols<CPW>(tmem_base + lane_base + static_cast<uint32_t>(acc * N + col0), v);
+                tc_fence_before_sync();
+                mbar_arrive(&acc_empty[acc]);
+                const int t = I.tile0 + jt;
+                const int j = t * kTileKeys + eq * 32 + lane;
+                const uint32_t vm = tile_mask<CPW, W_PAD>(colmask, col0, t, j, P, L);
+                float accum[HPW];
+#pragma unroll
+                for (int h = 0; h < HPW; ++h) accum[h] = 0.f;
+                if (vm == kFullMask) {
+#pragma unroll
+                    for (int i = 0; i < CPW; ++i)
+                        accum[kSplitHead ? 0 : i / W_PAD] += ex2_approx(fmaf(v[i], p.sl2, -st_a[i]));
+                } else {
+#pragma unroll
+                    for (int i = 0; i < CPW; ++i) {
+                        const float e = ex2_approx(fmaf(v[i], p.sl2, -st_a[i]));
+                        accum[kSplitHead ? 0 : i / W_PAD] += ((vm >> i) & 1u) ? e : 0.f;
+                    }
+                }
+                const bool key_ok = j < L;
+                const size_t col = static_cast<size_t>(U.seq_start) + j;
+                if constexpr (kSplitHead) {
+                    float* xs = xsum + acc * 128;
+                    if (wg == 1) xs[eq * 32 + lane] = accum[0];
+                    named_bar_sync(2, kEpiThreads);
+                    if (wg == 0 && key_ok)
+                        p.scores[static_cast<size_t>(first) * p.T + col] = accum[0] + xs[eq * 32 + lane];
+                } else if (key_ok) {
+#pragma unroll
+                    for (int h = 0; h < HPW; ++h) {
+                        const int hg = wg * HPW + h;
+                        if (hg < nheads) p.scores[static_cast<size_t>(first + hg) * p.T + col] = accum[h];
+                    }
+                }
             }
         }
         if (!ok) {
             *abort = 1;
-            record_error(p.status, kDevTimeout, 10 * PASS + 3);
+            record_error(p.status, kDevTimeout, 14);
         }
     }
 
@@ -494,9 +548,9 @@ __global__ void __launch_bounds__(256, 1) score_kernel(const __grid_constant__ S
 // ------------------------------------------------------------------------------ host side
 namespace {
 
-template <int PASS, int N, int W_PAD>
+template <int N, int W_PAD>
 cudaError_t launch_one(const ScoreParams& p, int grid, cudaStream_t stream) {
-    auto kern = score_kernel<PASS, N, W_PAD>;
+    auto kern = score_kernel<N, W_PAD>;
     constexpr int smem = SmemLayout<N>::kDynamic;
     static bool configured = false;  // benign race: the attribute call is idempotent
     if (!configured) {
@@ -504,21 +558,30 @@ cudaError_t launch_one(const ScoreParams& p, int grid, cudaStream_t stream) {
         if (e != cudaSuccess) return e;
         configured = true;
     }
-    kern<<<grid, 256, smem, stream>>>(p);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg;
+    memset(&cfg, 0, sizeof cfg);
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;  // all CTAs co-resident: the unit waits need it
+    attr[0].val.cooperative = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, p);
 }
 
-template <int PASS>
 cudaError_t dispatch(const ScoreParams& p, int n_cols, int w_pad, int grid, cudaStream_t st) {
     if (n_cols == 32) {
-        if (w_pad == 8) return launch_one<PASS, 32, 8>(p, grid, st);
-        if (w_pad == 16) return launch_one<PASS, 32, 16>(p, grid, st);
-        if (w_pad == 32) return launch_one<PASS, 32, 32>(p, grid, st);
+        if (w_pad == 8) return launch_one<32, 8>(p, grid, st);
+        if (w_pad == 16) return launch_one<32, 16>(p, grid, st);
+        if (w_pad == 32) return launch_one<32, 32>(p, grid, st);
     } else if (n_cols == 64) {
-        if (w_pad == 8) return launch_one<PASS, 64, 8>(p, grid, st);
-        if (w_pad == 16) return launch_one<PASS, 64, 16>(p, grid, st);
-        if (w_pad == 32) return launch_one<PASS, 64, 32>(p, grid, st);
-        if (w_pad == 64) return launch_one<PASS, 64, 64>(p, grid, st);
+        if (w_pad == 8) return launch_one<64, 8>(p, grid, st);
+        if (w_pad == 16) return launch_one<64, 16>(p, grid, st);
+        if (w_pad == 32) return launch_one<64, 32>(p, grid, st);
+        if (w_pad == 64) return launch_one<64, 64>(p, grid, st);
     }
     return cudaErrorInvalidValue;
 }
@@ -526,23 +589,22 @@ cudaError_t dispatch(const ScoreParams& p, int n_cols, int w_pad, int grid, cuda
 }  // namespace
 
 cudaError_t launch_score(const ScoreLaunch& L, cudaStream_t stream) {
-    static_assert(sizeof(ScoreParams) < 4096, "kernel parameters");
-    ScoreParams p;
+    static_assert(sizeof(ScoreParams) <= 32000, "kernel parameters");
+    static ScoreParams p;  // ~25 KB, kept off the host stack; calls are serialised by `mu`
+    static std::mutex mu;
+    std::lock_guard<std::mutex> lock(mu);
     memset(&p, 0, sizeof(p));
     p.tmap_k = L.tmap_k;
     p.q_win = reinterpret_cast<const __nv_bfloat16*>(L.q_win);
     p.cu_seqlens = L.cu_seqlens_dev;
     p.partials = reinterpret_cast<float2*>(L.partials);
+    p.counters = L.counters;
     p.scores = L.scores;
     p.status = L.status;
     p.S = L.S;
     p.T = L.T;
     p.Hq = L.Hq;
     p.w = L.w;
-    p.nb = L.nb;
-    p.n_items = L.n_items;
-    p.chunk_tiles = L.chunk_tiles;
-    p.skip_le = L.skip_le;
     p.cu_hash = L.cu_hash;
     p.sl2 = L.softmax_scale * 1.4426950408889634f;
     for (int b = 0; b < L.nb; ++b) {
@@ -551,13 +613,19 @@ cudaError_t launch_score(const ScoreLaunch& L, cudaStream_t stream) {
         p.batch_nheads[b] = static_cast<int16_t>(L.batch_nheads[b]);
     }
     for (int i = 0; i < L.n_sel; ++i) p.sel_heads[i] = static_cast<int16_t>(L.sel_heads[i]);
-    if (L.n_items == 0) return cudaSuccess;
-    const int grid = L.n_items < L.grid ? L.n_items : L.grid;
-    cudaError_t e = dispatch<1>(p, L.n_cols, L.w_pad, grid, stream);
-    if (e != cudaSuccess || !L.scores) return e;
-    return dispatch<2>(p, L.n_cols, L.w_pad, grid, stream);
+    // One launch per slice of rounds whose items and units fit the parameter tables.
+    for (const ScoreSlice& sl : L.slices) {
+        p.n_rounds = sl.n_rounds;
+        p.n_items = sl.n_rounds * L.grid;
+        p.n_units = sl.n_units;
+        memcpy(p.items, L.items.data() + sl.item0, sizeof(ScoreItem) * p.n_items);
+        memcpy(p.units, L.units.data() + sl.unit0, sizeof(ScoreUnit) * p.n_units);
+        cudaError_t e = cudaMemsetAsync(L.counters, 0, sizeof(int) * sl.n_units, stream);
+        if (e != cudaSuccess) return e;
+        e = dispatch(p, L.n_cols, L.w_pad, L.grid, stream);
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
 }
-
-int score_partials_stride(int n_cols) { return n_cols; }
 
 }  // namespace ckv
