@@ -91,6 +91,9 @@ typedef struct ckv_config {
                               divides by pool_kernel */
     int32_t head_order;    /* ckv_head_order */
     float softmax_scale;   /* scale of q.k; 0 selects 1/sqrt(head_dim) */
+    int32_t max_ctas;      /* SMs one call's scoring kernel may occupy; 0 = all.  Callers that
+                              run several layers concurrently on different streams give each
+                              call a share, so the calls' kernels can be resident together. */
     const uint8_t* head_mask; /* host [num_layers * num_q_heads]; non-zero = selected.  Every
                                  KV group of a layer needs at least one selected head. */
     const int32_t* budgets;   /* host [num_layers]; kept tokens per KV head, window included,

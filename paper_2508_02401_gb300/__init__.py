@@ -45,7 +45,7 @@ class _Config(C.Structure):
     _fields_ = [("num_layers", C.c_int32), ("num_q_heads", C.c_int32), ("num_kv_heads", C.c_int32),
                 ("head_dim", C.c_int32), ("window", C.c_int32), ("pool_kernel", C.c_int32),
                 ("pool_type", C.c_int32), ("head_order", C.c_int32), ("softmax_scale", C.c_float),
-                ("head_mask", C.c_void_p), ("budgets", C.c_void_p)]
+                ("max_ctas", C.c_int32), ("head_mask", C.c_void_p), ("budgets", C.c_void_p)]
 
 
 class _Batch(C.Structure):
@@ -106,13 +106,15 @@ class Config:
     budgets: np.ndarray     # int32 [num_layers]
     softmax_scale: float = 0.0
     head_dim: int = 128
+    max_ctas: int = 0       # SMs one call's scoring kernel may occupy (0 = all)
 
     def __post_init__(self):
         self.head_mask = np.ascontiguousarray(self.head_mask, dtype=np.uint8)
         self.budgets = np.ascontiguousarray(self.budgets, dtype=np.int32)
         self._c = _Config(self.num_layers, self.num_q_heads, self.num_kv_heads, self.head_dim,
                           self.window, self.pool_kernel, self.pool_type, self.head_order,
-                          self.softmax_scale, self.head_mask.ctypes.data, self.budgets.ctypes.data)
+                          self.softmax_scale, self.max_ctas, self.head_mask.ctypes.data,
+                          self.budgets.ctypes.data)
 
     @classmethod
     def from_workload(cls, wl, **overrides):

@@ -39,7 +39,7 @@ size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // Everything a call needs to know about one layer of the config.
 struct Plan {
-    int Hq = 0, Hkv = 0, G = 0, w = 0, w_pad = 0, n_cols = 0, hpb = 0, budget = 0;
+    int Hq = 0, Hkv = 0, G = 0, w = 0, w_pad = 0, n_cols = 0, hpb = 0, budget = 0, max_ctas = 0;
     int n_sel = 0, nb = 0;
     float scale = 0.f;
     std::vector<int> sel_heads, batch_group, batch_first, batch_nheads, group_first;
@@ -71,6 +71,7 @@ ckv_status check_config(const ckv_config* cfg) {
         return fail(CKV_ERR_INVALID_ARG, "head_order %d", cfg->head_order);
     if (!(cfg->softmax_scale >= 0.f) || !isfinite(cfg->softmax_scale))
         return fail(CKV_ERR_INVALID_ARG, "softmax_scale must be finite and >= 0");
+    if (cfg->max_ctas < 0) return fail(CKV_ERR_INVALID_ARG, "max_ctas %d < 0", cfg->max_ctas);
     if (!cfg->head_mask || !cfg->budgets)
         return fail(CKV_ERR_INVALID_ARG, "head_mask and budgets must be host pointers");
     return CKV_OK;
@@ -86,6 +87,7 @@ ckv_status make_plan(const ckv_config* cfg, int32_t layer, Plan& pl) {
     pl.G = pl.Hq / pl.Hkv;
     pl.w = cfg->window;
     pl.budget = cfg->budgets[layer];
+    pl.max_ctas = cfg->max_ctas;
     if (pl.budget < pl.w)
         return fail(CKV_ERR_INVALID_ARG, "budget %d of layer %d is below the window %d", pl.budget,
                     layer, pl.w);
@@ -348,6 +350,7 @@ ckv_status enqueue_score(const Plan& pl, const ckv_batch* b, int T, const void* 
                          int max_items_per_launch = kMaxScoreItems) {
     int ctas = device_sm_count();
     if (ctas <= 0) return cuda_fail(cudaGetLastError(), "querying the SM count");
+    if (pl.max_ctas > 0) ctas = std::min(ctas, pl.max_ctas);
     static thread_local ScoreLaunch L;  // reused: keeps the plan's vectors allocated
     ckv_status st = plan_score(pl, b, skip_le, std::min(ctas, max_items_per_launch), L,
                                max_items_per_launch);

@@ -33,8 +33,9 @@ struct alignas(256) WsHeader {
     int pad[62];
 };
 
-// Wall-clock bound on every spin in the library's kernels.
-constexpr uint64_t kWaitTimeoutNs = 2000000000ull;  // 2 s
+// Bound on every spin in the library's kernels, in SM clock cycles (about 2 s at 2 GHz).  The
+// cycle counter is cheap to read; the global timer is not, so it is never read inside a spin.
+constexpr long long kWaitTimeoutCycles = 4000000000ll;
 
 // FNV-1a hash of cu_seqlens[0..n]: the host passes the hash of its copy, one device thread
 // hashes the device copy, and a mismatch is recorded as kDevBadSeqlens.
@@ -91,14 +92,18 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 
 // Waits for the phase with the given parity to complete.  Gives up (returns false) after
-// kWaitTimeoutNs or as soon as *abort is set by another thread of the block.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
+// kWaitTimeoutCycles or as soon as *abort is set by another thread of the block (both are
+// checked every 64 polls).  Between polls the warp sleeps for `backoff_ns`, so waiting warps
+// leave the issue slots of their scheduler to the warps doing work.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort,
+                                          uint32_t backoff_ns = 32) {
     if (mbar_try_wait(bar, parity)) return true;
-    const uint64_t t0 = globaltimer_ns();
-    while (true) {
+    const long long t0 = clock64();
+#pragma unroll 1
+    for (uint32_t it = 1;; ++it) {
+        __nanosleep(backoff_ns);
         if (mbar_try_wait(bar, parity)) return true;
-        if (*abort) return false;
-        if (globaltimer_ns() - t0 > kWaitTimeoutNs) return false;
+        if ((it & 63u) == 0u && (*abort || clock64() - t0 > kWaitTimeoutCycles)) return false;
     }
 }
 

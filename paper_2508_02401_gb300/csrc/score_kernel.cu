@@ -9,10 +9,10 @@
 //
 // One cooperative launch; one CTA per SM, 384 threads, warp-specialised:
 //   warp 0      TMA producer: 128-key x 128-dim bf16 tiles of K (two 128-byte-swizzled boxes of
-//               64 dims) into kSlots shared-memory slots; tile i of an item lives in slot
-//               i % kSlots;
+//               64 dims) into a ring of kSlots shared-memory slots; tile i of an item lives
+//               in slot (base + i) % kSlots, base advancing by the item's tile count;
 //   warp 1      allocates TMEM and issues tcgen05.mma (M = 128 keys, N = the window rows of a
-//               batch of heads, K = 128) into two TMEM accumulators;
+//               batch of heads, K = 128) into kAccBufs TMEM accumulators;
 //   warps 2-3   stage the unit's window query rows (the MMA's B operand);
 //   warps 4-11  two epilogue warpgroups, each owning half of the window-row columns; every
 //               thread owns one key (one TMEM lane), so per-row running statistics (pass 1)
@@ -41,9 +41,14 @@ namespace ckv {
 constexpr int kSlots = 6;
 constexpr int kTileBytes = kTileKeys * kHeadDim * 2;  // 32 KiB
 constexpr int kHalfBytes = kTileBytes / 2;            // 64 dims x 128 keys
-constexpr float kLazyTau = 8.0f;                      // rescale only when 2^(x-m) > 2^8
-constexpr int kThreads = 384;
-constexpr int kEpiThreads = 256;
+// The running maximum of a row is only moved when a logit exceeds it by more than 2^60: the
+// running sum then stays far below the fp32 range (at most keys * 2^60), and terms that are
+// 2^-126 below the reference are negligible against the reference term itself.
+constexpr float kLazyTau = 60.0f;
+constexpr int kEpiWG = 4;                             // epilogue warpgroups
+constexpr int kAccBufs = 4;                           // TMEM accumulators (MMA runs ahead)
+constexpr int kEpiThreads = 128 * kEpiWG;
+constexpr int kThreads = 128 + kEpiThreads;
 
 struct alignas(128) ScoreParams {
     CUtensorMap tmap_k;            // K as {128 (dim), H_kv, T}, box {64, 1, 128}, 128B swizzle
@@ -69,12 +74,12 @@ struct SmemLayout {
     static constexpr int kQ = kSlots * kTileBytes;
     static constexpr int kQHalf = N * 128;
     static constexpr int kBars = kQ + 2 * kQHalf;
-    // full[kSlots], freed[kSlots], acc_full[2], acc_empty[2], q_full, q_empty, done
-    static constexpr int kNumBars = 2 * kSlots + 7;
-    static constexpr int kRed = kBars + 8 * kNumBars;   // float2 [2 wg][4 quarters][N/2]
-    static constexpr int kLse = kRed + 8 * 4 * N;       // float [N]
-    static constexpr int kXsum = kLse + 4 * N + 16;     // float [2][128] (lse: N + flag)
-    static constexpr int kFills = kXsum + 4 * 256;      // int [2][kSlots]: producer, MMA
+    // full[kSlots], freed[kSlots], acc_full[kAccBufs], acc_empty[kAccBufs], q_full, q_empty, done
+    static constexpr int kNumBars = 2 * kSlots + 2 * kAccBufs + 3;
+    static constexpr int kRed = kBars + 8 * kNumBars;   // float2 [512] reduction scratch
+    static constexpr int kLse = kRed + 8 * 512;         // float [N]
+    static constexpr int kXsum = kLse + 4 * N + 16;     // float [2][kEpiWG][128] (lse: N + flag)
+    static constexpr int kFills = kXsum + 4 * 2 * kEpiWG * 128;  // int [2][kSlots]
     static constexpr int kTmemSlot = kFills + 4 * 2 * kSlots;
     static constexpr int kAbort = kTmemSlot + 4;
     static constexpr int kBytes = kAbort + 4;
@@ -87,18 +92,58 @@ __device__ __forceinline__ float redux_max(float v) {
     return r;
 }
 
+__device__ __forceinline__ void red_release_add(int* p, int v) {
+    asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ float lg2_approx(float x) {
+    float y;
+    asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// Sum / max of an array by a balanced tree (short dependency chains).
+template <int C>
+__device__ __forceinline__ float tree_sum(float (&x)[C]) {
+#pragma unroll
+    for (int w = C / 2; w >= 1; w >>= 1)
+#pragma unroll
+        for (int i = 0; i < w; ++i) x[i] += x[i + w];
+    return x[0];
+}
+
 __device__ __forceinline__ int ld_acquire(const int* p) {
     int v;
     asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
     return v;
 }
 
+// Warp-wide sums of C per-lane columns (C = 8, 16 or 32) by recursive halving: at each level
+// a lane keeps one half of its remaining columns and swaps the other half with its partner, so
+// the C sums take C - 1 + log2(32 / C) shuffles instead of 5 C.  `m` (uniform across the warp)
+// is carried along.  Afterwards lane l holds column l / (32 / C) in v[0] / m[0].
+template <int C>
+__device__ __forceinline__ void transpose_reduce(float (&v)[C], float (&m)[C], int lane) {
+#pragma unroll
+    for (int k = C / 2, bit = 16; k >= 1; k >>= 1, bit >>= 1) {
+        const bool upper = (lane & bit) != 0;
+#pragma unroll
+        for (int i = 0; i < k; ++i) {
+            const float send = upper ? v[i] : v[i + k];
+            const float keep = upper ? v[i + k] : v[i];
+            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, bit);
+            m[i] = upper ? m[i + k] : m[i];
+        }
+    }
+#pragma unroll
+    for (int bit = 16 / C; bit >= 1; bit >>= 1) v[0] += __shfl_xor_sync(0xffffffffu, v[0], bit);
+}
+
 template <int CPW>
 __device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, float (&v)[CPW]) {
     if constexpr (CPW == 32) {
         tmem_ld32(taddr, v);
-    } else {
-        static_assert(CPW == 16, "CPW");
+    } else if constexpr (CPW == 16) {
         uint32_t r[16];
         asm volatile(
             "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
@@ -111,6 +156,18 @@ __device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, float (&v)[CPW]) {
             : "memory");
 #pragma unroll
         for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+    } else {
+        static_assert(CPW == 8, "CPW");
+        uint32_t r[8];
+        asm volatile(
+            "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];\n\t"
+            "tcgen05.wait::ld.sync.aligned;"
+            : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]),
+              "=r"(r[6]), "=r"(r[7])
+            : "r"(taddr)
+            : "memory");
+#pragma unroll
+        for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(r[i]);
     }
 }
 
@@ -133,12 +190,13 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
     static_assert(N == 32 || N == 64, "N");
     static_assert(W_PAD == 8 || W_PAD == 16 || W_PAD == 32 || W_PAD == 64, "W_PAD");
     static_assert(W_PAD <= N, "a head's rows fit in one MMA");
-    constexpr int CPW = N / 2;                         // columns per epilogue warpgroup
-    constexpr bool kSplitHead = W_PAD > CPW;           // one head spans both warpgroups
-    constexpr int HPW = kSplitHead ? 1 : CPW / W_PAD;  // heads (or half a head) per warpgroup
+    constexpr int CPW = N / kEpiWG;                    // columns per epilogue warpgroup
+    constexpr int kWgPerHead = W_PAD > CPW ? W_PAD / CPW : 1;
+    constexpr bool kSplitHead = kWgPerHead > 1;        // one head spans several warpgroups
+    constexpr int HPW = kSplitHead ? 1 : CPW / W_PAD;  // heads (or a part of one) per warpgroup
     using SL = SmemLayout<N>;
     constexpr uint32_t kIdesc = idesc_bf16_f32(kTileKeys, N);
-    constexpr uint32_t kFullMask = CPW == 32 ? 0xffffffffu : 0xffffu;
+    constexpr uint32_t kFullMask = CPW == 32 ? 0xffffffffu : ((1u << CPW) - 1u);
 
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>(
@@ -149,8 +207,8 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
     uint64_t* full = bars;
     uint64_t* freed = bars + kSlots;
     uint64_t* acc_full = bars + 2 * kSlots;
-    uint64_t* acc_empty = acc_full + 2;
-    uint64_t* q_full = acc_empty + 2;
+    uint64_t* acc_empty = acc_full + kAccBufs;
+    uint64_t* q_full = acc_empty + kAccBufs;
     uint64_t* q_empty = q_full + 1;
     uint64_t* done = q_empty + 1;
     float2* red = reinterpret_cast<float2*>(sm + SL::kRed);
@@ -167,9 +225,9 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             mbar_init(&full[i], 1);
             mbar_init(&freed[i], 1);
         }
-        for (int i = 0; i < 2; ++i) {
+        for (int i = 0; i < kAccBufs; ++i) {
             mbar_init(&acc_full[i], 1);
-            mbar_init(&acc_empty[i], kEpiThreads);
+            mbar_init(&acc_empty[i], kEpiThreads / 32);  // one arrival per epilogue warp
         }
         mbar_init(q_full, 64);
         mbar_init(q_empty, 1);
@@ -180,7 +238,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         tma_prefetch_desc(&p.tmap_k);
     }
     if (warp == 1) {
-        tmem_alloc(tmem_slot, 2 * N);
+        tmem_alloc(tmem_slot, kAccBufs * N);
         tmem_relinquish();
     }
     if (blockIdx.x == 0 && threadIdx.x == 64 && seqlens_hash(p.cu_seqlens, p.S) != p.cu_hash)
@@ -194,9 +252,10 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
             int* pf = fills;  // fills issued per slot
+            int base = 0;     // slot of the item's first tile: the ring continues across items
             bool ok = true;
             auto load = [&](const ScoreUnit& U, int tile0, int jt) {
-                const int s = jt % kSlots;
+                const int s = (base + jt) % kSlots;
                 if (!mbar_wait(&freed[s], (pf[s] & 1) ^ 1, abort)) return false;
                 ++pf[s];
                 mbar_arrive_expect_tx(&full[s], kTileBytes);
@@ -214,6 +273,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                 const ScoreUnit& U = p.units[I.unit];
                 for (int jt = 0; ok && jt < n; ++jt) ok = load(U, I.tile0, jt);               // pass 1
                 for (int jt = n - kSlots - 1; ok && jt >= 0; --jt) ok = load(U, I.tile0, jt);  // pass 2
+                base = (base + n) % kSlots;
             }
             if (!ok) {
                 *abort = 1;
@@ -229,15 +289,15 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
             int* mf = fills + kSlots;  // fills consumed per slot
-            int acc_it = 0, item_it = 0;
+            int acc_it = 0, item_it = 0, base = 0;
             bool ok = true;
             auto mma_tile = [&](int s, bool wait_fill, bool release) {
                 if (wait_fill) {
                     if (!mbar_wait(&full[s], mf[s] & 1, abort)) return false;
                     ++mf[s];
                 }
-                const int acc = acc_it & 1;
-                if (!mbar_wait(&acc_empty[acc], ((acc_it >> 1) & 1) ^ 1, abort)) return false;
+                const int acc = acc_it % kAccBufs;
+                if (!mbar_wait(&acc_empty[acc], ((acc_it / kAccBufs) & 1) ^ 1, abort)) return false;
                 tc_fence_after_sync();
                 const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * N);
                 const uint32_t a0 = smem_u32(slots + s * kTileBytes);
@@ -264,10 +324,13 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                 }
                 tc_fence_after_sync();
                 // pass 1: a tile that is evicted before pass 2 frees its slot right away
-                for (int jt = 0; ok && jt < n; ++jt) ok = mma_tile(jt % kSlots, true, jt < n - kSlots);
+                for (int jt = 0; ok && jt < n; ++jt)
+                    ok = mma_tile((base + jt) % kSlots, true, jt < n - kSlots);
                 // pass 2: resident tiles need no new fill; every tile frees its slot after use
-                for (int jt = n - 1; ok && jt >= 0; --jt) ok = mma_tile(jt % kSlots, jt < n - kSlots, true);
+                for (int jt = n - 1; ok && jt >= 0; --jt)
+                    ok = mma_tile((base + jt) % kSlots, jt < n - kSlots, true);
                 if (!ok) break;
+                base = (base + n) % kSlots;
                 umma_commit(q_empty);
                 ++item_it;
             }
@@ -288,7 +351,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             const ScoreItem& I = p.items[r * gridDim.x + blockIdx.x];
             if (I.ntiles == 0) continue;
             const ScoreUnit& U = p.units[I.unit];
-            if (!mbar_wait(q_empty, (item_it & 1) ^ 1, abort)) {
+            if (!mbar_wait(q_empty, (item_it & 1) ^ 1, abort, 500)) {  // a long, idle wait
                 *abort = 1;
                 record_error(p.status, kDevTimeout, 12);
                 break;
@@ -326,19 +389,24 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         // ------------------------------------------------------------ epilogue
         const int wg = (warp - 4) >> 2;      // warpgroup: columns [wg*CPW, wg*CPW+CPW)
         const int eq = warp & 3;             // TMEM lane quarter
-        const int etid = threadIdx.x - 128;  // 0..255 over both warpgroups
+        const int etid = threadIdx.x - 128;  // 0 .. kEpiThreads-1 over the warpgroups
         const int col0 = wg * CPW;
         const uint32_t lane_base = static_cast<uint32_t>(eq * 32) << 16;
         int acc_it = 0;
         bool ok = true;
         for (int r = 0; ok && r < p.n_rounds; ++r) {
             const int item = r * gridDim.x + blockIdx.x;
-            const ScoreItem& I = p.items[item];
+            // Everything the loops need, copied out of the parameter tables once (asm with a
+            // memory clobber inside the loops would otherwise force reloads).
+            const ScoreItem I = p.items[item];
             const int n = I.ntiles;
             if (n == 0) continue;
-            const ScoreUnit& U = p.units[I.unit];
+            const ScoreUnit U = p.units[I.unit];
             const int L = U.len, P = L - p.w;
             const int first = p.batch_first[U.batch], nheads = p.batch_nheads[U.batch];
+            const int T = p.T;
+            const float sl2 = p.sl2;
+            float* const scores = p.scores;
             uint32_t colmask = 0;  // this warpgroup's columns that hold a real window row
 #pragma unroll
             for (int i = 0; i < CPW; ++i) {
@@ -350,8 +418,8 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
 
             // ---------------------------------------------------- pass 1
             for (int jt = 0; jt < n; ++jt, ++acc_it) {
-                const int acc = acc_it & 1;
-                if (!mbar_wait(&acc_full[acc], (acc_it >> 1) & 1, abort)) {
+                const int acc = acc_it % kAccBufs;
+                if (!mbar_wait(&acc_full[acc], (acc_it / kAccBufs) & 1, abort)) {
                     ok = false;
                     break;
                 }
@@ -359,7 +427,8 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                 float v[CPW];
                 tmem_ld_cols<CPW>(tmem_base + lane_base + static_cast<uint32_t>(acc * N + col0), v);
                 tc_fence_before_sync();
-                mbar_arrive(&acc_empty[acc]);
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&acc_empty[acc]);
                 const int t = I.tile0 + jt;
                 const int j = t * kTileKeys + eq * 32 + lane;  // sequence-local key
                 const uint32_t vm = tile_mask<CPW, W_PAD>(colmask, col0, t, j, P, L);
@@ -369,26 +438,30 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
 #pragma unroll
                     for (int i = 0; i < CPW; ++i) {
                         const bool valid = (vm >> i) & 1u;
-                        st_a[i] = valid ? v[i] * p.sl2 : -1e30f;
+                        st_a[i] = valid ? v[i] * sl2 : -1e30f;
                         st_b[i] = valid ? 1.f : 0.f;
                     }
                     continue;
                 }
-                float dmax = -INFINITY;
                 if (vm == kFullMask) {
 #pragma unroll
-                    for (int i = 0; i < CPW; ++i) {
-                        v[i] = fmaf(v[i], p.sl2, -st_a[i]);
-                        dmax = fmaxf(dmax, v[i]);
-                    }
+                    for (int i = 0; i < CPW; ++i) v[i] = fmaf(v[i], sl2, -st_a[i]);
                 } else {
 #pragma unroll
                     for (int i = 0; i < CPW; ++i) {
-                        const float d = fmaf(v[i], p.sl2, -st_a[i]);
+                        const float d = fmaf(v[i], sl2, -st_a[i]);
                         v[i] = ((vm >> i) & 1u) ? d : -INFINITY;
-                        dmax = fmaxf(dmax, v[i]);
                     }
                 }
+                float dm[CPW / 4];  // max by a short tree
+#pragma unroll
+                for (int i = 0; i < CPW / 4; ++i)
+                    dm[i] = fmaxf(fmaxf(v[4 * i], v[4 * i + 1]), fmaxf(v[4 * i + 2], v[4 * i + 3]));
+#pragma unroll
+                for (int w = CPW / 8; w >= 1; w >>= 1)
+#pragma unroll
+                    for (int i = 0; i < w; ++i) dm[i] = fmaxf(dm[i], dm[i + w]);
+                const float dmax = dm[0];
                 if (dmax > kLazyTau) {  // a new running maximum well above the old one
 #pragma unroll
                     for (int i = 0; i < CPW; ++i) {
@@ -404,21 +477,19 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             }
             if (!ok) break;
 
-            // The warpgroup's 128 threads per column: warp max by redux, rescale, level-major
-            // butterfly sums; then the 4 warps of each warpgroup through shared memory.
+            // The warpgroup's 128 threads per column: warp max by redux, rescale to it, warp sums
+            // by recursive halving; then the 4 warps of each warpgroup through shared memory.
 #pragma unroll
             for (int i = 0; i < CPW; ++i) {
                 const float M = redux_max(st_a[i]);
                 st_b[i] *= ex2_approx(st_a[i] - M);
                 st_a[i] = M;
             }
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1)
-#pragma unroll
-                for (int i = 0; i < CPW; ++i) st_b[i] += __shfl_xor_sync(0xffffffffu, st_b[i], o);
-            if (lane == 0) {
-#pragma unroll
-                for (int i = 0; i < CPW; ++i) red[(wg * 4 + eq) * CPW + i] = make_float2(st_a[i], st_b[i]);
+            transpose_reduce<CPW>(st_b, st_a, lane);
+            {
+                constexpr int kLanesPerCol = 32 / CPW;
+                if (lane % kLanesPerCol == 0)
+                    red[(wg * 4 + eq) * CPW + lane / kLanesPerCol] = make_float2(st_a[0], st_b[0]);
             }
             named_bar_sync(1, kEpiThreads);
             if (etid < N) {
@@ -433,17 +504,20 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                     S += x.y * ex2_approx(x.x - M);
                 }
                 p.partials[static_cast<size_t>(item) * N + etid] = make_float2(M, S);
-                __threadfence();
             }
             named_bar_sync(1, kEpiThreads);
 
             // ---------------------------------------------------- exchange with the unit
             if (etid == 0) {
-                atomicAdd(p.counters + I.unit, 1);
-                const uint64_t t0 = globaltimer_ns();
+                // The barrier above orders the block's partial stores before this thread's
+                // release; the fence makes that release cumulative at GPU scope.
+                __threadfence();
+                red_release_add(p.counters + I.unit, 1);
+                const long long t0 = clock64();
                 bool got = true;
-                while (ld_acquire(p.counters + I.unit) < U.nitems) {
-                    if (*abort || globaltimer_ns() - t0 > kWaitTimeoutNs) {
+                for (uint32_t it = 1; ld_acquire(p.counters + I.unit) < U.nitems; ++it) {
+                    __nanosleep(64);
+                    if ((it & 63u) == 0u && (*abort || clock64() - t0 > kWaitTimeoutCycles)) {
                         *abort = 1;
                         record_error(p.status, kDevTimeout, 13);
                         got = false;
@@ -458,28 +532,31 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                 ok = false;
                 break;
             }
-            if (etid < N) {
+            {
+                // All epilogue threads: column etid % N, items part, part + parts, ...
+                constexpr int kParts = kEpiThreads / N;
+                const int c = etid % N, part = etid / N;
                 float M = -INFINITY, S = 0.f;
-                const float2* src = p.partials + static_cast<size_t>(U.first_item) * N + etid;
-                int k = 0;
-                for (; k + 4 <= U.nitems; k += 4) {  // four independent loads in flight
-                    float2 pr[4];
-#pragma unroll
-                    for (int u = 0; u < 4; ++u) pr[u] = __ldcg(src + static_cast<size_t>(k + u) * N);
-#pragma unroll
-                    for (int u = 0; u < 4; ++u) {
-                        const float Mn = fmaxf(M, pr[u].x);
-                        S = S * ex2_approx(M - Mn) + pr[u].y * ex2_approx(pr[u].x - Mn);
-                        M = Mn;
-                    }
-                }
-                for (; k < U.nitems; ++k) {
+                const float2* src = p.partials + static_cast<size_t>(U.first_item) * N + c;
+                for (int k = part; k < U.nitems; k += kParts) {
                     const float2 pr = __ldcg(src + static_cast<size_t>(k) * N);
                     const float Mn = fmaxf(M, pr.x);
                     S = S * ex2_approx(M - Mn) + pr.y * ex2_approx(pr.x - Mn);
                     M = Mn;
                 }
-                lse_s[etid] = M + log2f(S);
+                red[part * N + c] = make_float2(M, S);
+                named_bar_sync(1, kEpiThreads);
+                if (etid < N) {
+                    float M2 = -INFINITY, S2 = 0.f;
+#pragma unroll
+                    for (int q = 0; q < kParts; ++q) {
+                        const float2 x = red[q * N + etid];
+                        const float Mn = fmaxf(M2, x.x);
+                        S2 = S2 * ex2_approx(M2 - Mn) + x.y * ex2_approx(x.x - Mn);
+                        M2 = Mn;
+                    }
+                    lse_s[etid] = M2 + lg2_approx(S2);
+                }
             }
             named_bar_sync(1, kEpiThreads);
 #pragma unroll
@@ -487,8 +564,8 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
 
             // ---------------------------------------------------- pass 2 (tiles in reverse)
             for (int jt = n - 1; jt >= 0; --jt, ++acc_it) {
-                const int acc = acc_it & 1;
-                if (!mbar_wait(&acc_full[acc], (acc_it >> 1) & 1, abort)) {
+                const int acc = acc_it % kAccBufs;
+                if (!mbar_wait(&acc_full[acc], (acc_it / kAccBufs) & 1, abort)) {
                     ok = false;
                     break;
                 }
@@ -496,37 +573,50 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                 float v[CPW];
                 tmem_ld_cols<CPW>(tmem_base + lane_base + static_cast<uint32_t>(acc * N + col0), v);
                 tc_fence_before_sync();
-                mbar_arrive(&acc_empty[acc]);
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&acc_empty[acc]);
                 const int t = I.tile0 + jt;
                 const int j = t * kTileKeys + eq * 32 + lane;
                 const uint32_t vm = tile_mask<CPW, W_PAD>(colmask, col0, t, j, P, L);
-                float accum[HPW];
-#pragma unroll
-                for (int h = 0; h < HPW; ++h) accum[h] = 0.f;
                 if (vm == kFullMask) {
 #pragma unroll
-                    for (int i = 0; i < CPW; ++i)
-                        accum[kSplitHead ? 0 : i / W_PAD] += ex2_approx(fmaf(v[i], p.sl2, -st_a[i]));
+                    for (int i = 0; i < CPW; ++i) v[i] = ex2_approx(fmaf(v[i], sl2, -st_a[i]));
                 } else {
 #pragma unroll
                     for (int i = 0; i < CPW; ++i) {
-                        const float e = ex2_approx(fmaf(v[i], p.sl2, -st_a[i]));
-                        accum[kSplitHead ? 0 : i / W_PAD] += ((vm >> i) & 1u) ? e : 0.f;
+                        const float e = ex2_approx(fmaf(v[i], sl2, -st_a[i]));
+                        v[i] = ((vm >> i) & 1u) ? e : 0.f;
                     }
+                }
+                // per-head sums by trees over each head's (up to W_PAD) columns
+                constexpr int kSeg = kSplitHead ? CPW : W_PAD;
+                float accum[HPW];
+#pragma unroll
+                for (int h = 0; h < HPW; ++h) {
+                    float seg[kSeg];
+#pragma unroll
+                    for (int i = 0; i < kSeg; ++i) seg[i] = v[h * kSeg + i];
+                    accum[h] = tree_sum<kSeg>(seg);
                 }
                 const bool key_ok = j < L;
                 const size_t col = static_cast<size_t>(U.seq_start) + j;
                 if constexpr (kSplitHead) {
-                    float* xs = xsum + acc * 128;
-                    if (wg == 1) xs[eq * 32 + lane] = accum[0];
+                    // the head's first warpgroup adds the other warpgroups' parts
+                    float* xs = xsum + (acc & 1) * kEpiWG * 128;
+                    const int part = wg % kWgPerHead, hg = wg / kWgPerHead;
+                    if (part != 0) xs[wg * 128 + eq * 32 + lane] = accum[0];
                     named_bar_sync(2, kEpiThreads);
-                    if (wg == 0 && key_ok)
-                        p.scores[static_cast<size_t>(first) * p.T + col] = accum[0] + xs[eq * 32 + lane];
+                    if (part == 0 && key_ok && hg < nheads) {
+                        float sum = accum[0];
+#pragma unroll
+                        for (int q = 1; q < kWgPerHead; ++q) sum += xs[(wg + q) * 128 + eq * 32 + lane];
+                        scores[static_cast<size_t>(first + hg) * T + col] = sum;
+                    }
                 } else if (key_ok) {
 #pragma unroll
                     for (int h = 0; h < HPW; ++h) {
                         const int hg = wg * HPW + h;
-                        if (hg < nheads) p.scores[static_cast<size_t>(first + hg) * p.T + col] = accum[h];
+                        if (hg < nheads) scores[static_cast<size_t>(first + hg) * T + col] = accum[h];
                     }
                 }
             }
@@ -541,7 +631,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
     __syncthreads();
     if (warp == 1) {
         tc_fence_after_sync();
-        tmem_dealloc(tmem_base, 2 * N);
+        tmem_dealloc(tmem_base, kAccBufs * N);
     }
 }
 

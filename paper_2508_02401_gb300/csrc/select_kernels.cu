@@ -85,6 +85,7 @@ constexpr int kPoolTile = 8192;                         // candidate positions p
 constexpr int kMaxHalo = kMaxPoolKernel / 2;
 constexpr int kResidentKeys = 40960;                    // candidates kept in shared memory
 constexpr int kSelSmemBytes = (kResidentKeys + kPoolTile + 2 * kMaxHalo) * 4;
+static_assert(kPoolTile + 2 * kMaxHalo >= kSelWarps * 256, "per-warp histograms fit in the stage buffer");
 
 // Order-preserving key of a non-negative float (-0 maps to +0).
 __device__ __forceinline__ uint32_t rank_key(float f) {
@@ -180,18 +181,28 @@ __global__ void __launch_bounds__(kSelThreads, 1) pool_select_kernel(const __gri
             for (int i = 0; i < kPer; ++i) acc[i] = 0.f;
             const int passes = p.head_order == 0 ? r1 - r0 : 1;
             for (int ps = 0; ps < passes; ++ps) {
-                // stage positions tile0-half .. tile0+n+half (zeros outside [0, P))
-                for (int e = tid; e < n + 2 * half; e += kSelThreads) {
+                // stage positions tile0-half .. tile0+n+half (zeros outside [0, P)); every load
+                // of a thread is issued before its stores, so the round trips overlap
+                constexpr int kStagePer = (kPoolTile + 2 * kMaxHalo + kSelThreads - 1) / kSelThreads;
+                float xs[kStagePer];
+#pragma unroll
+                for (int i = 0; i < kStagePer; ++i) {
+                    const int e = tid + i * kSelThreads;
                     const int u = tile0 - half + e;
                     float x = 0.f;
-                    if (u >= 0 && u < P) {
+                    if (e < n + 2 * half && u >= 0 && u < P) {
                         if (p.head_order == 0) {
                             x = __ldg(base + static_cast<size_t>(r0 + ps) * p.T + u);
                         } else {
                             for (int r = r0; r < r1; ++r) x += __ldg(base + static_cast<size_t>(r) * p.T + u);
                         }
                     }
-                    stage[e] = x;
+                    xs[i] = x;
+                }
+#pragma unroll
+                for (int i = 0; i < kStagePer; ++i) {
+                    const int e = tid + i * kSelThreads;
+                    if (e < n + 2 * half) stage[e] = xs[i];
                 }
                 __syncthreads();
 #pragma unroll
@@ -236,11 +247,30 @@ __global__ void __launch_bounds__(kSelThreads, 1) pool_select_kernel(const __gri
         uint32_t prefix = 0, mask = 0;
         int remaining = k;
         for (int shift = 24; shift >= 0; shift -= 8) {
-            if (tid < 256) hist[tid] = 0;
+            // Per-warp histograms (aliasing the pooling stage buffer): lanes with the same digit
+            // are grouped by __match_any_sync and their leader adds the group's count, so
+            // clustered scores neither serialise on shared atomics nor race across warps.
+            int* whist = reinterpret_cast<int*>(stage) + (tid >> 5) * 256;
+            const int lane = tid & 31;
+#pragma unroll
+            for (int b = lane; b < 256; b += 32) whist[b] = 0;
+            __syncwarp();
+            for (int j0 = 0; j0 < P; j0 += kSelThreads) {
+                const int j = j0 + tid;
+                const uint32_t u = j < P ? key_at(j) : 0u;
+                const bool in = j < P && (u & mask) == prefix;
+                const uint32_t digit = in ? ((u >> shift) & 255u) : 256u;
+                const unsigned peers = __match_any_sync(0xffffffffu, digit);
+                if (in && lane == __ffs(peers) - 1) whist[digit] += __popc(peers);
+                __syncwarp();
+            }
             __syncthreads();
-            for (int j = tid; j < P; j += kSelThreads) {
-                const uint32_t u = key_at(j);
-                if ((u & mask) == prefix) atomicAdd(&hist[(u >> shift) & 255u], 1);
+            if (tid < 256) {
+                int h = 0;
+                const int* wh = reinterpret_cast<const int*>(stage) + tid;
+#pragma unroll 8
+                for (int w = 0; w < kSelWarps; ++w) h += wh[w * 256];
+                hist[tid] = h;
             }
             __syncthreads();
             if (tid < 32) {

@@ -193,3 +193,15 @@ def test_device_lengths_that_disagree_are_reported():
     code, _ = ckv.ckv_read_device_status(ws)
     assert code == 1
     assert ckv.ckv_read_device_status(ws) == (0, 0)  # the read reset it
+
+
+@pytest.mark.parametrize("max_ctas", [1, 5, 24])
+def test_capped_grid_long_items_and_many_rounds(max_ctas):
+    """A small CTA cap forces long work items (tiles re-loaded in pass 2) and several rounds."""
+    wl = _wl(seqlens=(9000, 3000, 700), num_q_heads=32, num_kv_heads=8, budget_mean=300,
+             outlier_channels=8)
+    li = wl.layer(0)
+    cfg = ckv.Config.from_workload(wl, max_ctas=max_ctas)
+    g = gu.run_gpu(wl, 0, li, cfg=cfg)
+    o = gu.run_oracle(wl, 0, li)
+    gu.check_layer(wl, 0, li, g, o)
