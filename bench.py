@@ -237,9 +237,8 @@ def run_ours(args):
     ms_per_step = ms / args.steps
     value = world * nl * T / (ms_per_step / 1e3)
 
-    launches_per_step = 0
-    for l, d in enumerate(layers):
-        launches_per_step += 4 + (1 if d["t_keep"] > 0 else 0)
+    # per layer: the scoring kernel, then pool_hist, threshold and compact (gather fused)
+    launches_per_step = 4 * nl
 
     # --- scoring stage (the dominant kernels): a graph of every layer's ckv_score_window,
     # timed with events on its stream; the average per layer is one pass-1 + pass-2 pair.

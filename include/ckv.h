@@ -37,7 +37,9 @@
  *     are recorded in the workspace's status word and reported by ckv_read_device_status.
  *   - Device pointers must be 16-byte aligned, the workspace 256-byte aligned.
  *   - A workspace may be reused by calls that are ordered on one stream; calls that may run
- *     concurrently need separate workspaces.  Zero it once (cudaMemset) before its first use.
+ *     concurrently need separate workspaces.  Zero it once (cudaMemset) before its first use,
+ *     and again after a call that returned CKV_ERR_CUDA: the selection keeps a histogram there
+ *     that each call leaves zeroed for the next.
  */
 #ifndef CKV_H
 #define CKV_H

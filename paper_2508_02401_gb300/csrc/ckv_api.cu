@@ -249,12 +249,22 @@ ckv_status plan_score(const Plan& pl, const ckv_batch* b, int skip_le, int ctas,
 }
 
 struct WsLayout {
-    size_t header = 0, partials = 0, counters = 0, scores = 0, pooled = 0, total = 0;
+    size_t header = 0, partials = 0, counters = 0, scores = 0, pooled = 0;
+    size_t hist = 0, info = 0, chunk_off = 0, total = 0;
+    int max_chunks = 0;
 };
 
+int max_seqlen(const ckv_batch* b) {
+    int m = 0;
+    for (int s = 0; s < b->num_seqs; ++s)
+        m = std::max(m, b->cu_seqlens_host[s + 1] - b->cu_seqlens_host[s]);
+    return m;
+}
+
 WsLayout ws_layout(const Plan& pl, const ckv_batch* b, int T) {
-    (void)b;
     WsLayout l;
+    const size_t units = static_cast<size_t>(b->num_seqs) * pl.Hkv;
+    l.max_chunks = select_chunks(max_seqlen(b));
     size_t off = round_up(sizeof(WsHeader), kWsAlign);
     l.partials = off;
     off = round_up(off + static_cast<size_t>(kMaxScoreItems) * kMaxCols * sizeof(float2), kWsAlign);
@@ -264,6 +274,12 @@ WsLayout ws_layout(const Plan& pl, const ckv_batch* b, int T) {
     off = round_up(off + static_cast<size_t>(pl.n_sel) * T * sizeof(float), kWsAlign);
     l.pooled = off;
     off = round_up(off + static_cast<size_t>(pl.Hkv) * T * sizeof(float), kWsAlign);
+    l.hist = off;  // zero outside a call: the selection leaves it as it found it
+    off = round_up(off + units * select_hist_ints() * sizeof(int), kWsAlign);
+    l.info = off;
+    off = round_up(off + units * 4 * sizeof(int), kWsAlign);
+    l.chunk_off = off;
+    off = round_up(off + units * l.max_chunks * sizeof(int), kWsAlign);
     l.total = off;
     return l;
 }
@@ -384,9 +400,16 @@ ckv_status enqueue_score(const Plan& pl, const ckv_batch* b, int T, const void* 
 }
 
 SelectLaunch select_launch(const Plan& pl, const ckv_batch* b, int T, int T_keep, int skip_le,
-                           const ckv_config* cfg, void* ws) {
+                           const ckv_config* cfg, void* ws, const WsLayout* l) {
     SelectLaunch L;
     memset(&L, 0, sizeof L);
+    if (l) {
+        uint8_t* w8 = static_cast<uint8_t*>(ws);
+        L.hist = reinterpret_cast<int*>(w8 + l->hist);
+        L.info = reinterpret_cast<int*>(w8 + l->info);
+        L.chunk_off = reinterpret_cast<int*>(w8 + l->chunk_off);
+        L.max_chunks = l->max_chunks;
+    }
     L.cu_seqlens_dev = b->cu_seqlens_dev;
     L.status = static_cast<int*>(ws);
     L.S = b->num_seqs;
@@ -482,7 +505,7 @@ ckv_status ckv_pool(const ckv_config* cfg, int32_t layer, const ckv_batch* batch
     if ((st = check_batch(batch, &T)) || (st = check_kv(scores, "scores", T)) ||
         (st = check_kv(pooled, "pooled", T)))
         return st;
-    SelectLaunch L = select_launch(pl, batch, T, 0, -1, cfg, nullptr);
+    SelectLaunch L = select_launch(pl, batch, T, 0, -1, cfg, nullptr, nullptr);
     L.scores = scores;
     L.pooled = pooled;
     const cudaError_t e = launch_pool(L, reinterpret_cast<cudaStream_t>(stream));
@@ -503,7 +526,7 @@ ckv_status ckv_select_topk(const ckv_config* cfg, int32_t layer, const ckv_batch
     const int64_t tk = keep_total(batch, pl.budget);
     if (tk > 0 && !idx) return fail(CKV_ERR_INVALID_ARG, "idx is NULL");
     if (!cu_keep_dev) return fail(CKV_ERR_INVALID_ARG, "cu_keep_dev is NULL");
-    SelectLaunch L = select_launch(pl, batch, T, static_cast<int>(tk), -1, cfg, workspace);
+    SelectLaunch L = select_launch(pl, batch, T, static_cast<int>(tk), -1, cfg, workspace, &l);
     L.pooled = const_cast<float*>(pooled);
     L.idx = idx;
     L.cu_keep_dev = cu_keep_dev;
@@ -583,34 +606,23 @@ ckv_status ckv_compress_layer(const ckv_config* cfg, int32_t layer, const ckv_ba
     if ((st = enqueue_score(pl, batch, T, q_win, k, tok_stride, head_stride, scores, workspace, l,
                             skip_le, s)))
         return st;
-    SelectLaunch L = select_launch(pl, batch, T, static_cast<int>(tk), skip_le, cfg, workspace);
+    SelectLaunch L = select_launch(pl, batch, T, static_cast<int>(tk), skip_le, cfg, workspace, &l);
     L.scores = scores;
     L.pooled = pooled;
     L.idx = idx;
     L.cu_keep_dev = cu_keep_dev;
-    L.from_scores = 1;                      // pooling is fused into the selection kernel
+    L.from_scores = 1;                      // pooling is fused into the selection
     L.write_pooled = pooled_out != nullptr;
-    cudaError_t e = launch_select(L, s);
-    if (e != cudaSuccess) return cuda_fail(e, "launching the pool + selection kernel");
-    if (tk == 0) return CKV_OK;
-    GatherLaunch G;
-    G.k = k;
-    G.v = v;
-    G.tok_stride = tok_stride;
-    G.head_stride = head_stride;
-    G.idx = idx;
-    G.cu_keep_dev = cu_keep_dev;
-    G.cu_seqlens_dev = batch->cu_seqlens_dev;
-    G.k_out = k_out;
-    G.v_out = v_out;
-    G.status = static_cast<int*>(workspace);
-    G.S = batch->num_seqs;
-    G.T = T;
-    G.Hkv = pl.Hkv;
-    G.T_keep = static_cast<int>(tk);
-    G.cu_hash = seqlens_hash(batch->cu_seqlens_host, batch->num_seqs);
-    e = launch_gather(G, s);
-    return e == cudaSuccess ? CKV_OK : cuda_fail(e, "launching the gather kernel");
+    if (tk > 0) {                           // and so is the gather
+        L.k = k;
+        L.v = v;
+        L.tok_stride = tok_stride;
+        L.head_stride = head_stride;
+        L.k_out = k_out;
+        L.v_out = v_out;
+    }
+    const cudaError_t e = launch_select(L, s);
+    return e == cudaSuccess ? CKV_OK : cuda_fail(e, "launching the pool, selection and gather kernels");
 }
 
 ckv_status ckv_read_device_status(void* workspace, ckv_stream stream, int32_t reset,

@@ -70,10 +70,22 @@ struct SelectLaunch {
     int pool_kernel, pool_type, head_order;
     int skip_le;                // pooled is produced only for sequences with L > skip_le
     int from_scores;            // select: pool the scores on the fly (else read pooled)
-    int write_pooled;           // select with from_scores: also store the pooled scores
+    int write_pooled;           // with from_scores: also store the pooled scores (zeros
+                                //   at window positions and unselected sequences)
     uint32_t cu_hash;
     const int* group_first;     // [H_kv+1] first score row of each group
+    int* hist;                  // [S*H_kv][select_hist_ints()] workspace
+    int* info;                  // [S*H_kv][4] workspace
+    int* chunk_off;             // [S*H_kv][max_chunks] workspace
+    int max_chunks;             // select_chunks(longest sequence)
+    const void* k;              // optional fused gather (nullptr: none)
+    const void* v;
+    int64_t tok_stride, head_stride;
+    void* k_out;
+    void* v_out;
 };
+int select_chunks(int max_len);
+size_t select_hist_ints();
 cudaError_t launch_pool(const SelectLaunch& L, cudaStream_t stream);
 cudaError_t launch_select(const SelectLaunch& L, cudaStream_t stream);
 
