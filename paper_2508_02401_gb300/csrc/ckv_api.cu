@@ -14,6 +14,8 @@
 #include "ckv_device.cuh"
 #include "ckv_internal.h"
 
+#include <limits.h>
+
 namespace ckv {
 namespace {
 
@@ -250,7 +252,7 @@ ckv_status plan_score(const Plan& pl, const ckv_batch* b, int skip_le, int ctas,
 
 struct WsLayout {
     size_t header = 0, partials = 0, counters = 0, scores = 0, pooled = 0;
-    size_t hist = 0, info = 0, chunk_off = 0, total = 0;
+    size_t hist = 0, arrivals = 0, chunk_start = 0, buckets = 0, info = 0, chunk_off = 0, total = 0;
     int max_chunks = 0;
 };
 
@@ -276,6 +278,12 @@ WsLayout ws_layout(const Plan& pl, const ckv_batch* b, int T) {
     off = round_up(off + static_cast<size_t>(pl.Hkv) * T * sizeof(float), kWsAlign);
     l.hist = off;  // zero outside a call: the selection leaves it as it found it
     off = round_up(off + units * select_hist_ints() * sizeof(int), kWsAlign);
+    l.arrivals = off;  // zero outside a call, like hist
+    off = round_up(off + units * sizeof(int), kWsAlign);
+    l.chunk_start = off;
+    off = round_up(off + units * l.max_chunks * select_hist_ints() * sizeof(int), kWsAlign);
+    l.buckets = off;
+    off = round_up(off + units * l.max_chunks * select_chunk_positions() * 8, kWsAlign);
     l.info = off;
     off = round_up(off + units * 4 * sizeof(int), kWsAlign);
     l.chunk_off = off;
@@ -406,6 +414,9 @@ SelectLaunch select_launch(const Plan& pl, const ckv_batch* b, int T, int T_keep
     if (l) {
         uint8_t* w8 = static_cast<uint8_t*>(ws);
         L.hist = reinterpret_cast<int*>(w8 + l->hist);
+        L.arrivals = reinterpret_cast<int*>(w8 + l->arrivals);
+        L.chunk_start = reinterpret_cast<int*>(w8 + l->chunk_start);
+        L.buckets = w8 + l->buckets;
         L.info = reinterpret_cast<int*>(w8 + l->info);
         L.chunk_off = reinterpret_cast<int*>(w8 + l->chunk_off);
         L.max_chunks = l->max_chunks;
@@ -424,6 +435,13 @@ SelectLaunch select_launch(const Plan& pl, const ckv_batch* b, int T, int T_keep
     L.skip_le = skip_le;
     L.cu_hash = seqlens_hash(b->cu_seqlens_host, b->num_seqs);
     L.group_first = pl.group_first.data();
+    L.min_len = INT_MAX;
+    L.max_len = 0;
+    for (int s = 0; s < b->num_seqs; ++s) {
+        const int len = b->cu_seqlens_host[s + 1] - b->cu_seqlens_host[s];
+        L.min_len = std::min(L.min_len, len);
+        L.max_len = std::max(L.max_len, len);
+    }
     return L;
 }
 

@@ -74,10 +74,14 @@ struct SelectLaunch {
                                 //   at window positions and unselected sequences)
     uint32_t cu_hash;
     const int* group_first;     // [H_kv+1] first score row of each group
-    int* hist;                  // [S*H_kv][select_hist_ints()] workspace
+    int* hist;                  // [S*H_kv][select_hist_ints()] workspace, zero between calls
+    int* arrivals;              // [S*H_kv] workspace, zero between calls
+    int* chunk_start;           // [S*H_kv][max_chunks][select_hist_ints()] workspace
+    void* buckets;              // [S*H_kv][max_chunks][select_chunk_positions()] 8-byte pairs
     int* info;                  // [S*H_kv][4] workspace
     int* chunk_off;             // [S*H_kv][max_chunks] workspace
     int max_chunks;             // select_chunks(longest sequence)
+    int min_len, max_len;       // shortest and longest sequence (host lengths)
     const void* k;              // optional fused gather (nullptr: none)
     const void* v;
     int64_t tok_stride, head_stride;
@@ -86,6 +90,8 @@ struct SelectLaunch {
 };
 int select_chunks(int max_len);
 size_t select_hist_ints();
+int select_chunk_positions();
+int select_unit_len();  // units up to this length take the one-block path
 cudaError_t launch_pool(const SelectLaunch& L, cudaStream_t stream);
 cudaError_t launch_select(const SelectLaunch& L, cudaStream_t stream);
 

@@ -8,6 +8,7 @@
 #include <limits.h>
 #include <string.h>
 
+#include <algorithm>
 #include <mutex>
 
 namespace ckv {
@@ -72,42 +73,66 @@ __global__ void __launch_bounds__(256) pool_kernel(const __grid_constant__ PoolP
 }
 
 // ------------------------------------------------------------------------ selection
-// Three kernels per call, each over (sequence, KV head) units:
-//   pool_hist   grid (unit, chunk): pools one chunk of kChunk candidate positions and adds the
-//               chunk's histogram of the top 11 bits of the order-preserving score keys to the
-//               unit's histogram in the workspace;
-//   threshold   one block per unit: the exact k-th largest key, the position up to which the
-//               keys equal to it are kept (lowest positions first, as a stable sort by
-//               descending score would keep them), and each chunk's output offset;
-//   compact     grid (unit, chunk): writes the chunk's kept positions in position order and,
-//               when asked, copies their K/V rows into the compacted cache; chunk 0 also
-//               writes the window.
-// The histogram is zero outside a call: threshold clears each unit's copy once it has read it.
+// Per (sequence, KV head) unit: pool the scores (or read given pooled scores), take the k
+// largest as order-preserving keys (ties: lowest positions first, as a stable sort by
+// descending score keeps them), write their positions in position order followed by the
+// window, and copy their K/V rows into the compacted cache when asked.
+//
+// Units of up to kUnitLen tokens are done by one 1024-thread block each (select_unit_kernel):
+// every key stays in a register, and the k-th largest is found digit by digit (11, 11 and 10
+// bits) with shared-memory counts.
+//
+// Longer units are cut into chunks of kChunk positions:
+//   select_kernel  grid (unit, chunk): pools the chunk, counts its keys by their first digit
+//                  into the unit's histogram and stores them grouped by that digit, highest
+//                  first.  The last chunk block of a unit to finish gathers the keys of the
+//                  digit that holds the k-th largest from every chunk's group and finds the
+//                  threshold key, the tie cutoff position and each chunk's output offset.
+//   compact_kernel grid (unit, chunk): writes the chunk's kept positions in position order and
+//                  copies their rows; chunk 0 also writes the window.
+// The unit histograms and arrival counters are zero outside a call: the last block of each
+// unit clears them once it has read them.
 constexpr int kChunk = 4096;                 // candidate positions per chunk
 constexpr int kChunkShift = 12;
 constexpr int kHistBins = 2048;              // digits of up to 11 bits
 constexpr int kHistShift = 21;               // the first digit is bits 31..21 of a key
-constexpr int kPHThreads = 512;              // pool_hist and compact
-constexpr int kPHPer = kChunk / kPHThreads;  // positions per thread
-constexpr int kPHWarps = kPHThreads / 32;
-constexpr int kWarpSpan = kChunk / kPHWarps; // compact: contiguous positions per warp
+constexpr int kSelThreads = 512;             // select_kernel and compact_kernel
+constexpr int kSelWarps = kSelThreads / 32;
+constexpr int kPHPer = kChunk / kSelThreads; // contiguous positions per thread
+constexpr int kWarpSpan = kChunk / kSelWarps; // compact: contiguous positions per warp
 constexpr int kMaxHalo = kMaxPoolKernel / 2;
 constexpr int kStageFloats = kChunk + 2 * kMaxHalo;
-constexpr int kThThreads = 1024;             // threshold
-constexpr int kCandCap = 8192;               // threshold: candidates kept in shared memory
+constexpr int kStageLoads = (kStageFloats + kSelThreads - 1) / kSelThreads;
+constexpr int kCandCap = 8192;               // candidates held in shared memory
+constexpr int kTieCap = 256;                 // ties ranked pairwise up to this many
 constexpr int kCompactSmem = kChunk * 4;     // compact: the chunk's kept positions
-constexpr uint32_t kTaken = 0xFFFFFFFEu;     // candidate markers (the top bit excludes them
-constexpr uint32_t kDropped = 0xFFFFFFFFu;   // from the tie-position select)
+constexpr uint32_t kTaken = 0xFFFFFFFEu;     // tie-select markers; the top bit keeps both out
+constexpr uint32_t kDropped = 0xFFFFFFFFu;   //   of the position select
+constexpr int kUnitThreads = 1024;           // select_unit_kernel
+constexpr int kUnitPer = 16;
+constexpr int kUnitLen = kUnitThreads * kUnitPer;
+constexpr int kUnitStage = kUnitLen + 2 * kMaxHalo;
+constexpr int kUnitStageLoads = (kUnitStage + kUnitThreads - 1) / kUnitThreads;
 static_assert(kWarpSpan % 32 == 0 && (1 << kChunkShift) == kChunk, "chunk shape");
 
+// Shared-memory index of staged element e: one pad word per 32 keeps the contiguous
+// per-thread reads of the pooling free of bank conflicts.
+__device__ __forceinline__ int sidx(int e) { return e + (e >> 5); }
+constexpr int stage_words(int n) { return n + (n >> 5) + 2; }
+constexpr int kUnitSmem = stage_words(kUnitStage) * 4;
+constexpr int kSelStageSmem = stage_words(kStageFloats) * 4;
+
 struct SelectParams {
-    const float* scores;   // [n_sel, T]: pooled in pool_hist when from_scores != 0
+    const float* scores;   // [n_sel, T]: pooled here when from_scores != 0
     float* pooled;         // [H_kv, T]
     int32_t* idx;          // [H_kv, T_keep]
     int32_t* cu_keep;      // [S+1]
     const int32_t* cu_seqlens;
     int* status;
-    int* hist;             // [units][kHistBins]
+    int* hist;             // [units][kHistBins] first-digit counts
+    int* arrivals;         // [units] chunk blocks done
+    int* chunk_start;      // [units][max_chunks][kHistBins] start of each digit group
+    uint2* buckets;        // [units][max_chunks][kChunk] (key, position) grouped by digit
     int* info;             // [units][4]: threshold key, tie cutoff position
     int* chunk_off;        // [units][max_chunks]: output offset of each chunk's kept positions
     const uint4* k;        // gather source (nullptr: no gather); strides in 16-byte units
@@ -120,6 +145,12 @@ struct SelectParams {
     uint32_t cu_hash;
     int16_t group_first[kMaxQHeads + 1];
 };
+
+__device__ __forceinline__ int atomic_add_acq_rel(int* p, int v) {
+    int old;
+    asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+    return old;
+}
 
 // Order-preserving unsigned key of a float (-0 and +0 share one key).
 __device__ __forceinline__ uint32_t rank_key(float f) {
@@ -154,7 +185,7 @@ __device__ __forceinline__ bool unit_geo(const SelectParams& p, int unit, UnitGe
     return true;
 }
 
-// Block-wide exclusive prefix sum over NT threads in thread order; *total gets the sum.
+// Block-wide exclusive prefix sum in thread order over NT threads; *total gets the sum.
 template <int NT>
 __device__ __forceinline__ int block_excl_scan(int v, int* scratch, int* total) {
     constexpr int NW = NT / 32;
@@ -185,6 +216,165 @@ __device__ __forceinline__ int block_excl_scan(int v, int* scratch, int* total) 
     return r;
 }
 
+// The digit d of a kHistBins-bin histogram with count(bins above d) < r <= count(bins >= d),
+// r >= 1: *s_digit = d, *s_above = count(bins above d).  Thread 0 owns the highest bins.
+template <int NT>
+__device__ __forceinline__ void find_digit(const int* hist, int r, int* scratch, int* s_digit,
+                                           int* s_above) {
+    constexpr int PER = kHistBins / NT;
+    if (threadIdx.x == 0) {
+        *s_digit = 0;
+        *s_above = 0;
+    }
+    const int base = (NT - 1 - static_cast<int>(threadIdx.x)) * PER;
+    int local = 0;
+#pragma unroll
+    for (int q = 0; q < PER; ++q) local += hist[base + q];
+    int tot;
+    const int above = block_excl_scan<NT>(local, scratch, &tot);
+    if (above < r && above + local >= r) {
+        int acc = above;
+        for (int q = PER - 1; q >= 0; --q) {
+            const int h = hist[base + q];
+            if (acc + h >= r) {
+                *s_digit = base + q;
+                *s_above = acc;
+                break;
+            }
+            acc += h;
+        }
+    }
+    __syncthreads();
+}
+
+// Adds a thread's run-aggregated counts of PER consecutive digits to a shared histogram:
+// consecutive keys of a thread are neighbouring positions and often share a digit.
+template <int PER>
+__device__ __forceinline__ void add_runs(int* hist, const uint32_t (&bins)[PER], int nvalid) {
+#pragma unroll
+    for (int i = 0; i < PER; ++i) {
+        if (i < nvalid && (i == 0 || bins[i] != bins[i - 1])) {
+            int len = 1;
+            bool run = true;
+#pragma unroll
+            for (int q = i + 1; q < PER; ++q) {
+                run = run && q < nvalid && bins[q] == bins[i];
+                len += run ? 1 : 0;
+            }
+            atomicAdd(&hist[bins[i]], len);
+        }
+    }
+}
+
+// Stages the sum of score rows [ra, rb) at sequence positions base-half .. base+n+half-1
+// (zero outside [0, P)) into st, element e at st[sidx(e)]; loads are coalesced and all of a
+// row's loads of a thread are issued before its stores.
+template <int NT, int LOADS>
+__device__ __forceinline__ void stage_rows(float* st, const float* scores, size_t T, int t0, int ra,
+                                           int rb, int base, int half, int n, int P) {
+    const int ne = n + 2 * half, tid = threadIdx.x;
+    float xs[LOADS];
+#pragma unroll
+    for (int i = 0; i < LOADS; ++i) xs[i] = 0.f;
+    for (int r = ra; r < rb; ++r) {
+        const float* row = scores + static_cast<size_t>(r) * T + t0;
+#pragma unroll
+        for (int i = 0; i < LOADS; ++i) {
+            const int e = tid + i * NT;
+            const int uu = base - half + e;
+            if (e < ne && uu >= 0 && uu < P) xs[i] += __ldg(row + uu);
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < LOADS; ++i) {
+        const int e = tid + i * NT;
+        if (e < ne) st[sidx(e)] = xs[i];
+    }
+}
+
+// Pools PER consecutive outputs from the stage: output i reads staged elements
+// jl+i .. jl+i+2*HALF.  Same arithmetic, in the same order, as pool_kernel: the staged zeros
+// outside [0, P) leave a max of non-negative scores and a left-to-right sum unchanged.
+template <int HALF, int PER>
+__device__ __forceinline__ void pool_window(const float* st, int jl, int nvalid, bool is_max, float kf,
+                                            float (&acc)[PER]) {
+    float w[PER + 2 * HALF];
+#pragma unroll
+    for (int i = 0; i < PER + 2 * HALF; ++i) w[i] = st[sidx(jl + i)];
+#pragma unroll
+    for (int i = 0; i < PER; ++i) {
+        if (i < nvalid) {
+            float m = w[i];
+            if (is_max) {
+#pragma unroll
+                for (int t = 1; t <= 2 * HALF; ++t) m = fmaxf(m, w[i + t]);
+                acc[i] += m;
+            } else {
+#pragma unroll
+                for (int t = 1; t <= 2 * HALF; ++t) m += w[i + t];
+                acc[i] += m / kf;  // IEEE division, as in pool_kernel
+            }
+        }
+    }
+}
+
+template <int PER>
+__device__ __forceinline__ void pool_any(const float* st, int jl, int nvalid, int half, bool is_max,
+                                         float kf, float (&acc)[PER]) {
+    if (half == 3) {
+        pool_window<3, PER>(st, jl, nvalid, is_max, kf, acc);
+    } else if (half == 2) {
+        pool_window<2, PER>(st, jl, nvalid, is_max, kf, acc);
+    } else {
+#pragma unroll
+        for (int i = 0; i < PER; ++i) {
+            if (i < nvalid) {
+                float m = st[sidx(jl + i)];
+                for (int t = 1; t <= 2 * half; ++t)
+                    m = is_max ? fmaxf(m, st[sidx(jl + i + t)]) : m + st[sidx(jl + i + t)];
+                acc[i] += is_max ? m : m / kf;
+            }
+        }
+    }
+}
+
+// Pooled scores of positions base+jl .. base+jl+PER-1 (jl = PER * thread) of unit u, computed
+// from the scores (from_scores) or read from p.pooled.  Ends with the stage free again.
+template <int NT, int PER, int LOADS>
+__device__ __forceinline__ void pooled_values(const SelectParams& p, const UnitGeo& u, float* st, int base,
+                                              int n, float (&acc)[PER]) {
+    const int jl = threadIdx.x * PER, nvalid = n - jl;
+#pragma unroll
+    for (int i = 0; i < PER; ++i) acc[i] = 0.f;
+    if (p.from_scores) {
+        const int half = p.pool_kernel >> 1;
+        const bool is_max = p.pool_type == 0;
+        const float kf = static_cast<float>(p.pool_kernel);
+        const int r0 = p.group_first[u.g], r1 = p.group_first[u.g + 1];
+        const bool per_head = p.head_order == 0;
+        const int passes = per_head ? r1 - r0 : 1;
+        for (int ps = 0; ps < passes; ++ps) {
+            const int ra = per_head ? r0 + ps : r0, rb = per_head ? ra + 1 : r1;
+            stage_rows<NT, LOADS>(st, p.scores, p.T, u.t0, ra, rb, base, half, n, u.P);
+            __syncthreads();
+            pool_any<PER>(st, jl, nvalid, half, is_max, kf, acc);
+            __syncthreads();
+        }
+    } else {
+        const float* src = p.pooled + static_cast<size_t>(u.g) * p.T + u.t0 + base;
+#pragma unroll
+        for (int i = 0; i < LOADS; ++i) {
+            const int e = threadIdx.x + i * NT;
+            if (e < n) st[sidx(e)] = __ldg(src + e);
+        }
+        __syncthreads();
+#pragma unroll
+        for (int i = 0; i < PER; ++i)
+            if (i < nvalid) acc[i] = st[sidx(jl + i)];
+        __syncthreads();
+    }
+}
+
 // Copies the K and V rows of sequence-local positions list[0..m) to output rows
 // out_row0 + 0..m-1 of KV head g: a warp per row (16 lanes for K, 16 for V), four rows in
 // flight per warp.
@@ -210,399 +400,446 @@ __device__ __forceinline__ void copy_rows(const SelectParams& p, const UnitGeo& 
     }
 }
 
-__global__ void __launch_bounds__(kPHThreads) pool_hist_kernel(const __grid_constant__ SelectParams p) {
-    extern __shared__ float stage[];  // [kStageFloats]
+// ------------------------------------------------------------------ units of up to kUnitLen
+__global__ void __launch_bounds__(kUnitThreads, 1) select_unit_kernel(const __grid_constant__ SelectParams p) {
+    extern __shared__ __align__(16) float ust[];  // pooling stage, then the kept list
     __shared__ int hist[kHistBins];
-    const int unit = blockIdx.x, c = blockIdx.y, tid = threadIdx.x, lane = tid & 31;
-    if (unit == 0 && c == 0 && tid == 0 && seqlens_hash(p.cu_seqlens, p.S) != p.cu_hash)
-        record_error(p.status, kDevBadSeqlens, 200);
+    __shared__ int scratch[33];
+    __shared__ int s_digit, s_above, s_cut;
+    constexpr int NT = kUnitThreads, PER = kUnitPer;
+    const int unit = blockIdx.x, tid = threadIdx.x;
+    if (unit == 0 && tid == 0 && seqlens_hash(p.cu_seqlens, p.S) != p.cu_hash)
+        record_error(p.status, kDevBadSeqlens, 230);
     UnitGeo u;
     if (!unit_geo(p, unit, u)) return;
+    if (u.L > kUnitLen) return;  // a long unit: the chunked kernels take it
+    if (u.g == 0 && tid == 0) {
+        p.cu_keep[u.s + 1] = u.keep_off + u.n_keep;
+        if (u.s == 0) p.cu_keep[0] = 0;
+    }
+    int32_t* out = p.idx + static_cast<size_t>(u.g) * p.T_keep + u.keep_off;
     float* pooled = p.pooled + static_cast<size_t>(u.g) * p.T + u.t0;
-    const int j0 = c * kChunk;
+    int* list = reinterpret_cast<int*>(ust);
     const bool zeros = p.from_scores && p.write_pooled;
-    if (u.L <= p.budget) {  // kept whole: nothing to select; its pooled scores read as 0
-        if (zeros)
-            for (int j = j0 + tid; j < min(u.L, j0 + kChunk); j += kPHThreads) pooled[j] = 0.f;
+    if (u.L <= p.budget) {  // kept whole; its pooled scores read as 0
+        for (int e = tid; e < u.L; e += NT) {
+            out[e] = e;
+            list[e] = e;
+            if (zeros) pooled[e] = 0.f;
+        }
+        __syncthreads();
+        if (p.k) copy_rows(p, u, list, u.L, u.keep_off);
         return;
     }
+    const int P = u.P, k = u.k;
     if (zeros)  // window positions are not candidates
-        for (int j = max(j0, u.P) + tid; j < min(u.L, j0 + kChunk); j += kPHThreads) pooled[j] = 0.f;
-    if (j0 >= u.P) return;
-    const int n = min(kChunk, u.P - j0);
-    float acc[kPHPer];
+        for (int j = P + tid; j < u.L; j += NT) pooled[j] = 0.f;
+    const int jb = tid * PER, nvalid = P - jb;
+    float acc[PER];
+    pooled_values<NT, PER, kUnitStageLoads>(p, u, ust, 0, P, acc);
+    if (zeros)
 #pragma unroll
-    for (int i = 0; i < kPHPer; ++i) acc[i] = 0.f;
-    if (p.from_scores) {
-        // Same arithmetic, in the same order, as pool_kernel: the zeros staged outside [0, P)
-        // leave a max of non-negative scores and a sum unchanged.
-        const int half = p.pool_kernel >> 1;
-        const bool is_max = p.pool_type == 0;
-        const float kf = static_cast<float>(p.pool_kernel);
-        const int r0 = p.group_first[u.g], r1 = p.group_first[u.g + 1];
-        const float* base = p.scores + u.t0;
-        const int passes = p.head_order == 0 ? r1 - r0 : 1;
-        for (int ps = 0; ps < passes; ++ps) {
-            // stage positions j0-half .. j0+n+half-1; each thread issues all its loads first
-            constexpr int kStagePer = (kStageFloats + kPHThreads - 1) / kPHThreads;
-            float xs[kStagePer];
+        for (int i = 0; i < PER; ++i)
+            if (i < nvalid) pooled[jb + i] = acc[i];
+    uint32_t key[PER], bins[PER];
 #pragma unroll
-            for (int i = 0; i < kStagePer; ++i) {
-                const int e = tid + i * kPHThreads;
-                const int uu = j0 - half + e;
-                float x = 0.f;
-                if (e < n + 2 * half && uu >= 0 && uu < u.P) {
-                    if (p.head_order == 0) {
-                        x = __ldg(base + static_cast<size_t>(r0 + ps) * p.T + uu);
-                    } else {
-                        for (int r = r0; r < r1; ++r) x += __ldg(base + static_cast<size_t>(r) * p.T + uu);
-                    }
-                }
-                xs[i] = x;
-            }
-#pragma unroll
-            for (int i = 0; i < kStagePer; ++i) {
-                const int e = tid + i * kPHThreads;
-                if (e < n + 2 * half) stage[e] = xs[i];
-            }
+    for (int i = 0; i < PER; ++i) {
+        key[i] = rank_key(acc[i]);
+        bins[i] = key[i] >> kHistShift;
+    }
+    // the k-th largest key, digit by digit (k = 0 keeps only the window: no key is above
+    // 0xffffffff and no position is at or below -1)
+    uint32_t thr = 0xFFFFFFFFu;
+    int pos_cut = -1;
+    if (k > 0) {
+        for (int b = tid; b < kHistBins; b += NT) hist[b] = 0;
+        if (tid == 0) s_cut = INT_MAX;
+        __syncthreads();
+        add_runs<PER>(hist, bins, nvalid);
+        __syncthreads();
+        find_digit<NT>(hist, k, scratch, &s_digit, &s_above);
+        uint32_t prefix = static_cast<uint32_t>(s_digit) << kHistShift, mask = 0x7FFu << kHistShift;
+        int r = k - s_above, n_eq = hist[s_digit];
+        __syncthreads();
+#pragma unroll 1
+        for (int level = 0; level < 2; ++level) {
+            const int shift = level == 0 ? 10 : 0;
+            const uint32_t dmask = level == 0 ? 0x7FFu : 0x3FFu;
+            for (int b = tid; b < kHistBins; b += NT) hist[b] = 0;
             __syncthreads();
 #pragma unroll
-            for (int i = 0; i < kPHPer; ++i) {
-                const int jl = tid + i * kPHThreads;  // its window: stage[jl .. jl + 2*half]
-                if (jl < n) {
-                    float m = stage[jl];
-                    if (is_max) {
-                        for (int t = 1; t <= 2 * half; ++t) m = fmaxf(m, stage[jl + t]);
-                        acc[i] += m;
-                    } else {
-                        for (int t = 1; t <= 2 * half; ++t) m += stage[jl + t];
-                        acc[i] += m / kf;  // IEEE division, as in pool_kernel
+            for (int i = 0; i < PER; ++i)
+                if (i < nvalid && (key[i] & mask) == prefix) atomicAdd(&hist[(key[i] >> shift) & dmask], 1);
+            __syncthreads();
+            find_digit<NT>(hist, r, scratch, &s_digit, &s_above);
+            prefix |= static_cast<uint32_t>(s_digit) << shift;
+            mask |= dmask << shift;
+            r -= s_above;
+            n_eq = hist[s_digit];
+            __syncthreads();
+        }
+        thr = prefix;
+        const int need_eq = r;  // keys equal to thr that are kept: the lowest positions
+        pos_cut = INT_MAX;
+        if (need_eq < n_eq) {
+            int ne = 0;
+#pragma unroll
+            for (int i = 0; i < PER; ++i) ne += (i < nvalid && key[i] == thr) ? 1 : 0;
+            int tot;
+            const int before = block_excl_scan<NT>(ne, scratch, &tot);  // thread order = position order
+            if (before < need_eq && before + ne >= need_eq) {
+                int c = before;
+#pragma unroll
+                for (int i = 0; i < PER; ++i) {
+                    if (i < nvalid && key[i] == thr) {
+                        ++c;
+                        if (c == need_eq) s_cut = jb + i;
                     }
                 }
             }
             __syncthreads();
-        }
-#pragma unroll
-        for (int i = 0; i < kPHPer; ++i) {
-            const int jl = tid + i * kPHThreads;
-            if (jl < n) pooled[j0 + jl] = acc[i];
-        }
-    } else {
-#pragma unroll
-        for (int i = 0; i < kPHPer; ++i) {
-            const int jl = tid + i * kPHThreads;
-            acc[i] = jl < n ? __ldg(pooled + j0 + jl) : 0.f;
+            pos_cut = s_cut;
         }
     }
-    // the chunk's histogram of the first digit, then into the unit's histogram
-    for (int b = tid; b < kHistBins; b += kPHThreads) hist[b] = 0;
-    __syncthreads();
+    // the kept positions in order, then the window
+    uint32_t taken = 0;
+    int cnt = 0;
 #pragma unroll
-    for (int i = 0; i < kPHPer; ++i) {
-        const int jl = tid + i * kPHThreads;
-        const bool in = jl < n;
-        const uint32_t bin = in ? (rank_key(acc[i]) >> kHistShift) : static_cast<uint32_t>(kHistBins);
-        const unsigned peers = __match_any_sync(0xffffffffu, bin);
-        if (in && lane == __ffs(peers) - 1) atomicAdd(&hist[bin], __popc(peers));
+    for (int i = 0; i < PER; ++i) {
+        if (i < nvalid && (key[i] > thr || (key[i] == thr && jb + i <= pos_cut))) {
+            taken |= 1u << i;
+            ++cnt;
+        }
     }
-    __syncthreads();
-    int* gh = p.hist + static_cast<size_t>(unit) * kHistBins;
-    for (int b = tid; b < kHistBins; b += kPHThreads) {
-        const int h = hist[b];
-        if (h) atomicAdd(gh + b, h);
-    }
-}
-
-// The digit d of a kHistBins-bin histogram with count(bins above d) < r <= count(bins >= d)
-// (r >= 1): *s_digit = d, *s_above = count(bins above d).  Thread 0 owns the highest bins.
-__device__ __forceinline__ void find_digit(const int* hist, int r, int* scratch, int* s_digit,
-                                           int* s_above) {
-    constexpr int PER = kHistBins / kThThreads;
-    if (threadIdx.x == 0) {
-        *s_digit = 0;
-        *s_above = 0;
-    }
-    const int base = (kThThreads - 1 - static_cast<int>(threadIdx.x)) * PER;
-    int local = 0;
-#pragma unroll
-    for (int q = 0; q < PER; ++q) local += hist[base + q];
     int tot;
-    const int above = block_excl_scan<kThThreads>(local, scratch, &tot);
-    if (above < r && above + local >= r) {
-        int acc = above;
-        for (int q = PER - 1; q >= 0; --q) {
-            const int h = hist[base + q];
-            if (acc + h >= r) {
-                *s_digit = base + q;
-                *s_above = acc;
-                break;
-            }
-            acc += h;
+    int rk = block_excl_scan<NT>(cnt, scratch, &tot);
+    if (tot != k) {
+        if (tid == 0) record_error(p.status, kDevBadIndex, 330 + unit);
+        return;
+    }
+#pragma unroll
+    for (int i = 0; i < PER; ++i) {
+        if ((taken >> i) & 1u) {
+            out[rk] = jb + i;
+            list[rk] = jb + i;
+            ++rk;
         }
     }
+    for (int i = tid; i < p.w; i += NT) {
+        out[k + i] = P + i;
+        list[k + i] = P + i;
+    }
     __syncthreads();
+    if (p.k) copy_rows(p, u, list, p.budget, u.keep_off);
 }
 
-struct SelectState {
-    int hist[kHistBins];
+// ------------------------------------------------------------------ longer units, in chunks
+struct SelectShared {
+    int hist[kHistBins];   // chunk counts, then group starts; the unit's counts in the last block
+    int fill[kHistBins];   // group fill pointers
     int scratch[33];
-    int digit, above, n_cand, cut_chunk, cut_take, cut_pos;
+    int digit, above, last, n_cand, n_tie, cut;
 };
 
-// The r-th largest (r >= 1) of the values vals[0..n) whose bits under `mask` equal `prefix`,
-// found digit by digit over the `bits` lower bits.  *r_eq gets how many of the copies of the
-// result rank within the first r, *n_eq how many copies there are.
-__device__ uint32_t smem_select(const uint32_t* vals, int n, uint32_t prefix, uint32_t mask, int bits,
-                                int r, SelectState& st, int* r_eq, int* n_eq) {
+// The r-th largest (r >= 1) of the values get(0..n) whose bits under `mask` equal `prefix`,
+// digit by digit over the `bits` lower bits.  *r_eq gets how many copies of the result rank
+// within the first r, *n_eq how many copies there are.  Uses (and leaves garbage in) sh.hist.
+template <class Get>
+__device__ uint32_t radix_select(Get get, int n, uint32_t prefix, uint32_t mask, int bits, int r,
+                                 SelectShared& sh, int* r_eq, int* n_eq) {
     const int tid = threadIdx.x, lane = tid & 31;
     int last = 0;
     while (bits > 0) {
         const int d = bits > 11 ? 11 : bits;
         const int shift = bits - d;
         const uint32_t dmask = (1u << d) - 1u;
-        for (int b = tid; b < kHistBins; b += kThThreads) st.hist[b] = 0;
+        for (int b = tid; b < kHistBins; b += kSelThreads) sh.hist[b] = 0;
         __syncthreads();
-        for (int i0 = 0; i0 < n; i0 += kThThreads) {
+        for (int i0 = 0; i0 < n; i0 += kSelThreads) {
             const int i = i0 + tid;
-            const uint32_t x = i < n ? vals[i] : 0u;
+            const uint32_t x = i < n ? get(i) : 0u;
             const bool in = i < n && (x & mask) == prefix;
-            const uint32_t bin = in ? (x >> shift) & dmask : static_cast<uint32_t>(kHistBins);
-            const unsigned peers = __match_any_sync(0xffffffffu, bin);
-            if (in && lane == __ffs(peers) - 1) atomicAdd(&st.hist[bin], __popc(peers));
+            if (__any_sync(0xffffffffu, in)) {
+                const uint32_t bin = in ? (x >> shift) & dmask : static_cast<uint32_t>(kHistBins);
+                const unsigned peers = __match_any_sync(0xffffffffu, bin);
+                if (in && lane == __ffs(peers) - 1) atomicAdd(&sh.hist[bin], __popc(peers));
+            }
         }
         __syncthreads();
-        find_digit(st.hist, r, st.scratch, &st.digit, &st.above);
-        const int dg = st.digit;
-        last = st.hist[dg];
+        find_digit<kSelThreads>(sh.hist, r, sh.scratch, &sh.digit, &sh.above);
+        const int dg = sh.digit;
+        last = sh.hist[dg];
         prefix |= static_cast<uint32_t>(dg) << shift;
         mask |= dmask << shift;
-        r -= st.above;
+        r -= sh.above;
         bits -= d;
-        __syncthreads();  // everyone has read hist and digit before they are reused
+        __syncthreads();  // hist and digit are read before the next digit reuses them
     }
     *r_eq = r;
     *n_eq = last;
     return prefix;
 }
 
-__global__ void __launch_bounds__(kThThreads, 1) threshold_kernel(const __grid_constant__ SelectParams p) {
-    extern __shared__ uint32_t th_smem[];  // cand_key[kCandCap] cand_pos[kCandCap] cnt eqc [max_chunks]
-    __shared__ SelectState st;
-    uint32_t* cand_key = th_smem;
-    int* cand_pos = reinterpret_cast<int*>(th_smem + kCandCap);
-    int* cnt = reinterpret_cast<int*>(th_smem + 2 * kCandCap);
-    int* eqc = cnt + p.max_chunks;
-    const int unit = blockIdx.x, tid = threadIdx.x, lane = tid & 31;
-    // take the unit's first-digit histogram and leave zeros behind for the next call
+// The threshold of one unit, run by the last of its chunk blocks (see select_kernel).
+// dyn: cand_key[kCandCap] cand_pos[kCandCap] above[max_chunks] coff[max_chunks+1] cnt[max_chunks]
+//      tie_pos[kTieCap]
+__device__ __noinline__ void unit_threshold(const SelectParams& p, const UnitGeo& u, int unit, int nch,
+                                            SelectShared& sh, uint32_t* dyn) {
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    uint32_t* cand_key = dyn;
+    int* cand_pos = reinterpret_cast<int*>(dyn + kCandCap);
+    int* above = reinterpret_cast<int*>(dyn + 2 * kCandCap);
+    int* coff = above + p.max_chunks;
+    int* cnt = coff + p.max_chunks + 1;
+    int* tie_pos = cnt + p.max_chunks;
+    int* info = p.info + unit * 4;
+    int* out_off = p.chunk_off + static_cast<size_t>(unit) * p.max_chunks;
+    const int P = u.P, k = u.k;
+    // the unit's digit counts, left zeroed for the next call
     int* gh = p.hist + static_cast<size_t>(unit) * kHistBins;
-    for (int b = tid; b < kHistBins; b += kThThreads) {
-        st.hist[b] = __ldcg(gh + b);
+    for (int b = tid; b < kHistBins; b += kSelThreads) {
+        sh.hist[b] = __ldcg(gh + b);
         __stcg(gh + b, 0);
     }
-    UnitGeo u;
-    if (!unit_geo(p, unit, u)) return;
-    if (u.L <= p.budget) return;
-    const int P = u.P, k = u.k, nch = (P + kChunk - 1) / kChunk;
-    int* info = p.info + unit * 4;
-    int* coff = p.chunk_off + static_cast<size_t>(unit) * p.max_chunks;
-    if (nch > p.max_chunks) {
-        if (tid == 0) record_error(p.status, kDevBadSeqlens, 210);
-        return;
+    if (tid == 0) {
+        p.arrivals[unit] = 0;
+        sh.n_tie = 0;
+        sh.cut = INT_MAX;
     }
+    __syncthreads();
     if (k == 0) {  // only the window is kept
         if (tid == 0) {
             info[0] = -1;  // key 0xffffffff: no key is above it
             info[1] = -1;
         }
-        for (int c = tid; c < nch; c += kThThreads) coff[c] = 0;
+        for (int c = tid; c < nch; c += kSelThreads) out_off[c] = 0;
         return;
     }
-    const float* pooled = p.pooled + static_cast<size_t>(u.g) * p.T + u.t0;
-    for (int c = tid; c < nch; c += kThThreads) {
-        cnt[c] = 0;
-        eqc[c] = 0;
-    }
-    if (tid == 0) st.n_cand = 0;
-    __syncthreads();
-    find_digit(st.hist, k, st.scratch, &st.digit, &st.above);
-    const uint32_t d1 = static_cast<uint32_t>(st.digit);
-    const int r1 = k - st.above;           // rank of the k-th key within its first-digit bin
-    const int bin_count = st.hist[d1];
-    uint32_t thr;
-    int pos_cut;
-    if (bin_count <= kCandCap) {
-        // One pass over the keys: count the keys of higher bins per chunk (all kept) and
-        // collect the keys of bin d1 with their positions; the rest works in shared memory.
-        for (int j0 = 0; j0 < P; j0 += 4 * kThThreads) {
-            uint32_t key[4];
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const int j = j0 + q * kThThreads + tid;
-                key[q] = j < P ? rank_key(__ldcg(pooled + j)) : 0u;
-            }
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const int j = j0 + q * kThThreads + tid;  // a warp's 32 positions share a chunk
-                const uint32_t b = key[q] >> kHistShift;
-                const unsigned ba = __ballot_sync(0xffffffffu, j < P && b > d1);
-                const unsigned bc = __ballot_sync(0xffffffffu, j < P && b == d1);
-                if (lane == 0 && ba) atomicAdd(&cnt[(j0 + q * kThThreads + (tid & ~31)) >> kChunkShift], __popc(ba));
-                if (bc) {
-                    int slot = 0;
-                    if (lane == 0) slot = atomicAdd(&st.n_cand, __popc(bc));
-                    slot = __shfl_sync(0xffffffffu, slot, 0) + __popc(bc & ((1u << lane) - 1u));
-                    if (((bc >> lane) & 1u) && slot < kCandCap) {
-                        cand_key[slot] = key[q];
-                        cand_pos[slot] = j;
-                    }
-                }
-            }
-        }
-        __syncthreads();
-        const int n = st.n_cand;
-        if (n != bin_count) {  // the keys changed between the two reads
-            if (tid == 0) record_error(p.status, kDevBadIndex, 310 + unit);
-            return;
-        }
-        int need_eq, n_eq;
-        thr = smem_select(cand_key, n, d1 << kHistShift, 0x7FFu << kHistShift, kHistShift, r1, st,
-                          &need_eq, &n_eq);
-        // mark the candidates: above the threshold, tied with it (by position), or dropped
-        for (int i = tid; i < n; i += kThThreads) {
-            const uint32_t x = cand_key[i];
-            cand_key[i] = x > thr ? kTaken : (x == thr ? 0x7FFFFFFFu - static_cast<uint32_t>(cand_pos[i]) : kDropped);
-        }
-        __syncthreads();
-        pos_cut = INT_MAX;  // every tie is kept
-        if (need_eq < n_eq) {  // the need_eq-th smallest tie position, as the largest 0x7fffffff - pos
-            int r_eq, n_eq2;
-            const uint32_t v = smem_select(cand_key, n, 0u, 0x80000000u, 31, need_eq, st, &r_eq, &n_eq2);
-            pos_cut = static_cast<int>(0x7FFFFFFFu - v);
-        }
-        for (int i = tid; i < n; i += kThThreads) {
-            const uint32_t x = cand_key[i];
-            if (x == kTaken || (x < 0x80000000u && static_cast<int>(0x7FFFFFFFu - x) <= pos_cut))
-                atomicAdd(&cnt[cand_pos[i] >> kChunkShift], 1);
-        }
-        __syncthreads();
-    } else {
-        // Too many keys share the first digit: two more digit passes over all of the unit's
-        // keys, then per-chunk counts of the keys above and equal to the threshold.
-        uint32_t prefix = d1 << kHistShift, mask = 0x7FFu << kHistShift;
-        int r = r1, last = 0;
-#pragma unroll 1
-        for (int level = 0; level < 2; ++level) {
-            const int shift = level == 0 ? 10 : 0;
-            const uint32_t dmask = level == 0 ? 0x7FFu : 0x3FFu;
-            for (int b = tid; b < kHistBins; b += kThThreads) st.hist[b] = 0;
-            __syncthreads();
-            for (int j0 = 0; j0 < P; j0 += 4 * kThThreads) {
-                uint32_t key[4];
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const int j = j0 + q * kThThreads + tid;
-                    key[q] = j < P ? rank_key(__ldcg(pooled + j)) : 0u;
-                }
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const int j = j0 + q * kThThreads + tid;
-                    const bool in = j < P && (key[q] & mask) == prefix;
-                    const uint32_t bin = in ? ((key[q] >> shift) & dmask) : static_cast<uint32_t>(kHistBins);
-                    const unsigned peers = __match_any_sync(0xffffffffu, bin);
-                    if (in && lane == __ffs(peers) - 1) atomicAdd(&st.hist[bin], __popc(peers));
-                }
-            }
-            __syncthreads();
-            find_digit(st.hist, r, st.scratch, &st.digit, &st.above);
-            last = st.hist[st.digit];
-            prefix |= static_cast<uint32_t>(st.digit) << shift;
-            mask |= dmask << shift;
-            r -= st.above;
-            __syncthreads();
-        }
-        thr = prefix;
-        const int need_eq = r, n_eq = last;
-        for (int j0 = 0; j0 < P; j0 += 4 * kThThreads) {
-            uint32_t key[4];
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const int j = j0 + q * kThThreads + tid;
-                key[q] = j < P ? rank_key(__ldcg(pooled + j)) : 0u;
-            }
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const int j = j0 + q * kThThreads + tid;
-                const unsigned bg = __ballot_sync(0xffffffffu, j < P && key[q] > thr);
-                const unsigned be = __ballot_sync(0xffffffffu, j < P && key[q] == thr);
-                if (lane == 0 && (bg | be)) {
-                    const int c = (j0 + q * kThThreads + (tid & ~31)) >> kChunkShift;
-                    if (bg) atomicAdd(&cnt[c], __popc(bg));
-                    if (be) atomicAdd(&eqc[c], __popc(be));
-                }
-            }
-        }
-        __syncthreads();
-        pos_cut = INT_MAX;
-        if (need_eq < n_eq) {
-            // the chunk holding the need_eq-th tie in position order, then a walk through it
-            if (tid == 0) {
-                int before = 0, cc = nch - 1;
-                for (int c = 0; c < nch; ++c) {
-                    if (before + eqc[c] >= need_eq) {
-                        cc = c;
-                        break;
-                    }
-                    before += eqc[c];
-                }
-                st.cut_chunk = cc;
-                st.cut_take = need_eq - before;
-                st.cut_pos = INT_MAX;
-            }
-            __syncthreads();
-            const int cc = st.cut_chunk, take = st.cut_take;
-            int seen = 0;
-            for (int b0 = cc * kChunk; b0 < min(P, (cc + 1) * kChunk); b0 += kThThreads) {
-                const int j = b0 + tid;
-                const bool is_eq = j < P && rank_key(__ldcg(pooled + j)) == thr;
-                int tot;
-                const int rk = block_excl_scan<kThThreads>(is_eq ? 1 : 0, st.scratch, &tot);
-                if (is_eq && seen + rk == take - 1) st.cut_pos = j;
-                seen += tot;
-                if (seen >= take) break;  // uniform: every thread has the same `seen`
-            }
-            __syncthreads();
-            pos_cut = st.cut_pos;
-            for (int c = tid; c < nch; c += kThThreads)
-                cnt[c] += c < cc ? eqc[c] : (c == cc ? take : 0);
-        } else {
-            for (int c = tid; c < nch; c += kThThreads) cnt[c] += eqc[c];
-        }
-        __syncthreads();
-    }
-    // output offsets of the chunks: an exclusive scan of their kept counts
+    find_digit<kSelThreads>(sh.hist, k, sh.scratch, &sh.digit, &sh.above);
+    const uint32_t d1 = static_cast<uint32_t>(sh.digit);
+    const int r1 = k - sh.above;  // rank of the k-th key among the keys of digit d1
+    const int n = sh.hist[d1];
+    // per chunk: keys of higher digits (all kept) and the group of digit d1
+    const int* cs = p.chunk_start + static_cast<size_t>(unit) * p.max_chunks * kHistBins;
     int carry = 0;
-    for (int c0 = 0; c0 < nch; c0 += kThThreads) {
+    for (int c0 = 0; c0 < nch; c0 += kSelThreads) {
+        const int c = c0 + tid;
+        int m = 0;
+        if (c < nch) {
+            const int a = __ldcg(cs + static_cast<size_t>(c) * kHistBins + d1);
+            const int e = d1 == 0 ? min(kChunk, P - c * kChunk)
+                                  : __ldcg(cs + static_cast<size_t>(c) * kHistBins + d1 - 1);
+            above[c] = a;
+            m = e - a;
+        }
+        int tot;
+        const int r = block_excl_scan<kSelThreads>(m, sh.scratch, &tot);
+        if (c < nch) coff[c] = carry + r;
+        carry += tot;
+    }
+    if (tid == 0) coff[nch] = carry;
+    __syncthreads();
+    if (carry != n) {
+        if (tid == 0) record_error(p.status, kDevBadIndex, 300 + unit);
+        return;
+    }
+    const uint2* bk = p.buckets + static_cast<size_t>(unit) * p.max_chunks * kChunk;
+    // candidate i: from shared memory, or found in its chunk's group when there are too many
+    const bool in_smem = n <= kCandCap;
+    if (in_smem) {
+        for (int c = warp; c < nch; c += kSelWarps) {
+            const int a = above[c], o = coff[c], m = coff[c + 1] - o;
+            for (int i = lane; i < m; i += 32) {
+                const uint2 e = __ldcg(bk + static_cast<size_t>(c) * kChunk + a + i);
+                cand_key[o + i] = e.x;
+                cand_pos[o + i] = static_cast<int>(e.y);
+            }
+        }
+        __syncthreads();
+    }
+    auto cand = [&](int i) -> uint2 {
+        if (in_smem) return make_uint2(cand_key[i], static_cast<uint32_t>(cand_pos[i]));
+        int lo = 0, hi = nch - 1;  // the chunk c with coff[c] <= i < coff[c+1]
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (coff[mid] <= i) lo = mid;
+            else hi = mid - 1;
+        }
+        return __ldcg(bk + static_cast<size_t>(lo) * kChunk + above[lo] + (i - coff[lo]));
+    };
+    int need_eq, n_eq;
+    const uint32_t thr = radix_select([&](int i) { return cand(i).x; }, n, d1 << kHistShift,
+                                      0x7FFu << kHistShift, kHistShift, r1, sh, &need_eq, &n_eq);
+    // Of the candidates equal to thr the need_eq lowest positions are kept: ranked pairwise
+    // when there are few, else found as the need_eq-th largest 0x7fffffff - position.
+    int pos_cut = INT_MAX;
+    if (need_eq < n_eq) {
+        if (n_eq <= kTieCap) {
+            for (int i0 = 0; i0 < n; i0 += kSelThreads) {
+                const int i = i0 + tid;
+                const bool eq = i < n && cand(i).x == thr;
+                const unsigned b = __ballot_sync(0xffffffffu, eq);
+                if (b) {
+                    int at = 0;
+                    if (lane == 0) at = atomicAdd(&sh.n_tie, __popc(b));
+                    at = __shfl_sync(0xffffffffu, at, 0) + __popc(b & ((1u << lane) - 1u));
+                    if (eq) tie_pos[at] = static_cast<int>(cand(i).y);
+                }
+            }
+            __syncthreads();
+            if (tid < n_eq) {
+                const int mine = tie_pos[tid];
+                int rank = 0;
+                for (int q = 0; q < n_eq; ++q) rank += tie_pos[q] < mine ? 1 : 0;
+                if (rank == need_eq - 1) sh.cut = mine;
+            }
+        } else {
+            auto mark = [&](int i) -> uint32_t {
+                const uint2 e = cand(i);
+                return e.x > thr ? kTaken : (e.x == thr ? 0x7FFFFFFFu - e.y : kDropped);
+            };
+            int r_eq, n_eq2;
+            const uint32_t v = radix_select(mark, n, 0u, 0x80000000u, 31, need_eq, sh, &r_eq, &n_eq2);
+            if (tid == 0) sh.cut = static_cast<int>(0x7FFFFFFFu - v);
+        }
+        __syncthreads();
+        pos_cut = sh.cut;
+    }
+    for (int c = tid; c < nch; c += kSelThreads) cnt[c] = above[c];
+    __syncthreads();
+    for (int i = tid; i < n; i += kSelThreads) {
+        const uint2 e = cand(i);
+        if (e.x > thr || (e.x == thr && static_cast<int>(e.y) <= pos_cut))
+            atomicAdd(&cnt[e.y >> kChunkShift], 1);
+    }
+    __syncthreads();
+    carry = 0;
+    for (int c0 = 0; c0 < nch; c0 += kSelThreads) {
         const int c = c0 + tid;
         int tot;
-        const int r = block_excl_scan<kThThreads>(c < nch ? cnt[c] : 0, st.scratch, &tot);
-        if (c < nch) coff[c] = carry + r;
+        const int r = block_excl_scan<kSelThreads>(c < nch ? cnt[c] : 0, sh.scratch, &tot);
+        if (c < nch) out_off[c] = carry + r;
         carry += tot;
     }
     if (tid == 0) {
         info[0] = static_cast<int>(thr);
         info[1] = pos_cut;
-        if (carry != k) record_error(p.status, kDevBadIndex, 300 + unit);
+        if (carry != k) record_error(p.status, kDevBadIndex, 310 + unit);
     }
 }
 
-__global__ void __launch_bounds__(kPHThreads) compact_kernel(const __grid_constant__ SelectParams p) {
+__global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_constant__ SelectParams p) {
+    extern __shared__ __align__(16) uint32_t dyn[];  // pooling stage, later the threshold's arrays
+    __shared__ SelectShared sh;
+    constexpr int PER = kPHPer;
+    const int unit = blockIdx.x, c = blockIdx.y, tid = threadIdx.x;
+    if (unit == 0 && c == 0 && tid == 0 && seqlens_hash(p.cu_seqlens, p.S) != p.cu_hash)
+        record_error(p.status, kDevBadSeqlens, 200);
+    UnitGeo u;
+    if (!unit_geo(p, unit, u)) return;
+    if (u.L <= kUnitLen) return;  // select_unit_kernel takes it
+    float* pooled = p.pooled + static_cast<size_t>(u.g) * p.T + u.t0;
+    const int j0 = c * kChunk;
+    const bool zeros = p.from_scores && p.write_pooled;
+    if (u.L <= p.budget) {  // kept whole: nothing to select; its pooled scores read as 0
+        if (zeros)
+            for (int j = j0 + tid; j < min(u.L, j0 + kChunk); j += kSelThreads) pooled[j] = 0.f;
+        return;
+    }
+    const int nch = (u.P + kChunk - 1) / kChunk;
+    if (nch > p.max_chunks) {  // longer than the host lengths said: leave the unit alone
+        if (c == 0 && tid == 0) record_error(p.status, kDevBadSeqlens, 210);
+        return;
+    }
+    if (zeros)  // window positions are not candidates
+        for (int j = max(j0, u.P) + tid; j < min(u.L, j0 + kChunk); j += kSelThreads) pooled[j] = 0.f;
+    if (j0 >= u.P) return;
+    const int n = min(kChunk, u.P - j0);
+    const int jl = tid * PER, nvalid = n - jl;
+    float acc[PER];
+    pooled_values<kSelThreads, PER, kStageLoads>(p, u, reinterpret_cast<float*>(dyn), j0, n, acc);
+    if (p.from_scores)  // the compaction reads them back
+#pragma unroll
+        for (int i = 0; i < PER; ++i)
+            if (i < nvalid) pooled[j0 + jl + i] = acc[i];
+    uint32_t key[PER], bins[PER];
+#pragma unroll
+    for (int i = 0; i < PER; ++i) {
+        key[i] = rank_key(acc[i]);
+        bins[i] = key[i] >> kHistShift;
+    }
+    // first-digit counts of the chunk
+    for (int b = tid; b < kHistBins; b += kSelThreads) sh.hist[b] = 0;
+    __syncthreads();
+    add_runs<PER>(sh.hist, bins, nvalid);
+    __syncthreads();
+    // group starts, highest digit first; the unit's counts
+    const size_t slot = static_cast<size_t>(unit) * p.max_chunks + c;
+    int* cs = p.chunk_start + slot * kHistBins;
+    int* gh = p.hist + static_cast<size_t>(unit) * kHistBins;
+    {
+        constexpr int BPT = kHistBins / kSelThreads;
+        const int base = (kSelThreads - 1 - tid) * BPT;
+        int h[BPT], local = 0;
+#pragma unroll
+        for (int q = BPT - 1; q >= 0; --q) {
+            h[q] = sh.hist[base + q];
+            local += h[q];
+        }
+        int tot;
+        int start = block_excl_scan<kSelThreads>(local, sh.scratch, &tot);
+#pragma unroll
+        for (int q = BPT - 1; q >= 0; --q) {
+            sh.fill[base + q] = start;
+            cs[base + q] = start;
+            if (h[q]) atomicAdd(gh + base + q, h[q]);
+            start += h[q];
+        }
+    }
+    __syncthreads();
+    // the chunk's (key, position) pairs grouped by first digit; a run of equal digits takes
+    // consecutive slots
+    uint2* bk = p.buckets + slot * kChunk;
+    {
+        int at = 0;
+#pragma unroll
+        for (int i = 0; i < PER; ++i) {
+            if (i < nvalid) {
+                if (i == 0 || bins[i] != bins[i - 1]) {
+                    int len = 1;
+                    bool run = true;
+#pragma unroll
+                    for (int q = i + 1; q < PER; ++q) {
+                        run = run && q < nvalid && bins[q] == bins[i];
+                        len += run ? 1 : 0;
+                    }
+                    at = atomicAdd(&sh.fill[bins[i]], len);
+                } else {
+                    ++at;
+                }
+                bk[at] = make_uint2(key[i], static_cast<uint32_t>(j0 + jl + i));
+            }
+        }
+    }
+    // The last chunk block of the unit to get here computes the unit's threshold.  The
+    // barrier orders the block's stores before thread 0's release; its acquire, and the
+    // barrier after it, order the other blocks' stores before this block's reads.
+    __syncthreads();
+    if (tid == 0) sh.last = atomic_add_acq_rel(p.arrivals + unit, 1) == nch - 1;
+    __syncthreads();
+    if (!sh.last) return;
+    unit_threshold(p, u, unit, nch, sh, dyn);
+}
+
+__global__ void __launch_bounds__(kSelThreads) compact_kernel(const __grid_constant__ SelectParams p) {
     extern __shared__ int list[];  // [kChunk] the chunk's kept positions, in order
-    __shared__ int wbase[kPHWarps + 1];
+    __shared__ int wbase[kSelWarps + 1];
     const int unit = blockIdx.x, c = blockIdx.y, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     if (unit == 0 && c == 0 && tid == 0 && seqlens_hash(p.cu_seqlens, p.S) != p.cu_hash)
         record_error(p.status, kDevBadSeqlens, 220);
     UnitGeo u;
     if (!unit_geo(p, unit, u)) return;
+    if (u.L <= kUnitLen) return;  // select_unit_kernel took it
     if (u.g == 0 && c == 0 && tid == 0) {
         p.cu_keep[u.s + 1] = u.keep_off + u.n_keep;
         if (u.s == 0) p.cu_keep[0] = 0;
@@ -611,7 +848,7 @@ __global__ void __launch_bounds__(kPHThreads) compact_kernel(const __grid_consta
     const int j0 = c * kChunk;
     if (u.L <= p.budget) {  // kept whole
         const int m = max(0, min(u.L, j0 + kChunk) - j0);
-        for (int e = tid; e < m; e += kPHThreads) {
+        for (int e = tid; e < m; e += kSelThreads) {
             out[j0 + e] = j0 + e;
             list[e] = j0 + e;
         }
@@ -621,7 +858,7 @@ __global__ void __launch_bounds__(kPHThreads) compact_kernel(const __grid_consta
     }
     const int P = u.P, k = u.k;
     if (c == 0) {  // the window closes the list
-        for (int i = tid; i < p.w; i += kPHThreads) {
+        for (int i = tid; i < p.w; i += kSelThreads) {
             out[k + i] = P + i;
             list[i] = P + i;
         }
@@ -655,15 +892,15 @@ __global__ void __launch_bounds__(kPHThreads) compact_kernel(const __grid_consta
     __syncthreads();
     if (tid == 0) {
         int a = 0;
-        for (int x = 0; x < kPHWarps; ++x) {
+        for (int x = 0; x < kSelWarps; ++x) {
             const int t = wbase[x];
             wbase[x] = a;
             a += t;
         }
-        wbase[kPHWarps] = a;
+        wbase[kSelWarps] = a;
     }
     __syncthreads();
-    const int tot = wbase[kPHWarps];
+    const int tot = wbase[kSelWarps];
     if (base < 0 || base + tot > k) {
         if (tid == 0) record_error(p.status, kDevBadIndex, 320 + unit);
         return;
@@ -682,7 +919,6 @@ __global__ void __launch_bounds__(kPHThreads) compact_kernel(const __grid_consta
     __syncthreads();
     if (p.k) copy_rows(p, u, list, tot, u.keep_off + base);
 }
-
 struct GatherParams {
     const uint4* k;
     const uint4* v;
@@ -753,6 +989,9 @@ cudaError_t launch_select(const SelectLaunch& L, cudaStream_t stream) {
     p.cu_seqlens = L.cu_seqlens_dev;
     p.status = L.status;
     p.hist = L.hist;
+    p.arrivals = L.arrivals;
+    p.chunk_start = L.chunk_start;
+    p.buckets = reinterpret_cast<uint2*>(L.buckets);
     p.info = L.info;
     p.chunk_off = L.chunk_off;
     p.k = reinterpret_cast<const uint4*>(L.k);
@@ -778,34 +1017,43 @@ cudaError_t launch_select(const SelectLaunch& L, cudaStream_t stream) {
     const int units = L.S * L.Hkv;
     if (units == 0 || L.max_chunks == 0) return cudaSuccess;
     if (L.max_chunks > 65535) return cudaErrorInvalidConfiguration;
-    const size_t th_smem = sizeof(uint32_t) * 2 * kCandCap + sizeof(int) * 2 * static_cast<size_t>(L.max_chunks);
-    static size_t th_smem_set = 0;
+    const size_t sel_smem = std::max(static_cast<size_t>(kSelStageSmem),
+                                     sizeof(uint32_t) * 2 * kCandCap +
+                                         sizeof(int) * (3 * static_cast<size_t>(L.max_chunks) + 1 + kTieCap));
+    static size_t sel_smem_set = 0;
     static bool configured = false;
     cudaError_t e;
     if (!configured) {
-        e = cudaFuncSetAttribute(pool_hist_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kStageFloats * 4);
-        if (e != cudaSuccess) return e;
         e = cudaFuncSetAttribute(compact_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kCompactSmem);
+        if (e != cudaSuccess) return e;
+        e = cudaFuncSetAttribute(select_unit_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kUnitSmem);
         if (e != cudaSuccess) return e;
         configured = true;
     }
-    if (th_smem > th_smem_set) {
-        e = cudaFuncSetAttribute(threshold_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 static_cast<int>(th_smem));
+    if (sel_smem > sel_smem_set) {
+        e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 static_cast<int>(sel_smem));
         if (e != cudaSuccess) return e;
-        th_smem_set = th_smem;
+        sel_smem_set = sel_smem;
     }
-    const dim3 grid(units, L.max_chunks);
-    pool_hist_kernel<<<grid, kPHThreads, kStageFloats * 4, stream>>>(p);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    threshold_kernel<<<units, kThThreads, th_smem, stream>>>(p);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    compact_kernel<<<grid, kPHThreads, kCompactSmem, stream>>>(p);
-    return cudaGetLastError();
+    if (L.min_len <= kUnitLen) {
+        select_unit_kernel<<<units, kUnitThreads, kUnitSmem, stream>>>(p);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+    if (L.max_len > kUnitLen) {
+        const dim3 grid(units, L.max_chunks);
+        select_kernel<<<grid, kSelThreads, sel_smem, stream>>>(p);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        compact_kernel<<<grid, kSelThreads, kCompactSmem, stream>>>(p);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+    return cudaSuccess;
 }
 
 int select_chunks(int max_len) { return max(1, (max_len + kChunk - 1) / kChunk); }
 size_t select_hist_ints() { return kHistBins; }
+int select_chunk_positions() { return kChunk; }
+int select_unit_len() { return kUnitLen; }
 
 cudaError_t launch_gather(const GatherLaunch& L, cudaStream_t stream) {
     GatherParams p;
