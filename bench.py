@@ -35,7 +35,15 @@ HBM_FALLBACK_GBS = 6800.0
 
 # dram__bytes_read.sum + dram__bytes_write.sum per launch pair of the scoring stage, from the
 # ncu capture summarised in profiles/, keyed by the sha256 of the kernel source it was taken on.
-SCORE_TRAFFIC = {}
+# DRAM bytes (read + write) per scoring launch (one layer of llama8b_l8192) from the ncu
+# capture summarised in profiles/score_kernel_llama8b_l8192.md, keyed by the sha256 of the
+# kernel source it was taken on; a changed kernel reports null until it is captured again.
+SCORE_TRAFFIC = {
+    "32d2a5579cdc99ed22368dd49779372e10ef36016648c6a00524df233b42391b": 16976128,
+}
+# Sequences up to this many tokens are selected by one block per (sequence, KV head)
+# (one launch); longer ones by the chunked kernels (two launches).
+SELECT_UNIT_LEN = 16384
 
 
 def _args():
@@ -237,8 +245,10 @@ def run_ours(args):
     ms_per_step = ms / args.steps
     value = world * nl * T / (ms_per_step / 1e3)
 
-    # per layer: the scoring kernel, then pool_hist, threshold and compact (gather fused)
-    launches_per_step = 4 * nl
+    # per layer: the scoring kernel, then the selection (pool, top-k, compaction and gather)
+    lens = list(wl.seqlens)
+    per_layer = 1 + (1 if min(lens) <= SELECT_UNIT_LEN else 0) + (2 if max(lens) > SELECT_UNIT_LEN else 0)
+    launches_per_step = per_layer * nl
 
     # --- scoring stage (the dominant kernels): a graph of every layer's ckv_score_window,
     # timed with events on its stream; the average per layer is one pass-1 + pass-2 pair.
@@ -378,7 +388,9 @@ def _cpu_baseline(wl, host_layers, seconds):
     cores = oracle.threads(0)
     t0 = time.perf_counter()
     done = 0
-    for l, li in enumerate(host_layers):
+    while True:  # sweeps of the layers, in order, until `seconds` have passed
+        l = done % len(host_layers)
+        li = host_layers[l]
         oracle.compress_layer(li.q_win, li.k, li.v, wl.cu_seqlens(), wl.head_mask()[l],
                               int(wl.budgets()[l]), wl.window, wl.pool_kernel,
                               0 if wl.pool_type == "max" else 1,
@@ -388,8 +400,9 @@ def _cpu_baseline(wl, host_layers, seconds):
             break
     dt = time.perf_counter() - t0
     return {"value": round(done * wl.total_tokens / dt, 2), "unit": UNIT, "cores": cores,
-            "kind": "oracle", "sample": f"{done} of {wl.num_layers} layers, whole layers, "
-                                        f"{dt:.1f} s, OpenMP over (sequence, KV head)"}
+            "kind": "oracle", "sample": f"{done} layer calls (sweeps over the {len(host_layers)} "
+                                        f"layers), whole layers, {dt:.1f} s, OpenMP over "
+                                        "(sequence, KV head)"}
 
 
 def run_reference(args):
