@@ -146,8 +146,11 @@ int64_t keep_total(const ckv_batch* b, int budget) {
 
 // Splits every (sequence, head batch) unit's key tiles into items of at most `c` tiles and
 // packs units whole into rounds of at most `ctas` items; `c` minimises an estimate of the
-// launch's time: per round, the longest item, plus the tiles of it that do not stay resident
-// in the kernel's shared-memory slots (they are loaded a second time), plus a fixed cost.
+// launch's time in tile loads per CTA.  Pass 1 of a round streams while the previous round
+// exchanges its statistics and runs pass 2, so a round costs its item length, or the
+// exchange plus pass 2 of the round before when that is longer; the last round adds its own
+// exchange and pass 2.  Items longer than kL2Tiles are charged their excess again: their
+// pass-2 re-reads fall out of the CTA's share of L2.
 ckv_status plan_score(const Plan& pl, const ckv_batch* b, int skip_le, int ctas, ScoreLaunch& L,
                       int max_items_per_launch) {
     struct RawUnit {
@@ -168,9 +171,11 @@ ckv_status plan_score(const Plan& pl, const ckv_batch* b, int skip_le, int ctas,
     L.slices.clear();
     if (raw.empty()) return CKV_OK;
     if (b->num_seqs > 65535) return fail(CKV_ERR_UNSUPPORTED, "more than 65535 sequences");
-    constexpr int kResident = 6, kFixed = 3;
+    constexpr int kL2Tiles = 8;        // 2 items x 8 tiles x 32 KiB x 152 CTAs ~ 78 MB of L2
+    constexpr double kExchange = 4.0;  // the exchange, in tile-load times
+    constexpr double kPass2 = 0.4;     // pass 2 per tile from L2, relative to a pass-1 load
     int best_c = -1;
-    long long best_cost = 0;
+    double best_cost = 0;
     for (int c = 1; c <= max_tiles; ++c) {
         long long rounds = 0;
         int cur = 0;
@@ -189,7 +194,9 @@ ckv_status plan_score(const Plan& pl, const ckv_batch* b, int skip_le, int ctas,
         }
         if (!feasible) continue;
         rounds += cur > 0;
-        const long long cost = rounds * (c + std::max(0, c - kResident) + kFixed);
+        const double per_round = std::max(static_cast<double>(c), kPass2 * c + kExchange) +
+                                 std::max(0, c - kL2Tiles);
+        const double cost = rounds * per_round + kPass2 * c + kExchange;
         if (best_c < 0 || cost < best_cost) {
             best_c = c;
             best_cost = cost;
@@ -337,6 +344,25 @@ EncodeTiledFn encode_fn() {
 }
 
 // K viewed as {128 (dim), H_kv, T} with a {64, 1, 128} box and the 128-byte swizzle.
+// The window queries [S, w, H_q, 128] as {128 (dim), H_q, S*w (row)}: one box is 64 dims of
+// rows_per_box consecutive window rows of one head, 128-byte swizzled like the MMA operand.
+ckv_status make_q_map(CUtensorMap* map, const void* q, int Hq, int S, int w, int rows_per_box) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return fail(CKV_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
+    const cuuint64_t dims[3] = {static_cast<cuuint64_t>(kHeadDim), static_cast<cuuint64_t>(Hq),
+                                static_cast<cuuint64_t>(S) * static_cast<cuuint64_t>(w)};
+    const cuuint64_t strides[2] = {static_cast<cuuint64_t>(kHeadDim) * 2,
+                                   static_cast<cuuint64_t>(Hq) * kHeadDim * 2};
+    const cuuint32_t box[3] = {64, 1, static_cast<cuuint32_t>(rows_per_box)};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    const CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(q), dims,
+                          strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                          CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(CKV_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", static_cast<int>(r));
+    return CKV_OK;
+}
+
 ckv_status make_k_map(CUtensorMap* map, const void* k, int Hkv, int T, int64_t tok, int64_t head) {
     EncodeTiledFn fn = encode_fn();
     if (!fn) return fail(CKV_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
@@ -381,6 +407,7 @@ ckv_status enqueue_score(const Plan& pl, const ckv_batch* b, int T, const void* 
     if (st) return st;
     if (L.slices.empty()) return CKV_OK;
     if ((st = make_k_map(&L.tmap_k, k, pl.Hkv, T, tok, head))) return st;
+    if ((st = make_q_map(&L.tmap_q, q_win, pl.Hq, b->num_seqs, pl.w, pl.w_pad))) return st;
     uint8_t* w8 = static_cast<uint8_t*>(ws);
     L.q_win = q_win;
     L.cu_seqlens_dev = b->cu_seqlens_dev;

@@ -36,6 +36,7 @@ struct ScoreSlice {
 
 struct ScoreLaunch {
     CUtensorMap tmap_k;
+    CUtensorMap tmap_q;    // the window queries, boxes of w_pad rows x 64 dims
     const void* q_win;
     const int32_t* cu_seqlens_dev;
     void* partials;        // float2 [items per launch, n_cols]

@@ -4,31 +4,32 @@
 //
 // for every selected head h of a KV group, every window row r and every key j of a sequence
 // (P = L - w).  A row's normaliser lse needs every key before any probability can be summed
-// over rows, so each key tile is used twice -- once for the row statistics, once for the
-// probabilities -- and kept in shared memory in between.
-//
-// One cooperative launch; one CTA per SM, 384 threads, warp-specialised:
-//   warp 0      TMA producer: 128-key x 128-dim bf16 tiles of K (two 128-byte-swizzled boxes of
-//               64 dims) into a ring of kSlots shared-memory slots; tile i of an item lives
-//               in slot (base + i) % kSlots, base advancing by the item's tile count;
-//   warp 1      allocates TMEM and issues tcgen05.mma (M = 128 keys, N = the window rows of a
-//               batch of heads, K = 128) into kAccBufs TMEM accumulators;
-//   warps 2-3   stage the unit's window query rows (the MMA's B operand);
-//   warps 4-11  two epilogue warpgroups, each owning half of the window-row columns; every
-//               thread owns one key (one TMEM lane), so per-row running statistics (pass 1)
-//               and per-key sums over rows (pass 2) are thread-local.
+// over rows, so each key tile is used twice: once for the row statistics (pass 1), once for
+// the probabilities (pass 2).
 //
 // Work: a unit is (sequence, batch of selected heads of one KV group); its key tiles are cut
-// into items (chunks).  Per item:
-//   pass 1  tiles in increasing order: per-thread running (max, sum of 2^(x - max)) per row,
-//           rescaled only when a logit exceeds the running max by more than 2^8; then the
-//           CTA's per-row partial goes to global memory and the unit's arrival counter is
-//           incremented;
-//   wait    until every item of the unit has published its partial (a bounded spin; all CTAs
-//           of a launch are co-resident, and a unit's items all belong to one round);
-//   pass 2  tiles in decreasing order, so the last kSlots tiles are still resident and only
-//           older ones are loaded again: exp2(x - lse) summed over each head's rows.
-// Items are dealt out in rounds of gridDim.x; CTA b takes item (round * gridDim.x + b).
+// into items of a few tiles, and the items are dealt out in rounds of gridDim.x (CTA b takes
+// item round * gridDim.x + b; all items of a unit are in one round).  One cooperative
+// launch, one CTA per SM, 640 threads, warp-specialised:
+//   warp 0       pass-1 producer: per item, TMA loads of the window query rows (the MMA's B
+//                operand) into one of three buffers, then of its 128-key x 128-dim bf16 K
+//                tiles (two 128-byte-swizzled boxes of 64 dims) into a ring of kP1Slots slots;
+//   warp 1       allocates TMEM and issues tcgen05.mma (M = 128 keys, N = the window rows of a
+//                head batch, K = 128) for both passes, into four pass-1 and four pass-2 TMEM
+//                accumulators, taking whichever ring has a tile ready;
+//   warp 2       pass-2 producer: the same tiles again into a ring of kP2Slots slots, issued
+//                once an item's pass-1 loads are out, so they are served by L2;
+//   warp 3       publisher: once an item's pass-1 partials are stored, one release on the
+//                unit's arrival counter;
+//   warps 4-11   pass 1, one warpgroup per 32 columns: each thread owns one key (one TMEM
+//                lane), keeps a running (max, sum of 2^(x - max)) per column, and at the end of
+//                the item the warpgroup's per-column partial goes to global memory, followed by
+//                a release on the unit's arrival counter;
+//   warps 12-19  pass 2, one warpgroup per 32 columns: once every item of the unit has
+//                arrived (a bounded acquire spin) they combine the partials into lse and sum
+//                exp2(x - lse) over each head's rows per key.
+// Pass 1 of an item overlaps the exchange and pass 2 of the item before it, so HBM keeps
+// streaming while the CTAs wait for each other.
 #include "ckv_device.cuh"
 #include "ckv_internal.h"
 
@@ -38,20 +39,23 @@
 
 namespace ckv {
 
-constexpr int kSlots = 6;
+constexpr int kP1Slots = 3;                           // pass-1 ring (HBM)
+constexpr int kP2Slots = 2;                           // pass-2 ring (L2)
+constexpr int kAcc = 4;                               // TMEM accumulators per pass
+constexpr int kQBufs = 3;                             // query-row buffers: pass 1 runs two items ahead
 constexpr int kTileBytes = kTileKeys * kHeadDim * 2;  // 32 KiB
 constexpr int kHalfBytes = kTileBytes / 2;            // 64 dims x 128 keys
-// The running maximum of a row is only moved when a logit exceeds it by more than 2^60: the
-// running sum then stays far below the fp32 range (at most keys * 2^60), and terms that are
-// 2^-126 below the reference are negligible against the reference term itself.
+// The running maximum of a column is only moved when a logit exceeds it by more than 2^60:
+// the running sum then stays far below the fp32 range (at most keys * 2^60), and terms that
+// are 2^-126 below the reference are negligible against the reference term itself.
 constexpr float kLazyTau = 60.0f;
-constexpr int kEpiWG = 4;                             // epilogue warpgroups
-constexpr int kAccBufs = 4;                           // TMEM accumulators (MMA runs ahead)
-constexpr int kEpiThreads = 128 * kEpiWG;
-constexpr int kThreads = 128 + kEpiThreads;
+constexpr int kCols = 32;                             // columns per epilogue warpgroup
+constexpr int kThreads = 512;
+constexpr int kWarpA = 4, kWarpB = 12;                // first pass-1 / pass-2 warp
 
 struct alignas(128) ScoreParams {
     CUtensorMap tmap_k;            // K as {128 (dim), H_kv, T}, box {64, 1, 128}, 128B swizzle
+    CUtensorMap tmap_q;            // q_win as {128, H_q, S*w}, box {64, 1, W_PAD}, 128B swizzle
     const __nv_bfloat16* q_win;    // [S, w, H_q, 128] packed
     const int32_t* cu_seqlens;     // device [S+1] (checked against cu_hash)
     float2* partials;              // [n_items, N]: (max, sum) per window-row column
@@ -71,16 +75,22 @@ struct alignas(128) ScoreParams {
 
 template <int N>
 struct SmemLayout {
-    static constexpr int kQ = kSlots * kTileBytes;
-    static constexpr int kQHalf = N * 128;
-    static constexpr int kBars = kQ + 2 * kQHalf;
-    // full[kSlots], freed[kSlots], acc_full[kAccBufs], acc_empty[kAccBufs], q_full, q_empty, done
-    static constexpr int kNumBars = 2 * kSlots + 2 * kAccBufs + 3;
-    static constexpr int kRed = kBars + 8 * kNumBars;   // float2 [512] reduction scratch
-    static constexpr int kLse = kRed + 8 * 512;         // float [N]
-    static constexpr int kXsum = kLse + 4 * N + 16;     // float [2][kEpiWG][128] (lse: N + flag)
-    static constexpr int kFills = kXsum + 4 * 2 * kEpiWG * 128;  // int [2][kSlots]
-    static constexpr int kTmemSlot = kFills + 4 * 2 * kSlots;
+    static constexpr int kP1 = 0;
+    static constexpr int kP2 = kP1 + kP1Slots * kTileBytes;
+    static constexpr int kQ = kP2 + kP2Slots * kTileBytes;
+    static constexpr int kQBytes = N * 256;             // one item's rows: N x 128 bf16
+    static constexpr int kQHalf = N * 128;              // 64 dims of them
+    static constexpr int kBars = kQ + kQBufs * kQBytes;
+    // mbarrier indices, in this order
+    static constexpr int kFull1 = 0, kFree1 = kFull1 + kP1Slots, kFull2 = kFree1 + kP1Slots,
+                         kFree2 = kFull2 + kP2Slots, kAFull = kFree2 + kP2Slots,
+                         kAEmpty = kAFull + kAcc, kBFull = kAEmpty + kAcc, kBEmpty = kBFull + kAcc,
+                         kQFull = kBEmpty + kAcc, kQEmpty = kQFull + kQBufs,
+                         kDone = kQEmpty + kQBufs, kGroup = kDone + 1,  // A0 A1 B
+                         kPubFull = kGroup + 3, kPubEmpty = kPubFull + 2,
+                         kNumBars = kPubEmpty + 2;
+    static constexpr int kIssued = kBars + 8 * kNumBars; // items whose pass-1 loads are issued
+    static constexpr int kTmemSlot = kIssued + 4;
     static constexpr int kAbort = kTmemSlot + 4;
     static constexpr int kBytes = kAbort + 4;
     static constexpr int kDynamic = kBytes + 1024;      // slack to align the base to 1024 B
@@ -122,6 +132,24 @@ __device__ __forceinline__ int ld_acquire(const int* p) {
 // a lane keeps one half of its remaining columns and swaps the other half with its partner, so
 // the C sums take C - 1 + log2(32 / C) shuffles instead of 5 C.  `m` (uniform across the warp)
 // is carried along.  Afterwards lane l holds column l / (32 / C) in v[0] / m[0].
+template <int R>
+__device__ __forceinline__ void setmaxnreg_inc() {
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(R));
+}
+template <int R>
+__device__ __forceinline__ void setmaxnreg_dec() {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(R));
+}
+
+// A barrier of one epilogue warpgroup built on an mbarrier of 128 arrivals, so that the wait
+// is bounded like every other wait of the kernel.
+__device__ __forceinline__ bool group_sync(uint64_t* bar, uint32_t& phase, volatile int* abort) {
+    mbar_arrive(bar);
+    const bool ok = mbar_wait(bar, phase, abort);
+    phase ^= 1;
+    return ok;
+}
+
 template <int C>
 __device__ __forceinline__ void transpose_reduce(float (&v)[C], float (&m)[C], int lane) {
 #pragma unroll
@@ -171,6 +199,33 @@ __device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, float (&v)[CPW]) {
     }
 }
 
+// tcgen05.ld of 16 columns without the wait: the registers are not valid until tmem_ld_wait,
+// and reg_fence then ties every later use to the wait.
+__device__ __forceinline__ void tmem_ld16_nowait(uint32_t taddr, float (&v)[16]) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr)
+        : "memory");
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__device__ __forceinline__ void tmem_ld_wait() {
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void reg_fence(float (&v)[16]) {
+    asm volatile(""
+                 : "+f"(v[0]), "+f"(v[1]), "+f"(v[2]), "+f"(v[3]), "+f"(v[4]), "+f"(v[5]),
+                   "+f"(v[6]), "+f"(v[7]), "+f"(v[8]), "+f"(v[9]), "+f"(v[10]), "+f"(v[11]),
+                   "+f"(v[12]), "+f"(v[13]), "+f"(v[14]), "+f"(v[15]));
+}
+
 // Valid-column mask of one thread for a tile: columns holding a real window row that sees
 // key j.  Row r of a head sees key j iff r >= j - P (causal window); keys >= L are padding.
 template <int CPW, int W_PAD>
@@ -190,55 +245,76 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
     static_assert(N == 32 || N == 64, "N");
     static_assert(W_PAD == 8 || W_PAD == 16 || W_PAD == 32 || W_PAD == 64, "W_PAD");
     static_assert(W_PAD <= N, "a head's rows fit in one MMA");
-    constexpr int CPW = N / kEpiWG;                    // columns per epilogue warpgroup
-    constexpr int kWgPerHead = W_PAD > CPW ? W_PAD / CPW : 1;
-    constexpr bool kSplitHead = kWgPerHead > 1;        // one head spans several warpgroups
-    constexpr int HPW = kSplitHead ? 1 : CPW / W_PAD;  // heads (or a part of one) per warpgroup
+    constexpr int kNW = N / kCols;                      // warpgroups per pass
+    constexpr int kTmemCols = 2 * kAcc * N;           // pass-1 accumulators, then pass-2
     using SL = SmemLayout<N>;
     constexpr uint32_t kIdesc = idesc_bf16_f32(kTileKeys, N);
-    constexpr uint32_t kFullMask = CPW == 32 ? 0xffffffffu : ((1u << CPW) - 1u);
 
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-    uint8_t* slots = sm;
+    uint8_t* ring1 = sm + SL::kP1;
+    uint8_t* ring2 = sm + SL::kP2;
     uint8_t* qbuf = sm + SL::kQ;
     uint64_t* bars = reinterpret_cast<uint64_t*>(sm + SL::kBars);
-    uint64_t* full = bars;
-    uint64_t* freed = bars + kSlots;
-    uint64_t* acc_full = bars + 2 * kSlots;
-    uint64_t* acc_empty = acc_full + kAccBufs;
-    uint64_t* q_full = acc_empty + kAccBufs;
-    uint64_t* q_empty = q_full + 1;
-    uint64_t* done = q_empty + 1;
-    float2* red = reinterpret_cast<float2*>(sm + SL::kRed);
-    float* lse_s = reinterpret_cast<float*>(sm + SL::kLse);
-    float* xsum = reinterpret_cast<float*>(sm + SL::kXsum);
-    int* fills = reinterpret_cast<int*>(sm + SL::kFills);
+    uint64_t* full1 = bars + SL::kFull1;
+    uint64_t* free1 = bars + SL::kFree1;
+    uint64_t* full2 = bars + SL::kFull2;
+    uint64_t* free2 = bars + SL::kFree2;
+    uint64_t* a_full = bars + SL::kAFull;
+    uint64_t* a_empty = bars + SL::kAEmpty;
+    uint64_t* b_full = bars + SL::kBFull;
+    uint64_t* b_empty = bars + SL::kBEmpty;
+    uint64_t* q_full = bars + SL::kQFull;
+    uint64_t* q_empty = bars + SL::kQEmpty;
+    uint64_t* done = bars + SL::kDone;
+    uint64_t* group = bars + SL::kGroup;        // one per epilogue warpgroup: A0 A1 B
+    uint64_t* pub_full = bars + SL::kPubFull;   // pass-1 partials of an item stored (item parity)
+    uint64_t* pub_empty = bars + SL::kPubEmpty;
+    // scratch of the epilogues (static, so that its accesses are shared-memory instructions)
+    __shared__ float2 red_a[2][2][128];  // [item parity][warpgroup][warp * 32 + lane]
+    __shared__ float2 red_b[256];        // [part * N + column]
+    __shared__ float lse_s[64];
+    __shared__ volatile int verdict[1];
+    volatile int* issued = reinterpret_cast<volatile int*>(sm + SL::kIssued);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + SL::kTmemSlot);
     volatile int* abort = reinterpret_cast<volatile int*>(sm + SL::kAbort);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     if (threadIdx.x == 0) {
-        for (int i = 0; i < kSlots; ++i) {
-            mbar_init(&full[i], 1);
-            mbar_init(&freed[i], 1);
+        for (int i = 0; i < kP1Slots; ++i) {
+            mbar_init(&full1[i], 1);
+            mbar_init(&free1[i], 1);
         }
-        for (int i = 0; i < kAccBufs; ++i) {
-            mbar_init(&acc_full[i], 1);
-            mbar_init(&acc_empty[i], kEpiThreads / 32);  // one arrival per epilogue warp
+        for (int i = 0; i < kP2Slots; ++i) {
+            mbar_init(&full2[i], 1);
+            mbar_init(&free2[i], 1);
         }
-        mbar_init(q_full, 64);
-        mbar_init(q_empty, 1);
+        for (int i = 0; i < kAcc; ++i) {
+            mbar_init(&a_full[i], 1);
+            mbar_init(&a_empty[i], 4 * kNW);  // one arrival per pass-1 warp
+            mbar_init(&b_full[i], 1);
+            mbar_init(&b_empty[i], 4);        // one arrival per pass-2 warp
+        }
+        for (int i = 0; i < kQBufs; ++i) {
+            mbar_init(&q_full[i], 1);
+            mbar_init(&q_empty[i], 1);
+        }
         mbar_init(done, 1);
-        for (int i = 0; i < 2 * kSlots; ++i) fills[i] = 0;
+        for (int i = 0; i < 3; ++i) mbar_init(&group[i], 128);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&pub_full[i], 32 * kNW);
+            mbar_init(&pub_empty[i], 1);
+        }
+        *issued = 0;
         *abort = 0;
         fence_mbar_init();
         tma_prefetch_desc(&p.tmap_k);
+        tma_prefetch_desc(&p.tmap_q);
     }
     if (warp == 1) {
-        tmem_alloc(tmem_slot, kAccBufs * N);
+        tmem_alloc(tmem_slot, kTmemCols);
         tmem_relinquish();
     }
     if (blockIdx.x == 0 && threadIdx.x == 64 && seqlens_hash(p.cu_seqlens, p.S) != p.cu_hash)
@@ -247,61 +323,102 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
     __syncthreads();
     tc_fence_after_sync();
     const uint32_t tmem_base = *tmem_slot;
+    // Registers: launched at 128 per thread (512 x 128 = 65536); on entry the producer/MMA/
+    // query warpgroup gives up to 56, which leaves room for the two pass-1 warpgroups' 160;
+    // the pass-2 warpgroup keeps 128 (128*56 + 256*160 + 128*128 = 64512).
+    const int R = p.n_rounds;
+    const int G = gridDim.x;
+    auto item_of = [&](int r) -> const ScoreItem& { return p.items[r * G + blockIdx.x]; };
 
-    if (warp == 0) {
-        // ------------------------------------------------------------ TMA producer
+    if (warp < kWarpA) {
+    setmaxnreg_dec<56>();
+    if (warp == 0 || warp == 2) {
+        // ------------------------------------------------------------ TMA producers
         if (lane == 0) {
-            int* pf = fills;  // fills issued per slot
-            int base = 0;     // slot of the item's first tile: the ring continues across items
+            const bool first = warp == 0;
+            const int nslots = first ? kP1Slots : kP2Slots;
+            uint8_t* ring = first ? ring1 : ring2;
+            uint64_t* full = first ? full1 : full2;
+            uint64_t* freed = first ? free1 : free2;
+            int use = 0, it = 0;
             bool ok = true;
-            auto load = [&](const ScoreUnit& U, int tile0, int jt) {
-                const int s = (base + jt) % kSlots;
-                if (!mbar_wait(&freed[s], (pf[s] & 1) ^ 1, abort)) return false;
-                ++pf[s];
-                mbar_arrive_expect_tx(&full[s], kTileBytes);
-                uint8_t* dst = slots + s * kTileBytes;
-                const int tok = U.seq_start + (tile0 + jt) * kTileKeys;
-                const int g = p.batch_group[U.batch];
-                tma_load_3d(dst, &p.tmap_k, &full[s], 0, g, tok);
-                tma_load_3d(dst + kHalfBytes, &p.tmap_k, &full[s], 64, g, tok);
-                return true;
-            };
-            for (int r = 0; ok && r < p.n_rounds; ++r) {
-                const ScoreItem& I = p.items[r * gridDim.x + blockIdx.x];
+            for (int r = 0; ok && r < R; ++r) {
+                const ScoreItem& I = item_of(r);
                 const int n = I.ntiles;
                 if (n == 0) continue;
+                if (!first) {  // pass 2 follows the item's pass-1 loads, so it reads L2
+                    const long long t0 = clock64();
+                    for (uint32_t k = 1; *issued <= it; ++k) {
+                        __nanosleep(64);
+                        if ((k & 63u) == 0u && (*abort || clock64() - t0 > kWaitTimeoutCycles)) {
+                            ok = false;
+                            break;
+                        }
+                    }
+                    if (!ok) break;
+                }
                 const ScoreUnit& U = p.units[I.unit];
-                for (int jt = 0; ok && jt < n; ++jt) ok = load(U, I.tile0, jt);               // pass 1
-                for (int jt = n - kSlots - 1; ok && jt >= 0; --jt) ok = load(U, I.tile0, jt);  // pass 2
-                base = (base + n) % kSlots;
+                const int g = p.batch_group[U.batch];
+                if (first) {
+                    // The item's window query rows: per head of the batch two boxes of 64
+                    // dims x W_PAD rows in the MMA's 128-byte-swizzled layout.  Rows past w
+                    // (the next sequence's, or zeros past the end) and head slots past the
+                    // batch's heads land in columns that the epilogues mask out.
+                    const int qb = it % kQBufs;
+                    if (!mbar_wait(&q_empty[qb], ((it / kQBufs) & 1) ^ 1, abort)) {
+                        ok = false;
+                        break;
+                    }
+                    uint8_t* qdst = qbuf + qb * SL::kQBytes;
+                    const int first_row = p.batch_first[U.batch], nheads = p.batch_nheads[U.batch];
+                    mbar_arrive_expect_tx(&q_full[qb], static_cast<uint32_t>(nheads * W_PAD * 256));
+                    for (int slot = 0; slot < nheads; ++slot) {
+                        const int h = p.sel_heads[first_row + slot];
+                        uint8_t* d = qdst + slot * W_PAD * 128;
+                        tma_load_3d(d, &p.tmap_q, &q_full[qb], 0, h, U.seq * p.w);
+                        tma_load_3d(d + SL::kQHalf, &p.tmap_q, &q_full[qb], 64, h, U.seq * p.w);
+                    }
+                }
+                for (int jt = 0; ok && jt < n; ++jt, ++use) {
+                    const int s = use % nslots;
+                    if (!mbar_wait(&freed[s], ((use / nslots) & 1) ^ 1, abort)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(&full[s], kTileBytes);
+                    uint8_t* dst = ring + s * kTileBytes;
+                    const int tok = U.seq_start + (I.tile0 + jt) * kTileKeys;
+                    tma_load_3d(dst, &p.tmap_k, &full[s], 0, g, tok);
+                    tma_load_3d(dst + kHalfBytes, &p.tmap_k, &full[s], 64, g, tok);
+                }
+                ++it;
+                if (first) *issued = it;
             }
             if (!ok) {
                 *abort = 1;
-                record_error(p.status, kDevTimeout, 10);
+                record_error(p.status, kDevTimeout, first ? 10 : 15);
             }
             // Let every issued copy land before the block may exit.
-            for (int s = 0; s < kSlots; ++s) {
+            const int last = use;
+            for (int k = (last > nslots ? last - nslots : 0); k < last; ++k) {
                 volatile int never = 0;
-                if (pf[s] > 0) mbar_wait(&full[s], (pf[s] - 1) & 1, &never);
+                mbar_wait(&full[k % nslots], (k / nslots) & 1, &never);
             }
+            if (first)
+                for (int k = (it > kQBufs ? it - kQBufs : 0); k < it; ++k) {
+                    volatile int never = 0;
+                    mbar_wait(&q_full[k % kQBufs], (k / kQBufs) & 1, &never);
+                }
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
-            int* mf = fills + kSlots;  // fills consumed per slot
-            int acc_it = 0, item_it = 0, base = 0;
-            bool ok = true;
-            auto mma_tile = [&](int s, bool wait_fill, bool release) {
-                if (wait_fill) {
-                    if (!mbar_wait(&full[s], mf[s] & 1, abort)) return false;
-                    ++mf[s];
-                }
-                const int acc = acc_it % kAccBufs;
-                if (!mbar_wait(&acc_empty[acc], ((acc_it / kAccBufs) & 1) ^ 1, abort)) return false;
-                tc_fence_after_sync();
-                const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * N);
-                const uint32_t a0 = smem_u32(slots + s * kTileBytes);
-                const uint32_t b0 = smem_u32(qbuf);
+            auto next_item = [&](int r) {
+                while (r < R && item_of(r).ntiles == 0) ++r;
+                return r;
+            };
+            auto mma = [&](const uint8_t* a_tile, const uint8_t* q, uint32_t d_tmem) {
+                const uint32_t a0 = smem_u32(a_tile), b0 = smem_u32(q);
 #pragma unroll
                 for (int kk = 0; kk < kHeadDim / 16; ++kk) {
                     const uint32_t koff = (kk & 3) * 32;
@@ -309,30 +426,69 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                     const uint64_t bd = sdesc_k_major_sw128(b0 + (kk >> 2) * SL::kQHalf + koff);
                     umma_bf16(d_tmem, ad, bd, kIdesc, kk > 0 ? 1u : 0u);
                 }
-                umma_commit(&acc_full[acc]);
-                if (release) umma_commit(&freed[s]);
-                ++acc_it;
-                return true;
             };
-            for (int r = 0; ok && r < p.n_rounds; ++r) {
-                const ScoreItem& I = p.items[r * gridDim.x + blockIdx.x];
-                const int n = I.ntiles;
-                if (n == 0) continue;
-                if (!mbar_wait(q_full, item_it & 1, abort)) {
-                    ok = false;
-                    break;
+            int r1 = next_item(0), it1 = 0, jt1 = 0, use1 = 0, a_it = 0;
+            int r2 = r1, it2 = 0, jt2 = 0, use2 = 0, b_it = 0;
+            bool q_ready = false, ok = true;
+            long long t0 = clock64();
+            uint32_t idle = 0;
+            while (r1 < R || r2 < R) {
+                bool did = false;
+                // pass 2 of an item whose pass-1 products are all issued
+                if (r2 < R && it2 < it1) {
+                    const int s = use2 % kP2Slots, acc = b_it % kAcc;
+                    if (mbar_test(&full2[s], (use2 / kP2Slots) & 1) &&
+                        mbar_test(&b_empty[acc], ((b_it / kAcc) & 1) ^ 1)) {
+                        tc_fence_after_sync();
+                        mma(ring2 + s * kTileBytes, qbuf + (it2 % kQBufs) * SL::kQBytes,
+                            tmem_base + static_cast<uint32_t>((kAcc + acc) * N));
+                        umma_commit(&b_full[acc]);
+                        umma_commit(&free2[s]);
+                        ++use2;
+                        ++b_it;
+                        if (++jt2 == item_of(r2).ntiles) {
+                            umma_commit(&q_empty[it2 % kQBufs]);  // the item's query rows are free
+                            r2 = next_item(r2 + 1);
+                            ++it2;
+                            jt2 = 0;
+                        }
+                        did = true;
+                    }
                 }
-                tc_fence_after_sync();
-                // pass 1: a tile that is evicted before pass 2 frees its slot right away
-                for (int jt = 0; ok && jt < n; ++jt)
-                    ok = mma_tile((base + jt) % kSlots, true, jt < n - kSlots);
-                // pass 2: resident tiles need no new fill; every tile frees its slot after use
-                for (int jt = n - 1; ok && jt >= 0; --jt)
-                    ok = mma_tile((base + jt) % kSlots, jt < n - kSlots, true);
-                if (!ok) break;
-                base = (base + n) % kSlots;
-                umma_commit(q_empty);
-                ++item_it;
+                if (r1 < R) {
+                    if (!q_ready) {
+                        q_ready = mbar_test(&q_full[it1 % kQBufs], (it1 / kQBufs) & 1);
+                        if (q_ready) tc_fence_after_sync();
+                    }
+                    const int s = use1 % kP1Slots, acc = a_it % kAcc;
+                    if (q_ready && mbar_test(&full1[s], (use1 / kP1Slots) & 1) &&
+                        mbar_test(&a_empty[acc], ((a_it / kAcc) & 1) ^ 1)) {
+                        tc_fence_after_sync();
+                        mma(ring1 + s * kTileBytes, qbuf + (it1 % kQBufs) * SL::kQBytes,
+                            tmem_base + static_cast<uint32_t>(acc * N));
+                        umma_commit(&a_full[acc]);
+                        umma_commit(&free1[s]);
+                        ++use1;
+                        ++a_it;
+                        if (++jt1 == item_of(r1).ntiles) {
+                            r1 = next_item(r1 + 1);
+                            ++it1;
+                            jt1 = 0;
+                            q_ready = false;
+                        }
+                        did = true;
+                    }
+                }
+                if (did) {
+                    idle = 0;
+                    t0 = clock64();
+                } else {
+                    __nanosleep(20);
+                    if ((++idle & 63u) == 0u && (*abort || clock64() - t0 > kWaitTimeoutCycles)) {
+                        ok = false;
+                        break;
+                    }
+                }
             }
             if (!ok) {
                 *abort = 1;
@@ -343,62 +499,178 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             mbar_wait(done, 0, &never);
         }
         __syncwarp();
-    } else if (warp < 4) {
-        // ------------------------------------------------------------ query-row staging
-        const int tid = threadIdx.x - 64;
-        int item_it = 0;
-        for (int r = 0; r < p.n_rounds; ++r) {
-            const ScoreItem& I = p.items[r * gridDim.x + blockIdx.x];
-            if (I.ntiles == 0) continue;
-            const ScoreUnit& U = p.units[I.unit];
-            if (!mbar_wait(q_empty, (item_it & 1) ^ 1, abort, 500)) {  // a long, idle wait
-                *abort = 1;
-                record_error(p.status, kDevTimeout, 12);
-                break;
-            }
-            const int first = p.batch_first[U.batch], nheads = p.batch_nheads[U.batch];
-            // Each thread owns one 16-byte chunk c of rows r0, r0+4, ...; every load is issued
-            // before any store.
-            constexpr int kPer = N * 16 / 64;
-            const int c = tid & 15, r0 = tid >> 4;
-            uint4 vals[kPer];
-#pragma unroll
-            for (int i = 0; i < kPer; ++i) {
-                const int row = r0 + 4 * i;
-                const int slot = row / W_PAD, rr = row % W_PAD;
-                vals[i] = make_uint4(0u, 0u, 0u, 0u);
-                if (slot < nheads && rr < p.w) {
-                    const int h = p.sel_heads[first + slot];
-                    const uint4* src = reinterpret_cast<const uint4*>(
-                        p.q_win + ((static_cast<size_t>(U.seq) * p.w + rr) * p.Hq + h) * kHeadDim);
-                    vals[i] = __ldg(src + c);
+    } else if (warp == 3) {
+        // ------------------------------------------------------------ publisher
+        // Once both pass-1 warpgroups have stored an item's partials, one release on the
+        // unit's arrival counter makes them visible GPU-wide; the GPU-scope fence this takes
+        // stalls only this lane, not the pass-1 warps.
+        if (lane == 0) {
+            int it = 0;
+            for (int r = 0; r < R; ++r) {
+                const ScoreItem& I = item_of(r);
+                if (I.ntiles == 0) continue;
+                if (!mbar_wait(&pub_full[it & 1], (it >> 1) & 1, abort, 64)) {
+                    *abort = 1;
+                    record_error(p.status, kDevTimeout, 17);
+                    break;
                 }
+                __threadfence();
+                red_release_add(p.counters + I.unit, kNW);
+                mbar_arrive(&pub_empty[it & 1]);
+                ++it;
             }
+        }
+    }
+    } else if (warp < kWarpB) {
+        // ------------------------------------------------------------ pass 1
+        setmaxnreg_inc<160>();
+        const int wg = (warp - kWarpA) >> 2;  // columns [wg*32, wg*32+32)
+        if (wg < kNW) {
+            const int eq = warp & 3;            // TMEM lane quarter
+            const int wtid = threadIdx.x - (kWarpA + 4 * wg) * 32;  // 0 .. 127
+            const int col0 = wg * kCols;
+            const uint32_t lane_base = static_cast<uint32_t>(eq * 32) << 16;
+            uint64_t* gbar = &group[wg];
+            uint32_t gphase = 0;
+            int a_it = 0, a_item = 0;
+            bool ok = true;
+            for (int r = 0; ok && r < R; ++r) {
+                const int item = r * G + blockIdx.x;
+                const ScoreItem I = p.items[item];
+                const int n = I.ntiles;
+                if (n == 0) continue;
+                const ScoreUnit U = p.units[I.unit];
+                const int L = U.len, P = L - p.w, nheads = p.batch_nheads[U.batch];
+                const float sl2 = p.sl2;
+                uint32_t colmask = 0;  // this warpgroup's columns that hold a real window row
 #pragma unroll
-            for (int i = 0; i < kPer; ++i) {
-                const int row = r0 + 4 * i;
-                const int half = c >> 3, cc = c & 7;
-                *reinterpret_cast<uint4*>(qbuf + half * SL::kQHalf + row * 128 +
-                                          ((cc ^ (row & 7)) << 4)) = vals[i];
+                for (int i = 0; i < kCols; ++i) {
+                    const int c = col0 + i;
+                    if ((c % W_PAD) < p.w && (c / W_PAD) < nheads) colmask |= 1u << i;
+                }
+                float m[kCols], sm_[kCols];  // running max (log2 units) and sum relative to it
+                for (int jt = 0; jt < n; ++jt, ++a_it) {
+                    const int acc = a_it % kAcc;
+                    if (!mbar_wait(&a_full[acc], (a_it / kAcc) & 1, abort)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after_sync();
+                    const int t = I.tile0 + jt;
+                    const int j = t * kTileKeys + eq * 32 + lane;  // sequence-local key
+                    const uint32_t vm = tile_mask<kCols, W_PAD>(colmask, col0, t, j, P, L);
+                    const uint32_t taddr = tmem_base + lane_base + static_cast<uint32_t>(acc * N + col0);
+                    // both halves of 16 columns in flight, then one wait
+                    float vv[2][16];
+                    tmem_ld16_nowait(taddr, vv[0]);
+                    tmem_ld16_nowait(taddr + 16, vv[1]);
+                    tmem_ld_wait();
+                    reg_fence(vv[0]);
+                    reg_fence(vv[1]);
+                    tc_fence_before_sync();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&a_empty[acc]);  // the accumulator is free
+#pragma unroll
+                    for (int hh = 0; hh < 2; ++hh) {
+                        float (&v)[16] = vv[hh];
+                        const uint32_t hm = (vm >> (16 * hh)) & 0xffffu;
+                        float* mh = m + 16 * hh;
+                        float* sh = sm_ + 16 * hh;
+                        if (jt == 0) {
+                            // The thread's first key of the item seeds each column's running
+                            // max.  A row that cannot see this key cannot see its later keys.
+#pragma unroll
+                            for (int i = 0; i < 16; ++i) {
+                                const bool valid = (hm >> i) & 1u;
+                                mh[i] = valid ? v[i] * sl2 : -1e30f;
+                                sh[i] = valid ? 1.f : 0.f;
+                            }
+                            continue;
+                        }
+                        if (hm == 0xffffu) {
+#pragma unroll
+                            for (int i = 0; i < 16; ++i) v[i] = fmaf(v[i], sl2, -mh[i]);
+                        } else {
+#pragma unroll
+                            for (int i = 0; i < 16; ++i) {
+                                const float d = fmaf(v[i], sl2, -mh[i]);
+                                v[i] = ((hm >> i) & 1u) ? d : -INFINITY;
+                            }
+                        }
+                        float dm[4];  // max by a short tree
+#pragma unroll
+                        for (int i = 0; i < 4; ++i)
+                            dm[i] = fmaxf(fmaxf(v[4 * i], v[4 * i + 1]), fmaxf(v[4 * i + 2], v[4 * i + 3]));
+                        if (fmaxf(fmaxf(dm[0], dm[1]), fmaxf(dm[2], dm[3])) > kLazyTau) {
+                            // a new running maximum well above the old one
+#pragma unroll
+                            for (int i = 0; i < 16; ++i) {
+                                if (v[i] > kLazyTau) {
+                                    sh[i] *= ex2_approx(-v[i]);
+                                    mh[i] += v[i];
+                                    v[i] = 0.f;
+                                }
+                            }
+                        }
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) sh[i] += ex2_approx(v[i]);
+                    }
+                }
+                if (!ok) break;
+                // Per column over the warpgroup's 128 keys: warp max by redux, rescale to it,
+                // warp sums by recursive halving, then the 4 warps through shared memory.
+#pragma unroll
+                for (int i = 0; i < kCols; ++i) {
+                    const float M = redux_max(m[i]);
+                    sm_[i] *= ex2_approx(m[i] - M);
+                    m[i] = M;
+                }
+                transpose_reduce<kCols>(sm_, m, lane);  // lane l: column l
+                float2* red = red_a[a_item & 1][wg];
+                red[eq * 32 + lane] = make_float2(m[0], sm_[0]);
+                if (!group_sync(gbar, gphase, abort)) {
+                    ok = false;
+                    break;
+                }
+                if (wtid < kCols) {
+                    float M = red[wtid].x;
+#pragma unroll
+                    for (int q = 1; q < 4; ++q) M = fmaxf(M, red[q * 32 + wtid].x);
+                    float S = 0.f;
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const float2 x = red[q * 32 + wtid];
+                        S += x.y * ex2_approx(x.x - M);
+                    }
+                    // the publisher has released the item two back that used this phase
+                    if (!mbar_wait(&pub_empty[a_item & 1], ((a_item >> 1) & 1) ^ 1, abort)) {
+                        ok = false;
+                        break;
+                    }
+                    p.partials[static_cast<size_t>(item) * N + col0 + wtid] = make_float2(M, S);
+                    mbar_arrive(&pub_full[a_item & 1]);
+                }
+                ++a_item;
             }
-            fence_proxy_async_smem();
-            mbar_arrive(q_full);
-            ++item_it;
+            if (!ok) {
+                *abort = 1;
+                record_error(p.status, kDevTimeout, 14);
+            }
         }
     } else {
-        // ------------------------------------------------------------ epilogue
-        const int wg = (warp - 4) >> 2;      // warpgroup: columns [wg*CPW, wg*CPW+CPW)
-        const int eq = warp & 3;             // TMEM lane quarter
-        const int etid = threadIdx.x - 128;  // 0 .. kEpiThreads-1 over the warpgroups
-        const int col0 = wg * CPW;
+        // ------------------------------------------------------------ pass 2
+        // One warpgroup over all N columns; lse sits in shared memory and is read by every
+        // lane of a warp at the same address.
+        const int eq = warp & 3;
+        const int wtid = threadIdx.x - kWarpB * 32;  // 0 .. 127
         const uint32_t lane_base = static_cast<uint32_t>(eq * 32) << 16;
-        int acc_it = 0;
+        uint64_t* gbar = &group[2];
+        uint32_t gphase = 0;
+        constexpr int kHeads = N / W_PAD;  // head slots of the MMA's columns
+        int b_it = 0;
         bool ok = true;
-        for (int r = 0; ok && r < p.n_rounds; ++r) {
-            const int item = r * gridDim.x + blockIdx.x;
-            // Everything the loops need, copied out of the parameter tables once (asm with a
-            // memory clobber inside the loops would otherwise force reloads).
-            const ScoreItem I = p.items[item];
+        for (int r = 0; ok && r < R; ++r) {
+            const ScoreItem I = p.items[r * G + blockIdx.x];
             const int n = I.ntiles;
             if (n == 0) continue;
             const ScoreUnit U = p.units[I.unit];
@@ -407,223 +679,151 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             const int T = p.T;
             const float sl2 = p.sl2;
             float* const scores = p.scores;
-            uint32_t colmask = 0;  // this warpgroup's columns that hold a real window row
+            uint64_t colmask = 0;  // columns that hold a real window row
 #pragma unroll
-            for (int i = 0; i < CPW; ++i) {
-                const int c = col0 + i;
-                if ((c % W_PAD) < p.w && (c / W_PAD) < nheads) colmask |= 1u << i;
-            }
-            float st_a[CPW];  // pass 1: running max (log2 units); pass 2: lse (log2 units)
-            float st_b[CPW];  // pass 1: running sum relative to st_a
-
-            // ---------------------------------------------------- pass 1
-            for (int jt = 0; jt < n; ++jt, ++acc_it) {
-                const int acc = acc_it % kAccBufs;
-                if (!mbar_wait(&acc_full[acc], (acc_it / kAccBufs) & 1, abort)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after_sync();
-                float v[CPW];
-                tmem_ld_cols<CPW>(tmem_base + lane_base + static_cast<uint32_t>(acc * N + col0), v);
-                tc_fence_before_sync();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&acc_empty[acc]);
-                const int t = I.tile0 + jt;
-                const int j = t * kTileKeys + eq * 32 + lane;  // sequence-local key
-                const uint32_t vm = tile_mask<CPW, W_PAD>(colmask, col0, t, j, P, L);
-                if (jt == 0) {
-                    // The thread's first key of the item seeds each row's running maximum.  A
-                    // row that cannot see this key cannot see the thread's later keys either.
-#pragma unroll
-                    for (int i = 0; i < CPW; ++i) {
-                        const bool valid = (vm >> i) & 1u;
-                        st_a[i] = valid ? v[i] * sl2 : -1e30f;
-                        st_b[i] = valid ? 1.f : 0.f;
-                    }
-                    continue;
-                }
-                if (vm == kFullMask) {
-#pragma unroll
-                    for (int i = 0; i < CPW; ++i) v[i] = fmaf(v[i], sl2, -st_a[i]);
-                } else {
-#pragma unroll
-                    for (int i = 0; i < CPW; ++i) {
-                        const float d = fmaf(v[i], sl2, -st_a[i]);
-                        v[i] = ((vm >> i) & 1u) ? d : -INFINITY;
-                    }
-                }
-                float dm[CPW / 4];  // max by a short tree
-#pragma unroll
-                for (int i = 0; i < CPW / 4; ++i)
-                    dm[i] = fmaxf(fmaxf(v[4 * i], v[4 * i + 1]), fmaxf(v[4 * i + 2], v[4 * i + 3]));
-#pragma unroll
-                for (int w = CPW / 8; w >= 1; w >>= 1)
-#pragma unroll
-                    for (int i = 0; i < w; ++i) dm[i] = fmaxf(dm[i], dm[i + w]);
-                const float dmax = dm[0];
-                if (dmax > kLazyTau) {  // a new running maximum well above the old one
-#pragma unroll
-                    for (int i = 0; i < CPW; ++i) {
-                        if (v[i] > kLazyTau) {
-                            st_b[i] *= ex2_approx(-v[i]);
-                            st_a[i] += v[i];
-                            v[i] = 0.f;
-                        }
-                    }
-                }
-#pragma unroll
-                for (int i = 0; i < CPW; ++i) st_b[i] += ex2_approx(v[i]);
-            }
-            if (!ok) break;
-
-            // The warpgroup's 128 threads per column: warp max by redux, rescale to it, warp sums
-            // by recursive halving; then the 4 warps of each warpgroup through shared memory.
-#pragma unroll
-            for (int i = 0; i < CPW; ++i) {
-                const float M = redux_max(st_a[i]);
-                st_b[i] *= ex2_approx(st_a[i] - M);
-                st_a[i] = M;
-            }
-            transpose_reduce<CPW>(st_b, st_a, lane);
-            {
-                constexpr int kLanesPerCol = 32 / CPW;
-                if (lane % kLanesPerCol == 0)
-                    red[(wg * 4 + eq) * CPW + lane / kLanesPerCol] = make_float2(st_a[0], st_b[0]);
-            }
-            named_bar_sync(1, kEpiThreads);
-            if (etid < N) {
-                const int cw = etid / CPW, ci = etid % CPW;
-                float M = red[(cw * 4) * CPW + ci].x;
-#pragma unroll
-                for (int q = 1; q < 4; ++q) M = fmaxf(M, red[(cw * 4 + q) * CPW + ci].x);
-                float S = 0.f;
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const float2 x = red[(cw * 4 + q) * CPW + ci];
-                    S += x.y * ex2_approx(x.x - M);
-                }
-                p.partials[static_cast<size_t>(item) * N + etid] = make_float2(M, S);
-            }
-            named_bar_sync(1, kEpiThreads);
-
+            for (int c = 0; c < N; ++c)
+                if ((c % W_PAD) < p.w && (c / W_PAD) < nheads) colmask |= 1ull << c;
             // ---------------------------------------------------- exchange with the unit
-            if (etid == 0) {
-                // The barrier above orders the block's partial stores before this thread's
-                // release; the fence makes that release cumulative at GPU scope.
-                __threadfence();
-                red_release_add(p.counters + I.unit, 1);
+            if (wtid == 0) {
+                const int target = U.nitems * kNW;
                 const long long t0 = clock64();
                 bool got = true;
-                for (uint32_t it = 1; ld_acquire(p.counters + I.unit) < U.nitems; ++it) {
+                for (uint32_t k = 1; ld_acquire(p.counters + I.unit) < target; ++k) {
                     __nanosleep(64);
-                    if ((it & 63u) == 0u && (*abort || clock64() - t0 > kWaitTimeoutCycles)) {
-                        *abort = 1;
-                        record_error(p.status, kDevTimeout, 13);
+                    if ((k & 63u) == 0u && (*abort || clock64() - t0 > kWaitTimeoutCycles)) {
                         got = false;
                         break;
                     }
                 }
                 __threadfence();
-                lse_s[N] = got ? 1.f : 0.f;  // one verdict for the whole epilogue
+                verdict[0] = got ? 1 : 0;
             }
-            named_bar_sync(1, kEpiThreads);
-            if (lse_s[N] == 0.f) {
+            if (!group_sync(gbar, gphase, abort) || verdict[0] == 0) {
                 ok = false;
                 break;
             }
             {
-                // All epilogue threads: column etid % N, items part, part + parts, ...
-                constexpr int kParts = kEpiThreads / N;
-                const int c = etid % N, part = etid / N;
-                float M = -INFINITY, S = 0.f;
-                const float2* src = p.partials + static_cast<size_t>(U.first_item) * N + c;
-                for (int k = part; k < U.nitems; k += kParts) {
-                    const float2 pr = __ldcg(src + static_cast<size_t>(k) * N);
-                    const float Mn = fmaxf(M, pr.x);
-                    S = S * ex2_approx(M - Mn) + pr.y * ex2_approx(pr.x - Mn);
-                    M = Mn;
+                // Column pairs (2c, 2c+1) by 16-byte loads, items split over the parts; up
+                // to kU loads in flight per thread (a unit can have ~150 items).
+                constexpr int kPairs = N / 2, kParts = 128 / kPairs, kU = 20;
+                static_assert(kParts * N <= 256, "red_b holds 256 entries");
+                const int c2 = wtid % kPairs, part = wtid / kPairs;
+                float M0 = -INFINITY, S0 = 0.f, M1 = -INFINITY, S1 = 0.f;
+                const float4* src =
+                    reinterpret_cast<const float4*>(p.partials + static_cast<size_t>(U.first_item) * N) + c2;
+                for (int k0 = part; k0 < U.nitems; k0 += kParts * kU) {
+                    float4 pr[kU];
+#pragma unroll
+                    for (int u = 0; u < kU; ++u) {
+                        const int k = k0 + u * kParts;
+                        pr[u] = k < U.nitems ? __ldcg(src + static_cast<size_t>(k) * kPairs)
+                                             : make_float4(-INFINITY, 0.f, -INFINITY, 0.f);
+                    }
+#pragma unroll
+                    for (int u = 0; u < kU; ++u) {
+                        float Mn = fmaxf(M0, pr[u].x);
+                        if (Mn > -INFINITY) {
+                            S0 = S0 * ex2_approx(M0 - Mn) + pr[u].y * ex2_approx(pr[u].x - Mn);
+                            M0 = Mn;
+                        }
+                        Mn = fmaxf(M1, pr[u].z);
+                        if (Mn > -INFINITY) {
+                            S1 = S1 * ex2_approx(M1 - Mn) + pr[u].w * ex2_approx(pr[u].z - Mn);
+                            M1 = Mn;
+                        }
+                    }
                 }
-                red[part * N + c] = make_float2(M, S);
-                named_bar_sync(1, kEpiThreads);
-                if (etid < N) {
+                red_b[part * N + 2 * c2] = make_float2(M0, S0);
+                red_b[part * N + 2 * c2 + 1] = make_float2(M1, S1);
+                if (!group_sync(gbar, gphase, abort)) {
+                    ok = false;
+                    break;
+                }
+                if (wtid < N) {  // part 0 always holds item 0, so M2 turns finite first
                     float M2 = -INFINITY, S2 = 0.f;
 #pragma unroll
                     for (int q = 0; q < kParts; ++q) {
-                        const float2 x = red[q * N + etid];
+                        const float2 x = red_b[q * N + wtid];
                         const float Mn = fmaxf(M2, x.x);
                         S2 = S2 * ex2_approx(M2 - Mn) + x.y * ex2_approx(x.x - Mn);
                         M2 = Mn;
                     }
-                    lse_s[etid] = M2 + lg2_approx(S2);
+                    lse_s[wtid] = M2 + lg2_approx(S2);
+                }
+                if (!group_sync(gbar, gphase, abort)) {
+                    ok = false;
+                    break;
                 }
             }
-            named_bar_sync(1, kEpiThreads);
-#pragma unroll
-            for (int i = 0; i < CPW; ++i) st_a[i] = lse_s[col0 + i];
-
-            // ---------------------------------------------------- pass 2 (tiles in reverse)
-            for (int jt = n - 1; jt >= 0; --jt, ++acc_it) {
-                const int acc = acc_it % kAccBufs;
-                if (!mbar_wait(&acc_full[acc], (acc_it / kAccBufs) & 1, abort)) {
+            // ---------------------------------------------------- the item's tiles
+            for (int jt = 0; jt < n; ++jt, ++b_it) {
+                const int acc = b_it % kAcc;
+                if (!mbar_wait(&b_full[acc], (b_it / kAcc) & 1, abort)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after_sync();
-                float v[CPW];
-                tmem_ld_cols<CPW>(tmem_base + lane_base + static_cast<uint32_t>(acc * N + col0), v);
-                tc_fence_before_sync();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&acc_empty[acc]);
                 const int t = I.tile0 + jt;
                 const int j = t * kTileKeys + eq * 32 + lane;
-                const uint32_t vm = tile_mask<CPW, W_PAD>(colmask, col0, t, j, P, L);
-                if (vm == kFullMask) {
+                // columns that see key j: all real ones, except in the window's own tiles
+                uint64_t vm = colmask;
+                const bool edge = (t * kTileKeys + kTileKeys - 1 >= P) || (t * kTileKeys + kTileKeys > L);
+                if (edge) {
+                    uint64_t cm = 0;
+                    if (j < L) {
 #pragma unroll
-                    for (int i = 0; i < CPW; ++i) v[i] = ex2_approx(fmaf(v[i], sl2, -st_a[i]));
-                } else {
+                        for (int c = 0; c < N; ++c) cm |= static_cast<uint64_t>((c % W_PAD) >= j - P) << c;
+                    }
+                    vm &= cm;
+                }
+                const uint32_t taddr = tmem_base + lane_base + static_cast<uint32_t>((kAcc + acc) * N);
+                // every 16-column chunk in flight, then one wait
+                float vv[N / 16][16];
 #pragma unroll
-                    for (int i = 0; i < CPW; ++i) {
-                        const float e = ex2_approx(fmaf(v[i], sl2, -st_a[i]));
-                        v[i] = ((vm >> i) & 1u) ? e : 0.f;
+                for (int hh = 0; hh < N / 16; ++hh) tmem_ld16_nowait(taddr + hh * 16, vv[hh]);
+                tmem_ld_wait();
+#pragma unroll
+                for (int hh = 0; hh < N / 16; ++hh) reg_fence(vv[hh]);
+                tc_fence_before_sync();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&b_empty[acc]);  // the accumulator is free
+                float accum[kHeads];
+#pragma unroll
+                for (int h = 0; h < kHeads; ++h) accum[h] = 0.f;
+#pragma unroll
+                for (int hh = 0; hh < N / 16; ++hh) {
+                    float (&v)[16] = vv[hh];
+                    const uint32_t hm = static_cast<uint32_t>(vm >> (16 * hh)) & 0xffffu;
+                    if (hm == 0xffffu) {
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) v[i] = ex2_approx(fmaf(v[i], sl2, -lse_s[16 * hh + i]));
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) {
+                            const float e = ex2_approx(fmaf(v[i], sl2, -lse_s[16 * hh + i]));
+                            v[i] = ((hm >> i) & 1u) ? e : 0.f;
+                        }
+                    }
+                    constexpr int kPiece = W_PAD < 16 ? W_PAD : 16;  // a head's columns in this chunk
+#pragma unroll
+                    for (int q = 0; q < 16 / kPiece; ++q) {
+                        float seg[kPiece];
+#pragma unroll
+                        for (int i = 0; i < kPiece; ++i) seg[i] = v[q * kPiece + i];
+                        accum[(16 * hh + q * kPiece) / W_PAD] += tree_sum<kPiece>(seg);
                     }
                 }
-                // per-head sums by trees over each head's (up to W_PAD) columns
-                constexpr int kSeg = kSplitHead ? CPW : W_PAD;
-                float accum[HPW];
+                if (j < L) {
+                    const size_t col = static_cast<size_t>(U.seq_start) + j;
 #pragma unroll
-                for (int h = 0; h < HPW; ++h) {
-                    float seg[kSeg];
-#pragma unroll
-                    for (int i = 0; i < kSeg; ++i) seg[i] = v[h * kSeg + i];
-                    accum[h] = tree_sum<kSeg>(seg);
-                }
-                const bool key_ok = j < L;
-                const size_t col = static_cast<size_t>(U.seq_start) + j;
-                if constexpr (kSplitHead) {
-                    // the head's first warpgroup adds the other warpgroups' parts
-                    float* xs = xsum + (acc & 1) * kEpiWG * 128;
-                    const int part = wg % kWgPerHead, hg = wg / kWgPerHead;
-                    if (part != 0) xs[wg * 128 + eq * 32 + lane] = accum[0];
-                    named_bar_sync(2, kEpiThreads);
-                    if (part == 0 && key_ok && hg < nheads) {
-                        float sum = accum[0];
-#pragma unroll
-                        for (int q = 1; q < kWgPerHead; ++q) sum += xs[(wg + q) * 128 + eq * 32 + lane];
-                        scores[static_cast<size_t>(first + hg) * T + col] = sum;
-                    }
-                } else if (key_ok) {
-#pragma unroll
-                    for (int h = 0; h < HPW; ++h) {
-                        const int hg = wg * HPW + h;
-                        if (hg < nheads) scores[static_cast<size_t>(first + hg) * T + col] = accum[h];
-                    }
+                    for (int h = 0; h < kHeads; ++h)
+                        if (h < nheads) scores[static_cast<size_t>(first + h) * T + col] = accum[h];
                 }
             }
         }
         if (!ok) {
             *abort = 1;
-            record_error(p.status, kDevTimeout, 14);
+            record_error(p.status, kDevTimeout, 16);
         }
     }
 
@@ -631,7 +831,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
     __syncthreads();
     if (warp == 1) {
         tc_fence_after_sync();
-        tmem_dealloc(tmem_base, kAccBufs * N);
+        tmem_dealloc(tmem_base, kTmemCols);
     }
 }
 
@@ -685,6 +885,7 @@ cudaError_t launch_score(const ScoreLaunch& L, cudaStream_t stream) {
     std::lock_guard<std::mutex> lock(mu);
     memset(&p, 0, sizeof(p));
     p.tmap_k = L.tmap_k;
+    p.tmap_q = L.tmap_q;
     p.q_win = reinterpret_cast<const __nv_bfloat16*>(L.q_win);
     p.cu_seqlens = L.cu_seqlens_dev;
     p.partials = reinterpret_cast<float2*>(L.partials);
