@@ -340,6 +340,9 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             uint8_t* ring = first ? ring1 : ring2;
             uint64_t* full = first ? full1 : full2;
             uint64_t* freed = first ? free1 : free2;
+            // Pass-1 tiles are read again by pass 2 shortly after: ask L2 to keep them, and
+            // to drop them first once pass 2 has read them.
+            const uint64_t policy = first ? l2_policy_evict_last() : l2_policy_evict_first();
             int use = 0, it = 0;
             bool ok = true;
             for (int r = 0; ok && r < R; ++r) {
@@ -388,8 +391,8 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                     mbar_arrive_expect_tx(&full[s], kTileBytes);
                     uint8_t* dst = ring + s * kTileBytes;
                     const int tok = U.seq_start + (I.tile0 + jt) * kTileKeys;
-                    tma_load_3d(dst, &p.tmap_k, &full[s], 0, g, tok);
-                    tma_load_3d(dst + kHalfBytes, &p.tmap_k, &full[s], 64, g, tok);
+                    tma_load_3d_hint(dst, &p.tmap_k, &full[s], 0, g, tok, policy);
+                    tma_load_3d_hint(dst + kHalfBytes, &p.tmap_k, &full[s], 64, g, tok, policy);
                 }
                 ++it;
                 if (first) *issued = it;
@@ -548,7 +551,14 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                     const int c = col0 + i;
                     if ((c % W_PAD) < p.w && (c / W_PAD) < nheads) colmask |= 1u << i;
                 }
-                float m[kCols], sm_[kCols];  // running max (log2 units) and sum relative to it
+                // Running max (log2 units) and sum relative to it.  -1e30 (not -inf) for a
+                // column with no visible key yet keeps the reductions below free of inf - inf.
+                float m[kCols], sm_[kCols];
+#pragma unroll
+                for (int i = 0; i < kCols; ++i) {
+                    m[i] = -1e30f;
+                    sm_[i] = 0.f;
+                }
                 for (int jt = 0; jt < n; ++jt, ++a_it) {
                     const int acc = a_it % kAcc;
                     if (!mbar_wait(&a_full[acc], (a_it / kAcc) & 1, abort)) {
@@ -576,44 +586,30 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                         const uint32_t hm = (vm >> (16 * hh)) & 0xffffu;
                         float* mh = m + 16 * hh;
                         float* sh = sm_ + 16 * hh;
-                        if (jt == 0) {
-                            // The thread's first key of the item seeds each column's running
-                            // max.  A row that cannot see this key cannot see its later keys.
+                        float d[16];
 #pragma unroll
-                            for (int i = 0; i < 16; ++i) {
-                                const bool valid = (hm >> i) & 1u;
-                                mh[i] = valid ? v[i] * sl2 : -1e30f;
-                                sh[i] = valid ? 1.f : 0.f;
-                            }
-                            continue;
-                        }
-                        if (hm == 0xffffu) {
-#pragma unroll
-                            for (int i = 0; i < 16; ++i) v[i] = fmaf(v[i], sl2, -mh[i]);
-                        } else {
-#pragma unroll
-                            for (int i = 0; i < 16; ++i) {
-                                const float d = fmaf(v[i], sl2, -mh[i]);
-                                v[i] = ((hm >> i) & 1u) ? d : -INFINITY;
-                            }
+                        for (int i = 0; i < 16; ++i) {
+                            const float x = fmaf(v[i], sl2, -mh[i]);
+                            d[i] = ((hm >> i) & 1u) ? x : -INFINITY;
                         }
                         float dm[4];  // max by a short tree
 #pragma unroll
                         for (int i = 0; i < 4; ++i)
-                            dm[i] = fmaxf(fmaxf(v[4 * i], v[4 * i + 1]), fmaxf(v[4 * i + 2], v[4 * i + 3]));
+                            dm[i] = fmaxf(fmaxf(d[4 * i], d[4 * i + 1]), fmaxf(d[4 * i + 2], d[4 * i + 3]));
                         if (fmaxf(fmaxf(dm[0], dm[1]), fmaxf(dm[2], dm[3])) > kLazyTau) {
-                            // a new running maximum well above the old one
+                            // A logit well above the running maximum (always so for a column's
+                            // first visible key): restart the column's sum relative to it.
 #pragma unroll
                             for (int i = 0; i < 16; ++i) {
-                                if (v[i] > kLazyTau) {
-                                    sh[i] *= ex2_approx(-v[i]);
-                                    mh[i] += v[i];
-                                    v[i] = 0.f;
+                                if (d[i] > kLazyTau) {
+                                    sh[i] *= ex2_approx(-d[i]);
+                                    mh[i] = v[i] * sl2;
+                                    d[i] = 0.f;
                                 }
                             }
                         }
 #pragma unroll
-                        for (int i = 0; i < 16; ++i) sh[i] += ex2_approx(v[i]);
+                        for (int i = 0; i < 16; ++i) sh[i] += ex2_approx(d[i]);
                     }
                 }
                 if (!ok) break;
@@ -794,15 +790,10 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                 for (int hh = 0; hh < N / 16; ++hh) {
                     float (&v)[16] = vv[hh];
                     const uint32_t hm = static_cast<uint32_t>(vm >> (16 * hh)) & 0xffffu;
-                    if (hm == 0xffffu) {
 #pragma unroll
-                        for (int i = 0; i < 16; ++i) v[i] = ex2_approx(fmaf(v[i], sl2, -lse_s[16 * hh + i]));
-                    } else {
-#pragma unroll
-                        for (int i = 0; i < 16; ++i) {
-                            const float e = ex2_approx(fmaf(v[i], sl2, -lse_s[16 * hh + i]));
-                            v[i] = ((hm >> i) & 1u) ? e : 0.f;
-                        }
+                    for (int i = 0; i < 16; ++i) {
+                        const float e = ex2_approx(fmaf(v[i], sl2, -lse_s[16 * hh + i]));
+                        v[i] = ((hm >> i) & 1u) ? e : 0.f;
                     }
                     constexpr int kPiece = W_PAD < 16 ? W_PAD : 16;  // a head's columns in this chunk
 #pragma unroll
