@@ -171,8 +171,9 @@ ckv_status plan_score(const Plan& pl, const ckv_batch* b, int skip_le, int ctas,
     L.slices.clear();
     if (raw.empty()) return CKV_OK;
     if (b->num_seqs > 65535) return fail(CKV_ERR_UNSUPPORTED, "more than 65535 sequences");
-    constexpr int kL2Tiles = 8;        // 2 items x 8 tiles x 32 KiB x 152 CTAs ~ 78 MB of L2
-    constexpr double kExchange = 4.0;  // the exchange, in tile-load times
+    constexpr int kL2Tiles = 16;       // 16 tiles x 32 KiB x 152 CTAs ~ 78 MB of L2, kept there
+                                       // by the kernel's evict-last hint until pass 2 reads it
+    constexpr double kExchange = 12.0; // publish, exchange and combine, in tile-load times
     constexpr double kPass2 = 0.4;     // pass 2 per tile from L2, relative to a pass-1 load
     int best_c = -1;
     double best_cost = 0;

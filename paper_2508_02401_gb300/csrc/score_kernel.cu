@@ -486,8 +486,10 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                     idle = 0;
                     t0 = clock64();
                 } else {
-                    __nanosleep(20);
-                    if ((++idle & 63u) == 0u && (*abort || clock64() - t0 > kWaitTimeoutCycles)) {
+                    // Nothing ready: back off (32 ns doubling to 256 ns), so that the polls do
+                    // not take issue slots from the epilogue warps of this SM sub-partition.
+                    __nanosleep(32u << (idle < 3u ? idle : 3u));
+                    if ((++idle & 15u) == 0u && (*abort || clock64() - t0 > kWaitTimeoutCycles)) {
                         ok = false;
                         break;
                     }
