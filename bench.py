@@ -39,7 +39,7 @@ HBM_FALLBACK_GBS = 6800.0
 # capture summarised in profiles/score_kernel_llama8b_l8192.md, keyed by the sha256 of the
 # kernel source it was taken on; a changed kernel reports null until it is captured again.
 SCORE_TRAFFIC = {
-    "32d2a5579cdc99ed22368dd49779372e10ef36016648c6a00524df233b42391b": 16976128,
+    "3893613cffe69c5ce65a7dba1aa62659a2b451aa6ab525761c01c5451a88608b": 16996096,
 }
 # Sequences up to this many tokens are selected by one block per (sequence, KV head)
 # (one launch); longer ones by the chunked kernels (two launches).
@@ -57,8 +57,9 @@ def _args():
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--layers", type=int, default=0, help="use only the first N layers (0 = all)")
     ap.add_argument("--breakdown", action="store_true", help="per-stage times on stderr")
-    ap.add_argument("--streams", type=int, default=4,
-                    help="layers are issued round-robin on this many streams (one workspace each)")
+    ap.add_argument("--streams", type=int, default=16,
+                    help="layers are issued round-robin on this many streams (one workspace each); "
+                         "each call is capped at SMs / streams CTAs")
     return ap.parse_args()
 
 
