@@ -166,6 +166,29 @@ CKV_API ckv_status ckv_compress_layer(const ckv_config* cfg, int32_t layer, cons
                               int32_t* cu_keep_dev, void* k_out, void* v_out, float* pooled_out,
                               void* workspace, size_t workspace_bytes, ckv_stream stream);
 
+/* Layer budgets (App. B, the paper's error-aware layer-adaptive allocation).  Host only; no
+ * GPU is needed.
+ *
+ * ckv_layer_error_scores: Eq. 11-13.  errors [num_datasets][num_layers] (host, row-major) are
+ * the per-layer compression errors e_d^(l) of Eq. 10 (finite, >= 0; each dataset's row must
+ * not sum to 0).  Each row is divided by its sum (Eq. 11), the rows are averaged (Eq. 12) and
+ * the average is divided by its sum (Eq. 13) into scores[num_layers] (host, caller-owned).
+ *
+ * ckv_allocate_budgets: Algorithm 1.  From scores[num_layers] (finite, >= 0, normally the
+ * output above) and the total budget B_total, every layer starts at min_budget (m), the rest
+ * B_total - m * num_layers is handed out as round(score * rest) (ties to even) clipped to
+ * [m, max_budget], and the difference left by rounding and clipping is settled one token at
+ * a time: added to the highest-scoring layer still below M, or taken from the lowest-scoring
+ * layer still above m (lowest layer index among equal scores).  The paper uses m = 32 and
+ * M = 3 * B_total / num_layers.  The budgets sum to B_total whenever
+ * m * num_layers <= B_total <= M * num_layers; otherwise every layer ends at m (or M).
+ * Writes budgets[num_layers] (host, caller-owned), usable as ckv_config.budgets. */
+CKV_API ckv_status ckv_layer_error_scores(const double* errors, int32_t num_datasets,
+                                          int32_t num_layers, double* scores);
+CKV_API ckv_status ckv_allocate_budgets(const double* scores, int32_t num_layers,
+                                        int64_t total_budget, int32_t min_budget,
+                                        int32_t max_budget, int32_t* budgets);
+
 /* Synchronises `stream`, then returns the workspace's device status: *code = 0 if no kernel
  * recorded an error since the last reset, else the first error (1 = cu_seqlens_dev disagrees
  * with the host copy, 2 = a wait timed out, 3 = an index out of range); *detail says where.

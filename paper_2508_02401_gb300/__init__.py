@@ -78,6 +78,8 @@ def load():
         "ckv_compress_layer": ([cfg, I32, bat, P, P, P, I64, I64, P, P, P, P, P, P, SZ, P], C.c_int),
         "ckv_read_device_status": ([P, P, I32, C.POINTER(I32), C.POINTER(I32)], C.c_int),
         "ckv_score_window_static": ([cfg, I32, bat, P, P, I64, I64, P, P, P], C.c_int),
+        "ckv_layer_error_scores": ([P, I32, I32, P], C.c_int),
+        "ckv_allocate_budgets": ([P, I32, I64, I32, I32, P], C.c_int),
     }
     for name, (args, res) in sigs.items():
         fn = getattr(lib, name)
@@ -187,6 +189,29 @@ def ckv_keep_lengths(cfg: Config, layer: int, batch: Batch):
     _check(load().ckv_keep_lengths(cfg.ref, layer, batch.ref, out.ctypes.data, C.byref(n_sel)),
            "ckv_keep_lengths")
     return out, n_sel.value
+
+
+def ckv_layer_error_scores(errors) -> np.ndarray:
+    """Eq. 11-13: per-layer scores (float64 [L]) from errors [datasets, L] (host)."""
+    e = np.ascontiguousarray(errors, dtype=np.float64)
+    if e.ndim != 2:
+        raise ValueError("errors must be [datasets, layers]")
+    out = np.zeros(e.shape[1], np.float64)
+    _check(load().ckv_layer_error_scores(e.ctypes.data, e.shape[0], e.shape[1], out.ctypes.data),
+           "ckv_layer_error_scores")
+    return out
+
+
+def ckv_allocate_budgets(scores, total_budget: int, min_budget: int = 32, max_budget: int | None = None):
+    """Algorithm 1: int32 [L] budgets; max_budget defaults to 3 * total_budget // L."""
+    s = np.ascontiguousarray(scores, dtype=np.float64)
+    L = s.shape[0]
+    if max_budget is None:
+        max_budget = 3 * int(total_budget) // max(L, 1)
+    out = np.zeros(L, np.int32)
+    _check(load().ckv_allocate_budgets(s.ctypes.data, L, int(total_budget), int(min_budget),
+                                       int(max_budget), out.ctypes.data), "ckv_allocate_budgets")
+    return out
 
 
 def ckv_score_window(cfg, layer, batch, q_win, k, scores, workspace, stream=None,

@@ -474,6 +474,15 @@ SelectLaunch select_launch(const Plan& pl, const ckv_batch* b, int T, int T_keep
 }
 
 }  // namespace
+
+// The last-error message for the other translation units (host-only entry points).
+ckv_status set_error(ckv_status st, const char* fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_msg, sizeof g_msg, fmt, ap);
+    va_end(ap);
+    return st;
+}
 }  // namespace ckv
 
 using namespace ckv;
