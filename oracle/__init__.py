@@ -46,7 +46,7 @@ def _load():
         lib.ckv_oracle_keep_lengths.argtypes = [C.c_int, P, C.c_int, P]
         lib.ckv_oracle_compress_layer.argtypes = [
             C.c_int, P, C.c_int, C.c_int, C.c_int, C.c_int, C.c_double, P, C.c_int,
-            C.c_int, C.c_int, C.c_int, P, P, P, P, P, P, P, P, P, P, C.c_int]
+            C.c_int, C.c_int, C.c_int, C.c_int, P, P, P, P, P, P, P, P, P, P, C.c_int]
         lib.ckv_oracle_threads.argtypes = [C.c_int]
         _lib = lib
     return _lib
@@ -104,16 +104,19 @@ def keep_lengths(cu_seqlens: np.ndarray, budget: int) -> np.ndarray:
     return out
 
 
+SCOPE_KV_HEAD, SCOPE_LAYER = 0, 1
+
+
 def compress_layer(q_win, k, v, cu_seqlens, head_mask, budget, window, pool_kernel, pool_type,
                    head_order, scale=None, want_scores=True, want_kv=True, groups=None,
-                   num_threads=0):
+                   num_threads=0, scope=SCOPE_KV_HEAD):
     """One layer of the compression step.  Arrays are bf16 bits (uint16), packed.
 
     q_win [S, w, Hq, d], k/v [T, Hkv, d], cu_seqlens [S+1], head_mask [Hq] (uint8).
-    Returns a dict with scores [n_sel, T] (float64), pooled [Hkv, T] (float64), cu_keep [S+1],
-    idx [Hkv, T_keep] (int32), k_out / v_out [T_keep, Hkv, d] (uint16).
-    ``groups`` (optional iterable of KV heads) restricts the work to those groups; rows of the
-    other groups are left as NaN / -1.
+    Returns a dict with scores [n_sel, T] (float64), pooled [Hkv, T] (float64; [1, T] with
+    scope=SCOPE_LAYER), cu_keep [S+1], idx [Hkv, T_keep] (int32), k_out / v_out
+    [T_keep, Hkv, d] (uint16).  ``groups`` (optional iterable of KV heads, KV-head scope only)
+    restricts the work to those groups; rows of the other groups are left as NaN / -1.
     """
     q_win = np.ascontiguousarray(q_win, dtype=np.uint16)
     k = np.ascontiguousarray(k, dtype=np.uint16)
@@ -129,7 +132,7 @@ def compress_layer(q_win, k, v, cu_seqlens, head_mask, budget, window, pool_kern
     Tk = int(cu_keep[-1])
     n_sel = int(mask.astype(bool).sum())
     scores = np.full((n_sel, T), np.nan) if want_scores else None
-    pooled = np.full((Hkv, T), np.nan)
+    pooled = np.full((Hkv if scope == SCOPE_KV_HEAD else 1, T), np.nan)
     idx = np.full((Hkv, Tk), -1, np.int32)
     k_out = np.zeros((Tk, Hkv, d), np.uint16) if want_kv else None
     v_out = np.zeros((Tk, Hkv, d), np.uint16) if want_kv else None
@@ -139,6 +142,6 @@ def compress_layer(q_win, k, v, cu_seqlens, head_mask, budget, window, pool_kern
         gf[list(groups)] = 1
     _check(_load().ckv_oracle_compress_layer(
         S, _p(cu), Hq, Hkv, d, window, float(scale), _p(mask), int(budget), int(pool_kernel),
-        int(pool_type), int(head_order), _p(q_win), _p(k), _p(v), _p(scores), _p(pooled),
+        int(pool_type), int(head_order), int(scope), _p(q_win), _p(k), _p(v), _p(scores), _p(pooled),
         None, _p(idx), _p(k_out), _p(v_out), _p(gf), int(num_threads)))
     return dict(scores=scores, pooled=pooled, cu_keep=cu_keep, idx=idx, k_out=k_out, v_out=v_out)

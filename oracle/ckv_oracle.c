@@ -23,7 +23,9 @@
  *   (iv)  both head orders are provided: pool each selected head then sum (the order of
  *         Sec. 3.3) or sum the selected heads then pool;
  *   (v)   heads are summed, not averaged (a positive rescale; the ranking is identical);
- *   (vi)  one index set per KV head, from the selected heads of its GQA group;
+ *   (vi)  one index set per KV head, from the selected heads of its GQA group (scope 0); or,
+ *         as Sec. 3.3 states it, one index set per layer from all of the layer's selected
+ *         heads, shared by every KV head (scope 1);
  *   (vii) the budget B counts the window: k = B - w candidates are kept; if L <= B every
  *         position is kept;
  *   (viii) ties in the selection go to the lower position;
@@ -193,17 +195,26 @@ int ckv_oracle_keep_lengths(int S, const int32_t* cu_seqlens, int budget, int32_
  *   k_out, v_out [T_keep, Hkv, d]  the kept rows
  * group_filter (optional, [Hkv]): when given, only groups with a non-zero entry are computed.
  */
+/*
+ * One layer of the step (Sec. 3.3).  scope 0: a vector, a selection and an index set per KV
+ * head g from the selected heads of group g.  scope 1: one vector and one selection per
+ * sequence from every selected head of the layer (each head against its own group's keys);
+ * the index set is repeated for every KV head and each KV head's rows are gathered with it.
+ * pooled has Hkv rows (scope 0) or 1 row (scope 1); idx and the outputs have Hkv rows.
+ */
 int ckv_oracle_compress_layer(int S, const int32_t* cu_seqlens, int Hq, int Hkv, int d, int w,
                               double scale, const uint8_t* head_mask, int budget,
-                              int pool_kernel, int pool_type, int head_order,
+                              int pool_kernel, int pool_type, int head_order, int scope,
                               const uint16_t* q_win, const uint16_t* k, const uint16_t* v,
                               double* scores, double* pooled, int32_t* cu_keep, int32_t* idx,
                               uint16_t* k_out, uint16_t* v_out, const uint8_t* group_filter,
                               int num_threads) {
     if (S < 0 || Hq < 1 || Hkv < 1 || Hq % Hkv != 0 || d < 1 || w < 1 || budget < w ||
         pool_kernel < 1 || pool_kernel % 2 == 0 || (pool_type != 0 && pool_type != 1) ||
-        (head_order != 0 && head_order != 1))
+        (head_order != 0 && head_order != 1) || (scope != 0 && scope != 1) ||
+        (scope == 1 && group_filter))
         return ORACLE_BAD_ARG;
+    const int n_vec = scope == 0 ? Hkv : 1; /* selections per sequence */
     const int G = Hq / Hkv;
     const int T = cu_seqlens[S];
     int32_t* keep = (int32_t*)malloc(sizeof(int32_t) * (size_t)(S + 1));
@@ -223,13 +234,14 @@ int ckv_oracle_compress_layer(int S, const int32_t* cu_seqlens, int Hq, int Hkv,
     const int Tk = keep[S];
     int n_sel = 0;
     for (int h = 0; h < Hq; ++h) sel_row[h] = head_mask[h] ? n_sel++ : -1;
-    for (int g = 0; g < Hkv; ++g) {
+    for (int g = 0; g < n_vec; ++g) {
         int any = 0;
-        for (int h = g * G; h < (g + 1) * G; ++h) any |= head_mask[h] != 0;
+        const int h0 = scope == 0 ? g * G : 0, h1 = scope == 0 ? (g + 1) * G : Hq;
+        for (int h = h0; h < h1; ++h) any |= head_mask[h] != 0;
         if (!any) {
             free(keep);
             free(sel_row);
-            return ORACLE_BAD_ARG; /* every KV group needs a selected head */
+            return ORACLE_BAD_ARG; /* every selection needs a selected head */
         }
     }
     int failed = 0;
@@ -237,8 +249,8 @@ int ckv_oracle_compress_layer(int S, const int32_t* cu_seqlens, int Hq, int Hkv,
     if (num_threads > 0) omp_set_num_threads(num_threads);
 #pragma omp parallel for schedule(dynamic, 1) reduction(| : failed)
 #endif
-    for (int unit = 0; unit < S * Hkv; ++unit) {
-        const int s = unit / Hkv, g = unit % Hkv;
+    for (int unit = 0; unit < S * n_vec; ++unit) {
+        const int s = unit / n_vec, g = unit % n_vec; /* g: the KV head, or 0 (scope 1) */
         if (group_filter && !group_filter[g]) continue;
         const int t0 = cu_seqlens[s];
         const int L = cu_seqlens[s + 1] - t0;
@@ -256,10 +268,11 @@ int ckv_oracle_compress_layer(int S, const int32_t* cu_seqlens, int Hq, int Hkv,
         }
         /* steps 1-3: per selected head, window attention summed over the window rows, then
          * pooled and summed over heads (head_order 0) or summed and then pooled (1) */
-        for (int h = g * G; h < (g + 1) * G; ++h) {
+        const int h0 = scope == 0 ? g * G : 0, h1 = scope == 0 ? (g + 1) * G : Hq;
+        for (int h = h0; h < h1; ++h) {
             if (!head_mask[h]) continue;
             const uint16_t* qh = q_win + ((long)s * w * Hq + h) * d;
-            const uint16_t* kg = k + ((long)t0 * Hkv + g) * d;
+            const uint16_t* kg = k + ((long)t0 * Hkv + h / G) * d; /* the head's own KV group */
             if (ckv_oracle_window_scores(L, w, d, scale, qh, (long)Hq * d, kg, (long)Hkv * d,
                                          a, lse, mass)) {
                 failed |= 1;
@@ -293,14 +306,17 @@ int ckv_oracle_compress_layer(int S, const int32_t* cu_seqlens, int Hq, int Hkv,
                 if (ckv_oracle_topk(acc, P, kc, out)) failed |= 1;
                 for (int i = 0; i < w; ++i) out[kc + i] = P + i;
             }
-            /* step 5: the kept K/V rows, in position order */
-            for (int i = 0; i < kn; ++i) {
-                if (idx) idx[(long)g * Tk + ks + i] = out[i];
-                long src = ((long)(t0 + out[i]) * Hkv + g) * d;
-                long dst = ((long)(ks + i) * Hkv + g) * d;
-                if (k_out) memcpy(k_out + dst, k + src, sizeof(uint16_t) * (size_t)d);
-                if (v_out) memcpy(v_out + dst, v + src, sizeof(uint16_t) * (size_t)d);
-            }
+            /* step 5: the kept K/V rows, in position order, for the KV head (scope 0) or for
+             * every KV head (scope 1) */
+            const int kv0 = scope == 0 ? g : 0, kv1 = scope == 0 ? g + 1 : Hkv;
+            for (int kv = kv0; kv < kv1; ++kv)
+                for (int i = 0; i < kn; ++i) {
+                    if (idx) idx[(long)kv * Tk + ks + i] = out[i];
+                    long src = ((long)(t0 + out[i]) * Hkv + kv) * d;
+                    long dst = ((long)(ks + i) * Hkv + kv) * d;
+                    if (k_out) memcpy(k_out + dst, k + src, sizeof(uint16_t) * (size_t)d);
+                    if (v_out) memcpy(v_out + dst, v + src, sizeof(uint16_t) * (size_t)d);
+                }
             free(out);
         }
         free(a); free(acc); free(tmp); free(lse); free(mass);

@@ -78,23 +78,28 @@ def _pool(x, kernel, pool_type):
 
 
 def compress_layer_reference(q_win, k, v, cu_seqlens, head_mask, budget, window, pool_kernel,
-                             pool_type, head_order, scale=None):
-    """Whole step for inputs where every sequence has L >= window.  bf16 bits in."""
+                             pool_type, head_order, scale=None, scope=0):
+    """Whole step for inputs where every sequence has L >= window.  bf16 bits in.
+
+    scope 0: one vector and selection per KV head g from the selected heads of group g;
+    scope 1: one per sequence from all selected heads (kept[(s, 0)], pooled row 0)."""
     qf, kf = widen(q_win), widen(k)
     S = len(cu_seqlens) - 1
     T, Hkv, d = k.shape
     Hq = q_win.shape[2]
     G = Hq // Hkv
     scale = 1.0 / math.sqrt(d) if scale is None else scale
-    pooled = np.zeros((Hkv, T))
+    n_vec = Hkv if scope == 0 else 1
+    pooled = np.zeros((n_vec, T))
     kept = {}
     for s in range(S):
         t0, t1 = int(cu_seqlens[s]), int(cu_seqlens[s + 1])
         L = t1 - t0
         P = L - window
-        for g in range(Hkv):
-            heads = [h for h in range(g * G, (g + 1) * G) if head_mask[h]]
-            vecs = [window_attention_matrix(qf[s, :, h, :], kf[t0:t1, g, :], scale)[:P]
+        for g in range(n_vec):
+            span = range(g * G, (g + 1) * G) if scope == 0 else range(Hq)
+            heads = [h for h in span if head_mask[h]]
+            vecs = [window_attention_matrix(qf[s, :, h, :], kf[t0:t1, h // G, :], scale)[:P]
                     for h in heads]
             if head_order == 0:
                 c = np.sum([_pool(a, pool_kernel, pool_type) for a in vecs], axis=0)

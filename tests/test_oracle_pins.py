@@ -281,3 +281,59 @@ def test_rejects_bad_arguments(oracle_lib):
     bad[:4] = 0                      # a group without a selected head
     with pytest.raises(ValueError):
         oracle_lib.compress_layer(li.q_win, li.k, li.v, wl.cu_seqlens(), bad, 24, 8, 5, 0, 0)
+
+
+# ---------------------------------------------------------------- layer scope (Sec. 3.3 as printed)
+@pytest.mark.parametrize("pool_type", ["max", "avg"])
+@pytest.mark.parametrize("head_order", ["pool_then_sum", "sum_then_pool"])
+def test_layer_scope_matches_independent_pipeline(oracle_lib, pool_type, head_order):
+    """One vector per sequence from every selected head, each against its own group's keys."""
+    wl = _tiny(pool_type=pool_type, head_order=head_order, seqlens=(96, 40, 120), budget_mean=30)
+    mask = np.array([0, 1, 1, 0, 0, 0, 1, 1], np.uint8)  # 4 heads over the two groups
+    out, li, m = _run(oracle_lib, wl, mask=mask, scope=oracle_lib.SCOPE_LAYER)
+    pooled, kept = ind.compress_layer_reference(
+        li.q_win, li.k, li.v, wl.cu_seqlens(), mask, 30, wl.window, wl.pool_kernel,
+        0 if pool_type == "max" else 1, 0 if head_order == "pool_then_sum" else 1, scope=1)
+    cu, ck = wl.cu_seqlens(), out["cu_keep"]
+    assert out["pooled"].shape[0] == 1
+    for s in range(wl.num_seqs):
+        P = wl.seqlens[s] - wl.window
+        np.testing.assert_allclose(out["pooled"][0, cu[s]:cu[s] + P], pooled[0, cu[s]:cu[s] + P],
+                                   rtol=1e-11)
+        for g in range(wl.num_kv_heads):  # the same positions for every KV head
+            np.testing.assert_array_equal(out["idx"][g, ck[s]:ck[s + 1]], kept[(s, 0)])
+    for g in range(wl.num_kv_heads):  # each KV head's own rows at those positions
+        for s in range(wl.num_seqs):
+            rows = cu[s] + out["idx"][g, ck[s]:ck[s + 1]]
+            np.testing.assert_array_equal(out["k_out"][ck[s]:ck[s + 1], g], li.k[rows, g])
+            np.testing.assert_array_equal(out["v_out"][ck[s]:ck[s + 1], g], li.v[rows, g])
+
+
+def test_layer_scope_vector_is_the_sum_of_the_groups_vectors(oracle_lib):
+    wl = _tiny(seqlens=(150, 70), budget_mean=40)
+    mask = np.array([1, 0, 1, 0, 0, 1, 0, 1], np.uint8)  # both groups have selected heads
+    per_group, _, _ = _run(oracle_lib, wl, mask=mask)
+    layer, _, _ = _run(oracle_lib, wl, mask=mask, scope=oracle_lib.SCOPE_LAYER)
+    cu = wl.cu_seqlens()
+    for s in range(wl.num_seqs):
+        P = wl.seqlens[s] - wl.window
+        a = per_group["pooled"][:, cu[s]:cu[s] + P].sum(axis=0)
+        np.testing.assert_allclose(layer["pooled"][0, cu[s]:cu[s] + P], a, rtol=1e-12)
+
+
+def test_layer_scope_with_one_kv_head_is_the_kv_head_scope(oracle_lib):
+    wl = _tiny(num_q_heads=4, num_kv_heads=1, heads_per_group=2, seqlens=(120, 60), budget_mean=30)
+    a, _, m = _run(oracle_lib, wl)
+    b, _, _ = _run(oracle_lib, wl, mask=m, scope=oracle_lib.SCOPE_LAYER)
+    for key in ("pooled", "idx", "k_out", "v_out", "cu_keep"):
+        np.testing.assert_array_equal(a[key], b[key])
+
+
+def test_layer_scope_allows_groups_without_selected_heads(oracle_lib):
+    wl = _tiny(seqlens=(100,), budget_mean=30)
+    mask = np.array([1, 1, 1, 0, 0, 0, 0, 0], np.uint8)  # every selected head in group 0
+    with pytest.raises(ValueError):
+        _run(oracle_lib, wl, mask=mask)  # the KV-head scope needs a head in every group
+    out, li, _ = _run(oracle_lib, wl, mask=mask, scope=oracle_lib.SCOPE_LAYER)
+    np.testing.assert_array_equal(out["idx"][0], out["idx"][1])
+    assert len(set(out["idx"][0].tolist())) == 30
