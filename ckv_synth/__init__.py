@@ -171,6 +171,8 @@ class Workload:
     plant_noise: bool = False
     seed: int = 20250802
     description: str = ""
+    heads_per_layer: int = 0         # > 0: that many selected heads per layer, from any group
+    scope: str = "kv_head"           # "kv_head" | "layer": one selection per KV head / per layer
 
     # ---- shapes -------------------------------------------------------------------------
     @property
@@ -194,10 +196,19 @@ class Workload:
     # ---- per-layer head mask and budgets -------------------------------------------------
     def head_mask(self) -> np.ndarray:
         """uint8 [num_layers, H_q]: 1 marks a selected (semantic retrieval) head."""
+        m = np.zeros((self.num_layers, self.num_q_heads), dtype=np.uint8)
+        if self.heads_per_layer > 0:  # heads_per_layer of the layer's heads, any groups
+            n = self.heads_per_layer
+            if n > self.num_q_heads:
+                raise ValueError("heads_per_layer must be at most num_q_heads")
+            for l in range(self.num_layers):
+                key = _stream_key(self.seed, _K_MASK, l, 1 << 16)
+                order = np.argsort(uniform_u64(key, 0, self.num_q_heads), kind="stable")
+                m[l, order[:n]] = 1
+            return m
         G, n = self.group_size, self.heads_per_group
         if not 1 <= n <= G:
             raise ValueError("heads_per_group must be in [1, group size]")
-        m = np.zeros((self.num_layers, self.num_q_heads), dtype=np.uint8)
         for l in range(self.num_layers):
             for g in range(self.num_kv_heads):
                 key = _stream_key(self.seed, _K_MASK, l, g)
@@ -271,6 +282,8 @@ class Workload:
             out[s] = pos
             for g in range(self.num_kv_heads):
                 heads = np.nonzero(mask[g * G:(g + 1) * G])[0] + g * G
+                if heads.size == 0:  # a group without a selected head: the layer's heads
+                    heads = np.nonzero(mask)[0]
                 u = qf[s][:, heads, :].reshape(-1, d).mean(axis=0)
                 u /= np.linalg.norm(u)
                 rows = np.broadcast_to(beta * u, (n, d)).copy()
@@ -314,6 +327,13 @@ _W = [
              budget_mean=512, outlier_channels=8, seed=20250802 + 4,
              description="8 ragged sequences in [4096, 32768], Qwen2.5-7B-shaped 28 layers, 28/4 "
                          "heads, mean budget 512, varlen packed"),
+    Workload(name="paper_llama8b_l8192", num_layers=32, num_q_heads=32, num_kv_heads=8,
+             seqlens=(8192,), window=8, heads_per_group=1, heads_per_layer=4, scope="layer",
+             pool_kernel=5, pool_type="avg", budget_mean=256, outlier_channels=8,
+             plant="tokens", plant_count=4, plant_beta=6.0, seed=20250802 + 5,
+             description="the paper's own hyper-parameters (App. A, Sec. 4.1): one index set per "
+                         "layer from the top-4 heads of the layer, w=8, avg pool 5; "
+                         "Llama-3.1-8B-shaped 32 layers, L=8192, 4 planted keys"),
 ]
 WORKLOAD_ORDER = [w.name for w in _W]
 WORKLOADS = {w.name: w for w in _W}

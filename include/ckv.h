@@ -22,10 +22,12 @@
  *                                     0 = packed: tok_stride = H_kv*128, head_stride = 128)
  *       scores [n_sel, T]   fp32      one row per selected head of the layer, in ascending
  *                                     query-head order (so grouped by KV head)
- *       pooled [H_kv, T]    fp32      combined, pooled scores on candidate positions; 0 at the
- *                                     window positions
+ *       pooled [n_vec, T]   fp32      combined, pooled scores on candidate positions; 0 at the
+ *                                     window positions; n_vec = H_kv (CKV_SCOPE_KV_HEAD) or 1
+ *                                     (CKV_SCOPE_LAYER)
  *       idx    [H_kv, T_keep] int32   kept sequence-local positions; the positions of sequence
- *                                     s for head g are idx[g*T_keep + cu_keep[s] ...]
+ *                                     s for head g are idx[g*T_keep + cu_keep[s] ...] (the same
+ *                                     for every g with CKV_SCOPE_LAYER)
  *       k_out, v_out [T_keep, H_kv, 128]  packed
  *     with T = cu_seqlens[S], T_keep = sum_s min(B_l, L_s).
  *   - The caller owns every buffer.  The library allocates no device or host memory during a
@@ -51,7 +53,7 @@
 extern "C" {
 #endif
 
-#define CKV_ABI_VERSION 1
+#define CKV_ABI_VERSION 2
 
 #if defined(__GNUC__)
 #define CKV_API __attribute__((visibility("default")))
@@ -69,6 +71,14 @@ typedef enum ckv_status {
     CKV_ERR_CUDA = 4,        /* a CUDA runtime call failed; see ckv_last_error_message() */
     CKV_ERR_DEVICE = 5       /* a kernel recorded an error in the workspace status word */
 } ckv_status;
+
+/* Which heads' vectors make one selection (Sec. 3.3). */
+typedef enum ckv_scope {
+    CKV_SCOPE_KV_HEAD = 0, /* one selection per KV head g from the selected heads of group g;
+                              each KV head keeps its own positions */
+    CKV_SCOPE_LAYER = 1    /* one selection per sequence from every selected head of the layer
+                              (the form Sec. 3.3 states); every KV head keeps those positions */
+} ckv_scope;
 
 typedef enum ckv_pool_type { CKV_POOL_MAX = 0, CKV_POOL_AVG = 1 } ckv_pool_type;
 
@@ -92,12 +102,15 @@ typedef struct ckv_config {
     int32_t pool_type;     /* ckv_pool_type: max ignores padding; avg counts zero padding and
                               divides by pool_kernel */
     int32_t head_order;    /* ckv_head_order */
+    int32_t scope;         /* ckv_scope; n_vec = num_kv_heads (CKV_SCOPE_KV_HEAD) or 1
+                              (CKV_SCOPE_LAYER) selections per sequence */
     float softmax_scale;   /* scale of q.k; 0 selects 1/sqrt(head_dim) */
     int32_t max_ctas;      /* SMs one call's scoring kernel may occupy; 0 = all.  Callers that
                               run several layers concurrently on different streams give each
                               call a share, so the calls' kernels can be resident together. */
-    const uint8_t* head_mask; /* host [num_layers * num_q_heads]; non-zero = selected.  Every
-                                 KV group of a layer needs at least one selected head. */
+    const uint8_t* head_mask; /* host [num_layers * num_q_heads]; non-zero = selected.  With
+                                 CKV_SCOPE_KV_HEAD every KV group of a layer needs at least one
+                                 selected head; with CKV_SCOPE_LAYER the layer needs one. */
     const int32_t* budgets;   /* host [num_layers]; kept tokens per KV head, window included,
                                  >= window */
 } ckv_config;
@@ -137,14 +150,16 @@ CKV_API ckv_status ckv_score_window(const ckv_config* cfg, int32_t layer, const 
                             size_t workspace_bytes, ckv_stream stream);
 
 /* Step 2 (Sec. 3.3 token-axis smoothing; App. A sizes): pooled[g, cu[s]+j] for
- * j < L_s - w from the scores of group g's selected heads, in cfg->head_order; 0 at window
- * positions.  Pooling runs over the candidate range only (window scores never enter it). */
+ * j < L_s - w from the scores of selection g's heads (group g's selected heads, or every
+ * selected head of the layer with CKV_SCOPE_LAYER), in cfg->head_order; 0 at window positions.
+ * Pooling runs over the candidate range only (window scores never enter it). */
 CKV_API ckv_status ckv_pool(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
                     const float* scores, float* pooled, ckv_stream stream);
 
 /* Step 3 (Sec. 3.3, top-N selection):
- * per (sequence, KV head), the B_l - w largest pooled candidates (ties: lower position first)
- * followed by the window positions, ascending; every position when L_s <= B_l.  Writes idx
+ * per (sequence, selection), the B_l - w largest pooled candidates (ties: lower position
+ * first) followed by the window positions, ascending; every position when L_s <= B_l.  Writes
+ * idx for the KV heads the selection serves (its own, or all of them with CKV_SCOPE_LAYER)
  * and cu_keep_dev[S+1] (device copy of ckv_keep_lengths). */
 CKV_API ckv_status ckv_select_topk(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
                            const float* pooled, int32_t* idx, int32_t* cu_keep_dev,

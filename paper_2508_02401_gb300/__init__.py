@@ -19,9 +19,11 @@ __all__ = [
     "ckv_workspace_size", "ckv_keep_lengths", "ckv_score_window", "ckv_pool", "ckv_select_topk",
     "ckv_gather_compact", "ckv_compress_layer", "ckv_read_device_status", "ckv_status_string",
     "ckv_abi_version", "ckv_score_window_static", "POOL_MAX", "POOL_AVG", "POOL_THEN_SUM", "SUM_THEN_POOL",
+    "SCOPE_KV_HEAD", "SCOPE_LAYER", "ckv_layer_error_scores", "ckv_allocate_budgets",
 ]
 
 POOL_MAX, POOL_AVG = 0, 1
+SCOPE_KV_HEAD, SCOPE_LAYER = 0, 1
 POOL_THEN_SUM, SUM_THEN_POOL = 0, 1
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _lib = None
@@ -44,7 +46,8 @@ _STATUS = {0: "CKV_OK", 1: "CKV_ERR_INVALID_ARG", 2: "CKV_ERR_UNSUPPORTED", 3: "
 class _Config(C.Structure):
     _fields_ = [("num_layers", C.c_int32), ("num_q_heads", C.c_int32), ("num_kv_heads", C.c_int32),
                 ("head_dim", C.c_int32), ("window", C.c_int32), ("pool_kernel", C.c_int32),
-                ("pool_type", C.c_int32), ("head_order", C.c_int32), ("softmax_scale", C.c_float),
+                ("pool_type", C.c_int32), ("head_order", C.c_int32), ("scope", C.c_int32),
+                ("softmax_scale", C.c_float),
                 ("max_ctas", C.c_int32), ("head_mask", C.c_void_p), ("budgets", C.c_void_p)]
 
 
@@ -109,13 +112,14 @@ class Config:
     softmax_scale: float = 0.0
     head_dim: int = 128
     max_ctas: int = 0       # SMs one call's scoring kernel may occupy (0 = all)
+    scope: int = SCOPE_KV_HEAD  # SCOPE_LAYER: one selection per sequence for all KV heads
 
     def __post_init__(self):
         self.head_mask = np.ascontiguousarray(self.head_mask, dtype=np.uint8)
         self.budgets = np.ascontiguousarray(self.budgets, dtype=np.int32)
         self._c = _Config(self.num_layers, self.num_q_heads, self.num_kv_heads, self.head_dim,
                           self.window, self.pool_kernel, self.pool_type, self.head_order,
-                          self.softmax_scale, self.max_ctas, self.head_mask.ctypes.data,
+                          self.scope, self.softmax_scale, self.max_ctas, self.head_mask.ctypes.data,
                           self.budgets.ctypes.data)
 
     @classmethod
@@ -124,9 +128,15 @@ class Config:
                   num_kv_heads=wl.num_kv_heads, window=wl.window, pool_kernel=wl.pool_kernel,
                   pool_type=POOL_MAX if wl.pool_type == "max" else POOL_AVG,
                   head_order=POOL_THEN_SUM if wl.head_order == "pool_then_sum" else SUM_THEN_POOL,
-                  head_mask=wl.head_mask(), budgets=wl.budgets(), head_dim=wl.head_dim)
+                  head_mask=wl.head_mask(), budgets=wl.budgets(), head_dim=wl.head_dim,
+                  scope=SCOPE_LAYER if getattr(wl, "scope", "kv_head") == "layer" else SCOPE_KV_HEAD)
         kw.update(overrides)
         return cls(**kw)
+
+    @property
+    def num_vectors(self) -> int:
+        """Selections per sequence: the rows of the pooled scores."""
+        return 1 if self.scope == SCOPE_LAYER else self.num_kv_heads
 
     @property
     def ref(self):

@@ -43,6 +43,8 @@ size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 struct Plan {
     int Hq = 0, Hkv = 0, G = 0, w = 0, w_pad = 0, n_cols = 0, hpb = 0, budget = 0, max_ctas = 0;
     int n_sel = 0, nb = 0;
+    int scope = CKV_SCOPE_KV_HEAD, n_vec = 0;  // selections per sequence: H_kv or 1
+    // group_first: first score row of each selection's heads (n_vec + 1 entries)
     float scale = 0.f;
     std::vector<int> sel_heads, batch_group, batch_first, batch_nheads, group_first;
 };
@@ -74,6 +76,8 @@ ckv_status check_config(const ckv_config* cfg) {
     if (!(cfg->softmax_scale >= 0.f) || !isfinite(cfg->softmax_scale))
         return fail(CKV_ERR_INVALID_ARG, "softmax_scale must be finite and >= 0");
     if (cfg->max_ctas < 0) return fail(CKV_ERR_INVALID_ARG, "max_ctas %d < 0", cfg->max_ctas);
+    if (cfg->scope != CKV_SCOPE_KV_HEAD && cfg->scope != CKV_SCOPE_LAYER)
+        return fail(CKV_ERR_INVALID_ARG, "scope %d", cfg->scope);
     if (!cfg->head_mask || !cfg->budgets)
         return fail(CKV_ERR_INVALID_ARG, "head_mask and budgets must be host pointers");
     return CKV_OK;
@@ -98,14 +102,16 @@ ckv_status make_plan(const ckv_config* cfg, int32_t layer, Plan& pl) {
     while (pl.w_pad < pl.w) pl.w_pad *= 2;
     pl.hpb = kMaxCols / pl.w_pad;
     const uint8_t* mask = cfg->head_mask + static_cast<size_t>(layer) * pl.Hq;
-    pl.group_first.assign(pl.Hkv + 1, 0);
+    pl.scope = cfg->scope;
+    pl.n_vec = pl.scope == CKV_SCOPE_LAYER ? 1 : pl.Hkv;
+    pl.group_first.assign(pl.n_vec + 1, 0);
     int max_heads = 0;
     for (int g = 0; g < pl.Hkv; ++g) {
-        pl.group_first[g] = pl.n_sel;
+        if (pl.scope == CKV_SCOPE_KV_HEAD) pl.group_first[g] = pl.n_sel;
         std::vector<int> heads;
         for (int h = g * pl.G; h < (g + 1) * pl.G; ++h)
             if (mask[h]) heads.push_back(h);
-        if (heads.empty())
+        if (heads.empty() && pl.scope == CKV_SCOPE_KV_HEAD)
             return fail(CKV_ERR_INVALID_ARG, "KV group %d of layer %d has no selected head", g, layer);
         for (size_t i = 0; i < heads.size(); i += pl.hpb) {
             const int n = std::min<int>(pl.hpb, static_cast<int>(heads.size() - i));
@@ -117,7 +123,8 @@ ckv_status make_plan(const ckv_config* cfg, int32_t layer, Plan& pl) {
         for (int h : heads) pl.sel_heads.push_back(h);
         pl.n_sel += static_cast<int>(heads.size());
     }
-    pl.group_first[pl.Hkv] = pl.n_sel;
+    if (pl.n_sel == 0) return fail(CKV_ERR_INVALID_ARG, "layer %d has no selected head", layer);
+    pl.group_first[pl.n_vec] = pl.n_sel;  // per layer: rows [0, n_sel) form one selection
     pl.nb = static_cast<int>(pl.batch_group.size());
     if (pl.nb > kMaxBatches) return fail(CKV_ERR_UNSUPPORTED, "too many head batches (%d)", pl.nb);
     pl.n_cols = (max_heads * pl.w_pad <= 32) ? 32 : 64;
@@ -273,7 +280,7 @@ int max_seqlen(const ckv_batch* b) {
 
 WsLayout ws_layout(const Plan& pl, const ckv_batch* b, int T) {
     WsLayout l;
-    const size_t units = static_cast<size_t>(b->num_seqs) * pl.Hkv;
+    const size_t units = static_cast<size_t>(b->num_seqs) * pl.n_vec;
     l.max_chunks = select_chunks(max_seqlen(b));
     size_t off = round_up(sizeof(WsHeader), kWsAlign);
     l.partials = off;
@@ -283,7 +290,7 @@ WsLayout ws_layout(const Plan& pl, const ckv_batch* b, int T) {
     l.scores = off;
     off = round_up(off + static_cast<size_t>(pl.n_sel) * T * sizeof(float), kWsAlign);
     l.pooled = off;
-    off = round_up(off + static_cast<size_t>(pl.Hkv) * T * sizeof(float), kWsAlign);
+    off = round_up(off + static_cast<size_t>(pl.n_vec) * T * sizeof(float), kWsAlign);
     l.hist = off;  // zero outside a call: the selection leaves it as it found it
     off = round_up(off + units * select_hist_ints() * sizeof(int), kWsAlign);
     l.arrivals = off;  // zero outside a call, like hist
@@ -463,6 +470,7 @@ SelectLaunch select_launch(const Plan& pl, const ckv_batch* b, int T, int T_keep
     L.skip_le = skip_le;
     L.cu_hash = seqlens_hash(b->cu_seqlens_host, b->num_seqs);
     L.group_first = pl.group_first.data();
+    L.n_vec = pl.n_vec;
     L.min_len = INT_MAX;
     L.max_len = 0;
     for (int s = 0; s < b->num_seqs; ++s) {

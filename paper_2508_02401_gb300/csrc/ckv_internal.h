@@ -74,7 +74,8 @@ struct SelectLaunch {
     int write_pooled;           // with from_scores: also store the pooled scores (zeros
                                 //   at window positions and unselected sequences)
     uint32_t cu_hash;
-    const int* group_first;     // [H_kv+1] first score row of each group
+    const int* group_first;     // [n_vec+1] first score row of each selection's heads
+    int n_vec;                  // selections per sequence: H_kv (per KV head) or 1 (per layer)
     int* hist;                  // [S*H_kv][select_hist_ints()] workspace, zero between calls
     int* arrivals;              // [S*H_kv] workspace, zero between calls
     int* chunk_start;           // [S*H_kv][max_chunks][select_hist_ints()] workspace

@@ -141,6 +141,7 @@ struct SelectParams {
     uint4* k_out;
     uint4* v_out;
     int S, T, Hkv, w, budget, T_keep, max_chunks;
+    int n_vec;             // selections per sequence: H_kv (per KV head) or 1 (per layer)
     int pool_kernel, pool_type, head_order, from_scores, write_pooled;
     uint32_t cu_hash;
     int16_t group_first[kMaxQHeads + 1];
@@ -160,14 +161,14 @@ __device__ __forceinline__ uint32_t rank_key(float f) {
 }
 
 struct UnitGeo {
-    int s, g, t0, L, P, k, keep_off, n_keep;
+    int s, g, t0, L, P, k, keep_off, n_keep;  // g: the selection (KV head, or 0 per layer)
 };
 
 // Geometry of unit (sequence s, KV head g), from the device cu_seqlens; false (and an error
 // recorded) if they are unusable.  Every thread of the block calls it.
 __device__ __forceinline__ bool unit_geo(const SelectParams& p, int unit, UnitGeo& u) {
-    u.s = unit / p.Hkv;
-    u.g = unit % p.Hkv;
+    u.s = unit / p.n_vec;
+    u.g = unit % p.n_vec;
     u.t0 = __ldg(p.cu_seqlens + u.s);
     u.L = __ldg(p.cu_seqlens + u.s + 1) - u.t0;
     int off = 0;  // kept tokens of the earlier sequences: lanes stride over them
@@ -378,13 +379,13 @@ __device__ __forceinline__ void pooled_values(const SelectParams& p, const UnitG
 // Copies the K and V rows of sequence-local positions list[0..m) to output rows
 // out_row0 + 0..m-1 of KV head g: a warp per row (16 lanes for K, 16 for V), four rows in
 // flight per warp.
-__device__ __forceinline__ void copy_rows(const SelectParams& p, const UnitGeo& u, const int* list,
-                                          int m, int out_row0) {
+__device__ __forceinline__ void copy_rows(const SelectParams& p, const UnitGeo& u, int kv,
+                                          const int* list, int m, int out_row0) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
     const int part = lane & 15;
     const uint4* src0 = (lane < 16 ? p.k : p.v) + static_cast<int64_t>(u.t0) * p.tok_stride +
-                        static_cast<int64_t>(u.g) * p.head_stride + part;
-    uint4* dst0 = (lane < 16 ? p.k_out : p.v_out) + static_cast<int64_t>(u.g) * 16 + part;
+                        static_cast<int64_t>(kv) * p.head_stride + part;
+    uint4* dst0 = (lane < 16 ? p.k_out : p.v_out) + static_cast<int64_t>(kv) * 16 + part;
     for (int e0 = warp; e0 < m; e0 += 4 * nw) {
         uint4 x[4];
 #pragma unroll
@@ -397,6 +398,19 @@ __device__ __forceinline__ void copy_rows(const SelectParams& p, const UnitGeo& 
             const int e = e0 + q * nw;
             if (e < m) dst0[static_cast<int64_t>(out_row0 + e) * p.Hkv * 16] = x[q];
         }
+    }
+}
+
+// Writes list[0..m) (sequence-local positions, in order) to the index rows at offset out_off
+// of the unit's kept tokens, and copies the K/V rows when asked, for every KV head that the
+// unit's selection serves: its own (per-KV-head scope) or all of them (per-layer scope).
+__device__ __forceinline__ void emit_kept(const SelectParams& p, const UnitGeo& u, const int* list,
+                                          int m, int out_off) {
+    const int per = p.Hkv / p.n_vec;
+    for (int kv = u.g * per; kv < (u.g + 1) * per; ++kv) {
+        int32_t* out = p.idx + static_cast<size_t>(kv) * p.T_keep + u.keep_off + out_off;
+        for (int e = threadIdx.x; e < m; e += blockDim.x) out[e] = list[e];
+        if (p.k) copy_rows(p, u, kv, list, m, u.keep_off + out_off);
     }
 }
 
@@ -417,18 +431,16 @@ __global__ void __launch_bounds__(kUnitThreads, 1) select_unit_kernel(const __gr
         p.cu_keep[u.s + 1] = u.keep_off + u.n_keep;
         if (u.s == 0) p.cu_keep[0] = 0;
     }
-    int32_t* out = p.idx + static_cast<size_t>(u.g) * p.T_keep + u.keep_off;
     float* pooled = p.pooled + static_cast<size_t>(u.g) * p.T + u.t0;
     int* list = reinterpret_cast<int*>(ust);
     const bool zeros = p.from_scores && p.write_pooled;
     if (u.L <= p.budget) {  // kept whole; its pooled scores read as 0
         for (int e = tid; e < u.L; e += NT) {
-            out[e] = e;
             list[e] = e;
             if (zeros) pooled[e] = 0.f;
         }
         __syncthreads();
-        if (p.k) copy_rows(p, u, list, u.L, u.keep_off);
+        emit_kept(p, u, list, u.L, 0);
         return;
     }
     const int P = u.P, k = u.k;
@@ -520,17 +532,13 @@ __global__ void __launch_bounds__(kUnitThreads, 1) select_unit_kernel(const __gr
 #pragma unroll
     for (int i = 0; i < PER; ++i) {
         if ((taken >> i) & 1u) {
-            out[rk] = jb + i;
             list[rk] = jb + i;
             ++rk;
         }
     }
-    for (int i = tid; i < p.w; i += NT) {
-        out[k + i] = P + i;
-        list[k + i] = P + i;
-    }
+    for (int i = tid; i < p.w; i += NT) list[k + i] = P + i;
     __syncthreads();
-    if (p.k) copy_rows(p, u, list, p.budget, u.keep_off);
+    emit_kept(p, u, list, p.budget, 0);
 }
 
 // ------------------------------------------------------------------ longer units, in chunks
@@ -844,26 +852,19 @@ __global__ void __launch_bounds__(kSelThreads) compact_kernel(const __grid_const
         p.cu_keep[u.s + 1] = u.keep_off + u.n_keep;
         if (u.s == 0) p.cu_keep[0] = 0;
     }
-    int32_t* out = p.idx + static_cast<size_t>(u.g) * p.T_keep + u.keep_off;
     const int j0 = c * kChunk;
     if (u.L <= p.budget) {  // kept whole
         const int m = max(0, min(u.L, j0 + kChunk) - j0);
-        for (int e = tid; e < m; e += kSelThreads) {
-            out[j0 + e] = j0 + e;
-            list[e] = j0 + e;
-        }
+        for (int e = tid; e < m; e += kSelThreads) list[e] = j0 + e;
         __syncthreads();
-        if (p.k) copy_rows(p, u, list, m, u.keep_off + j0);
+        emit_kept(p, u, list, m, j0);
         return;
     }
     const int P = u.P, k = u.k;
     if (c == 0) {  // the window closes the list
-        for (int i = tid; i < p.w; i += kSelThreads) {
-            out[k + i] = P + i;
-            list[i] = P + i;
-        }
+        for (int i = tid; i < p.w; i += kSelThreads) list[i] = P + i;
         __syncthreads();
-        if (p.k) copy_rows(p, u, list, p.w, u.keep_off + k);
+        emit_kept(p, u, list, p.w, k);
         __syncthreads();
     }
     if (j0 >= P) return;
@@ -909,15 +910,11 @@ __global__ void __launch_bounds__(kSelThreads) compact_kernel(const __grid_const
     const unsigned lt = (1u << lane) - 1u;
 #pragma unroll
     for (int q = 0; q < kIt; ++q) {
-        if ((bal[q] >> lane) & 1u) {
-            const int e = r + __popc(bal[q] & lt);
-            out[base + e] = js + q * 32;
-            list[e] = js + q * 32;
-        }
+        if ((bal[q] >> lane) & 1u) list[r + __popc(bal[q] & lt)] = js + q * 32;
         r += __popc(bal[q]);
     }
     __syncthreads();
-    if (p.k) copy_rows(p, u, list, tot, u.keep_off + base);
+    emit_kept(p, u, list, tot, base);
 }
 struct GatherParams {
     const uint4* k;
@@ -970,9 +967,9 @@ cudaError_t launch_pool(const SelectLaunch& L, cudaStream_t stream) {
     p.pool_type = L.pool_type;
     p.head_order = L.head_order;
     p.skip_le = L.skip_le;
-    for (int g = 0; g <= L.Hkv; ++g) p.group_first[g] = static_cast<int16_t>(L.group_first[g]);
+    for (int g = 0; g <= L.n_vec; ++g) p.group_first[g] = static_cast<int16_t>(L.group_first[g]);
     if (L.T == 0) return cudaSuccess;
-    dim3 grid((L.T + 255) / 256, L.Hkv);
+    dim3 grid((L.T + 255) / 256, L.n_vec);
     pool_kernel<<<grid, 256, 0, stream>>>(p);
     return cudaGetLastError();
 }
@@ -1007,14 +1004,15 @@ cudaError_t launch_select(const SelectLaunch& L, cudaStream_t stream) {
     p.budget = L.budget;
     p.T_keep = L.T_keep;
     p.max_chunks = L.max_chunks;
+    p.n_vec = L.n_vec;
     p.pool_kernel = L.pool_kernel;
     p.pool_type = L.pool_type;
     p.head_order = L.head_order;
     p.from_scores = L.from_scores;
     p.write_pooled = L.write_pooled;
     p.cu_hash = L.cu_hash;
-    for (int g = 0; g <= L.Hkv; ++g) p.group_first[g] = static_cast<int16_t>(L.group_first[g]);
-    const int units = L.S * L.Hkv;
+    for (int g = 0; g <= L.n_vec; ++g) p.group_first[g] = static_cast<int16_t>(L.group_first[g]);
+    const int units = L.S * L.n_vec;
     if (units == 0 || L.max_chunks == 0) return cudaSuccess;
     if (L.max_chunks > 65535) return cudaErrorInvalidConfiguration;
     const size_t sel_smem = std::max(static_cast<size_t>(kSelStageSmem),

@@ -39,7 +39,7 @@ def run_gpu(wl, layer, li, cfg=None, scores=True, stream=None, check_status=True
     ws = ckv.new_workspace(cfg, layer, batch)
     idx, cu_keep_dev, k_out, v_out, cu_keep = ckv.new_outputs(cfg, layer, batch)
     T = batch.total_tokens
-    pooled = torch.full((cfg.num_kv_heads, T), float("nan"), dtype=torch.float32, device="cuda")
+    pooled = torch.full((cfg.num_vectors, T), float("nan"), dtype=torch.float32, device="cuda")
     ckv.ckv_compress_layer(cfg, layer, batch, q, k, v, idx, cu_keep_dev, k_out, v_out, ws,
                            pooled_out=pooled, stream=stream)
     out = dict(cfg=cfg, cu_keep=cu_keep)
@@ -62,7 +62,8 @@ def run_oracle(wl, layer, li, mask=None, groups=None, want_kv=True):
                                  int(wl.budgets()[layer]), wl.window, wl.pool_kernel,
                                  0 if wl.pool_type == "max" else 1,
                                  0 if wl.head_order == "pool_then_sum" else 1,
-                                 want_kv=want_kv, groups=groups)
+                                 want_kv=want_kv, groups=groups,
+                                 scope=oracle.SCOPE_LAYER if wl.scope == "layer" else oracle.SCOPE_KV_HEAD)
 
 
 def assert_close_rows(gpu, orc, rtol=SCORE_RTOL, floor=SCORE_FLOOR, what="scores"):
@@ -90,15 +91,19 @@ def check_layer(wl, layer, li, g, o, groups=None, exact_select=True):
     groups = range(wl.num_kv_heads) if groups is None else groups
     sel_rows = np.nonzero(wl.head_mask()[layer])[0]
     G = wl.group_size
+    layer_scope = wl.scope == "layer"
+    if layer_scope:  # one selection per sequence, the same positions for every KV head
+        for gi in groups:
+            np.testing.assert_array_equal(g["idx"][gi], g["idx"][0])
     for s in range(wl.num_seqs):
         t0, t1 = int(cu[s]), int(cu[s + 1])
         L = t1 - t0
         P = L - w
-        for gi in groups:
-            # scores of the group's selected heads, every position
+        for gi in groups:  # scores of the group's selected heads, every position
             if "scores" in g and L > 0:
                 rows = [i for i, h in enumerate(sel_rows) if h // G == gi]
                 assert_close_rows(g["scores"][rows, t0:t1], o["scores"][rows, t0:t1])
+        for gi in ([0] if layer_scope else groups):  # the selections
             ix = g["idx"][gi, ck[s]:ck[s + 1]]
             if L <= B:
                 np.testing.assert_array_equal(ix, np.arange(L))

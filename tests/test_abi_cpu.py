@@ -47,7 +47,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 
 def test_version_and_status_strings(lib):
-    assert ckv.ckv_abi_version() == 1
+    assert ckv.ckv_abi_version() == 2
     assert ckv.ckv_status_string(0) == "CKV_OK"
     assert ckv.ckv_status_string(3) == "CKV_ERR_WORKSPACE"
 
@@ -99,6 +99,8 @@ def _call_compress(lib, cfg, batch, layer=0, q=_P, k=_P, v=_P, ws=_P, ws_bytes=1
     (dict(budgets=np.array([16, 64], np.int32)), 1),              # budget below the window
     (dict(head_mask=np.zeros((2, 32), np.uint8)), 1),             # group without a head
     (dict(num_q_heads=512, num_kv_heads=8, head_mask=np.ones((2, 512), np.uint8)), 2),
+    (dict(scope=2), 1),
+    (dict(scope=1, head_mask=np.zeros((2, 32), np.uint8)), 1),    # layer without a head
 ])
 def test_config_errors(lib, change, expect):
     cfg = _cfg(**change)
@@ -137,3 +139,12 @@ def test_python_errors_carry_the_message(lib):
 def test_valid_call_without_a_gpu_reports_cuda_error(lib):
     rc = _call_compress(lib, _cfg(), FakeBatch([0, 4096]))
     assert rc == 4
+
+
+def test_layer_scope_accepts_groups_without_heads(lib):
+    """Per-layer selection: heads in one group only is a valid config (it gets past every host
+    check, so on a machine without a GPU the call ends in CKV_ERR_CUDA)."""
+    m = np.zeros((2, 32), np.uint8)
+    m[:, :4] = 1
+    assert _call_compress(lib, _cfg(scope=1, head_mask=m), FakeBatch([0, 4096])) in (0, 4)
+    assert _call_compress(lib, _cfg(scope=0, head_mask=m), FakeBatch([0, 4096])) == 1

@@ -51,6 +51,14 @@ FUZZ = [
     dict(seqlens=(5000,), plant="span", plant_count=32, plant_beta=4.0, plant_noise=True,
          budget_mean=64, pool_type="avg"),
     dict(seqlens=(20000,), budget_mean=600, heads_per_group=1, pool_kernel=9),
+    # one selection per layer from heads anywhere in the layer (Sec. 3.3 as stated)
+    dict(scope="layer", heads_per_layer=3, seqlens=(1000, 77, 300), budget_mean=40),
+    dict(scope="layer", heads_per_layer=4, num_q_heads=32, num_kv_heads=8, window=8,
+         pool_kernel=5, pool_type="avg", seqlens=(4096, 333), budget_mean=128),
+    dict(scope="layer", heads_per_layer=1, num_q_heads=28, num_kv_heads=4, seqlens=(20000, 3000),
+         budget_mean=300, head_order="sum_then_pool"),
+    dict(scope="layer", heads_per_layer=6, num_q_heads=32, num_kv_heads=8, window=64,
+         seqlens=(1500, 9000), budget_mean=100),
 ]
 
 
@@ -80,6 +88,7 @@ def test_single_layer_workload_full():
     ("llama8b_l32768", (0, 5), None),
     ("needle_l131072", (7,), (0, 5)),
     ("ragged_qwen7b", (0, 27), None),
+    ("paper_llama8b_l8192", (0, 17, 31), None),
 ])
 def test_full_size_workloads(name, layers, groups):
     wl = cs.workload(name)
@@ -91,6 +100,10 @@ def test_full_size_workloads(name, layers, groups):
             g["scores"] = None
             g.pop("scores")
         gu.check_layer(wl, layer, li, g, o, groups=groups)
+        if wl.plant == "tokens":  # the planted keys are kept by every KV head
+            ck = o["cu_keep"]
+            for gi in range(wl.num_kv_heads):
+                assert set(li.planted[0].tolist()) <= set(g["idx"][gi, ck[0]:ck[1]].tolist())
         if wl.plant == "span":  # the needle span is kept by every KV head
             ck = o["cu_keep"]
             for gi in range(wl.num_kv_heads):

@@ -46,8 +46,12 @@ def test_workload_recipe(name):
     wl = cs.workload(name)
     m = wl.head_mask()
     assert m.shape == (wl.num_layers, wl.num_q_heads)
-    per_group = m.reshape(wl.num_layers, wl.num_kv_heads, wl.group_size).sum(-1)
-    assert np.all(per_group == wl.heads_per_group)
+    if wl.heads_per_layer > 0:  # that many heads per layer, anywhere in the layer
+        assert np.all(m.sum(-1) == wl.heads_per_layer)
+        assert len({tuple(np.nonzero(r)[0]) for r in m}) > 1  # layers differ
+    else:
+        per_group = m.reshape(wl.num_layers, wl.num_kv_heads, wl.group_size).sum(-1)
+        assert np.all(per_group == wl.heads_per_group)
     b = wl.budgets()
     assert b.sum() == wl.num_layers * wl.budget_mean
     assert b.min() >= max(wl.budget_min, wl.window) and b.max() <= 3 * wl.budget_mean
