@@ -204,6 +204,14 @@ CKV_API ckv_status ckv_allocate_budgets(const double* scores, int32_t num_layers
                                         int64_t total_budget, int32_t min_budget,
                                         int32_t max_budget, int32_t* budgets);
 
+/* Limit, for the calls enqueued after this one, of every bounded wait in which a kernel
+ * waits on another of its roles or on another CTA: 0 restores the default (about 2 s).  When
+ * a wait runs out the kernel sets CKV_DEV status 2 (a wait gave up) in the workspace status
+ * word, lets its own copies and MMAs finish, frees its tensor memory and returns; the results
+ * of that call are then undefined, the CUDA context stays usable.  Process-wide; meant for
+ * failure detection (and its tests), not for normal use. */
+CKV_API ckv_status ckv_set_wait_limit_us(uint32_t microseconds);
+
 /* Synchronises `stream`, then returns the workspace's device status: *code = 0 if no kernel
  * recorded an error since the last reset, else the first error (1 = cu_seqlens_dev disagrees
  * with the host copy, 2 = a wait timed out, 3 = an index out of range); *detail says where.

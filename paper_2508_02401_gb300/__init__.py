@@ -82,6 +82,7 @@ def load():
         "ckv_read_device_status": ([P, P, I32, C.POINTER(I32), C.POINTER(I32)], C.c_int),
         "ckv_score_window_static": ([cfg, I32, bat, P, P, I64, I64, P, P, P], C.c_int),
         "ckv_layer_error_scores": ([P, I32, I32, P], C.c_int),
+        "ckv_set_wait_limit_us": ([C.c_uint32], C.c_int),
         "ckv_allocate_budgets": ([P, I32, I64, I32, I32, P], C.c_int),
     }
     for name, (args, res) in sigs.items():
@@ -222,6 +223,11 @@ def ckv_allocate_budgets(scores, total_budget: int, min_budget: int = 32, max_bu
     _check(load().ckv_allocate_budgets(s.ctypes.data, L, int(total_budget), int(min_budget),
                                        int(max_budget), out.ctypes.data), "ckv_allocate_budgets")
     return out
+
+
+def ckv_set_wait_limit_us(microseconds: int):
+    """Limit of the kernels' bounded waits for later calls (0 = the default, about 2 s)."""
+    _check(load().ckv_set_wait_limit_us(int(microseconds)), "ckv_set_wait_limit_us")
 
 
 def ckv_score_window(cfg, layer, batch, q_win, k, scores, workspace, stream=None,

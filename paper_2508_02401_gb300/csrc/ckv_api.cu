@@ -16,6 +16,8 @@
 
 #include <limits.h>
 
+#include <atomic>
+
 namespace ckv {
 namespace {
 
@@ -483,6 +485,11 @@ SelectLaunch select_launch(const Plan& pl, const ckv_batch* b, int T, int T_keep
 
 }  // namespace
 
+// Limit of the kernels' bounded waits on other roles and other CTAs (ckv_set_wait_limit_us).
+std::atomic<long long> g_wait_cycles{kWaitTimeoutCycles};
+
+long long wait_limit_cycles() { return g_wait_cycles.load(std::memory_order_relaxed); }
+
 // The last-error message for the other translation units (host-only entry points).
 ckv_status set_error(ckv_status st, const char* fmt, ...) {
     va_list ap;
@@ -498,6 +505,23 @@ using namespace ckv;
 extern "C" {
 
 int32_t ckv_abi_version(void) { return CKV_ABI_VERSION; }
+
+ckv_status ckv_set_wait_limit_us(uint32_t microseconds) {
+    long long cycles = kWaitTimeoutCycles;
+    if (microseconds > 0) {
+        int khz = 0;  // SM clock; 2 GHz if there is no device to ask
+        int dev = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&khz, cudaDevAttrClockRate, dev) != cudaSuccess || khz <= 0) {
+            cudaGetLastError();
+            khz = 2000000;
+        }
+        cycles = static_cast<long long>(microseconds) * khz / 1000;
+        if (cycles < 1) cycles = 1;
+    }
+    g_wait_cycles.store(cycles, std::memory_order_relaxed);
+    return CKV_OK;
+}
 
 const char* ckv_status_string(ckv_status s) {
     switch (s) {

@@ -105,18 +105,19 @@ __device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
 }
 
 // Waits for the phase with the given parity to complete.  Gives up (returns false) after
-// kWaitTimeoutCycles or as soon as *abort is set by another thread of the block (both are
+// `limit` cycles or as soon as *abort is set by another thread of the block (both are
 // checked every 64 polls).  Between polls the warp sleeps for `backoff_ns`, so waiting warps
 // leave the issue slots of their scheduler to the warps doing work.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort,
-                                          uint32_t backoff_ns = 32) {
+                                          uint32_t backoff_ns = 32,
+                                          long long limit = kWaitTimeoutCycles) {
     if (mbar_try_wait(bar, parity)) return true;
     const long long t0 = clock64();
 #pragma unroll 1
     for (uint32_t it = 1;; ++it) {
         __nanosleep(backoff_ns);
         if (mbar_try_wait(bar, parity)) return true;
-        if ((it & 63u) == 0u && (*abort || clock64() - t0 > kWaitTimeoutCycles)) return false;
+        if ((it & 63u) == 0u && (*abort || clock64() - t0 > limit)) return false;
     }
 }
 

@@ -59,6 +59,7 @@ struct ScoreLaunch {
     std::vector<ScoreSlice> slices;
 };
 cudaError_t launch_score(const ScoreLaunch& L, cudaStream_t stream);
+long long wait_limit_cycles();  // the current limit of a bounded wait, in SM clock cycles
 
 struct SelectLaunch {
     const float* scores;        // [n_sel, T]

@@ -65,6 +65,7 @@ struct alignas(128) ScoreParams {
     int S, T, Hq, w, n_rounds, n_items, n_units;
     uint32_t cu_hash;
     float sl2;                     // softmax scale * log2(e)
+    long long wait_cycles;         // limit of a bounded wait (ckv_set_wait_limit_us)
     int16_t batch_group[kMaxBatches];   // KV head of each head batch
     int16_t batch_first[kMaxBatches];   // score row of the batch's first head
     int16_t batch_nheads[kMaxBatches];  // heads in the batch
@@ -143,9 +144,10 @@ __device__ __forceinline__ void setmaxnreg_dec() {
 
 // A barrier of one epilogue warpgroup built on an mbarrier of 128 arrivals, so that the wait
 // is bounded like every other wait of the kernel.
-__device__ __forceinline__ bool group_sync(uint64_t* bar, uint32_t& phase, volatile int* abort) {
+__device__ __forceinline__ bool group_sync(uint64_t* bar, uint32_t& phase, volatile int* abort,
+                                           long long limit) {
     mbar_arrive(bar);
-    const bool ok = mbar_wait(bar, phase, abort);
+    const bool ok = mbar_wait(bar, phase, abort, 32, limit);
     phase ^= 1;
     return ok;
 }
@@ -328,6 +330,9 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
     // the pass-2 warpgroup keeps 128 (128*56 + 256*160 + 128*128 = 64512).
     const int R = p.n_rounds;
     const int G = gridDim.x;
+    // Limit of the waits on other roles and other CTAs (the waits for this block's own copies
+    // and MMAs before it exits keep the long default, whatever this is).
+    const long long lim = p.wait_cycles;
     auto item_of = [&](int r) -> const ScoreItem& { return p.items[r * G + blockIdx.x]; };
 
     if (warp < kWarpA) {
@@ -353,7 +358,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                     const long long t0 = clock64();
                     for (uint32_t k = 1; *issued <= it; ++k) {
                         __nanosleep(64);
-                        if ((k & 63u) == 0u && (*abort || clock64() - t0 > kWaitTimeoutCycles)) {
+                        if ((k & 63u) == 0u && (*abort || clock64() - t0 > lim)) {
                             ok = false;
                             break;
                         }
@@ -368,7 +373,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                     // (the next sequence's, or zeros past the end) and head slots past the
                     // batch's heads land in columns that the epilogues mask out.
                     const int qb = it % kQBufs;
-                    if (!mbar_wait(&q_empty[qb], ((it / kQBufs) & 1) ^ 1, abort)) {
+                    if (!mbar_wait(&q_empty[qb], ((it / kQBufs) & 1) ^ 1, abort, 32, lim)) {
                         ok = false;
                         break;
                     }
@@ -384,7 +389,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                 }
                 for (int jt = 0; ok && jt < n; ++jt, ++use) {
                     const int s = use % nslots;
-                    if (!mbar_wait(&freed[s], ((use / nslots) & 1) ^ 1, abort)) {
+                    if (!mbar_wait(&freed[s], ((use / nslots) & 1) ^ 1, abort, 32, lim)) {
                         ok = false;
                         break;
                     }
@@ -489,7 +494,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                     // Nothing ready: back off (32 ns doubling to 256 ns), so that the polls do
                     // not take issue slots from the epilogue warps of this SM sub-partition.
                     __nanosleep(32u << (idle < 3u ? idle : 3u));
-                    if ((++idle & 15u) == 0u && (*abort || clock64() - t0 > kWaitTimeoutCycles)) {
+                    if ((++idle & 15u) == 0u && (*abort || clock64() - t0 > lim)) {
                         ok = false;
                         break;
                     }
@@ -514,7 +519,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             for (int r = 0; r < R; ++r) {
                 const ScoreItem& I = item_of(r);
                 if (I.ntiles == 0) continue;
-                if (!mbar_wait(&pub_full[it & 1], (it >> 1) & 1, abort, 64)) {
+                if (!mbar_wait(&pub_full[it & 1], (it >> 1) & 1, abort, 64, lim)) {
                     *abort = 1;
                     record_error(p.status, kDevTimeout, 17);
                     break;
@@ -563,7 +568,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                 }
                 for (int jt = 0; jt < n; ++jt, ++a_it) {
                     const int acc = a_it % kAcc;
-                    if (!mbar_wait(&a_full[acc], (a_it / kAcc) & 1, abort)) {
+                    if (!mbar_wait(&a_full[acc], (a_it / kAcc) & 1, abort, 32, lim)) {
                         ok = false;
                         break;
                     }
@@ -626,7 +631,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                 transpose_reduce<kCols>(sm_, m, lane);  // lane l: column l
                 float2* red = red_a[a_item & 1][wg];
                 red[eq * 32 + lane] = make_float2(m[0], sm_[0]);
-                if (!group_sync(gbar, gphase, abort)) {
+                if (!group_sync(gbar, gphase, abort, lim)) {
                     ok = false;
                     break;
                 }
@@ -641,7 +646,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                         S += x.y * ex2_approx(x.x - M);
                     }
                     // the publisher has released the item two back that used this phase
-                    if (!mbar_wait(&pub_empty[a_item & 1], ((a_item >> 1) & 1) ^ 1, abort)) {
+                    if (!mbar_wait(&pub_empty[a_item & 1], ((a_item >> 1) & 1) ^ 1, abort, 32, lim)) {
                         ok = false;
                         break;
                     }
@@ -688,7 +693,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                 bool got = true;
                 for (uint32_t k = 1; ld_acquire(p.counters + I.unit) < target; ++k) {
                     __nanosleep(64);
-                    if ((k & 63u) == 0u && (*abort || clock64() - t0 > kWaitTimeoutCycles)) {
+                    if ((k & 63u) == 0u && (*abort || clock64() - t0 > lim)) {
                         got = false;
                         break;
                     }
@@ -696,7 +701,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                 __threadfence();
                 verdict[0] = got ? 1 : 0;
             }
-            if (!group_sync(gbar, gphase, abort) || verdict[0] == 0) {
+            if (!group_sync(gbar, gphase, abort, lim) || verdict[0] == 0) {
                 ok = false;
                 break;
             }
@@ -733,7 +738,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                 }
                 red_b[part * N + 2 * c2] = make_float2(M0, S0);
                 red_b[part * N + 2 * c2 + 1] = make_float2(M1, S1);
-                if (!group_sync(gbar, gphase, abort)) {
+                if (!group_sync(gbar, gphase, abort, lim)) {
                     ok = false;
                     break;
                 }
@@ -748,7 +753,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                     }
                     lse_s[wtid] = M2 + lg2_approx(S2);
                 }
-                if (!group_sync(gbar, gphase, abort)) {
+                if (!group_sync(gbar, gphase, abort, lim)) {
                     ok = false;
                     break;
                 }
@@ -756,7 +761,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             // ---------------------------------------------------- the item's tiles
             for (int jt = 0; jt < n; ++jt, ++b_it) {
                 const int acc = b_it % kAcc;
-                if (!mbar_wait(&b_full[acc], (b_it / kAcc) & 1, abort)) {
+                if (!mbar_wait(&b_full[acc], (b_it / kAcc) & 1, abort, 32, lim)) {
                     ok = false;
                     break;
                 }
@@ -891,6 +896,7 @@ cudaError_t launch_score(const ScoreLaunch& L, cudaStream_t stream) {
     p.w = L.w;
     p.cu_hash = L.cu_hash;
     p.sl2 = L.softmax_scale * 1.4426950408889634f;
+    p.wait_cycles = wait_limit_cycles();
     for (int b = 0; b < L.nb; ++b) {
         p.batch_group[b] = static_cast<int16_t>(L.batch_group[b]);
         p.batch_first[b] = static_cast<int16_t>(L.batch_first[b]);

@@ -1,0 +1,44 @@
+"""Failure detection on the GPU without a fault: a bounded wait that runs out is reported in
+the workspace status word, the kernel returns, and the CUDA context stays usable.
+
+The wait limit is shortened to 1 us with ckv_set_wait_limit_us; with 4 CTAs for a 40k-token
+sequence every work item is ~80 key tiles long, so the cross-CTA exchange of each round waits
+far longer than that and gives up.  No flag, barrier or check is removed: every wait still
+ends, only sooner.
+"""
+import pytest
+import torch
+
+import ckv_synth as cs
+import oracle
+import paper_2508_02401_gb300 as ckv
+from tests import gpu_util as gu
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a GPU")
+    ckv.load()
+    oracle.build()
+
+
+def test_a_wait_that_runs_out_is_reported_and_the_context_stays_usable():
+    wl = cs.Workload(name="timeout", num_layers=1, num_q_heads=32, num_kv_heads=8,
+                     seqlens=(40000, 9000), window=32, heads_per_group=2, budget_mean=300,
+                     budget_uniform=True, outlier_channels=8, seed=5)
+    li = wl.layer(0)
+    cfg = ckv.Config.from_workload(wl, max_ctas=4)
+    ckv.ckv_set_wait_limit_us(1)
+    try:
+        g = gu.run_gpu(wl, 0, li, cfg=cfg, scores=False, check_status=False)
+    finally:
+        ckv.ckv_set_wait_limit_us(0)
+    assert g["status"][0] == 2, g["status"]  # a wait gave up
+    # the same call with the default limit: status clean, results right
+    g = gu.run_gpu(wl, 0, li, cfg=cfg)
+    o = gu.run_oracle(wl, 0, li, groups=(0, 5), want_kv=False)
+    g.pop("scores")
+    gu.check_layer(wl, 0, li, g, o, groups=(0, 5))
