@@ -57,6 +57,9 @@ def _args():
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--layers", type=int, default=0, help="use only the first N layers (0 = all)")
     ap.add_argument("--breakdown", action="store_true", help="per-stage times on stderr")
+    ap.add_argument("--score-path", choices=("auto", "resident", "reload"), default="auto",
+                    help="scoring kernel: logits kept in TMEM, K re-read in pass 2, or the "
+                         "library's choice")
     ap.add_argument("--streams", type=int, default=16,
                     help="layers are issued round-robin on this many streams (one workspace each); "
                          "each call is capped at SMs / streams CTAs")
@@ -159,7 +162,8 @@ def run_ours(args):
     wl = cs.workload(args.workload)
     if args.layers:
         wl = wl.with_(num_layers=args.layers)
-    cfg = ckv.Config.from_workload(wl)
+    path = {"auto": ckv.SCORE_AUTO, "resident": ckv.SCORE_RESIDENT, "reload": ckv.SCORE_RELOAD}[args.score_path]
+    cfg = ckv.Config.from_workload(wl, score_path=path)
     batch = ckv.Batch(wl.cu_seqlens(), device=f"cuda:{local}")
     T, Hkv, nl = wl.total_tokens, wl.num_kv_heads, wl.num_layers
 
@@ -178,7 +182,7 @@ def run_ours(args):
     nstreams = max(1, args.streams)
     if nstreams > 1:  # each stream's calls may occupy an equal share of the SMs
         sms = torch.cuda.get_device_properties(local).multi_processor_count
-        cfg = ckv.Config.from_workload(wl, max_ctas=sms // nstreams)
+        cfg = ckv.Config.from_workload(wl, max_ctas=sms // nstreams, score_path=path)
     wss = [torch.zeros(ws_bytes, dtype=torch.uint8, device="cuda") for _ in range(nstreams)]
     ws = wss[0]
     stream = torch.cuda.Stream()

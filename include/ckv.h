@@ -53,7 +53,7 @@
 extern "C" {
 #endif
 
-#define CKV_ABI_VERSION 2
+#define CKV_ABI_VERSION 3
 
 #if defined(__GNUC__)
 #define CKV_API __attribute__((visibility("default")))
@@ -79,6 +79,18 @@ typedef enum ckv_scope {
     CKV_SCOPE_LAYER = 1    /* one selection per sequence from every selected head of the layer
                               (the form Sec. 3.3 states); every KV head keeps those positions */
 } ckv_scope;
+
+/* Which scoring kernel runs the two passes over the keys (same scores either way). */
+typedef enum ckv_score_path {
+    CKV_SCORE_AUTO = 0,     /* resident when it fits and N = 32 (see below), otherwise reload */
+    CKV_SCORE_RESIDENT = 1, /* each key tile is read and multiplied once; pass 1 keeps its
+                               exponentials in tensor memory and pass 2 rescales them.  Needs
+                               every sequence's key tiles to fit one round of work items of at
+                               most 512 / N tiles (N = 32 or 64 window-row columns of a head
+                               batch); CKV_ERR_UNSUPPORTED if not */
+    CKV_SCORE_RELOAD = 2    /* pass 2 reads each key tile again (from L2 while it is there) and
+                               multiplies it again; no limit on the sequence length */
+} ckv_score_path;
 
 typedef enum ckv_pool_type { CKV_POOL_MAX = 0, CKV_POOL_AVG = 1 } ckv_pool_type;
 
@@ -108,6 +120,7 @@ typedef struct ckv_config {
     int32_t max_ctas;      /* SMs one call's scoring kernel may occupy; 0 = all.  Callers that
                               run several layers concurrently on different streams give each
                               call a share, so the calls' kernels can be resident together. */
+    int32_t score_path;    /* ckv_score_path */
     const uint8_t* head_mask; /* host [num_layers * num_q_heads]; non-zero = selected.  With
                                  CKV_SCOPE_KV_HEAD every KV group of a layer needs at least one
                                  selected head; with CKV_SCOPE_LAYER the layer needs one. */

@@ -25,6 +25,7 @@ __all__ = [
 POOL_MAX, POOL_AVG = 0, 1
 SCOPE_KV_HEAD, SCOPE_LAYER = 0, 1
 POOL_THEN_SUM, SUM_THEN_POOL = 0, 1
+SCORE_AUTO, SCORE_RESIDENT, SCORE_RELOAD = 0, 1, 2
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _lib = None
 
@@ -48,7 +49,8 @@ class _Config(C.Structure):
                 ("head_dim", C.c_int32), ("window", C.c_int32), ("pool_kernel", C.c_int32),
                 ("pool_type", C.c_int32), ("head_order", C.c_int32), ("scope", C.c_int32),
                 ("softmax_scale", C.c_float),
-                ("max_ctas", C.c_int32), ("head_mask", C.c_void_p), ("budgets", C.c_void_p)]
+                ("max_ctas", C.c_int32), ("score_path", C.c_int32), ("head_mask", C.c_void_p),
+                ("budgets", C.c_void_p)]
 
 
 class _Batch(C.Structure):
@@ -114,14 +116,15 @@ class Config:
     head_dim: int = 128
     max_ctas: int = 0       # SMs one call's scoring kernel may occupy (0 = all)
     scope: int = SCOPE_KV_HEAD  # SCOPE_LAYER: one selection per sequence for all KV heads
+    score_path: int = 0     # SCORE_AUTO / SCORE_RESIDENT / SCORE_RELOAD (the scoring kernel)
 
     def __post_init__(self):
         self.head_mask = np.ascontiguousarray(self.head_mask, dtype=np.uint8)
         self.budgets = np.ascontiguousarray(self.budgets, dtype=np.int32)
         self._c = _Config(self.num_layers, self.num_q_heads, self.num_kv_heads, self.head_dim,
                           self.window, self.pool_kernel, self.pool_type, self.head_order,
-                          self.scope, self.softmax_scale, self.max_ctas, self.head_mask.ctypes.data,
-                          self.budgets.ctypes.data)
+                          self.scope, self.softmax_scale, self.max_ctas, self.score_path,
+                          self.head_mask.ctypes.data, self.budgets.ctypes.data)
 
     @classmethod
     def from_workload(cls, wl, **overrides):

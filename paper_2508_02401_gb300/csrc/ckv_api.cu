@@ -44,6 +44,7 @@ size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 // Everything a call needs to know about one layer of the config.
 struct Plan {
     int Hq = 0, Hkv = 0, G = 0, w = 0, w_pad = 0, n_cols = 0, hpb = 0, budget = 0, max_ctas = 0;
+    int score_path = CKV_SCORE_AUTO;
     int n_sel = 0, nb = 0;
     int scope = CKV_SCOPE_KV_HEAD, n_vec = 0;  // selections per sequence: H_kv or 1
     // group_first: first score row of each selection's heads (n_vec + 1 entries)
@@ -78,6 +79,8 @@ ckv_status check_config(const ckv_config* cfg) {
     if (!(cfg->softmax_scale >= 0.f) || !isfinite(cfg->softmax_scale))
         return fail(CKV_ERR_INVALID_ARG, "softmax_scale must be finite and >= 0");
     if (cfg->max_ctas < 0) return fail(CKV_ERR_INVALID_ARG, "max_ctas %d < 0", cfg->max_ctas);
+    if (cfg->score_path < CKV_SCORE_AUTO || cfg->score_path > CKV_SCORE_RELOAD)
+        return fail(CKV_ERR_INVALID_ARG, "score_path %d", cfg->score_path);
     if (cfg->scope != CKV_SCOPE_KV_HEAD && cfg->scope != CKV_SCOPE_LAYER)
         return fail(CKV_ERR_INVALID_ARG, "scope %d", cfg->scope);
     if (!cfg->head_mask || !cfg->budgets)
@@ -96,6 +99,7 @@ ckv_status make_plan(const ckv_config* cfg, int32_t layer, Plan& pl) {
     pl.w = cfg->window;
     pl.budget = cfg->budgets[layer];
     pl.max_ctas = cfg->max_ctas;
+    pl.score_path = cfg->score_path;
     if (pl.budget < pl.w)
         return fail(CKV_ERR_INVALID_ARG, "budget %d of layer %d is below the window %d", pl.budget,
                     layer, pl.w);
@@ -155,11 +159,17 @@ int64_t keep_total(const ckv_batch* b, int budget) {
 
 // Splits every (sequence, head batch) unit's key tiles into items of at most `c` tiles and
 // packs units whole into rounds of at most `ctas` items; `c` minimises an estimate of the
-// launch's time in tile loads per CTA.  Pass 1 of a round streams while the previous round
-// exchanges its statistics and runs pass 2, so a round costs its item length, or the
-// exchange plus pass 2 of the round before when that is longer; the last round adds its own
-// exchange and pass 2.  Items longer than kL2Tiles are charged their excess again: their
-// pass-2 re-reads fall out of the CTA's share of L2.
+// launch's time in tile loads per CTA.
+//
+// Resident kernel (items of at most 512 / n_cols tiles, so that an item's logits fit in
+// TMEM): while an item waits for its unit's exchange and runs pass 2, the next item's MMAs can
+// fill the accumulators it leaves free and the ring can hold kRing more tiles; a round costs
+// its item length plus whatever of the exchange those do not cover.
+// Reload kernel: pass 1 of a round streams while the previous round exchanges its statistics
+// and runs pass 2, so a round costs its item length, or the exchange plus pass 2 of the round
+// before when that is longer; the last round adds its own exchange and pass 2.  Items longer
+// than kL2Tiles are charged their excess again: their pass-2 re-reads fall out of the CTA's
+// share of L2.
 ckv_status plan_score(const Plan& pl, const ckv_batch* b, int skip_le, int ctas, ScoreLaunch& L,
                       int max_items_per_launch) {
     struct RawUnit {
@@ -184,9 +194,26 @@ ckv_status plan_score(const Plan& pl, const ckv_batch* b, int skip_le, int ctas,
                                        // by the kernel's evict-last hint until pass 2 reads it
     constexpr double kExchange = 12.0; // publish, exchange and combine, in tile-load times
     constexpr double kPass2 = 0.4;     // pass 2 per tile from L2, relative to a pass-1 load
+    // The resident kernel when every unit fits one round of items that fit in TMEM.
+    const int c_res = 512 / pl.n_cols;
+    const bool fits = static_cast<long long>(max_tiles) <= static_cast<long long>(c_res) * ctas;
+    if (pl.score_path == CKV_SCORE_RESIDENT && !fits)
+        return fail(CKV_ERR_UNSUPPORTED,
+                    "resident scoring: a sequence of %d key tiles needs items of at most %d tiles "
+                    "on at least %d CTAs (%d available)", max_tiles, c_res,
+                    (max_tiles + c_res - 1) / c_res, ctas);
+    // Automatic choice: the resident kernel at N = 32, where TMEM holds two items of up to 8
+    // tiles, so the next item's MMAs proceed while this one waits for its unit's exchange; at
+    // N = 64 one 8-tile item fills TMEM and every exchange stalls the CTA, while the reload
+    // kernel runs pass 1 two items ahead through L2 (measured faster there).
+    L.resident = fits && (pl.score_path == CKV_SCORE_RESIDENT ||
+                          (pl.score_path == CKV_SCORE_AUTO && pl.n_cols == 32));
+    constexpr double kResExchange = 8.0;  // publish, exchange, combine and pass 2 from TMEM
+    const int ring = pl.n_cols == 64 ? 5 : 6;
+    const int c_hi = L.resident ? std::min(max_tiles, c_res) : max_tiles;
     int best_c = -1;
     double best_cost = 0;
-    for (int c = 1; c <= max_tiles; ++c) {
+    for (int c = 1; c <= c_hi; ++c) {
         long long rounds = 0;
         int cur = 0;
         bool feasible = c <= 65535;
@@ -204,9 +231,15 @@ ckv_status plan_score(const Plan& pl, const ckv_batch* b, int skip_le, int ctas,
         }
         if (!feasible) continue;
         rounds += cur > 0;
-        const double per_round = std::max(static_cast<double>(c), kPass2 * c + kExchange) +
-                                 std::max(0, c - kL2Tiles);
-        const double cost = rounds * per_round + kPass2 * c + kExchange;
+        double cost;
+        if (L.resident) {
+            const double per_round = c + std::max(0.0, kResExchange - (c_res - c) - ring);
+            cost = rounds * per_round + kResExchange;
+        } else {
+            const double per_round = std::max(static_cast<double>(c), kPass2 * c + kExchange) +
+                                     std::max(0, c - kL2Tiles);
+            cost = rounds * per_round + kPass2 * c + kExchange;
+        }
         if (best_c < 0 || cost < best_cost) {
             best_c = c;
             best_cost = cost;

@@ -104,20 +104,32 @@ __device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
     return ok != 0;
 }
 
+// try_wait with a suspend-time hint: the thread sleeps in the barrier unit until the phase
+// completes or about `ns` nanoseconds have passed, so a waiting warp takes no issue slots.
+__device__ __forceinline__ bool mbar_try_wait_for(uint64_t* bar, uint32_t parity, uint32_t ns) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity), "r"(ns)
+        : "memory");
+    return ok != 0;
+}
+
 // Waits for the phase with the given parity to complete.  Gives up (returns false) after
-// `limit` cycles or as soon as *abort is set by another thread of the block (both are
-// checked every 64 polls).  Between polls the warp sleeps for `backoff_ns`, so waiting warps
-// leave the issue slots of their scheduler to the warps doing work.
+// `limit` cycles or once *abort is set by another thread of the block; both are checked each
+// time a suspended try_wait (at most ~1 us) returns without the phase.
+constexpr uint32_t kSuspendNs = 1000;
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort,
-                                          uint32_t backoff_ns = 32,
                                           long long limit = kWaitTimeoutCycles) {
     if (mbar_try_wait(bar, parity)) return true;
     const long long t0 = clock64();
 #pragma unroll 1
-    for (uint32_t it = 1;; ++it) {
-        __nanosleep(backoff_ns);
-        if (mbar_try_wait(bar, parity)) return true;
-        if ((it & 63u) == 0u && (*abort || clock64() - t0 > limit)) return false;
+    for (;;) {
+        if (mbar_try_wait_for(bar, parity, kSuspendNs)) return true;
+        if (*abort || clock64() - t0 > limit) return false;
     }
 }
 

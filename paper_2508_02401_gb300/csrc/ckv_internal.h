@@ -47,6 +47,7 @@ struct ScoreLaunch {
     int w_pad, n_cols;     // rows per head in the MMA (8/16/32/64), MMA N (32/64)
     int nb;                // head batches
     int grid;              // CTAs (= items per round)
+    bool resident;         // score_resident.cu (logits kept in TMEM) instead of score_kernel.cu
     uint32_t cu_hash;      // seqlens_hash of the host copy of cu_seqlens
     float softmax_scale;
     int n_sel;

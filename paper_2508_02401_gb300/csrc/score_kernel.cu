@@ -10,7 +10,7 @@
 // Work: a unit is (sequence, batch of selected heads of one KV group); its key tiles are cut
 // into items of a few tiles, and the items are dealt out in rounds of gridDim.x (CTA b takes
 // item round * gridDim.x + b; all items of a unit are in one round).  One cooperative
-// launch, one CTA per SM, 640 threads, warp-specialised:
+// launch, one CTA per SM, 512 threads, warp-specialised:
 //   warp 0       pass-1 producer: per item, TMA loads of the window query rows (the MMA's B
 //                operand) into one of three buffers, then of its 128-key x 128-dim bf16 K
 //                tiles (two 128-byte-swizzled boxes of 64 dims) into a ring of kP1Slots slots;
@@ -22,16 +22,16 @@
 //   warp 3       publisher: once an item's pass-1 partials are stored, one release on the
 //                unit's arrival counter;
 //   warps 4-11   pass 1, one warpgroup per 32 columns: each thread owns one key (one TMEM
-//                lane), keeps a running (max, sum of 2^(x - max)) per column, and at the end of
-//                the item the warpgroup's per-column partial goes to global memory, followed by
-//                a release on the unit's arrival counter;
-//   warps 12-19  pass 2, one warpgroup per 32 columns: once every item of the unit has
-//                arrived (a bounded acquire spin) they combine the partials into lse and sum
-//                exp2(x - lse) over each head's rows per key.
+//                lane) and keeps a running (max, sum of 2^(x - max)) per column; at the end of
+//                the item the warpgroup's per-column partial goes to global memory;
+//   warps 12-15  pass 2, one warpgroup over all N columns: once every item of the unit has
+//                arrived (a bounded acquire spin) it combines the partials into lse and sums
+//                2^(x - lse) over each head's rows per key.
+// Only the last tiles of a sequence (the window's own keys, the padding past its end) need a
+// per-column mask; the others take an unmasked path of packed fp32 pair instructions.
 // Pass 1 of an item overlaps the exchange and pass 2 of the item before it, so HBM keeps
 // streaming while the CTAs wait for each other.
-#include "ckv_device.cuh"
-#include "ckv_internal.h"
+#include "score_common.cuh"
 
 #include <string.h>
 
@@ -43,36 +43,6 @@ constexpr int kP1Slots = 3;                           // pass-1 ring (HBM)
 constexpr int kP2Slots = 2;                           // pass-2 ring (L2)
 constexpr int kAcc = 4;                               // TMEM accumulators per pass
 constexpr int kQBufs = 3;                             // query-row buffers: pass 1 runs two items ahead
-constexpr int kTileBytes = kTileKeys * kHeadDim * 2;  // 32 KiB
-constexpr int kHalfBytes = kTileBytes / 2;            // 64 dims x 128 keys
-// The running maximum of a column is only moved when a logit exceeds it by more than 2^60:
-// the running sum then stays far below the fp32 range (at most keys * 2^60), and terms that
-// are 2^-126 below the reference are negligible against the reference term itself.
-constexpr float kLazyTau = 60.0f;
-constexpr int kCols = 32;                             // columns per epilogue warpgroup
-constexpr int kThreads = 512;
-constexpr int kWarpA = 4, kWarpB = 12;                // first pass-1 / pass-2 warp
-
-struct alignas(128) ScoreParams {
-    CUtensorMap tmap_k;            // K as {128 (dim), H_kv, T}, box {64, 1, 128}, 128B swizzle
-    CUtensorMap tmap_q;            // q_win as {128, H_q, S*w}, box {64, 1, W_PAD}, 128B swizzle
-    const __nv_bfloat16* q_win;    // [S, w, H_q, 128] packed
-    const int32_t* cu_seqlens;     // device [S+1] (checked against cu_hash)
-    float2* partials;              // [n_items, N]: (max, sum) per window-row column
-    int* counters;                 // [n_units] arrivals, zero at launch
-    float* scores;                 // [n_sel, T]
-    int* status;
-    int S, T, Hq, w, n_rounds, n_items, n_units;
-    uint32_t cu_hash;
-    float sl2;                     // softmax scale * log2(e)
-    long long wait_cycles;         // limit of a bounded wait (ckv_set_wait_limit_us)
-    int16_t batch_group[kMaxBatches];   // KV head of each head batch
-    int16_t batch_first[kMaxBatches];   // score row of the batch's first head
-    int16_t batch_nheads[kMaxBatches];  // heads in the batch
-    int16_t sel_heads[kMaxQHeads];      // query head of each score row
-    ScoreItem items[kMaxScoreItems];    // [n_rounds * gridDim.x]
-    ScoreUnit units[kMaxScoreUnits];
-};
 
 template <int N>
 struct SmemLayout {
@@ -96,151 +66,6 @@ struct SmemLayout {
     static constexpr int kBytes = kAbort + 4;
     static constexpr int kDynamic = kBytes + 1024;      // slack to align the base to 1024 B
 };
-
-__device__ __forceinline__ float redux_max(float v) {
-    float r;
-    asm volatile("redux.sync.max.f32 %0, %1, 0xffffffff;" : "=f"(r) : "f"(v));
-    return r;
-}
-
-__device__ __forceinline__ void red_release_add(int* p, int v) {
-    asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
-}
-
-__device__ __forceinline__ float lg2_approx(float x) {
-    float y;
-    asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-    return y;
-}
-
-// Sum / max of an array by a balanced tree (short dependency chains).
-template <int C>
-__device__ __forceinline__ float tree_sum(float (&x)[C]) {
-#pragma unroll
-    for (int w = C / 2; w >= 1; w >>= 1)
-#pragma unroll
-        for (int i = 0; i < w; ++i) x[i] += x[i + w];
-    return x[0];
-}
-
-__device__ __forceinline__ int ld_acquire(const int* p) {
-    int v;
-    asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-    return v;
-}
-
-// Warp-wide sums of C per-lane columns (C = 8, 16 or 32) by recursive halving: at each level
-// a lane keeps one half of its remaining columns and swaps the other half with its partner, so
-// the C sums take C - 1 + log2(32 / C) shuffles instead of 5 C.  `m` (uniform across the warp)
-// is carried along.  Afterwards lane l holds column l / (32 / C) in v[0] / m[0].
-template <int R>
-__device__ __forceinline__ void setmaxnreg_inc() {
-    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(R));
-}
-template <int R>
-__device__ __forceinline__ void setmaxnreg_dec() {
-    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(R));
-}
-
-// A barrier of one epilogue warpgroup built on an mbarrier of 128 arrivals, so that the wait
-// is bounded like every other wait of the kernel.
-__device__ __forceinline__ bool group_sync(uint64_t* bar, uint32_t& phase, volatile int* abort,
-                                           long long limit) {
-    mbar_arrive(bar);
-    const bool ok = mbar_wait(bar, phase, abort, 32, limit);
-    phase ^= 1;
-    return ok;
-}
-
-template <int C>
-__device__ __forceinline__ void transpose_reduce(float (&v)[C], float (&m)[C], int lane) {
-#pragma unroll
-    for (int k = C / 2, bit = 16; k >= 1; k >>= 1, bit >>= 1) {
-        const bool upper = (lane & bit) != 0;
-#pragma unroll
-        for (int i = 0; i < k; ++i) {
-            const float send = upper ? v[i] : v[i + k];
-            const float keep = upper ? v[i + k] : v[i];
-            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, bit);
-            m[i] = upper ? m[i + k] : m[i];
-        }
-    }
-#pragma unroll
-    for (int bit = 16 / C; bit >= 1; bit >>= 1) v[0] += __shfl_xor_sync(0xffffffffu, v[0], bit);
-}
-
-template <int CPW>
-__device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, float (&v)[CPW]) {
-    if constexpr (CPW == 32) {
-        tmem_ld32(taddr, v);
-    } else if constexpr (CPW == 16) {
-        uint32_t r[16];
-        asm volatile(
-            "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-            "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n\t"
-            "tcgen05.wait::ld.sync.aligned;"
-            : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]),
-              "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]),
-              "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-            : "r"(taddr)
-            : "memory");
-#pragma unroll
-        for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
-    } else {
-        static_assert(CPW == 8, "CPW");
-        uint32_t r[8];
-        asm volatile(
-            "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];\n\t"
-            "tcgen05.wait::ld.sync.aligned;"
-            : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]),
-              "=r"(r[6]), "=r"(r[7])
-            : "r"(taddr)
-            : "memory");
-#pragma unroll
-        for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(r[i]);
-    }
-}
-
-// tcgen05.ld of 16 columns without the wait: the registers are not valid until tmem_ld_wait,
-// and reg_fence then ties every later use to the wait.
-__device__ __forceinline__ void tmem_ld16_nowait(uint32_t taddr, float (&v)[16]) {
-    uint32_t r[16];
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
-          "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-        : "r"(taddr)
-        : "memory");
-#pragma unroll
-    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
-}
-
-__device__ __forceinline__ void tmem_ld_wait() {
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-}
-
-__device__ __forceinline__ void reg_fence(float (&v)[16]) {
-    asm volatile(""
-                 : "+f"(v[0]), "+f"(v[1]), "+f"(v[2]), "+f"(v[3]), "+f"(v[4]), "+f"(v[5]),
-                   "+f"(v[6]), "+f"(v[7]), "+f"(v[8]), "+f"(v[9]), "+f"(v[10]), "+f"(v[11]),
-                   "+f"(v[12]), "+f"(v[13]), "+f"(v[14]), "+f"(v[15]));
-}
-
-// Valid-column mask of one thread for a tile: columns holding a real window row that sees
-// key j.  Row r of a head sees key j iff r >= j - P (causal window); keys >= L are padding.
-template <int CPW, int W_PAD>
-__device__ __forceinline__ uint32_t tile_mask(uint32_t colmask, int col0, int t, int j, int P, int L) {
-    const bool edge = (t * kTileKeys + kTileKeys - 1 >= P) || (t * kTileKeys + kTileKeys > L);
-    if (!edge) return colmask;
-    if (j >= L) return 0u;
-    const int jr = j - P;
-    uint32_t cm = 0;
-#pragma unroll
-    for (int i = 0; i < CPW; ++i) cm |= (((col0 + i) % W_PAD) >= jr ? 1u : 0u) << i;
-    return colmask & cm;
-}
 
 template <int N, int W_PAD>
 __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constant__ ScoreParams p) {
@@ -276,7 +101,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
     // scratch of the epilogues (static, so that its accesses are shared-memory instructions)
     __shared__ float2 red_a[2][2][128];  // [item parity][warpgroup][warp * 32 + lane]
     __shared__ float2 red_b[256];        // [part * N + column]
-    __shared__ float lse_s[64];
+    __shared__ __align__(16) float nlse_s[64];  // -lse per column of the current pass-2 item
     __shared__ volatile int verdict[1];
     volatile int* issued = reinterpret_cast<volatile int*>(sm + SL::kIssued);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + SL::kTmemSlot);
@@ -315,6 +140,11 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         tma_prefetch_desc(&p.tmap_k);
         tma_prefetch_desc(&p.tmap_q);
     }
+    // Query slots of head batches with fewer heads than the MMA's columns are never loaded;
+    // zeros there keep those (unused) columns finite.
+    for (int i = threadIdx.x; i < kQBufs * SL::kQBytes / 16; i += kThreads)
+        reinterpret_cast<uint4*>(qbuf)[i] = make_uint4(0u, 0u, 0u, 0u);
+    fence_proxy_async_smem();
     if (warp == 1) {
         tmem_alloc(tmem_slot, kTmemCols);
         tmem_relinquish();
@@ -373,7 +203,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                     // (the next sequence's, or zeros past the end) and head slots past the
                     // batch's heads land in columns that the epilogues mask out.
                     const int qb = it % kQBufs;
-                    if (!mbar_wait(&q_empty[qb], ((it / kQBufs) & 1) ^ 1, abort, 32, lim)) {
+                    if (!mbar_wait(&q_empty[qb], ((it / kQBufs) & 1) ^ 1, abort, lim)) {
                         ok = false;
                         break;
                     }
@@ -389,7 +219,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                 }
                 for (int jt = 0; ok && jt < n; ++jt, ++use) {
                     const int s = use % nslots;
-                    if (!mbar_wait(&freed[s], ((use / nslots) & 1) ^ 1, abort, 32, lim)) {
+                    if (!mbar_wait(&freed[s], ((use / nslots) & 1) ^ 1, abort, lim)) {
                         ok = false;
                         break;
                     }
@@ -519,7 +349,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             for (int r = 0; r < R; ++r) {
                 const ScoreItem& I = item_of(r);
                 if (I.ntiles == 0) continue;
-                if (!mbar_wait(&pub_full[it & 1], (it >> 1) & 1, abort, 64, lim)) {
+                if (!mbar_wait(&pub_full[it & 1], (it >> 1) & 1, abort, lim)) {
                     *abort = 1;
                     record_error(p.status, kDevTimeout, 17);
                     break;
@@ -550,32 +380,29 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                 const int n = I.ntiles;
                 if (n == 0) continue;
                 const ScoreUnit U = p.units[I.unit];
-                const int L = U.len, P = L - p.w, nheads = p.batch_nheads[U.batch];
+                const int L = U.len, P = L - p.w;
                 const float sl2 = p.sl2;
-                uint32_t colmask = 0;  // this warpgroup's columns that hold a real window row
+                // Running maximum (log2 units, kept negated so that it is the FMA's addend) and
+                // the sum relative to it.  -1e30 (not -inf) for a column with no visible key
+                // yet keeps the reductions below free of inf - inf.
+                float nm[kCols], sm_[kCols];
 #pragma unroll
                 for (int i = 0; i < kCols; ++i) {
-                    const int c = col0 + i;
-                    if ((c % W_PAD) < p.w && (c / W_PAD) < nheads) colmask |= 1u << i;
-                }
-                // Running max (log2 units) and sum relative to it.  -1e30 (not -inf) for a
-                // column with no visible key yet keeps the reductions below free of inf - inf.
-                float m[kCols], sm_[kCols];
-#pragma unroll
-                for (int i = 0; i < kCols; ++i) {
-                    m[i] = -1e30f;
+                    nm[i] = 1e30f;
                     sm_[i] = 0.f;
                 }
                 for (int jt = 0; jt < n; ++jt, ++a_it) {
                     const int acc = a_it % kAcc;
-                    if (!mbar_wait(&a_full[acc], (a_it / kAcc) & 1, abort, 32, lim)) {
+                    if (!mbar_wait(&a_full[acc], (a_it / kAcc) & 1, abort, lim)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after_sync();
                     const int t = I.tile0 + jt;
                     const int j = t * kTileKeys + eq * 32 + lane;  // sequence-local key
-                    const uint32_t vm = tile_mask<kCols, W_PAD>(colmask, col0, t, j, P, L);
+                    // Tiles wholly before the window, inside the sequence: every key is seen by
+                    // every row, and the columns without a real row are never read, so no mask.
+                    const bool edge = (t * kTileKeys + kTileKeys - 1 >= P) || (t * kTileKeys + kTileKeys > L);
                     const uint32_t taddr = tmem_base + lane_base + static_cast<uint32_t>(acc * N + col0);
                     // both halves of 16 columns in flight, then one wait
                     float vv[2][16];
@@ -587,71 +414,26 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                     tc_fence_before_sync();
                     __syncwarp();
                     if (lane == 0) mbar_arrive(&a_empty[acc]);  // the accumulator is free
-#pragma unroll
-                    for (int hh = 0; hh < 2; ++hh) {
-                        float (&v)[16] = vv[hh];
-                        const uint32_t hm = (vm >> (16 * hh)) & 0xffffu;
-                        float* mh = m + 16 * hh;
-                        float* sh = sm_ + 16 * hh;
-                        float d[16];
-#pragma unroll
-                        for (int i = 0; i < 16; ++i) {
-                            const float x = fmaf(v[i], sl2, -mh[i]);
-                            d[i] = ((hm >> i) & 1u) ? x : -INFINITY;
-                        }
-                        float dm[4];  // max by a short tree
-#pragma unroll
-                        for (int i = 0; i < 4; ++i)
-                            dm[i] = fmaxf(fmaxf(d[4 * i], d[4 * i + 1]), fmaxf(d[4 * i + 2], d[4 * i + 3]));
-                        if (fmaxf(fmaxf(dm[0], dm[1]), fmaxf(dm[2], dm[3])) > kLazyTau) {
-                            // A logit well above the running maximum (always so for a column's
-                            // first visible key): restart the column's sum relative to it.
-#pragma unroll
-                            for (int i = 0; i < 16; ++i) {
-                                if (d[i] > kLazyTau) {
-                                    sh[i] *= ex2_approx(-d[i]);
-                                    mh[i] = v[i] * sl2;
-                                    d[i] = 0.f;
-                                }
-                            }
-                        }
-#pragma unroll
-                        for (int i = 0; i < 16; ++i) sh[i] += ex2_approx(d[i]);
+                    if (!edge) {
+                        stats_block<false, W_PAD, 0>(vv[0], nm, sm_, sl2, 0);
+                        stats_block<false, W_PAD, 16>(vv[1], nm + 16, sm_ + 16, sl2, 0);
+                    } else {
+                        // row r of a head sees key j iff r >= j - P; keys past L are padding
+                        // (columns without a real row are never read, so they need no mask)
+                        const int jr = (j < L ? j - P : (1 << 30)) - (W_PAD == 64 ? col0 : 0);
+                        stats_block<true, W_PAD, 0>(vv[0], nm, sm_, sl2, jr);
+                        stats_block<true, W_PAD, 16>(vv[1], nm + 16, sm_ + 16, sl2, jr);
                     }
                 }
-                if (!ok) break;
-                // Per column over the warpgroup's 128 keys: warp max by redux, rescale to it,
-                // warp sums by recursive halving, then the 4 warps through shared memory.
+                float m[kCols];
 #pragma unroll
-                for (int i = 0; i < kCols; ++i) {
-                    const float M = redux_max(m[i]);
-                    sm_[i] *= ex2_approx(m[i] - M);
-                    m[i] = M;
-                }
-                transpose_reduce<kCols>(sm_, m, lane);  // lane l: column l
-                float2* red = red_a[a_item & 1][wg];
-                red[eq * 32 + lane] = make_float2(m[0], sm_[0]);
-                if (!group_sync(gbar, gphase, abort, lim)) {
+                for (int i = 0; i < kCols; ++i) m[i] = -nm[i];
+                if (!ok) break;
+                if (!item_partials(m, sm_, red_a[a_item & 1][wg], eq, lane, wtid, gbar, gphase,
+                                   &pub_full[a_item & 1], &pub_empty[a_item & 1], (a_item >> 1) & 1,
+                                   p.partials + static_cast<size_t>(item) * N + col0, abort, lim)) {
                     ok = false;
                     break;
-                }
-                if (wtid < kCols) {
-                    float M = red[wtid].x;
-#pragma unroll
-                    for (int q = 1; q < 4; ++q) M = fmaxf(M, red[q * 32 + wtid].x);
-                    float S = 0.f;
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const float2 x = red[q * 32 + wtid];
-                        S += x.y * ex2_approx(x.x - M);
-                    }
-                    // the publisher has released the item two back that used this phase
-                    if (!mbar_wait(&pub_empty[a_item & 1], ((a_item >> 1) & 1) ^ 1, abort, 32, lim)) {
-                        ok = false;
-                        break;
-                    }
-                    p.partials[static_cast<size_t>(item) * N + col0 + wtid] = make_float2(M, S);
-                    mbar_arrive(&pub_full[a_item & 1]);
                 }
                 ++a_item;
             }
@@ -687,98 +469,21 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             for (int c = 0; c < N; ++c)
                 if ((c % W_PAD) < p.w && (c / W_PAD) < nheads) colmask |= 1ull << c;
             // ---------------------------------------------------- exchange with the unit
-            if (wtid == 0) {
-                const int target = U.nitems * kNW;
-                const long long t0 = clock64();
-                bool got = true;
-                for (uint32_t k = 1; ld_acquire(p.counters + I.unit) < target; ++k) {
-                    __nanosleep(64);
-                    if ((k & 63u) == 0u && (*abort || clock64() - t0 > lim)) {
-                        got = false;
-                        break;
-                    }
-                }
-                __threadfence();
-                verdict[0] = got ? 1 : 0;
-            }
-            if (!group_sync(gbar, gphase, abort, lim) || verdict[0] == 0) {
+            if (!unit_lse<N>(p, U, I.unit, wtid, gbar, gphase, verdict, red_b, nlse_s, colmask, abort, lim)) {
                 ok = false;
                 break;
-            }
-            {
-                // Column pairs (2c, 2c+1) by 16-byte loads, items split over the parts; up
-                // to kU loads in flight per thread (a unit can have ~150 items).
-                constexpr int kPairs = N / 2, kParts = 128 / kPairs, kU = 20;
-                static_assert(kParts * N <= 256, "red_b holds 256 entries");
-                const int c2 = wtid % kPairs, part = wtid / kPairs;
-                float M0 = -INFINITY, S0 = 0.f, M1 = -INFINITY, S1 = 0.f;
-                const float4* src =
-                    reinterpret_cast<const float4*>(p.partials + static_cast<size_t>(U.first_item) * N) + c2;
-                for (int k0 = part; k0 < U.nitems; k0 += kParts * kU) {
-                    float4 pr[kU];
-#pragma unroll
-                    for (int u = 0; u < kU; ++u) {
-                        const int k = k0 + u * kParts;
-                        pr[u] = k < U.nitems ? __ldcg(src + static_cast<size_t>(k) * kPairs)
-                                             : make_float4(-INFINITY, 0.f, -INFINITY, 0.f);
-                    }
-#pragma unroll
-                    for (int u = 0; u < kU; ++u) {
-                        float Mn = fmaxf(M0, pr[u].x);
-                        if (Mn > -INFINITY) {
-                            S0 = S0 * ex2_approx(M0 - Mn) + pr[u].y * ex2_approx(pr[u].x - Mn);
-                            M0 = Mn;
-                        }
-                        Mn = fmaxf(M1, pr[u].z);
-                        if (Mn > -INFINITY) {
-                            S1 = S1 * ex2_approx(M1 - Mn) + pr[u].w * ex2_approx(pr[u].z - Mn);
-                            M1 = Mn;
-                        }
-                    }
-                }
-                red_b[part * N + 2 * c2] = make_float2(M0, S0);
-                red_b[part * N + 2 * c2 + 1] = make_float2(M1, S1);
-                if (!group_sync(gbar, gphase, abort, lim)) {
-                    ok = false;
-                    break;
-                }
-                if (wtid < N) {  // part 0 always holds item 0, so M2 turns finite first
-                    float M2 = -INFINITY, S2 = 0.f;
-#pragma unroll
-                    for (int q = 0; q < kParts; ++q) {
-                        const float2 x = red_b[q * N + wtid];
-                        const float Mn = fmaxf(M2, x.x);
-                        S2 = S2 * ex2_approx(M2 - Mn) + x.y * ex2_approx(x.x - Mn);
-                        M2 = Mn;
-                    }
-                    lse_s[wtid] = M2 + lg2_approx(S2);
-                }
-                if (!group_sync(gbar, gphase, abort, lim)) {
-                    ok = false;
-                    break;
-                }
             }
             // ---------------------------------------------------- the item's tiles
             for (int jt = 0; jt < n; ++jt, ++b_it) {
                 const int acc = b_it % kAcc;
-                if (!mbar_wait(&b_full[acc], (b_it / kAcc) & 1, abort, 32, lim)) {
+                if (!mbar_wait(&b_full[acc], (b_it / kAcc) & 1, abort, lim)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after_sync();
                 const int t = I.tile0 + jt;
                 const int j = t * kTileKeys + eq * 32 + lane;
-                // columns that see key j: all real ones, except in the window's own tiles
-                uint64_t vm = colmask;
                 const bool edge = (t * kTileKeys + kTileKeys - 1 >= P) || (t * kTileKeys + kTileKeys > L);
-                if (edge) {
-                    uint64_t cm = 0;
-                    if (j < L) {
-#pragma unroll
-                        for (int c = 0; c < N; ++c) cm |= static_cast<uint64_t>((c % W_PAD) >= j - P) << c;
-                    }
-                    vm &= cm;
-                }
                 const uint32_t taddr = tmem_base + lane_base + static_cast<uint32_t>((kAcc + acc) * N);
                 // every 16-column chunk in flight, then one wait
                 float vv[N / 16][16];
@@ -791,25 +496,10 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&b_empty[acc]);  // the accumulator is free
                 float accum[kHeads];
-#pragma unroll
-                for (int h = 0; h < kHeads; ++h) accum[h] = 0.f;
-#pragma unroll
-                for (int hh = 0; hh < N / 16; ++hh) {
-                    float (&v)[16] = vv[hh];
-                    const uint32_t hm = static_cast<uint32_t>(vm >> (16 * hh)) & 0xffffu;
-#pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        const float e = ex2_approx(fmaf(v[i], sl2, -lse_s[16 * hh + i]));
-                        v[i] = ((hm >> i) & 1u) ? e : 0.f;
-                    }
-                    constexpr int kPiece = W_PAD < 16 ? W_PAD : 16;  // a head's columns in this chunk
-#pragma unroll
-                    for (int q = 0; q < 16 / kPiece; ++q) {
-                        float seg[kPiece];
-#pragma unroll
-                        for (int i = 0; i < kPiece; ++i) seg[i] = v[q * kPiece + i];
-                        accum[(16 * hh + q * kPiece) / W_PAD] += tree_sum<kPiece>(seg);
-                    }
+                if (!edge) {
+                    prob_sums<N, W_PAD, false>(vv, sl2, nlse_s, 0, accum);
+                } else {  // row r sees key j iff r >= j - P; keys past L are padding
+                    prob_sums<N, W_PAD, true>(vv, sl2, nlse_s, j < L ? j - P : (1 << 30), accum);
                 }
                 if (j < L) {
                     const size_t col = static_cast<size_t>(U.seq_start) + j;
@@ -912,7 +602,8 @@ cudaError_t launch_score(const ScoreLaunch& L, cudaStream_t stream) {
         memcpy(p.units, L.units.data() + sl.unit0, sizeof(ScoreUnit) * p.n_units);
         cudaError_t e = cudaMemsetAsync(L.counters, 0, sizeof(int) * sl.n_units, stream);
         if (e != cudaSuccess) return e;
-        e = dispatch(p, L.n_cols, L.w_pad, L.grid, stream);
+        e = L.resident ? launch_resident(p, L.n_cols, L.w_pad, L.grid, stream)
+                       : dispatch(p, L.n_cols, L.w_pad, L.grid, stream);
         if (e != cudaSuccess) return e;
     }
     return cudaSuccess;

@@ -47,7 +47,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 
 def test_version_and_status_strings(lib):
-    assert ckv.ckv_abi_version() == 2
+    assert ckv.ckv_abi_version() == 3
     assert ckv.ckv_status_string(0) == "CKV_OK"
     assert ckv.ckv_status_string(3) == "CKV_ERR_WORKSPACE"
 
@@ -100,6 +100,8 @@ def _call_compress(lib, cfg, batch, layer=0, q=_P, k=_P, v=_P, ws=_P, ws_bytes=1
     (dict(head_mask=np.zeros((2, 32), np.uint8)), 1),             # group without a head
     (dict(num_q_heads=512, num_kv_heads=8, head_mask=np.ones((2, 512), np.uint8)), 2),
     (dict(scope=2), 1),
+    (dict(score_path=3), 1),
+    (dict(score_path=-1), 1),
     (dict(scope=1, head_mask=np.zeros((2, 32), np.uint8)), 1),    # layer without a head
 ])
 def test_config_errors(lib, change, expect):

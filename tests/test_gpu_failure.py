@@ -1,9 +1,10 @@
 """Failure detection on the GPU without a fault: a bounded wait that runs out is reported in
 the workspace status word, the kernel returns, and the CUDA context stays usable.
 
-The wait limit is shortened to 1 us with ckv_set_wait_limit_us; with 4 CTAs for a 40k-token
-sequence every work item is ~80 key tiles long, so the cross-CTA exchange of each round waits
-far longer than that and gives up.  No flag, barrier or check is removed: every wait still
+The wait limit is shortened to 1 us with ckv_set_wait_limit_us.  With 4 CTAs for a 40k-token
+sequence (the kernel that re-reads K) every work item is ~80 key tiles long, so the cross-CTA
+exchange of each round waits far longer than that and gives up; in the kernel that keeps the
+logits in TMEM the first key tile alone takes longer than 1 us to arrive from HBM.  No flag, barrier or check is removed: every wait still
 ends, only sooner.
 """
 import pytest
@@ -25,12 +26,14 @@ def _built():
     oracle.build()
 
 
-def test_a_wait_that_runs_out_is_reported_and_the_context_stays_usable():
+@pytest.mark.parametrize("max_ctas,path", [(4, ckv.SCORE_RELOAD), (0, ckv.SCORE_RESIDENT)],
+                         ids=["reload", "resident"])
+def test_a_wait_that_runs_out_is_reported_and_the_context_stays_usable(max_ctas, path):
     wl = cs.Workload(name="timeout", num_layers=1, num_q_heads=32, num_kv_heads=8,
                      seqlens=(40000, 9000), window=32, heads_per_group=2, budget_mean=300,
                      budget_uniform=True, outlier_channels=8, seed=5)
     li = wl.layer(0)
-    cfg = ckv.Config.from_workload(wl, max_ctas=4)
+    cfg = ckv.Config.from_workload(wl, max_ctas=max_ctas, score_path=path)
     ckv.ckv_set_wait_limit_us(1)
     try:
         g = gu.run_gpu(wl, 0, li, cfg=cfg, scores=False, check_status=False)

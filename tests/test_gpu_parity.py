@@ -51,6 +51,8 @@ FUZZ = [
     dict(seqlens=(5000,), plant="span", plant_count=32, plant_beta=4.0, plant_noise=True,
          budget_mean=64, pool_type="avg"),
     dict(seqlens=(20000,), budget_mean=600, heads_per_group=1, pool_kernel=9),
+    # keys far above the rest, in later tiles of the work items: the column references move
+    dict(seqlens=(3000, 1700), plant="tokens", plant_count=24, plant_beta=9.0, budget_mean=64),
     # one selection per layer from heads anywhere in the layer (Sec. 3.3 as stated)
     dict(scope="layer", heads_per_layer=3, seqlens=(1000, 77, 300), budget_mean=40),
     dict(scope="layer", heads_per_layer=4, num_q_heads=32, num_kv_heads=8, window=8,
@@ -62,12 +64,17 @@ FUZZ = [
 ]
 
 
+PATHS = [ckv.SCORE_RESIDENT, ckv.SCORE_RELOAD]
+
+
+@pytest.mark.parametrize("path", PATHS, ids=["resident", "reload"])
 @pytest.mark.parametrize("case", range(len(FUZZ)))
-def test_fuzz_shapes(case):
+def test_fuzz_shapes(case, path):
     wl = _wl(**FUZZ[case])
+    cfg = ckv.Config.from_workload(wl, score_path=path)
     for layer in range(wl.num_layers):
         li = wl.layer(layer)
-        g = gu.run_gpu(wl, layer, li)
+        g = gu.run_gpu(wl, layer, li, cfg=cfg)
         o = gu.run_oracle(wl, layer, li)
         gu.check_layer(wl, layer, li, g, o)
 
@@ -83,18 +90,23 @@ def test_single_layer_workload_full():
         assert set(li.planted[0].tolist()) <= set(g["idx"][gi, ck[0]:ck[1]].tolist())
 
 
-@pytest.mark.parametrize("name,layers,groups", [
-    ("llama8b_l8192", (0, 13, 31), None),
-    ("llama8b_l32768", (0, 5), None),
-    ("needle_l131072", (7,), (0, 5)),
-    ("ragged_qwen7b", (0, 27), None),
-    ("paper_llama8b_l8192", (0, 17, 31), None),
+@pytest.mark.parametrize("name,layers,groups,path", [
+    ("llama8b_l8192", (0, 13, 31), None, ckv.SCORE_AUTO),
+    ("llama8b_l8192", (13,), None, ckv.SCORE_RELOAD),
+    ("llama8b_l32768", (0, 5), None, ckv.SCORE_AUTO),
+    ("needle_l131072", (7,), (0, 5), ckv.SCORE_AUTO),
+    ("needle_l131072", (7,), (3,), ckv.SCORE_RELOAD),
+    ("needle_l131072", (7,), (6,), ckv.SCORE_RESIDENT),
+    ("llama8b_l8192", (5,), None, ckv.SCORE_RESIDENT),
+    ("ragged_qwen7b", (0, 27), None, ckv.SCORE_AUTO),
+    ("paper_llama8b_l8192", (0, 17, 31), None, ckv.SCORE_AUTO),
 ])
-def test_full_size_workloads(name, layers, groups):
+def test_full_size_workloads(name, layers, groups, path):
     wl = cs.workload(name)
+    cfg = ckv.Config.from_workload(wl, score_path=path)
     for layer in layers:
         li = wl.layer(layer)
-        g = gu.run_gpu(wl, layer, li, scores=groups is None)
+        g = gu.run_gpu(wl, layer, li, cfg=cfg, scores=groups is None)
         o = gu.run_oracle(wl, layer, li, groups=groups, want_kv=False)
         if groups is not None:
             g["scores"] = None
@@ -208,13 +220,25 @@ def test_device_lengths_that_disagree_are_reported():
     assert ckv.ckv_read_device_status(ws) == (0, 0)  # the read reset it
 
 
-@pytest.mark.parametrize("max_ctas", [1, 5, 24])
-def test_capped_grid_long_items_and_many_rounds(max_ctas):
-    """A small CTA cap forces long work items (tiles re-loaded in pass 2) and several rounds."""
+@pytest.mark.parametrize("max_ctas,path", [(1, ckv.SCORE_AUTO), (5, ckv.SCORE_AUTO),
+                                           (24, ckv.SCORE_RELOAD), (9, ckv.SCORE_RESIDENT),
+                                           (24, ckv.SCORE_RESIDENT)])
+def test_capped_grid_long_items_and_many_rounds(max_ctas, path):
+    """A small CTA cap forces long work items (tiles re-loaded in pass 2, the only kernel that
+    takes them) and several rounds; 9 CTAs is the fewest that fit 9000 tokens in TMEM."""
     wl = _wl(seqlens=(9000, 3000, 700), num_q_heads=32, num_kv_heads=8, budget_mean=300,
              outlier_channels=8)
     li = wl.layer(0)
-    cfg = ckv.Config.from_workload(wl, max_ctas=max_ctas)
+    cfg = ckv.Config.from_workload(wl, max_ctas=max_ctas, score_path=path)
     g = gu.run_gpu(wl, 0, li, cfg=cfg)
     o = gu.run_oracle(wl, 0, li)
     gu.check_layer(wl, 0, li, g, o)
+
+
+def test_resident_path_reports_what_does_not_fit():
+    """9000 tokens are 71 key tiles: in TMEM (8 tiles per item at N = 64) they need 9 CTAs."""
+    wl = _wl(seqlens=(9000,), num_q_heads=32, num_kv_heads=8, budget_mean=300)
+    li = wl.layer(0)
+    cfg = ckv.Config.from_workload(wl, max_ctas=8, score_path=ckv.SCORE_RESIDENT)
+    with pytest.raises(ckv.CkvError, match="resident"):
+        gu.run_gpu(wl, 0, li, cfg=cfg)
