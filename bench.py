@@ -33,13 +33,13 @@ UNIT = "prefix tokens/s per layer"
 WORKLOAD = "llama8b_l8192"
 HBM_FALLBACK_GBS = 6800.0
 
-# dram__bytes_read.sum + dram__bytes_write.sum per launch pair of the scoring stage, from the
-# ncu capture summarised in profiles/, keyed by the sha256 of the kernel source it was taken on.
-# DRAM bytes (read + write) per scoring launch (one layer of llama8b_l8192) from the ncu
-# capture summarised in profiles/score_kernel_llama8b_l8192.md, keyed by the sha256 of the
-# kernel source it was taken on; a changed kernel reports null until it is captured again.
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) of one scoring launch (one layer)
+# per workload, from the ncu captures summarised in profiles/ (score_kernel_llama8b_l8192.md,
+# score_resident_paper_llama8b_l8192.md), keyed by the sha256 of the scoring kernels' sources
+# (SCORE_SOURCES); a changed kernel reports null until it is captured again.
+SCORE_SOURCES = ('score_kernel.cu', 'score_resident.cu', 'score_common.cuh', 'ckv_device.cuh')
 SCORE_TRAFFIC = {
-    "3893613cffe69c5ce65a7dba1aa62659a2b451aa6ab525761c01c5451a88608b": 16996096,
+    "0e24b44d442cf1e6c618608c61b1ead13c09ab6100d6d702e76236f3f28d9b31": {"llama8b_l8192": 16987904, "paper_llama8b_l8192": 8488704},
 }
 # Sequences up to this many tokens are selected by one block per (sequence, KV head)
 # (one launch); longer ones by the chunked kernels (two launches).
@@ -303,15 +303,20 @@ def run_ours(args):
                  "gather": stage(gather_all), "step": ms_per_step / nl}
         print("per-layer stage times (us): " + ", ".join(f"{k}={v * 1e3:.2f}" for k, v in parts.items()),
               file=sys.stderr, flush=True)
-    k_bytes = T * Hkv * 256
+    # K is read once per (token, KV head) whose group has a selected head in the layer
+    G = wl.num_q_heads // Hkv
+    scored = [int((cfg.head_mask[l].reshape(Hkv, G) != 0).any(axis=1).sum()) for l in range(nl)]
+    k_bytes = T * 256 * sum(scored) / nl
     score_gbs = k_bytes / (score_ms / 1e3) / 1e9
-    src = open(os.path.join(ROOT, "paper_2508_02401_gb300", "csrc", "score_kernel.cu"), "rb").read()
-    traffic = SCORE_TRAFFIC.get(hashlib.sha256(src).hexdigest())
-    roofline = {"bound": "hbm", "kernel": "score_kernel (ckv_score_window), per layer, layers "
+    digest = hashlib.sha256()
+    for f in SCORE_SOURCES:
+        digest.update(open(os.path.join(ROOT, "paper_2508_02401_gb300", "csrc", f), "rb").read())
+    traffic = SCORE_TRAFFIC.get(digest.hexdigest(), {}).get(args.workload)
+    roofline = {"bound": "hbm", "kernel": "scoring kernel (ckv_score_window), per layer, layers "
                                           f"overlapped on {nstreams} streams",
                 "achieved": round(score_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
                 "frac": round(score_gbs / hbm_peak, 4), "peak_kind": peak_kind,
-                "traffic": traffic, "algorithmic_bytes_per_launch": k_bytes,
+                "traffic": traffic, "algorithmic_bytes_per_launch": int(k_bytes),
                 "avg_launch_us": round(score_ms * 1e3, 2)}
     keep_bytes = sum(4 * 256 * Hkv * d["t_keep"] for d in layers) / nl
     layer_bytes = k_bytes + keep_bytes

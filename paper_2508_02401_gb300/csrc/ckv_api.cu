@@ -190,8 +190,9 @@ ckv_status plan_score(const Plan& pl, const ckv_batch* b, int skip_le, int ctas,
     L.slices.clear();
     if (raw.empty()) return CKV_OK;
     if (b->num_seqs > 65535) return fail(CKV_ERR_UNSUPPORTED, "more than 65535 sequences");
-    constexpr int kL2Tiles = 16;       // 16 tiles x 32 KiB x 152 CTAs ~ 78 MB of L2, kept there
-                                       // by the kernel's evict-last hint until pass 2 reads it
+    constexpr int kL2Tiles = 8;        // pass 1 runs up to two items ahead, so each CTA keeps
+                                       // ~2 items in L2 (evict-last hint) until pass 2 reads
+                                       // them: 2 x 8 tiles x 32 KiB x 152 CTAs ~ 80 MB
     constexpr double kExchange = 12.0; // publish, exchange and combine, in tile-load times
     constexpr double kPass2 = 0.4;     // pass 2 per tile from L2, relative to a pass-1 load
     // The resident kernel when every unit fits one round of items that fit in TMEM.
