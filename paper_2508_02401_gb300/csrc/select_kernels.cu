@@ -402,12 +402,12 @@ __device__ __forceinline__ void copy_rows(const SelectParams& p, const UnitGeo& 
 }
 
 // Writes list[0..m) (sequence-local positions, in order) to the index rows at offset out_off
-// of the unit's kept tokens, and copies the K/V rows when asked, for every KV head that the
-// unit's selection serves: its own (per-KV-head scope) or all of them (per-layer scope).
+// of the unit's kept tokens, and copies the K/V rows when asked, for KV heads [kv0, kv1) of
+// those the unit's selection serves: its own (per-KV-head scope) or all of them (per-layer
+// scope).
 __device__ __forceinline__ void emit_kept(const SelectParams& p, const UnitGeo& u, const int* list,
-                                          int m, int out_off) {
-    const int per = p.Hkv / p.n_vec;
-    for (int kv = u.g * per; kv < (u.g + 1) * per; ++kv) {
+                                          int m, int out_off, int kv0, int kv1) {
+    for (int kv = kv0; kv < kv1; ++kv) {
         int32_t* out = p.idx + static_cast<size_t>(kv) * p.T_keep + u.keep_off + out_off;
         for (int e = threadIdx.x; e < m; e += blockDim.x) out[e] = list[e];
         if (p.k) copy_rows(p, u, kv, list, m, u.keep_off + out_off);
@@ -421,26 +421,31 @@ __global__ void __launch_bounds__(kUnitThreads, 1) select_unit_kernel(const __gr
     __shared__ int scratch[33];
     __shared__ int s_digit, s_above, s_cut;
     constexpr int NT = kUnitThreads, PER = kUnitPer;
-    const int unit = blockIdx.x, tid = threadIdx.x;
-    if (unit == 0 && tid == 0 && seqlens_hash(p.cu_seqlens, p.S) != p.cu_hash)
+    // A selection that serves several KV heads (per-layer scope) is made by one block per KV
+    // head, each gathering its own head's rows: the selection is recomputed (from L2-resident
+    // scores) rather than one block copying every head's rows alone.
+    const int per = p.Hkv / p.n_vec;
+    const int unit = blockIdx.x / per, sub = blockIdx.x % per, tid = threadIdx.x;
+    if (blockIdx.x == 0 && tid == 0 && seqlens_hash(p.cu_seqlens, p.S) != p.cu_hash)
         record_error(p.status, kDevBadSeqlens, 230);
     UnitGeo u;
     if (!unit_geo(p, unit, u)) return;
     if (u.L > kUnitLen) return;  // a long unit: the chunked kernels take it
-    if (u.g == 0 && tid == 0) {
+    const int kv = u.g * per + sub;  // the KV head whose rows this block writes
+    if (u.g == 0 && sub == 0 && tid == 0) {
         p.cu_keep[u.s + 1] = u.keep_off + u.n_keep;
         if (u.s == 0) p.cu_keep[0] = 0;
     }
     float* pooled = p.pooled + static_cast<size_t>(u.g) * p.T + u.t0;
     int* list = reinterpret_cast<int*>(ust);
-    const bool zeros = p.from_scores && p.write_pooled;
+    const bool zeros = p.from_scores && p.write_pooled && sub == 0;
     if (u.L <= p.budget) {  // kept whole; its pooled scores read as 0
         for (int e = tid; e < u.L; e += NT) {
             list[e] = e;
             if (zeros) pooled[e] = 0.f;
         }
         __syncthreads();
-        emit_kept(p, u, list, u.L, 0);
+        emit_kept(p, u, list, u.L, 0, kv, kv + 1);
         return;
     }
     const int P = u.P, k = u.k;
@@ -538,7 +543,7 @@ __global__ void __launch_bounds__(kUnitThreads, 1) select_unit_kernel(const __gr
     }
     for (int i = tid; i < p.w; i += NT) list[k + i] = P + i;
     __syncthreads();
-    emit_kept(p, u, list, p.budget, 0);
+    emit_kept(p, u, list, p.budget, 0, kv, kv + 1);
 }
 
 // ------------------------------------------------------------------ longer units, in chunks
@@ -857,14 +862,14 @@ __global__ void __launch_bounds__(kSelThreads) compact_kernel(const __grid_const
         const int m = max(0, min(u.L, j0 + kChunk) - j0);
         for (int e = tid; e < m; e += kSelThreads) list[e] = j0 + e;
         __syncthreads();
-        emit_kept(p, u, list, m, j0);
+        emit_kept(p, u, list, m, j0, u.g * (p.Hkv / p.n_vec), (u.g + 1) * (p.Hkv / p.n_vec));
         return;
     }
     const int P = u.P, k = u.k;
     if (c == 0) {  // the window closes the list
         for (int i = tid; i < p.w; i += kSelThreads) list[i] = P + i;
         __syncthreads();
-        emit_kept(p, u, list, p.w, k);
+        emit_kept(p, u, list, p.w, k, u.g * (p.Hkv / p.n_vec), (u.g + 1) * (p.Hkv / p.n_vec));
         __syncthreads();
     }
     if (j0 >= P) return;
@@ -914,7 +919,7 @@ __global__ void __launch_bounds__(kSelThreads) compact_kernel(const __grid_const
         r += __popc(bal[q]);
     }
     __syncthreads();
-    emit_kept(p, u, list, tot, base);
+    emit_kept(p, u, list, tot, base, u.g * (p.Hkv / p.n_vec), (u.g + 1) * (p.Hkv / p.n_vec));
 }
 struct GatherParams {
     const uint4* k;
@@ -1035,7 +1040,7 @@ cudaError_t launch_select(const SelectLaunch& L, cudaStream_t stream) {
         sel_smem_set = sel_smem;
     }
     if (L.min_len <= kUnitLen) {
-        select_unit_kernel<<<units, kUnitThreads, kUnitSmem, stream>>>(p);
+        select_unit_kernel<<<units * (L.Hkv / L.n_vec), kUnitThreads, kUnitSmem, stream>>>(p);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
     if (L.max_len > kUnitLen) {
