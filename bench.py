@@ -46,6 +46,33 @@ SCORE_TRAFFIC = {
 SELECT_UNIT_LEN = 16384
 
 
+def _window_lse(q, k, cu_seqlens, w, Hq, Hkv):
+    """The window rows' lse, [Hq, S*w] fp32 natural log, as a prefill attention kernel returns
+    it: log sum_{j <= P+r} exp(q_r.k_j / sqrt(d)) (NaN for rows before the sequence start).
+    Plain PyTorch, for preparing the input of the given-lse path."""
+    import torch
+    S = len(cu_seqlens) - 1
+    G = Hq // Hkv
+    d = q.shape[-1]
+    out = torch.full((Hq, S * w), float("nan"), dtype=torch.float32, device=q.device)
+    for s in range(S):
+        t0, t1 = int(cu_seqlens[s]), int(cu_seqlens[s + 1])
+        L, P = t1 - t0, t1 - t0 - w
+        if L <= 0:
+            continue
+        for h in range(Hq):
+            qs = q[s, :, h].float()                       # [w, d]
+            ks = k[t0:t1, h // G].float()                 # [L, d]
+            logits = (qs @ ks.T) / (d ** 0.5)            # [w, L]
+            j = torch.arange(L, device=q.device)[None, :]
+            r = torch.arange(w, device=q.device)[:, None]
+            logits = logits.masked_fill(j > P + r, float("-inf"))
+            lse = torch.logsumexp(logits, dim=1)
+            lse[P + torch.arange(w, device=q.device) < 0] = float("nan")
+            out[h, s * w:(s + 1) * w] = lse
+    return out
+
+
 def _args():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -60,6 +87,9 @@ def _args():
     ap.add_argument("--score-path", choices=("auto", "resident", "reload"), default="auto",
                     help="scoring kernel: logits kept in TMEM, K re-read in pass 2, or the "
                          "library's choice")
+    ap.add_argument("--lse", action="store_true",
+                    help="the window rows' lse given (as a prefill attention kernel returns it): "
+                         "ckv_compress_layer_lse / ckv_score_window_lse, one pass over K")
     ap.add_argument("--max-ctas", type=int, default=0,
                     help="CTAs one call's scoring kernel may occupy (0 = SMs / 16, so that 16 "
                          "layers' scoring kernels are resident at once)")
@@ -181,6 +211,9 @@ def run_ours(args):
         idx, cu_keep_dev, k_out, v_out, cu_keep = ckv.new_outputs(cfg, l, batch)
         layers.append(dict(q=dev(li.q_win), k=dev(li.k), v=dev(li.v), idx=idx, cu_keep_dev=cu_keep_dev,
                            k_out=k_out, v_out=v_out, t_keep=int(cu_keep[-1])))
+        if args.lse:  # input preparation, outside every timed region
+            layers[-1]["lse"] = _window_lse(layers[-1]["q"], layers[-1]["k"], wl.cu_seqlens(), wl.window,
+                                            wl.num_q_heads, Hkv)
     ws_bytes = max(ckv.ckv_workspace_size(cfg, l, batch) for l in range(nl))
     # Layers are independent: by default each gets its own stream, and each call's scoring
     # kernel is capped at SMs / 16 CTAs, so that 16 of them are resident at once while the
@@ -204,10 +237,16 @@ def run_ours(args):
         for sd in side:
             stream.wait_stream(sd)
 
+    def compress(l, d, w, st):
+        if args.lse:
+            ckv.ckv_compress_layer_lse(cfg, l, batch, d["q"], d["k"], d["v"], d["lse"], d["idx"],
+                                       d["cu_keep_dev"], d["k_out"], d["v_out"], w, stream=st)
+        else:
+            ckv.ckv_compress_layer(cfg, l, batch, d["q"], d["k"], d["v"], d["idx"], d["cu_keep_dev"],
+                                   d["k_out"], d["v_out"], w, stream=st)
+
     def step():
-        over_layers(lambda l, d, w, st: ckv.ckv_compress_layer(
-            cfg, l, batch, d["q"], d["k"], d["v"], d["idx"], d["cu_keep_dev"], d["k_out"],
-            d["v_out"], w, stream=st))
+        over_layers(compress)
 
     with torch.cuda.stream(stream):
         for _ in range(max(1, args.warmup)):
@@ -287,9 +326,14 @@ def run_ours(args):
         torch.cuda.synchronize()
         return a.elapsed_time(b) / reps / nl  # ms per layer
 
+    def score_one(l, d, w, st):
+        if args.lse:
+            ckv.ckv_score_window_lse(cfg, l, batch, d["q"], d["k"], d["lse"], score_rows[l], w, stream=st)
+        else:
+            ckv.ckv_score_window(cfg, l, batch, d["q"], d["k"], score_rows[l], w, stream=st)
+
     def score_all():
-        over_layers(lambda l, d, w, st: ckv.ckv_score_window(cfg, l, batch, d["q"], d["k"],
-                                                             score_rows[l], w, stream=st))
+        over_layers(score_one)
 
     score_ms = stage(score_all)
     if args.breakdown:
@@ -317,7 +361,7 @@ def run_ours(args):
     digest = hashlib.sha256()
     for f in SCORE_SOURCES:
         digest.update(open(os.path.join(ROOT, "paper_2508_02401_gb300", "csrc", f), "rb").read())
-    traffic = SCORE_TRAFFIC.get(digest.hexdigest(), {}).get(args.workload)
+    traffic = SCORE_TRAFFIC.get(digest.hexdigest(), {}).get(args.workload + ("+lse" if args.lse else ""))
     roofline = {"bound": "hbm", "kernel": "scoring kernel (ckv_score_window), per layer, layers "
                                           f"overlapped on {nstreams} streams, {cap} CTAs per call",
                 "achieved": round(score_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
@@ -334,10 +378,11 @@ def run_ours(args):
         hq = [torch.from_numpy(h.q_win.view(np.int16)).view(torch.bfloat16).pin_memory() for h in host_layers]
         hk = [torch.from_numpy(h.k.view(np.int16)).view(torch.bfloat16).pin_memory() for h in host_layers]
         hv = [torch.from_numpy(h.v.view(np.int16)).view(torch.bfloat16).pin_memory() for h in host_layers]
+        hl = [d["lse"].cpu().pin_memory() for d in layers] if args.lse else []
         oi = [torch.empty(d["idx"].shape, dtype=torch.int32, pin_memory=True) for d in layers]
         ok = [torch.empty(d["k_out"].shape, dtype=torch.bfloat16, pin_memory=True) for d in layers]
         ov = [torch.empty(d["v_out"].shape, dtype=torch.bfloat16, pin_memory=True) for d in layers]
-        h2d = sum(x.numel() * 2 for x in hq + hk + hv)
+        h2d = sum(x.numel() * 2 for x in hq + hk + hv) + sum(x.numel() * 4 for x in hl)
         d2h = sum(x.numel() * x.element_size() for x in oi + ok + ov)
 
         def e2e_step():
@@ -345,8 +390,9 @@ def run_ours(args):
                 d["q"].copy_(hq[l], non_blocking=True)
                 d["k"].copy_(hk[l], non_blocking=True)
                 d["v"].copy_(hv[l], non_blocking=True)
-                ckv.ckv_compress_layer(cfg, l, batch, d["q"], d["k"], d["v"], d["idx"],
-                                       d["cu_keep_dev"], d["k_out"], d["v_out"], ws, stream=stream)
+                if args.lse:
+                    d["lse"].copy_(hl[l], non_blocking=True)
+                compress(l, d, ws, stream)
                 oi[l].copy_(d["idx"], non_blocking=True)
                 ok[l].copy_(d["k_out"], non_blocking=True)
                 ov[l].copy_(d["v_out"], non_blocking=True)
@@ -381,7 +427,9 @@ def run_ours(args):
                        "budget_total": int(wl.budgets().sum()), "parallelism": f"replicas{world}",
                        "l2": "inputs larger than L2 (distinct per-layer buffers, 1.07 GB per step)",
                        "graph": "one CUDA graph per step",
-                       "streams": f"layers round-robin on {nstreams} streams, scoring capped at {cap} CTAs per call"},
+                       "streams": f"layers round-robin on {nstreams} streams, scoring capped at {cap} CTAs per call",
+                       "lse": ("window-row lse given (PyTorch logsumexp outside the timed region; "
+                               "one pass over K)") if args.lse else "computed (two passes)"},
             "roofline": roofline,
             "layer_roofline": {"bound": "hbm", "achieved": round(layer_gbs, 1), "peak": hbm_peak,
                                "unit": "GB/s", "frac": round(layer_gbs / hbm_peak, 4),

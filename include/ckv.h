@@ -162,6 +162,22 @@ CKV_API ckv_status ckv_score_window(const ckv_config* cfg, int32_t layer, const 
                             int64_t head_stride, float* scores, void* workspace,
                             size_t workspace_bytes, ckv_stream stream);
 
+/* Step 1 with the window rows' normalisers given (the log-sum-exp that a prefill attention
+ * kernel returns per query row): the same scores as ckv_score_window, with lse_{h,r} read
+ * instead of computed, so K is read and multiplied once and no CTA waits for another.
+ *   lse: device fp32, natural log of sum_{j <= P+r} exp(scale * q_{h,r}.k_j) for query head
+ *        h and window row r of sequence s at lse[h * lse_head_stride + s * w + r] (the layout
+ *        of a varlen prefill's per-head lse over the window rows); lse_head_stride >= S * w,
+ *        0 selects S * w.  Only the selected heads' rows are read, and rows whose query
+ *        position is before the sequence start (L < w) are not read.  4-byte aligned.
+ * The result is exact for the true lse; any other value scales row r's probabilities by
+ * exp(lse_true - lse_given). */
+CKV_API ckv_status ckv_score_window_lse(const ckv_config* cfg, int32_t layer,
+                                        const ckv_batch* batch, const void* q_win, const void* k,
+                                        int64_t tok_stride, int64_t head_stride, const float* lse,
+                                        int64_t lse_head_stride, float* scores, void* workspace,
+                                        size_t workspace_bytes, ckv_stream stream);
+
 /* Step 2 (Sec. 3.3 token-axis smoothing; App. A sizes): pooled[g, cu[s]+j] for
  * j < L_s - w from the scores of selection g's heads (group g's selected heads, or every
  * selected head of the layer with CKV_SCOPE_LAYER), in cfg->head_order; 0 at window positions.
@@ -193,6 +209,16 @@ CKV_API ckv_status ckv_compress_layer(const ckv_config* cfg, int32_t layer, cons
                               int64_t tok_stride, int64_t head_stride, int32_t* idx,
                               int32_t* cu_keep_dev, void* k_out, void* v_out, float* pooled_out,
                               void* workspace, size_t workspace_bytes, ckv_stream stream);
+
+/* ckv_compress_layer with the window rows' lse given (layout as in ckv_score_window_lse). */
+CKV_API ckv_status ckv_compress_layer_lse(const ckv_config* cfg, int32_t layer,
+                                          const ckv_batch* batch, const void* q_win,
+                                          const void* k, const void* v, int64_t tok_stride,
+                                          int64_t head_stride, const float* lse,
+                                          int64_t lse_head_stride, int32_t* idx,
+                                          int32_t* cu_keep_dev, void* k_out, void* v_out,
+                                          float* pooled_out, void* workspace,
+                                          size_t workspace_bytes, ckv_stream stream);
 
 /* Layer budgets (App. B, the paper's error-aware layer-adaptive allocation).  Host only; no
  * GPU is needed.

@@ -44,9 +44,11 @@ def _load():
         lib.ckv_oracle_pool.argtypes = [P, C.c_int, C.c_int, C.c_int, P]
         lib.ckv_oracle_topk.argtypes = [P, C.c_int, C.c_int, P]
         lib.ckv_oracle_keep_lengths.argtypes = [C.c_int, P, C.c_int, P]
+        lib.ckv_oracle_window_scores_lse.argtypes = [C.c_int, C.c_int, C.c_int, C.c_double, P,
+                                                     C.c_long, P, C.c_long, P, P]
         lib.ckv_oracle_compress_layer.argtypes = [
             C.c_int, P, C.c_int, C.c_int, C.c_int, C.c_int, C.c_double, P, C.c_int,
-            C.c_int, C.c_int, C.c_int, C.c_int, P, P, P, P, P, P, P, P, P, P, C.c_int]
+            C.c_int, C.c_int, C.c_int, C.c_int, P, P, P, P, C.c_long, P, P, P, P, P, P, P, C.c_int]
         lib.ckv_oracle_threads.argtypes = [C.c_int]
         _lib = lib
     return _lib
@@ -83,6 +85,22 @@ def window_scores(q_rows: np.ndarray, k_rows: np.ndarray, scale: float | None = 
     return a, lse, mass
 
 
+def window_scores_lse(q_rows: np.ndarray, k_rows: np.ndarray, lse: np.ndarray,
+                      scale: float | None = None) -> np.ndarray:
+    """Window scores of one head with the rows' normalisers given (lse [w], natural log):
+    a [L] = sum over the rows that see key j of exp(s - lse_r)."""
+    q = np.ascontiguousarray(q_rows, dtype=np.uint16)
+    k = np.ascontiguousarray(k_rows, dtype=np.uint16)
+    lse = np.ascontiguousarray(lse, dtype=np.float64)
+    w, d = q.shape
+    L = k.shape[0]
+    assert lse.shape == (w,)
+    scale = 1.0 / np.sqrt(d) if scale is None else scale
+    a = np.empty(L, np.float64)
+    _check(_load().ckv_oracle_window_scores_lse(L, w, d, float(scale), _p(q), d, _p(k), d, _p(lse), _p(a)))
+    return a
+
+
 def pool(x: np.ndarray, kernel: int, pool_type: int) -> np.ndarray:
     x = np.ascontiguousarray(x, dtype=np.float64)
     y = np.empty_like(x)
@@ -109,7 +127,7 @@ SCOPE_KV_HEAD, SCOPE_LAYER = 0, 1
 
 def compress_layer(q_win, k, v, cu_seqlens, head_mask, budget, window, pool_kernel, pool_type,
                    head_order, scale=None, want_scores=True, want_kv=True, groups=None,
-                   num_threads=0, scope=SCOPE_KV_HEAD):
+                   num_threads=0, scope=SCOPE_KV_HEAD, lse=None):
     """One layer of the compression step.  Arrays are bf16 bits (uint16), packed.
 
     q_win [S, w, Hq, d], k/v [T, Hkv, d], cu_seqlens [S+1], head_mask [Hq] (uint8).
@@ -117,6 +135,8 @@ def compress_layer(q_win, k, v, cu_seqlens, head_mask, budget, window, pool_kern
     scope=SCOPE_LAYER), cu_keep [S+1], idx [Hkv, T_keep] (int32), k_out / v_out
     [T_keep, Hkv, d] (uint16).  ``groups`` (optional iterable of KV heads, KV-head scope only)
     restricts the work to those groups; rows of the other groups are left as NaN / -1.
+    ``lse`` (optional, [Hq, S*w] float64, natural log): the window rows' normalisers, used
+    instead of computing them.
     """
     q_win = np.ascontiguousarray(q_win, dtype=np.uint16)
     k = np.ascontiguousarray(k, dtype=np.uint16)
@@ -140,8 +160,14 @@ def compress_layer(q_win, k, v, cu_seqlens, head_mask, budget, window, pool_kern
     if groups is not None:
         gf = np.zeros(Hkv, np.uint8)
         gf[list(groups)] = 1
+    lse_arr, lse_stride = None, 0
+    if lse is not None:
+        lse_arr = np.ascontiguousarray(lse, dtype=np.float64)
+        assert lse_arr.ndim == 2 and lse_arr.shape[0] == Hq and lse_arr.shape[1] >= S * window
+        lse_stride = lse_arr.shape[1]
     _check(_load().ckv_oracle_compress_layer(
         S, _p(cu), Hq, Hkv, d, window, float(scale), _p(mask), int(budget), int(pool_kernel),
-        int(pool_type), int(head_order), int(scope), _p(q_win), _p(k), _p(v), _p(scores), _p(pooled),
-        None, _p(idx), _p(k_out), _p(v_out), _p(gf), int(num_threads)))
+        int(pool_type), int(head_order), int(scope), _p(q_win), _p(k), _p(v), _p(lse_arr),
+        int(lse_stride), _p(scores), _p(pooled), None, _p(idx), _p(k_out), _p(v_out), _p(gf),
+        int(num_threads)))
     return dict(scores=scores, pooled=pooled, cu_keep=cu_keep, idx=idx, k_out=k_out, v_out=v_out)

@@ -105,6 +105,33 @@ int ckv_oracle_window_scores(int L, int w, int d, double scale,
 }
 
 /*
+ * The same window scores with the rows' normalisers given (lse_in[r], natural log), as a
+ * prefill attention kernel returns them for its query rows (Sec. 3.3 with Eq. 2):
+ *   a[j] = sum over rows r that see key j of exp(s_{r,j} - lse_in[r]).
+ * Rows whose query position is negative (L < w) contribute nothing and lse_in[r] is not read.
+ */
+int ckv_oracle_window_scores_lse(int L, int w, int d, double scale,
+                                 const uint16_t* q, long q_row_stride,
+                                 const uint16_t* k, long k_row_stride,
+                                 const double* lse_in, double* a) {
+    if (L < 0 || w < 1 || d < 1 || !lse_in) return ORACLE_BAD_ARG;
+    int P = L - w;
+    for (int j = 0; j < L; ++j) a[j] = 0.0;
+    for (int r = 0; r < w; ++r) {
+        int qpos = P + r;
+        if (qpos < 0) continue;
+        const uint16_t* qr = q + (long)r * q_row_stride;
+        for (int j = 0; j <= qpos; ++j) {
+            const uint16_t* kj = k + (long)j * k_row_stride;
+            double dot = 0.0;
+            for (int c = 0; c < d; ++c) dot += widen_bf16(qr[c]) * widen_bf16(kj[c]);
+            a[j] += exp(scale * dot - lse_in[r]);
+        }
+    }
+    return ORACLE_OK;
+}
+
+/*
  * 1-D pooling along the token axis (Sec. 3.3; App. A uses kernel 5 with average pooling).
  * Stride 1, output length n, window [j - kernel/2, j + kernel/2] clipped to [0, n).
  *   type 0 (max): maximum over the clipped window (padded cells ignored);
@@ -201,11 +228,14 @@ int ckv_oracle_keep_lengths(int S, const int32_t* cu_seqlens, int budget, int32_
  * sequence from every selected head of the layer (each head against its own group's keys);
  * the index set is repeated for every KV head and each KV head's rows are gathered with it.
  * pooled has Hkv rows (scope 0) or 1 row (scope 1); idx and the outputs have Hkv rows.
+ * lse_in (optional): the window rows' normalisers, lse_in[h * lse_head_stride + s * w + r]
+ * (natural log), used instead of computing them (ckv_oracle_window_scores_lse).
  */
 int ckv_oracle_compress_layer(int S, const int32_t* cu_seqlens, int Hq, int Hkv, int d, int w,
                               double scale, const uint8_t* head_mask, int budget,
                               int pool_kernel, int pool_type, int head_order, int scope,
                               const uint16_t* q_win, const uint16_t* k, const uint16_t* v,
+                              const double* lse_in, long lse_head_stride,
                               double* scores, double* pooled, int32_t* cu_keep, int32_t* idx,
                               uint16_t* k_out, uint16_t* v_out, const uint8_t* group_filter,
                               int num_threads) {
@@ -273,8 +303,13 @@ int ckv_oracle_compress_layer(int S, const int32_t* cu_seqlens, int Hq, int Hkv,
             if (!head_mask[h]) continue;
             const uint16_t* qh = q_win + ((long)s * w * Hq + h) * d;
             const uint16_t* kg = k + ((long)t0 * Hkv + h / G) * d; /* the head's own KV group */
-            if (ckv_oracle_window_scores(L, w, d, scale, qh, (long)Hq * d, kg, (long)Hkv * d,
-                                         a, lse, mass)) {
+            const int ws_rc =
+                lse_in ? ckv_oracle_window_scores_lse(L, w, d, scale, qh, (long)Hq * d, kg,
+                                                      (long)Hkv * d,
+                                                      lse_in + (long)h * lse_head_stride + (long)s * w, a)
+                       : ckv_oracle_window_scores(L, w, d, scale, qh, (long)Hq * d, kg, (long)Hkv * d,
+                                                  a, lse, mass);
+            if (ws_rc) {
                 failed |= 1;
                 continue;
             }

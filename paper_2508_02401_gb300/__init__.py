@@ -83,6 +83,9 @@ def load():
         "ckv_compress_layer": ([cfg, I32, bat, P, P, P, I64, I64, P, P, P, P, P, P, SZ, P], C.c_int),
         "ckv_read_device_status": ([P, P, I32, C.POINTER(I32), C.POINTER(I32)], C.c_int),
         "ckv_score_window_static": ([cfg, I32, bat, P, P, I64, I64, P, P, P], C.c_int),
+        "ckv_score_window_lse": ([cfg, I32, bat, P, P, I64, I64, P, I64, P, P, SZ, P], C.c_int),
+        "ckv_compress_layer_lse": ([cfg, I32, bat, P, P, P, I64, I64, P, I64, P, P, P, P, P, P, SZ, P],
+                                   C.c_int),
         "ckv_layer_error_scores": ([P, I32, I32, P], C.c_int),
         "ckv_set_wait_limit_us": ([C.c_uint32], C.c_int),
         "ckv_allocate_budgets": ([P, I32, I64, I32, I32, P], C.c_int),
@@ -269,6 +272,27 @@ def ckv_compress_layer(cfg, layer, batch, q_win, k, v, idx, cu_keep_dev, k_out, 
                                      _ptr(k_out), _ptr(v_out), _ptr(pooled_out), _ptr(workspace),
                                      workspace.numel() * workspace.element_size(), _stream(stream)),
            "ckv_compress_layer")
+
+
+def ckv_score_window_lse(cfg, layer, batch, q_win, k, lse, scores, workspace, lse_head_stride=0,
+                         stream=None, tok_stride=0, head_stride=0):
+    """ckv_score_window with the window rows' lse given: lse [H_q, >= S*w] fp32 natural log."""
+    _check(load().ckv_score_window_lse(cfg.ref, layer, batch.ref, _ptr(q_win), _ptr(k), tok_stride,
+                                       head_stride, _ptr(lse), lse_head_stride, _ptr(scores),
+                                       _ptr(workspace), workspace.numel() * workspace.element_size(),
+                                       _stream(stream)), "ckv_score_window_lse")
+
+
+def ckv_compress_layer_lse(cfg, layer, batch, q_win, k, v, lse, idx, cu_keep_dev, k_out, v_out,
+                           workspace, lse_head_stride=0, pooled_out=None, stream=None, tok_stride=0,
+                           head_stride=0):
+    """ckv_compress_layer with the window rows' lse given (layout as ckv_score_window_lse)."""
+    _check(load().ckv_compress_layer_lse(cfg.ref, layer, batch.ref, _ptr(q_win), _ptr(k), _ptr(v),
+                                         tok_stride, head_stride, _ptr(lse), lse_head_stride,
+                                         _ptr(idx), _ptr(cu_keep_dev), _ptr(k_out), _ptr(v_out),
+                                         _ptr(pooled_out), _ptr(workspace),
+                                         workspace.numel() * workspace.element_size(), _stream(stream)),
+           "ckv_compress_layer_lse")
 
 
 def ckv_score_window_static(cfg, layer, batch, q_win, k, scores, status_out=None, stream=None,

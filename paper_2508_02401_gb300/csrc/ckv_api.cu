@@ -301,6 +301,101 @@ ckv_status plan_score(const Plan& pl, const ckv_batch* b, int skip_le, int ctas,
     return CKV_OK;
 }
 
+// Work of the single-pass kernel (window-row lse given): no exchange between CTAs, so the key
+// tiles of all (sequence, head batch) units, taken in order, are cut into `grid` runs of
+// (nearly) equal length, one per CTA; a run that crosses units becomes one item per unit.
+// Round r of the item table holds every CTA's r-th item.
+ckv_status plan_score_stream(const Plan& pl, const ckv_batch* b, int skip_le, int ctas, ScoreLaunch& L,
+                             int max_items_per_launch) {
+    struct RawUnit {
+        int seq, start, len, batch, tiles;
+    };
+    std::vector<RawUnit> raw;
+    int64_t total = 0;
+    for (int s = 0; s < b->num_seqs; ++s) {
+        const int t0 = b->cu_seqlens_host[s];
+        const int len = b->cu_seqlens_host[s + 1] - t0;
+        if (len <= skip_le || len <= 0) continue;
+        const int tiles = (len + kTileKeys - 1) / kTileKeys;
+        for (int bt = 0; bt < pl.nb; ++bt) {
+            raw.push_back({s, t0, len, bt, tiles});
+            total += tiles;
+        }
+    }
+    L.items.clear();
+    L.units.clear();
+    L.slices.clear();
+    L.resident = false;
+    if (raw.empty()) return CKV_OK;
+    if (b->num_seqs > 65535) return fail(CKV_ERR_UNSUPPORTED, "more than 65535 sequences");
+    const int grid = static_cast<int>(std::min<int64_t>(ctas, total));
+    const int64_t per = (total + grid - 1) / grid;
+    if (per > 65535) return fail(CKV_ERR_UNSUPPORTED, "more than 65535 key tiles per CTA");
+    struct Run {
+        int raw;         // index into raw
+        ScoreItem item;  // unit filled in per slice
+    };
+    std::vector<std::vector<Run>> runs(grid);
+    int cta = 0;
+    int64_t filled = 0;
+    for (int ui = 0; ui < static_cast<int>(raw.size()); ++ui) {
+        for (int t = 0; t < raw[ui].tiles;) {
+            const int take = static_cast<int>(std::min<int64_t>(raw[ui].tiles - t, per - filled));
+            runs[cta].push_back({ui, ScoreItem{0, static_cast<uint16_t>(take), static_cast<uint32_t>(t)}});
+            t += take;
+            filled += take;
+            if (filled == per && cta + 1 < grid) {
+                ++cta;
+                filled = 0;
+            }
+        }
+    }
+    size_t rounds = 0;
+    for (const auto& r : runs) rounds = std::max(rounds, r.size());
+    L.grid = grid;
+    const int max_rounds = std::max(1, max_items_per_launch / grid);
+    std::vector<int> local(raw.size(), -1);
+    size_t r = 0;
+    while (r < rounds) {
+        ScoreSlice sl{static_cast<int>(L.items.size()), 0, static_cast<int>(L.units.size()), 0};
+        std::vector<int> used;
+        while (r < rounds && sl.n_rounds < max_rounds) {
+            int fresh = 0;
+            for (int c = 0; c < grid; ++c)
+                if (r < runs[c].size() && local[runs[c][r].raw] < 0) ++fresh;  // an upper bound
+            if (sl.n_rounds > 0 && sl.n_units + fresh > kMaxScoreUnits) break;
+            for (int c = 0; c < grid; ++c) {
+                ScoreItem it{0, 0, 0};
+                if (r < runs[c].size()) {
+                    const int ui = runs[c][r].raw;
+                    if (local[ui] < 0) {
+                        if (sl.n_units >= kMaxScoreUnits)
+                            return fail(CKV_ERR_UNSUPPORTED, "too many scoring units in a round");
+                        local[ui] = sl.n_units++;
+                        used.push_back(ui);
+                        ScoreUnit su;
+                        su.seq_start = raw[ui].start;
+                        su.len = raw[ui].len;
+                        su.seq = static_cast<uint16_t>(raw[ui].seq);
+                        su.batch = static_cast<uint16_t>(raw[ui].batch);
+                        su.first_item = 0;  // no exchange: unused
+                        su.nitems = 0;
+                        L.units.push_back(su);
+                    }
+                    it = runs[c][r].item;
+                    it.unit = static_cast<uint16_t>(local[ui]);
+                }
+                L.items.push_back(it);
+            }
+            ++sl.n_rounds;
+            ++r;
+        }
+        for (int ui : used) local[ui] = -1;
+        L.slices.push_back(sl);
+    }
+    return CKV_OK;
+}
+
 struct WsLayout {
     size_t header = 0, partials = 0, counters = 0, scores = 0, pooled = 0;
     size_t hist = 0, arrivals = 0, chunk_start = 0, buckets = 0, info = 0, chunk_off = 0, total = 0;
@@ -441,14 +536,19 @@ namespace {
 ckv_status enqueue_score(const Plan& pl, const ckv_batch* b, int T, const void* q_win,
                          const void* k, int64_t tok, int64_t head, float* scores, void* ws,
                          const WsLayout& l, int skip_le, cudaStream_t stream,
-                         int max_items_per_launch = kMaxScoreItems) {
+                         int max_items_per_launch = kMaxScoreItems, const float* lse = nullptr,
+                         int64_t lse_head_stride = 0) {
     int ctas = device_sm_count();
     if (ctas <= 0) return cuda_fail(cudaGetLastError(), "querying the SM count");
     if (pl.max_ctas > 0) ctas = std::min(ctas, pl.max_ctas);
     static thread_local ScoreLaunch L;  // reused: keeps the plan's vectors allocated
-    ckv_status st = plan_score(pl, b, skip_le, std::min(ctas, max_items_per_launch), L,
-                               max_items_per_launch);
+    ckv_status st = lse ? plan_score_stream(pl, b, skip_le, std::min(ctas, max_items_per_launch), L,
+                                            max_items_per_launch)
+                        : plan_score(pl, b, skip_le, std::min(ctas, max_items_per_launch), L,
+                                     max_items_per_launch);
     if (st) return st;
+    L.lse = lse;
+    L.lse_head_stride = lse_head_stride;
     if (L.slices.empty()) return CKV_OK;
     if ((st = make_k_map(&L.tmap_k, k, pl.Hkv, T, tok, head))) return st;
     if ((st = make_q_map(&L.tmap_q, q_win, pl.Hq, b->num_seqs, pl.w, pl.w_pad))) return st;
@@ -599,10 +699,26 @@ ckv_status ckv_keep_lengths(const ckv_config* cfg, int32_t layer, const ckv_batc
     return CKV_OK;
 }
 
-ckv_status ckv_score_window(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
-                            const void* q_win, const void* k, int64_t tok_stride,
-                            int64_t head_stride, float* scores, void* workspace,
-                            size_t workspace_bytes, ckv_stream stream) {
+}  // extern "C"
+
+namespace {
+
+// The given lse array: device, 4-byte aligned, [H_q][lse_head_stride] with lse_head_stride >= S*w
+// (0 selects S*w).
+ckv_status check_lse(const Plan& pl, const ckv_batch* b, const float* lse, int64_t* stride) {
+    if (!lse) return fail(CKV_ERR_INVALID_ARG, "lse is NULL");
+    if (!aligned(lse, 4)) return fail(CKV_ERR_INVALID_ARG, "lse is not 4-byte aligned");
+    const int64_t rows = static_cast<int64_t>(b->num_seqs) * pl.w;
+    if (*stride == 0) *stride = rows;
+    if (*stride < rows) return fail(CKV_ERR_INVALID_ARG, "lse_head_stride %lld < S*w", (long long)*stride);
+    return CKV_OK;
+}
+
+ckv_status score_window_impl(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
+                             const void* q_win, const void* k, int64_t tok_stride,
+                             int64_t head_stride, const float* lse, int64_t lse_head_stride,
+                             float* scores, void* workspace, size_t workspace_bytes,
+                             ckv_stream stream) {
     Plan pl;
     ckv_status st = make_plan(cfg, layer, pl);
     if (st) return st;
@@ -613,8 +729,31 @@ ckv_status ckv_score_window(const ckv_config* cfg, int32_t layer, const ckv_batc
         (st = check_kv(scores, "scores", T)) ||
         (st = check_ws(pl, batch, T, workspace, workspace_bytes, &l)))
         return st;
+    if (lse && (st = check_lse(pl, batch, lse, &lse_head_stride))) return st;
     return enqueue_score(pl, batch, T, q_win, k, tok_stride, head_stride, scores, workspace, l, -1,
-                         reinterpret_cast<cudaStream_t>(stream));
+                         reinterpret_cast<cudaStream_t>(stream), kMaxScoreItems, lse, lse_head_stride);
+}
+
+}  // namespace
+
+extern "C" {
+
+ckv_status ckv_score_window(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
+                            const void* q_win, const void* k, int64_t tok_stride,
+                            int64_t head_stride, float* scores, void* workspace,
+                            size_t workspace_bytes, ckv_stream stream) {
+    return score_window_impl(cfg, layer, batch, q_win, k, tok_stride, head_stride, nullptr, 0,
+                             scores, workspace, workspace_bytes, stream);
+}
+
+ckv_status ckv_score_window_lse(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
+                                const void* q_win, const void* k, int64_t tok_stride,
+                                int64_t head_stride, const float* lse, int64_t lse_head_stride,
+                                float* scores, void* workspace, size_t workspace_bytes,
+                                ckv_stream stream) {
+    if (!lse) return fail(CKV_ERR_INVALID_ARG, "lse is NULL");
+    return score_window_impl(cfg, layer, batch, q_win, k, tok_stride, head_stride, lse,
+                             lse_head_stride, scores, workspace, workspace_bytes, stream);
 }
 
 ckv_status ckv_pool(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
@@ -697,11 +836,16 @@ ckv_status ckv_gather_compact(const ckv_config* cfg, const ckv_batch* batch, int
     return e == cudaSuccess ? CKV_OK : cuda_fail(e, "launching the gather kernel");
 }
 
-ckv_status ckv_compress_layer(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
-                              const void* q_win, const void* k, const void* v,
-                              int64_t tok_stride, int64_t head_stride, int32_t* idx,
-                              int32_t* cu_keep_dev, void* k_out, void* v_out, float* pooled_out,
-                              void* workspace, size_t workspace_bytes, ckv_stream stream) {
+}  // extern "C"
+
+namespace {
+
+ckv_status compress_layer_impl(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
+                               const void* q_win, const void* k, const void* v,
+                               int64_t tok_stride, int64_t head_stride, const float* lse,
+                               int64_t lse_head_stride, int32_t* idx, int32_t* cu_keep_dev,
+                               void* k_out, void* v_out, float* pooled_out, void* workspace,
+                               size_t workspace_bytes, ckv_stream stream) {
     Plan pl;
     ckv_status st = make_plan(cfg, layer, pl);
     if (st) return st;
@@ -713,6 +857,7 @@ ckv_status ckv_compress_layer(const ckv_config* cfg, int32_t layer, const ckv_ba
         return st;
     if (pooled_out && !aligned(pooled_out, 16))
         return fail(CKV_ERR_INVALID_ARG, "pooled_out is not 16-byte aligned");
+    if (lse && (st = check_lse(pl, batch, lse, &lse_head_stride))) return st;
     const int64_t tk = keep_total(batch, pl.budget);
     if (tk > INT32_MAX) return fail(CKV_ERR_UNSUPPORTED, "too many kept tokens");
     if (!cu_keep_dev) return fail(CKV_ERR_INVALID_ARG, "cu_keep_dev is NULL");
@@ -725,7 +870,7 @@ ckv_status ckv_compress_layer(const ckv_config* cfg, int32_t layer, const ckv_ba
     float* pooled = pooled_out ? pooled_out : reinterpret_cast<float*>(w8 + l.pooled);
     const int skip_le = pl.budget;  // sequences that fit the budget are kept whole
     if ((st = enqueue_score(pl, batch, T, q_win, k, tok_stride, head_stride, scores, workspace, l,
-                            skip_le, s)))
+                            skip_le, s, kMaxScoreItems, lse, lse_head_stride)))
         return st;
     SelectLaunch L = select_launch(pl, batch, T, static_cast<int>(tk), skip_le, cfg, workspace, &l);
     L.scores = scores;
@@ -744,6 +889,32 @@ ckv_status ckv_compress_layer(const ckv_config* cfg, int32_t layer, const ckv_ba
     }
     const cudaError_t e = launch_select(L, s);
     return e == cudaSuccess ? CKV_OK : cuda_fail(e, "launching the pool, selection and gather kernels");
+}
+
+}  // namespace
+
+extern "C" {
+
+ckv_status ckv_compress_layer(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
+                              const void* q_win, const void* k, const void* v,
+                              int64_t tok_stride, int64_t head_stride, int32_t* idx,
+                              int32_t* cu_keep_dev, void* k_out, void* v_out, float* pooled_out,
+                              void* workspace, size_t workspace_bytes, ckv_stream stream) {
+    return compress_layer_impl(cfg, layer, batch, q_win, k, v, tok_stride, head_stride, nullptr, 0,
+                               idx, cu_keep_dev, k_out, v_out, pooled_out, workspace,
+                               workspace_bytes, stream);
+}
+
+ckv_status ckv_compress_layer_lse(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
+                                  const void* q_win, const void* k, const void* v,
+                                  int64_t tok_stride, int64_t head_stride, const float* lse,
+                                  int64_t lse_head_stride, int32_t* idx, int32_t* cu_keep_dev,
+                                  void* k_out, void* v_out, float* pooled_out, void* workspace,
+                                  size_t workspace_bytes, ckv_stream stream) {
+    if (!lse) return fail(CKV_ERR_INVALID_ARG, "lse is NULL");
+    return compress_layer_impl(cfg, layer, batch, q_win, k, v, tok_stride, head_stride, lse,
+                               lse_head_stride, idx, cu_keep_dev, k_out, v_out, pooled_out,
+                               workspace, workspace_bytes, stream);
 }
 
 ckv_status ckv_read_device_status(void* workspace, ckv_stream stream, int32_t reset,

@@ -48,6 +48,8 @@ struct ScoreLaunch {
     int nb;                // head batches
     int grid;              // CTAs (= items per round)
     bool resident;         // score_resident.cu (logits kept in TMEM) instead of score_kernel.cu
+    const float* lse;      // given window-row lse [Hq][lse_head_stride] (score_lse.cu), or null
+    int64_t lse_head_stride;
     uint32_t cu_hash;      // seqlens_hash of the host copy of cu_seqlens
     float softmax_scale;
     int n_sel;

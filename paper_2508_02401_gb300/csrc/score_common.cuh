@@ -30,6 +30,8 @@ struct alignas(128) ScoreParams {
     uint32_t cu_hash;
     float sl2;                     // softmax scale * log2(e)
     long long wait_cycles;         // limit of a bounded wait (ckv_set_wait_limit_us)
+    const float* lse;              // given lse of the window rows (natural log), [Hq][lse_stride]
+    long long lse_stride;
     int16_t batch_group[kMaxBatches];   // KV head of each head batch
     int16_t batch_first[kMaxBatches];   // score row of the batch's first head
     int16_t batch_nheads[kMaxBatches];  // heads in the batch
@@ -410,5 +412,7 @@ __device__ __forceinline__ bool unit_lse(const ScoreParams& p, const ScoreUnit& 
 
 // Resident variant (score_resident.cu): launch of one (N, W_PAD) instance.
 cudaError_t launch_resident(const ScoreParams& p, int n_cols, int w_pad, int grid, cudaStream_t st);
+// Single pass with the rows' lse given (score_lse.cu).
+cudaError_t launch_given_lse(const ScoreParams& p, int n_cols, int w_pad, int grid, cudaStream_t st);
 
 }  // namespace ckv

@@ -587,6 +587,8 @@ cudaError_t launch_score(const ScoreLaunch& L, cudaStream_t stream) {
     p.cu_hash = L.cu_hash;
     p.sl2 = L.softmax_scale * 1.4426950408889634f;
     p.wait_cycles = wait_limit_cycles();
+    p.lse = L.lse;
+    p.lse_stride = L.lse_head_stride;
     for (int b = 0; b < L.nb; ++b) {
         p.batch_group[b] = static_cast<int16_t>(L.batch_group[b]);
         p.batch_first[b] = static_cast<int16_t>(L.batch_first[b]);
@@ -600,10 +602,14 @@ cudaError_t launch_score(const ScoreLaunch& L, cudaStream_t stream) {
         p.n_units = sl.n_units;
         memcpy(p.items, L.items.data() + sl.item0, sizeof(ScoreItem) * p.n_items);
         memcpy(p.units, L.units.data() + sl.unit0, sizeof(ScoreUnit) * p.n_units);
-        cudaError_t e = cudaMemsetAsync(L.counters, 0, sizeof(int) * sl.n_units, stream);
-        if (e != cudaSuccess) return e;
-        e = L.resident ? launch_resident(p, L.n_cols, L.w_pad, L.grid, stream)
-                       : dispatch(p, L.n_cols, L.w_pad, L.grid, stream);
+        cudaError_t e = cudaSuccess;
+        if (!L.lse) {  // the unit arrival counters of the exchange
+            e = cudaMemsetAsync(L.counters, 0, sizeof(int) * sl.n_units, stream);
+            if (e != cudaSuccess) return e;
+        }
+        e = L.lse ? launch_given_lse(p, L.n_cols, L.w_pad, L.grid, stream)
+            : L.resident ? launch_resident(p, L.n_cols, L.w_pad, L.grid, stream)
+                         : dispatch(p, L.n_cols, L.w_pad, L.grid, stream);
         if (e != cudaSuccess) return e;
     }
     return cudaSuccess;
