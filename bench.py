@@ -35,11 +35,15 @@ HBM_FALLBACK_GBS = 6800.0
 
 # DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) of one scoring launch (one layer)
 # per workload, from the ncu captures summarised in profiles/ (score_kernel_llama8b_l8192.md,
-# score_resident_paper_llama8b_l8192.md), keyed by the sha256 of the scoring kernels' sources
-# (SCORE_SOURCES); a changed kernel reports null until it is captured again.
-SCORE_SOURCES = ('score_kernel.cu', 'score_resident.cu', 'score_common.cuh', 'ckv_device.cuh')
+# score_resident_paper_llama8b_l8192.md, score_lse_llama8b_l8192.md; "+lse": bench.py --lse),
+# keyed by the sha256 of the scoring kernels' sources (SCORE_SOURCES); a changed kernel reports
+# null until it is captured again.
+SCORE_SOURCES = ('score_kernel.cu', 'score_resident.cu', 'score_lse.cu', 'score_common.cuh', 'ckv_device.cuh')
 SCORE_TRAFFIC = {
-    "0e24b44d442cf1e6c618608c61b1ead13c09ab6100d6d702e76236f3f28d9b31": {"llama8b_l8192": 16987904, "paper_llama8b_l8192": 8488704},
+    "e2ce6dd503dbedaf76fb38d0c48061e120265a4a3cee04f9733c613831effc5e": {
+        "llama8b_l8192": 16987904, "paper_llama8b_l8192": 8488704,
+        "llama8b_l8192+lse": 16948736, "needle_l131072+lse": 274966272,
+    },
 }
 # Sequences up to this many tokens are selected by one block per (sequence, KV head)
 # (one launch); longer ones by the chunked kernels (two launches).
