@@ -220,6 +220,27 @@ CKV_API ckv_status ckv_compress_layer_lse(const ckv_config* cfg, int32_t layer,
                                           float* pooled_out, void* workspace,
                                           size_t workspace_bytes, ckv_stream stream);
 
+/* Semantic Retrieval Score accumulation (Sec. 3.2, Eq. 5), the offline step that picks the
+ * heads: srs[h] += sum over decode steps t whose generated token is in the answer span A of
+ * sum_{j in A} a^h_{t,j}, for the layer's selected heads h (an all-ones head mask scores every
+ * head).  Per sequence s of the batch (one profiling prompt each):
+ *   k      [T, H_kv, d]: the context followed by the w generated tokens' keys; decode step t
+ *          (t < w = cfg->window) attends to keys 0..L_s-w+t (itself included);
+ *   q_dec  [S, w, H_q, d]: the decode steps' queries, laid out like q_win;
+ *   lse    the decode rows' lse (natural log), layout as in ckv_score_window_lse;
+ *   in_answer  device uint8 [S*w]: nonzero where step t's generated token is in A;
+ *   span   device int32 [S][2]: A = positions [a0, a1) of the sequence (a span outside
+ *          [0, L_s) is reported in the status word, kind 3, and skipped);
+ *   srs    device fp32 [H_q], accumulated (+=) so that calls over prompts and layers add up.
+ * The workspace is ckv_workspace_size's. */
+CKV_API ckv_status ckv_semantic_retrieval_scores(const ckv_config* cfg, int32_t layer,
+                                                 const ckv_batch* batch, const void* q_dec,
+                                                 const void* k, int64_t tok_stride,
+                                                 int64_t head_stride, const float* lse,
+                                                 int64_t lse_head_stride, const uint8_t* in_answer,
+                                                 const int32_t* span, float* srs, void* workspace,
+                                                 size_t workspace_bytes, ckv_stream stream);
+
 /* Layer budgets (App. B, the paper's error-aware layer-adaptive allocation).  Host only; no
  * GPU is needed.
  *

@@ -49,6 +49,8 @@ def _load():
         lib.ckv_oracle_compress_layer.argtypes = [
             C.c_int, P, C.c_int, C.c_int, C.c_int, C.c_int, C.c_double, P, C.c_int,
             C.c_int, C.c_int, C.c_int, C.c_int, P, P, P, P, C.c_long, P, P, P, P, P, P, P, C.c_int]
+        lib.ckv_oracle_srs.argtypes = [C.c_int, P, C.c_int, C.c_int, C.c_int, C.c_int, C.c_double,
+                                       P, P, P, P, P, P]
         lib.ckv_oracle_threads.argtypes = [C.c_int]
         _lib = lib
     return _lib
@@ -171,3 +173,24 @@ def compress_layer(q_win, k, v, cu_seqlens, head_mask, budget, window, pool_kern
         int(lse_stride), _p(scores), _p(pooled), None, _p(idx), _p(k_out), _p(v_out), _p(gf),
         int(num_threads)))
     return dict(scores=scores, pooled=pooled, cu_keep=cu_keep, idx=idx, k_out=k_out, v_out=v_out)
+
+
+def semantic_retrieval_scores(q_dec, k, cu_seqlens, head_mask, window, in_answer, span, scale=None):
+    """Eq. 5 per selected head, summed over the batch's sequences: float64 [Hq] (0 for heads
+    that are not selected).  q_dec [S, w, Hq, d], k [T, Hkv, d] (bf16 bits), in_answer [S*w],
+    span [S, 2] (sequence-local [a0, a1))."""
+    q = np.ascontiguousarray(q_dec, dtype=np.uint16)
+    k = np.ascontiguousarray(k, dtype=np.uint16)
+    cu = np.ascontiguousarray(cu_seqlens, dtype=np.int32)
+    mask = np.ascontiguousarray(head_mask, dtype=np.uint8)
+    flags = np.ascontiguousarray(in_answer, dtype=np.uint8)
+    sp = np.ascontiguousarray(span, dtype=np.int32)
+    S = cu.size - 1
+    T, Hkv, d = k.shape
+    Hq = q.shape[2]
+    assert q.shape == (S, window, Hq, d) and flags.size == S * window and sp.shape == (S, 2)
+    scale = 1.0 / np.sqrt(d) if scale is None else scale
+    out = np.zeros(Hq, np.float64)
+    _check(_load().ckv_oracle_srs(S, _p(cu), Hq, Hkv, d, window, float(scale), _p(mask), _p(q), _p(k),
+                                  _p(flags), _p(sp), _p(out)))
+    return out

@@ -361,6 +361,51 @@ int ckv_oracle_compress_layer(int S, const int32_t* cu_seqlens, int Hq, int Hkv,
     return failed ? ORACLE_NO_MEMORY : ORACLE_OK;
 }
 
+/*
+ * Semantic Retrieval Score (Sec. 3.2, Eq. 5), added into srs[Hq] for the selected heads:
+ *   srs[h] += sum over decode steps t with in_answer[s*w + t] of sum_{j in [a0, a1)} a^h_{t,j}
+ * per sequence s, where a^h_{t,j} is head h's attention of decode step t over keys
+ * 0..L_s-w+t (the context and the generated tokens up to itself; Eq. 2 with scale) and
+ * [a0, a1) = span[2s], span[2s+1] is the answer span.  q_dec [S, w, Hq, d], k [T, Hkv, d].
+ */
+int ckv_oracle_srs(int S, const int32_t* cu_seqlens, int Hq, int Hkv, int d, int w, double scale,
+                   const uint8_t* head_mask, const uint16_t* q_dec, const uint16_t* k,
+                   const uint8_t* in_answer, const int32_t* span, double* srs) {
+    if (S < 0 || Hq < 1 || Hkv < 1 || Hq % Hkv != 0 || d < 1 || w < 1) return ORACLE_BAD_ARG;
+    const int G = Hq / Hkv;
+    for (int s = 0; s < S; ++s) {
+        const int t0 = cu_seqlens[s], L = cu_seqlens[s + 1] - t0;
+        const int a0 = span[2 * s], a1 = span[2 * s + 1];
+        if (a0 < 0 || a1 < a0 || a1 > L) return ORACLE_BAD_ARG;
+        double* logit = (double*)malloc(sizeof(double) * (size_t)(L > 0 ? L : 1));
+        if (!logit) return ORACLE_NO_MEMORY;
+        for (int h = 0; h < Hq; ++h) {
+            if (!head_mask[h]) continue;
+            for (int t = 0; t < w; ++t) {
+                if (!in_answer[s * w + t]) continue;
+                const int last = L - w + t; /* the step's own position */
+                if (last < 0) continue;
+                const uint16_t* qt = q_dec + (((long)s * w + t) * Hq + h) * d;
+                double mx = -INFINITY;
+                for (int j = 0; j <= last; ++j) {
+                    const uint16_t* kj = k + ((long)(t0 + j) * Hkv + h / G) * d;
+                    double dot = 0.0;
+                    for (int c = 0; c < d; ++c) dot += widen_bf16(qt[c]) * widen_bf16(kj[c]);
+                    logit[j] = scale * dot;
+                    if (logit[j] > mx) mx = logit[j];
+                }
+                double z = 0.0;
+                for (int j = 0; j <= last; ++j) z += exp(logit[j] - mx);
+                double on_span = 0.0;
+                for (int j = a0; j < a1 && j <= last; ++j) on_span += exp(logit[j] - mx);
+                srs[h] += on_span / z;
+            }
+        }
+        free(logit);
+    }
+    return ORACLE_OK;
+}
+
 /* Number of threads an OpenMP region of this library uses when asked for n (0 = default). */
 int ckv_oracle_threads(int n) {
 #ifdef _OPENMP

@@ -84,6 +84,8 @@ def load():
         "ckv_read_device_status": ([P, P, I32, C.POINTER(I32), C.POINTER(I32)], C.c_int),
         "ckv_score_window_static": ([cfg, I32, bat, P, P, I64, I64, P, P, P], C.c_int),
         "ckv_score_window_lse": ([cfg, I32, bat, P, P, I64, I64, P, I64, P, P, SZ, P], C.c_int),
+        "ckv_semantic_retrieval_scores": ([cfg, I32, bat, P, P, I64, I64, P, I64, P, P, P, P, SZ, P],
+                                          C.c_int),
         "ckv_compress_layer_lse": ([cfg, I32, bat, P, P, P, I64, I64, P, I64, P, P, P, P, P, P, SZ, P],
                                    C.c_int),
         "ckv_layer_error_scores": ([P, I32, I32, P], C.c_int),
@@ -293,6 +295,17 @@ def ckv_compress_layer_lse(cfg, layer, batch, q_win, k, v, lse, idx, cu_keep_dev
                                          _ptr(pooled_out), _ptr(workspace),
                                          workspace.numel() * workspace.element_size(), _stream(stream)),
            "ckv_compress_layer_lse")
+
+
+def ckv_semantic_retrieval_scores(cfg, layer, batch, q_dec, k, lse, in_answer, span, srs, workspace,
+                                  lse_head_stride=0, stream=None, tok_stride=0, head_stride=0):
+    """Eq. 5: srs [H_q] += the selected heads' attention of the in-answer decode steps on the
+    answer span.  q_dec like q_win (w = cfg.window decode steps), k = context + generated keys,
+    lse [H_q, >= S*w], in_answer uint8 [S*w], span int32 [S, 2] (all device tensors)."""
+    _check(load().ckv_semantic_retrieval_scores(
+        cfg.ref, layer, batch.ref, _ptr(q_dec), _ptr(k), tok_stride, head_stride, _ptr(lse),
+        lse_head_stride, _ptr(in_answer), _ptr(span), _ptr(srs), _ptr(workspace),
+        workspace.numel() * workspace.element_size(), _stream(stream)), "ckv_semantic_retrieval_scores")
 
 
 def ckv_score_window_static(cfg, layer, batch, q_win, k, scores, status_out=None, stream=None,

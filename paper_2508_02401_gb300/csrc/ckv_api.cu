@@ -397,7 +397,7 @@ ckv_status plan_score_stream(const Plan& pl, const ckv_batch* b, int skip_le, in
 }
 
 struct WsLayout {
-    size_t header = 0, partials = 0, counters = 0, scores = 0, pooled = 0;
+    size_t header = 0, partials = 0, counters = 0, scores = 0, pooled = 0, srs_lse = 0;
     size_t hist = 0, arrivals = 0, chunk_start = 0, buckets = 0, info = 0, chunk_off = 0, total = 0;
     int max_chunks = 0;
 };
@@ -434,6 +434,8 @@ WsLayout ws_layout(const Plan& pl, const ckv_batch* b, int T) {
     off = round_up(off + units * 4 * sizeof(int), kWsAlign);
     l.chunk_off = off;
     off = round_up(off + units * l.max_chunks * sizeof(int), kWsAlign);
+    l.srs_lse = off;  // ckv_semantic_retrieval_scores: the masked lse of the decode rows
+    off = round_up(off + static_cast<size_t>(pl.Hq) * b->num_seqs * pl.w * sizeof(float), kWsAlign);
     l.total = off;
     return l;
 }
@@ -915,6 +917,52 @@ ckv_status ckv_compress_layer_lse(const ckv_config* cfg, int32_t layer, const ck
     return compress_layer_impl(cfg, layer, batch, q_win, k, v, tok_stride, head_stride, lse,
                                lse_head_stride, idx, cu_keep_dev, k_out, v_out, pooled_out,
                                workspace, workspace_bytes, stream);
+}
+
+ckv_status ckv_semantic_retrieval_scores(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
+                                         const void* q_dec, const void* k, int64_t tok_stride,
+                                         int64_t head_stride, const float* lse, int64_t lse_head_stride,
+                                         const uint8_t* in_answer, const int32_t* span, float* srs,
+                                         void* workspace, size_t workspace_bytes, ckv_stream stream) {
+    Plan pl;
+    ckv_status st = make_plan(cfg, layer, pl);
+    if (st) return st;
+    int T = 0;
+    WsLayout l;
+    if ((st = check_batch(batch, &T)) || (st = resolve_strides(pl, &tok_stride, &head_stride)) ||
+        (st = check_kv(q_dec, "q_dec", T)) || (st = check_kv(k, "k", T)) ||
+        (st = check_ws(pl, batch, T, workspace, workspace_bytes, &l)) ||
+        (st = check_lse(pl, batch, lse, &lse_head_stride)))
+        return st;
+    if (!in_answer || !span || !srs) return fail(CKV_ERR_INVALID_ARG, "in_answer, span and srs are required");
+    if (!aligned(span, 4) || !aligned(srs, 4)) return fail(CKV_ERR_INVALID_ARG, "span or srs is misaligned");
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    uint8_t* w8 = static_cast<uint8_t*>(workspace);
+    SrsLaunch L;
+    memset(&L, 0, sizeof L);
+    L.lse = lse;
+    L.lse_stride = lse_head_stride;
+    L.in_answer = in_answer;
+    float* scores = reinterpret_cast<float*>(w8 + l.scores);
+    L.lse_masked = reinterpret_cast<float*>(w8 + l.srs_lse);
+    L.scores = scores;
+    L.span = span;
+    L.cu_seqlens_dev = batch->cu_seqlens_dev;
+    L.sel_heads = pl.sel_heads.data();
+    L.srs = srs;
+    L.status = static_cast<int*>(workspace);
+    L.S = batch->num_seqs;
+    L.T = T;
+    L.Hq = pl.Hq;
+    L.w = pl.w;
+    L.n_sel = pl.n_sel;
+    cudaError_t e = launch_srs_mask(L, s);
+    if (e != cudaSuccess) return cuda_fail(e, "launching the lse mask kernel");
+    if ((st = enqueue_score(pl, batch, T, q_dec, k, tok_stride, head_stride, scores, workspace, l, -1, s,
+                            kMaxScoreItems, L.lse_masked, static_cast<int64_t>(batch->num_seqs) * pl.w)))
+        return st;
+    e = launch_srs_span(L, s);
+    return e == cudaSuccess ? CKV_OK : cuda_fail(e, "launching the span-sum kernel");
 }
 
 ckv_status ckv_read_device_status(void* workspace, ckv_stream stream, int32_t reset,

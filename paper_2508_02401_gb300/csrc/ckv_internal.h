@@ -116,6 +116,23 @@ struct GatherLaunch {
 };
 cudaError_t launch_gather(const GatherLaunch& L, cudaStream_t stream);
 
+// Semantic Retrieval Score support (Eq. 5, srs_kernels.cu).
+struct SrsLaunch {
+    const float* lse;         // [Hq][lse_stride] the decode rows' lse
+    int64_t lse_stride;
+    const uint8_t* in_answer; // [S*w] the step's generated token is in the answer span
+    float* lse_masked;        // [Hq][S*w] out: lse, or +inf where in_answer is 0
+    const float* scores;      // [n_sel, T]
+    const int32_t* span;      // [S][2] answer span [a0, a1), sequence-local
+    const int32_t* cu_seqlens_dev;
+    const int* sel_heads;     // host [n_sel]: query head of each score row
+    float* srs;               // [Hq] accumulated
+    int* status;
+    int S, T, Hq, w, n_sel;
+};
+cudaError_t launch_srs_mask(const SrsLaunch& L, cudaStream_t stream);
+cudaError_t launch_srs_span(const SrsLaunch& L, cudaStream_t stream);
+
 int device_sm_count();
 
 }  // namespace ckv
