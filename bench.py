@@ -91,6 +91,9 @@ def _args():
     ap.add_argument("--score-path", choices=("auto", "resident", "reload"), default="auto",
                     help="scoring kernel: logits kept in TMEM, K re-read in pass 2, or the "
                          "library's choice")
+    ap.add_argument("--srs", action="store_true",
+                    help="time the Semantic Retrieval Score accumulation (Eq. 5) instead: every "
+                         "head scored, the window rows as decode steps, all of them in the answer")
     ap.add_argument("--lse", action="store_true",
                     help="the window rows' lse given (as a prefill attention kernel returns it): "
                          "ckv_compress_layer_lse / ckv_score_window_lse, one pass over K")
@@ -518,10 +521,101 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+def run_srs(args):
+    """ckv_semantic_retrieval_scores over every layer of the workload: the window queries act as
+    the decode steps (all flagged as answer tokens), the answer span is 64 positions from a third
+    of each sequence, every query head is scored.  One JSON line; 1 GPU."""
+    import numpy as np
+    import torch
+
+    import __graft_entry__ as entry
+    import ckv_synth as cs
+    entry.build()
+    import paper_2508_02401_gb300 as ckv
+
+    wl = cs.workload(args.workload)
+    if args.layers:
+        wl = wl.with_(num_layers=args.layers)
+    nl, T, Hkv, Hq = wl.num_layers, wl.total_tokens, wl.num_kv_heads, wl.num_q_heads
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    nstreams = args.streams if args.streams > 0 else nl
+    cap = args.max_ctas if args.max_ctas > 0 else max(1, sms // 16)
+    cfg = ckv.Config.from_workload(wl, head_mask=np.ones((nl, Hq), np.uint8), max_ctas=cap)
+    batch = ckv.Batch(wl.cu_seqlens())
+    cu = wl.cu_seqlens()
+    lens = np.diff(cu)
+    span = torch.from_numpy(np.array([[L // 3, min(L, L // 3 + 64)] for L in lens], np.int32)).cuda()
+    flags = torch.ones(wl.num_seqs * wl.window, dtype=torch.uint8, device="cuda")
+    layers = []
+    for l in range(nl):
+        li = wl.layer(l)
+        q = torch.from_numpy(li.q_win.view(np.int16)).cuda().view(torch.bfloat16)
+        k = torch.from_numpy(li.k.view(np.int16)).cuda().view(torch.bfloat16)
+        layers.append(dict(q=q, k=k, lse=_window_lse(q, k, cu, wl.window, Hq, Hkv)))
+    srs = torch.zeros(Hq, dtype=torch.float32, device="cuda")
+    ws_bytes = max(ckv.ckv_workspace_size(cfg, l, batch) for l in range(nl))
+    wss = [torch.zeros(ws_bytes, dtype=torch.uint8, device="cuda") for _ in range(nstreams)]
+    stream = torch.cuda.Stream()
+    side = [torch.cuda.Stream() for _ in range(nstreams)]
+
+    def step():
+        for sd in side:
+            sd.wait_stream(stream)
+        for l, d in enumerate(layers):
+            ckv.ckv_semantic_retrieval_scores(cfg, l, batch, d["q"], d["k"], d["lse"], flags, span, srs,
+                                              wss[l % nstreams], stream=side[l % nstreams])
+        for sd in side:
+            stream.wait_stream(sd)
+
+    with torch.cuda.stream(stream):
+        for _ in range(max(1, args.warmup)):
+            step()
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        step()
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            graph.replay()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(0) as clk:
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(args.steps):
+                graph.replay()
+            e1.record(stream)
+        torch.cuda.synchronize()
+    for w in wss:
+        code, detail = ckv.ckv_read_device_status(w, stream=stream)
+        if code != 0:
+            raise RuntimeError(f"device status {code} ({detail}) after the timed region")
+    ms_per_step = e0.elapsed_time(e1) / args.steps
+    hbm_peak, peak_kind = _peaks()
+    k_bytes = T * Hkv * 256  # K read once per (token, KV head): the floor; each head batch reads it
+    gbs = k_bytes * nl / (ms_per_step / 1e3) / 1e9
+    line = {
+        "metric": "SRS accumulation (Eq. 5) prefix tokens/s per layer", "value": round(nl * T / (ms_per_step / 1e3), 1),
+        "unit": UNIT, "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(ms_per_step, 5), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": wl.name, "layers": nl, "seq_len": T, "q_heads": Hq, "kv_heads": Hkv,
+                   "decode_steps": wl.window, "heads_scored": Hq,
+                   "streams": f"layers round-robin on {nstreams} streams, scoring capped at {cap} CTAs per call"},
+        "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": hbm_peak, "unit": "GB/s",
+                     "frac": round(gbs / hbm_peak, 4), "peak_kind": peak_kind, "traffic": None,
+                     "algorithmic_bytes_per_layer": k_bytes},
+        "clocks": clk.summary(), "gpu_launches": 3 * nl * args.steps,
+    }
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = _args()
     if args.impl == "reference":
         run_reference(args)
+    elif args.srs:
+        run_srs(args)
     else:
         run_ours(args)
 
