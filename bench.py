@@ -392,17 +392,38 @@ def run_ours(args):
         h2d = sum(x.numel() * 2 for x in hq + hk + hv) + sum(x.numel() * 4 for x in hl)
         d2h = sum(x.numel() * x.element_size() for x in oi + ok + ov)
 
+        # Per layer: its inputs on one of two copy streams, its compression on its own stream once
+        # they have landed, its outputs back on a read-back stream once it is done; the copies of
+        # one layer overlap the other layers' compressions.
+        copy_streams = [torch.cuda.Stream() for _ in range(2)]
+        back = torch.cuda.Stream()
+        every = copy_streams + side + [back]
+
         def e2e_step():
+            for st in every:
+                st.wait_stream(stream)
             for l, d in enumerate(layers):
-                d["q"].copy_(hq[l], non_blocking=True)
-                d["k"].copy_(hk[l], non_blocking=True)
-                d["v"].copy_(hv[l], non_blocking=True)
-                if args.lse:
-                    d["lse"].copy_(hl[l], non_blocking=True)
-                compress(l, d, ws, stream)
-                oi[l].copy_(d["idx"], non_blocking=True)
-                ok[l].copy_(d["k_out"], non_blocking=True)
-                ov[l].copy_(d["v_out"], non_blocking=True)
+                cp = copy_streams[l % len(copy_streams)]
+                with torch.cuda.stream(cp):
+                    d["q"].copy_(hq[l], non_blocking=True)
+                    d["k"].copy_(hk[l], non_blocking=True)
+                    d["v"].copy_(hv[l], non_blocking=True)
+                    if args.lse:
+                        d["lse"].copy_(hl[l], non_blocking=True)
+                landed = torch.cuda.Event()
+                landed.record(cp)
+                st = side[l % nstreams]
+                st.wait_event(landed)
+                compress(l, d, wss[l % nstreams], st)
+                done = torch.cuda.Event()
+                done.record(st)
+                back.wait_event(done)
+                with torch.cuda.stream(back):
+                    oi[l].copy_(d["idx"], non_blocking=True)
+                    ok[l].copy_(d["k_out"], non_blocking=True)
+                    ov[l].copy_(d["v_out"], non_blocking=True)
+            for st in every:
+                stream.wait_stream(st)
 
         with torch.cuda.stream(stream):
             for _ in range(2):
