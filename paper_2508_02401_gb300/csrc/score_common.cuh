@@ -56,16 +56,6 @@ __device__ __forceinline__ float lg2_approx(float x) {
     return y;
 }
 
-// Sum / max of an array by a balanced tree (short dependency chains).
-template <int C>
-__device__ __forceinline__ float tree_sum(float (&x)[C]) {
-#pragma unroll
-    for (int w = C / 2; w >= 1; w >>= 1)
-#pragma unroll
-        for (int i = 0; i < w; ++i) x[i] += x[i + w];
-    return x[0];
-}
-
 // Packed fp32 pairs (sm_100+): one instruction for two lanes' worth of FMA / add, with the
 // same IEEE rounding as the scalar forms.
 __device__ __forceinline__ void fma2(float& d0, float& d1, float a0, float a1, float b0, float b1,
@@ -154,38 +144,6 @@ __device__ __forceinline__ void transpose_reduce(float (&v)[C], float (&m)[C], i
     }
 #pragma unroll
     for (int bit = 16 / C; bit >= 1; bit >>= 1) v[0] += __shfl_xor_sync(0xffffffffu, v[0], bit);
-}
-
-template <int CPW>
-__device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, float (&v)[CPW]) {
-    if constexpr (CPW == 32) {
-        tmem_ld32(taddr, v);
-    } else if constexpr (CPW == 16) {
-        uint32_t r[16];
-        asm volatile(
-            "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-            "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n\t"
-            "tcgen05.wait::ld.sync.aligned;"
-            : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]),
-              "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]),
-              "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-            : "r"(taddr)
-            : "memory");
-#pragma unroll
-        for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
-    } else {
-        static_assert(CPW == 8, "CPW");
-        uint32_t r[8];
-        asm volatile(
-            "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];\n\t"
-            "tcgen05.wait::ld.sync.aligned;"
-            : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]),
-              "=r"(r[6]), "=r"(r[7])
-            : "r"(taddr)
-            : "memory");
-#pragma unroll
-        for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(r[i]);
-    }
 }
 
 // tcgen05.ld of 16 columns without the wait: the registers are not valid until tmem_ld_wait,
