@@ -122,6 +122,30 @@ def _dist():
     return rank, world, local
 
 
+# Replicas only: the ranks share nothing in the data path; they meet for the barriers around
+# the timed region and for the maximum of their times.
+def _rank_barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def _max_over_ranks(ms, world, device):
+    """The largest of the ranks' times (every rank gets it)."""
+    if world <= 1:
+        return ms
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(ms)], device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def _job_throughput(world, units_per_rank, ms_per_step):
+    """Whole-job units per second: every rank processes its own units in the slowest rank's time."""
+    return world * units_per_rank / (ms_per_step / 1e3)
+
+
 # ----------------------------------------------------------------------------- clocks
 _REASONS = {0x1: "gpu_idle", 0x2: "applications_clocks_setting", 0x4: "sw_power_cap",
             0x8: "hw_slowdown", 0x10: "sync_boost", 0x20: "sw_thermal_slowdown",
@@ -273,9 +297,7 @@ def run_ours(args):
     torch.cuda.synchronize()
 
     def barrier():
-        if world > 1:
-            import torch.distributed as dist
-            dist.barrier()
+        _rank_barrier(world)
 
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(local) as clk:
@@ -288,19 +310,14 @@ def run_ours(args):
             e1.record(stream)
         torch.cuda.synchronize()
         barrier()
-    ms = e0.elapsed_time(e1)
+    ms = _max_over_ranks(e0.elapsed_time(e1), world, "cuda")
     clocks = clk.summary()
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
     for w in wss:
         code, detail = ckv.ckv_read_device_status(w, stream=stream)
         if code != 0:
             raise RuntimeError(f"device status {code} ({detail}) after the timed region")
     ms_per_step = ms / args.steps
-    value = world * nl * T / (ms_per_step / 1e3)
+    value = _job_throughput(world, nl * T, ms_per_step)
 
     # per layer: the scoring kernel, then the selection (pool, top-k, compaction and gather)
     lens = list(wl.seqlens)
