@@ -113,6 +113,7 @@ constexpr int kUnitPer = 16;
 constexpr int kUnitLen = kUnitThreads * kUnitPer;
 constexpr int kUnitStage = kUnitLen + 2 * kMaxHalo;
 constexpr int kUnitStageLoads = (kUnitStage + kUnitThreads - 1) / kUnitThreads;
+constexpr int kUnitCandMax = 1024;            // first-digit ties ranked pairwise up to this many
 static_assert(kWarpSpan % 32 == 0 && (1 << kChunkShift) == kChunk, "chunk shape");
 
 // Shared-memory index of staged element e: one pad word per 32 keeps the contiguous
@@ -293,6 +294,38 @@ __device__ __forceinline__ void stage_rows(float* st, const float* scores, size_
     }
 }
 
+__device__ __forceinline__ void cp_async4(float* dst, const float* src) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+    asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+}
+
+// Stages score rows ra .. ra+nr-1 (each alone, not summed) at sequence positions
+// base-half .. base+n+half-1 (zero outside [0, P)), row i at st + i*words, element e at
+// sidx(e): every copy of every row is issued (asynchronously, no registers held) before the
+// wait, so the rows take one round trip together.
+template <int NT, int LOADS>
+__device__ __forceinline__ void stage_rows_async(float* st, int words, const float* scores, size_t T,
+                                                 int t0, int ra, int nr, int base, int half, int n,
+                                                 int P) {
+    const int ne = n + 2 * half, tid = threadIdx.x;
+    for (int i = 0; i < nr; ++i) {
+        const float* row = scores + static_cast<size_t>(ra + i) * T + t0;
+        float* dst = st + i * words;
+#pragma unroll
+        for (int q = 0; q < LOADS; ++q) {
+            const int e = tid + q * NT;
+            const int uu = base - half + e;
+            if (e < ne) {
+                if (uu >= 0 && uu < P) cp_async4(dst + sidx(e), row + uu);
+                else dst[sidx(e)] = 0.f;
+            }
+        }
+    }
+    cp_async_wait_all();
+}
+
 // Pools PER consecutive outputs from the stage: output i reads staged elements
 // jl+i .. jl+i+2*HALF.  Same arithmetic, in the same order, as pool_kernel: the staged zeros
 // outside [0, P) leave a max of non-negative scores and a left-to-right sum unchanged.
@@ -322,6 +355,10 @@ __device__ __forceinline__ void pool_window(const float* st, int jl, int nvalid,
 template <int PER>
 __device__ __forceinline__ void pool_any(const float* st, int jl, int nvalid, int half, bool is_max,
                                          float kf, float (&acc)[PER]) {
+    // A thread with no output reads nothing: its window would start past the staged row (and,
+    // for the last of several staged rows, past the stage).  A thread with outputs reads at most
+    // PER - 1 elements past its row's last staged one.
+    if (nvalid <= 0) return;
     if (half == 3) {
         pool_window<3, PER>(st, jl, nvalid, is_max, kf, acc);
     } else if (half == 2) {
@@ -341,7 +378,9 @@ __device__ __forceinline__ void pool_any(const float* st, int jl, int nvalid, in
 
 // Pooled scores of positions base+jl .. base+jl+PER-1 (jl = PER * thread) of unit u, computed
 // from the scores (from_scores) or read from p.pooled.  Ends with the stage free again.
-template <int NT, int PER, int LOADS>
+// WORDS is the stage's capacity: with the heads pooled one by one, as many rows as fit are
+// staged together.
+template <int NT, int PER, int LOADS, int WORDS>
 __device__ __forceinline__ void pooled_values(const SelectParams& p, const UnitGeo& u, float* st, int base,
                                               int n, float (&acc)[PER]) {
     const int jl = threadIdx.x * PER, nvalid = n - jl;
@@ -352,11 +391,19 @@ __device__ __forceinline__ void pooled_values(const SelectParams& p, const UnitG
         const bool is_max = p.pool_type == 0;
         const float kf = static_cast<float>(p.pool_kernel);
         const int r0 = p.group_first[u.g], r1 = p.group_first[u.g + 1];
-        const bool per_head = p.head_order == 0;
-        const int passes = per_head ? r1 - r0 : 1;
-        for (int ps = 0; ps < passes; ++ps) {
-            const int ra = per_head ? r0 + ps : r0, rb = per_head ? ra + 1 : r1;
-            stage_rows<NT, LOADS>(st, p.scores, p.T, u.t0, ra, rb, base, half, n, u.P);
+        if (p.head_order == 0) {  // pool each head, then sum (in head order)
+            const int words = stage_words(n + 2 * half);
+            // rows that fit, with room for the last row's readers to run PER words past it
+            const int fit = max(1, (WORDS - PER) / words);
+            for (int ra = r0; ra < r1; ra += fit) {
+                const int nr = min(fit, r1 - ra);
+                stage_rows_async<NT, LOADS>(st, words, p.scores, p.T, u.t0, ra, nr, base, half, n, u.P);
+                __syncthreads();
+                for (int i = 0; i < nr; ++i) pool_any<PER>(st + i * words, jl, nvalid, half, is_max, kf, acc);
+                __syncthreads();
+            }
+        } else {  // sum the heads, then pool
+            stage_rows<NT, LOADS>(st, p.scores, p.T, u.t0, r0, r1, base, half, n, u.P);
             __syncthreads();
             pool_any<PER>(st, jl, nvalid, half, is_max, kf, acc);
             __syncthreads();
@@ -377,8 +424,9 @@ __device__ __forceinline__ void pooled_values(const SelectParams& p, const UnitG
 }
 
 // Copies the K and V rows of sequence-local positions list[0..m) to output rows
-// out_row0 + 0..m-1 of KV head g: a warp per row (16 lanes for K, 16 for V), four rows in
-// flight per warp.
+// out_row0 + 0..m-1 of KV head g: a warp per row (16 lanes for K, 16 for V), kRowsInFlight
+// rows in flight per warp.
+constexpr int kRowsInFlight = 8;
 __device__ __forceinline__ void copy_rows(const SelectParams& p, const UnitGeo& u, int kv,
                                           const int* list, int m, int out_row0) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
@@ -386,15 +434,15 @@ __device__ __forceinline__ void copy_rows(const SelectParams& p, const UnitGeo& 
     const uint4* src0 = (lane < 16 ? p.k : p.v) + static_cast<int64_t>(u.t0) * p.tok_stride +
                         static_cast<int64_t>(kv) * p.head_stride + part;
     uint4* dst0 = (lane < 16 ? p.k_out : p.v_out) + static_cast<int64_t>(kv) * 16 + part;
-    for (int e0 = warp; e0 < m; e0 += 4 * nw) {
-        uint4 x[4];
+    for (int e0 = warp; e0 < m; e0 += kRowsInFlight * nw) {
+        uint4 x[kRowsInFlight];
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
+        for (int q = 0; q < kRowsInFlight; ++q) {
             const int e = e0 + q * nw;
             if (e < m) x[q] = __ldg(src0 + static_cast<int64_t>(list[e]) * p.tok_stride);
         }
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
+        for (int q = 0; q < kRowsInFlight; ++q) {
             const int e = e0 + q * nw;
             if (e < m) dst0[static_cast<int64_t>(out_row0 + e) * p.Hkv * 16] = x[q];
         }
@@ -419,7 +467,8 @@ __global__ void __launch_bounds__(kUnitThreads, 1) select_unit_kernel(const __gr
     extern __shared__ __align__(16) float ust[];  // pooling stage, then the kept list
     __shared__ int hist[kHistBins];
     __shared__ int scratch[33];
-    __shared__ int s_digit, s_above, s_cut;
+    __shared__ int s_digit, s_above, s_cut, s_cnt;
+    __shared__ uint32_t s_thr;
     constexpr int NT = kUnitThreads, PER = kUnitPer;
     // A selection that serves several KV heads (per-layer scope) is made by one block per KV
     // head, each gathering its own head's rows: the selection is recomputed (from L2-resident
@@ -453,7 +502,7 @@ __global__ void __launch_bounds__(kUnitThreads, 1) select_unit_kernel(const __gr
         for (int j = P + tid; j < u.L; j += NT) pooled[j] = 0.f;
     const int jb = tid * PER, nvalid = P - jb;
     float acc[PER];
-    pooled_values<NT, PER, kUnitStageLoads>(p, u, ust, 0, P, acc);
+    pooled_values<NT, PER, kUnitStageLoads, stage_words(kUnitStage)>(p, u, ust, 0, P, acc);
     if (zeros)
 #pragma unroll
         for (int i = 0; i < PER; ++i)
@@ -478,44 +527,73 @@ __global__ void __launch_bounds__(kUnitThreads, 1) select_unit_kernel(const __gr
         uint32_t prefix = static_cast<uint32_t>(s_digit) << kHistShift, mask = 0x7FFu << kHistShift;
         int r = k - s_above, n_eq = hist[s_digit];
         __syncthreads();
-#pragma unroll 1
-        for (int level = 0; level < 2; ++level) {
-            const int shift = level == 0 ? 10 : 0;
-            const uint32_t dmask = level == 0 ? 0x7FFu : 0x3FFu;
-            for (int b = tid; b < kHistBins; b += NT) hist[b] = 0;
+        if (n_eq <= kUnitCandMax) {
+            // Few keys share the k-th key's first digit: gather them and rank them exactly, by
+            // key descending then position ascending; the r-th is the threshold key, its
+            // position the tie cutoff.  (The stage is free again: it holds the pairs.)
+            uint2* cand = reinterpret_cast<uint2*>(ust);
+            const uint32_t d = static_cast<uint32_t>(s_digit);
+            if (tid == 0) s_cnt = 0;
             __syncthreads();
 #pragma unroll
             for (int i = 0; i < PER; ++i)
-                if (i < nvalid && (key[i] & mask) == prefix) atomicAdd(&hist[(key[i] >> shift) & dmask], 1);
+                if (i < nvalid && bins[i] == d) cand[atomicAdd(&s_cnt, 1)] = make_uint2(key[i], jb + i);
             __syncthreads();
-            find_digit<NT>(hist, r, scratch, &s_digit, &s_above);
-            prefix |= static_cast<uint32_t>(s_digit) << shift;
-            mask |= dmask << shift;
-            r -= s_above;
-            n_eq = hist[s_digit];
-            __syncthreads();
-        }
-        thr = prefix;
-        const int need_eq = r;  // keys equal to thr that are kept: the lowest positions
-        pos_cut = INT_MAX;
-        if (need_eq < n_eq) {
-            int ne = 0;
-#pragma unroll
-            for (int i = 0; i < PER; ++i) ne += (i < nvalid && key[i] == thr) ? 1 : 0;
-            int tot;
-            const int before = block_excl_scan<NT>(ne, scratch, &tot);  // thread order = position order
-            if (before < need_eq && before + ne >= need_eq) {
-                int c = before;
-#pragma unroll
-                for (int i = 0; i < PER; ++i) {
-                    if (i < nvalid && key[i] == thr) {
-                        ++c;
-                        if (c == need_eq) s_cut = jb + i;
-                    }
+            for (int c = tid; c < n_eq; c += NT) {
+                const uint2 me = cand[c];
+                int ahead = 0;
+                for (int q = 0; q < n_eq; ++q) {
+                    const uint2 o = cand[q];
+                    ahead += (o.x > me.x || (o.x == me.x && o.y < me.y)) ? 1 : 0;
+                }
+                if (ahead == r - 1) {
+                    s_thr = me.x;
+                    s_cut = static_cast<int>(me.y);
                 }
             }
             __syncthreads();
+            thr = s_thr;
             pos_cut = s_cut;
+        } else {
+#pragma unroll 1
+            for (int level = 0; level < 2; ++level) {
+                const int shift = level == 0 ? 10 : 0;
+                const uint32_t dmask = level == 0 ? 0x7FFu : 0x3FFu;
+                for (int b = tid; b < kHistBins; b += NT) hist[b] = 0;
+                __syncthreads();
+#pragma unroll
+                for (int i = 0; i < PER; ++i)
+                    if (i < nvalid && (key[i] & mask) == prefix) atomicAdd(&hist[(key[i] >> shift) & dmask], 1);
+                __syncthreads();
+                find_digit<NT>(hist, r, scratch, &s_digit, &s_above);
+                prefix |= static_cast<uint32_t>(s_digit) << shift;
+                mask |= dmask << shift;
+                r -= s_above;
+                n_eq = hist[s_digit];
+                __syncthreads();
+            }
+            thr = prefix;
+            const int need_eq = r;  // keys equal to thr that are kept: the lowest positions
+            pos_cut = INT_MAX;
+            if (need_eq < n_eq) {
+                int ne = 0;
+#pragma unroll
+                for (int i = 0; i < PER; ++i) ne += (i < nvalid && key[i] == thr) ? 1 : 0;
+                int tot;
+                const int before = block_excl_scan<NT>(ne, scratch, &tot);  // thread order = position order
+                if (before < need_eq && before + ne >= need_eq) {
+                    int c = before;
+#pragma unroll
+                    for (int i = 0; i < PER; ++i) {
+                        if (i < nvalid && key[i] == thr) {
+                            ++c;
+                            if (c == need_eq) s_cut = jb + i;
+                        }
+                    }
+                }
+                __syncthreads();
+                pos_cut = s_cut;
+            }
         }
     }
     // the kept positions in order, then the window
@@ -770,7 +848,8 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
     const int n = min(kChunk, u.P - j0);
     const int jl = tid * PER, nvalid = n - jl;
     float acc[PER];
-    pooled_values<kSelThreads, PER, kStageLoads>(p, u, reinterpret_cast<float*>(dyn), j0, n, acc);
+    pooled_values<kSelThreads, PER, kStageLoads, stage_words(kStageFloats)>(p, u, reinterpret_cast<float*>(dyn),
+                                                                            j0, n, acc);
     if (p.from_scores)  // the compaction reads them back
 #pragma unroll
         for (int i = 0; i < PER; ++i)
