@@ -40,9 +40,9 @@ HBM_FALLBACK_GBS = 6800.0
 # null until it is captured again.
 SCORE_SOURCES = ('score_kernel.cu', 'score_resident.cu', 'score_lse.cu', 'score_common.cuh', 'ckv_device.cuh')
 SCORE_TRAFFIC = {
-    "e2ce6dd503dbedaf76fb38d0c48061e120265a4a3cee04f9733c613831effc5e": {
-        "llama8b_l8192": 16987904, "paper_llama8b_l8192": 8488704,
-        "llama8b_l8192+lse": 16948736, "needle_l131072+lse": 274966272,
+    "a73eeb2e6dadd90875af204f73bc575a255a509fc1ae824331b36d2fdc214004": {
+        "llama8b_l8192": 16992768, "paper_llama8b_l8192": 8493056,
+        "llama8b_l8192+lse": 16950528, "needle_l131072+lse": 274175232,
     },
 }
 # Sequences up to this many tokens are selected by one block per (sequence, KV head)
