@@ -11,14 +11,15 @@
 // into items of a few tiles, and the items are dealt out in rounds of gridDim.x (CTA b takes
 // item round * gridDim.x + b; all items of a unit are in one round).  One cooperative
 // launch, one CTA per SM, 512 threads, warp-specialised:
-//   warp 0       pass-1 producer: per item, TMA loads of the window query rows (the MMA's B
-//                operand) into one of three buffers, then of its 128-key x 128-dim bf16 K
-//                tiles (two 128-byte-swizzled boxes of 64 dims) into a ring of kP1Slots slots;
-//   warp 1       allocates TMEM and issues tcgen05.mma (M = 128 keys, N = the window rows of a
-//                head batch, K = 128) for both passes, into four pass-1 and four pass-2 TMEM
-//                accumulators, taking whichever ring has a tile ready;
-//   warp 2       pass-2 producer: the same tiles again into a ring of kP2Slots slots, issued
-//                once an item's pass-1 loads are out, so they are served by L2;
+//   warp 0       TMA producer for both passes, one polling thread: per item, TMA loads of the
+//                window query rows (the MMA's B operand) into one of three buffers, then of its
+//                128-key x 128-dim bf16 K tiles (two 128-byte-swizzled boxes of 64 dims) into
+//                the pass-1 ring of kP1Slots slots; the same tiles again into the pass-2 ring
+//                of kP2Slots slots once the item's pass-1 loads are out, so they come from L2;
+//   warp 1       allocates TMEM and issues the pass-1 tcgen05.mma (M = 128 keys, N = the
+//                window rows of a head batch, K = 128) into four pass-1 TMEM accumulators;
+//   warp 2       issues the pass-2 tcgen05.mma into four pass-2 accumulators (two issuing
+//                threads, so that neither pass's issue waits behind the other's);
 //   warp 3       publisher: once an item's pass-1 partials are stored, one release on the
 //                unit's arrival counter;
 //   warps 4-11   pass 1, one warpgroup per 32 columns: each thread owns one key (one TMEM
@@ -57,11 +58,10 @@ struct SmemLayout {
                          kFree2 = kFull2 + kP2Slots, kAFull = kFree2 + kP2Slots,
                          kAEmpty = kAFull + kAcc, kBFull = kAEmpty + kAcc, kBEmpty = kBFull + kAcc,
                          kQFull = kBEmpty + kAcc, kQEmpty = kQFull + kQBufs,
-                         kDone = kQEmpty + kQBufs, kGroup = kDone + 1,  // A0 A1 B
+                         kDone = kQEmpty + kQBufs, kGroup = kDone + 2,  // A0 A1 B
                          kPubFull = kGroup + 3, kPubEmpty = kPubFull + 2,
                          kNumBars = kPubEmpty + 2;
-    static constexpr int kIssued = kBars + 8 * kNumBars; // items whose pass-1 loads are issued
-    static constexpr int kTmemSlot = kIssued + 4;
+    static constexpr int kTmemSlot = kBars + 8 * kNumBars;
     static constexpr int kAbort = kTmemSlot + 4;
     static constexpr int kBytes = kAbort + 4;
     static constexpr int kDynamic = kBytes + 1024;      // slack to align the base to 1024 B
@@ -103,7 +103,6 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
     __shared__ float2 red_b[256];        // [part * N + column]
     __shared__ __align__(16) float nlse_s[64];  // -lse per column of the current pass-2 item
     __shared__ volatile int verdict[1];
-    volatile int* issued = reinterpret_cast<volatile int*>(sm + SL::kIssued);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + SL::kTmemSlot);
     volatile int* abort = reinterpret_cast<volatile int*>(sm + SL::kAbort);
 
@@ -126,15 +125,15 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         }
         for (int i = 0; i < kQBufs; ++i) {
             mbar_init(&q_full[i], 1);
-            mbar_init(&q_empty[i], 1);
+            mbar_init(&q_empty[i], 2);  // one commit per pass
         }
-        mbar_init(done, 1);
+        mbar_init(&done[0], 1);
+        mbar_init(&done[1], 1);
         for (int i = 0; i < 3; ++i) mbar_init(&group[i], 128);
         for (int i = 0; i < 2; ++i) {
             mbar_init(&pub_full[i], 32 * kNW);
             mbar_init(&pub_empty[i], 1);
         }
-        *issued = 0;
         *abort = 0;
         fence_mbar_init();
         tma_prefetch_desc(&p.tmap_k);
@@ -167,163 +166,102 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
 
     if (warp < kWarpA) {
     setmaxnreg_dec<56>();
-    if (warp == 0 || warp == 2) {
-        // ------------------------------------------------------------ TMA producers
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer
+        // Both rings from one thread that polls: a pass-1 slot still in use must not hold up
+        // a pass-2 load, nor the other way round.
         if (lane == 0) {
-            const bool first = warp == 0;
-            const int nslots = first ? kP1Slots : kP2Slots;
-            uint8_t* ring = first ? ring1 : ring2;
-            uint64_t* full = first ? full1 : full2;
-            uint64_t* freed = first ? free1 : free2;
-            // Pass-1 tiles are read again by pass 2 shortly after: ask L2 to keep them, and
-            // to drop them first once pass 2 has read them.
-            const uint64_t policy = first ? l2_policy_evict_last() : l2_policy_evict_first();
-            int use = 0, it = 0;
-            bool ok = true;
-            for (int r = 0; ok && r < R; ++r) {
-                const ScoreItem& I = item_of(r);
-                const int n = I.ntiles;
-                if (n == 0) continue;
-                if (!first) {  // pass 2 follows the item's pass-1 loads, so it reads L2
-                    const long long t0 = clock64();
-                    for (uint32_t k = 1; *issued <= it; ++k) {
-                        __nanosleep(64);
-                        if ((k & 63u) == 0u && (*abort || clock64() - t0 > lim)) {
-                            ok = false;
-                            break;
-                        }
-                    }
-                    if (!ok) break;
-                }
-                const ScoreUnit& U = p.units[I.unit];
-                const int g = p.batch_group[U.batch];
-                if (first) {
-                    // The item's window query rows: per head of the batch two boxes of 64
-                    // dims x W_PAD rows in the MMA's 128-byte-swizzled layout.  Rows past w
-                    // (the next sequence's, or zeros past the end) and head slots past the
-                    // batch's heads land in columns that the epilogues mask out.
-                    const int qb = it % kQBufs;
-                    if (!mbar_wait(&q_empty[qb], ((it / kQBufs) & 1) ^ 1, abort, lim)) {
-                        ok = false;
-                        break;
-                    }
-                    uint8_t* qdst = qbuf + qb * SL::kQBytes;
-                    const int first_row = p.batch_first[U.batch], nheads = p.batch_nheads[U.batch];
-                    mbar_arrive_expect_tx(&q_full[qb], static_cast<uint32_t>(nheads * W_PAD * 256));
-                    for (int slot = 0; slot < nheads; ++slot) {
-                        const int h = p.sel_heads[first_row + slot];
-                        uint8_t* d = qdst + slot * W_PAD * 128;
-                        tma_load_3d(d, &p.tmap_q, &q_full[qb], 0, h, U.seq * p.w);
-                        tma_load_3d(d + SL::kQHalf, &p.tmap_q, &q_full[qb], 64, h, U.seq * p.w);
-                    }
-                }
-                for (int jt = 0; ok && jt < n; ++jt, ++use) {
-                    const int s = use % nslots;
-                    if (!mbar_wait(&freed[s], ((use / nslots) & 1) ^ 1, abort, lim)) {
-                        ok = false;
-                        break;
-                    }
-                    mbar_arrive_expect_tx(&full[s], kTileBytes);
-                    uint8_t* dst = ring + s * kTileBytes;
-                    const int tok = U.seq_start + (I.tile0 + jt) * kTileKeys;
-                    tma_load_3d_hint(dst, &p.tmap_k, &full[s], 0, g, tok, policy);
-                    tma_load_3d_hint(dst + kHalfBytes, &p.tmap_k, &full[s], 64, g, tok, policy);
-                }
-                ++it;
-                if (first) *issued = it;
-            }
-            if (!ok) {
-                *abort = 1;
-                record_error(p.status, kDevTimeout, first ? 10 : 15);
-            }
-            // Let every issued copy land before the block may exit.
-            const int last = use;
-            for (int k = (last > nslots ? last - nslots : 0); k < last; ++k) {
-                volatile int never = 0;
-                mbar_wait(&full[k % nslots], (k / nslots) & 1, &never);
-            }
-            if (first)
-                for (int k = (it > kQBufs ? it - kQBufs : 0); k < it; ++k) {
-                    volatile int never = 0;
-                    mbar_wait(&q_full[k % kQBufs], (k / kQBufs) & 1, &never);
-                }
-        }
-    } else if (warp == 1) {
-        // ------------------------------------------------------------ MMA issuer
-        if (lane == 0) {
+            // Pass-1 tiles are read again by pass 2 shortly after: ask L2 to keep them, and to
+            // drop them first once pass 2 has read them.
+            const uint64_t pol1 = l2_policy_evict_last(), pol2 = l2_policy_evict_first();
             auto next_item = [&](int r) {
                 while (r < R && item_of(r).ntiles == 0) ++r;
                 return r;
             };
-            auto mma = [&](const uint8_t* a_tile, const uint8_t* q, uint32_t d_tmem) {
-                const uint32_t a0 = smem_u32(a_tile), b0 = smem_u32(q);
-#pragma unroll
-                for (int kk = 0; kk < kHeadDim / 16; ++kk) {
-                    const uint32_t koff = (kk & 3) * 32;
-                    const uint64_t ad = sdesc_k_major_sw128(a0 + (kk >> 2) * kHalfBytes + koff);
-                    const uint64_t bd = sdesc_k_major_sw128(b0 + (kk >> 2) * SL::kQHalf + koff);
-                    umma_bf16(d_tmem, ad, bd, kIdesc, kk > 0 ? 1u : 0u);
-                }
-            };
-            int r1 = next_item(0), it1 = 0, jt1 = 0, use1 = 0, a_it = 0;
-            int r2 = r1, it2 = 0, jt2 = 0, use2 = 0, b_it = 0;
-            bool q_ready = false, ok = true;
+            int r1 = next_item(0), jt1 = 0, it1 = 0, use1 = 0;
+            int r2 = r1, jt2 = 0, it2 = 0, use2 = 0;
+            ScoreItem I1{}, I2{};
+            ScoreUnit U1{}, U2{};
+            if (r1 < R) {
+                I1 = I2 = item_of(r1);
+                U1 = U2 = p.units[I1.unit];
+            }
+            bool q_out = false, ok = true;
             long long t0 = clock64();
             uint32_t idle = 0;
             while (r1 < R || r2 < R) {
                 bool did = false;
-                // pass 2 of an item whose pass-1 products are all issued
-                if (r2 < R && it2 < it1) {
-                    const int s = use2 % kP2Slots, acc = b_it % kAcc;
-                    if (mbar_test(&full2[s], (use2 / kP2Slots) & 1) &&
-                        mbar_test(&b_empty[acc], ((b_it / kAcc) & 1) ^ 1)) {
-                        tc_fence_after_sync();
-                        mma(ring2 + s * kTileBytes, qbuf + (it2 % kQBufs) * SL::kQBytes,
-                            tmem_base + static_cast<uint32_t>((kAcc + acc) * N));
-                        umma_commit(&b_full[acc]);
-                        umma_commit(&free2[s]);
-                        ++use2;
-                        ++b_it;
-                        if (++jt2 == item_of(r2).ntiles) {
-                            umma_commit(&q_empty[it2 % kQBufs]);  // the item's query rows are free
-                            r2 = next_item(r2 + 1);
-                            ++it2;
-                            jt2 = 0;
+                if (r1 < R) {
+                    if (!q_out) {
+                        // The item's window query rows: per head of the batch two boxes of 64
+                        // dims x W_PAD rows in the MMA's 128-byte-swizzled layout.  Rows past w
+                        // (the next sequence's, or zeros past the end) and head slots past the
+                        // batch's heads land in columns that the epilogues mask out.
+                        const int qb = it1 % kQBufs;
+                        if (mbar_test(&q_empty[qb], ((it1 / kQBufs) & 1) ^ 1)) {
+                            uint8_t* qdst = qbuf + qb * SL::kQBytes;
+                            const int first_row = p.batch_first[U1.batch], nheads = p.batch_nheads[U1.batch];
+                            mbar_arrive_expect_tx(&q_full[qb], static_cast<uint32_t>(nheads * W_PAD * 256));
+                            for (int slot = 0; slot < nheads; ++slot) {
+                                const int h = p.sel_heads[first_row + slot];
+                                uint8_t* d = qdst + slot * W_PAD * 128;
+                                tma_load_3d(d, &p.tmap_q, &q_full[qb], 0, h, U1.seq * p.w);
+                                tma_load_3d(d + SL::kQHalf, &p.tmap_q, &q_full[qb], 64, h, U1.seq * p.w);
+                            }
+                            q_out = true;
+                            did = true;
                         }
+                    }
+                    const int s = use1 % kP1Slots;
+                    if (q_out && mbar_test(&free1[s], ((use1 / kP1Slots) & 1) ^ 1)) {
+                        mbar_arrive_expect_tx(&full1[s], kTileBytes);
+                        uint8_t* dst = ring1 + s * kTileBytes;
+                        const int g = p.batch_group[U1.batch];
+                        const int tok = U1.seq_start + (I1.tile0 + jt1) * kTileKeys;
+                        tma_load_3d_hint(dst, &p.tmap_k, &full1[s], 0, g, tok, pol1);
+                        tma_load_3d_hint(dst + kHalfBytes, &p.tmap_k, &full1[s], 64, g, tok, pol1);
+                        ++use1;
                         did = true;
+                        if (++jt1 == I1.ntiles) {
+                            jt1 = 0;
+                            ++it1;
+                            q_out = false;
+                            r1 = next_item(r1 + 1);
+                            if (r1 < R) {
+                                I1 = item_of(r1);
+                                U1 = p.units[I1.unit];
+                            }
+                        }
                     }
                 }
-                if (r1 < R) {
-                    if (!q_ready) {
-                        q_ready = mbar_test(&q_full[it1 % kQBufs], (it1 / kQBufs) & 1);
-                        if (q_ready) tc_fence_after_sync();
-                    }
-                    const int s = use1 % kP1Slots, acc = a_it % kAcc;
-                    if (q_ready && mbar_test(&full1[s], (use1 / kP1Slots) & 1) &&
-                        mbar_test(&a_empty[acc], ((a_it / kAcc) & 1) ^ 1)) {
-                        tc_fence_after_sync();
-                        mma(ring1 + s * kTileBytes, qbuf + (it1 % kQBufs) * SL::kQBytes,
-                            tmem_base + static_cast<uint32_t>(acc * N));
-                        umma_commit(&a_full[acc]);
-                        umma_commit(&free1[s]);
-                        ++use1;
-                        ++a_it;
-                        if (++jt1 == item_of(r1).ntiles) {
-                            r1 = next_item(r1 + 1);
-                            ++it1;
-                            jt1 = 0;
-                            q_ready = false;
-                        }
+                // pass 2 of an item follows its pass-1 loads, so that it reads L2
+                if (r2 < R && it2 < it1) {
+                    const int s = use2 % kP2Slots;
+                    if (mbar_test(&free2[s], ((use2 / kP2Slots) & 1) ^ 1)) {
+                        mbar_arrive_expect_tx(&full2[s], kTileBytes);
+                        uint8_t* dst = ring2 + s * kTileBytes;
+                        const int g = p.batch_group[U2.batch];
+                        const int tok = U2.seq_start + (I2.tile0 + jt2) * kTileKeys;
+                        tma_load_3d_hint(dst, &p.tmap_k, &full2[s], 0, g, tok, pol2);
+                        tma_load_3d_hint(dst + kHalfBytes, &p.tmap_k, &full2[s], 64, g, tok, pol2);
+                        ++use2;
                         did = true;
+                        if (++jt2 == I2.ntiles) {
+                            jt2 = 0;
+                            ++it2;
+                            r2 = next_item(r2 + 1);
+                            if (r2 < R) {
+                                I2 = item_of(r2);
+                                U2 = p.units[I2.unit];
+                            }
+                        }
                     }
                 }
                 if (did) {
                     idle = 0;
                     t0 = clock64();
                 } else {
-                    // Nothing ready: back off (32 ns doubling to 256 ns), so that the polls do
-                    // not take issue slots from the epilogue warps of this SM sub-partition.
-                    __nanosleep(32u << (idle < 3u ? idle : 3u));
+                    __nanosleep(32u << (idle < 1u ? idle : 1u));
                     if ((++idle & 15u) == 0u && (*abort || clock64() - t0 > lim)) {
                         ok = false;
                         break;
@@ -332,11 +270,73 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             }
             if (!ok) {
                 *abort = 1;
-                record_error(p.status, kDevTimeout, 11);
+                record_error(p.status, kDevTimeout, 10);
             }
-            umma_commit(done);
+            // Let every issued copy land before the block may exit.
             volatile int never = 0;
-            mbar_wait(done, 0, &never);
+            for (int k = (use1 > kP1Slots ? use1 - kP1Slots : 0); k < use1; ++k)
+                mbar_wait(&full1[k % kP1Slots], (k / kP1Slots) & 1, &never);
+            for (int k = (use2 > kP2Slots ? use2 - kP2Slots : 0); k < use2; ++k)
+                mbar_wait(&full2[k % kP2Slots], (k / kP2Slots) & 1, &never);
+            const int nq = it1 + (q_out ? 1 : 0);
+            for (int k = (nq > kQBufs ? nq - kQBufs : 0); k < nq; ++k)
+                mbar_wait(&q_full[k % kQBufs], (k / kQBufs) & 1, &never);
+        }
+    } else if (warp == 1 || warp == 2) {
+        // ------------------------------------------------------------ MMA issuers
+        // warp 1: pass 1, warp 2: pass 2, so that neither pass's issue waits behind the other's.
+        if (lane == 0) {
+            const bool first = warp == 1;
+            const int nslots = first ? kP1Slots : kP2Slots;
+            const uint8_t* ring = first ? ring1 : ring2;
+            uint64_t* full = first ? full1 : full2;
+            uint64_t* freed = first ? free1 : free2;
+            uint64_t* acc_full = first ? a_full : b_full;
+            uint64_t* acc_empty = first ? a_empty : b_empty;
+            uint64_t* fin = first ? done : done + 1;
+            const uint32_t d0 = tmem_base + static_cast<uint32_t>((first ? 0 : kAcc) * N);
+            int it = 0, use = 0;
+            bool ok = true;
+            for (int r = 0; ok && r < R; ++r) {
+                const int n = item_of(r).ntiles;
+                if (n == 0) continue;
+                const int qb = it % kQBufs;
+                if (!mbar_wait(&q_full[qb], (it / kQBufs) & 1, abort, lim)) {
+                    ok = false;
+                    break;
+                }
+                const uint32_t b0 = smem_u32(qbuf + qb * SL::kQBytes);
+                for (int jt = 0; jt < n; ++jt, ++use) {
+                    const int s = use % nslots, acc = use % kAcc;
+                    if (!mbar_wait(&full[s], (use / nslots) & 1, abort, lim) ||
+                        !mbar_wait(&acc_empty[acc], ((use / kAcc) & 1) ^ 1, abort, lim)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after_sync();
+                    const uint32_t a0 = smem_u32(ring + s * kTileBytes);
+                    const uint32_t d = d0 + static_cast<uint32_t>(acc * N);
+#pragma unroll
+                    for (int kk = 0; kk < kHeadDim / 16; ++kk) {
+                        const uint32_t koff = (kk & 3) * 32;
+                        const uint64_t ad = sdesc_k_major_sw128(a0 + (kk >> 2) * kHalfBytes + koff);
+                        const uint64_t bd = sdesc_k_major_sw128(b0 + (kk >> 2) * SL::kQHalf + koff);
+                        umma_bf16(d, ad, bd, kIdesc, kk > 0 ? 1u : 0u);
+                    }
+                    umma_commit(&acc_full[acc]);
+                    umma_commit(&freed[s]);
+                }
+                if (!ok) break;
+                umma_commit(&q_empty[qb]);  // this pass is done with the item's query rows
+                ++it;
+            }
+            if (!ok) {
+                *abort = 1;
+                record_error(p.status, kDevTimeout, first ? 11 : 12);
+            }
+            umma_commit(fin);
+            volatile int never = 0;
+            mbar_wait(fin, 0, &never);
         }
         __syncwarp();
     } else if (warp == 3) {
