@@ -115,14 +115,22 @@ __device__ __forceinline__ void setmaxnreg_dec() {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(R));
 }
 
-// A barrier of one epilogue warpgroup built on an mbarrier of 128 arrivals, so that the wait
-// is bounded like every other wait of the kernel.
+// A barrier of one epilogue warpgroup on an mbarrier of kGroupArrivals arrivals, one per warp:
+// each warp converges, its lane 0 arrives and waits (bounded, like every other wait of the
+// kernel), and the warp converges again, which carries the ordering to the other lanes.
+constexpr int kGroupArrivals = 4;
 __device__ __forceinline__ bool group_sync(uint64_t* bar, uint32_t& phase, volatile int* abort,
                                            long long limit) {
-    mbar_arrive(bar);
-    const bool ok = mbar_wait(bar, phase, abort, limit);
+    __syncwarp();
+    int ok = 1;
+    if ((threadIdx.x & 31) == 0) {
+        mbar_arrive(bar);
+        ok = mbar_wait(bar, phase, abort, limit) ? 1 : 0;
+    }
+    __syncwarp();
+    ok = __shfl_sync(0xffffffffu, ok, 0);
     phase ^= 1;
-    return ok;
+    return ok != 0;
 }
 
 // Warp-wide sums of C per-lane columns (C = 8, 16 or 32) by recursive halving: at each level
@@ -320,8 +328,7 @@ __device__ __forceinline__ bool unit_lse(const ScoreParams& p, const ScoreUnit& 
                 break;
             }
         }
-        __threadfence();
-        verdict[0] = got ? 1 : 0;
+        verdict[0] = got ? 1 : 0;  // the acquire load orders the reads of the partials below
     }
     if (!group_sync(gbar, gphase, abort, lim) || verdict[0] == 0) return false;
     constexpr int kPairs = N / 2, kParts = 128 / kPairs, kU = 20;

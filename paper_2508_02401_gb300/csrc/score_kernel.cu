@@ -60,12 +60,70 @@ struct SmemLayout {
                          kQFull = kBEmpty + kAcc, kQEmpty = kQFull + kQBufs,
                          kDone = kQEmpty + kQBufs, kGroup = kDone + 2,  // A0 A1 B
                          kPubFull = kGroup + 3, kPubEmpty = kPubFull + 2,
-                         kNumBars = kPubEmpty + 2;
+                         kLseFull = kPubEmpty + 2, kLseEmpty = kLseFull + 2,
+                         kNumBars = kLseEmpty + 2;
     static constexpr int kTmemSlot = kBars + 8 * kNumBars;
     static constexpr int kAbort = kTmemSlot + 4;
     static constexpr int kBytes = kAbort + 4;
     static constexpr int kDynamic = kBytes + 1024;      // slack to align the base to 1024 B
 };
+
+// The unit's -lse per column (log2 units, -inf for a column without a real window row or
+// without a visible key) from its items' partials, by one warp: lane 0 waits (bounded acquire
+// spin) until every item of the unit has published, then lane l combines the column pair
+// (2l, 2l + 1) over the items, kU partials in flight.
+template <int N, int W_PAD>
+__device__ __forceinline__ bool warp_unit_lse(const ScoreParams& p, const ScoreUnit& U, int unit,
+                                              int lane, float* nlse, volatile int* abort,
+                                              long long lim) {
+    constexpr int kNW = N / kCols, kPairs = N / 2, kU = 4;
+    int got = 1;
+    if (lane == 0) {
+        const int target = U.nitems * kNW;
+        const long long t0 = clock64();
+        for (uint32_t k = 1; ld_acquire(p.counters + unit) < target; ++k) {
+            __nanosleep(32);
+            if ((k & 63u) == 0u && (*abort || clock64() - t0 > lim)) {
+                got = 0;
+                break;
+            }
+        }
+    }
+    __syncwarp();  // the acquire above orders the other lanes' reads of the partials too
+    if (__shfl_sync(0xffffffffu, got, 0) == 0) return false;
+    if (lane < kPairs) {
+        const float4* src = reinterpret_cast<const float4*>(p.partials + static_cast<size_t>(U.first_item) * N) + lane;
+        float M0 = -INFINITY, S0 = 0.f, M1 = -INFINITY, S1 = 0.f;
+        for (int k0 = 0; k0 < U.nitems; k0 += kU) {
+            float4 pr[kU];
+#pragma unroll
+            for (int u = 0; u < kU; ++u)
+                pr[u] = k0 + u < U.nitems ? __ldcg(src + static_cast<size_t>(k0 + u) * kPairs)
+                                          : make_float4(-INFINITY, 0.f, -INFINITY, 0.f);
+#pragma unroll
+            for (int u = 0; u < kU; ++u) {
+                float Mn = fmaxf(M0, pr[u].x);
+                if (Mn > -INFINITY) {
+                    S0 = S0 * ex2_approx(M0 - Mn) + pr[u].y * ex2_approx(pr[u].x - Mn);
+                    M0 = Mn;
+                }
+                Mn = fmaxf(M1, pr[u].z);
+                if (Mn > -INFINITY) {
+                    S1 = S1 * ex2_approx(M1 - Mn) + pr[u].w * ex2_approx(pr[u].z - Mn);
+                    M1 = Mn;
+                }
+            }
+        }
+        const int nheads = p.batch_nheads[U.batch];
+        const int c0 = 2 * lane, c1 = c0 + 1;
+        const bool real0 = (c0 % W_PAD) < p.w && (c0 / W_PAD) < nheads;
+        const bool real1 = (c1 % W_PAD) < p.w && (c1 / W_PAD) < nheads;
+        nlse[c0] = real0 && S0 > 0.f ? -(M0 + lg2_approx(S0)) : -INFINITY;
+        nlse[c1] = real1 && S1 > 0.f ? -(M1 + lg2_approx(S1)) : -INFINITY;
+    }
+    __syncwarp();
+    return true;
+}
 
 template <int N, int W_PAD>
 __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constant__ ScoreParams p) {
@@ -98,11 +156,11 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
     uint64_t* group = bars + SL::kGroup;        // one per epilogue warpgroup: A0 A1 B
     uint64_t* pub_full = bars + SL::kPubFull;   // pass-1 partials of an item stored (item parity)
     uint64_t* pub_empty = bars + SL::kPubEmpty;
+    uint64_t* lse_full = bars + SL::kLseFull;   // a unit's lse is in nlse_s[item parity]
+    uint64_t* lse_empty = bars + SL::kLseEmpty; // pass 2 is done with nlse_s[item parity]
     // scratch of the epilogues (static, so that its accesses are shared-memory instructions)
     __shared__ float2 red_a[2][2][128];  // [item parity][warpgroup][warp * 32 + lane]
-    __shared__ float2 red_b[256];        // [part * N + column]
-    __shared__ __align__(16) float nlse_s[64];  // -lse per column of the current pass-2 item
-    __shared__ volatile int verdict[1];
+    __shared__ __align__(16) float nlse_s[2][64];  // -lse per column, by item parity
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + SL::kTmemSlot);
     volatile int* abort = reinterpret_cast<volatile int*>(sm + SL::kAbort);
 
@@ -129,10 +187,12 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         }
         mbar_init(&done[0], 1);
         mbar_init(&done[1], 1);
-        for (int i = 0; i < 3; ++i) mbar_init(&group[i], 128);
+        for (int i = 0; i < 3; ++i) mbar_init(&group[i], kGroupArrivals);
         for (int i = 0; i < 2; ++i) {
             mbar_init(&pub_full[i], 32 * kNW);
             mbar_init(&pub_empty[i], 1);
+            mbar_init(&lse_full[i], 1);
+            mbar_init(&lse_empty[i], 4);  // one arrival per pass-2 warp
         }
         *abort = 0;
         fence_mbar_init();
@@ -340,25 +400,40 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         }
         __syncwarp();
     } else if (warp == 3) {
-        // ------------------------------------------------------------ publisher
-        // Once both pass-1 warpgroups have stored an item's partials, one release on the
-        // unit's arrival counter makes them visible GPU-wide; the GPU-scope fence this takes
-        // stalls only this lane, not the pass-1 warps.
-        if (lane == 0) {
-            int it = 0;
-            for (int r = 0; r < R; ++r) {
-                const ScoreItem& I = item_of(r);
-                if (I.ntiles == 0) continue;
-                if (!mbar_wait(&pub_full[it & 1], (it >> 1) & 1, abort, lim)) {
-                    *abort = 1;
-                    record_error(p.status, kDevTimeout, 17);
-                    break;
+        // ------------------------------------------------------------ publisher and combiner
+        // Per item: once both pass-1 warpgroups have stored its partials (their pub_full
+        // arrival releases them to lane 0 at CTA scope), one release add on the unit's arrival
+        // counter makes them visible GPU-wide (a release is cumulative).  Then the warp waits
+        // for the unit's other items, combines all their partials into the unit's lse and
+        // leaves it in nlse_s for pass 2, which meanwhile still works on the item before: the
+        // exchange stays off pass 2's path unless pass 1 elsewhere is late.
+        int it = 0;
+        bool ok = true;
+        for (int r = 0; r < R; ++r) {
+            const ScoreItem I = item_of(r);
+            if (I.ntiles == 0) continue;
+            const int buf = it & 1;
+            int good = 1;
+            if (lane == 0) {
+                if (!mbar_wait(&pub_full[buf], (it >> 1) & 1, abort, lim)) {
+                    good = 0;
+                } else {
+                    red_release_add(p.counters + I.unit, kNW);
+                    mbar_arrive(&pub_empty[buf]);
+                    good = mbar_wait(&lse_empty[buf], ((it >> 1) & 1) ^ 1, abort, lim) ? 1 : 0;
                 }
-                __threadfence();
-                red_release_add(p.counters + I.unit, kNW);
-                mbar_arrive(&pub_empty[it & 1]);
-                ++it;
             }
+            if (__shfl_sync(0xffffffffu, good, 0) == 0 ||
+                !warp_unit_lse<N, W_PAD>(p, p.units[I.unit], I.unit, lane, nlse_s[buf], abort, lim)) {
+                ok = false;
+                break;
+            }
+            if (lane == 0) mbar_arrive(&lse_full[buf]);
+            ++it;
+        }
+        if (!ok && lane == 0) {
+            *abort = 1;
+            record_error(p.status, kDevTimeout, 17);
         }
     }
     } else if (warp < kWarpB) {
@@ -447,12 +522,9 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         // One warpgroup over all N columns; lse sits in shared memory and is read by every
         // lane of a warp at the same address.
         const int eq = warp & 3;
-        const int wtid = threadIdx.x - kWarpB * 32;  // 0 .. 127
         const uint32_t lane_base = static_cast<uint32_t>(eq * 32) << 16;
-        uint64_t* gbar = &group[2];
-        uint32_t gphase = 0;
         constexpr int kHeads = N / W_PAD;  // head slots of the MMA's columns
-        int b_it = 0;
+        int b_it = 0, n_item = 0;
         bool ok = true;
         for (int r = 0; ok && r < R; ++r) {
             const ScoreItem I = p.items[r * G + blockIdx.x];
@@ -464,15 +536,16 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             const int T = p.T;
             const float sl2 = p.sl2;
             float* const scores = p.scores;
-            uint64_t colmask = 0;  // columns that hold a real window row
-#pragma unroll
-            for (int c = 0; c < N; ++c)
-                if ((c % W_PAD) < p.w && (c / W_PAD) < nheads) colmask |= 1ull << c;
-            // ---------------------------------------------------- exchange with the unit
-            if (!unit_lse<N>(p, U, I.unit, wtid, gbar, gphase, verdict, red_b, nlse_s, colmask, abort, lim)) {
+            // ---------------------------------------------------- the unit's lse (warp 3)
+            const int buf = n_item & 1;
+            int good = 1;
+            if (lane == 0) good = mbar_wait(&lse_full[buf], (n_item >> 1) & 1, abort, lim) ? 1 : 0;
+            __syncwarp();
+            if (__shfl_sync(0xffffffffu, good, 0) == 0) {
                 ok = false;
                 break;
             }
+            const float* nlse = nlse_s[buf];
             // ---------------------------------------------------- the item's tiles
             for (int jt = 0; jt < n; ++jt, ++b_it) {
                 const int acc = b_it % kAcc;
@@ -497,9 +570,9 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                 if (lane == 0) mbar_arrive(&b_empty[acc]);  // the accumulator is free
                 float accum[kHeads];
                 if (!edge) {
-                    prob_sums<N, W_PAD, false>(vv, sl2, nlse_s, 0, accum);
+                    prob_sums<N, W_PAD, false>(vv, sl2, nlse, 0, accum);
                 } else {  // row r sees key j iff r >= j - P; keys past L are padding
-                    prob_sums<N, W_PAD, true>(vv, sl2, nlse_s, j < L ? j - P : (1 << 30), accum);
+                    prob_sums<N, W_PAD, true>(vv, sl2, nlse, j < L ? j - P : (1 << 30), accum);
                 }
                 if (j < L) {
                     const size_t col = static_cast<size_t>(U.seq_start) + j;
@@ -508,6 +581,9 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                         if (h < nheads) scores[static_cast<size_t>(first + h) * T + col] = accum[h];
                 }
             }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&lse_empty[buf]);  // this warp is done with the lse
+            ++n_item;
         }
         if (!ok) {
             *abort = 1;

@@ -93,7 +93,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_lse_kernel(const __grid_con
             mbar_init(&q_empty[i], 1);
         }
         mbar_init(done, 1);
-        for (int i = 0; i < kEpiWG; ++i) mbar_init(&group[i], 128);
+        for (int i = 0; i < kEpiWG; ++i) mbar_init(&group[i], kGroupArrivals);
         *abort = 0;
         fence_mbar_init();
         tma_prefetch_desc(&p.tmap_k);

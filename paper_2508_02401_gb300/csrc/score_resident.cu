@@ -186,7 +186,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_resident_kernel(const __gri
             mbar_init(&q_empty[i], 1);
         }
         mbar_init(done, 1);
-        for (int i = 0; i < 3; ++i) mbar_init(&group[i], 128);
+        for (int i = 0; i < 3; ++i) mbar_init(&group[i], kGroupArrivals);
         for (int i = 0; i < 2; ++i) {
             mbar_init(&pub_full[i], 32 * kNW);
             mbar_init(&pub_empty[i], 1);
@@ -339,7 +339,6 @@ __global__ void __launch_bounds__(kThreads, 1) score_resident_kernel(const __gri
                         record_error(p.status, kDevTimeout, 22);
                         break;
                     }
-                    __threadfence();
                     red_release_add(p.counters + I.unit, kNW);
                     mbar_arrive(&pub_empty[it & 1]);
                     ++it;
