@@ -193,8 +193,11 @@ ckv_status plan_score(const Plan& pl, const ckv_batch* b, int skip_le, int ctas,
     constexpr int kL2Tiles = 8;        // pass 1 runs up to two items ahead, so each CTA keeps
                                        // ~2 items in L2 (evict-last hint) until pass 2 reads
                                        // them: 2 x 8 tiles x 32 KiB x 152 CTAs ~ 80 MB
-    constexpr double kExchange = 12.0; // publish, exchange and combine, in tile-load times
-    constexpr double kPass2 = 0.4;     // pass 2 per tile from L2, relative to a pass-1 load
+    constexpr double kExchange = 4.0;  // publish, exchange and combine, in tile-load times
+                                       // (combined ahead of pass 2, so mostly hidden)
+    constexpr double kPass2 = 1.0;     // pass 2 per tile from L2, relative to a pass-1 load:
+                                       // measured about as fast (each pass has its own issuer
+                                       // and ring, and both share the SM's copy bandwidth)
     // The resident kernel when every unit fits one round of items that fit in TMEM.
     const int c_res = 512 / pl.n_cols;
     const bool fits = static_cast<long long>(max_tiles) <= static_cast<long long>(c_res) * ctas;
