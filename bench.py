@@ -35,14 +35,15 @@ HBM_FALLBACK_GBS = 6800.0
 
 # DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) of one scoring launch (one layer)
 # per workload, from the ncu captures summarised in profiles/ (score_kernel_llama8b_l8192.md,
-# score_resident_paper_llama8b_l8192.md, score_lse_llama8b_l8192.md; "+lse": bench.py --lse),
+# score_kernel_needle_l131072.md, score_resident_paper_llama8b_l8192.md,
+# score_lse_llama8b_l8192.md; "+lse": bench.py --lse),
 # keyed by the sha256 of the scoring kernels' sources (SCORE_SOURCES); a changed kernel reports
-# null until it is captured again.
+# null until it is captured again.  Figures that ncu printed in MB are rounded to 10 kB.
 SCORE_SOURCES = ('score_kernel.cu', 'score_resident.cu', 'score_lse.cu', 'score_common.cuh', 'ckv_device.cuh')
 SCORE_TRAFFIC = {
-    "a73eeb2e6dadd90875af204f73bc575a255a509fc1ae824331b36d2fdc214004": {
-        "llama8b_l8192": 16992768, "paper_llama8b_l8192": 8493056,
-        "llama8b_l8192+lse": 16950528, "needle_l131072+lse": 274175232,
+    "7342ede02588be85a088ff789a14e1dd86c0b927d5aa47aa56ddda71f6d6a90d": {
+        "llama8b_l8192": 16989952, "paper_llama8b_l8192": 8500000, "needle_l131072": 299342080,
+        "llama8b_l8192+lse": 16950000, "needle_l131072+lse": 274310000,
     },
 }
 # Sequences up to this many tokens are selected by one block per (sequence, KV head)

@@ -306,6 +306,12 @@ __device__ __forceinline__ bool item_partials(float (&m)[kCols], float (&s)[kCol
     return true;
 }
 
+template <int N>
+__device__ __forceinline__ bool unit_combine(const ScoreParams& p, const ScoreUnit& U, int wtid,
+                                             uint64_t* gbar, uint32_t& gphase, float2* red_b,
+                                             float* nlse, uint64_t colmask, volatile int* abort,
+                                             long long lim);
+
 // The unit's lse per column, for the pass-2 warpgroup (128 threads): thread 0 waits (bounded
 // acquire spin) until every item of the unit has published its partials, then the warpgroup
 // combines them -- column pairs by 16-byte loads, the items split over kParts groups of
@@ -331,6 +337,16 @@ __device__ __forceinline__ bool unit_lse(const ScoreParams& p, const ScoreUnit& 
         verdict[0] = got ? 1 : 0;  // the acquire load orders the reads of the partials below
     }
     if (!group_sync(gbar, gphase, abort, lim) || verdict[0] == 0) return false;
+    return unit_combine<N>(p, U, wtid, gbar, gphase, red_b, nlse, colmask, abort, lim);
+}
+
+// The combining part of unit_lse, for a warpgroup that already knows (by an acquire, carried
+// to it by a CTA-scope barrier) that every item of the unit has published its partials.
+template <int N>
+__device__ __forceinline__ bool unit_combine(const ScoreParams& p, const ScoreUnit& U, int wtid,
+                                             uint64_t* gbar, uint32_t& gphase, float2* red_b,
+                                             float* nlse, uint64_t colmask, volatile int* abort,
+                                             long long lim) {
     constexpr int kPairs = N / 2, kParts = 128 / kPairs, kU = 20;
     static_assert(kParts * N <= 256, "red_b holds 256 entries");
     const int c2 = wtid % kPairs, part = wtid / kPairs;

@@ -44,6 +44,7 @@ constexpr int kP1Slots = 3;                           // pass-1 ring (HBM)
 constexpr int kP2Slots = 2;                           // pass-2 ring (L2)
 constexpr int kAcc = 4;                               // TMEM accumulators per pass
 constexpr int kQBufs = 3;                             // query-row buffers: pass 1 runs two items ahead
+constexpr int kWarpCombineMax = 16;                   // units of more items: pass 2 combines (128 threads)
 
 template <int N>
 struct SmemLayout {
@@ -70,12 +71,13 @@ struct SmemLayout {
 
 // The unit's -lse per column (log2 units, -inf for a column without a real window row or
 // without a visible key) from its items' partials, by one warp: lane 0 waits (bounded acquire
-// spin) until every item of the unit has published, then lane l combines the column pair
-// (2l, 2l + 1) over the items, kU partials in flight.
+// spin) until every item of the unit has published, then, if `combine`, lane l combines the
+// column pair (2l, 2l + 1) over the items, kU partials in flight (a unit of many items is
+// combined by the pass-2 warpgroup instead, which has the threads for more loads in flight).
 template <int N, int W_PAD>
 __device__ __forceinline__ bool warp_unit_lse(const ScoreParams& p, const ScoreUnit& U, int unit,
-                                              int lane, float* nlse, volatile int* abort,
-                                              long long lim) {
+                                              int lane, float* nlse, bool combine,
+                                              volatile int* abort, long long lim) {
     constexpr int kNW = N / kCols, kPairs = N / 2, kU = 4;
     int got = 1;
     if (lane == 0) {
@@ -91,7 +93,7 @@ __device__ __forceinline__ bool warp_unit_lse(const ScoreParams& p, const ScoreU
     }
     __syncwarp();  // the acquire above orders the other lanes' reads of the partials too
     if (__shfl_sync(0xffffffffu, got, 0) == 0) return false;
-    if (lane < kPairs) {
+    if (combine && lane < kPairs) {
         const float4* src = reinterpret_cast<const float4*>(p.partials + static_cast<size_t>(U.first_item) * N) + lane;
         float M0 = -INFINITY, S0 = 0.f, M1 = -INFINITY, S1 = 0.f;
         for (int k0 = 0; k0 < U.nitems; k0 += kU) {
@@ -161,6 +163,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
     // scratch of the epilogues (static, so that its accesses are shared-memory instructions)
     __shared__ float2 red_a[2][2][128];  // [item parity][warpgroup][warp * 32 + lane]
     __shared__ __align__(16) float nlse_s[2][64];  // -lse per column, by item parity
+    __shared__ float2 red_b[256];                     // pass-2 combine of a many-item unit
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + SL::kTmemSlot);
     volatile int* abort = reinterpret_cast<volatile int*>(sm + SL::kAbort);
 
@@ -423,8 +426,10 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                     good = mbar_wait(&lse_empty[buf], ((it >> 1) & 1) ^ 1, abort, lim) ? 1 : 0;
                 }
             }
+            const ScoreUnit& U = p.units[I.unit];
             if (__shfl_sync(0xffffffffu, good, 0) == 0 ||
-                !warp_unit_lse<N, W_PAD>(p, p.units[I.unit], I.unit, lane, nlse_s[buf], abort, lim)) {
+                !warp_unit_lse<N, W_PAD>(p, U, I.unit, lane, nlse_s[buf], U.nitems <= kWarpCombineMax,
+                                         abort, lim)) {
                 ok = false;
                 break;
             }
@@ -522,7 +527,10 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         // One warpgroup over all N columns; lse sits in shared memory and is read by every
         // lane of a warp at the same address.
         const int eq = warp & 3;
+        const int wtid = threadIdx.x - kWarpB * 32;  // 0 .. 127
         const uint32_t lane_base = static_cast<uint32_t>(eq * 32) << 16;
+        uint64_t* gbar = &group[2];
+        uint32_t gphase = 0;
         constexpr int kHeads = N / W_PAD;  // head slots of the MMA's columns
         int b_it = 0, n_item = 0;
         bool ok = true;
@@ -544,6 +552,16 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             if (__shfl_sync(0xffffffffu, good, 0) == 0) {
                 ok = false;
                 break;
+            }
+            if (U.nitems > kWarpCombineMax) {  // warp 3 only acquired: combine here
+                uint64_t colmask = 0;           // columns that hold a real window row
+#pragma unroll
+                for (int c = 0; c < N; ++c)
+                    if ((c % W_PAD) < p.w && (c / W_PAD) < nheads) colmask |= 1ull << c;
+                if (!unit_combine<N>(p, U, wtid, gbar, gphase, red_b, nlse_s[buf], colmask, abort, lim)) {
+                    ok = false;
+                    break;
+                }
             }
             const float* nlse = nlse_s[buf];
             // ---------------------------------------------------- the item's tiles
