@@ -95,6 +95,9 @@ def _args():
     ap.add_argument("--srs", action="store_true",
                     help="time the Semantic Retrieval Score accumulation (Eq. 5) instead: every "
                          "head scored, the window rows as decode steps, all of them in the answer")
+    ap.add_argument("--split-select", action="store_true",
+                    help="each layer as ckv_score_window then ckv_select_compact, the selection "
+                         "on a stream of its own, so that the next layer's scoring need not wait")
     ap.add_argument("--lse", action="store_true",
                     help="the window rows' lse given (as a prefill attention kernel returns it): "
                          "ckv_compress_layer_lse / ckv_score_window_lse, one pass over K")
@@ -259,33 +262,55 @@ def run_ours(args):
     ws = wss[0]
     stream = torch.cuda.Stream()
     side = [torch.cuda.Stream() for _ in range(nstreams)]
+    if args.split_select:  # per layer a score buffer; per stream a selection stream + workspace
+        sel_side = [torch.cuda.Stream() for _ in range(nstreams)]
+        sel_wss = [torch.zeros(ws_bytes, dtype=torch.uint8, device="cuda") for _ in range(nstreams)]
+        n_sel_max = max(ckv.ckv_keep_lengths(cfg, l, batch)[1] for l in range(nl))
+        for d in layers:
+            d["scores"] = torch.empty((n_sel_max, T), dtype=torch.float32, device="cuda")
 
-    def over_layers(fn):
+    def over_layers(fn, selections=False):
         # Layers are independent: layer l runs on side stream l % nstreams with its own
-        # workspace, so the calls of consecutive layers overlap on the GPU.
+        # workspace, so the calls of consecutive layers overlap on the GPU (and, with
+        # `selections`, its selection on the matching selection stream).
         for sd in side:
             sd.wait_stream(stream)
         for l, d in enumerate(layers):
             fn(l, d, wss[l % nstreams], side[l % nstreams])
-        for sd in side:
+        for sd in side + (sel_side if selections else []):
             stream.wait_stream(sd)
 
     def compress(l, d, w, st):
+        if args.split_select:
+            i = l % nstreams
+            if args.lse:
+                ckv.ckv_score_window_lse(cfg, l, batch, d["q"], d["k"], d["lse"], d["scores"], w,
+                                         stream=st)
+            else:
+                ckv.ckv_score_window(cfg, l, batch, d["q"], d["k"], d["scores"], w, stream=st)
+            ev = torch.cuda.Event()
+            ev.record(st)
+            sel_side[i].wait_event(ev)
+            ckv.ckv_select_compact(cfg, l, batch, d["scores"], d["k"], d["v"], d["idx"],
+                                   d["cu_keep_dev"], d["k_out"], d["v_out"], sel_wss[i],
+                                   stream=sel_side[i])
+            return sel_side[i]  # the stream on which the layer's outputs are complete
         if args.lse:
             ckv.ckv_compress_layer_lse(cfg, l, batch, d["q"], d["k"], d["v"], d["lse"], d["idx"],
                                        d["cu_keep_dev"], d["k_out"], d["v_out"], w, stream=st)
         else:
             ckv.ckv_compress_layer(cfg, l, batch, d["q"], d["k"], d["v"], d["idx"], d["cu_keep_dev"],
                                    d["k_out"], d["v_out"], w, stream=st)
+        return st
 
     def step():
-        over_layers(compress)
+        over_layers(compress, selections=args.split_select)
 
     with torch.cuda.stream(stream):
         for _ in range(max(1, args.warmup)):
             step()
     torch.cuda.synchronize()
-    for w in wss:
+    for w in wss + (sel_wss if args.split_select else []):
         code, detail = ckv.ckv_read_device_status(w, stream=stream)
         if code != 0:
             raise RuntimeError(f"device status {code} ({detail}) after warm-up")
@@ -314,7 +339,7 @@ def run_ours(args):
         barrier()
     ms = _max_over_ranks(e0.elapsed_time(e1), world, "cuda")
     clocks = clk.summary()
-    for w in wss:
+    for w in wss + (sel_wss if args.split_select else []):
         code, detail = ckv.ckv_read_device_status(w, stream=stream)
         if code != 0:
             raise RuntimeError(f"device status {code} ({detail}) after the timed region")
@@ -416,7 +441,7 @@ def run_ours(args):
         # one layer overlap the other layers' compressions.
         copy_streams = [torch.cuda.Stream() for _ in range(2)]
         back = torch.cuda.Stream()
-        every = copy_streams + side + [back]
+        every = copy_streams + side + [back] + (sel_side if args.split_select else [])
 
         def e2e_step():
             for st in every:
@@ -433,9 +458,9 @@ def run_ours(args):
                 landed.record(cp)
                 st = side[l % nstreams]
                 st.wait_event(landed)
-                compress(l, d, wss[l % nstreams], st)
+                out_st = compress(l, d, wss[l % nstreams], st)
                 done = torch.cuda.Event()
-                done.record(st)
+                done.record(out_st)
                 back.wait_event(done)
                 with torch.cuda.stream(back):
                     oi[l].copy_(d["idx"], non_blocking=True)
@@ -476,7 +501,9 @@ def run_ours(args):
                        "graph": "one CUDA graph per step",
                        "streams": f"layers round-robin on {nstreams} streams, scoring capped at {cap} CTAs per call",
                        "lse": ("window-row lse given (PyTorch logsumexp outside the timed region; "
-                               "one pass over K)") if args.lse else "computed (two passes)"},
+                               "one pass over K)") if args.lse else "computed (two passes)",
+                       "calls": ("ckv_score_window + ckv_select_compact, the selection on a stream "
+                                 "of its own") if args.split_select else "ckv_compress_layer"},
             "roofline": roofline,
             "layer_roofline": {"bound": "hbm", "achieved": round(layer_gbs, 1), "peak": hbm_peak,
                                "unit": "GB/s", "frac": round(layer_gbs / hbm_peak, 4),

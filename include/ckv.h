@@ -53,7 +53,7 @@
 extern "C" {
 #endif
 
-#define CKV_ABI_VERSION 3
+#define CKV_ABI_VERSION 4
 
 #if defined(__GNUC__)
 #define CKV_API __attribute__((visibility("default")))
@@ -201,6 +201,21 @@ CKV_API ckv_status ckv_gather_compact(const ckv_config* cfg, const ckv_batch* ba
                               int64_t head_stride, const int32_t* idx,
                               const int32_t* cu_keep_dev, void* k_out, void* v_out,
                               void* workspace, size_t workspace_bytes, ckv_stream stream);
+
+/* Steps 2-4 for one layer, fused (the selection half of ckv_compress_layer): pooling, top-k,
+ * compaction and the K/V gather from the scores ckv_score_window (or ckv_score_window_lse)
+ * wrote.  Splitting a layer into these two calls lets a caller put each layer's selection on
+ * a stream of its own, so that the next layer's scoring need not wait for it.
+ *   scores: device fp32 [n_sel, T] as ckv_score_window writes it (row i = the layer's i-th
+ *           selected head), 16-byte aligned; read only for sequences with L_s > B_l.
+ *   k, v, tok_stride, head_stride, idx, cu_keep_dev, k_out, v_out, pooled_out: as for
+ *           ckv_compress_layer.  The workspace may be another call's than the scoring's. */
+CKV_API ckv_status ckv_select_compact(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
+                                      const float* scores, const void* k, const void* v,
+                                      int64_t tok_stride, int64_t head_stride, int32_t* idx,
+                                      int32_t* cu_keep_dev, void* k_out, void* v_out,
+                                      float* pooled_out, void* workspace, size_t workspace_bytes,
+                                      ckv_stream stream);
 
 /* Steps 1-4 for one layer.  Sequences with L_s <= B_l are copied whole without being scored.
  * pooled_out may be NULL (then the pooled scores stay in the workspace). */

@@ -17,7 +17,8 @@ import numpy as np
 __all__ = [
     "CkvError", "Config", "Batch", "lib_path", "load",
     "ckv_workspace_size", "ckv_keep_lengths", "ckv_score_window", "ckv_pool", "ckv_select_topk",
-    "ckv_gather_compact", "ckv_compress_layer", "ckv_read_device_status", "ckv_status_string",
+    "ckv_gather_compact", "ckv_select_compact", "ckv_compress_layer", "ckv_read_device_status",
+    "ckv_status_string",
     "ckv_abi_version", "ckv_score_window_static", "POOL_MAX", "POOL_AVG", "POOL_THEN_SUM", "SUM_THEN_POOL",
     "SCOPE_KV_HEAD", "SCOPE_LAYER", "ckv_layer_error_scores", "ckv_allocate_budgets",
 ]
@@ -80,6 +81,7 @@ def load():
         "ckv_pool": ([cfg, I32, bat, P, P, P], C.c_int),
         "ckv_select_topk": ([cfg, I32, bat, P, P, P, P, SZ, P], C.c_int),
         "ckv_gather_compact": ([cfg, bat, I32, P, P, I64, I64, P, P, P, P, P, SZ, P], C.c_int),
+        "ckv_select_compact": ([cfg, I32, bat, P, P, P, I64, I64, P, P, P, P, P, P, SZ, P], C.c_int),
         "ckv_compress_layer": ([cfg, I32, bat, P, P, P, I64, I64, P, P, P, P, P, P, SZ, P], C.c_int),
         "ckv_read_device_status": ([P, P, I32, C.POINTER(I32), C.POINTER(I32)], C.c_int),
         "ckv_score_window_static": ([cfg, I32, bat, P, P, I64, I64, P, P, P], C.c_int),
@@ -265,6 +267,16 @@ def ckv_gather_compact(cfg, batch, t_keep, k, v, idx, cu_keep_dev, k_out, v_out,
                                      _ptr(v_out), _ptr(workspace),
                                      workspace.numel() * workspace.element_size(), _stream(stream)),
            "ckv_gather_compact")
+
+
+def ckv_select_compact(cfg, layer, batch, scores, k, v, idx, cu_keep_dev, k_out, v_out, workspace,
+                       pooled_out=None, stream=None, tok_stride=0, head_stride=0):
+    """Pool, top-k, compaction and gather of one layer from ckv_score_window's scores."""
+    _check(load().ckv_select_compact(cfg.ref, layer, batch.ref, _ptr(scores), _ptr(k), _ptr(v),
+                                     tok_stride, head_stride, _ptr(idx), _ptr(cu_keep_dev),
+                                     _ptr(k_out), _ptr(v_out), _ptr(pooled_out), _ptr(workspace),
+                                     workspace.numel() * workspace.element_size(), _stream(stream)),
+           "ckv_select_compact")
 
 
 def ckv_compress_layer(cfg, layer, batch, q_win, k, v, idx, cu_keep_dev, k_out, v_out, workspace,

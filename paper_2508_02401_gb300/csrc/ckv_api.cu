@@ -845,40 +845,17 @@ ckv_status ckv_gather_compact(const ckv_config* cfg, const ckv_batch* batch, int
 
 namespace {
 
-ckv_status compress_layer_impl(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
-                               const void* q_win, const void* k, const void* v,
-                               int64_t tok_stride, int64_t head_stride, const float* lse,
-                               int64_t lse_head_stride, int32_t* idx, int32_t* cu_keep_dev,
-                               void* k_out, void* v_out, float* pooled_out, void* workspace,
-                               size_t workspace_bytes, ckv_stream stream) {
-    Plan pl;
-    ckv_status st = make_plan(cfg, layer, pl);
-    if (st) return st;
-    int T = 0;
-    WsLayout l;
-    if ((st = check_batch(batch, &T)) || (st = resolve_strides(pl, &tok_stride, &head_stride)) ||
-        (st = check_kv(q_win, "q_win", T)) || (st = check_kv(k, "k", T)) ||
-        (st = check_kv(v, "v", T)) || (st = check_ws(pl, batch, T, workspace, workspace_bytes, &l)))
-        return st;
-    if (pooled_out && !aligned(pooled_out, 16))
-        return fail(CKV_ERR_INVALID_ARG, "pooled_out is not 16-byte aligned");
-    if (lse && (st = check_lse(pl, batch, lse, &lse_head_stride))) return st;
-    const int64_t tk = keep_total(batch, pl.budget);
-    if (tk > INT32_MAX) return fail(CKV_ERR_UNSUPPORTED, "too many kept tokens");
-    if (!cu_keep_dev) return fail(CKV_ERR_INVALID_ARG, "cu_keep_dev is NULL");
-    if (tk > 0 && (st = check_kv(idx, "idx", 1))) return st;
-    if (tk > 0 && ((st = check_kv(k_out, "k_out", 1)) || (st = check_kv(v_out, "v_out", 1))))
-        return st;
-    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+// The fused selection (pool, top-k, compaction, gather) of one layer from `scores`.
+ckv_status enqueue_select_fused(const Plan& pl, const ckv_config* cfg, const ckv_batch* batch, int T,
+                                const float* scores, const void* k, const void* v,
+                                int64_t tok_stride, int64_t head_stride, int32_t* idx,
+                                int32_t* cu_keep_dev, void* k_out, void* v_out, float* pooled_out,
+                                void* workspace, WsLayout& l, int64_t tk, cudaStream_t s) {
     uint8_t* w8 = static_cast<uint8_t*>(workspace);
-    float* scores = reinterpret_cast<float*>(w8 + l.scores);
     float* pooled = pooled_out ? pooled_out : reinterpret_cast<float*>(w8 + l.pooled);
     const int skip_le = pl.budget;  // sequences that fit the budget are kept whole
-    if ((st = enqueue_score(pl, batch, T, q_win, k, tok_stride, head_stride, scores, workspace, l,
-                            skip_le, s, kMaxScoreItems, lse, lse_head_stride)))
-        return st;
     SelectLaunch L = select_launch(pl, batch, T, static_cast<int>(tk), skip_le, cfg, workspace, &l);
-    L.scores = scores;
+    L.scores = const_cast<float*>(scores);
     L.pooled = pooled;
     L.idx = idx;
     L.cu_keep_dev = cu_keep_dev;
@@ -896,9 +873,79 @@ ckv_status compress_layer_impl(const ckv_config* cfg, int32_t layer, const ckv_b
     return e == cudaSuccess ? CKV_OK : cuda_fail(e, "launching the pool, selection and gather kernels");
 }
 
+// Checks of the selection's outputs, shared by the fused calls; *tk_out = kept tokens.
+ckv_status check_select_outputs(const ckv_batch* batch, const Plan& pl, int32_t* idx,
+                                int32_t* cu_keep_dev, void* k_out, void* v_out, float* pooled_out,
+                                int64_t* tk_out) {
+    ckv_status st;
+    if (pooled_out && !aligned(pooled_out, 16))
+        return fail(CKV_ERR_INVALID_ARG, "pooled_out is not 16-byte aligned");
+    const int64_t tk = keep_total(batch, pl.budget);
+    if (tk > INT32_MAX) return fail(CKV_ERR_UNSUPPORTED, "too many kept tokens");
+    if (!cu_keep_dev) return fail(CKV_ERR_INVALID_ARG, "cu_keep_dev is NULL");
+    if (tk > 0 && (st = check_kv(idx, "idx", 1))) return st;
+    if (tk > 0 && ((st = check_kv(k_out, "k_out", 1)) || (st = check_kv(v_out, "v_out", 1))))
+        return st;
+    *tk_out = tk;
+    return CKV_OK;
+}
+
+ckv_status compress_layer_impl(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
+                               const void* q_win, const void* k, const void* v,
+                               int64_t tok_stride, int64_t head_stride, const float* lse,
+                               int64_t lse_head_stride, int32_t* idx, int32_t* cu_keep_dev,
+                               void* k_out, void* v_out, float* pooled_out, void* workspace,
+                               size_t workspace_bytes, ckv_stream stream) {
+    Plan pl;
+    ckv_status st = make_plan(cfg, layer, pl);
+    if (st) return st;
+    int T = 0;
+    WsLayout l;
+    if ((st = check_batch(batch, &T)) || (st = resolve_strides(pl, &tok_stride, &head_stride)) ||
+        (st = check_kv(q_win, "q_win", T)) || (st = check_kv(k, "k", T)) ||
+        (st = check_kv(v, "v", T)) || (st = check_ws(pl, batch, T, workspace, workspace_bytes, &l)))
+        return st;
+    if (lse && (st = check_lse(pl, batch, lse, &lse_head_stride))) return st;
+    int64_t tk = 0;
+    if ((st = check_select_outputs(batch, pl, idx, cu_keep_dev, k_out, v_out, pooled_out, &tk)))
+        return st;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    float* scores = reinterpret_cast<float*>(static_cast<uint8_t*>(workspace) + l.scores);
+    const int skip_le = pl.budget;  // sequences that fit the budget are kept whole
+    if ((st = enqueue_score(pl, batch, T, q_win, k, tok_stride, head_stride, scores, workspace, l,
+                            skip_le, s, kMaxScoreItems, lse, lse_head_stride)))
+        return st;
+    return enqueue_select_fused(pl, cfg, batch, T, scores, k, v, tok_stride, head_stride, idx,
+                                cu_keep_dev, k_out, v_out, pooled_out, workspace, l, tk, s);
+}
+
 }  // namespace
 
 extern "C" {
+
+ckv_status ckv_select_compact(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
+                              const float* scores, const void* k, const void* v,
+                              int64_t tok_stride, int64_t head_stride, int32_t* idx,
+                              int32_t* cu_keep_dev, void* k_out, void* v_out, float* pooled_out,
+                              void* workspace, size_t workspace_bytes, ckv_stream stream) {
+    Plan pl;
+    ckv_status st = make_plan(cfg, layer, pl);
+    if (st) return st;
+    int T = 0;
+    WsLayout l;
+    if ((st = check_batch(batch, &T)) || (st = resolve_strides(pl, &tok_stride, &head_stride)) ||
+        (st = check_kv(k, "k", T)) || (st = check_kv(v, "v", T)) ||
+        (st = check_ws(pl, batch, T, workspace, workspace_bytes, &l)))
+        return st;
+    if (!scores) return fail(CKV_ERR_INVALID_ARG, "scores is NULL");
+    if (!aligned(scores, 16)) return fail(CKV_ERR_INVALID_ARG, "scores is not 16-byte aligned");
+    int64_t tk = 0;
+    if ((st = check_select_outputs(batch, pl, idx, cu_keep_dev, k_out, v_out, pooled_out, &tk)))
+        return st;
+    return enqueue_select_fused(pl, cfg, batch, T, scores, k, v, tok_stride, head_stride, idx,
+                                cu_keep_dev, k_out, v_out, pooled_out, workspace, l, tk,
+                                reinterpret_cast<cudaStream_t>(stream));
+}
 
 ckv_status ckv_compress_layer(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
                               const void* q_win, const void* k, const void* v,

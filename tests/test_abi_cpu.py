@@ -47,7 +47,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 
 def test_version_and_status_strings(lib):
-    assert ckv.ckv_abi_version() == 3
+    assert ckv.ckv_abi_version() == 4
     assert ckv.ckv_status_string(0) == "CKV_OK"
     assert ckv.ckv_status_string(3) == "CKV_ERR_WORKSPACE"
 

@@ -122,6 +122,19 @@ def test_full_size_workloads(name, layers, groups, path):
                 assert set(li.planted[0].tolist()) <= set(g["idx"][gi, ck[0]:ck[1]].tolist())
 
 
+@pytest.mark.parametrize("max_ctas", [9, 3])
+def test_reload_kernel_over_many_rounds(max_ctas):
+    """The reload kernel with its grid capped as the benchmark caps it: each CTA runs several
+    rounds of items, so the double-buffered lse of the publisher warp is reused across rounds,
+    and every unit has few enough items for that warp to combine them."""
+    wl = cs.workload("llama8b_l8192")
+    cfg = ckv.Config.from_workload(wl, score_path=ckv.SCORE_RELOAD, max_ctas=max_ctas)
+    li = wl.layer(13)
+    g = gu.run_gpu(wl, 13, li, cfg=cfg)
+    o = gu.run_oracle(wl, 13, li, want_kv=False)
+    gu.check_layer(wl, 13, li, g, o)
+
+
 def test_unselected_heads_are_ignored():
     wl = _wl(seqlens=(3000, 400))
     li = wl.layer(0)
@@ -181,6 +194,47 @@ def test_standalone_entry_points_match_the_fused_call():
             rows = [i for i, h in enumerate(sel) if h // 4 == gi]
             ref = sum(oracle.pool(sc[r, t0:t0 + P], wl.pool_kernel, 1) for r in rows)
             np.testing.assert_allclose(pl[gi, t0:t0 + P], ref, rtol=1e-5, atol=1e-30)
+
+
+def test_split_score_and_select_match_the_fused_call():
+    """ckv_score_window then ckv_select_compact (its own workspace, another stream) give the
+    fused call's indices, pooled scores and gathered rows bit for bit."""
+    wl = _wl(seqlens=(9000, 300, 20, 2500), num_q_heads=32, num_kv_heads=8)
+    layer = 1
+    li = wl.layer(layer)
+    cfg = ckv.Config.from_workload(wl)
+    batch = ckv.Batch(wl.cu_seqlens())
+    q, k, v = gu.to_dev(li.q_win), gu.to_dev(li.k), gu.to_dev(li.v)
+    ws_score, ws_select = ckv.new_workspace(cfg, layer, batch), ckv.new_workspace(cfg, layer, batch)
+    _, n_sel = ckv.ckv_keep_lengths(cfg, layer, batch)
+    T = batch.total_tokens
+    scores = torch.empty((n_sel, T), dtype=torch.float32, device="cuda")
+    pooled = torch.full((cfg.num_vectors, T), float("nan"), dtype=torch.float32, device="cuda")
+    idx, cu_keep_dev, k_out, v_out, cu_keep = ckv.new_outputs(cfg, layer, batch)
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+    ckv.ckv_score_window(cfg, layer, batch, q, k, scores, ws_score, stream=s1)
+    ev = torch.cuda.Event()
+    ev.record(s1)
+    s2.wait_event(ev)
+    ckv.ckv_select_compact(cfg, layer, batch, scores, k, v, idx, cu_keep_dev, k_out, v_out,
+                           ws_select, pooled_out=pooled, stream=s2)
+    torch.cuda.synchronize()
+    assert ckv.ckv_read_device_status(ws_score) == (0, 0)
+    assert ckv.ckv_read_device_status(ws_select) == (0, 0)
+    fused = gu.run_gpu(wl, layer, li)
+    np.testing.assert_array_equal(idx.cpu().numpy(), fused["idx"])
+    np.testing.assert_array_equal(cu_keep_dev.cpu().numpy(), fused["cu_keep_dev"])
+    np.testing.assert_array_equal(gu.to_host(k_out), fused["k_out"])
+    np.testing.assert_array_equal(gu.to_host(v_out), fused["v_out"])
+    # sequences that fit the budget are not scored by the fused call: compare pooled elsewhere
+    pl, fp = pooled.cpu().numpy(), fused["pooled"]
+    cu = wl.cu_seqlens()
+    for s_ in range(wl.num_seqs):
+        if wl.seqlens[s_] > int(wl.budgets()[layer]):
+            np.testing.assert_array_equal(pl[:, cu[s_]:cu[s_ + 1]], fp[:, cu[s_]:cu[s_ + 1]])
+    with pytest.raises(ckv.CkvError, match="aligned"):
+        ckv.ckv_select_compact(cfg, layer, batch, scores.view(-1)[1:], k, v, idx, cu_keep_dev,
+                               k_out, v_out, ws_select)
 
 
 def test_strided_kv_layout():
