@@ -21,6 +21,9 @@ __all__ = [
     "ckv_status_string",
     "ckv_abi_version", "ckv_score_window_static", "POOL_MAX", "POOL_AVG", "POOL_THEN_SUM", "SUM_THEN_POOL",
     "SCOPE_KV_HEAD", "SCOPE_LAYER", "ckv_layer_error_scores", "ckv_allocate_budgets",
+    "SCORE_AUTO", "SCORE_RESIDENT", "SCORE_RELOAD", "ckv_score_window_lse",
+    "ckv_compress_layer_lse", "ckv_semantic_retrieval_scores", "ckv_set_wait_limit_us",
+    "new_workspace", "new_outputs",
 ]
 
 POOL_MAX, POOL_AVG = 0, 1
