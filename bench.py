@@ -41,7 +41,7 @@ HBM_FALLBACK_GBS = 6800.0
 # null until it is captured again.  Figures that ncu printed in MB are rounded to 10 kB.
 SCORE_SOURCES = ('score_kernel.cu', 'score_resident.cu', 'score_lse.cu', 'score_common.cuh', 'ckv_device.cuh')
 SCORE_TRAFFIC = {
-    "7342ede02588be85a088ff789a14e1dd86c0b927d5aa47aa56ddda71f6d6a90d": {
+    "50ca48de509577f3973443051d675ffae0d66af5da371b0bba5e4bf4ff8adf7d": {
         "llama8b_l8192": 16989952, "paper_llama8b_l8192": 8500000, "needle_l131072": 299342080,
         "llama8b_l8192+lse": 16950000, "needle_l131072+lse": 274310000,
     },

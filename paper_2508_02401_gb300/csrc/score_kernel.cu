@@ -20,13 +20,16 @@
 //                window rows of a head batch, K = 128) into four pass-1 TMEM accumulators;
 //   warp 2       issues the pass-2 tcgen05.mma into four pass-2 accumulators (two issuing
 //                threads, so that neither pass's issue waits behind the other's);
-//   warp 3       publisher: once an item's pass-1 partials are stored, one release on the
-//                unit's arrival counter;
+//   warp 3       publisher and combiner: once an item's pass-1 partials are stored, one
+//                release on the unit's arrival counter; then a bounded acquire spin until every
+//                item of the unit has arrived and (for a unit of at most kWarpCombineMax items)
+//                the combine of their partials into the unit's lse, left in shared memory for
+//                pass 2 while pass 2 still works on the item before;
 //   warps 4-11   pass 1, one warpgroup per 32 columns: each thread owns one key (one TMEM
 //                lane) and keeps a running (max, sum of 2^(x - max)) per column; at the end of
 //                the item the warpgroup's per-column partial goes to global memory;
-//   warps 12-15  pass 2, one warpgroup over all N columns: once every item of the unit has
-//                arrived (a bounded acquire spin) it combines the partials into lse and sums
+//   warps 12-15  pass 2, one warpgroup over all N columns: takes the unit's lse from warp 3
+//                (combining it itself, 128 threads, for a unit of more items) and sums
 //                2^(x - lse) over each head's rows per key.
 // Only the last tiles of a sequence (the window's own keys, the padding past its end) need a
 // per-column mask; the others take an unmasked path of packed fp32 pair instructions.
