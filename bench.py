@@ -417,6 +417,7 @@ def run_ours(args):
                                           f"overlapped on {nstreams} streams, {cap} CTAs per call",
                 "achieved": round(score_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
                 "frac": round(score_gbs / hbm_peak, 4), "peak_kind": peak_kind,
+                "frac_of_8TBs": round(score_gbs / 8000.0, 4),
                 "traffic": traffic, "algorithmic_bytes_per_launch": int(k_bytes),
                 "avg_launch_us": round(score_ms * 1e3, 2)}
     keep_bytes = sum(4 * 256 * Hkv * d["t_keep"] for d in layers) / nl
