@@ -131,6 +131,26 @@ def test_argument_errors(lib):
     assert "workspace" in ckv.load().ckv_last_error_message().decode() or True
 
 
+def _call_select(lib, cfg, batch, scores=_P, k=_P, v=_P, ws=_P, ws_bytes=1 << 30, cu_keep=_P):
+    return lib.ckv_select_compact(cfg.ref, 0, batch.ref, scores, k, v, 0, 0, _P, cu_keep, _P, _P,
+                                  None, ws, ws_bytes, None)
+
+
+def test_select_compact_argument_errors(lib):
+    """ckv_select_compact validates like ckv_compress_layer, plus its scores pointer (NULL or
+    not 16-byte aligned); every check returns before a launch."""
+    cfg, b = _cfg(), FakeBatch([0, 4096, 5000])
+    assert _call_select(lib, cfg, b, scores=None) == 1
+    assert b"scores" in lib.ckv_last_error_message()
+    assert _call_select(lib, cfg, b, scores=_P + 4) == 1
+    assert b"aligned" in lib.ckv_last_error_message()
+    assert _call_select(lib, cfg, b, k=_P + 8) == 1
+    assert _call_select(lib, cfg, b, ws=None) == 3
+    assert _call_select(lib, cfg, b, ws_bytes=1024) == 3
+    assert _call_select(lib, cfg, b, cu_keep=None) == 1
+    assert _call_select(lib, cfg, FakeBatch([0, 4096, 4000])) == 1
+
+
 def test_python_errors_carry_the_message(lib):
     cfg = _cfg(window=0)
     with pytest.raises(ckv.CkvError, match="window"):
