@@ -8,9 +8,11 @@ or budget allocation); it only decides *what data* the method is run on.
 Random numbers come from a counter-based generator: output ``i`` of stream ``key`` is the
 SplitMix64 finaliser (Steele, Lea & Flood, "Fast splittable pseudorandom number generators",
 OOPSLA 2014) applied to ``key + (i + 1) * 0x9E3779B97F4A7C15`` (mod 2**64).  Normals use the
-Box-Muller transform on two 32-bit uniforms per 64-bit draw.  Every tensor of every layer has
-its own stream, so any layer (or any subset of layers) is generated on its own, in any order,
-with the same bits.
+Box-Muller transform on the two 32-bit halves of each 64-bit draw, in double precision, rounded
+to float32.  Every tensor of every layer has its own stream, so any layer (or any subset of
+layers) is generated on its own, in any order, with the same bits.  The bulk draws run in a
+small C library (``synth.c``, built with gcc on first use, OpenMP over the draws); the stream
+itself is also written out in numpy (``uniform_u64``), and the two agree bit for bit.
 
 Recipe per tensor (generate fp32 -> outlier channels -> planted keys -> round to bf16 once):
   * Q window rows, K, V ~ N(0, 1).
@@ -30,13 +32,16 @@ Recipe per tensor (generate fp32 -> outlier channels -> planted keys -> round to
 from __future__ import annotations
 
 from dataclasses import dataclass, field, replace
+import ctypes
 import math
+import os
+import subprocess
 
 import numpy as np
 
 __all__ = [
     "Workload", "LayerInputs", "WORKLOADS", "WORKLOAD_ORDER", "workload",
-    "bf16_bits", "bf16_to_f32", "normals", "uniform_u64",
+    "bf16_bits", "bf16_to_f32", "normals", "normals_bf16", "uniform_u64", "build",
 ]
 
 _GOLDEN = 0x9E3779B97F4A7C15
@@ -70,43 +75,57 @@ def uniform_u64(key: int, start: int, count: int) -> np.ndarray:
     return z
 
 
-def _normals_into(out: np.ndarray, key: int, p0: int, n: int) -> None:
-    z = uniform_u64(key, p0, n)
-    inv32 = np.float32(1.0 / 4294967296.0)
-    u1 = ((z >> np.uint64(32)).astype(np.float32) + np.float32(0.5)) * inv32
-    u2 = ((z & np.uint64(0xFFFFFFFF)).astype(np.float32) + np.float32(0.5)) * inv32
-    rad = np.sqrt(np.float32(-2.0) * np.log(u1))
-    ang = np.float32(2.0 * math.pi) * u2
-    o = out[2 * p0: 2 * (p0 + n)]
-    o[0::2] = (rad * np.cos(ang))[: (len(o) + 1) // 2]
-    o[1::2] = (rad * np.sin(ang))[: len(o) // 2]
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "synth.c")
+_LIB_PATH = os.path.join(_HERE, "libckv_synth.so")
+_lib = None
 
 
-def normals(key: int, count: int, chunk: int = 1 << 20) -> np.ndarray:
-    """``count`` standard normals (float32) from stream ``key`` (Box-Muller, 2 per draw).
+def build(force: bool = False) -> str:
+    """Compiles the bulk-draw library (gcc, C11, OpenMP, no FMA contraction) next to this file."""
+    if force or not os.path.exists(_LIB_PATH) or os.path.getmtime(_LIB_PATH) < os.path.getmtime(_SRC):
+        tmp = _LIB_PATH + f".{os.getpid()}.tmp"
+        subprocess.check_call(["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fopenmp",
+                               "-ffp-contract=off", "-o", tmp, _SRC, "-lm"])
+        os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
 
-    The transform runs in float32 (the values are rounded to bfloat16 afterwards); chunks are
-    independent slices of the stream and are filled by a thread pool.
-    """
-    out = np.empty(count, dtype=np.float32)
-    pairs = (count + 1) // 2
-    starts = list(range(0, pairs, chunk))
-    if len(starts) <= 1:
-        for p0 in starts:
-            _normals_into(out, key, p0, min(chunk, pairs - p0))
-        return out
-    from concurrent.futures import ThreadPoolExecutor
-    with ThreadPoolExecutor(max_workers=min(len(starts), _threads())) as ex:
-        list(ex.map(lambda p0: _normals_into(out, key, p0, min(chunk, pairs - p0)), starts))
+
+def _load():
+    global _lib
+    if _lib is None:
+        build()
+        lib = ctypes.CDLL(_LIB_PATH)
+        P, I64, U64 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_uint64
+        lib.synth_u64.argtypes = [U64, I64, I64, P]
+        lib.synth_normals_f32.argtypes = [U64, I64, P]
+        lib.synth_normals_bf16.argtypes = [U64, I64, P, I64, P]
+        _lib = lib
+    return _lib
+
+
+def uniform_u64_fast(key: int, start: int, count: int) -> np.ndarray:
+    """The same draws as ``uniform_u64``, from the C library."""
+    out = np.empty(count, dtype=np.uint64)
+    _load().synth_u64(key & _M64, start, count, out.ctypes.data_as(ctypes.c_void_p))
     return out
 
 
-def _threads() -> int:
-    import os
-    try:
-        return max(1, len(os.sched_getaffinity(0)))
-    except AttributeError:  # pragma: no cover
-        return max(1, os.cpu_count() or 1)
+def normals(key: int, count: int) -> np.ndarray:
+    """``count`` standard normals (float32) from stream ``key`` (Box-Muller, 2 per draw)."""
+    out = np.empty(count, dtype=np.float32)
+    _load().synth_normals_f32(key & _M64, count, out.ctypes.data_as(ctypes.c_void_p))
+    return out
+
+
+def normals_bf16(key: int, count: int, scale: np.ndarray | None = None) -> np.ndarray:
+    """The first ``count`` normals of stream ``key``, element i multiplied in float32 by
+    ``scale.flat[i % scale.size]`` (when given), rounded to bfloat16; returns the uint16 bits."""
+    out = np.empty(count, dtype=np.uint16)
+    sc = None if scale is None else np.ascontiguousarray(scale, dtype=np.float32).ravel()
+    _load().synth_normals_bf16(key & _M64, count, None if sc is None else sc.ctypes.data_as(ctypes.c_void_p),
+                               0 if sc is None else sc.size, out.ctypes.data_as(ctypes.c_void_p))
+    return out
 
 
 def _randint(key: int, start: int, count: int, lo: int, hi: int) -> np.ndarray:
@@ -243,19 +262,21 @@ class Workload:
         S, w, Hq, Hkv, d = self.num_seqs, self.window, self.num_q_heads, self.num_kv_heads, self.head_dim
         T, G = self.total_tokens, self.group_size
         cu = self.cu_seqlens()
-        q32 = normals(_stream_key(self.seed, _K_Q, l), S * w * Hq * d).reshape(S, w, Hq, d)
-        q_bits = bf16_bits(q32)
-        k32 = normals(_stream_key(self.seed, _K_K, l), T * Hkv * d).reshape(T, Hkv, d)
+        q_bits = normals_bf16(_stream_key(self.seed, _K_Q, l), S * w * Hq * d).reshape(S, w, Hq, d)
+        scale = None
         if self.outlier_channels:
+            scale = np.ones((Hkv, d), dtype=np.float32)
             for g in range(Hkv):
                 key = _stream_key(self.seed, _K_OUTLIER, l, g)
                 ch = np.argsort(uniform_u64(key, 0, d), kind="stable")[: self.outlier_channels]
-                k32[:, g, ch] *= np.float32(self.outlier_scale)
-        planted = self._plant(l, q_bits, k32, cu)
-        v32 = normals(_stream_key(self.seed, _K_V, l), T * Hkv * d).reshape(T, Hkv, d)
-        return LayerInputs(q_win=q_bits, k=bf16_bits(k32), v=bf16_bits(v32), planted=planted)
+                scale[g, ch] = np.float32(self.outlier_scale)
+        k_bits = normals_bf16(_stream_key(self.seed, _K_K, l), T * Hkv * d, scale).reshape(T, Hkv, d)
+        planted = self._plant(l, q_bits, k_bits, cu)
+        v_bits = normals_bf16(_stream_key(self.seed, _K_V, l), T * Hkv * d).reshape(T, Hkv, d)
+        return LayerInputs(q_win=q_bits, k=k_bits, v=v_bits, planted=planted)
 
-    def _plant(self, l, q_bits, k32, cu) -> np.ndarray:
+    def _plant(self, l, q_bits, k_bits, cu) -> np.ndarray:
+        """Overwrites the planted keys' rows of ``k_bits`` (bf16 bits) in place."""
         S, w, d, G = self.num_seqs, self.window, self.head_dim, self.group_size
         if self.plant == "none" or self.plant_count == 0:
             return np.zeros((S, 0), dtype=np.int64)
@@ -290,7 +311,7 @@ class Workload:
                 if self.plant_noise:
                     rows += normals(_stream_key(self.seed, _K_PLANT_NOISE, l, s * 4096 + g),
                                     n * d).reshape(n, d)
-                k32[cu[s] + pos, g, :] = rows.astype(np.float32)
+                k_bits[cu[s] + pos, g, :] = bf16_bits(rows.astype(np.float32))
         return out
 
 

@@ -90,3 +90,17 @@ def test_span_plant_is_contiguous():
     li = wl.layer(1)
     span = li.planted[0]
     assert np.all(np.diff(span) == 1) and len(span) == 64 and span[-1] < 4096 - 32
+
+
+def test_bulk_draws_equal_the_numpy_stream():
+    """The C library's draws are the numpy definition of the stream, bit for bit."""
+    for key, start, n in ((7, 0, 1000), (2**63 + 12345, 999, 4097), (0, 10**9, 64)):
+        np.testing.assert_array_equal(cs.uniform_u64_fast(key, start, n), cs.uniform_u64(key, start, n))
+
+
+def test_bf16_normals_are_the_rounded_float32_normals():
+    scale = np.array([1.0, 10.0, 0.5], np.float32)
+    n = cs.normals(77, 3001)
+    np.testing.assert_array_equal(cs.normals_bf16(77, 3001), cs.bf16_bits(n))
+    np.testing.assert_array_equal(cs.normals_bf16(77, 3001, scale),
+                                  cs.bf16_bits(n * np.resize(scale, 3001)))
