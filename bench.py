@@ -2,14 +2,14 @@
 """Benchmark of the CompressKV prefill KV-compression step on GB300.
 
 One step = ckv_compress_layer (score + pool + top-k + gather) for every layer of the
-Llama-3.1-8B-shaped workload (32 layers, 32 query / 8 KV heads, d = 128, one sequence of 8192
-prefix tokens, w = 32, 2 selected heads per group, max-pool 7, layer budgets summing to
-32 x 256), on synthetic seeded inputs already resident in HBM.  Each layer has its own K/V/Q
-buffers, so one step streams 1.07 GB (far more than the 129 MB L2); the step is replayed from a
-CUDA graph.
+needle-style long-prefix workload (Llama-3.1-8B-shaped: 32 layers, 32 query / 8 KV heads,
+d = 128, one sequence of 131072 prefix tokens with a planted 64-token span, w = 32, 2 selected
+heads per group, max-pool 7, 128 tokens kept per KV head), on synthetic seeded inputs already
+resident in HBM.  Each layer has its own K/V/Q buffers, so one step streams far more than the
+129 MB L2; the step is replayed from a CUDA graph.  `--workload` picks another workload.
 
 Prints one JSON line (rank 0).  `--impl reference` times the fp64 CPU oracle instead (the
-reference arm of this build), on bounded samples of the same workload.
+reference arm of this build) on whole layers of the same workload.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 """
@@ -30,15 +30,13 @@ sys.path.insert(0, ROOT)
 
 METRIC = "KV-compress prefix tokens/s per layer (score+topk+gather); % of HBM peak"
 UNIT = "prefix tokens/s per layer"
-WORKLOAD = "llama8b_l8192"
+WORKLOAD = "needle_l131072"
 HBM_FALLBACK_GBS = 6800.0
 
 # DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) of one scoring launch (one layer)
-# per workload, from the ncu captures summarised in profiles/ (score_kernel_llama8b_l8192.md,
-# score_kernel_needle_l131072.md, score_resident_paper_llama8b_l8192.md,
-# score_lse_llama8b_l8192.md; "+lse": bench.py --lse),
-# keyed by the sha256 of the scoring kernels' sources (SCORE_SOURCES); a changed kernel reports
-# null until it is captured again.  Figures that ncu printed in MB are rounded to 10 kB.
+# per workload, from the ncu summaries under profiles/ ("+lse": bench.py --lse), keyed by the
+# sha256 of the scoring kernels' sources (SCORE_SOURCES); a changed kernel reports null until
+# it is captured again.  Figures that ncu printed in MB are rounded to 10 kB.
 SCORE_SOURCES = ('score_kernel.cu', 'score_resident.cu', 'score_lse.cu', 'score_common.cuh', 'ckv_device.cuh')
 SCORE_TRAFFIC = {
     "50ca48de509577f3973443051d675ffae0d66af5da371b0bba5e4bf4ff8adf7d": {
@@ -81,12 +79,15 @@ def _window_lse(q, k, cu_seqlens, w, Hq, Hkv):
 def _args():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--workload", default=WORKLOAD)
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--min-seconds", type=float, default=1.0,
+                    help="the K-step timed region is repeated until this much GPU time has been "
+                         "timed (at least 3 times); the median repetition is reported")
     ap.add_argument("--layers", type=int, default=0, help="use only the first N layers (0 = all)")
     ap.add_argument("--breakdown", action="store_true", help="per-stage times on stderr")
     ap.add_argument("--score-path", choices=("auto", "resident", "reload"), default="auto",
@@ -148,6 +149,20 @@ def _max_over_ranks(ms, world, device):
 def _job_throughput(world, units_per_rank, ms_per_step):
     """Whole-job units per second: every rank processes its own units in the slowest rank's time."""
     return world * units_per_rank / (ms_per_step / 1e3)
+
+
+def _workload_config(wl, world):
+    """The workload both arms run, as the `config` of their JSON lines."""
+    d = wl.head_dim
+    per_layer = (wl.num_seqs * wl.window * wl.num_q_heads * d + 2 * wl.total_tokens * wl.num_kv_heads * d) * 2
+    step_gb = per_layer * wl.num_layers / 1e9
+    return {"workload": wl.name, "layers": wl.num_layers, "seq_len": wl.total_tokens,
+            "seqs": wl.num_seqs, "q_heads": wl.num_q_heads, "kv_heads": wl.num_kv_heads,
+            "head_dim": d, "window": wl.window, "heads_per_group": wl.heads_per_group,
+            "heads_per_layer": wl.heads_per_layer, "scope": wl.scope,
+            "pool": f"{wl.pool_type}{wl.pool_kernel}", "head_order": wl.head_order,
+            "budget_total": int(wl.budgets().sum()), "parallelism": f"replicas{world}",
+            "l2": f"inputs larger than L2 (distinct per-layer buffers, {step_gb:.2f} GB per step)"}
 
 
 # ----------------------------------------------------------------------------- clocks
@@ -326,18 +341,26 @@ def run_ours(args):
     def barrier():
         _rank_barrier(world)
 
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    # The timed region: exactly `steps` graph replays between a barrier and a synchronize on
+    # both sides, repeated until at least `min_seconds` of GPU time (and 3 repetitions) so
+    # that the clock sampler sees the GPU under load; the median repetition is reported.
+    reps_ms = []
     with ClockSampler(local) as clk:
-        barrier()
-        torch.cuda.synchronize()
-        with torch.cuda.stream(stream):
-            e0.record(stream)
-            for _ in range(args.steps):
-                graph.replay()
-            e1.record(stream)
-        torch.cuda.synchronize()
-        barrier()
-    ms = _max_over_ranks(e0.elapsed_time(e1), world, "cuda")
+        while len(reps_ms) < 3 or sum(reps_ms) < 1e3 * args.min_seconds:
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            barrier()
+            torch.cuda.synchronize()
+            with torch.cuda.stream(stream):
+                e0.record(stream)
+                for _ in range(args.steps):
+                    graph.replay()
+                e1.record(stream)
+            torch.cuda.synchronize()
+            barrier()
+            reps_ms.append(_max_over_ranks(e0.elapsed_time(e1), world, "cuda"))
+            if len(reps_ms) >= 1000:
+                break
+    ms = statistics.median(reps_ms)
     clocks = clk.summary()
     for w in wss + (sel_wss if args.split_select else []):
         code, detail = ckv.ckv_read_device_status(w, stream=stream)
@@ -345,6 +368,24 @@ def run_ours(args):
             raise RuntimeError(f"device status {code} ({detail}) after the timed region")
     ms_per_step = ms / args.steps
     value = _job_throughput(world, nl * T, ms_per_step)
+
+    # --- the same step issued eagerly (no graph): the host's wall time per call (argument
+    # checks, planning, tensor-map encoding and the launches, through the Python binding) and
+    # the GPU time of a step issued that way.
+    eager_reps = 3
+    host_s = []
+    ea, eb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        ea.record(stream)
+        for _ in range(eager_reps):
+            t_issue = time.perf_counter()
+            step()
+            host_s.append(time.perf_counter() - t_issue)
+        eb.record(stream)
+    torch.cuda.synchronize()
+    eager = {"host_us_per_call": round(statistics.median(host_s) / nl * 1e6, 2),
+             "gpu_ms_per_step": round(ea.elapsed_time(eb) / eager_reps, 5)}
 
     # per layer: the scoring kernel, then the selection (pool, top-k, compaction and gather)
     lens = list(wl.seqlens)
@@ -481,8 +522,12 @@ def run_ours(args):
             b.record(stream)
         torch.cuda.synchronize()
         e2e_ms = a.elapsed_time(b) / args.e2e_steps
+        h2d_peak = _h2d_peak(torch, stream)
+        h2d_gbs = h2d / (e2e_ms / 1e3) / 1e9
         e2e = {"value": world * nl * T / (e2e_ms / 1e3), "unit": UNIT, "ms_per_step": round(e2e_ms, 4),
-               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+               "h2d_gbs": round(h2d_gbs, 1), "h2d_peak_gbs": round(h2d_peak, 1),
+               "frac_of_h2d_peak": round(h2d_gbs / h2d_peak, 4)}
 
     cpu = None
     if rank == 0 and world == 1 and args.cpu_seconds > 0:
@@ -494,17 +539,19 @@ def run_ours(args):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 5),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic",
-            "config": {"workload": wl.name, "layers": nl, "seq_len": T, "q_heads": wl.num_q_heads,
-                       "kv_heads": Hkv, "head_dim": 128, "window": wl.window,
-                       "heads_per_group": wl.heads_per_group, "pool": f"{wl.pool_type}{wl.pool_kernel}",
-                       "budget_total": int(wl.budgets().sum()), "parallelism": f"replicas{world}",
-                       "l2": "inputs larger than L2 (distinct per-layer buffers, 1.07 GB per step)",
-                       "graph": "one CUDA graph per step",
-                       "streams": f"layers round-robin on {nstreams} streams, scoring capped at {cap} CTAs per call",
-                       "lse": ("window-row lse given (PyTorch logsumexp outside the timed region; "
-                               "one pass over K)") if args.lse else "computed (two passes)",
-                       "calls": ("ckv_score_window + ckv_select_compact, the selection on a stream "
-                                 "of its own") if args.split_select else "ckv_compress_layer"},
+            "config": _workload_config(wl, world),
+            "run": {"graph": "one CUDA graph per step",
+                    "streams": f"layers round-robin on {nstreams} streams, scoring capped at {cap} CTAs per call",
+                    "lse": ("window-row lse given (PyTorch logsumexp outside the timed region; "
+                            "one pass over K)") if args.lse else "computed (two passes)",
+                    "calls": ("ckv_score_window + ckv_select_compact, the selection on a stream "
+                              "of its own") if args.split_select else "ckv_compress_layer",
+                    "repetitions": len(reps_ms),
+                    "ms_per_step_spread": {"min": round(min(reps_ms) / args.steps, 5),
+                                           "median": round(ms_per_step, 5),
+                                           "max": round(max(reps_ms) / args.steps, 5)},
+                    "timed_gpu_s": round(sum(reps_ms) / 1e3, 3),
+                    "eager": eager},
             "roofline": roofline,
             "layer_roofline": {"bound": "hbm", "achieved": round(layer_gbs, 1), "peak": hbm_peak,
                                "unit": "GB/s", "frac": round(layer_gbs / hbm_peak, 4),
@@ -519,12 +566,35 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+def _h2d_peak(torch, stream, nbytes=1 << 30, reps=5):
+    """A plain host-to-device copy of one pinned 1 GiB buffer: the best of `reps`, in GB/s."""
+    h = torch.empty(nbytes, dtype=torch.uint8, pin_memory=True)
+    d = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    best = float("inf")
+    with torch.cuda.stream(stream):
+        for _ in range(reps):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            d.copy_(h, non_blocking=True)
+            b.record(stream)
+            torch.cuda.synchronize()
+            best = min(best, a.elapsed_time(b))
+    del h, d
+    return nbytes / (best / 1e3) / 1e9
+
+
 # ----------------------------------------------------------------------------- the oracle
+def _oracle_cores(wl, threads):
+    """Threads that the oracle keeps busy: it runs OpenMP over (sequence, selection) units."""
+    units = wl.num_seqs * (1 if wl.scope == "layer" else wl.num_kv_heads)
+    return min(threads, units)
+
+
 def _cpu_baseline(wl, host_layers, seconds):
     """The fp64 oracle as it stands, whole layers in order until `seconds` have passed."""
     import oracle
     oracle.build()
-    cores = oracle.threads(0)
+    cores = _oracle_cores(wl, oracle.threads(0))
     t0 = time.perf_counter()
     done = 0
     while True:  # sweeps of the layers, in order, until `seconds` have passed
@@ -533,18 +603,21 @@ def _cpu_baseline(wl, host_layers, seconds):
         oracle.compress_layer(li.q_win, li.k, li.v, wl.cu_seqlens(), wl.head_mask()[l],
                               int(wl.budgets()[l]), wl.window, wl.pool_kernel,
                               0 if wl.pool_type == "max" else 1,
-                              0 if wl.head_order == "pool_then_sum" else 1)
+                              0 if wl.head_order == "pool_then_sum" else 1,
+                              scope=1 if wl.scope == "layer" else 0)
         done += 1
         if time.perf_counter() - t0 >= seconds:
             break
     dt = time.perf_counter() - t0
     return {"value": round(done * wl.total_tokens / dt, 2), "unit": UNIT, "cores": cores,
-            "kind": "oracle", "sample": f"{done} layer calls (sweeps over the {len(host_layers)} "
-                                        f"layers), whole layers, {dt:.1f} s, OpenMP over "
-                                        "(sequence, KV head)"}
+            "kind": "oracle", "sample": f"{done} whole-layer calls (layers in order), {dt:.1f} s, "
+                                        f"OpenMP over (sequence, KV head) units on "
+                                        f"{oracle.threads(0)} host threads"}
 
 
 def run_reference(args):
+    """The reference arm: the fp64 oracle as it stands, on all host cores, one whole layer of the
+    workload per step (cycling over its first four layers), as the GPU line's cpu_baseline."""
     rank, world, local = _dist()
     if rank != 0:
         return
@@ -552,38 +625,39 @@ def run_reference(args):
     import oracle
     oracle.build()
     wl = cs.workload(args.workload)
-    cores = oracle.threads(0)
-    li_cache = {}
+    if args.layers:
+        wl = wl.with_(num_layers=args.layers)
+    cores = _oracle_cores(wl, oracle.threads(0))
+    masks, budgets, cu = wl.head_mask(), wl.budgets(), wl.cu_seqlens()
+    cache = {}
+    n_distinct = min(wl.num_layers, 4)
 
     def sample(i):
-        l = i % wl.num_layers
-        if l not in li_cache:
-            li_cache.clear()
-            li_cache[l] = wl.layer(l)
-        li = li_cache[l]
-        g = (i // wl.num_layers) % wl.num_kv_heads
-        oracle.compress_layer(li.q_win, li.k, li.v, wl.cu_seqlens(), wl.head_mask()[l],
-                              int(wl.budgets()[l]), wl.window, wl.pool_kernel,
-                              0 if wl.pool_type == "max" else 1,
-                              0 if wl.head_order == "pool_then_sum" else 1, groups=[g])
+        l = i % n_distinct
+        if l not in cache:
+            cache[l] = wl.layer(l)
+        li = cache[l]
+        t = time.perf_counter()
+        oracle.compress_layer(li.q_win, li.k, li.v, cu, masks[l], int(budgets[l]), wl.window,
+                              wl.pool_kernel, 0 if wl.pool_type == "max" else 1,
+                              0 if wl.head_order == "pool_then_sum" else 1,
+                              scope=1 if wl.scope == "layer" else 0)
+        return time.perf_counter() - t
 
     for i in range(args.warmup):
         sample(i)
-    times = []
-    for i in range(args.steps):
-        t = time.perf_counter()
-        sample(args.warmup + i)
-        times.append(time.perf_counter() - t)
-    per_unit = statistics.mean(times)
-    value = wl.total_tokens / (per_unit * wl.num_kv_heads)  # a layer = H_kv (seq, head) units
+    times = [sample(args.warmup + i) for i in range(args.steps)]
+    per_layer = statistics.mean(times)
+    value = wl.total_tokens / per_layer
     line = {"impl": "reference", "metric": METRIC, "value": round(value, 2), "unit": UNIT,
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
-            "ms_per_step": round(per_unit * 1e3, 3), "higher_is_better": True, "scaling": "weak",
+            "ms_per_step": round(per_layer * 1e3, 3), "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": wl.name, "layers": wl.num_layers, "seq_len": wl.total_tokens,
-                       "parallelism": "host cores"},
+            "config": _workload_config(wl, world),
             "cpu_baseline": {"value": round(value, 2), "unit": UNIT, "cores": cores, "kind": "oracle",
-                             "sample": "one (layer, KV head) unit of the workload per step"},
+                             "sample": f"one whole layer per step (layers 0..{n_distinct - 1} in turn), "
+                                       f"OpenMP over (sequence, KV head) units on "
+                                       f"{oracle.threads(0)} host threads"},
             "e2e": {"value": round(value, 2), "unit": UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)

@@ -1065,7 +1065,10 @@ ckv_status ckv_score_window_static(const ckv_config* cfg, int32_t layer, const c
     if (dev < 0 || dev >= kMaxDevices) return fail(CKV_ERR_UNSUPPORTED, "device index %d", dev);
     int ctas = device_sm_count();
     if (ctas <= 0) return cuda_fail(cudaGetLastError(), "querying the SM count");
+    if (pl.max_ctas > 0) ctas = std::min(ctas, pl.max_ctas);  // the CTAs enqueue_score plans for
     {
+        // The same plan as the launch below makes: its work items, over all of its launches,
+        // must fit the array (each launch's items are also bounded by the array's size).
         static thread_local ScoreLaunch probe;
         if ((st = plan_score(pl, batch, -1, std::min(ctas, CKV_STATIC_SCRATCH_ITEMS), probe,
                              CKV_STATIC_SCRATCH_ITEMS)))

@@ -10,6 +10,9 @@ Tolerances (the GPU accumulates in fp32, the oracle in fp64):
     are within 1e-3 of each other, otherwise every token clearly above / below the threshold
     band must be in / out;
   * gathered K/V: bit-exact against the input rows at the GPU's indices.
+
+Every output buffer of `run_gpu` sits between canary bytes that are checked after the calls:
+a kernel that writes past an output's end (or before its start) fails the test.
 """
 from __future__ import annotations
 
@@ -31,28 +34,66 @@ def to_host(t: torch.Tensor) -> np.ndarray:
     return t.view(torch.int16).cpu().numpy().view(np.uint16)
 
 
+GUARD_BYTES = 4096          # canary bytes before and after every output buffer
+GUARD_BYTE = 0xA5
+
+
+class Guarded:
+    """A device buffer with canary bytes on both sides: `view` is what the library writes;
+    `check()` asserts that nothing was written outside it (compute-sanitizer stands in)."""
+
+    def __init__(self, shape, dtype, fill=None):
+        n = int(np.prod(shape)) * torch.empty((), dtype=dtype).element_size()
+        self.raw = torch.full((GUARD_BYTES + n + GUARD_BYTES,), GUARD_BYTE, dtype=torch.uint8,
+                              device="cuda")
+        self.view = self.raw[GUARD_BYTES:GUARD_BYTES + n].view(dtype).view(shape)
+        if fill is not None:
+            self.view.fill_(fill)
+        self.what = f"{tuple(shape)} {dtype}"
+
+    def check(self):
+        head = self.raw[:GUARD_BYTES].cpu().numpy()
+        tail = self.raw[-GUARD_BYTES:].cpu().numpy()
+        assert np.all(head == GUARD_BYTE) and np.all(tail == GUARD_BYTE), \
+            f"a kernel wrote outside the output buffer {self.what}"
+
+
+def guarded_outputs(cfg, layer, batch):
+    """(idx, cu_keep_dev, k_out, v_out) as canary-guarded buffers, and the host cu_keep."""
+    cu_keep, _ = ckv.ckv_keep_lengths(cfg, layer, batch)
+    tk = int(cu_keep[-1])
+    H = cfg.num_kv_heads
+    return (Guarded((H, tk), torch.int32, -7), Guarded((batch.num_seqs + 1,), torch.int32, -7),
+            Guarded((tk, H, 128), torch.bfloat16), Guarded((tk, H, 128), torch.bfloat16), cu_keep)
+
+
 def run_gpu(wl, layer, li, cfg=None, scores=True, stream=None, check_status=True):
-    """compress_layer (+ score_window when asked) for one layer; numpy outputs."""
+    """compress_layer (+ score_window when asked) for one layer; numpy outputs.  Every output
+    buffer carries canaries on both sides, checked after the calls."""
     cfg = cfg or ckv.Config.from_workload(wl)
     batch = ckv.Batch(wl.cu_seqlens())
     q, k, v = to_dev(li.q_win), to_dev(li.k), to_dev(li.v)
     ws = ckv.new_workspace(cfg, layer, batch)
-    idx, cu_keep_dev, k_out, v_out, cu_keep = ckv.new_outputs(cfg, layer, batch)
+    gidx, gck, gk, gv, cu_keep = guarded_outputs(cfg, layer, batch)
     T = batch.total_tokens
-    pooled = torch.full((cfg.num_vectors, T), float("nan"), dtype=torch.float32, device="cuda")
-    ckv.ckv_compress_layer(cfg, layer, batch, q, k, v, idx, cu_keep_dev, k_out, v_out, ws,
-                           pooled_out=pooled, stream=stream)
+    gpooled = Guarded((cfg.num_vectors, T), torch.float32, float("nan"))
+    ckv.ckv_compress_layer(cfg, layer, batch, q, k, v, gidx.view, gck.view, gk.view, gv.view, ws,
+                           pooled_out=gpooled.view, stream=stream)
+    guards = [gidx, gck, gk, gv, gpooled]
     out = dict(cfg=cfg, cu_keep=cu_keep)
     if scores:
         _, n_sel = ckv.ckv_keep_lengths(cfg, layer, batch)
-        sc = torch.full((n_sel, T), float("nan"), dtype=torch.float32, device="cuda")
-        ckv.ckv_score_window(cfg, layer, batch, q, k, sc, ws, stream=stream)
-        out["scores"] = sc.cpu().numpy()
+        gsc = Guarded((n_sel, T), torch.float32, float("nan"))
+        ckv.ckv_score_window(cfg, layer, batch, q, k, gsc.view, ws, stream=stream)
+        guards.append(gsc)
+        out["scores"] = gsc.view.cpu().numpy()
     code, detail = ckv.ckv_read_device_status(ws, stream=stream)
     if check_status:
         assert code == 0, f"device status {code} ({detail})"
-    out.update(status=(code, detail), pooled=pooled.cpu().numpy(), idx=idx.cpu().numpy(),
-               cu_keep_dev=cu_keep_dev.cpu().numpy(), k_out=to_host(k_out), v_out=to_host(v_out))
+    for g in guards:
+        g.check()
+    out.update(status=(code, detail), pooled=gpooled.view.cpu().numpy(), idx=gidx.view.cpu().numpy(),
+               cu_keep_dev=gck.view.cpu().numpy(), k_out=to_host(gk.view), v_out=to_host(gv.view))
     return out
 
 

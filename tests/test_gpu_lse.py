@@ -84,14 +84,19 @@ def test_scores_and_layer_with_given_lse(case, max_ctas):
     T = batch.total_tokens
     _, n_sel = ckv.ckv_keep_lengths(cfg, 0, batch)
     ws = ckv.new_workspace(cfg, 0, batch)
-    sc = torch.full((n_sel, T), float("nan"), dtype=torch.float32, device="cuda")
+    gsc = gu.Guarded((n_sel, T), torch.float32, float("nan"))
+    sc = gsc.view
     ckv.ckv_score_window_lse(cfg, 0, batch, q, k, lse32, sc, ws, lse_head_stride=lse64.shape[1])
-    idx, cu_keep_dev, k_out, v_out, cu_keep = ckv.new_outputs(cfg, 0, batch)
-    pooled = torch.full((cfg.num_vectors, T), float("nan"), dtype=torch.float32, device="cuda")
+    *gouts, cu_keep = gu.guarded_outputs(cfg, 0, batch)
+    idx, cu_keep_dev, k_out, v_out = (g_.view for g_ in gouts)
+    gpl = gu.Guarded((cfg.num_vectors, T), torch.float32, float("nan"))
+    pooled = gpl.view
     ckv.ckv_compress_layer_lse(cfg, 0, batch, q, k, v, lse32, idx, cu_keep_dev, k_out, v_out, ws,
                                lse_head_stride=lse64.shape[1], pooled_out=pooled)
     code, detail = ckv.ckv_read_device_status(ws)
     assert code == 0, (code, detail)
+    for g_ in [gsc, gpl, *gouts]:
+        g_.check()
     g = dict(cfg=cfg, cu_keep=cu_keep, scores=sc.cpu().numpy(), pooled=pooled.cpu().numpy(),
              idx=idx.cpu().numpy(), cu_keep_dev=cu_keep_dev.cpu().numpy(),
              k_out=gu.to_host(k_out), v_out=gu.to_host(v_out))
@@ -109,10 +114,12 @@ def test_given_lse_agrees_with_the_computing_path():
     q, k = gu.to_dev(li.q_win), gu.to_dev(li.k)
     lse32 = torch.from_numpy(_oracle_lse(wl, li).astype(np.float32)).cuda()
     _, n_sel = ckv.ckv_keep_lengths(cfg, 0, batch)
-    sc = torch.full((n_sel, batch.total_tokens), float("nan"), dtype=torch.float32, device="cuda")
+    gsc = gu.Guarded((n_sel, batch.total_tokens), torch.float32, float("nan"))
+    sc = gsc.view
     ws = ckv.new_workspace(cfg, 0, batch)
     ckv.ckv_score_window_lse(cfg, 0, batch, q, k, lse32, sc, ws)
     assert ckv.ckv_read_device_status(ws) == (0, 0)
+    gsc.check()
     gu.assert_close_rows(sc.cpu().numpy(), g1["scores"], rtol=2e-3)
 
 

@@ -61,6 +61,10 @@ FUZZ = [
          budget_mean=300, head_order="sum_then_pool"),
     dict(scope="layer", heads_per_layer=6, num_q_heads=32, num_kv_heads=8, window=64,
          seqlens=(1500, 9000), budget_mean=100),
+    # pool kernels wider than the candidate range, L = w, L = w + 1, empty sequences
+    dict(window=8, pool_kernel=9, seqlens=(12, 13, 9, 0, 17, 300, 8), budget_mean=10),
+    dict(window=4, pool_kernel=63, heads_per_group=1, seqlens=(40, 70, 5, 0, 200), budget_mean=12,
+         pool_type="avg"),
 ]
 
 
@@ -165,17 +169,17 @@ def test_standalone_entry_points_match_the_fused_call():
     ws = ckv.new_workspace(cfg, layer, batch)
     cu_keep, n_sel = ckv.ckv_keep_lengths(cfg, layer, batch)
     T, tk = batch.total_tokens, int(cu_keep[-1])
-    scores = torch.empty((n_sel, T), dtype=torch.float32, device="cuda")
-    pooled = torch.empty((8, T), dtype=torch.float32, device="cuda")
-    idx = torch.empty((8, tk), dtype=torch.int32, device="cuda")
-    cu_keep_dev = torch.empty(4, dtype=torch.int32, device="cuda")
-    k_out = torch.empty((tk, 8, 128), dtype=torch.bfloat16, device="cuda")
-    v_out = torch.empty_like(k_out)
+    guards = [gu.Guarded((n_sel, T), torch.float32), gu.Guarded((8, T), torch.float32),
+              gu.Guarded((8, tk), torch.int32), gu.Guarded((4,), torch.int32),
+              gu.Guarded((tk, 8, 128), torch.bfloat16), gu.Guarded((tk, 8, 128), torch.bfloat16)]
+    scores, pooled, idx, cu_keep_dev, k_out, v_out = (g_.view for g_ in guards)
     ckv.ckv_score_window(cfg, layer, batch, q, k, scores, ws)
     ckv.ckv_pool(cfg, layer, batch, scores, pooled)
     ckv.ckv_select_topk(cfg, layer, batch, pooled, idx, cu_keep_dev, ws)
     ckv.ckv_gather_compact(cfg, batch, tk, k, v, idx, cu_keep_dev, k_out, v_out, ws)
     assert ckv.ckv_read_device_status(ws) == (0, 0)
+    for g_ in guards:
+        g_.check()
     fused = gu.run_gpu(wl, layer, li)
     np.testing.assert_array_equal(scores.cpu().numpy(), fused["scores"])
     np.testing.assert_array_equal(idx.cpu().numpy(), fused["idx"])
@@ -208,9 +212,11 @@ def test_split_score_and_select_match_the_fused_call():
     ws_score, ws_select = ckv.new_workspace(cfg, layer, batch), ckv.new_workspace(cfg, layer, batch)
     _, n_sel = ckv.ckv_keep_lengths(cfg, layer, batch)
     T = batch.total_tokens
-    scores = torch.empty((n_sel, T), dtype=torch.float32, device="cuda")
-    pooled = torch.full((cfg.num_vectors, T), float("nan"), dtype=torch.float32, device="cuda")
-    idx, cu_keep_dev, k_out, v_out, cu_keep = ckv.new_outputs(cfg, layer, batch)
+    gsc = gu.Guarded((n_sel, T), torch.float32)
+    gpl = gu.Guarded((cfg.num_vectors, T), torch.float32, float("nan"))
+    *gouts, cu_keep = gu.guarded_outputs(cfg, layer, batch)
+    scores, pooled = gsc.view, gpl.view
+    idx, cu_keep_dev, k_out, v_out = (g_.view for g_ in gouts)
     s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
     ckv.ckv_score_window(cfg, layer, batch, q, k, scores, ws_score, stream=s1)
     ev = torch.cuda.Event()
@@ -221,6 +227,8 @@ def test_split_score_and_select_match_the_fused_call():
     torch.cuda.synchronize()
     assert ckv.ckv_read_device_status(ws_score) == (0, 0)
     assert ckv.ckv_read_device_status(ws_select) == (0, 0)
+    for g_ in [gsc, gpl, *gouts]:
+        g_.check()
     fused = gu.run_gpu(wl, layer, li)
     np.testing.assert_array_equal(idx.cpu().numpy(), fused["idx"])
     np.testing.assert_array_equal(cu_keep_dev.cpu().numpy(), fused["cu_keep_dev"])
@@ -248,10 +256,13 @@ def test_strided_kv_layout():
     kv = torch.stack([gu.to_dev(li.k), gu.to_dev(li.v)], dim=1).contiguous()  # [T, 2, 8, 128]
     k_view, v_view = kv[:, 0], kv[:, 1]
     ws = ckv.new_workspace(cfg, layer, batch)
-    idx, cu_keep_dev, k_out, v_out, _ = ckv.new_outputs(cfg, layer, batch)
+    *gouts, _ = gu.guarded_outputs(cfg, layer, batch)
+    idx, cu_keep_dev, k_out, v_out = (g_.view for g_ in gouts)
     ckv.ckv_compress_layer(cfg, layer, batch, gu.to_dev(li.q_win), k_view, v_view, idx, cu_keep_dev,
                            k_out, v_out, ws, tok_stride=2 * 8 * 128, head_stride=128)
     assert ckv.ckv_read_device_status(ws) == (0, 0)
+    for g_ in gouts:
+        g_.check()
     np.testing.assert_array_equal(idx.cpu().numpy(), ref["idx"])
     np.testing.assert_array_equal(gu.to_host(k_out), ref["k_out"])
     np.testing.assert_array_equal(gu.to_host(v_out), ref["v_out"])
@@ -266,11 +277,14 @@ def test_device_lengths_that_disagree_are_reported():
     batch = ckv.Batch(wl.cu_seqlens(),
                       cu_seqlens_dev=torch.tensor([0, 1500, 3000], dtype=torch.int32, device="cuda"))
     ws = ckv.new_workspace(cfg, 0, batch)
-    idx, cu_keep_dev, k_out, v_out, _ = ckv.new_outputs(cfg, 0, batch)
+    *gouts, _ = gu.guarded_outputs(cfg, 0, batch)
+    idx, cu_keep_dev, k_out, v_out = (g_.view for g_ in gouts)
     ckv.ckv_compress_layer(cfg, 0, batch, gu.to_dev(li.q_win), gu.to_dev(li.k), gu.to_dev(li.v),
                            idx, cu_keep_dev, k_out, v_out, ws)
     code, _ = ckv.ckv_read_device_status(ws)
     assert code == 1
+    for g_ in gouts:
+        g_.check()
     assert ckv.ckv_read_device_status(ws) == (0, 0)  # the read reset it
 
 

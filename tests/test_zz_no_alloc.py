@@ -26,12 +26,8 @@ def _lib():
     ckv.load()
 
 
-def test_static_scratch_matches_workspace_entry_point_twice():
-    wl = cs.Workload(name="noalloc", num_layers=1, num_q_heads=32, num_kv_heads=8,
-                     seqlens=(6000, 1300, 45), window=32, heads_per_group=2, budget_mean=128,
-                     budget_uniform=True, outlier_channels=8, seed=3)
+def _static_against_workspace(wl, cfg):
     li = wl.layer(0)
-    cfg = ckv.Config.from_workload(wl)
     batch = ckv.Batch(wl.cu_seqlens())
     q, k = gu.to_dev(li.q_win), gu.to_dev(li.k)
     _, n_sel = ckv.ckv_keep_lengths(cfg, 0, batch)
@@ -45,14 +41,34 @@ def test_static_scratch_matches_workspace_entry_point_twice():
     lib = ckv.load()
     stream = torch.cuda.current_stream().cuda_stream
     for _ in range(2):
-        out = torch.full((n_sel, T), float("nan"), dtype=torch.float32, device="cuda")
+        gout = gu.Guarded((n_sel, T), torch.float32, float("nan"))
+        out = gout.view
         status = torch.full((2,), -1, dtype=torch.int32, device="cuda")
         rc = lib.ckv_score_window_static(cfg.ref, 0, batch.ref, q.data_ptr(), k.data_ptr(), 0, 0,
                                          out.data_ptr(), status.data_ptr(), C.c_void_p(stream))
         assert rc == 0, lib.ckv_last_error_message()
         torch.cuda.synchronize()
         assert status.tolist() == [0, 0]
+        gout.check()
         gu.assert_close_rows(out.cpu().numpy(), ref)
+
+
+@pytest.mark.parametrize("path,max_ctas", [("auto", 0), ("reload", 3), ("resident", 0)])
+def test_static_scratch_matches_workspace_entry_point_twice(path, max_ctas):
+    wl = cs.Workload(name="noalloc", num_layers=1, num_q_heads=32, num_kv_heads=8,
+                     seqlens=(6000, 1300, 45), window=32, heads_per_group=2, budget_mean=128,
+                     budget_uniform=True, outlier_channels=8, seed=3)
+    sp = {"auto": ckv.SCORE_AUTO, "reload": ckv.SCORE_RELOAD, "resident": ckv.SCORE_RESIDENT}[path]
+    _static_against_workspace(wl, ckv.Config.from_workload(wl, score_path=sp, max_ctas=max_ctas))
+
+
+def test_static_scratch_over_several_launches():
+    # 400 short sequences, one KV head: 400 units of one item each, more units than one launch's
+    # unit table holds (384), so the call is split into two launches that reuse the array.
+    wl = cs.Workload(name="noalloc_many", num_layers=1, num_q_heads=2, num_kv_heads=1,
+                     seqlens=tuple(100 + (i * 37) % 90 for i in range(400)), window=16,
+                     heads_per_group=1, budget_mean=48, budget_uniform=True, seed=9)
+    _static_against_workspace(wl, ckv.Config.from_workload(wl))
 
 
 def test_static_scratch_rejects_work_beyond_its_size():
