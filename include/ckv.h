@@ -53,7 +53,7 @@
 extern "C" {
 #endif
 
-#define CKV_ABI_VERSION 4
+#define CKV_ABI_VERSION 5
 
 #if defined(__GNUC__)
 #define CKV_API __attribute__((visibility("default")))
@@ -217,6 +217,46 @@ CKV_API ckv_status ckv_select_compact(const ckv_config* cfg, int32_t layer, cons
                                       float* pooled_out, void* workspace, size_t workspace_bytes,
                                       ckv_stream stream);
 
+/* One layer of a multi-layer call (ckv_score_windows, ckv_compress_layers).  The layers of a
+ * call share the config and the batch; each brings its own buffers. */
+typedef struct ckv_layer_io {
+    int32_t layer;                 /* index into the config's head_mask and budgets */
+    const void* q_win;             /* [S, w, H_q, 128] */
+    const void* k;                 /* [T, H_kv, 128] with the strides below */
+    const void* v;                 /* ckv_compress_layers only; the same strides as k */
+    int64_t tok_stride;            /* of k and v, in elements; 0 = packed */
+    int64_t head_stride;
+    float* scores;                 /* ckv_score_windows: [n_sel, T] out, as ckv_score_window */
+    int32_t* idx;                  /* ckv_compress_layers: outputs as for ckv_compress_layer */
+    int32_t* cu_keep_dev;
+    void* k_out;
+    void* v_out;
+    float* pooled_out;             /* may be NULL */
+} ckv_layer_io;
+
+/* Workspace bytes for a multi-layer call over io[0..n_layers) (enough for either entry point). */
+CKV_API ckv_status ckv_workspace_size_layers(const ckv_config* cfg, int32_t n_layers,
+                                             const ckv_layer_io* io, const ckv_batch* batch,
+                                             size_t* bytes);
+
+/* Step 1 for several layers at once: for each io[i], what ckv_score_window(cfg, io[i].layer,
+ * ...) writes to io[i].scores.  Every layer's two passes run in one persistent launch (one per
+ * 32 layers, and per 512 sequences), so the GPU streams one layer's keys while it exchanges
+ * another's row statistics; the per-call start and tail are paid once.  Always the two-pass
+ * kernel that re-reads K in pass 2 (cfg->score_path is ignored).  cfg->max_ctas caps the CTAs
+ * of the launch (0 = all SMs), which leaves the other SMs to work issued on other streams. */
+CKV_API ckv_status ckv_score_windows(const ckv_config* cfg, int32_t n_layers,
+                                     const ckv_layer_io* io, const ckv_batch* batch,
+                                     void* workspace, size_t workspace_bytes, ckv_stream stream);
+
+/* Steps 1-4 for several layers: for each io[i], what ckv_compress_layer(cfg, io[i].layer, ...)
+ * writes.  The layers are scored as by ckv_score_windows (into the workspace), then each
+ * layer's selection runs in order on the same stream.  Sequences with L_s at most every
+ * layer's budget are copied whole without being scored. */
+CKV_API ckv_status ckv_compress_layers(const ckv_config* cfg, int32_t n_layers,
+                                       const ckv_layer_io* io, const ckv_batch* batch,
+                                       void* workspace, size_t workspace_bytes, ckv_stream stream);
+
 /* Steps 1-4 for one layer.  Sequences with L_s <= B_l are copied whole without being scored.
  * pooled_out may be NULL (then the pooled scores stay in the workspace). */
 CKV_API ckv_status ckv_compress_layer(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
@@ -289,7 +329,9 @@ CKV_API ckv_status ckv_set_wait_limit_us(uint32_t microseconds);
 
 /* Synchronises `stream`, then returns the workspace's device status: *code = 0 if no kernel
  * recorded an error since the last reset, else the first error (1 = cu_seqlens_dev disagrees
- * with the host copy, 2 = a wait timed out, 3 = an index out of range); *detail says where.
+ * with the host copy, 2 = a wait timed out, 3 = an index out of range, 4 = a window row's
+ * largest logit beyond +-700, which the two-pass kernel's fp64 row sums cannot hold); *detail
+ * says where.
  * With reset != 0 the status word is cleared afterwards. */
 CKV_API ckv_status ckv_read_device_status(void* workspace, ckv_stream stream, int32_t reset,
                                   int32_t* code, int32_t* detail);
@@ -297,16 +339,19 @@ CKV_API ckv_status ckv_read_device_status(void* workspace, ckv_stream stream, in
 /* ckv_score_window for callers that cannot allocate device memory (no counterpart in the
  * paper).  Some callers have no allocator to hand: code running inside a host-side engine
  * whose memory pool is owned elsewhere, or code that must not grow the process's device
- * footprint after start-up.  This variant takes no workspace.  Its scratch (the per-chunk
- * softmax partials, per-unit arrival counters and a status word) is a fixed, file-scope
- * device array of
- * CKV_STATIC_SCRATCH_BYTES that every GPU loading the library holds until the process exits.
+ * footprint after start-up.  This variant takes no workspace.  Its scratch (the softmax
+ * exchange of the scoring kernel -- per-item partials of the TMEM-resident kernel, or per-unit
+ * sums of the two-pass kernel -- arrival counters and a status word) is a fixed, file-scope
+ * device array of CKV_STATIC_SCRATCH_BYTES that every GPU loading the library holds until the
+ * process exits.
  *   - Same arguments, results and layouts as ckv_score_window, minus the workspace.
  *   - The first call on a device looks up the array's device address (once per device, with
  *     that device current); make that first call before any stream capture.
- *   - Calls whose work needs more scratch than the array holds (more than
- *     CKV_STATIC_SCRATCH_ITEMS work items) return CKV_ERR_UNSUPPORTED before enqueuing
- *     anything; ckv_score_window has no such limit.
+ *   - Calls whose work needs more scratch than the array holds return CKV_ERR_UNSUPPORTED
+ *     before enqueuing anything: on the resident kernel more than CKV_STATIC_SCRATCH_ITEMS
+ *     work items over the call; on the two-pass kernel more than CKV_STATIC_SCRATCH_UNITS
+ *     (head batch, sequence) units in one launch, which takes up to 512 sequences.
+ *     ckv_score_window has no such limit.
  *   - Every call shares the one array: calls that may overlap on the GPU (other streams,
  *     other host threads) race and must be serialised by the caller.
  *   - Each call clears the status word first.  If status_out (device, 2 x int32) is not NULL,
@@ -314,7 +359,8 @@ CKV_API ckv_status ckv_read_device_status(void* workspace, ckv_stream stream, in
  *     the end of the call, in stream order.
  *   - Allocates nothing: no cudaMalloc, cudaFree or allocating library call. */
 #define CKV_STATIC_SCRATCH_ITEMS 1024
-#define CKV_STATIC_SCRATCH_BYTES (256 + CKV_STATIC_SCRATCH_ITEMS * 64 * 8 + 2048)
+#define CKV_STATIC_SCRATCH_UNITS 1024
+#define CKV_STATIC_SCRATCH_BYTES (256 + CKV_STATIC_SCRATCH_ITEMS * 64 * 8 + 4096)
 CKV_API ckv_status ckv_score_window_static(const ckv_config* cfg, int32_t layer,
                                            const ckv_batch* batch, const void* q_win,
                                            const void* k, int64_t tok_stride,

@@ -23,7 +23,8 @@ __all__ = [
     "SCOPE_KV_HEAD", "SCOPE_LAYER", "ckv_layer_error_scores", "ckv_allocate_budgets",
     "SCORE_AUTO", "SCORE_RESIDENT", "SCORE_RELOAD", "ckv_score_window_lse",
     "ckv_compress_layer_lse", "ckv_semantic_retrieval_scores", "ckv_set_wait_limit_us",
-    "new_workspace", "new_outputs",
+    "new_workspace", "new_outputs", "LayerIO", "ckv_workspace_size_layers", "ckv_score_windows",
+    "ckv_compress_layers", "new_layers_workspace",
 ]
 
 POOL_MAX, POOL_AVG = 0, 1
@@ -55,6 +56,13 @@ class _Config(C.Structure):
                 ("softmax_scale", C.c_float),
                 ("max_ctas", C.c_int32), ("score_path", C.c_int32), ("head_mask", C.c_void_p),
                 ("budgets", C.c_void_p)]
+
+
+class _LayerIO(C.Structure):
+    _fields_ = [("layer", C.c_int32), ("q_win", C.c_void_p), ("k", C.c_void_p), ("v", C.c_void_p),
+                ("tok_stride", C.c_int64), ("head_stride", C.c_int64), ("scores", C.c_void_p),
+                ("idx", C.c_void_p), ("cu_keep_dev", C.c_void_p), ("k_out", C.c_void_p),
+                ("v_out", C.c_void_p), ("pooled_out", C.c_void_p)]
 
 
 class _Batch(C.Structure):
@@ -96,6 +104,9 @@ def load():
         "ckv_layer_error_scores": ([P, I32, I32, P], C.c_int),
         "ckv_set_wait_limit_us": ([C.c_uint32], C.c_int),
         "ckv_allocate_budgets": ([P, I32, I64, I32, I32, P], C.c_int),
+        "ckv_workspace_size_layers": ([cfg, I32, P, bat, C.POINTER(SZ)], C.c_int),
+        "ckv_score_windows": ([cfg, I32, P, bat, P, SZ, P], C.c_int),
+        "ckv_compress_layers": ([cfg, I32, P, bat, P, SZ, P], C.c_int),
     }
     for name, (args, res) in sigs.items():
         fn = getattr(lib, name)
@@ -329,6 +340,63 @@ def ckv_score_window_static(cfg, layer, batch, q_win, k, scores, status_out=None
     _check(load().ckv_score_window_static(cfg.ref, layer, batch.ref, _ptr(q_win), _ptr(k),
                                           tok_stride, head_stride, _ptr(scores), _ptr(status_out),
                                           _stream(stream)), "ckv_score_window_static")
+
+
+@dataclass
+class LayerIO:
+    """One layer of a multi-layer call (ckv_layer_io): the layer index and its tensors."""
+    layer: int
+    q_win: object
+    k: object
+    v: object = None
+    scores: object = None       # ckv_score_windows
+    idx: object = None          # ckv_compress_layers
+    cu_keep_dev: object = None
+    k_out: object = None
+    v_out: object = None
+    pooled_out: object = None
+    tok_stride: int = 0
+    head_stride: int = 0
+
+
+def _layer_ios(ios):
+    arr = (_LayerIO * len(ios))()
+    for i, x in enumerate(ios):
+        arr[i] = _LayerIO(x.layer, *(None if t is None else t.data_ptr() for t in (x.q_win, x.k, x.v)),
+                          x.tok_stride, x.head_stride,
+                          *(None if t is None else t.data_ptr()
+                            for t in (x.scores, x.idx, x.cu_keep_dev, x.k_out, x.v_out, x.pooled_out)))
+    return arr
+
+
+def ckv_workspace_size_layers(cfg, ios, batch) -> int:
+    n = C.c_size_t(0)
+    arr = _layer_ios(ios)
+    _check(load().ckv_workspace_size_layers(cfg.ref, len(ios), arr, batch.ref, C.byref(n)),
+           "ckv_workspace_size_layers")
+    return n.value
+
+
+def new_layers_workspace(cfg, ios, batch, device="cuda"):
+    """A zeroed workspace of ckv_workspace_size_layers bytes (uint8 tensor)."""
+    import torch
+    return torch.zeros(ckv_workspace_size_layers(cfg, ios, batch), dtype=torch.uint8, device=device)
+
+
+def ckv_score_windows(cfg, ios, batch, workspace, stream=None):
+    """ckv_score_window for every LayerIO of `ios` (their `scores`), in one persistent launch."""
+    arr = _layer_ios(ios)
+    _check(load().ckv_score_windows(cfg.ref, len(ios), arr, batch.ref, _ptr(workspace),
+                                    workspace.numel() * workspace.element_size(), _stream(stream)),
+           "ckv_score_windows")
+
+
+def ckv_compress_layers(cfg, ios, batch, workspace, stream=None):
+    """ckv_compress_layer for every LayerIO of `ios`: one scoring launch, then the selections."""
+    arr = _layer_ios(ios)
+    _check(load().ckv_compress_layers(cfg.ref, len(ios), arr, batch.ref, _ptr(workspace),
+                                      workspace.numel() * workspace.element_size(), _stream(stream)),
+           "ckv_compress_layers")
 
 
 def ckv_read_device_status(workspace, stream=None, reset=True):

@@ -157,19 +157,14 @@ int64_t keep_total(const ckv_batch* b, int budget) {
     return t;
 }
 
-// Splits every (sequence, head batch) unit's key tiles into items of at most `c` tiles and
-// packs units whole into rounds of at most `ctas` items; `c` minimises an estimate of the
-// launch's time in tile loads per CTA.
-//
-// Resident kernel (items of at most 512 / n_cols tiles, so that an item's logits fit in
-// TMEM): while an item waits for its unit's exchange and runs pass 2, the next item's MMAs can
-// fill the accumulators it leaves free and the ring can hold kRing more tiles; a round costs
-// its item length plus whatever of the exchange those do not cover.
-// Reload kernel: pass 1 of a round streams while the previous round exchanges its statistics
-// and runs pass 2, so a round costs its item length, or the exchange plus pass 2 of the round
-// before when that is longer; the last round adds its own exchange and pass 2.  Items longer
-// than kL2Tiles are charged their excess again: their pass-2 re-reads fall out of the CTA's
-// share of L2.
+// Work of the TMEM-resident scoring kernel (score_resident.cu): splits every (sequence, head
+// batch) unit's key tiles into items of at most `c` tiles (c <= 512 / n_cols, so that an
+// item's logits fit in TMEM) and packs units whole into rounds of at most `ctas` items; `c`
+// minimises an estimate of the launch's time in tile loads per CTA.  While an item waits for
+// its unit's exchange and runs pass 2, the next item's MMAs can fill the accumulators it
+// leaves free and the ring can hold `ring` more tiles; a round costs its item length plus
+// whatever of the exchange those do not cover.  CKV_ERR_UNSUPPORTED if a unit does not fit
+// one round.
 ckv_status plan_score(const Plan& pl, const ckv_batch* b, int skip_le, int ctas, ScoreLaunch& L,
                       int max_items_per_launch) {
     struct RawUnit {
@@ -188,33 +183,18 @@ ckv_status plan_score(const Plan& pl, const ckv_batch* b, int skip_le, int ctas,
     L.items.clear();
     L.units.clear();
     L.slices.clear();
+    L.resident = true;
     if (raw.empty()) return CKV_OK;
     if (b->num_seqs > 65535) return fail(CKV_ERR_UNSUPPORTED, "more than 65535 sequences");
-    constexpr int kL2Tiles = 8;        // pass 1 runs up to two items ahead, so each CTA keeps
-                                       // ~2 items in L2 (evict-last hint) until pass 2 reads
-                                       // them: 2 x 8 tiles x 32 KiB x 152 CTAs ~ 80 MB
-    constexpr double kExchange = 4.0;  // publish, exchange and combine, in tile-load times
-                                       // (combined ahead of pass 2, so mostly hidden)
-    constexpr double kPass2 = 1.0;     // pass 2 per tile from L2, relative to a pass-1 load:
-                                       // measured about as fast (each pass has its own issuer
-                                       // and ring, and both share the SM's copy bandwidth)
-    // The resident kernel when every unit fits one round of items that fit in TMEM.
     const int c_res = 512 / pl.n_cols;
-    const bool fits = static_cast<long long>(max_tiles) <= static_cast<long long>(c_res) * ctas;
-    if (pl.score_path == CKV_SCORE_RESIDENT && !fits)
+    if (static_cast<long long>(max_tiles) > static_cast<long long>(c_res) * ctas)
         return fail(CKV_ERR_UNSUPPORTED,
                     "resident scoring: a sequence of %d key tiles needs items of at most %d tiles "
                     "on at least %d CTAs (%d available)", max_tiles, c_res,
                     (max_tiles + c_res - 1) / c_res, ctas);
-    // Automatic choice: the resident kernel at N = 32, where TMEM holds two items of up to 8
-    // tiles, so the next item's MMAs proceed while this one waits for its unit's exchange; at
-    // N = 64 one 8-tile item fills TMEM and every exchange stalls the CTA, while the reload
-    // kernel runs pass 1 two items ahead through L2 (measured faster there).
-    L.resident = fits && (pl.score_path == CKV_SCORE_RESIDENT ||
-                          (pl.score_path == CKV_SCORE_AUTO && pl.n_cols == 32));
     constexpr double kResExchange = 8.0;  // publish, exchange, combine and pass 2 from TMEM
     const int ring = pl.n_cols == 64 ? 5 : 6;
-    const int c_hi = L.resident ? std::min(max_tiles, c_res) : max_tiles;
+    const int c_hi = std::min(max_tiles, c_res);
     int best_c = -1;
     double best_cost = 0;
     for (int c = 1; c <= c_hi; ++c) {
@@ -235,15 +215,8 @@ ckv_status plan_score(const Plan& pl, const ckv_batch* b, int skip_le, int ctas,
         }
         if (!feasible) continue;
         rounds += cur > 0;
-        double cost;
-        if (L.resident) {
-            const double per_round = c + std::max(0.0, kResExchange - (c_res - c) - ring);
-            cost = rounds * per_round + kResExchange;
-        } else {
-            const double per_round = std::max(static_cast<double>(c), kPass2 * c + kExchange) +
-                                     std::max(0, c - kL2Tiles);
-            cost = rounds * per_round + kPass2 * c + kExchange;
-        }
+        const double per_round = c + std::max(0.0, kResExchange - (c_res - c) - ring);
+        const double cost = rounds * per_round + kResExchange;
         if (best_c < 0 || cost < best_cost) {
             best_c = c;
             best_cost = cost;
@@ -400,7 +373,8 @@ ckv_status plan_score_stream(const Plan& pl, const ckv_batch* b, int skip_le, in
 }
 
 struct WsLayout {
-    size_t header = 0, partials = 0, counters = 0, scores = 0, pooled = 0, srs_lse = 0;
+    size_t header = 0, partials = 0, counters = 0, sums = 0, unit_counters = 0, scores = 0,
+           pooled = 0, srs_lse = 0;
     size_t hist = 0, arrivals = 0, chunk_start = 0, buckets = 0, info = 0, chunk_off = 0, total = 0;
     int max_chunks = 0;
 };
@@ -421,6 +395,13 @@ WsLayout ws_layout(const Plan& pl, const ckv_batch* b, int T) {
     off = round_up(off + static_cast<size_t>(kMaxScoreItems) * kMaxCols * sizeof(float2), kWsAlign);
     l.counters = off;
     off = round_up(off + kMaxScoreUnits * sizeof(int), kWsAlign);
+    // the two-pass kernel's exchange: per (head batch, sequence) unit, an fp64 sum per column
+    // and an arrival counter
+    const size_t score_units = static_cast<size_t>(pl.nb) * b->num_seqs;
+    l.sums = off;
+    off = round_up(off + score_units * kMaxCols * sizeof(double), kWsAlign);
+    l.unit_counters = off;
+    off = round_up(off + score_units * sizeof(int), kWsAlign);
     l.scores = off;
     off = round_up(off + static_cast<size_t>(pl.n_sel) * T * sizeof(float), kWsAlign);
     l.pooled = off;
@@ -538,6 +519,138 @@ int device_sm_count() {
 
 namespace {
 
+// ---------------------------------------------------------------- two-pass scoring (reload)
+// One layer of a scoring call on the two-pass kernel of score_layers.cu.
+struct LayerJob {
+    const Plan* pl;
+    const void* q_win;
+    const void* k;
+    int64_t tok, head;
+    float* scores;
+};
+
+constexpr int kMinItemTiles = 4;  // shortest work item, in key tiles
+
+// Enqueues the two-pass scoring of `jobs` (layers sharing the batch and the window): one
+// persistent launch per group of consecutive layers and per chunk of up to kMaxLaunchSeqs
+// sequences whose tables fit the kernel's parameters.  Sequences of at most skip_le tokens are
+// skipped.  `sums`/`counters` hold the exchange of every (head batch, sequence) unit of one
+// launch (each launch clears them first; launches are ordered on `stream`).
+ckv_status enqueue_layers(const std::vector<LayerJob>& jobs, const ckv_batch* b, int T, void* sums,
+                          int* counters, int* status, int skip_le, int max_ctas, cudaStream_t stream) {
+    if (jobs.empty()) return CKV_OK;
+    int ctas = device_sm_count();
+    if (ctas <= 0) return cuda_fail(cudaGetLastError(), "querying the SM count");
+    if (max_ctas > 0) ctas = std::min(ctas, max_ctas);
+    const int S = b->num_seqs;
+    int max_tiles = 0;
+    for (int s = 0; s < S; ++s) {
+        const int len = b->cu_seqlens_host[s + 1] - b->cu_seqlens_host[s];
+        if (len > skip_le && len > 0) max_tiles = std::max(max_tiles, (len + kTileKeys - 1) / kTileKeys);
+    }
+    if (max_tiles == 0) return CKV_OK;
+    // Items of c tiles, with at most `ctas` items per unit: a unit's items then lie in at most
+    // three consecutive rounds of the launch, which the kernel's two-item lead of pass 1 covers.
+    const int c = std::max(kMinItemTiles, (max_tiles + ctas - 1) / ctas);
+    const int w_pad = jobs[0].pl->w_pad, w = jobs[0].pl->w;
+    static thread_local LayersLaunch L;
+    const uint32_t hash = seqlens_hash(b->cu_seqlens_host, S);
+    size_t j0 = 0;
+    while (j0 < jobs.size()) {
+        // the layers of this launch: as many as the parameter tables hold
+        size_t j1 = j0;
+        int nb = 0, nsel = 0, n_cols = 32;
+        while (j1 < jobs.size() && static_cast<int>(j1 - j0) < kMaxLaunchLayers &&
+               nb + jobs[j1].pl->nb <= kMaxLaunchBatches && nsel + jobs[j1].pl->n_sel <= kMaxLaunchSel) {
+            nb += jobs[j1].pl->nb;
+            nsel += jobs[j1].pl->n_sel;
+            n_cols = std::max(n_cols, jobs[j1].pl->n_cols);
+            ++j1;
+        }
+        if (j1 == j0) return fail(CKV_ERR_UNSUPPORTED, "a layer has more head batches than one launch holds");
+        L.layers.clear();
+        L.batch_layer.clear();
+        L.batch_group.clear();
+        L.batch_first.clear();
+        L.batch_nheads.clear();
+        L.batch_sel.clear();
+        L.sel_heads.clear();
+        for (size_t j = j0; j < j1; ++j) {
+            const LayerJob& J = jobs[j];
+            LayersLayer ly;
+            ckv_status st;
+            if ((st = make_k_map(&ly.tmap_k, J.k, J.pl->Hkv, T, J.tok, J.head))) return st;
+            if ((st = make_q_map(&ly.tmap_q, J.q_win, J.pl->Hq, S, w, w_pad))) return st;
+            ly.scores = J.scores;
+            const int sel_base = static_cast<int>(L.sel_heads.size());
+            for (int bt = 0; bt < J.pl->nb; ++bt) {
+                L.batch_layer.push_back(static_cast<int16_t>(j - j0));
+                L.batch_group.push_back(static_cast<int16_t>(J.pl->batch_group[bt]));
+                L.batch_first.push_back(static_cast<int16_t>(J.pl->batch_first[bt]));
+                L.batch_nheads.push_back(static_cast<int16_t>(J.pl->batch_nheads[bt]));
+                L.batch_sel.push_back(static_cast<int16_t>(sel_base + J.pl->batch_first[bt]));
+            }
+            for (int h : J.pl->sel_heads) L.sel_heads.push_back(static_cast<int16_t>(h));
+            L.layers.push_back(ly);
+        }
+        for (int s0 = 0; s0 < S; s0 += kMaxLaunchSeqs) {  // chunks of sequences
+            const int s1 = std::min(S, s0 + kMaxLaunchSeqs);
+            L.seq_start.clear();
+            L.seq_len.clear();
+            L.seq_item0.assign(1, 0);
+            for (int s = s0; s < s1; ++s) {
+                const int len = b->cu_seqlens_host[s + 1] - b->cu_seqlens_host[s];
+                const int tiles = len > skip_le && len > 0 ? (len + kTileKeys - 1) / kTileKeys : 0;
+                L.seq_start.push_back(b->cu_seqlens_host[s]);
+                L.seq_len.push_back(len);
+                L.seq_item0.push_back(L.seq_item0.back() + (tiles + c - 1) / c);
+            }
+            if (L.seq_item0.back() == 0) continue;
+            if (static_cast<int64_t>(L.seq_item0.back()) * nb > INT32_MAX)
+                return fail(CKV_ERR_UNSUPPORTED, "too many scoring work items");
+            L.seq0 = s0;
+            L.S_all = S;
+            L.cu_seqlens_dev = b->cu_seqlens_dev;
+            L.sums = static_cast<double*>(sums);
+            L.counters = counters;
+            L.status = status;
+            L.T = T;
+            L.w = w;
+            L.w_pad = w_pad;
+            L.n_cols = n_cols;
+            L.c = c;
+            L.grid = ctas;
+            L.cu_hash = hash;
+            L.softmax_scale = jobs[j0].pl->scale;
+            const cudaError_t e = launch_score_layers(L, stream);
+            if (e != cudaSuccess) return cuda_fail(e, "launching the two-pass scoring kernel");
+        }
+        j0 = j1;
+    }
+    return CKV_OK;
+}
+
+// Whether the single-layer scoring runs on the TMEM-resident kernel (score_resident.cu); the
+// two-pass reload kernel otherwise.  CKV_ERR_UNSUPPORTED when the caller asked for the resident
+// kernel and a sequence does not fit it.
+ckv_status resident_choice(const Plan& pl, const ckv_batch* b, int skip_le, int ctas, bool* resident) {
+    int max_tiles = 0;
+    for (int s = 0; s < b->num_seqs; ++s) {
+        const int len = b->cu_seqlens_host[s + 1] - b->cu_seqlens_host[s];
+        if (len > skip_le && len > 0) max_tiles = std::max(max_tiles, (len + kTileKeys - 1) / kTileKeys);
+    }
+    const int c_res = 512 / pl.n_cols;
+    const bool fits = static_cast<long long>(max_tiles) <= static_cast<long long>(c_res) * ctas;
+    if (pl.score_path == CKV_SCORE_RESIDENT && !fits)
+        return fail(CKV_ERR_UNSUPPORTED,
+                    "resident scoring: a sequence of %d key tiles needs items of at most %d tiles "
+                    "on at least %d CTAs (%d available)", max_tiles, c_res,
+                    (max_tiles + c_res - 1) / c_res, ctas);
+    *resident = fits && (pl.score_path == CKV_SCORE_RESIDENT ||
+                         (pl.score_path == CKV_SCORE_AUTO && pl.n_cols == 32));
+    return CKV_OK;
+}
+
 ckv_status enqueue_score(const Plan& pl, const ckv_batch* b, int T, const void* q_win,
                          const void* k, int64_t tok, int64_t head, float* scores, void* ws,
                          const WsLayout& l, int skip_le, cudaStream_t stream,
@@ -546,6 +659,17 @@ ckv_status enqueue_score(const Plan& pl, const ckv_batch* b, int T, const void* 
     int ctas = device_sm_count();
     if (ctas <= 0) return cuda_fail(cudaGetLastError(), "querying the SM count");
     if (pl.max_ctas > 0) ctas = std::min(ctas, pl.max_ctas);
+    if (!lse) {
+        bool resident = false;
+        ckv_status st = resident_choice(pl, b, skip_le, std::min(ctas, max_items_per_launch), &resident);
+        if (st) return st;
+        if (!resident) {  // the two-pass kernel
+            uint8_t* w8 = static_cast<uint8_t*>(ws);
+            const std::vector<LayerJob> jobs{LayerJob{&pl, q_win, k, tok, head, scores}};
+            return enqueue_layers(jobs, b, T, w8 + l.sums, reinterpret_cast<int*>(w8 + l.unit_counters),
+                                  reinterpret_cast<int*>(w8), skip_le, ctas, stream);
+        }
+    }
     static thread_local ScoreLaunch L;  // reused: keeps the plan's vectors allocated
     ckv_status st = lse ? plan_score_stream(pl, b, skip_le, std::min(ctas, max_items_per_launch), L,
                                             max_items_per_launch)
@@ -969,6 +1093,153 @@ ckv_status ckv_compress_layer_lse(const ckv_config* cfg, int32_t layer, const ck
                                workspace, workspace_bytes, stream);
 }
 
+}  // extern "C"
+
+namespace {
+
+// Workspace of a multi-layer call: the header and one layer's selection scratch (the layout of
+// the layer needing the most), the two-pass kernel's exchange for every (head batch, sequence)
+// unit of the call's layers, then each layer's scores (ckv_compress_layers).
+struct LayersWs {
+    WsLayout sel;
+    size_t sums = 0, counters = 0, total = 0;
+    std::vector<size_t> scores;
+};
+
+ckv_status prepare_layers(const ckv_config* cfg, int32_t n_layers, const ckv_layer_io* io,
+                          const ckv_batch* b, std::vector<Plan>& pls, int* T, LayersWs* lw) {
+    ckv_status st;
+    if (n_layers < 1) return fail(CKV_ERR_INVALID_ARG, "n_layers %d < 1", n_layers);
+    if (!io) return fail(CKV_ERR_INVALID_ARG, "io is NULL");
+    if ((st = check_batch(b, T))) return st;
+    pls.assign(n_layers, Plan());
+    size_t units = 0, best = 0;
+    for (int i = 0; i < n_layers; ++i) {
+        if ((st = make_plan(cfg, io[i].layer, pls[i]))) return st;
+        units += static_cast<size_t>(pls[i].nb) * b->num_seqs;
+        const WsLayout l = ws_layout(pls[i], b, *T);
+        if (i == 0 || l.total > best) {
+            best = l.total;
+            lw->sel = l;
+        }
+    }
+    size_t off = round_up(lw->sel.total, kWsAlign);
+    lw->sums = off;
+    off = round_up(off + units * kMaxCols * sizeof(double), kWsAlign);
+    lw->counters = off;
+    off = round_up(off + units * sizeof(int), kWsAlign);
+    lw->scores.assign(n_layers, 0);
+    for (int i = 0; i < n_layers; ++i) {
+        lw->scores[i] = off;
+        off = round_up(off + static_cast<size_t>(pls[i].n_sel) * *T * sizeof(float), kWsAlign);
+    }
+    lw->total = off;
+    return CKV_OK;
+}
+
+ckv_status check_layers_ws(const LayersWs& lw, void* ws, size_t bytes, bool with_scores) {
+    if (!ws) return fail(CKV_ERR_WORKSPACE, "workspace is NULL");
+    if (!aligned(ws, kWsAlign)) return fail(CKV_ERR_WORKSPACE, "workspace not 256-byte aligned");
+    const size_t need = with_scores ? lw.total : lw.scores.empty() ? lw.total : lw.scores[0];
+    if (bytes < need) return fail(CKV_ERR_WORKSPACE, "workspace %zu bytes < required %zu", bytes, need);
+    return CKV_OK;
+}
+
+// The scoring jobs of a multi-layer call; scores in the workspace when `own_scores`.
+ckv_status layer_jobs(const std::vector<Plan>& pls, const ckv_layer_io* io, int T, uint8_t* w8,
+                      const LayersWs& lw, bool own_scores, std::vector<LayerJob>& jobs,
+                      std::vector<int64_t>& tok, std::vector<int64_t>& head) {
+    ckv_status st;
+    const int n = static_cast<int>(pls.size());
+    jobs.clear();
+    tok.assign(n, 0);
+    head.assign(n, 0);
+    for (int i = 0; i < n; ++i) {
+        tok[i] = io[i].tok_stride;
+        head[i] = io[i].head_stride;
+        if ((st = resolve_strides(pls[i], &tok[i], &head[i])) || (st = check_kv(io[i].q_win, "q_win", T)) ||
+            (st = check_kv(io[i].k, "k", T)))
+            return st;
+        if (pls[i].w != pls[0].w) return fail(CKV_ERR_INVALID_ARG, "layers with different windows");
+        float* sc = own_scores ? reinterpret_cast<float*>(w8 + lw.scores[i]) : io[i].scores;
+        if (!own_scores && (st = check_kv(sc, "scores", T))) return st;
+        jobs.push_back(LayerJob{&pls[i], io[i].q_win, io[i].k, tok[i], head[i], sc});
+    }
+    return CKV_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+ckv_status ckv_workspace_size_layers(const ckv_config* cfg, int32_t n_layers, const ckv_layer_io* io,
+                                     const ckv_batch* batch, size_t* bytes) {
+    std::vector<Plan> pls;
+    LayersWs lw;
+    int T = 0;
+    ckv_status st = prepare_layers(cfg, n_layers, io, batch, pls, &T, &lw);
+    if (st) return st;
+    if (!bytes) return fail(CKV_ERR_INVALID_ARG, "bytes is NULL");
+    *bytes = lw.total;
+    return CKV_OK;
+}
+
+ckv_status ckv_score_windows(const ckv_config* cfg, int32_t n_layers, const ckv_layer_io* io,
+                             const ckv_batch* batch, void* workspace, size_t workspace_bytes,
+                             ckv_stream stream) {
+    static thread_local std::vector<Plan> pls;
+    static thread_local std::vector<LayerJob> jobs;
+    static thread_local std::vector<int64_t> tok, head;
+    LayersWs lw;
+    int T = 0;
+    ckv_status st;
+    if ((st = prepare_layers(cfg, n_layers, io, batch, pls, &T, &lw)) ||
+        (st = check_layers_ws(lw, workspace, workspace_bytes, false)))
+        return st;
+    uint8_t* w8 = static_cast<uint8_t*>(workspace);
+    if ((st = layer_jobs(pls, io, T, w8, lw, false, jobs, tok, head))) return st;
+    return enqueue_layers(jobs, batch, T, w8 + lw.sums, reinterpret_cast<int*>(w8 + lw.counters),
+                          reinterpret_cast<int*>(w8), -1, cfg->max_ctas,
+                          reinterpret_cast<cudaStream_t>(stream));
+}
+
+ckv_status ckv_compress_layers(const ckv_config* cfg, int32_t n_layers, const ckv_layer_io* io,
+                               const ckv_batch* batch, void* workspace, size_t workspace_bytes,
+                               ckv_stream stream) {
+    static thread_local std::vector<Plan> pls;
+    static thread_local std::vector<LayerJob> jobs;
+    static thread_local std::vector<int64_t> tok, head;
+    LayersWs lw;
+    int T = 0;
+    ckv_status st;
+    if ((st = prepare_layers(cfg, n_layers, io, batch, pls, &T, &lw)) ||
+        (st = check_layers_ws(lw, workspace, workspace_bytes, true)))
+        return st;
+    uint8_t* w8 = static_cast<uint8_t*>(workspace);
+    if ((st = layer_jobs(pls, io, T, w8, lw, true, jobs, tok, head))) return st;
+    std::vector<int64_t> tks(n_layers, 0);
+    int min_budget = INT_MAX;
+    for (int i = 0; i < n_layers; ++i) {
+        if ((st = check_kv(io[i].v, "v", T)) ||
+            (st = check_select_outputs(batch, pls[i], io[i].idx, io[i].cu_keep_dev, io[i].k_out,
+                                       io[i].v_out, io[i].pooled_out, &tks[i])))
+            return st;
+        min_budget = std::min(min_budget, pls[i].budget);
+    }
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    // sequences that fit every layer's budget are kept whole by every selection
+    if ((st = enqueue_layers(jobs, batch, T, w8 + lw.sums, reinterpret_cast<int*>(w8 + lw.counters),
+                             reinterpret_cast<int*>(w8), min_budget, cfg->max_ctas, s)))
+        return st;
+    WsLayout sel = lw.sel;
+    for (int i = 0; i < n_layers; ++i)
+        if ((st = enqueue_select_fused(pls[i], cfg, batch, T, jobs[i].scores, io[i].k, io[i].v, tok[i],
+                                       head[i], io[i].idx, io[i].cu_keep_dev, io[i].k_out, io[i].v_out,
+                                       io[i].pooled_out, workspace, sel, tks[i], s)))
+            return st;
+    return CKV_OK;
+}
+
 ckv_status ckv_semantic_retrieval_scores(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
                                          const void* q_dec, const void* k, int64_t tok_stride,
                                          int64_t head_stride, const float* lse, int64_t lse_head_stride,
@@ -1066,7 +1337,10 @@ ckv_status ckv_score_window_static(const ckv_config* cfg, int32_t layer, const c
     int ctas = device_sm_count();
     if (ctas <= 0) return cuda_fail(cudaGetLastError(), "querying the SM count");
     if (pl.max_ctas > 0) ctas = std::min(ctas, pl.max_ctas);  // the CTAs enqueue_score plans for
-    {
+    bool resident = false;
+    if ((st = resident_choice(pl, batch, -1, std::min(ctas, CKV_STATIC_SCRATCH_ITEMS), &resident)))
+        return st;
+    if (resident) {
         // The same plan as the launch below makes: its work items, over all of its launches,
         // must fit the array (each launch's items are also bounded by the array's size).
         static thread_local ScoreLaunch probe;
@@ -1078,6 +1352,14 @@ ckv_status ckv_score_window_static(const ckv_config* cfg, int32_t layer, const c
             return fail(CKV_ERR_UNSUPPORTED,
                         "this batch needs %d scratch work items; the static scratch holds %d "
                         "(use ckv_score_window with a workspace)", n_items, CKV_STATIC_SCRATCH_ITEMS);
+    } else {
+        // The two-pass kernel's exchange: one fp64 sum per column and a counter per (head
+        // batch, sequence) unit of a launch (a launch takes up to kMaxLaunchSeqs sequences).
+        const int units = pl.nb * std::min(batch->num_seqs, kMaxLaunchSeqs);
+        if (units > CKV_STATIC_SCRATCH_UNITS)
+            return fail(CKV_ERR_UNSUPPORTED,
+                        "this batch needs %d scratch units; the static scratch holds %d "
+                        "(use ckv_score_window with a workspace)", units, CKV_STATIC_SCRATCH_UNITS);
     }
     // Once per device, with that device current: the device address of the scratch array.
     std::call_once(g_scratch_once[dev], [dev] {
@@ -1091,10 +1373,15 @@ ckv_status ckv_score_window_static(const ckv_config* cfg, int32_t layer, const c
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     e = cudaMemsetAsync(scratch, 0, 2 * sizeof(int32_t), s);  // the status word starts at zero
     if (e != cudaSuccess) return cuda_fail(e, "clearing the static status word");
+    // Layout: the status header, then either kernel's exchange (they never run in one call).
+    static_assert(CKV_STATIC_SCRATCH_ITEMS * kMaxCols * sizeof(float2) ==
+                      CKV_STATIC_SCRATCH_UNITS * kMaxCols * sizeof(double), "scratch regions");
     WsLayout l;
     l.header = 0;
     l.partials = sizeof(WsHeader);
     l.counters = l.partials + static_cast<size_t>(CKV_STATIC_SCRATCH_ITEMS) * kMaxCols * sizeof(float2);
+    l.sums = l.partials;
+    l.unit_counters = l.counters;
     l.total = CKV_STATIC_SCRATCH_BYTES;
     if ((st = enqueue_score(pl, batch, T, q_win, k, tok_stride, head_stride, scores, scratch, l, -1, s,
                             CKV_STATIC_SCRATCH_ITEMS)))

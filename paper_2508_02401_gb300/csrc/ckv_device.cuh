@@ -24,6 +24,7 @@ enum DeviceCode : int {
     kDevBadSeqlens = 1,  // cu_seqlens on the device disagree with the host copy
     kDevTimeout = 2,     // a bounded wait gave up
     kDevBadIndex = 3,    // an index read from device memory was out of range
+    kDevRange = 4,       // a window row's largest logit is beyond the supported range
 };
 
 // Workspace header: status code, detail, then padding to 256 bytes.

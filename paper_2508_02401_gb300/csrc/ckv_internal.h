@@ -62,6 +62,34 @@ struct ScoreLaunch {
     std::vector<ScoreSlice> slices;
 };
 cudaError_t launch_score(const ScoreLaunch& L, cudaStream_t stream);
+
+// Multi-layer scoring (score_layers.cu): both passes, K re-read from L2 in pass 2, every unit
+// of every layer of the launch in one persistent cooperative kernel.
+constexpr int kMaxLaunchLayers = 32;
+constexpr int kMaxLaunchBatches = 512;   // head batches over the launch's layers
+constexpr int kMaxLaunchSel = 1024;      // head slots over the launch's layers
+constexpr int kMaxLaunchSeqs = 512;
+struct LayersLayer {
+    CUtensorMap tmap_k;
+    CUtensorMap tmap_q;
+    float* scores;       // [n_sel of the layer, T]
+};
+struct LayersLaunch {
+    std::vector<LayersLayer> layers;
+    // flat over the layers' head batches, in layer order
+    std::vector<int16_t> batch_layer, batch_group, batch_first, batch_nheads, batch_sel;
+    std::vector<int16_t> sel_heads;  // query head of each head slot, batch after batch
+    std::vector<int32_t> seq_start, seq_len, seq_item0;  // [S], [S], [S+1] of sequences seq0 ...
+    int seq0, S_all;     // the launch's first sequence; sequences in the batch (for the hash)
+    const int32_t* cu_seqlens_dev;
+    double* sums;        // [batches * S][n_cols]
+    int* counters;       // [batches * S]
+    int* status;
+    int T, w, w_pad, n_cols, c, grid;
+    uint32_t cu_hash;
+    float softmax_scale;
+};
+cudaError_t launch_score_layers(const LayersLaunch& L, cudaStream_t stream);
 long long wait_limit_cycles();  // the current limit of a bounded wait, in SM clock cycles
 
 struct SelectLaunch {

@@ -1,40 +1,48 @@
-// Window-attention scoring (arxiv 2508.02401, Sec. 3.3 with the attention of Eq. 2):
+// Window-attention scoring of several layers in one persistent launch (arxiv 2508.02401,
+// Sec. 3.3 with the attention of Eq. 2):
 //
 //   a_h[j] = sum_{r < w, j <= P+r} exp(s_{h,r,j} - lse_{h,r}),   s_{h,r,j} = scale * q_{h,r}.k_j
 //
-// for every selected head h of a KV group, every window row r and every key j of a sequence
-// (P = L - w).  A row's normaliser lse needs every key before any probability can be summed
-// over rows, so each key tile is used twice: once for the row statistics (pass 1), once for
-// the probabilities (pass 2).
+// for every selected head h of every KV group of every layer of the launch, every window row r
+// and every key j of a sequence (P = L - w).  A row's normaliser lse needs every key before any
+// probability can be summed over rows, so each key tile is used twice: once for the row
+// statistics (pass 1, from HBM), once for the probabilities (pass 2, from L2).
 //
-// Work: a unit is (sequence, batch of selected heads of one KV group); its key tiles are cut
-// into items of a few tiles, and the items are dealt out in rounds of gridDim.x (CTA b takes
-// item round * gridDim.x + b; all items of a unit are in one round).  One cooperative
-// launch, one CTA per SM, 512 threads, warp-specialised:
+// Work: a unit is (layer, head batch of one KV group, sequence); its key tiles are cut into
+// items of at most c tiles.  The items of all units, unit after unit, form one sequence that
+// the CTAs take round-robin (CTA b: items b, b + G, b + 2G, ...), so every CTA streams its
+// share of every unit and a unit's items are spread over consecutive CTAs.  The host picks c
+// so that a unit has at most G items: its items then lie in at most three consecutive rounds,
+// and since pass 1 may run up to two items ahead of pass 2 in every CTA, every unit's pass 1
+// completes before any CTA needs that unit's normalisers (no wait can close a cycle).
+//
+// Exchange: at the end of an item, pass 1 adds, per window-row column, its keys' sum
+// sum_j 2^(x_j) (x = logit * log2 e, as s * 2^m with the item's maximum m) in fp64 to the
+// unit's accumulator with one atomic add, and one arrival per pass-1 warpgroup is counted on
+// the unit's counter.  A unit's lse per column is log2 of its accumulator once the counter is
+// complete: one read of N doubles, whatever the number of items.  fp64 holds 2^(+-1022), so
+// a column's largest logit must lie within +-700 (natural log units); beyond that the status
+// word reports kDevRange.
+//
+// One cooperative launch, one CTA per SM, 512 threads, warp-specialised:
 //   warp 0       TMA producer for both passes, one polling thread: per item, TMA loads of the
-//                window query rows (the MMA's B operand) into one of three buffers, then of its
-//                128-key x 128-dim bf16 K tiles (two 128-byte-swizzled boxes of 64 dims) into
-//                the pass-1 ring of kP1Slots slots; the same tiles again into the pass-2 ring
-//                of kP2Slots slots once the item's pass-1 loads are out, so they come from L2;
+//                window query rows into one of kQBufs buffers, then of its 128-key x 128-dim
+//                bf16 K tiles (two 128-byte-swizzled boxes of 64 dims) into the pass-1 ring
+//                (evict-last: pass 2 reads them again soon); the same tiles again into the
+//                pass-2 ring (evict-first) once the item's pass-1 loads are out;
 //   warp 1       allocates TMEM and issues the pass-1 tcgen05.mma (M = 128 keys, N = the
-//                window rows of a head batch, K = 128) into four pass-1 TMEM accumulators;
-//   warp 2       issues the pass-2 tcgen05.mma into four pass-2 accumulators (two issuing
-//                threads, so that neither pass's issue waits behind the other's);
-//   warp 3       publisher and combiner: once an item's pass-1 partials are stored, one
-//                release on the unit's arrival counter; then a bounded acquire spin until every
-//                item of the unit has arrived and (for a unit of at most kWarpCombineMax items)
-//                the combine of their partials into the unit's lse, left in shared memory for
-//                pass 2 while pass 2 still works on the item before;
+//                window rows of a head batch, K = 128) into four pass-1 accumulators;
+//   warp 2       issues the pass-2 tcgen05.mma into four pass-2 accumulators;
+//   warp 3       publisher: once an item's pass-1 sums are added, one release on the unit's
+//                counter; then a bounded acquire spin until the unit is complete and the
+//                unit's -lse per column into shared memory for pass 2, which meanwhile still
+//                works on the item before;
 //   warps 4-11   pass 1, one warpgroup per 32 columns: each thread owns one key (one TMEM
-//                lane) and keeps a running (max, sum of 2^(x - max)) per column; at the end of
-//                the item the warpgroup's per-column partial goes to global memory;
-//   warps 12-15  pass 2, one warpgroup over all N columns: takes the unit's lse from warp 3
-//                (combining it itself, 128 threads, for a unit of more items) and sums
-//                2^(x - lse) over each head's rows per key.
+//                lane) and keeps a running (max, sum of 2^(x - max)) per column;
+//   warps 12-15  pass 2, one warpgroup over all N columns: sums 2^(x - lse) over each head's
+//                rows per key and writes the scores.
 // Only the last tiles of a sequence (the window's own keys, the padding past its end) need a
 // per-column mask; the others take an unmasked path of packed fp32 pair instructions.
-// Pass 1 of an item overlaps the exchange and pass 2 of the item before it, so HBM keeps
-// streaming while the CTAs wait for each other.
 #include "score_common.cuh"
 
 #include <string.h>
@@ -43,14 +51,69 @@
 
 namespace ckv {
 
-constexpr int kP1Slots = 3;                           // pass-1 ring (HBM)
-constexpr int kP2Slots = 2;                           // pass-2 ring (L2)
-constexpr int kAcc = 4;                               // TMEM accumulators per pass
-constexpr int kQBufs = 3;                             // query-row buffers: pass 1 runs two items ahead
-constexpr int kWarpCombineMax = 16;                   // units of more items: pass 2 combines (128 threads)
+namespace {
+
+constexpr int kP1Slots = 3;   // pass-1 ring (HBM)
+constexpr int kP2Slots = 2;   // pass-2 ring (L2)
+constexpr int kAcc = 4;       // TMEM accumulators per pass
+constexpr int kQBufs = 3;     // query-row buffers: pass 1 runs up to two items ahead of pass 2
+constexpr double kMaxLog2 = 1010.0;  // |log2| of a column's largest term that fp64 can hold
+
+struct alignas(128) LayersParams {
+    CUtensorMap tmap_k[kMaxLaunchLayers];  // K of each layer: {128, H_kv, T}, box {64, 1, 128}
+    CUtensorMap tmap_q[kMaxLaunchLayers];  // q_win of each layer: {128, H_q, S*w}, box {64, 1, W_PAD}
+    float* scores[kMaxLaunchLayers];       // [n_sel of the layer, T]
+    const int32_t* cu_seqlens;             // device [S+1] (checked against cu_hash)
+    double* sums;                          // [n_units][N]: per column, sum of 2^(x) over the unit
+    int* counters;                         // [n_units] arrivals, zero at launch
+    int* status;
+    int S, T, w, n_items, items_per_lb, c, n_layers;
+    int seq0, S_all;                       // the launch's first sequence, sequences of the batch
+    uint32_t cu_hash;
+    float sl2;                             // softmax scale * log2(e)
+    long long wait_cycles;
+    int16_t batch_layer[kMaxLaunchBatches];   // layer (launch-local) of each flat head batch
+    int16_t batch_group[kMaxLaunchBatches];   // KV head
+    int16_t batch_first[kMaxLaunchBatches];   // score row (in its layer) of the batch's first head
+    int16_t batch_nheads[kMaxLaunchBatches];
+    int16_t batch_sel[kMaxLaunchBatches];     // index into sel_heads of the batch's first head
+    int16_t sel_heads[kMaxLaunchSel];         // query head of each head slot
+    int32_t seq_start[kMaxLaunchSeqs];        // of the launch's sequences seq0, seq0 + 1, ...
+    int32_t seq_len[kMaxLaunchSeqs];
+    int32_t seq_item0[kMaxLaunchSeqs + 1];    // first item of each sequence within a head batch
+};
+static_assert(sizeof(LayersParams) <= 32000, "kernel parameters");
+
+struct Item {
+    int layer, batch, seq, unit, tile0, ntiles, start, len, nitems;
+};
+
+// Work item i of the launch: head batch i / M, then the sequence whose items hold i % M.
+__device__ __forceinline__ Item get_item(const LayersParams& p, int i) {
+    Item it;
+    const int lb = i / p.items_per_lb;
+    const int r = i - lb * p.items_per_lb;
+    int lo = 0, hi = p.S - 1;  // the last sequence whose first item is at or before r
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (p.seq_item0[mid] <= r) lo = mid;
+        else hi = mid - 1;
+    }
+    it.batch = lb;
+    it.layer = p.batch_layer[lb];
+    it.seq = lo;
+    it.unit = lb * p.S + lo;
+    it.start = p.seq_start[lo];
+    it.len = p.seq_len[lo];
+    it.nitems = p.seq_item0[lo + 1] - p.seq_item0[lo];
+    it.tile0 = (r - p.seq_item0[lo]) * p.c;
+    const int tiles = (it.len + kTileKeys - 1) / kTileKeys;
+    it.ntiles = min(p.c, tiles - it.tile0);
+    return it;
+}
 
 template <int N>
-struct SmemLayout {
+struct LayersSmem {
     static constexpr int kP1 = 0;
     static constexpr int kP2 = kP1 + kP1Slots * kTileBytes;
     static constexpr int kQ = kP2 + kP2Slots * kTileBytes;
@@ -71,73 +134,57 @@ struct SmemLayout {
     static constexpr int kBytes = kAbort + 4;
     static constexpr int kDynamic = kBytes + 1024;      // slack to align the base to 1024 B
 };
+// dynamic + the kernel's static shared memory (under 5 KB) within the 227 KB a block may use
+static_assert(LayersSmem<64>::kDynamic + 5 * 1024 <= 232448, "shared memory, N = 64");
 
-// The unit's -lse per column (log2 units, -inf for a column without a real window row or
-// without a visible key) from its items' partials, by one warp: lane 0 waits (bounded acquire
-// spin) until every item of the unit has published, then, if `combine`, lane l combines the
-// column pair (2l, 2l + 1) over the items, kU partials in flight (a unit of many items is
-// combined by the pass-2 warpgroup instead, which has the threads for more loads in flight).
-template <int N, int W_PAD>
-__device__ __forceinline__ bool warp_unit_lse(const ScoreParams& p, const ScoreUnit& U, int unit,
-                                              int lane, float* nlse, bool combine,
-                                              volatile int* abort, long long lim) {
-    constexpr int kNW = N / kCols, kPairs = N / 2, kU = 4;
-    int got = 1;
-    if (lane == 0) {
-        const int target = U.nitems * kNW;
-        const long long t0 = clock64();
-        for (uint32_t k = 1; ld_acquire(p.counters + unit) < target; ++k) {
-            __nanosleep(32);
-            if ((k & 63u) == 0u && (*abort || clock64() - t0 > lim)) {
-                got = 0;
-                break;
-            }
-        }
-    }
-    __syncwarp();  // the acquire above orders the other lanes' reads of the partials too
-    if (__shfl_sync(0xffffffffu, got, 0) == 0) return false;
-    if (combine && lane < kPairs) {
-        const float4* src = reinterpret_cast<const float4*>(p.partials + static_cast<size_t>(U.first_item) * N) + lane;
-        float M0 = -INFINITY, S0 = 0.f, M1 = -INFINITY, S1 = 0.f;
-        for (int k0 = 0; k0 < U.nitems; k0 += kU) {
-            float4 pr[kU];
+// End of a pass-1 item for one warpgroup of kCols columns: per column, the warp maximum by
+// redux and the sums rescaled to it, the warps' sums by recursive halving, then the four warps
+// through shared memory `red`; thread c < kCols adds column c's sum, as an fp64 multiple of
+// its maximum's power of two, to the unit's accumulator `sums[c]` once the publisher has
+// released the previous use of this pub_full/pub_empty pair, and arrives on pub_full.
+__device__ __forceinline__ bool item_sums(float (&m)[kCols], float (&s)[kCols], float2* red, int eq,
+                                          int lane, int wtid, uint64_t* gbar, uint32_t& gphase,
+                                          uint64_t* pub_full, uint64_t* pub_empty, uint32_t pub_phase,
+                                          double* sums, int* status, volatile int* abort,
+                                          long long lim) {
 #pragma unroll
-            for (int u = 0; u < kU; ++u)
-                pr[u] = k0 + u < U.nitems ? __ldcg(src + static_cast<size_t>(k0 + u) * kPairs)
-                                          : make_float4(-INFINITY, 0.f, -INFINITY, 0.f);
-#pragma unroll
-            for (int u = 0; u < kU; ++u) {
-                float Mn = fmaxf(M0, pr[u].x);
-                if (Mn > -INFINITY) {
-                    S0 = S0 * ex2_approx(M0 - Mn) + pr[u].y * ex2_approx(pr[u].x - Mn);
-                    M0 = Mn;
-                }
-                Mn = fmaxf(M1, pr[u].z);
-                if (Mn > -INFINITY) {
-                    S1 = S1 * ex2_approx(M1 - Mn) + pr[u].w * ex2_approx(pr[u].z - Mn);
-                    M1 = Mn;
-                }
-            }
-        }
-        const int nheads = p.batch_nheads[U.batch];
-        const int c0 = 2 * lane, c1 = c0 + 1;
-        const bool real0 = (c0 % W_PAD) < p.w && (c0 / W_PAD) < nheads;
-        const bool real1 = (c1 % W_PAD) < p.w && (c1 / W_PAD) < nheads;
-        nlse[c0] = real0 && S0 > 0.f ? -(M0 + lg2_approx(S0)) : -INFINITY;
-        nlse[c1] = real1 && S1 > 0.f ? -(M1 + lg2_approx(S1)) : -INFINITY;
+    for (int i = 0; i < kCols; ++i) {
+        const float M = redux_max(m[i]);
+        s[i] *= ex2_approx(m[i] - M);
+        m[i] = M;
     }
-    __syncwarp();
+    transpose_reduce<kCols>(s, m, lane);  // lane l: column l
+    red[eq * 32 + lane] = make_float2(m[0], s[0]);
+    if (!group_sync(gbar, gphase, abort, lim)) return false;
+    if (wtid < kCols) {
+        float M = red[wtid].x;
+#pragma unroll
+        for (int q = 1; q < 4; ++q) M = fmaxf(M, red[q * 32 + wtid].x);
+        float S = 0.f;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const float2 x = red[q * 32 + wtid];
+            S += x.y * ex2_approx(x.x - M);
+        }
+        if (!mbar_wait(pub_empty, pub_phase ^ 1, abort, lim)) return false;
+        if (S > 0.f) {
+            if (!(fabs(static_cast<double>(M)) <= kMaxLog2)) record_error(status, kDevRange, wtid);
+            else atomicAdd(sums + wtid, static_cast<double>(S) * exp2(static_cast<double>(M)));
+        }
+        __threadfence();  // the add is performed before the publisher's release below
+        mbar_arrive(pub_full);
+    }
     return true;
 }
 
 template <int N, int W_PAD>
-__global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constant__ ScoreParams p) {
+__global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_constant__ LayersParams p) {
     static_assert(N == 32 || N == 64, "N");
     static_assert(W_PAD == 8 || W_PAD == 16 || W_PAD == 32 || W_PAD == 64, "W_PAD");
     static_assert(W_PAD <= N, "a head's rows fit in one MMA");
     constexpr int kNW = N / kCols;                      // warpgroups per pass
-    constexpr int kTmemCols = 2 * kAcc * N;           // pass-1 accumulators, then pass-2
-    using SL = SmemLayout<N>;
+    constexpr int kTmemCols = 2 * kAcc * N;             // pass-1 accumulators, then pass-2
+    using SL = LayersSmem<N>;
     constexpr uint32_t kIdesc = idesc_bf16_f32(kTileKeys, N);
 
     extern __shared__ uint8_t smem_raw[];
@@ -159,18 +206,19 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
     uint64_t* q_empty = bars + SL::kQEmpty;
     uint64_t* done = bars + SL::kDone;
     uint64_t* group = bars + SL::kGroup;        // one per epilogue warpgroup: A0 A1 B
-    uint64_t* pub_full = bars + SL::kPubFull;   // pass-1 partials of an item stored (item parity)
+    uint64_t* pub_full = bars + SL::kPubFull;   // pass-1 sums of an item added (item parity)
     uint64_t* pub_empty = bars + SL::kPubEmpty;
     uint64_t* lse_full = bars + SL::kLseFull;   // a unit's lse is in nlse_s[item parity]
     uint64_t* lse_empty = bars + SL::kLseEmpty; // pass 2 is done with nlse_s[item parity]
     // scratch of the epilogues (static, so that its accesses are shared-memory instructions)
     __shared__ float2 red_a[2][2][128];  // [item parity][warpgroup][warp * 32 + lane]
     __shared__ __align__(16) float nlse_s[2][64];  // -lse per column, by item parity
-    __shared__ float2 red_b[256];                     // pass-2 combine of a many-item unit
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + SL::kTmemSlot);
     volatile int* abort = reinterpret_cast<volatile int*>(sm + SL::kAbort);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int G = gridDim.x;
+    const int n_items = p.n_items;
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < kP1Slots; ++i) {
@@ -202,8 +250,10 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         }
         *abort = 0;
         fence_mbar_init();
-        tma_prefetch_desc(&p.tmap_k);
-        tma_prefetch_desc(&p.tmap_q);
+    }
+    if (warp == 0 && lane < p.n_layers) {  // every layer's tensor maps, one lane each
+        tma_prefetch_desc(&p.tmap_k[lane]);
+        tma_prefetch_desc(&p.tmap_q[lane]);
     }
     // Query slots of head batches with fewer heads than the MMA's columns are never loaded;
     // zeros there keep those (unused) columns finite.
@@ -214,21 +264,18 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         tmem_alloc(tmem_slot, kTmemCols);
         tmem_relinquish();
     }
-    if (blockIdx.x == 0 && threadIdx.x == 64 && seqlens_hash(p.cu_seqlens, p.S) != p.cu_hash)
+    if (blockIdx.x == 0 && threadIdx.x == 64 && seqlens_hash(p.cu_seqlens, p.S_all) != p.cu_hash)
         record_error(p.status, kDevBadSeqlens, 100);
     tc_fence_before_sync();
     __syncthreads();
     tc_fence_after_sync();
     const uint32_t tmem_base = *tmem_slot;
     // Registers: launched at 128 per thread (512 x 128 = 65536); on entry the producer/MMA/
-    // query warpgroup gives up to 56, which leaves room for the two pass-1 warpgroups' 160;
+    // publisher warpgroup gives up to 56, which leaves room for the two pass-1 warpgroups' 160;
     // the pass-2 warpgroup keeps 128 (128*56 + 256*160 + 128*128 = 64512).
-    const int R = p.n_rounds;
-    const int G = gridDim.x;
     // Limit of the waits on other roles and other CTAs (the waits for this block's own copies
     // and MMAs before it exits keep the long default, whatever this is).
     const long long lim = p.wait_cycles;
-    auto item_of = [&](int r) -> const ScoreItem& { return p.items[r * G + blockIdx.x]; };
 
     if (warp < kWarpA) {
     setmaxnreg_dec<56>();
@@ -240,24 +287,16 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             // Pass-1 tiles are read again by pass 2 shortly after: ask L2 to keep them, and to
             // drop them first once pass 2 has read them.
             const uint64_t pol1 = l2_policy_evict_last(), pol2 = l2_policy_evict_first();
-            auto next_item = [&](int r) {
-                while (r < R && item_of(r).ntiles == 0) ++r;
-                return r;
-            };
-            int r1 = next_item(0), jt1 = 0, it1 = 0, use1 = 0;
-            int r2 = r1, jt2 = 0, it2 = 0, use2 = 0;
-            ScoreItem I1{}, I2{};
-            ScoreUnit U1{}, U2{};
-            if (r1 < R) {
-                I1 = I2 = item_of(r1);
-                U1 = U2 = p.units[I1.unit];
-            }
+            int i1 = blockIdx.x, jt1 = 0, it1 = 0, use1 = 0;
+            int i2 = blockIdx.x, jt2 = 0, it2 = 0, use2 = 0;
+            Item I1{}, I2{};
+            if (i1 < n_items) I1 = I2 = get_item(p, i1);
             bool q_out = false, ok = true;
             long long t0 = clock64();
             uint32_t idle = 0;
-            while (r1 < R || r2 < R) {
+            while (i1 < n_items || i2 < n_items) {
                 bool did = false;
-                if (r1 < R) {
+                if (i1 < n_items) {
                     if (!q_out) {
                         // The item's window query rows: per head of the batch two boxes of 64
                         // dims x W_PAD rows in the MMA's 128-byte-swizzled layout.  Rows past w
@@ -266,13 +305,15 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                         const int qb = it1 % kQBufs;
                         if (mbar_test(&q_empty[qb], ((it1 / kQBufs) & 1) ^ 1)) {
                             uint8_t* qdst = qbuf + qb * SL::kQBytes;
-                            const int first_row = p.batch_first[U1.batch], nheads = p.batch_nheads[U1.batch];
+                            const int nheads = p.batch_nheads[I1.batch], sel0 = p.batch_sel[I1.batch];
+                            const CUtensorMap* qm = &p.tmap_q[I1.layer];
                             mbar_arrive_expect_tx(&q_full[qb], static_cast<uint32_t>(nheads * W_PAD * 256));
                             for (int slot = 0; slot < nheads; ++slot) {
-                                const int h = p.sel_heads[first_row + slot];
+                                const int h = p.sel_heads[sel0 + slot];
                                 uint8_t* d = qdst + slot * W_PAD * 128;
-                                tma_load_3d(d, &p.tmap_q, &q_full[qb], 0, h, U1.seq * p.w);
-                                tma_load_3d(d + SL::kQHalf, &p.tmap_q, &q_full[qb], 64, h, U1.seq * p.w);
+                                const int row = (p.seq0 + I1.seq) * p.w;
+                                tma_load_3d(d, qm, &q_full[qb], 0, h, row);
+                                tma_load_3d(d + SL::kQHalf, qm, &q_full[qb], 64, h, row);
                             }
                             q_out = true;
                             did = true;
@@ -282,44 +323,40 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                     if (q_out && mbar_test(&free1[s], ((use1 / kP1Slots) & 1) ^ 1)) {
                         mbar_arrive_expect_tx(&full1[s], kTileBytes);
                         uint8_t* dst = ring1 + s * kTileBytes;
-                        const int g = p.batch_group[U1.batch];
-                        const int tok = U1.seq_start + (I1.tile0 + jt1) * kTileKeys;
-                        tma_load_3d_hint(dst, &p.tmap_k, &full1[s], 0, g, tok, pol1);
-                        tma_load_3d_hint(dst + kHalfBytes, &p.tmap_k, &full1[s], 64, g, tok, pol1);
+                        const int g = p.batch_group[I1.batch];
+                        const int tok = I1.start + (I1.tile0 + jt1) * kTileKeys;
+                        const CUtensorMap* km = &p.tmap_k[I1.layer];
+                        tma_load_3d_hint(dst, km, &full1[s], 0, g, tok, pol1);
+                        tma_load_3d_hint(dst + kHalfBytes, km, &full1[s], 64, g, tok, pol1);
                         ++use1;
                         did = true;
                         if (++jt1 == I1.ntiles) {
                             jt1 = 0;
                             ++it1;
                             q_out = false;
-                            r1 = next_item(r1 + 1);
-                            if (r1 < R) {
-                                I1 = item_of(r1);
-                                U1 = p.units[I1.unit];
-                            }
+                            i1 += G;
+                            if (i1 < n_items) I1 = get_item(p, i1);
                         }
                     }
                 }
                 // pass 2 of an item follows its pass-1 loads, so that it reads L2
-                if (r2 < R && it2 < it1) {
+                if (i2 < n_items && it2 < it1) {
                     const int s = use2 % kP2Slots;
                     if (mbar_test(&free2[s], ((use2 / kP2Slots) & 1) ^ 1)) {
                         mbar_arrive_expect_tx(&full2[s], kTileBytes);
                         uint8_t* dst = ring2 + s * kTileBytes;
-                        const int g = p.batch_group[U2.batch];
-                        const int tok = U2.seq_start + (I2.tile0 + jt2) * kTileKeys;
-                        tma_load_3d_hint(dst, &p.tmap_k, &full2[s], 0, g, tok, pol2);
-                        tma_load_3d_hint(dst + kHalfBytes, &p.tmap_k, &full2[s], 64, g, tok, pol2);
+                        const int g = p.batch_group[I2.batch];
+                        const int tok = I2.start + (I2.tile0 + jt2) * kTileKeys;
+                        const CUtensorMap* km = &p.tmap_k[I2.layer];
+                        tma_load_3d_hint(dst, km, &full2[s], 0, g, tok, pol2);
+                        tma_load_3d_hint(dst + kHalfBytes, km, &full2[s], 64, g, tok, pol2);
                         ++use2;
                         did = true;
                         if (++jt2 == I2.ntiles) {
                             jt2 = 0;
                             ++it2;
-                            r2 = next_item(r2 + 1);
-                            if (r2 < R) {
-                                I2 = item_of(r2);
-                                U2 = p.units[I2.unit];
-                            }
+                            i2 += G;
+                            if (i2 < n_items) I2 = get_item(p, i2);
                         }
                     }
                 }
@@ -363,9 +400,8 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             const uint32_t d0 = tmem_base + static_cast<uint32_t>((first ? 0 : kAcc) * N);
             int it = 0, use = 0;
             bool ok = true;
-            for (int r = 0; ok && r < R; ++r) {
-                const int n = item_of(r).ntiles;
-                if (n == 0) continue;
+            for (int i = blockIdx.x; ok && i < n_items; i += G) {
+                const int n = get_item(p, i).ntiles;
                 const int qb = it % kQBufs;
                 if (!mbar_wait(&q_full[qb], (it / kQBufs) & 1, abort, lim)) {
                     ok = false;
@@ -406,18 +442,16 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         }
         __syncwarp();
     } else if (warp == 3) {
-        // ------------------------------------------------------------ publisher and combiner
-        // Per item: once both pass-1 warpgroups have stored its partials (their pub_full
-        // arrival releases them to lane 0 at CTA scope), one release add on the unit's arrival
-        // counter makes them visible GPU-wide (a release is cumulative).  Then the warp waits
-        // for the unit's other items, combines all their partials into the unit's lse and
-        // leaves it in nlse_s for pass 2, which meanwhile still works on the item before: the
-        // exchange stays off pass 2's path unless pass 1 elsewhere is late.
+        // ------------------------------------------------------------ publisher
+        // Per item: once both pass-1 warpgroups have added its sums (each thread's fence
+        // ordered its add before its pub_full arrival), one release add on the unit's counter.
+        // Then the warp waits until every item of the unit has arrived and leaves the unit's
+        // -lse per column in nlse_s for pass 2, which meanwhile still works on the item
+        // before: the exchange stays off pass 2's path unless pass 1 elsewhere is late.
         int it = 0;
         bool ok = true;
-        for (int r = 0; r < R; ++r) {
-            const ScoreItem I = item_of(r);
-            if (I.ntiles == 0) continue;
+        for (int i = blockIdx.x; i < n_items; i += G) {
+            const Item I = get_item(p, i);
             const int buf = it & 1;
             int good = 1;
             if (lane == 0) {
@@ -428,14 +462,35 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                     mbar_arrive(&pub_empty[buf]);
                     good = mbar_wait(&lse_empty[buf], ((it >> 1) & 1) ^ 1, abort, lim) ? 1 : 0;
                 }
+                if (good) {  // bounded acquire spin until every item of the unit has arrived
+                    const int target = I.nitems * kNW;
+                    const long long t0 = clock64();
+                    for (uint32_t k = 1; ld_acquire(p.counters + I.unit) < target; ++k) {
+                        __nanosleep(32);
+                        if ((k & 63u) == 0u && (*abort || clock64() - t0 > lim)) {
+                            good = 0;
+                            break;
+                        }
+                    }
+                }
             }
-            const ScoreUnit& U = p.units[I.unit];
-            if (__shfl_sync(0xffffffffu, good, 0) == 0 ||
-                !warp_unit_lse<N, W_PAD>(p, U, I.unit, lane, nlse_s[buf], U.nitems <= kWarpCombineMax,
-                                         abort, lim)) {
+            __syncwarp();  // the acquire above orders the other lanes' reads of the sums too
+            if (__shfl_sync(0xffffffffu, good, 0) == 0) {
                 ok = false;
                 break;
             }
+            if (lane < N / 2) {
+                const double* src = p.sums + static_cast<size_t>(I.unit) * N;
+                const int nheads = p.batch_nheads[I.batch];
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    const int c = 2 * lane + e;
+                    const double v = __ldcg(src + c);
+                    const bool real = (c % W_PAD) < p.w && (c / W_PAD) < nheads;
+                    nlse_s[buf][c] = real && v > 0.0 ? -static_cast<float>(log2(v)) : -INFINITY;
+                }
+            }
+            __syncwarp();
             if (lane == 0) mbar_arrive(&lse_full[buf]);
             ++it;
         }
@@ -457,22 +512,19 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             uint32_t gphase = 0;
             int a_it = 0, a_item = 0;
             bool ok = true;
-            for (int r = 0; ok && r < R; ++r) {
-                const int item = r * G + blockIdx.x;
-                const ScoreItem I = p.items[item];
+            for (int i = blockIdx.x; ok && i < n_items; i += G) {
+                const Item I = get_item(p, i);
                 const int n = I.ntiles;
-                if (n == 0) continue;
-                const ScoreUnit U = p.units[I.unit];
-                const int L = U.len, P = L - p.w;
+                const int L = I.len, P = L - p.w;
                 const float sl2 = p.sl2;
                 // Running maximum (log2 units, kept negated so that it is the FMA's addend) and
                 // the sum relative to it.  -1e30 (not -inf) for a column with no visible key
                 // yet keeps the reductions below free of inf - inf.
                 float nm[kCols], sm_[kCols];
 #pragma unroll
-                for (int i = 0; i < kCols; ++i) {
-                    nm[i] = 1e30f;
-                    sm_[i] = 0.f;
+                for (int c = 0; c < kCols; ++c) {
+                    nm[c] = 1e30f;
+                    sm_[c] = 0.f;
                 }
                 for (int jt = 0; jt < n; ++jt, ++a_it) {
                     const int acc = a_it % kAcc;
@@ -487,8 +539,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                     // every row, and the columns without a real row are never read, so no mask.
                     const bool edge = (t * kTileKeys + kTileKeys - 1 >= P) || (t * kTileKeys + kTileKeys > L);
                     const uint32_t taddr = tmem_base + lane_base + static_cast<uint32_t>(acc * N + col0);
-                    // both halves of 16 columns in flight, then one wait
-                    float vv[2][16];
+                    float vv[2][16];  // both halves of 16 columns in flight, then one wait
                     tmem_ld16_nowait(taddr, vv[0]);
                     tmem_ld16_nowait(taddr + 16, vv[1]);
                     tmem_ld_wait();
@@ -510,11 +561,11 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                 }
                 float m[kCols];
 #pragma unroll
-                for (int i = 0; i < kCols; ++i) m[i] = -nm[i];
+                for (int c = 0; c < kCols; ++c) m[c] = -nm[c];
                 if (!ok) break;
-                if (!item_partials(m, sm_, red_a[a_item & 1][wg], eq, lane, wtid, gbar, gphase,
-                                   &pub_full[a_item & 1], &pub_empty[a_item & 1], (a_item >> 1) & 1,
-                                   p.partials + static_cast<size_t>(item) * N + col0, abort, lim)) {
+                if (!item_sums(m, sm_, red_a[a_item & 1][wg], eq, lane, wtid, gbar, gphase,
+                               &pub_full[a_item & 1], &pub_empty[a_item & 1], (a_item >> 1) & 1,
+                               p.sums + static_cast<size_t>(I.unit) * N + col0, p.status, abort, lim)) {
                     ok = false;
                     break;
                 }
@@ -530,23 +581,19 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         // One warpgroup over all N columns; lse sits in shared memory and is read by every
         // lane of a warp at the same address.
         const int eq = warp & 3;
-        const int wtid = threadIdx.x - kWarpB * 32;  // 0 .. 127
         const uint32_t lane_base = static_cast<uint32_t>(eq * 32) << 16;
-        uint64_t* gbar = &group[2];
-        uint32_t gphase = 0;
         constexpr int kHeads = N / W_PAD;  // head slots of the MMA's columns
         int b_it = 0, n_item = 0;
         bool ok = true;
-        for (int r = 0; ok && r < R; ++r) {
-            const ScoreItem I = p.items[r * G + blockIdx.x];
-            const int n = I.ntiles;
-            if (n == 0) continue;
-            const ScoreUnit U = p.units[I.unit];
-            const int L = U.len, P = L - p.w;
-            const int first = p.batch_first[U.batch], nheads = p.batch_nheads[U.batch];
-            const int T = p.T;
+        for (int i = blockIdx.x; ok && i < n_items; i += G) {
+            const Item I = get_item(p, i);
+            const int n = I.ntiles, tile0 = I.tile0;
+            const int L = I.len, P = L - p.w;
+            const int nheads = p.batch_nheads[I.batch];
+            const size_t T = static_cast<size_t>(p.T);
             const float sl2 = p.sl2;
-            float* const scores = p.scores;
+            // the batch's first score row, at the sequence's first token
+            float* const out = p.scores[I.layer] + static_cast<size_t>(p.batch_first[I.batch]) * T + I.start;
             // ---------------------------------------------------- the unit's lse (warp 3)
             const int buf = n_item & 1;
             int good = 1;
@@ -555,16 +602,6 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             if (__shfl_sync(0xffffffffu, good, 0) == 0) {
                 ok = false;
                 break;
-            }
-            if (U.nitems > kWarpCombineMax) {  // warp 3 only acquired: combine here
-                uint64_t colmask = 0;           // columns that hold a real window row
-#pragma unroll
-                for (int c = 0; c < N; ++c)
-                    if ((c % W_PAD) < p.w && (c / W_PAD) < nheads) colmask |= 1ull << c;
-                if (!unit_combine<N>(p, U, wtid, gbar, gphase, red_b, nlse_s[buf], colmask, abort, lim)) {
-                    ok = false;
-                    break;
-                }
             }
             const float* nlse = nlse_s[buf];
             // ---------------------------------------------------- the item's tiles
@@ -575,12 +612,11 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                     break;
                 }
                 tc_fence_after_sync();
-                const int t = I.tile0 + jt;
+                const int t = tile0 + jt;
                 const int j = t * kTileKeys + eq * 32 + lane;
                 const bool edge = (t * kTileKeys + kTileKeys - 1 >= P) || (t * kTileKeys + kTileKeys > L);
                 const uint32_t taddr = tmem_base + lane_base + static_cast<uint32_t>((kAcc + acc) * N);
-                // every 16-column chunk in flight, then one wait
-                float vv[N / 16][16];
+                float vv[N / 16][16];  // every 16-column chunk in flight, then one wait
 #pragma unroll
                 for (int hh = 0; hh < N / 16; ++hh) tmem_ld16_nowait(taddr + hh * 16, vv[hh]);
                 tmem_ld_wait();
@@ -596,10 +632,9 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                     prob_sums<N, W_PAD, true>(vv, sl2, nlse, j < L ? j - P : (1 << 30), accum);
                 }
                 if (j < L) {
-                    const size_t col = static_cast<size_t>(U.seq_start) + j;
 #pragma unroll
                     for (int h = 0; h < kHeads; ++h)
-                        if (h < nheads) scores[static_cast<size_t>(first + h) * T + col] = accum[h];
+                        if (h < nheads) out[h * T + j] = accum[h];
                 }
             }
             __syncwarp();
@@ -620,13 +655,10 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
     }
 }
 
-// ------------------------------------------------------------------------------ host side
-namespace {
-
 template <int N, int W_PAD>
-cudaError_t launch_one(const ScoreParams& p, int grid, cudaStream_t stream) {
-    auto kern = score_kernel<N, W_PAD>;
-    constexpr int smem = SmemLayout<N>::kDynamic;
+cudaError_t launch_one(const LayersParams& p, int grid, cudaStream_t stream) {
+    auto kern = score_layers_kernel<N, W_PAD>;
+    constexpr int smem = LayersSmem<N>::kDynamic;
     static bool configured = false;  // benign race: the attribute call is idempotent
     if (!configured) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
@@ -647,7 +679,7 @@ cudaError_t launch_one(const ScoreParams& p, int grid, cudaStream_t stream) {
     return cudaLaunchKernelEx(&cfg, kern, p);
 }
 
-cudaError_t dispatch(const ScoreParams& p, int n_cols, int w_pad, int grid, cudaStream_t st) {
+cudaError_t dispatch(const LayersParams& p, int n_cols, int w_pad, int grid, cudaStream_t st) {
     if (n_cols == 32) {
         if (w_pad == 8) return launch_one<32, 8>(p, grid, st);
         if (w_pad == 16) return launch_one<32, 16>(p, grid, st);
@@ -663,53 +695,59 @@ cudaError_t dispatch(const ScoreParams& p, int n_cols, int w_pad, int grid, cuda
 
 }  // namespace
 
-cudaError_t launch_score(const ScoreLaunch& L, cudaStream_t stream) {
-    static_assert(sizeof(ScoreParams) <= 32000, "kernel parameters");
-    static ScoreParams p;  // ~25 KB, kept off the host stack; calls are serialised by `mu`
+cudaError_t launch_score_layers(const LayersLaunch& L, cudaStream_t stream) {
+    static LayersParams p;  // ~22 KB, kept off the host stack; calls are serialised by `mu`
     static std::mutex mu;
     std::lock_guard<std::mutex> lock(mu);
     memset(&p, 0, sizeof(p));
-    p.tmap_k = L.tmap_k;
-    p.tmap_q = L.tmap_q;
-    p.q_win = reinterpret_cast<const __nv_bfloat16*>(L.q_win);
+    const int nl = static_cast<int>(L.layers.size());
+    const int nb = static_cast<int>(L.batch_layer.size());
+    const int ns = static_cast<int>(L.seq_start.size());
+    if (nl < 1 || nl > kMaxLaunchLayers || nb < 1 || nb > kMaxLaunchBatches ||
+        static_cast<int>(L.sel_heads.size()) > kMaxLaunchSel || ns < 1 || ns > kMaxLaunchSeqs)
+        return cudaErrorInvalidValue;
+    for (int l = 0; l < nl; ++l) {
+        p.tmap_k[l] = L.layers[l].tmap_k;
+        p.tmap_q[l] = L.layers[l].tmap_q;
+        p.scores[l] = L.layers[l].scores;
+    }
     p.cu_seqlens = L.cu_seqlens_dev;
-    p.partials = reinterpret_cast<float2*>(L.partials);
+    p.sums = L.sums;
     p.counters = L.counters;
-    p.scores = L.scores;
     p.status = L.status;
-    p.S = L.S;
+    p.S = ns;
     p.T = L.T;
-    p.Hq = L.Hq;
     p.w = L.w;
+    p.items_per_lb = L.seq_item0[ns];
+    p.n_items = nb * p.items_per_lb;
+    p.c = L.c;
+    p.n_layers = nl;
+    p.seq0 = L.seq0;
+    p.S_all = L.S_all;
     p.cu_hash = L.cu_hash;
     p.sl2 = L.softmax_scale * 1.4426950408889634f;
     p.wait_cycles = wait_limit_cycles();
-    p.lse = L.lse;
-    p.lse_stride = L.lse_head_stride;
-    for (int b = 0; b < L.nb; ++b) {
-        p.batch_group[b] = static_cast<int16_t>(L.batch_group[b]);
-        p.batch_first[b] = static_cast<int16_t>(L.batch_first[b]);
-        p.batch_nheads[b] = static_cast<int16_t>(L.batch_nheads[b]);
+    for (int b = 0; b < nb; ++b) {
+        p.batch_layer[b] = L.batch_layer[b];
+        p.batch_group[b] = L.batch_group[b];
+        p.batch_first[b] = L.batch_first[b];
+        p.batch_nheads[b] = L.batch_nheads[b];
+        p.batch_sel[b] = L.batch_sel[b];
     }
-    for (int i = 0; i < L.n_sel; ++i) p.sel_heads[i] = static_cast<int16_t>(L.sel_heads[i]);
-    // One launch per slice of rounds whose items and units fit the parameter tables.
-    for (const ScoreSlice& sl : L.slices) {
-        p.n_rounds = sl.n_rounds;
-        p.n_items = sl.n_rounds * L.grid;
-        p.n_units = sl.n_units;
-        memcpy(p.items, L.items.data() + sl.item0, sizeof(ScoreItem) * p.n_items);
-        memcpy(p.units, L.units.data() + sl.unit0, sizeof(ScoreUnit) * p.n_units);
-        cudaError_t e = cudaSuccess;
-        if (!L.lse) {  // the unit arrival counters of the exchange
-            e = cudaMemsetAsync(L.counters, 0, sizeof(int) * sl.n_units, stream);
-            if (e != cudaSuccess) return e;
-        }
-        e = L.lse ? launch_given_lse(p, L.n_cols, L.w_pad, L.grid, stream)
-            : L.resident ? launch_resident(p, L.n_cols, L.w_pad, L.grid, stream)
-                         : dispatch(p, L.n_cols, L.w_pad, L.grid, stream);
-        if (e != cudaSuccess) return e;
+    for (size_t i = 0; i < L.sel_heads.size(); ++i) p.sel_heads[i] = L.sel_heads[i];
+    for (int s = 0; s < ns; ++s) {
+        p.seq_start[s] = L.seq_start[s];
+        p.seq_len[s] = L.seq_len[s];
+        p.seq_item0[s] = L.seq_item0[s];
     }
-    return cudaSuccess;
+    p.seq_item0[ns] = L.seq_item0[ns];
+    if (p.n_items == 0) return cudaSuccess;
+    // the exchange's accumulators and arrival counters start at zero
+    const size_t n_units = static_cast<size_t>(nb) * ns;
+    cudaError_t e = cudaMemsetAsync(L.sums, 0, n_units * L.n_cols * sizeof(double), stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(L.counters, 0, n_units * sizeof(int), stream);
+    if (e != cudaSuccess) return e;
+    return dispatch(p, L.n_cols, L.w_pad, std::min(L.grid, p.n_items), stream);
 }
 
 }  // namespace ckv

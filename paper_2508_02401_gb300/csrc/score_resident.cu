@@ -30,6 +30,8 @@
 // the ring keeps loading meanwhile.
 #include "score_common.cuh"
 
+#include <mutex>
+
 #include <string.h>
 
 namespace ckv {
@@ -575,6 +577,57 @@ cudaError_t launch_resident(const ScoreParams& p, int n_cols, int w_pad, int gri
         if (w_pad == 64) return launch_res<64, 64>(p, grid, st);
     }
     return cudaErrorInvalidValue;
+}
+
+// The kernels that take the work-item tables of ScoreParams: the TMEM-resident two-pass kernel
+// (above) and the single pass with the window rows' lse given (score_lse.cu).  One launch per
+// slice of rounds whose items and units fit the parameter tables.
+cudaError_t launch_score(const ScoreLaunch& L, cudaStream_t stream) {
+    static_assert(sizeof(ScoreParams) <= 32000, "kernel parameters");
+    static ScoreParams p;  // ~25 KB, kept off the host stack; calls are serialised by `mu`
+    static std::mutex mu;
+    std::lock_guard<std::mutex> lock(mu);
+    memset(&p, 0, sizeof(p));
+    p.tmap_k = L.tmap_k;
+    p.tmap_q = L.tmap_q;
+    p.q_win = reinterpret_cast<const __nv_bfloat16*>(L.q_win);
+    p.cu_seqlens = L.cu_seqlens_dev;
+    p.partials = reinterpret_cast<float2*>(L.partials);
+    p.counters = L.counters;
+    p.scores = L.scores;
+    p.status = L.status;
+    p.S = L.S;
+    p.T = L.T;
+    p.Hq = L.Hq;
+    p.w = L.w;
+    p.cu_hash = L.cu_hash;
+    p.sl2 = L.softmax_scale * 1.4426950408889634f;
+    p.wait_cycles = wait_limit_cycles();
+    p.lse = L.lse;
+    p.lse_stride = L.lse_head_stride;
+    for (int b = 0; b < L.nb; ++b) {
+        p.batch_group[b] = static_cast<int16_t>(L.batch_group[b]);
+        p.batch_first[b] = static_cast<int16_t>(L.batch_first[b]);
+        p.batch_nheads[b] = static_cast<int16_t>(L.batch_nheads[b]);
+    }
+    for (int i = 0; i < L.n_sel; ++i) p.sel_heads[i] = static_cast<int16_t>(L.sel_heads[i]);
+    if (!L.lse && !L.resident) return cudaErrorInvalidValue;  // two-pass reload: score_layers.cu
+    for (const ScoreSlice& sl : L.slices) {
+        p.n_rounds = sl.n_rounds;
+        p.n_items = sl.n_rounds * L.grid;
+        p.n_units = sl.n_units;
+        memcpy(p.items, L.items.data() + sl.item0, sizeof(ScoreItem) * p.n_items);
+        memcpy(p.units, L.units.data() + sl.unit0, sizeof(ScoreUnit) * p.n_units);
+        cudaError_t e = cudaSuccess;
+        if (!L.lse) {  // the unit arrival counters of the exchange
+            e = cudaMemsetAsync(L.counters, 0, sizeof(int) * sl.n_units, stream);
+            if (e != cudaSuccess) return e;
+        }
+        e = L.lse ? launch_given_lse(p, L.n_cols, L.w_pad, L.grid, stream)
+                  : launch_resident(p, L.n_cols, L.w_pad, L.grid, stream);
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
 }
 
 }  // namespace ckv

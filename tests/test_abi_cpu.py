@@ -30,7 +30,8 @@ def _declared():
 def test_header_declares_the_boundary():
     names = _declared()
     for n in ("ckv_score_window", "ckv_pool", "ckv_select_topk", "ckv_gather_compact",
-              "ckv_compress_layer", "ckv_workspace_size", "ckv_keep_lengths",
+              "ckv_compress_layer", "ckv_workspace_size", "ckv_keep_lengths", "ckv_score_windows",
+              "ckv_compress_layers", "ckv_workspace_size_layers",
               "ckv_read_device_status", "ckv_status_string"):
         assert n in names
 
@@ -47,7 +48,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 
 def test_version_and_status_strings(lib):
-    assert ckv.ckv_abi_version() == 4
+    assert ckv.ckv_abi_version() == 5
     assert ckv.ckv_status_string(0) == "CKV_OK"
     assert ckv.ckv_status_string(3) == "CKV_ERR_WORKSPACE"
 
@@ -170,3 +171,63 @@ def test_layer_scope_accepts_groups_without_heads(lib):
     m[:, :4] = 1
     assert _call_compress(lib, _cfg(scope=1, head_mask=m), FakeBatch([0, 4096])) in (0, 4)
     assert _call_compress(lib, _cfg(scope=0, head_mask=m), FakeBatch([0, 4096])) == 1
+
+
+class _FakeT:
+    """A stand-in device tensor for the binding: only its address matters on the host."""
+
+    def __init__(self, addr):
+        self.addr = addr
+
+    def data_ptr(self):
+        return self.addr
+
+
+def _ios(n, **kw):
+    out = []
+    for i in range(n):
+        d = dict(layer=i % 2, q_win=_FakeT(_P), k=_FakeT(_P), v=_FakeT(_P), scores=_FakeT(_P),
+                 idx=_FakeT(_P), cu_keep_dev=_FakeT(_P), k_out=_FakeT(_P), v_out=_FakeT(_P))
+        d.update(kw)
+        out.append(ckv.LayerIO(**d))
+    return out
+
+
+def test_layers_workspace_grows_with_the_layers(lib):
+    cfg, b = _cfg(), FakeBatch([0, 4096, 5000])
+    one = ckv.ckv_workspace_size_layers(cfg, _ios(1), b)
+    four = ckv.ckv_workspace_size_layers(cfg, _ios(4), b)
+    assert one >= ckv.ckv_workspace_size(cfg, 0, b)
+    # each extra layer adds its scores [n_sel, T] and its units' exchange
+    assert four - one >= 3 * 8 * 5000 * 4
+
+
+def test_layers_argument_errors(lib):
+    cfg, b = _cfg(), FakeBatch([0, 4096, 5000])
+    ios = _ios(3)
+    arr = ckv._layer_ios(ios)
+    assert lib.ckv_score_windows(cfg.ref, 0, arr, b.ref, _P, 1 << 30, None) == 1      # no layer
+    assert lib.ckv_score_windows(cfg.ref, 3, None, b.ref, _P, 1 << 30, None) == 1     # io NULL
+    assert lib.ckv_score_windows(cfg.ref, 3, arr, b.ref, _P, 1024, None) == 3         # too small
+    assert lib.ckv_score_windows(cfg.ref, 3, arr, b.ref, _P + 64, 1 << 30, None) == 3  # misaligned
+    bad = ckv._layer_ios(_ios(3, layer=5))
+    assert lib.ckv_score_windows(cfg.ref, 3, bad, b.ref, _P, 1 << 30, None) == 1      # layer range
+    bad = ckv._layer_ios(_ios(2) + _ios(1, k=_FakeT(_P + 8)))
+    assert lib.ckv_score_windows(cfg.ref, 3, bad, b.ref, _P, 1 << 30, None) == 1      # misaligned k
+    bad = ckv._layer_ios(_ios(3, scores=None))
+    assert lib.ckv_score_windows(cfg.ref, 3, bad, b.ref, _P, 1 << 30, None) == 1      # no scores
+    bad = ckv._layer_ios(_ios(3, v=None))
+    assert lib.ckv_compress_layers(cfg.ref, 3, bad, b.ref, _P, 1 << 30, None) == 1    # no v
+    bad = ckv._layer_ios(_ios(3, cu_keep_dev=None))
+    assert lib.ckv_compress_layers(cfg.ref, 3, bad, b.ref, _P, 1 << 30, None) == 1
+    # the fused call needs room for every layer's scores; the scoring call does not
+    need = ckv.ckv_workspace_size_layers(cfg, ios, b)
+    assert lib.ckv_compress_layers(cfg.ref, 3, arr, b.ref, _P, need - 256, None) == 3
+
+
+@pytest.mark.skipif(__import__("torch").cuda.is_available(), reason="CPU-only behaviour")
+def test_valid_layers_call_without_a_gpu_reports_cuda_error(lib):
+    cfg, b = _cfg(), FakeBatch([0, 4096, 5000])
+    arr = ckv._layer_ios(_ios(3))
+    assert lib.ckv_score_windows(cfg.ref, 3, arr, b.ref, _P, 1 << 30, None) == 4
+    assert lib.ckv_compress_layers(cfg.ref, 3, arr, b.ref, _P, 1 << 30, None) == 4
