@@ -96,15 +96,21 @@ def _args():
     ap.add_argument("--srs", action="store_true",
                     help="time the Semantic Retrieval Score accumulation (Eq. 5) instead: every "
                          "head scored, the window rows as decode steps, all of them in the answer")
+    ap.add_argument("--calls", choices=("layers", "layer"), default="layers",
+                    help="layers: one ckv_compress_layers call over every layer of the step (one "
+                         "persistent scoring launch, then the selections); layer: one "
+                         "ckv_compress_layer call per layer, layers round-robin on streams")
     ap.add_argument("--split-select", action="store_true",
-                    help="each layer as ckv_score_window then ckv_select_compact, the selection "
-                         "on a stream of its own, so that the next layer's scoring need not wait")
+                    help="with --calls layer: each layer as ckv_score_window then "
+                         "ckv_select_compact, the selection on a stream of its own, so that the "
+                         "next layer's scoring need not wait")
     ap.add_argument("--lse", action="store_true",
                     help="the window rows' lse given (as a prefill attention kernel returns it): "
                          "ckv_compress_layer_lse / ckv_score_window_lse, one pass over K")
     ap.add_argument("--max-ctas", type=int, default=0,
-                    help="CTAs one call's scoring kernel may occupy (0 = SMs / 16, so that 16 "
-                         "layers' scoring kernels are resident at once)")
+                    help="CTAs one call's scoring kernel may occupy (0: all SMs with --calls "
+                         "layers; SMs / 16 with --calls layer, so that 16 layers' scoring kernels "
+                         "are resident at once)")
     ap.add_argument("--streams", type=int, default=0,
                     help="layers are issued round-robin on this many streams (one workspace each); "
                          "0 = min(layers, 16)")
@@ -284,6 +290,19 @@ def run_ours(args):
         for d in layers:
             d["scores"] = torch.empty((n_sel_max, T), dtype=torch.float32, device="cuda")
 
+    # One call for every layer of the step: ckv_compress_layers (the layers' scoring in one
+    # persistent launch over all SMs, then the selections), with the window rows' lse computed.
+    multi = args.calls == "layers" and not args.lse and not args.split_select
+    if multi:
+        cap = args.max_ctas if args.max_ctas > 0 else 0
+        cfg = ckv.Config.from_workload(wl, max_ctas=cap, score_path=path)
+        nstreams = 1
+        ios = [ckv.LayerIO(layer=l, q_win=d["q"], k=d["k"], v=d["v"], idx=d["idx"],
+                           cu_keep_dev=d["cu_keep_dev"], k_out=d["k_out"], v_out=d["v_out"])
+               for l, d in enumerate(layers)]
+        wss = [ckv.new_layers_workspace(cfg, ios, batch)]
+        ws = wss[0]
+
     def over_layers(fn, selections=False):
         # Layers are independent: layer l runs on side stream l % nstreams with its own
         # workspace, so the calls of consecutive layers overlap on the GPU (and, with
@@ -319,7 +338,10 @@ def run_ours(args):
         return st
 
     def step():
-        over_layers(compress, selections=args.split_select)
+        if multi:
+            ckv.ckv_compress_layers(cfg, ios, batch, ws, stream=stream)
+        else:
+            over_layers(compress, selections=args.split_select)
 
     with torch.cuda.stream(stream):
         for _ in range(max(1, args.warmup)):
@@ -389,8 +411,11 @@ def run_ours(args):
 
     # per layer: the scoring kernel, then the selection (pool, top-k, compaction and gather)
     lens = list(wl.seqlens)
-    per_layer = 1 + (1 if min(lens) <= SELECT_UNIT_LEN else 0) + (2 if max(lens) > SELECT_UNIT_LEN else 0)
-    launches_per_step = per_layer * nl
+    sel_per_layer = (1 if min(lens) <= SELECT_UNIT_LEN else 0) + (2 if max(lens) > SELECT_UNIT_LEN else 0)
+    if multi:  # one scoring launch per 32 layers and per 512 sequences, then the selections
+        launches_per_step = -(-nl // 32) * -(-wl.num_seqs // 512) + sel_per_layer * nl
+    else:
+        launches_per_step = (1 + sel_per_layer) * nl
 
     # --- scoring stage (the dominant kernels): a graph of every layer's ckv_score_window,
     # timed with events on its stream; the average per layer is one pass-1 + pass-2 pair.
@@ -425,7 +450,14 @@ def run_ours(args):
             ckv.ckv_score_window(cfg, l, batch, d["q"], d["k"], score_rows[l], w, stream=st)
 
     def score_all():
-        over_layers(score_one)
+        if multi:
+            ckv.ckv_score_windows(cfg, score_ios, batch, ws, stream=stream)
+        else:
+            over_layers(score_one)
+
+    if multi:
+        score_ios = [ckv.LayerIO(layer=l, q_win=d["q"], k=d["k"], scores=score_rows[l])
+                     for l, d in enumerate(layers)]
 
     score_ms = stage(score_all)
     if args.breakdown:
@@ -454,8 +486,11 @@ def run_ours(args):
     for f in SCORE_SOURCES:
         digest.update(open(os.path.join(ROOT, "paper_2508_02401_gb300", "csrc", f), "rb").read())
     traffic = SCORE_TRAFFIC.get(digest.hexdigest(), {}).get(args.workload + ("+lse" if args.lse else ""))
-    roofline = {"bound": "hbm", "kernel": "scoring kernel (ckv_score_window), per layer, layers "
-                                          f"overlapped on {nstreams} streams, {cap} CTAs per call",
+    kernel_desc = ("two-pass scoring kernel (ckv_score_windows): every layer of the step in one "
+                   f"persistent launch on {cap or sms} CTAs; per layer" if multi else
+                   "scoring kernel (ckv_score_window), per layer, layers overlapped on "
+                   f"{nstreams} streams, {cap} CTAs per call")
+    roofline = {"bound": "hbm", "kernel": kernel_desc,
                 "achieved": round(score_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
                 "frac": round(score_gbs / hbm_peak, 4), "peak_kind": peak_kind,
                 "frac_of_8TBs": round(score_gbs / 8000.0, 4),
@@ -485,7 +520,41 @@ def run_ours(args):
         back = torch.cuda.Stream()
         every = copy_streams + side + [back] + (sel_side if args.split_select else [])
 
+        E = 4  # layers per ckv_compress_layers call in the end-to-end step
+
+        def e2e_step_multi():
+            # Per chunk of E layers: its inputs on one of two copy streams, one
+            # ckv_compress_layers call on the compute stream once they have landed, its outputs
+            # back on the read-back stream; the copies overlap the other chunks' compressions.
+            for st in copy_streams + [back]:
+                st.wait_stream(stream)
+            for c0 in range(0, nl, E):
+                cp = copy_streams[(c0 // E) % len(copy_streams)]
+                with torch.cuda.stream(cp):
+                    for l in range(c0, min(nl, c0 + E)):
+                        d = layers[l]
+                        d["q"].copy_(hq[l], non_blocking=True)
+                        d["k"].copy_(hk[l], non_blocking=True)
+                        d["v"].copy_(hv[l], non_blocking=True)
+                landed = torch.cuda.Event()
+                landed.record(cp)
+                stream.wait_event(landed)
+                ckv.ckv_compress_layers(cfg, ios[c0:c0 + E], batch, ws, stream=stream)
+                done = torch.cuda.Event()
+                done.record(stream)
+                back.wait_event(done)
+                with torch.cuda.stream(back):
+                    for l in range(c0, min(nl, c0 + E)):
+                        oi[l].copy_(layers[l]["idx"], non_blocking=True)
+                        ok[l].copy_(layers[l]["k_out"], non_blocking=True)
+                        ov[l].copy_(layers[l]["v_out"], non_blocking=True)
+            for st in copy_streams + [back]:
+                stream.wait_stream(st)
+
         def e2e_step():
+            if multi:
+                e2e_step_multi()
+                return
             for st in every:
                 st.wait_stream(stream)
             for l, d in enumerate(layers):
@@ -541,11 +610,13 @@ def run_ours(args):
             "data": "synthetic",
             "config": _workload_config(wl, world),
             "run": {"graph": "one CUDA graph per step",
-                    "streams": f"layers round-robin on {nstreams} streams, scoring capped at {cap} CTAs per call",
+                    "streams": ("one stream" if multi else
+                                f"layers round-robin on {nstreams} streams, scoring capped at {cap} CTAs per call"),
                     "lse": ("window-row lse given (PyTorch logsumexp outside the timed region; "
                             "one pass over K)") if args.lse else "computed (two passes)",
-                    "calls": ("ckv_score_window + ckv_select_compact, the selection on a stream "
-                              "of its own") if args.split_select else "ckv_compress_layer",
+                    "calls": ("ckv_compress_layers over every layer of the step" if multi else
+                              "ckv_score_window + ckv_select_compact, the selection on a stream "
+                              "of its own" if args.split_select else "ckv_compress_layer per layer"),
                     "repetitions": len(reps_ms),
                     "ms_per_step_spread": {"min": round(min(reps_ms) / args.steps, 5),
                                            "median": round(ms_per_step, 5),

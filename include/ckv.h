@@ -330,7 +330,7 @@ CKV_API ckv_status ckv_set_wait_limit_us(uint32_t microseconds);
 /* Synchronises `stream`, then returns the workspace's device status: *code = 0 if no kernel
  * recorded an error since the last reset, else the first error (1 = cu_seqlens_dev disagrees
  * with the host copy, 2 = a wait timed out, 3 = an index out of range, 4 = a window row's
- * largest logit beyond +-700, which the two-pass kernel's fp64 row sums cannot hold); *detail
+ * largest logit beyond +-680, which the two-pass kernel's fp64 row sums cannot hold); *detail
  * says where.
  * With reset != 0 the status word is cleared afterwards. */
 CKV_API ckv_status ckv_read_device_status(void* workspace, ckv_stream stream, int32_t reset,

@@ -21,7 +21,7 @@
 // unit's accumulator with one atomic add, and one arrival per pass-1 warpgroup is counted on
 // the unit's counter.  A unit's lse per column is log2 of its accumulator once the counter is
 // complete: one read of N doubles, whatever the number of items.  fp64 holds 2^(+-1022), so
-// a column's largest logit must lie within +-700 (natural log units); beyond that the status
+// a column's largest logit must lie within +-680 (natural log units); beyond that the status
 // word reports kDevRange.
 //
 // One cooperative launch, one CTA per SM, 512 threads, warp-specialised:
@@ -57,7 +57,9 @@ constexpr int kP1Slots = 3;   // pass-1 ring (HBM)
 constexpr int kP2Slots = 2;   // pass-2 ring (L2)
 constexpr int kAcc = 4;       // TMEM accumulators per pass
 constexpr int kQBufs = 3;     // query-row buffers: pass 1 runs up to two items ahead of pass 2
-constexpr double kMaxLog2 = 1010.0;  // |log2| of a column's largest term that fp64 can hold
+// Largest |log2| of an item's column maximum: an item's sum is then below 2^1000 (at most
+// 2^10 keys), and the sum of up to 2^20 items stays below fp64's 2^1024.
+constexpr double kMaxLog2 = 990.0;
 
 struct alignas(128) LayersParams {
     CUtensorMap tmap_k[kMaxLaunchLayers];  // K of each layer: {128, H_kv, T}, box {64, 1, 128}
