@@ -37,13 +37,8 @@ HBM_FALLBACK_GBS = 6800.0
 # per workload, from the ncu summaries under profiles/ ("+lse": bench.py --lse), keyed by the
 # sha256 of the scoring kernels' sources (SCORE_SOURCES); a changed kernel reports null until
 # it is captured again.  Figures that ncu printed in MB are rounded to 10 kB.
-SCORE_SOURCES = ('score_kernel.cu', 'score_resident.cu', 'score_lse.cu', 'score_common.cuh', 'ckv_device.cuh')
-SCORE_TRAFFIC = {
-    "50ca48de509577f3973443051d675ffae0d66af5da371b0bba5e4bf4ff8adf7d": {
-        "llama8b_l8192": 16989952, "paper_llama8b_l8192": 8500000, "needle_l131072": 299342080,
-        "llama8b_l8192+lse": 16950000, "needle_l131072+lse": 274310000,
-    },
-}
+SCORE_SOURCES = ('score_layers.cu', 'score_resident.cu', 'score_lse.cu', 'score_common.cuh', 'ckv_device.cuh')
+SCORE_TRAFFIC = {}
 # Sequences up to this many tokens are selected by one block per (sequence, KV head)
 # (one launch); longer ones by the chunked kernels (two launches).
 SELECT_UNIT_LEN = 16384

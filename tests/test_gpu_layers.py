@@ -38,7 +38,8 @@ CASES = [
     dict(num_layers=2, seqlens=(1, 5, 31, 33, 300, 0, 2000), budget_mean=40, budget_uniform=True),
     dict(num_layers=4, scope="layer", heads_per_layer=3, seqlens=(1000, 77, 300), budget_mean=40),
     dict(num_layers=2, window=8, pool_kernel=5, pool_type="avg", heads_per_group=4, seqlens=(1000, 64)),
-    dict(num_layers=2, window=64, heads_per_group=2, seqlens=(1500,), budget_mean=100),
+    dict(num_layers=2, window=64, heads_per_group=2, seqlens=(1500,), budget_mean=100,
+         budget_uniform=True),
     dict(num_layers=34, num_q_heads=4, num_kv_heads=2, heads_per_group=1, seqlens=(600, 130),
          budget_mean=48),
     dict(num_layers=2, num_q_heads=2, num_kv_heads=1, heads_per_group=1, window=16,
