@@ -241,7 +241,7 @@ CKV_API ckv_status ckv_workspace_size_layers(const ckv_config* cfg, int32_t n_la
 
 /* Step 1 for several layers at once: for each io[i], what ckv_score_window(cfg, io[i].layer,
  * ...) writes to io[i].scores.  Every layer's two passes run in one persistent launch (one per
- * 32 layers, and per 512 sequences), so the GPU streams one layer's keys while it exchanges
+ * 32 layers, and per 256 sequences), so the GPU streams one layer's keys while it exchanges
  * another's row statistics; the per-call start and tail are paid once.  Always the two-pass
  * kernel that re-reads K in pass 2 (cfg->score_path is ignored).  cfg->max_ctas caps the CTAs
  * of the launch (0 = all SMs), which leaves the other SMs to work issued on other streams. */
@@ -350,7 +350,7 @@ CKV_API ckv_status ckv_read_device_status(void* workspace, ckv_stream stream, in
  *   - Calls whose work needs more scratch than the array holds return CKV_ERR_UNSUPPORTED
  *     before enqueuing anything: on the resident kernel more than CKV_STATIC_SCRATCH_ITEMS
  *     work items over the call; on the two-pass kernel more than CKV_STATIC_SCRATCH_UNITS
- *     (head batch, sequence) units in one launch, which takes up to 512 sequences.
+ *     (head batch, sequence) units in one launch, which takes up to 256 sequences.
  *     ckv_score_window has no such limit.
  *   - Every call shares the one array: calls that may overlap on the GPU (other streams,
  *     other host threads) race and must be serialised by the caller.
@@ -360,7 +360,7 @@ CKV_API ckv_status ckv_read_device_status(void* workspace, ckv_stream stream, in
  *   - Allocates nothing: no cudaMalloc, cudaFree or allocating library call. */
 #define CKV_STATIC_SCRATCH_ITEMS 1024
 #define CKV_STATIC_SCRATCH_UNITS 1024
-#define CKV_STATIC_SCRATCH_BYTES (256 + CKV_STATIC_SCRATCH_ITEMS * 64 * 8 + 4096)
+#define CKV_STATIC_SCRATCH_BYTES (256 + CKV_STATIC_SCRATCH_ITEMS * 64 * 8 + 8192)
 CKV_API ckv_status ckv_score_window_static(const ckv_config* cfg, int32_t layer,
                                            const ckv_batch* batch, const void* q_win,
                                            const void* k, int64_t tok_stride,

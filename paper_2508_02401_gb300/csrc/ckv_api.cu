@@ -400,8 +400,8 @@ WsLayout ws_layout(const Plan& pl, const ckv_batch* b, int T) {
     const size_t score_units = static_cast<size_t>(pl.nb) * b->num_seqs;
     l.sums = off;
     off = round_up(off + score_units * kMaxCols * sizeof(double), kWsAlign);
-    l.unit_counters = off;
-    off = round_up(off + score_units * sizeof(int), kWsAlign);
+    l.unit_counters = off;  // and, after them, the kernel's item counter
+    off = round_up(off + (score_units + 1) * sizeof(int), kWsAlign);
     l.scores = off;
     off = round_up(off + static_cast<size_t>(pl.n_sel) * T * sizeof(float), kWsAlign);
     l.pooled = off;
@@ -529,13 +529,40 @@ struct LayerJob {
     float* scores;
 };
 
-constexpr int kMinItemTiles = 4;  // shortest work item, in key tiles
+// The items of one launch of the two-pass kernel: unit (lb, s), of tiles[s] key tiles, is
+// split into m = ceil(tiles / c) items of balanced length, unit after unit (head batch major);
+// `units` ends with an entry holding the total.  c is kItemTiles, or more where a unit would
+// otherwise have more items than the launch has CTAs (the kernel's progress argument needs at
+// most G).  Short items let the faster SMs take more of the work and keep the tiles that pass
+// 2 re-reads few enough to stay in L2.
+constexpr int kItemTiles = 8;
+void plan_items(const std::vector<int>& tiles, int n_lb, int G, std::vector<LaunchUnit>& units) {
+    units.clear();
+    int max_tiles = 0;
+    for (int t : tiles) max_tiles = std::max(max_tiles, t);
+    const int c = std::max(kItemTiles, (max_tiles + G - 1) / G);
+    int item = 0;
+    for (int lb = 0; lb < n_lb; ++lb)
+        for (int s = 0; s < static_cast<int>(tiles.size()); ++s) {
+            const int t = tiles[s];
+            if (t == 0) continue;
+            units.push_back(LaunchUnit{static_cast<int16_t>(lb), static_cast<int16_t>(s), item});
+            item += std::min(t, (t + c - 1) / c);
+        }
+    units.push_back(LaunchUnit{0, 0, item});
+}
+
+// Sequences per launch of the two-pass kernel when a layer has up to max_nb head batches: one
+// layer's units of one chunk always fit a launch's unit table.
+int launch_seq_chunk(int max_nb) {
+    return std::max(1, std::min(kMaxLaunchSeqs, kMaxLaunchUnits / std::max(1, max_nb)));
+}
 
 // Enqueues the two-pass scoring of `jobs` (layers sharing the batch and the window): one
-// persistent launch per group of consecutive layers and per chunk of up to kMaxLaunchSeqs
-// sequences whose tables fit the kernel's parameters.  Sequences of at most skip_le tokens are
-// skipped.  `sums`/`counters` hold the exchange of every (head batch, sequence) unit of one
-// launch (each launch clears them first; launches are ordered on `stream`).
+// persistent launch per chunk of sequences (launch_seq_chunk) and per group of consecutive
+// layers whose tables fit the kernel's parameters.  Sequences of at most skip_le tokens are
+// skipped.  `sums`/`counters` hold the exchange of every unit of one launch (each launch
+// clears them first; launches are ordered on `stream`).
 ckv_status enqueue_layers(const std::vector<LayerJob>& jobs, const ckv_batch* b, int T, void* sums,
                           int* counters, int* status, int skip_le, int max_ctas, cudaStream_t stream) {
     if (jobs.empty()) return CKV_OK;
@@ -543,71 +570,71 @@ ckv_status enqueue_layers(const std::vector<LayerJob>& jobs, const ckv_batch* b,
     if (ctas <= 0) return cuda_fail(cudaGetLastError(), "querying the SM count");
     if (max_ctas > 0) ctas = std::min(ctas, max_ctas);
     const int S = b->num_seqs;
-    int max_tiles = 0;
-    for (int s = 0; s < S; ++s) {
-        const int len = b->cu_seqlens_host[s + 1] - b->cu_seqlens_host[s];
-        if (len > skip_le && len > 0) max_tiles = std::max(max_tiles, (len + kTileKeys - 1) / kTileKeys);
-    }
-    if (max_tiles == 0) return CKV_OK;
-    // Items of c tiles, with at most `ctas` items per unit: a unit's items then lie in at most
-    // three consecutive rounds of the launch, which the kernel's two-item lead of pass 1 covers.
-    const int c = std::max(kMinItemTiles, (max_tiles + ctas - 1) / ctas);
     const int w_pad = jobs[0].pl->w_pad, w = jobs[0].pl->w;
     static thread_local LayersLaunch L;
     const uint32_t hash = seqlens_hash(b->cu_seqlens_host, S);
-    size_t j0 = 0;
-    while (j0 < jobs.size()) {
-        // the layers of this launch: as many as the parameter tables hold
-        size_t j1 = j0;
-        int nb = 0, nsel = 0, n_cols = 32;
-        while (j1 < jobs.size() && static_cast<int>(j1 - j0) < kMaxLaunchLayers &&
-               nb + jobs[j1].pl->nb <= kMaxLaunchBatches && nsel + jobs[j1].pl->n_sel <= kMaxLaunchSel) {
-            nb += jobs[j1].pl->nb;
-            nsel += jobs[j1].pl->n_sel;
-            n_cols = std::max(n_cols, jobs[j1].pl->n_cols);
-            ++j1;
+    std::vector<int> tiles;
+    int max_nb = 1;
+    for (const LayerJob& J : jobs) max_nb = std::max(max_nb, J.pl->nb);
+    const int chunk = launch_seq_chunk(max_nb);
+    for (int s0 = 0; s0 < S; s0 += chunk) {  // chunks of sequences
+        const int s1 = std::min(S, s0 + chunk);
+        tiles.clear();
+        L.seq_start.clear();
+        L.seq_len.clear();
+        int active = 0;
+        for (int s = s0; s < s1; ++s) {
+            const int len = b->cu_seqlens_host[s + 1] - b->cu_seqlens_host[s];
+            const int t = len > skip_le && len > 0 ? (len + kTileKeys - 1) / kTileKeys : 0;
+            if (t > 32767) return fail(CKV_ERR_UNSUPPORTED, "a sequence of more than 2^22 tokens");
+            tiles.push_back(t);
+            active += t > 0;
+            L.seq_start.push_back(b->cu_seqlens_host[s]);
+            L.seq_len.push_back(len);
         }
-        if (j1 == j0) return fail(CKV_ERR_UNSUPPORTED, "a layer has more head batches than one launch holds");
-        L.layers.clear();
-        L.batch_layer.clear();
-        L.batch_group.clear();
-        L.batch_first.clear();
-        L.batch_nheads.clear();
-        L.batch_sel.clear();
-        L.sel_heads.clear();
-        for (size_t j = j0; j < j1; ++j) {
-            const LayerJob& J = jobs[j];
-            LayersLayer ly;
-            ckv_status st;
-            if ((st = make_k_map(&ly.tmap_k, J.k, J.pl->Hkv, T, J.tok, J.head))) return st;
-            if ((st = make_q_map(&ly.tmap_q, J.q_win, J.pl->Hq, S, w, w_pad))) return st;
-            ly.scores = J.scores;
-            const int sel_base = static_cast<int>(L.sel_heads.size());
-            for (int bt = 0; bt < J.pl->nb; ++bt) {
-                L.batch_layer.push_back(static_cast<int16_t>(j - j0));
-                L.batch_group.push_back(static_cast<int16_t>(J.pl->batch_group[bt]));
-                L.batch_first.push_back(static_cast<int16_t>(J.pl->batch_first[bt]));
-                L.batch_nheads.push_back(static_cast<int16_t>(J.pl->batch_nheads[bt]));
-                L.batch_sel.push_back(static_cast<int16_t>(sel_base + J.pl->batch_first[bt]));
+        if (active == 0) continue;
+        size_t j0 = 0;
+        while (j0 < jobs.size()) {
+            // the layers of this launch: as many as the parameter tables hold
+            size_t j1 = j0;
+            int nb = 0, nsel = 0, n_cols = 32;
+            while (j1 < jobs.size() && static_cast<int>(j1 - j0) < kMaxLaunchLayers &&
+                   nb + jobs[j1].pl->nb <= kMaxLaunchBatches &&
+                   nsel + jobs[j1].pl->n_sel <= kMaxLaunchSel &&
+                   (nb + jobs[j1].pl->nb) * active <= kMaxLaunchUnits) {
+                nb += jobs[j1].pl->nb;
+                nsel += jobs[j1].pl->n_sel;
+                n_cols = std::max(n_cols, jobs[j1].pl->n_cols);
+                ++j1;
             }
-            for (int h : J.pl->sel_heads) L.sel_heads.push_back(static_cast<int16_t>(h));
-            L.layers.push_back(ly);
-        }
-        for (int s0 = 0; s0 < S; s0 += kMaxLaunchSeqs) {  // chunks of sequences
-            const int s1 = std::min(S, s0 + kMaxLaunchSeqs);
-            L.seq_start.clear();
-            L.seq_len.clear();
-            L.seq_item0.assign(1, 0);
-            for (int s = s0; s < s1; ++s) {
-                const int len = b->cu_seqlens_host[s + 1] - b->cu_seqlens_host[s];
-                const int tiles = len > skip_le && len > 0 ? (len + kTileKeys - 1) / kTileKeys : 0;
-                L.seq_start.push_back(b->cu_seqlens_host[s]);
-                L.seq_len.push_back(len);
-                L.seq_item0.push_back(L.seq_item0.back() + (tiles + c - 1) / c);
+            if (j1 == j0)
+                return fail(CKV_ERR_UNSUPPORTED, "a layer's head batches and sequences exceed one launch's tables");
+            L.layers.clear();
+            L.batch_layer.clear();
+            L.batch_group.clear();
+            L.batch_first.clear();
+            L.batch_nheads.clear();
+            L.batch_sel.clear();
+            L.sel_heads.clear();
+            for (size_t j = j0; j < j1; ++j) {
+                const LayerJob& J = jobs[j];
+                LayersLayer ly;
+                ckv_status st;
+                if ((st = make_k_map(&ly.tmap_k, J.k, J.pl->Hkv, T, J.tok, J.head))) return st;
+                if ((st = make_q_map(&ly.tmap_q, J.q_win, J.pl->Hq, S, w, w_pad))) return st;
+                ly.scores = J.scores;
+                const int sel_base = static_cast<int>(L.sel_heads.size());
+                for (int bt = 0; bt < J.pl->nb; ++bt) {
+                    L.batch_layer.push_back(static_cast<int16_t>(j - j0));
+                    L.batch_group.push_back(static_cast<int16_t>(J.pl->batch_group[bt]));
+                    L.batch_first.push_back(static_cast<int16_t>(J.pl->batch_first[bt]));
+                    L.batch_nheads.push_back(static_cast<int16_t>(J.pl->batch_nheads[bt]));
+                    L.batch_sel.push_back(static_cast<int16_t>(sel_base + J.pl->batch_first[bt]));
+                }
+                for (int h : J.pl->sel_heads) L.sel_heads.push_back(static_cast<int16_t>(h));
+                L.layers.push_back(ly);
             }
-            if (L.seq_item0.back() == 0) continue;
-            if (static_cast<int64_t>(L.seq_item0.back()) * nb > INT32_MAX)
-                return fail(CKV_ERR_UNSUPPORTED, "too many scoring work items");
+            plan_items(tiles, nb, ctas, L.units);
             L.seq0 = s0;
             L.S_all = S;
             L.cu_seqlens_dev = b->cu_seqlens_dev;
@@ -618,14 +645,13 @@ ckv_status enqueue_layers(const std::vector<LayerJob>& jobs, const ckv_batch* b,
             L.w = w;
             L.w_pad = w_pad;
             L.n_cols = n_cols;
-            L.c = c;
             L.grid = ctas;
             L.cu_hash = hash;
             L.softmax_scale = jobs[j0].pl->scale;
             const cudaError_t e = launch_score_layers(L, stream);
             if (e != cudaSuccess) return cuda_fail(e, "launching the two-pass scoring kernel");
+            j0 = j1;
         }
-        j0 = j1;
     }
     return CKV_OK;
 }
@@ -1102,8 +1128,8 @@ namespace {
 // unit of the call's layers, then each layer's scores (ckv_compress_layers).
 struct LayersWs {
     WsLayout sel;
-    size_t sums = 0, counters = 0, total = 0;
-    std::vector<size_t> scores;
+    size_t sums = 0, counters = 0, next_unit = 0, total = 0;
+    std::vector<size_t> scores, keys;  // per layer (ckv_compress_layers)
 };
 
 ckv_status prepare_layers(const ckv_config* cfg, int32_t n_layers, const ckv_layer_io* io,
@@ -1126,12 +1152,17 @@ ckv_status prepare_layers(const ckv_config* cfg, int32_t n_layers, const ckv_lay
     size_t off = round_up(lw->sel.total, kWsAlign);
     lw->sums = off;
     off = round_up(off + units * kMaxCols * sizeof(double), kWsAlign);
-    lw->counters = off;
-    off = round_up(off + units * sizeof(int), kWsAlign);
+    lw->counters = off;  // and, after them, the kernel's item counter
+    off = round_up(off + (units + 1) * sizeof(int), kWsAlign);
+    lw->next_unit = off;  // the selection kernel's work counter
+    off = round_up(off + sizeof(int), kWsAlign);
     lw->scores.assign(n_layers, 0);
+    lw->keys.assign(n_layers, 0);
     for (int i = 0; i < n_layers; ++i) {
         lw->scores[i] = off;
         off = round_up(off + static_cast<size_t>(pls[i].n_sel) * *T * sizeof(float), kWsAlign);
+        lw->keys[i] = off;  // the selection's keys of the pooled scores, [n_vec, T]
+        off = round_up(off + static_cast<size_t>(pls[i].n_vec) * *T * sizeof(uint32_t), kWsAlign);
     }
     lw->total = off;
     return CKV_OK;
@@ -1231,13 +1262,35 @@ ckv_status ckv_compress_layers(const ckv_config* cfg, int32_t n_layers, const ck
     if ((st = enqueue_layers(jobs, batch, T, w8 + lw.sums, reinterpret_cast<int*>(w8 + lw.counters),
                              reinterpret_cast<int*>(w8), min_budget, cfg->max_ctas, s)))
         return st;
-    WsLayout sel = lw.sel;
-    for (int i = 0; i < n_layers; ++i)
-        if ((st = enqueue_select_fused(pls[i], cfg, batch, T, jobs[i].scores, io[i].k, io[i].v, tok[i],
-                                       head[i], io[i].idx, io[i].cu_keep_dev, io[i].k_out, io[i].v_out,
-                                       io[i].pooled_out, workspace, sel, tks[i], s)))
-            return st;
-    return CKV_OK;
+    // every layer's selection in one launch (one per 32 layers)
+    static thread_local std::vector<SelectLaunch> sls;
+    static thread_local std::vector<uint32_t*> keys;
+    sls.assign(n_layers, SelectLaunch{});
+    keys.assign(n_layers, nullptr);
+    for (int i = 0; i < n_layers; ++i) {
+        SelectLaunch& L = sls[i];
+        L = select_launch(pls[i], batch, T, static_cast<int>(tks[i]), pls[i].budget, cfg, workspace, &lw.sel);
+        L.scores = jobs[i].scores;
+        L.pooled = io[i].pooled_out;
+        L.write_pooled = io[i].pooled_out != nullptr;
+        L.from_scores = 1;
+        L.idx = io[i].idx;
+        L.cu_keep_dev = io[i].cu_keep_dev;
+        if (tks[i] > 0) {
+            L.k = io[i].k;
+            L.v = io[i].v;
+            L.tok_stride = tok[i];
+            L.head_stride = head[i];
+            L.k_out = io[i].k_out;
+            L.v_out = io[i].v_out;
+        }
+        keys[i] = reinterpret_cast<uint32_t*>(w8 + lw.keys[i]);
+    }
+    const int sms = device_sm_count();
+    if (sms <= 0) return cuda_fail(cudaGetLastError(), "querying the SM count");
+    const cudaError_t e = launch_select_layers(sls.data(), keys.data(), n_layers,
+                                               reinterpret_cast<int*>(w8 + lw.next_unit), sms, s);
+    return e == cudaSuccess ? CKV_OK : cuda_fail(e, "launching the multi-layer selection kernel");
 }
 
 ckv_status ckv_semantic_retrieval_scores(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,
@@ -1354,8 +1407,8 @@ ckv_status ckv_score_window_static(const ckv_config* cfg, int32_t layer, const c
                         "(use ckv_score_window with a workspace)", n_items, CKV_STATIC_SCRATCH_ITEMS);
     } else {
         // The two-pass kernel's exchange: one fp64 sum per column and a counter per (head
-        // batch, sequence) unit of a launch (a launch takes up to kMaxLaunchSeqs sequences).
-        const int units = pl.nb * std::min(batch->num_seqs, kMaxLaunchSeqs);
+        // batch, sequence) unit of a launch (a launch takes launch_seq_chunk sequences).
+        const int units = pl.nb * std::min(batch->num_seqs, launch_seq_chunk(pl.nb));
         if (units > CKV_STATIC_SCRATCH_UNITS)
             return fail(CKV_ERR_UNSUPPORTED,
                         "this batch needs %d scratch units; the static scratch holds %d "

@@ -64,11 +64,19 @@ struct ScoreLaunch {
 cudaError_t launch_score(const ScoreLaunch& L, cudaStream_t stream);
 
 // Multi-layer scoring (score_layers.cu): both passes, K re-read from L2 in pass 2, every unit
-// of every layer of the launch in one persistent cooperative kernel.
+// of every layer of the launch in one persistent cooperative kernel.  A unit is (head batch,
+// sequence); its key tiles are split into m items of balanced length (m at most the launch's
+// CTAs), and the CTAs take the items, unit after unit, from a global counter.
 constexpr int kMaxLaunchLayers = 32;
-constexpr int kMaxLaunchBatches = 512;   // head batches over the launch's layers
-constexpr int kMaxLaunchSel = 1024;      // head slots over the launch's layers
-constexpr int kMaxLaunchSeqs = 512;
+constexpr int kMaxLaunchBatches = 256;   // head batches over the launch's layers
+constexpr int kMaxLaunchSel = 512;       // head slots over the launch's layers
+constexpr int kMaxLaunchSeqs = 256;
+constexpr int kMaxLaunchUnits = 1536;
+struct LaunchUnit {
+    int16_t lb;      // flat head batch
+    int16_t seq;     // sequence within the launch
+    int32_t item0;   // first item; the unit's m items are item0 .. next unit's item0 - 1
+};
 struct LayersLayer {
     CUtensorMap tmap_k;
     CUtensorMap tmap_q;
@@ -79,13 +87,14 @@ struct LayersLaunch {
     // flat over the layers' head batches, in layer order
     std::vector<int16_t> batch_layer, batch_group, batch_first, batch_nheads, batch_sel;
     std::vector<int16_t> sel_heads;  // query head of each head slot, batch after batch
-    std::vector<int32_t> seq_start, seq_len, seq_item0;  // [S], [S], [S+1] of sequences seq0 ...
+    std::vector<int32_t> seq_start, seq_len;   // [S] of the launch's sequences seq0 ...
+    std::vector<LaunchUnit> units;             // unit after unit, then one entry closing the table
     int seq0, S_all;     // the launch's first sequence; sequences in the batch (for the hash)
     const int32_t* cu_seqlens_dev;
-    double* sums;        // [batches * S][n_cols]
-    int* counters;       // [batches * S]
+    double* sums;        // [units][n_cols]
+    int* counters;       // [units + 1]: arrivals per unit, then the item counter
     int* status;
-    int T, w, w_pad, n_cols, c, grid;
+    int T, w, w_pad, n_cols, grid;
     uint32_t cu_hash;
     float softmax_scale;
 };
@@ -128,6 +137,11 @@ int select_chunk_positions();
 int select_unit_len();  // units up to this length take the one-block path
 cudaError_t launch_pool(const SelectLaunch& L, cudaStream_t stream);
 cudaError_t launch_select(const SelectLaunch& L, cudaStream_t stream);
+// The selections of several layers (one SelectLaunch each, pooling from their scores) in one
+// launch per 32 layers: keys[i] is a [n_vec, T] uint32 scratch of layer i, next_unit a work
+// counter (cleared by the call).
+cudaError_t launch_select_layers(const SelectLaunch* Ls, uint32_t* const* keys, int n_layers,
+                                 int* next_unit, int grid, cudaStream_t stream);
 
 struct GatherLaunch {
     const void* k;

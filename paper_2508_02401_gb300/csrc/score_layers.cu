@@ -8,39 +8,43 @@
 // probability can be summed over rows, so each key tile is used twice: once for the row
 // statistics (pass 1, from HBM), once for the probabilities (pass 2, from L2).
 //
-// Work: a unit is (layer, head batch of one KV group, sequence); its key tiles are cut into
-// items of at most c tiles.  The items of all units, unit after unit, form one sequence that
-// the CTAs take round-robin (CTA b: items b, b + G, b + 2G, ...), so every CTA streams its
-// share of every unit and a unit's items are spread over consecutive CTAs.  The host picks c
-// so that a unit has at most G items: its items then lie in at most three consecutive rounds,
-// and since pass 1 may run up to two items ahead of pass 2 in every CTA, every unit's pass 1
-// completes before any CTA needs that unit's normalisers (no wait can close a cycle).
+// Work: a unit is (layer, head batch of one KV group, sequence); its key tiles are split into
+// m items of balanced length, m at most the CTAs of the launch.  The items of all units, unit
+// after unit, form one sequence; the CTAs take them dynamically, one at a time, from a global
+// counter, as each CTA becomes ready to start one (its query buffer is free).  The SMs do not
+// stream HBM equally fast, and taking items on demand lets the faster ones take more, so that
+// a unit's items finish close together and pass 2 re-reads its tiles while they are still in
+// L2.  No wait can close a cycle: a CTA waits only for units it holds an item of, a unit's
+// items are taken before any later unit's, and a CTA takes an item only when it can run its
+// pass 1 (up to two items ahead of its pass 2); if a unit's items were all held by CTAs that
+// cannot start them, each would hold three of the unit's items, more than the G it has.
 //
-// Exchange: at the end of an item, pass 1 adds, per window-row column, its keys' sum
-// sum_j 2^(x_j) (x = logit * log2 e, as s * 2^m with the item's maximum m) in fp64 to the
-// unit's accumulator with one atomic add, and one arrival per pass-1 warpgroup is counted on
-// the unit's counter.  A unit's lse per column is log2 of its accumulator once the counter is
-// complete: one read of N doubles, whatever the number of items.  fp64 holds 2^(+-1022), so
-// a column's largest logit must lie within +-680 (natural log units); beyond that the status
-// word reports kDevRange.
+// Exchange: at the end of an item, pass 1 leaves, per window-row column, its keys' sum
+// sum_j 2^(x_j) (x = logit * log2 e) as (m, s) with the item's maximum m in shared memory; a
+// publisher warp adds each s * 2^m in fp64 to the unit's accumulator with one atomic add and
+// counts the item's arrival on the unit's counter with a release (the wait for its adds to
+// land stays off pass 1's path).  A unit's lse per column is log2 of its accumulator once the
+// counter is complete: one read of N doubles, whatever the number of items.  fp64 holds 2^(+-1022), so a column's largest logit must lie within +-680 (natural
+// log units); beyond that the status word reports kDevRange.
 //
 // One cooperative launch, one CTA per SM, 512 threads, warp-specialised:
-//   warp 0       TMA producer for both passes, one polling thread: per item, TMA loads of the
-//                window query rows into one of kQBufs buffers, then of its 128-key x 128-dim
-//                bf16 K tiles (two 128-byte-swizzled boxes of 64 dims) into the pass-1 ring
-//                (evict-last: pass 2 reads them again soon); the same tiles again into the
-//                pass-2 ring (evict-first) once the item's pass-1 loads are out;
+//   warp 0       the producer, one polling thread: takes the CTA's next item from the global
+//                counter and posts it to the other roles (a ring of item indices in shared
+//                memory); per item, TMA loads of the window query rows into one of kQBufs
+//                buffers, then of its 128-key x 128-dim bf16 K tiles (two 128-byte-swizzled
+//                boxes of 64 dims) into the pass-1 ring (evict-last: pass 2 reads them again
+//                soon); the same tiles again into the pass-2 ring (evict-first) once the
+//                item's pass-1 loads are out;
 //   warp 1       allocates TMEM and issues the pass-1 tcgen05.mma (M = 128 keys, N = the
 //                window rows of a head batch, K = 128) into four pass-1 accumulators;
 //   warp 2       issues the pass-2 tcgen05.mma into four pass-2 accumulators;
-//   warp 3       publisher: once an item's pass-1 sums are added, one release on the unit's
-//                counter; then a bounded acquire spin until the unit is complete and the
-//                unit's -lse per column into shared memory for pass 2, which meanwhile still
-//                works on the item before;
+//   warp 3       the publisher: per item, the fp64 atomic adds of its column sums and the
+//                release of its arrival on the unit's counter;
 //   warps 4-11   pass 1, one warpgroup per 32 columns: each thread owns one key (one TMEM
 //                lane) and keeps a running (max, sum of 2^(x - max)) per column;
-//   warps 12-15  pass 2, one warpgroup over all N columns: sums 2^(x - lse) over each head's
-//                rows per key and writes the scores.
+//   warps 12-15  pass 2, one warpgroup over all N columns: per item, a bounded acquire spin
+//                until the item's unit is complete and the unit's -lse per column from its
+//                accumulator, then per key the sums of 2^(x - lse) over each head's rows.
 // Only the last tiles of a sequence (the window's own keys, the padding past its end) need a
 // per-column mask; the others take an unmasked path of packed fp32 pair instructions.
 #include "score_common.cuh"
@@ -57,6 +61,7 @@ constexpr int kP1Slots = 3;   // pass-1 ring (HBM)
 constexpr int kP2Slots = 2;   // pass-2 ring (L2)
 constexpr int kAcc = 4;       // TMEM accumulators per pass
 constexpr int kQBufs = 3;     // query-row buffers: pass 1 runs up to two items ahead of pass 2
+constexpr int kItemRing = 8;  // item indices posted by the producer (more than any role's lag)
 // Largest |log2| of an item's column maximum: an item's sum is then below 2^1000 (at most
 // 2^10 keys), and the sum of up to 2^20 items stays below fp64's 2^1024.
 constexpr double kMaxLog2 = 990.0;
@@ -67,9 +72,9 @@ struct alignas(128) LayersParams {
     float* scores[kMaxLaunchLayers];       // [n_sel of the layer, T]
     const int32_t* cu_seqlens;             // device [S+1] (checked against cu_hash)
     double* sums;                          // [n_units][N]: per column, sum of 2^(x) over the unit
-    int* counters;                         // [n_units] arrivals, zero at launch
+    int* counters;                         // [n_units] arrivals, then the item counter; zero at launch
     int* status;
-    int S, T, w, n_items, items_per_lb, c, n_layers;
+    int S, T, w, n_units, n_items, n_layers;
     int seq0, S_all;                       // the launch's first sequence, sequences of the batch
     uint32_t cu_hash;
     float sl2;                             // softmax scale * log2(e)
@@ -82,7 +87,7 @@ struct alignas(128) LayersParams {
     int16_t sel_heads[kMaxLaunchSel];         // query head of each head slot
     int32_t seq_start[kMaxLaunchSeqs];        // of the launch's sequences seq0, seq0 + 1, ...
     int32_t seq_len[kMaxLaunchSeqs];
-    int32_t seq_item0[kMaxLaunchSeqs + 1];    // first item of each sequence within a head batch
+    LaunchUnit units[kMaxLaunchUnits + 1];    // units[n_units].item0 = n_items
 };
 static_assert(sizeof(LayersParams) <= 32000, "kernel parameters");
 
@@ -90,27 +95,29 @@ struct Item {
     int layer, batch, seq, unit, tile0, ntiles, start, len, nitems;
 };
 
-// Work item i of the launch: head batch i / M, then the sequence whose items hold i % M.
+// Item i of the launch: the unit whose items hold i, and the (i - item0)-th of its m balanced
+// pieces of key tiles.
 __device__ __forceinline__ Item get_item(const LayersParams& p, int i) {
     Item it;
-    const int lb = i / p.items_per_lb;
-    const int r = i - lb * p.items_per_lb;
-    int lo = 0, hi = p.S - 1;  // the last sequence whose first item is at or before r
+    int lo = 0, hi = p.n_units - 1;  // the last unit whose first item is at or before i
     while (lo < hi) {
         const int mid = (lo + hi + 1) >> 1;
-        if (p.seq_item0[mid] <= r) lo = mid;
+        if (p.units[mid].item0 <= i) lo = mid;
         else hi = mid - 1;
     }
-    it.batch = lb;
-    it.layer = p.batch_layer[lb];
-    it.seq = lo;
-    it.unit = lb * p.S + lo;
-    it.start = p.seq_start[lo];
-    it.len = p.seq_len[lo];
-    it.nitems = p.seq_item0[lo + 1] - p.seq_item0[lo];
-    it.tile0 = (r - p.seq_item0[lo]) * p.c;
+    const LaunchUnit U = p.units[lo];
+    const int m = p.units[lo + 1].item0 - U.item0;
+    const int k = i - U.item0;
+    it.unit = lo;
+    it.batch = U.lb;
+    it.layer = p.batch_layer[U.lb];
+    it.seq = U.seq;
+    it.start = p.seq_start[U.seq];
+    it.len = p.seq_len[U.seq];
+    it.nitems = m;
     const int tiles = (it.len + kTileKeys - 1) / kTileKeys;
-    it.ntiles = min(p.c, tiles - it.tile0);
+    it.tile0 = k * tiles / m;
+    it.ntiles = (k + 1) * tiles / m - it.tile0;
     return it;
 }
 
@@ -129,26 +136,36 @@ struct LayersSmem {
                          kQFull = kBEmpty + kAcc, kQEmpty = kQFull + kQBufs,
                          kDone = kQEmpty + kQBufs, kGroup = kDone + 2,  // A0 A1 B
                          kPubFull = kGroup + 3, kPubEmpty = kPubFull + 2,
-                         kLseFull = kPubEmpty + 2, kLseEmpty = kLseFull + 2,
-                         kNumBars = kLseEmpty + 2;
-    static constexpr int kTmemSlot = kBars + 8 * kNumBars;
+                         kItemFull = kPubEmpty + 2, kItemFree = kItemFull + kItemRing,
+                         kNumBars = kItemFree + kItemRing;
+    static constexpr int kItems = kBars + 8 * kNumBars;  // int[kItemRing]: posted item indices
+    static constexpr int kTmemSlot = kItems + 4 * kItemRing;
     static constexpr int kAbort = kTmemSlot + 4;
     static constexpr int kBytes = kAbort + 4;
     static constexpr int kDynamic = kBytes + 1024;      // slack to align the base to 1024 B
 };
-// dynamic + the kernel's static shared memory (under 5 KB) within the 227 KB a block may use
-static_assert(LayersSmem<64>::kDynamic + 5 * 1024 <= 232448, "shared memory, N = 64");
+// dynamic + the kernel's static shared memory (under 6 KB) within the 227 KB a block may use
+static_assert(LayersSmem<64>::kDynamic + 6 * 1024 <= 232448, "shared memory, N = 64");
+
+// The index of the CTA's it-th item (-1 once its stream has ended), after the producer posted
+// it; false if the wait gave up.
+__device__ __forceinline__ bool wait_item(uint64_t* item_full, const int* items, int it, int* gi,
+                                          volatile int* abort, long long lim) {
+    const int k = it % kItemRing;
+    if (!mbar_wait(&item_full[k], (it / kItemRing) & 1, abort, lim)) return false;
+    *gi = items[k];
+    return true;
+}
 
 // End of a pass-1 item for one warpgroup of kCols columns: per column, the warp maximum by
 // redux and the sums rescaled to it, the warps' sums by recursive halving, then the four warps
-// through shared memory `red`; thread c < kCols adds column c's sum, as an fp64 multiple of
-// its maximum's power of two, to the unit's accumulator `sums[c]` once the publisher has
-// released the previous use of this pub_full/pub_empty pair, and arrives on pub_full.
+// through shared memory `red`; thread c < kCols (the warpgroup's first warp) leaves column c's
+// (max, sum) in `out[c]` once the publisher is done with that buffer's previous item, and
+// arrives on pub_full.
 __device__ __forceinline__ bool item_sums(float (&m)[kCols], float (&s)[kCols], float2* red, int eq,
                                           int lane, int wtid, uint64_t* gbar, uint32_t& gphase,
                                           uint64_t* pub_full, uint64_t* pub_empty, uint32_t pub_phase,
-                                          double* sums, int* status, volatile int* abort,
-                                          long long lim) {
+                                          float2* out, volatile int* abort, long long lim) {
 #pragma unroll
     for (int i = 0; i < kCols; ++i) {
         const float M = redux_max(m[i]);
@@ -169,14 +186,18 @@ __device__ __forceinline__ bool item_sums(float (&m)[kCols], float (&s)[kCols], 
             S += x.y * ex2_approx(x.x - M);
         }
         if (!mbar_wait(pub_empty, pub_phase ^ 1, abort, lim)) return false;
-        if (S > 0.f) {
-            if (!(fabs(static_cast<double>(M)) <= kMaxLog2)) record_error(status, kDevRange, wtid);
-            else atomicAdd(sums + wtid, static_cast<double>(S) * exp2(static_cast<double>(M)));
-        }
-        __threadfence();  // the add is performed before the publisher's release below
+        out[wtid] = make_float2(M, S);
         mbar_arrive(pub_full);
     }
     return true;
+}
+
+// s * 2^M as a double, for |M| <= kMaxLog2: the power of two of floor(M) exactly (built from
+// the exponent bits), the rest in fp32.
+__device__ __forceinline__ double scaled_sum(float M, float S) {
+    const float e = floorf(M);
+    const double p2 = __longlong_as_double(static_cast<long long>(static_cast<int>(e) + 1023) << 52);
+    return static_cast<double>(S * ex2_approx(M - e)) * p2;
 }
 
 template <int N, int W_PAD>
@@ -208,18 +229,19 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
     uint64_t* q_empty = bars + SL::kQEmpty;
     uint64_t* done = bars + SL::kDone;
     uint64_t* group = bars + SL::kGroup;        // one per epilogue warpgroup: A0 A1 B
-    uint64_t* pub_full = bars + SL::kPubFull;   // pass-1 sums of an item added (item parity)
-    uint64_t* pub_empty = bars + SL::kPubEmpty;
-    uint64_t* lse_full = bars + SL::kLseFull;   // a unit's lse is in nlse_s[item parity]
-    uint64_t* lse_empty = bars + SL::kLseEmpty; // pass 2 is done with nlse_s[item parity]
+    uint64_t* pub_full = bars + SL::kPubFull;   // pass 1 left an item's sums in pub_s[item parity]
+    uint64_t* pub_empty = bars + SL::kPubEmpty; // the publisher is done with pub_s[item parity]
+    uint64_t* item_full = bars + SL::kItemFull; // items[k] holds the CTA's next item index
+    uint64_t* item_free = bars + SL::kItemFree; // every role has read items[k]
+    int* items = reinterpret_cast<int*>(sm + SL::kItems);
     // scratch of the epilogues (static, so that its accesses are shared-memory instructions)
     __shared__ float2 red_a[2][2][128];  // [item parity][warpgroup][warp * 32 + lane]
-    __shared__ __align__(16) float nlse_s[2][64];  // -lse per column, by item parity
+    __shared__ float2 pub_s[2][64];      // [item parity][column]: (max, sum) of an item
+    __shared__ __align__(16) float nlse_s[64];  // -lse per column of pass 2's item
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + SL::kTmemSlot);
     volatile int* abort = reinterpret_cast<volatile int*>(sm + SL::kAbort);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int G = gridDim.x;
     const int n_items = p.n_items;
 
     if (threadIdx.x == 0) {
@@ -245,10 +267,12 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
         mbar_init(&done[1], 1);
         for (int i = 0; i < 3; ++i) mbar_init(&group[i], kGroupArrivals);
         for (int i = 0; i < 2; ++i) {
-            mbar_init(&pub_full[i], 32 * kNW);
+            mbar_init(&pub_full[i], 32 * kNW);  // the columns' threads of each pass-1 warpgroup
             mbar_init(&pub_empty[i], 1);
-            mbar_init(&lse_full[i], 1);
-            mbar_init(&lse_empty[i], 4);  // one arrival per pass-2 warp
+        }
+        for (int i = 0; i < kItemRing; ++i) {
+            mbar_init(&item_full[i], 1);
+            mbar_init(&item_free[i], 4);  // one arrival per pass-2 warp, once it has read the entry
         }
         *abort = 0;
         fence_mbar_init();
@@ -273,7 +297,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
     tc_fence_after_sync();
     const uint32_t tmem_base = *tmem_slot;
     // Registers: launched at 128 per thread (512 x 128 = 65536); on entry the producer/MMA/
-    // publisher warpgroup gives up to 56, which leaves room for the two pass-1 warpgroups' 160;
+    // lse warpgroup gives up to 56, which leaves room for the two pass-1 warpgroups' 160;
     // the pass-2 warpgroup keeps 128 (128*56 + 256*160 + 128*128 = 64512).
     // Limit of the waits on other roles and other CTAs (the waits for this block's own copies
     // and MMAs before it exits keep the long default, whatever this is).
@@ -282,47 +306,62 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
     if (warp < kWarpA) {
     setmaxnreg_dec<56>();
     if (warp == 0) {
-        // ------------------------------------------------------------ TMA producer
-        // Both rings from one thread that polls: a pass-1 slot still in use must not hold up
-        // a pass-2 load, nor the other way round.
+        // ------------------------------------------------------------ producer
+        // Items, and the tiles of both passes, from one thread that polls: a pass-1 slot still
+        // in use must not hold up a pass-2 load, nor the other way round.
         if (lane == 0) {
             // Pass-1 tiles are read again by pass 2 shortly after: ask L2 to keep them, and to
             // drop them first once pass 2 has read them.
             const uint64_t pol1 = l2_policy_evict_last(), pol2 = l2_policy_evict_first();
-            int i1 = blockIdx.x, jt1 = 0, it1 = 0, use1 = 0;
-            int i2 = blockIdx.x, jt2 = 0, it2 = 0, use2 = 0;
+            int* next_item = p.counters + p.n_units;
+            // The window query rows of an item into query buffer qb (completion on q_full[qb]):
+            // per head of the batch two boxes of 64 dims x W_PAD rows in the MMA's
+            // 128-byte-swizzled layout.  Rows past w (the next sequence's, or zeros past the
+            // end) and head slots past the batch's heads land in columns that the epilogues
+            // mask out.
+            auto load_q = [&](const Item& I, int qb) {
+                uint8_t* qdst = qbuf + qb * SL::kQBytes;
+                const int nheads = p.batch_nheads[I.batch], sel0 = p.batch_sel[I.batch];
+                const CUtensorMap* qm = &p.tmap_q[I.layer];
+                mbar_arrive_expect_tx(&q_full[qb], static_cast<uint32_t>(nheads * W_PAD * 256));
+                const int row = (p.seq0 + I.seq) * p.w;
+                for (int slot = 0; slot < nheads; ++slot) {
+                    const int h = p.sel_heads[sel0 + slot];
+                    uint8_t* d = qdst + slot * W_PAD * 128;
+                    tma_load_3d(d, qm, &q_full[qb], 0, h, row);
+                    tma_load_3d(d + SL::kQHalf, qm, &q_full[qb], 64, h, row);
+                }
+            };
+            // it1: items taken (pass-1 cursor on the last one); it2: pass-2 cursor
+            int it1 = 0, jt1 = 0, use1 = 0, it2 = 0, jt2 = 0, use2 = 0, have2 = -1;
             Item I1{}, I2{};
-            if (i1 < n_items) I1 = I2 = get_item(p, i1);
-            bool q_out = false, ok = true;
+            bool have1 = false, ended = false, ok = true;
             long long t0 = clock64();
             uint32_t idle = 0;
-            while (i1 < n_items || i2 < n_items) {
+            while (true) {
                 bool did = false;
-                if (i1 < n_items) {
-                    if (!q_out) {
-                        // The item's window query rows: per head of the batch two boxes of 64
-                        // dims x W_PAD rows in the MMA's 128-byte-swizzled layout.  Rows past w
-                        // (the next sequence's, or zeros past the end) and head slots past the
-                        // batch's heads land in columns that the epilogues mask out.
-                        const int qb = it1 % kQBufs;
-                        if (mbar_test(&q_empty[qb], ((it1 / kQBufs) & 1) ^ 1)) {
-                            uint8_t* qdst = qbuf + qb * SL::kQBytes;
-                            const int nheads = p.batch_nheads[I1.batch], sel0 = p.batch_sel[I1.batch];
-                            const CUtensorMap* qm = &p.tmap_q[I1.layer];
-                            mbar_arrive_expect_tx(&q_full[qb], static_cast<uint32_t>(nheads * W_PAD * 256));
-                            for (int slot = 0; slot < nheads; ++slot) {
-                                const int h = p.sel_heads[sel0 + slot];
-                                uint8_t* d = qdst + slot * W_PAD * 128;
-                                const int row = (p.seq0 + I1.seq) * p.w;
-                                tma_load_3d(d, qm, &q_full[qb], 0, h, row);
-                                tma_load_3d(d + SL::kQHalf, qm, &q_full[qb], 64, h, row);
-                            }
-                            q_out = true;
-                            did = true;
+                if (!have1 && !ended) {
+                    // Take the next item once its query buffer and its ring entry are free.
+                    const int qb = it1 % kQBufs, k = it1 % kItemRing;
+                    if (mbar_test(&q_empty[qb], ((it1 / kQBufs) & 1) ^ 1) &&
+                        mbar_test(&item_free[k], ((it1 / kItemRing) & 1) ^ 1)) {
+                        const int gi = atomicAdd(next_item, 1);
+                        items[k] = gi < n_items ? gi : -1;
+                        mbar_arrive(&item_full[k]);  // releases items[k] to the other roles
+                        if (gi >= n_items) {
+                            ended = true;
+                        } else {
+                            I1 = get_item(p, gi);
+                            load_q(I1, qb);
+                            have1 = true;
+                            jt1 = 0;
                         }
+                        did = true;
                     }
+                }
+                if (have1) {
                     const int s = use1 % kP1Slots;
-                    if (q_out && mbar_test(&free1[s], ((use1 / kP1Slots) & 1) ^ 1)) {
+                    if (mbar_test(&free1[s], ((use1 / kP1Slots) & 1) ^ 1)) {
                         mbar_arrive_expect_tx(&full1[s], kTileBytes);
                         uint8_t* dst = ring1 + s * kTileBytes;
                         const int g = p.batch_group[I1.batch];
@@ -333,16 +372,17 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
                         ++use1;
                         did = true;
                         if (++jt1 == I1.ntiles) {
-                            jt1 = 0;
+                            have1 = false;
                             ++it1;
-                            q_out = false;
-                            i1 += G;
-                            if (i1 < n_items) I1 = get_item(p, i1);
                         }
                     }
                 }
                 // pass 2 of an item follows its pass-1 loads, so that it reads L2
-                if (i2 < n_items && it2 < it1) {
+                if (it2 < it1) {
+                    if (have2 != it2) {
+                        I2 = get_item(p, items[it2 % kItemRing]);
+                        have2 = it2;
+                    }
                     const int s = use2 % kP2Slots;
                     if (mbar_test(&free2[s], ((use2 / kP2Slots) & 1) ^ 1)) {
                         mbar_arrive_expect_tx(&full2[s], kTileBytes);
@@ -357,11 +397,10 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
                         if (++jt2 == I2.ntiles) {
                             jt2 = 0;
                             ++it2;
-                            i2 += G;
-                            if (i2 < n_items) I2 = get_item(p, i2);
                         }
                     }
                 }
+                if (ended && !have1 && it2 == it1) break;
                 if (did) {
                     idle = 0;
                     t0 = clock64();
@@ -383,7 +422,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
                 mbar_wait(&full1[k % kP1Slots], (k / kP1Slots) & 1, &never);
             for (int k = (use2 > kP2Slots ? use2 - kP2Slots : 0); k < use2; ++k)
                 mbar_wait(&full2[k % kP2Slots], (k / kP2Slots) & 1, &never);
-            const int nq = it1 + (q_out ? 1 : 0);
+            const int nq = it1 + (have1 ? 1 : 0);
             for (int k = (nq > kQBufs ? nq - kQBufs : 0); k < nq; ++k)
                 mbar_wait(&q_full[k % kQBufs], (k / kQBufs) & 1, &never);
         }
@@ -400,10 +439,16 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
             uint64_t* acc_empty = first ? a_empty : b_empty;
             uint64_t* fin = first ? done : done + 1;
             const uint32_t d0 = tmem_base + static_cast<uint32_t>((first ? 0 : kAcc) * N);
-            int it = 0, use = 0;
+            int use = 0;
             bool ok = true;
-            for (int i = blockIdx.x; ok && i < n_items; i += G) {
-                const int n = get_item(p, i).ntiles;
+            for (int it = 0; ok; ++it) {
+                int gi = -1;
+                if (!wait_item(item_full, items, it, &gi, abort, lim)) {
+                    ok = false;
+                    break;
+                }
+                if (gi < 0) break;
+                const int n = get_item(p, gi).ntiles;
                 const int qb = it % kQBufs;
                 if (!mbar_wait(&q_full[qb], (it / kQBufs) & 1, abort, lim)) {
                     ok = false;
@@ -432,7 +477,6 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
                 }
                 if (!ok) break;
                 umma_commit(&q_empty[qb]);  // this pass is done with the item's query rows
-                ++it;
             }
             if (!ok) {
                 *abort = 1;
@@ -445,56 +489,41 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
         __syncwarp();
     } else if (warp == 3) {
         // ------------------------------------------------------------ publisher
-        // Per item: once both pass-1 warpgroups have added its sums (each thread's fence
-        // ordered its add before its pub_full arrival), one release add on the unit's counter.
-        // Then the warp waits until every item of the unit has arrived and leaves the unit's
-        // -lse per column in nlse_s for pass 2, which meanwhile still works on the item
-        // before: the exchange stays off pass 2's path unless pass 1 elsewhere is late.
-        int it = 0;
+        // Per item: once both pass-1 warpgroups have left its column sums (pub_full), lane l
+        // adds columns l and l + 32 to the unit's fp64 accumulator, every lane fences its adds,
+        // and lane 0 releases the item's arrival on the unit's counter.
         bool ok = true;
-        for (int i = blockIdx.x; i < n_items; i += G) {
-            const Item I = get_item(p, i);
-            const int buf = it & 1;
-            int good = 1;
-            if (lane == 0) {
-                if (!mbar_wait(&pub_full[buf], (it >> 1) & 1, abort, lim)) {
-                    good = 0;
-                } else {
-                    red_release_add(p.counters + I.unit, kNW);
-                    mbar_arrive(&pub_empty[buf]);
-                    good = mbar_wait(&lse_empty[buf], ((it >> 1) & 1) ^ 1, abort, lim) ? 1 : 0;
-                }
-                if (good) {  // bounded acquire spin until every item of the unit has arrived
-                    const int target = I.nitems * kNW;
-                    const long long t0 = clock64();
-                    for (uint32_t k = 1; ld_acquire(p.counters + I.unit) < target; ++k) {
-                        __nanosleep(32);
-                        if ((k & 63u) == 0u && (*abort || clock64() - t0 > lim)) {
-                            good = 0;
-                            break;
-                        }
-                    }
-                }
-            }
-            __syncwarp();  // the acquire above orders the other lanes' reads of the sums too
+        for (int it = 0;; ++it) {
+            int gi = -1, good = 1;
+            if (lane == 0) good = wait_item(item_full, items, it, &gi, abort, lim) ? 1 : 0;
+            gi = __shfl_sync(0xffffffffu, gi, 0);
             if (__shfl_sync(0xffffffffu, good, 0) == 0) {
                 ok = false;
                 break;
             }
-            if (lane < N / 2) {
-                const double* src = p.sums + static_cast<size_t>(I.unit) * N;
-                const int nheads = p.batch_nheads[I.batch];
+            if (gi < 0) break;
+            const Item I = get_item(p, gi);
+            const int buf = it & 1;
+            if (lane == 0) good = mbar_wait(&pub_full[buf], (it >> 1) & 1, abort, lim) ? 1 : 0;
+            if (__shfl_sync(0xffffffffu, good, 0) == 0) {
+                ok = false;
+                break;
+            }
+            double* dst = p.sums + static_cast<size_t>(I.unit) * N;
 #pragma unroll
-                for (int e = 0; e < 2; ++e) {
-                    const int c = 2 * lane + e;
-                    const double v = __ldcg(src + c);
-                    const bool real = (c % W_PAD) < p.w && (c / W_PAD) < nheads;
-                    nlse_s[buf][c] = real && v > 0.0 ? -static_cast<float>(log2(v)) : -INFINITY;
+            for (int c = lane; c < N; c += 32) {
+                const float2 ms = pub_s[buf][c];
+                if (ms.y > 0.f) {
+                    if (!(fabsf(ms.x) <= static_cast<float>(kMaxLog2))) record_error(p.status, kDevRange, c);
+                    else atomicAdd(dst + c, scaled_sum(ms.x, ms.y));
                 }
             }
+            __threadfence();  // this lane's adds are performed before the release below
             __syncwarp();
-            if (lane == 0) mbar_arrive(&lse_full[buf]);
-            ++it;
+            if (lane == 0) {
+                red_release_add(p.counters + I.unit, 1);
+                mbar_arrive(&pub_empty[buf]);
+            }
         }
         if (!ok && lane == 0) {
             *abort = 1;
@@ -512,10 +541,16 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
             const uint32_t lane_base = static_cast<uint32_t>(eq * 32) << 16;
             uint64_t* gbar = &group[wg];
             uint32_t gphase = 0;
-            int a_it = 0, a_item = 0;
+            int a_it = 0;
             bool ok = true;
-            for (int i = blockIdx.x; ok && i < n_items; i += G) {
-                const Item I = get_item(p, i);
+            for (int it = 0; ok; ++it) {
+                int gi = -1;
+                if (!wait_item(item_full, items, it, &gi, abort, lim)) {
+                    ok = false;
+                    break;
+                }
+                if (gi < 0) break;
+                const Item I = get_item(p, gi);
                 const int n = I.ntiles;
                 const int L = I.len, P = L - p.w;
                 const float sl2 = p.sl2;
@@ -565,13 +600,12 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
 #pragma unroll
                 for (int c = 0; c < kCols; ++c) m[c] = -nm[c];
                 if (!ok) break;
-                if (!item_sums(m, sm_, red_a[a_item & 1][wg], eq, lane, wtid, gbar, gphase,
-                               &pub_full[a_item & 1], &pub_empty[a_item & 1], (a_item >> 1) & 1,
-                               p.sums + static_cast<size_t>(I.unit) * N + col0, p.status, abort, lim)) {
+                if (!item_sums(m, sm_, red_a[it & 1][wg], eq, lane, wtid, gbar, gphase,
+                               &pub_full[it & 1], &pub_empty[it & 1], (it >> 1) & 1,
+                               pub_s[it & 1] + col0, abort, lim)) {
                     ok = false;
                     break;
                 }
-                ++a_item;
             }
             if (!ok) {
                 *abort = 1;
@@ -583,12 +617,25 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
         // One warpgroup over all N columns; lse sits in shared memory and is read by every
         // lane of a warp at the same address.
         const int eq = warp & 3;
+        const int wtid = threadIdx.x - kWarpB * 32;  // 0 .. 127
         const uint32_t lane_base = static_cast<uint32_t>(eq * 32) << 16;
         constexpr int kHeads = N / W_PAD;  // head slots of the MMA's columns
-        int b_it = 0, n_item = 0;
+        uint32_t gphase = 0;
+        int b_it = 0;
         bool ok = true;
-        for (int i = blockIdx.x; ok && i < n_items; i += G) {
-            const Item I = get_item(p, i);
+        for (int it = 0; ok; ++it) {
+            int gi = -1, good = 1;
+            if (lane == 0) good = wait_item(item_full, items, it, &gi, abort, lim) ? 1 : 0;
+            gi = __shfl_sync(0xffffffffu, gi, 0);
+            if (__shfl_sync(0xffffffffu, good, 0) == 0) {
+                ok = false;
+                break;
+            }
+            if (gi < 0) break;
+            // pass 2 reads an item's ring entry last: once each of its warps has, the producer
+            // may post another item there
+            if (lane == 0) mbar_arrive(&item_free[it % kItemRing]);
+            const Item I = get_item(p, gi);
             const int n = I.ntiles, tile0 = I.tile0;
             const int L = I.len, P = L - p.w;
             const int nheads = p.batch_nheads[I.batch];
@@ -596,16 +643,40 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
             const float sl2 = p.sl2;
             // the batch's first score row, at the sequence's first token
             float* const out = p.scores[I.layer] + static_cast<size_t>(p.batch_first[I.batch]) * T + I.start;
-            // ---------------------------------------------------- the unit's lse (warp 3)
-            const int buf = n_item & 1;
-            int good = 1;
-            if (lane == 0) good = mbar_wait(&lse_full[buf], (n_item >> 1) & 1, abort, lim) ? 1 : 0;
-            __syncwarp();
-            if (__shfl_sync(0xffffffffu, good, 0) == 0) {
+            // ---------------------------------------------------- the unit's lse
+            // a bounded acquire spin until every item of the unit has arrived, carried to the
+            // warpgroup by its barrier; then -lse per column from the accumulator
+            if (threadIdx.x == kWarpB * 32) {
+                const long long t0 = clock64();
+                for (uint32_t k = 1; ld_acquire(p.counters + I.unit) < I.nitems; ++k) {
+                    __nanosleep(32);
+                    if ((k & 63u) == 0u && (*abort || clock64() - t0 > lim)) {
+                        *abort = 1;
+                        break;
+                    }
+                }
+            }
+            if (!group_sync(&group[2], gphase, abort, lim) || *abort) {
                 ok = false;
                 break;
             }
-            const float* nlse = nlse_s[buf];
+            if (wtid < N) {
+                const int c = wtid;
+                const double v = __ldcg(p.sums + static_cast<size_t>(I.unit) * N + c);
+                const bool real = (c % W_PAD) < p.w && (c / W_PAD) < nheads;
+                // log2 v = e + log2 f with v = f * 2^e, f in [1, 2) (v is a normal double: its
+                // largest term is at least 2^-990)
+                const unsigned long long bits = static_cast<unsigned long long>(__double_as_longlong(v));
+                const int ex = static_cast<int>((bits >> 52) & 0x7FFull) - 1023;
+                const float f = static_cast<float>(__longlong_as_double(static_cast<long long>(
+                    (bits & 0x000FFFFFFFFFFFFFull) | 0x3FF0000000000000ull)));
+                nlse_s[c] = real && v > 0.0 ? -(static_cast<float>(ex) + lg2_approx(f)) : -INFINITY;
+            }
+            if (!group_sync(&group[2], gphase, abort, lim)) {
+                ok = false;
+                break;
+            }
+            const float* nlse = nlse_s;
             // ---------------------------------------------------- the item's tiles
             for (int jt = 0; jt < n; ++jt, ++b_it) {
                 const int acc = b_it % kAcc;
@@ -639,9 +710,11 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
                         if (h < nheads) out[h * T + j] = accum[h];
                 }
             }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&lse_empty[buf]);  // this warp is done with the lse
-            ++n_item;
+            // every warp is done with nlse_s before the next item's lse overwrites it
+            if (!group_sync(&group[2], gphase, abort, lim)) {
+                ok = false;
+                break;
+            }
         }
         if (!ok) {
             *abort = 1;
@@ -695,19 +768,23 @@ cudaError_t dispatch(const LayersParams& p, int n_cols, int w_pad, int grid, cud
     return cudaErrorInvalidValue;
 }
 
+
 }  // namespace
 
 cudaError_t launch_score_layers(const LayersLaunch& L, cudaStream_t stream) {
-    static LayersParams p;  // ~22 KB, kept off the host stack; calls are serialised by `mu`
+    static LayersParams p;  // ~30 KB, kept off the host stack; calls are serialised by `mu`
     static std::mutex mu;
     std::lock_guard<std::mutex> lock(mu);
     memset(&p, 0, sizeof(p));
     const int nl = static_cast<int>(L.layers.size());
     const int nb = static_cast<int>(L.batch_layer.size());
     const int ns = static_cast<int>(L.seq_start.size());
+    const int nu = static_cast<int>(L.units.size()) - 1;  // the last entry closes the table
     if (nl < 1 || nl > kMaxLaunchLayers || nb < 1 || nb > kMaxLaunchBatches ||
-        static_cast<int>(L.sel_heads.size()) > kMaxLaunchSel || ns < 1 || ns > kMaxLaunchSeqs)
+        static_cast<int>(L.sel_heads.size()) > kMaxLaunchSel || ns < 1 || ns > kMaxLaunchSeqs ||
+        nu < 0 || nu > kMaxLaunchUnits || L.grid < 1)
         return cudaErrorInvalidValue;
+    if (nu == 0) return cudaSuccess;
     for (int l = 0; l < nl; ++l) {
         p.tmap_k[l] = L.layers[l].tmap_k;
         p.tmap_q[l] = L.layers[l].tmap_q;
@@ -720,34 +797,31 @@ cudaError_t launch_score_layers(const LayersLaunch& L, cudaStream_t stream) {
     p.S = ns;
     p.T = L.T;
     p.w = L.w;
-    p.items_per_lb = L.seq_item0[ns];
-    p.n_items = nb * p.items_per_lb;
-    p.c = L.c;
+    p.n_units = nu;
+    p.n_items = L.units[nu].item0;
     p.n_layers = nl;
     p.seq0 = L.seq0;
     p.S_all = L.S_all;
     p.cu_hash = L.cu_hash;
     p.sl2 = L.softmax_scale * 1.4426950408889634f;
     p.wait_cycles = wait_limit_cycles();
-    for (int b = 0; b < nb; ++b) {
-        p.batch_layer[b] = L.batch_layer[b];
-        p.batch_group[b] = L.batch_group[b];
-        p.batch_first[b] = L.batch_first[b];
-        p.batch_nheads[b] = L.batch_nheads[b];
-        p.batch_sel[b] = L.batch_sel[b];
+    for (int i = 0; i < nb; ++i) {
+        p.batch_layer[i] = L.batch_layer[i];
+        p.batch_group[i] = L.batch_group[i];
+        p.batch_first[i] = L.batch_first[i];
+        p.batch_nheads[i] = L.batch_nheads[i];
+        p.batch_sel[i] = L.batch_sel[i];
     }
     for (size_t i = 0; i < L.sel_heads.size(); ++i) p.sel_heads[i] = L.sel_heads[i];
     for (int s = 0; s < ns; ++s) {
         p.seq_start[s] = L.seq_start[s];
         p.seq_len[s] = L.seq_len[s];
-        p.seq_item0[s] = L.seq_item0[s];
     }
-    p.seq_item0[ns] = L.seq_item0[ns];
+    for (int u = 0; u <= nu; ++u) p.units[u] = L.units[u];
     if (p.n_items == 0) return cudaSuccess;
-    // the exchange's accumulators and arrival counters start at zero
-    const size_t n_units = static_cast<size_t>(nb) * ns;
-    cudaError_t e = cudaMemsetAsync(L.sums, 0, n_units * L.n_cols * sizeof(double), stream);
-    if (e == cudaSuccess) e = cudaMemsetAsync(L.counters, 0, n_units * sizeof(int), stream);
+    // the exchange's accumulators, its arrival counters and the item counter start at zero
+    cudaError_t e = cudaMemsetAsync(L.sums, 0, static_cast<size_t>(nu) * L.n_cols * sizeof(double), stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(L.counters, 0, static_cast<size_t>(nu + 1) * sizeof(int), stream);
     if (e != cudaSuccess) return e;
     return dispatch(p, L.n_cols, L.w_pad, std::min(L.grid, p.n_items), stream);
 }

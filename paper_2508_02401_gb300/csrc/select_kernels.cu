@@ -1037,6 +1037,275 @@ __global__ void __launch_bounds__(256) gather_kernel(const __grid_constant__ Gat
     *dst = __ldg(src);
 }
 
+// ------------------------------------------------------------------ many layers at once
+// Selection of every (layer, sequence, selection) unit of a multi-layer call in one launch:
+// the CTAs take units from a global counter, and one CTA does a unit whole, streaming over its
+// candidate positions in chunks of kLsChunk (so that no length is too long and little sits in
+// shared memory): (A) pools the chunk, stores its order-preserving keys in a scratch row (and
+// the pooled scores when asked) and counts their first digits; the k-th largest key's digit
+// follows from the counts; (B) gathers the keys with that digit (at most kLsCand) and ranks
+// them exactly, by key and then position, or else refines the threshold digit by digit over
+// the scratch keys and finds the tie cutoff by a position-ordered scan; (C) writes the kept
+// positions in order, a chunk at a time (a block scan per chunk), copies their K/V rows, and
+// appends the window.  The same keys, ties and order as select_unit_kernel and the chunked
+// kernels.
+constexpr int kLsThreads = 512;
+constexpr int kLsPer = 16;
+constexpr int kLsChunk = kLsThreads * kLsPer;                    // 8192 positions
+constexpr int kLsStageFloats = kLsChunk + 2 * kMaxHalo;
+constexpr int kLsStageLoads = (kLsStageFloats + kLsThreads - 1) / kLsThreads;
+constexpr int kLsWords = 2 * stage_words(kLsStageFloats);        // two score rows at once
+constexpr int kLsSmem = kLsWords * 4;
+constexpr int kLsCand = 2048;                                    // first-digit ties ranked in place
+constexpr int kSelMaxLayers = 32;
+
+struct SelectLayersParams {
+    SelectParams layer[kSelMaxLayers];
+    uint32_t* keys[kSelMaxLayers];   // per layer [n_vec, T]: the keys of the pooled scores
+    int* next_unit;                  // work counter, zero at launch
+    int n_layers, units_per_layer;   // units_per_layer = S * n_vec
+};
+
+// The keys at src[jb .. jb + kLsPer) (zero past nvalid); 16-byte loads when src is 16-byte
+// aligned (jb is a multiple of kLsPer).
+__device__ __forceinline__ void load_keys(const uint32_t* src, int jb, int nvalid, uint32_t (&key)[kLsPer]) {
+    if (nvalid >= kLsPer && (reinterpret_cast<uintptr_t>(src) & 15u) == 0) {
+#pragma unroll
+        for (int q = 0; q < kLsPer / 4; ++q) {
+            const uint4 x = __ldcg(reinterpret_cast<const uint4*>(src + jb) + q);
+            key[4 * q] = x.x;
+            key[4 * q + 1] = x.y;
+            key[4 * q + 2] = x.z;
+            key[4 * q + 3] = x.w;
+        }
+    } else {
+#pragma unroll
+        for (int i = 0; i < kLsPer; ++i) key[i] = i < nvalid ? __ldcg(src + jb + i) : 0u;
+    }
+}
+
+__global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __grid_constant__ SelectLayersParams P) {
+    extern __shared__ __align__(16) float st[];  // pooling stage; the kept list of a chunk
+    __shared__ int hist[kHistBins];
+    __shared__ int scratch[33];
+    __shared__ int s_digit, s_above, s_cut, s_cnt, s_unit;
+    __shared__ uint32_t s_thr;
+    __shared__ uint2 cand[kLsCand];
+    constexpr int NT = kLsThreads, PER = kLsPer;
+    const int tid = threadIdx.x;
+    if (blockIdx.x == 0 && tid == 0) {
+        const SelectParams& p0 = P.layer[0];
+        if (seqlens_hash(p0.cu_seqlens, p0.S) != p0.cu_hash) record_error(p0.status, kDevBadSeqlens, 240);
+    }
+    const int n_units = P.n_layers * P.units_per_layer;
+    for (;;) {
+        if (tid == 0) s_unit = atomicAdd(P.next_unit, 1);
+        __syncthreads();
+        const int gu = s_unit;
+        __syncthreads();
+        if (gu >= n_units) break;
+        const int li = gu / P.units_per_layer, unit = gu % P.units_per_layer;
+        const SelectParams& p = P.layer[li];
+        UnitGeo u;
+        if (!unit_geo(p, unit, u)) continue;
+        const int kv0 = p.n_vec == p.Hkv ? u.g : 0, kv1 = p.n_vec == p.Hkv ? u.g + 1 : p.Hkv;
+        if (u.g == 0 && tid == 0) {
+            p.cu_keep[u.s + 1] = u.keep_off + u.n_keep;
+            if (u.s == 0) p.cu_keep[0] = 0;
+        }
+        float* pooled = p.write_pooled ? p.pooled + static_cast<size_t>(u.g) * p.T + u.t0 : nullptr;
+        int* list = reinterpret_cast<int*>(st);
+        if (u.L <= p.budget) {  // kept whole; its pooled scores read as 0
+            for (int e0 = 0; e0 < u.L; e0 += kLsChunk) {
+                const int m = min(kLsChunk, u.L - e0);
+                for (int e = tid; e < m; e += NT) {
+                    list[e] = e0 + e;
+                    if (pooled) pooled[e0 + e] = 0.f;
+                }
+                __syncthreads();
+                emit_kept(p, u, list, m, e0, kv0, kv1);
+                __syncthreads();
+            }
+            continue;
+        }
+        const int Pn = u.P, k = u.k;
+        uint32_t* keys = P.keys[li] + static_cast<size_t>(u.g) * p.T + u.t0;
+        if (pooled)  // window positions are not candidates
+            for (int j = Pn + tid; j < u.L; j += NT) pooled[j] = 0.f;
+        // (A) pooled scores, keys and first-digit counts, chunk by chunk
+        for (int b = tid; b < kHistBins; b += NT) hist[b] = 0;
+        __syncthreads();
+        for (int base = 0; base < Pn; base += kLsChunk) {
+            const int n = min(kLsChunk, Pn - base);
+            const int jb = tid * PER, nvalid = n - jb;
+            float acc[PER];
+            pooled_values<NT, PER, kLsStageLoads, kLsWords>(p, u, st, base, n, acc);
+            uint32_t key[PER], bins[PER];
+#pragma unroll
+            for (int i = 0; i < PER; ++i) {
+                key[i] = rank_key(acc[i]);
+                bins[i] = key[i] >> kHistShift;
+            }
+            // 16-byte stores where the rows are 16-byte aligned (base + jb is a multiple of 16)
+            if (nvalid >= PER && (reinterpret_cast<uintptr_t>(keys) & 15u) == 0 &&
+                (!pooled || (reinterpret_cast<uintptr_t>(pooled) & 15u) == 0)) {
+#pragma unroll
+                for (int q = 0; q < PER / 4; ++q) {
+                    reinterpret_cast<uint4*>(keys + base + jb)[q] =
+                        make_uint4(key[4 * q], key[4 * q + 1], key[4 * q + 2], key[4 * q + 3]);
+                    if (pooled)
+                        reinterpret_cast<float4*>(pooled + base + jb)[q] =
+                            make_float4(acc[4 * q], acc[4 * q + 1], acc[4 * q + 2], acc[4 * q + 3]);
+                }
+            } else {
+#pragma unroll
+                for (int i = 0; i < PER; ++i)
+                    if (i < nvalid) {
+                        keys[base + jb + i] = key[i];
+                        if (pooled) pooled[base + jb + i] = acc[i];
+                    }
+            }
+            add_runs<PER>(hist, bins, nvalid);
+        }
+        __syncthreads();  // also orders the key stores before the reads below (same block)
+        // (B) the k-th largest key thr, and the last position cut of a kept key equal to it
+        // (k = 0 keeps only the window: no key is above 0xffffffff, no position at or below -1)
+        uint32_t thr = 0xFFFFFFFFu;
+        int pos_cut = -1;
+        if (k > 0) {
+            if (tid == 0) s_cut = INT_MAX;
+            find_digit<NT>(hist, k, scratch, &s_digit, &s_above);
+            const uint32_t d1 = static_cast<uint32_t>(s_digit);
+            int r = k - s_above, n_eq = hist[d1];
+            __syncthreads();
+            if (n_eq <= kLsCand) {
+                if (tid == 0) s_cnt = 0;
+                __syncthreads();
+                for (int base = 0; base < Pn; base += kLsChunk) {
+                    const int jb = tid * PER, nvalid = min(kLsChunk, Pn - base) - jb;
+                    uint32_t key[PER];
+                    load_keys(keys + base, jb, nvalid, key);
+#pragma unroll
+                    for (int i = 0; i < PER; ++i)
+                        if (i < nvalid && (key[i] >> kHistShift) == d1) {
+                            const int c = atomicAdd(&s_cnt, 1);
+                            if (c < kLsCand) cand[c] = make_uint2(key[i], base + jb + i);
+                        }
+                }
+                __syncthreads();
+                for (int c = tid; c < n_eq; c += NT) {
+                    const uint2 me = cand[c];
+                    int ahead = 0;
+                    for (int q = 0; q < n_eq; ++q) {
+                        const uint2 o = cand[q];
+                        ahead += (o.x > me.x || (o.x == me.x && o.y < me.y)) ? 1 : 0;
+                    }
+                    if (ahead == r - 1) {
+                        s_thr = me.x;
+                        s_cut = static_cast<int>(me.y);
+                    }
+                }
+                __syncthreads();
+                thr = s_thr;
+                pos_cut = s_cut;
+            } else {
+                uint32_t prefix = d1 << kHistShift, mask = 0x7FFu << kHistShift;
+#pragma unroll 1
+                for (int level = 0; level < 2; ++level) {
+                    const int shift = level == 0 ? 10 : 0;
+                    const uint32_t dmask = level == 0 ? 0x7FFu : 0x3FFu;
+                    for (int b = tid; b < kHistBins; b += NT) hist[b] = 0;
+                    __syncthreads();
+                    for (int base = 0; base < Pn; base += kLsChunk) {
+                        const int jb = tid * PER, nvalid = min(kLsChunk, Pn - base) - jb;
+                        uint32_t key[PER];
+                        load_keys(keys + base, jb, nvalid, key);
+#pragma unroll
+                        for (int i = 0; i < PER; ++i)
+                            if (i < nvalid && (key[i] & mask) == prefix)
+                                atomicAdd(&hist[(key[i] >> shift) & dmask], 1);
+                    }
+                    __syncthreads();
+                    find_digit<NT>(hist, r, scratch, &s_digit, &s_above);
+                    prefix |= static_cast<uint32_t>(s_digit) << shift;
+                    mask |= dmask << shift;
+                    r -= s_above;
+                    n_eq = hist[s_digit];
+                    __syncthreads();
+                }
+                thr = prefix;
+                const int need_eq = r;  // keys equal to thr that are kept: the lowest positions
+                pos_cut = INT_MAX;
+                if (need_eq < n_eq) {
+                    int seen = 0;  // keys equal to thr in the chunks before
+                    for (int base = 0; base < Pn && seen < need_eq; base += kLsChunk) {
+                        const int jb = tid * PER, nvalid = min(kLsChunk, Pn - base) - jb;
+                        uint32_t key[PER];
+                        load_keys(keys + base, jb, nvalid, key);
+                        int ne = 0;
+#pragma unroll
+                        for (int i = 0; i < PER; ++i) ne += (i < nvalid && key[i] == thr) ? 1 : 0;
+                        int tot;
+                        const int before = seen + block_excl_scan<NT>(ne, scratch, &tot);
+                        if (before < need_eq && before + ne >= need_eq) {
+                            int c = before;
+#pragma unroll
+                            for (int i = 0; i < PER; ++i) {
+                                if (i < nvalid && key[i] == thr) {
+                                    ++c;
+                                    if (c == need_eq) s_cut = base + jb + i;
+                                }
+                            }
+                        }
+                        seen += tot;
+                    }
+                    __syncthreads();
+                    pos_cut = s_cut;
+                }
+            }
+        }
+        // (C) the kept positions in order, chunk by chunk, with their K/V rows; then the window
+        int written = 0;
+        for (int base = 0; base < Pn; base += kLsChunk) {
+            const int jb = tid * PER, nvalid = min(kLsChunk, Pn - base) - jb;
+            uint32_t key[PER];
+            load_keys(keys + base, jb, nvalid, key);
+            uint32_t taken = 0;
+            int cnt = 0;
+#pragma unroll
+            for (int i = 0; i < PER; ++i) {
+                const int j = base + jb + i;
+                if (i < nvalid && (key[i] > thr || (key[i] == thr && j <= pos_cut))) {
+                    taken |= 1u << i;
+                    ++cnt;
+                }
+            }
+            int tot;
+            int rk = block_excl_scan<NT>(cnt, scratch, &tot);
+            if (written + tot > k) break;  // checked below
+#pragma unroll
+            for (int i = 0; i < PER; ++i) {
+                if ((taken >> i) & 1u) {
+                    list[rk] = base + jb + i;
+                    ++rk;
+                }
+            }
+            __syncthreads();
+            emit_kept(p, u, list, tot, written, kv0, kv1);
+            written += tot;
+            __syncthreads();
+        }
+        if (written != k) {
+            if (tid == 0) record_error(p.status, kDevBadIndex, 340 + unit);
+            continue;
+        }
+        for (int i = tid; i < p.w; i += NT) list[i] = Pn + i;
+        __syncthreads();
+        emit_kept(p, u, list, p.w, k, kv0, kv1);
+        __syncthreads();
+    }
+}
+
 }  // namespace
 
 cudaError_t launch_pool(const SelectLaunch& L, cudaStream_t stream) {
@@ -1158,6 +1427,70 @@ cudaError_t launch_gather(const GatherLaunch& L, cudaStream_t stream) {
     if (rows == 0) return cudaSuccess;
     gather_kernel<<<static_cast<unsigned>((rows + 7) / 8), 256, 0, stream>>>(p);
     return cudaGetLastError();
+}
+
+// The selection of several layers in one launch (select_layers_kernel); Ls[i] as for
+// launch_select with from_scores = 1, and keys[i] a [n_vec, T] scratch per layer.  One launch per
+// kSelMaxLayers layers; `next_unit` (kSelMaxLayers-aligned count of ints) is the work counter
+// of each launch and is cleared first.
+cudaError_t launch_select_layers(const SelectLaunch* Ls, uint32_t* const* keys, int n_layers,
+                                 int* next_unit, int grid, cudaStream_t stream) {
+    static SelectLayersParams P;  // ~25 KB; calls are serialised by `mu`
+    static std::mutex mu;
+    static_assert(sizeof(SelectLayersParams) <= 32000, "kernel parameters");
+    std::lock_guard<std::mutex> lock(mu);
+    static bool configured = false;
+    if (!configured) {
+        const cudaError_t e = cudaFuncSetAttribute(select_layers_kernel,
+                                                   cudaFuncAttributeMaxDynamicSharedMemorySize, kLsSmem);
+        if (e != cudaSuccess) return e;
+        configured = true;
+    }
+    for (int l0 = 0; l0 < n_layers; l0 += kSelMaxLayers) {
+        const int nl = std::min(kSelMaxLayers, n_layers - l0);
+        memset(&P, 0, sizeof P);
+        for (int i = 0; i < nl; ++i) {
+            const SelectLaunch& L = Ls[l0 + i];
+            SelectParams& p = P.layer[i];
+            p.scores = L.scores;
+            p.pooled = L.pooled;
+            p.idx = L.idx;
+            p.cu_keep = L.cu_keep_dev;
+            p.cu_seqlens = L.cu_seqlens_dev;
+            p.status = L.status;
+            p.k = reinterpret_cast<const uint4*>(L.k);
+            p.v = reinterpret_cast<const uint4*>(L.v);
+            p.tok_stride = L.tok_stride / 8;
+            p.head_stride = L.head_stride / 8;
+            p.k_out = reinterpret_cast<uint4*>(L.k_out);
+            p.v_out = reinterpret_cast<uint4*>(L.v_out);
+            p.S = L.S;
+            p.T = L.T;
+            p.Hkv = L.Hkv;
+            p.w = L.w;
+            p.budget = L.budget;
+            p.T_keep = L.T_keep;
+            p.n_vec = L.n_vec;
+            p.pool_kernel = L.pool_kernel;
+            p.pool_type = L.pool_type;
+            p.head_order = L.head_order;
+            p.from_scores = 1;
+            p.write_pooled = L.write_pooled;
+            p.cu_hash = L.cu_hash;
+            for (int g = 0; g <= L.n_vec; ++g) p.group_first[g] = static_cast<int16_t>(L.group_first[g]);
+            P.keys[i] = keys[l0 + i];
+        }
+        P.n_layers = nl;
+        P.units_per_layer = Ls[l0].S * Ls[l0].n_vec;
+        P.next_unit = next_unit;
+        const int units = nl * P.units_per_layer;
+        if (units == 0) continue;
+        cudaError_t e = cudaMemsetAsync(next_unit, 0, sizeof(int), stream);
+        if (e != cudaSuccess) return e;
+        select_layers_kernel<<<std::min(grid, units), kLsThreads, kLsSmem, stream>>>(P);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+    return cudaSuccess;
 }
 
 }  // namespace ckv
