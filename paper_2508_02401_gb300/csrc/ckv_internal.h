@@ -8,7 +8,20 @@
 
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 namespace ckv {
+
+// A host-side NVTX range around one kernel launch, named for the kernel, so that a profiler or
+// timeline tool that attaches sees which library call each launch came from (ranges opened
+// while a CUDA graph is captured mark the capture).  With no tool attached, the push and the pop
+// go through NVTX's empty function table.
+struct NvtxRange {
+    explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+    ~NvtxRange() { nvtxRangePop(); }
+    NvtxRange(const NvtxRange&) = delete;
+    NvtxRange& operator=(const NvtxRange&) = delete;
+};
 
 // A scoring work item: `ntiles` key tiles (128 keys each) of one unit, from tile `tile0`.
 struct ScoreItem {

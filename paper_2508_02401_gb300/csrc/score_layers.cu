@@ -751,6 +751,7 @@ cudaError_t launch_one(const LayersParams& p, int grid, cudaStream_t stream) {
     attr[0].val.cooperative = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
+    NvtxRange range("score_layers_kernel");
     return cudaLaunchKernelEx(&cfg, kern, p);
 }
 

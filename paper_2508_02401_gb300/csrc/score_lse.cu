@@ -329,6 +329,7 @@ cudaError_t launch_lse(const ScoreParams& p, int grid, cudaStream_t stream) {
         if (e != cudaSuccess) return e;
         configured = true;
     }
+    NvtxRange range("score_lse_kernel");
     kern<<<grid, kThreads, smem, stream>>>(p);
     return cudaGetLastError();
 }

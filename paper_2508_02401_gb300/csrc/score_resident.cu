@@ -560,6 +560,7 @@ cudaError_t launch_res(const ScoreParams& p, int grid, cudaStream_t stream) {
     attr[0].val.cooperative = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
+    NvtxRange range("score_resident_kernel");
     return cudaLaunchKernelEx(&cfg, kern, p);
 }
 

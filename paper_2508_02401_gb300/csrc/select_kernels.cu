@@ -1323,6 +1323,7 @@ cudaError_t launch_pool(const SelectLaunch& L, cudaStream_t stream) {
     for (int g = 0; g <= L.n_vec; ++g) p.group_first[g] = static_cast<int16_t>(L.group_first[g]);
     if (L.T == 0) return cudaSuccess;
     dim3 grid((L.T + 255) / 256, L.n_vec);
+    NvtxRange range("pool_kernel");
     pool_kernel<<<grid, 256, 0, stream>>>(p);
     return cudaGetLastError();
 }
@@ -1388,10 +1389,12 @@ cudaError_t launch_select(const SelectLaunch& L, cudaStream_t stream) {
         sel_smem_set = sel_smem;
     }
     if (L.min_len <= kUnitLen) {
+        NvtxRange range("select_unit_kernel");
         select_unit_kernel<<<units * (L.Hkv / L.n_vec), kUnitThreads, kUnitSmem, stream>>>(p);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
     if (L.max_len > kUnitLen) {
+        NvtxRange range("select_kernel+compact_kernel");
         const dim3 grid(units, L.max_chunks);
         select_kernel<<<grid, kSelThreads, sel_smem, stream>>>(p);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
@@ -1425,6 +1428,7 @@ cudaError_t launch_gather(const GatherLaunch& L, cudaStream_t stream) {
     p.cu_hash = L.cu_hash;
     const long long rows = static_cast<long long>(L.T_keep) * L.Hkv;
     if (rows == 0) return cudaSuccess;
+    NvtxRange range("gather_kernel");
     gather_kernel<<<static_cast<unsigned>((rows + 7) / 8), 256, 0, stream>>>(p);
     return cudaGetLastError();
 }
@@ -1487,6 +1491,7 @@ cudaError_t launch_select_layers(const SelectLaunch* Ls, uint32_t* const* keys, 
         if (units == 0) continue;
         cudaError_t e = cudaMemsetAsync(next_unit, 0, sizeof(int), stream);
         if (e != cudaSuccess) return e;
+        NvtxRange range("select_layers_kernel");
         select_layers_kernel<<<std::min(grid, units), kLsThreads, kLsSmem, stream>>>(P);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }

@@ -72,6 +72,7 @@ cudaError_t launch_srs_mask(const SrsLaunch& L, cudaStream_t stream) {
     const int64_t n = static_cast<int64_t>(L.Hq) * rows;
     if (n == 0) return cudaSuccess;
     const int blocks = static_cast<int>(std::min<int64_t>((n + 255) / 256, 4096));
+    NvtxRange range("srs_mask_kernel");
     srs_mask_kernel<<<blocks, 256, 0, stream>>>(L.lse, L.lse_stride, L.in_answer, L.lse_masked, L.Hq, rows);
     return cudaGetLastError();
 }
@@ -89,6 +90,7 @@ cudaError_t launch_srs_span(const SrsLaunch& L, cudaStream_t stream) {
     p.T = L.T;
     p.S = L.S;
     for (int i = 0; i < L.n_sel; ++i) p.sel_heads[i] = static_cast<int16_t>(L.sel_heads[i]);
+    NvtxRange range("srs_span_kernel");
     srs_span_kernel<<<dim3(L.n_sel, L.S), 256, 0, stream>>>(p);
     return cudaGetLastError();
 }
