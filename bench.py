@@ -104,8 +104,8 @@ def _args():
                          "ckv_compress_layer_lse / ckv_score_window_lse, one pass over K")
     ap.add_argument("--max-ctas", type=int, default=0,
                     help="CTAs one call's scoring kernel may occupy (0: all SMs with --calls "
-                         "layers; SMs / 16 with --calls layer, so that 16 layers' scoring kernels "
-                         "are resident at once)")
+                         "layers; SMs / streams with --calls layer, so that one scoring kernel "
+                         "per stream is resident at once)")
     ap.add_argument("--streams", type=int, default=0,
                     help="layers are issued round-robin on this many streams (one workspace each); "
                          "0 = min(layers, 16)")
@@ -266,13 +266,13 @@ def run_ours(args):
             layers[-1]["lse"] = _window_lse(layers[-1]["q"], layers[-1]["k"], wl.cu_seqlens(), wl.window,
                                             wl.num_q_heads, Hkv)
     ws_bytes = max(ckv.ckv_workspace_size(cfg, l, batch) for l in range(nl))
-    # Layers are independent: by default they go round-robin on 16 streams, and each call's
-    # scoring kernel is capped at SMs / 16 CTAs, so that 16 of them are resident at once (in
-    # even waves: a stream's next layer starts when its previous one is done) and the SMs
-    # they leave free run the selections in between.
+    # Layers are independent: by default they go round-robin on min(layers, 16) streams, and
+    # each call's scoring kernel is capped at SMs / streams CTAs, so that one per stream is
+    # resident at once (in even waves: a stream's next layer starts when its previous one is
+    # done) and the SMs they leave free run the selections in between.
     nstreams = args.streams if args.streams > 0 else min(nl, 16)
     sms = torch.cuda.get_device_properties(local).multi_processor_count
-    cap = args.max_ctas if args.max_ctas > 0 else max(1, sms // 16)
+    cap = args.max_ctas if args.max_ctas > 0 else max(1, sms // nstreams)
     cfg = ckv.Config.from_workload(wl, max_ctas=cap, score_path=path)
     wss = [torch.zeros(ws_bytes, dtype=torch.uint8, device="cuda") for _ in range(nstreams)]
     ws = wss[0]
@@ -747,7 +747,7 @@ def run_srs(args):
     nl, T, Hkv, Hq = wl.num_layers, wl.total_tokens, wl.num_kv_heads, wl.num_q_heads
     sms = torch.cuda.get_device_properties(0).multi_processor_count
     nstreams = args.streams if args.streams > 0 else min(nl, 16)
-    cap = args.max_ctas if args.max_ctas > 0 else max(1, sms // 16)
+    cap = args.max_ctas if args.max_ctas > 0 else max(1, sms // nstreams)
     cfg = ckv.Config.from_workload(wl, head_mask=np.ones((nl, Hq), np.uint8), max_ctas=cap)
     batch = ckv.Batch(wl.cu_seqlens())
     cu = wl.cu_seqlens()

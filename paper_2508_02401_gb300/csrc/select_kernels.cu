@@ -250,22 +250,26 @@ __device__ __forceinline__ void find_digit(const int* hist, int r, int* scratch,
 }
 
 // Adds a thread's run-aggregated counts of PER consecutive digits to a shared histogram:
-// consecutive keys of a thread are neighbouring positions and often share a digit.
+// consecutive keys of a thread are neighbouring positions and often share a digit, so one
+// atomic add per run of equal digits (a linear scan) instead of one per key.
 template <int PER>
 __device__ __forceinline__ void add_runs(int* hist, const uint32_t (&bins)[PER], int nvalid) {
+    if (nvalid <= 0) return;
+    uint32_t cur = bins[0];
+    int len = 1;
 #pragma unroll
-    for (int i = 0; i < PER; ++i) {
-        if (i < nvalid && (i == 0 || bins[i] != bins[i - 1])) {
-            int len = 1;
-            bool run = true;
-#pragma unroll
-            for (int q = i + 1; q < PER; ++q) {
-                run = run && q < nvalid && bins[q] == bins[i];
-                len += run ? 1 : 0;
+    for (int i = 1; i < PER; ++i) {
+        if (i < nvalid) {
+            if (bins[i] == cur) {
+                ++len;
+            } else {
+                atomicAdd(&hist[cur], len);
+                cur = bins[i];
+                len = 1;
             }
-            atomicAdd(&hist[bins[i]], len);
         }
     }
+    atomicAdd(&hist[cur], len);
 }
 
 // Stages the sum of score rows [ra, rb) at sequence positions base-half .. base+n+half-1
@@ -297,16 +301,18 @@ __device__ __forceinline__ void stage_rows(float* st, const float* scores, size_
 __device__ __forceinline__ void cp_async4(float* dst, const float* src) {
     asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
 }
-__device__ __forceinline__ void cp_async_wait_all() {
-    asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait_group() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
-// Stages score rows ra .. ra+nr-1 (each alone, not summed) at sequence positions
-// base-half .. base+n+half-1 (zero outside [0, P)), row i at st + i*words, element e at
-// sidx(e): every copy of every row is issued (asynchronously, no registers held) before the
-// wait, so the rows take one round trip together.
+// Issues the copies that stage score rows ra .. ra+nr-1 (each alone, not summed) at sequence
+// positions base-half .. base+n+half-1 (zero outside [0, P)), row i at st + i*words, element e
+// at sidx(e), and commits them as one group: every copy of every row is issued
+// (asynchronously, no registers held) before any wait, so the rows take one round trip together.
 template <int NT, int LOADS>
-__device__ __forceinline__ void stage_rows_async(float* st, int words, const float* scores, size_t T,
+__device__ __forceinline__ void stage_rows_issue(float* st, int words, const float* scores, size_t T,
                                                  int t0, int ra, int nr, int base, int half, int n,
                                                  int P) {
     const int ne = n + 2 * half, tid = threadIdx.x;
@@ -323,7 +329,16 @@ __device__ __forceinline__ void stage_rows_async(float* st, int words, const flo
             }
         }
     }
-    cp_async_wait_all();
+    cp_async_commit();
+}
+
+// The same, waiting for this thread's copies to land.
+template <int NT, int LOADS>
+__device__ __forceinline__ void stage_rows_async(float* st, int words, const float* scores, size_t T,
+                                                 int t0, int ra, int nr, int base, int half, int n,
+                                                 int P) {
+    stage_rows_issue<NT, LOADS>(st, words, scores, T, t0, ra, nr, base, half, n, P);
+    cp_async_wait_group<0>();
 }
 
 // Pools PER consecutive outputs from the stage: output i reads staged elements
@@ -1041,22 +1056,25 @@ __global__ void __launch_bounds__(256) gather_kernel(const __grid_constant__ Gat
 // Selection of every (layer, sequence, selection) unit of a multi-layer call in one launch:
 // the CTAs take units from a global counter, and one CTA does a unit whole, streaming over its
 // candidate positions in chunks of kLsChunk (so that no length is too long and little sits in
-// shared memory): (A) pools the chunk, stores its order-preserving keys in a scratch row (and
-// the pooled scores when asked) and counts their first digits; the k-th largest key's digit
-// follows from the counts; (B) gathers the keys with that digit (at most kLsCand) and ranks
-// them exactly, by key and then position, or else refines the threshold digit by digit over
-// the scratch keys and finds the tie cutoff by a position-ordered scan; (C) writes the kept
-// positions in order, a chunk at a time (a block scan per chunk), copies their K/V rows, and
-// appends the window.  The same keys, ties and order as select_unit_kernel and the chunked
-// kernels.
+// shared memory): (A) pools the chunk (the next chunk's score rows copied in meanwhile),
+// stores its order-preserving keys in a scratch row (and the pooled scores when asked) and
+// counts their first digits; the k-th largest key's digit follows from the counts; (B) refines
+// the threshold by two more digits (11 and 10 bits), counting over the keys that share the
+// digits so far: gathered into shared memory when at most kLsCand share the first digit, else
+// read again from the scratch row; the tie cutoff among keys equal to the threshold is their
+// rank by position, in shared memory when at most kLsTies were gathered, else by a
+// position-ordered scan of the scratch row; (C) writes the kept positions in order, a chunk at
+// a time (a block scan per chunk), copies their K/V rows, and appends the window.  The same
+// keys, ties and order as select_unit_kernel and the chunked kernels.
 constexpr int kLsThreads = 512;
 constexpr int kLsPer = 16;
 constexpr int kLsChunk = kLsThreads * kLsPer;                    // 8192 positions
 constexpr int kLsStageFloats = kLsChunk + 2 * kMaxHalo;
 constexpr int kLsStageLoads = (kLsStageFloats + kLsThreads - 1) / kLsThreads;
-constexpr int kLsWords = 2 * stage_words(kLsStageFloats);        // two score rows at once
+constexpr int kLsWords = 4 * stage_words(kLsStageFloats);        // four score rows at once
 constexpr int kLsSmem = kLsWords * 4;
-constexpr int kLsCand = 2048;                                    // first-digit ties ranked in place
+constexpr int kLsCand = 2048;   // keys sharing the k-th key's first digit gathered in shared memory
+constexpr int kLsTies = 256;    // keys equal to the k-th key ranked by position in shared memory
 constexpr int kSelMaxLayers = 32;
 
 struct SelectLayersParams {
@@ -1081,6 +1099,17 @@ __device__ __forceinline__ void load_keys(const uint32_t* src, int jb, int nvali
     } else {
 #pragma unroll
         for (int i = 0; i < kLsPer; ++i) key[i] = i < nvalid ? __ldcg(src + jb + i) : 0u;
+    }
+}
+
+// The keys of a thread in the chunk after the one at `base` (zeros when there is none).
+__device__ __forceinline__ void next_keys(const uint32_t* keys, int base, int Pn, int jb, uint32_t (&key)[kLsPer]) {
+    const int nb = base + kLsChunk;
+    if (nb < Pn) {
+        load_keys(keys + nb, jb, min(kLsChunk, Pn - nb) - jb, key);
+    } else {
+#pragma unroll
+        for (int i = 0; i < kLsPer; ++i) key[i] = 0u;
     }
 }
 
@@ -1134,12 +1163,39 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
             for (int j = Pn + tid; j < u.L; j += NT) pooled[j] = 0.f;
         // (A) pooled scores, keys and first-digit counts, chunk by chunk
         for (int b = tid; b < kHistBins; b += NT) hist[b] = 0;
+        // With the heads pooled one by one and two chunks' rows fitting the stage, the next
+        // chunk's rows are copied in while this chunk is pooled (two buffers of nr rows).
+        const int half = p.pool_kernel >> 1;
+        const int r0 = p.group_first[u.g], nr = p.group_first[u.g + 1] - r0;
+        const int words = stage_words(kLsChunk + 2 * half);
+        const bool piped = p.from_scores && p.head_order == 0 && 2 * nr * words + PER <= kLsWords;
+        if (piped)
+            stage_rows_issue<NT, kLsStageLoads>(st, words, p.scores, p.T, u.t0, r0, nr, 0, half,
+                                                min(kLsChunk, Pn), u.P);
         __syncthreads();
-        for (int base = 0; base < Pn; base += kLsChunk) {
+        for (int base = 0, c = 0; base < Pn; base += kLsChunk, ++c) {
             const int n = min(kLsChunk, Pn - base);
             const int jb = tid * PER, nvalid = n - jb;
             float acc[PER];
-            pooled_values<NT, PER, kLsStageLoads, kLsWords>(p, u, st, base, n, acc);
+            if (piped) {
+                const float* cur = st + (c & 1) * nr * words;
+                if (base + kLsChunk < Pn) {
+                    stage_rows_issue<NT, kLsStageLoads>(st + ((c + 1) & 1) * nr * words, words, p.scores,
+                                                        p.T, u.t0, r0, nr, base + kLsChunk, half,
+                                                        min(kLsChunk, Pn - base - kLsChunk), u.P);
+                    cp_async_wait_group<1>();
+                } else {
+                    cp_async_wait_group<0>();
+                }
+                __syncthreads();
+#pragma unroll
+                for (int i = 0; i < PER; ++i) acc[i] = 0.f;
+                for (int i = 0; i < nr; ++i)
+                    pool_any<PER>(cur + i * words, jb, nvalid, half, p.pool_type == 0,
+                                  static_cast<float>(p.pool_kernel), acc);
+            } else {
+                pooled_values<NT, PER, kLsStageLoads, kLsWords>(p, u, st, base, n, acc);
+            }
             uint32_t key[PER], bins[PER];
 #pragma unroll
             for (int i = 0; i < PER; ++i) {
@@ -1166,6 +1222,7 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
                     }
             }
             add_runs<PER>(hist, bins, nvalid);
+            if (piped) __syncthreads();  // every thread is done with this chunk's buffer
         }
         __syncthreads();  // also orders the key stores before the reads below (same block)
         // (B) the k-th largest key thr, and the last position cut of a kept key equal to it
@@ -1177,45 +1234,45 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
             find_digit<NT>(hist, k, scratch, &s_digit, &s_above);
             const uint32_t d1 = static_cast<uint32_t>(s_digit);
             int r = k - s_above, n_eq = hist[d1];
+            const int n_first = n_eq;
             __syncthreads();
-            if (n_eq <= kLsCand) {
+            // The keys with the k-th key's first digit: gathered into shared memory when there
+            // are at most kLsCand of them (the usual case), else read again from the scratch row.
+            const bool in_smem = n_eq <= kLsCand;
+            if (in_smem) {
                 if (tid == 0) s_cnt = 0;
                 __syncthreads();
+                uint32_t key[PER];  // this chunk's keys; the next chunk's are loaded meanwhile
+                load_keys(keys, tid * PER, min(kLsChunk, Pn) - tid * PER, key);
                 for (int base = 0; base < Pn; base += kLsChunk) {
                     const int jb = tid * PER, nvalid = min(kLsChunk, Pn - base) - jb;
-                    uint32_t key[PER];
-                    load_keys(keys + base, jb, nvalid, key);
+                    uint32_t nxt[PER];
+                    next_keys(keys, base, Pn, jb, nxt);
 #pragma unroll
                     for (int i = 0; i < PER; ++i)
                         if (i < nvalid && (key[i] >> kHistShift) == d1) {
                             const int c = atomicAdd(&s_cnt, 1);
                             if (c < kLsCand) cand[c] = make_uint2(key[i], base + jb + i);
                         }
+#pragma unroll
+                    for (int i = 0; i < PER; ++i) key[i] = nxt[i];
                 }
-                __syncthreads();
-                for (int c = tid; c < n_eq; c += NT) {
-                    const uint2 me = cand[c];
-                    int ahead = 0;
-                    for (int q = 0; q < n_eq; ++q) {
-                        const uint2 o = cand[q];
-                        ahead += (o.x > me.x || (o.x == me.x && o.y < me.y)) ? 1 : 0;
-                    }
-                    if (ahead == r - 1) {
-                        s_thr = me.x;
-                        s_cut = static_cast<int>(me.y);
-                    }
-                }
-                __syncthreads();
-                thr = s_thr;
-                pos_cut = s_cut;
-            } else {
-                uint32_t prefix = d1 << kHistShift, mask = 0x7FFu << kHistShift;
+            }
+            // Two more digits (11 and 10 bits) of the k-th key, by counts of the keys that share
+            // the digits so far: over the gathered candidates or over the scratch row.
+            uint32_t prefix = d1 << kHistShift, mask = 0x7FFu << kHistShift;
 #pragma unroll 1
-                for (int level = 0; level < 2; ++level) {
-                    const int shift = level == 0 ? 10 : 0;
-                    const uint32_t dmask = level == 0 ? 0x7FFu : 0x3FFu;
-                    for (int b = tid; b < kHistBins; b += NT) hist[b] = 0;
-                    __syncthreads();
+            for (int level = 0; level < 2; ++level) {
+                const int shift = level == 0 ? 10 : 0;
+                const uint32_t dmask = level == 0 ? 0x7FFu : 0x3FFu;
+                for (int b = tid; b < kHistBins; b += NT) hist[b] = 0;
+                __syncthreads();
+                if (in_smem) {
+                    for (int c = tid; c < n_first; c += NT) {
+                        const uint32_t kk = cand[c].x;
+                        if ((kk & mask) == prefix) atomicAdd(&hist[(kk >> shift) & dmask], 1);
+                    }
+                } else {
                     for (int base = 0; base < Pn; base += kLsChunk) {
                         const int jb = tid * PER, nvalid = min(kLsChunk, Pn - base) - jb;
                         uint32_t key[PER];
@@ -1225,18 +1282,39 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
                             if (i < nvalid && (key[i] & mask) == prefix)
                                 atomicAdd(&hist[(key[i] >> shift) & dmask], 1);
                     }
-                    __syncthreads();
-                    find_digit<NT>(hist, r, scratch, &s_digit, &s_above);
-                    prefix |= static_cast<uint32_t>(s_digit) << shift;
-                    mask |= dmask << shift;
-                    r -= s_above;
-                    n_eq = hist[s_digit];
-                    __syncthreads();
                 }
-                thr = prefix;
-                const int need_eq = r;  // keys equal to thr that are kept: the lowest positions
-                pos_cut = INT_MAX;
-                if (need_eq < n_eq) {
+                __syncthreads();
+                find_digit<NT>(hist, r, scratch, &s_digit, &s_above);
+                prefix |= static_cast<uint32_t>(s_digit) << shift;
+                mask |= dmask << shift;
+                r -= s_above;
+                n_eq = hist[s_digit];  // now: the keys equal to the k-th key
+                __syncthreads();
+            }
+            thr = prefix;
+            const int need_eq = r;  // keys equal to thr that are kept: the lowest positions
+            pos_cut = INT_MAX;
+            if (need_eq < n_eq) {
+                if (in_smem && n_eq <= kLsTies) {
+                    // the candidates equal to thr, ranked by position in shared memory (the
+                    // counts are no longer needed: their array holds the positions)
+                    int* eq = hist;
+                    if (tid == 0) s_cnt = 0;
+                    __syncthreads();
+                    for (int c = tid; c < n_first; c += NT) {
+                        const uint2 x = cand[c];
+                        if (x.x == thr) eq[atomicAdd(&s_cnt, 1)] = static_cast<int>(x.y);
+                    }
+                    __syncthreads();
+                    for (int i = tid; i < n_eq; i += NT) {
+                        const int me = eq[i];
+                        int ahead = 0;
+                        for (int q = 0; q < n_eq; ++q) ahead += eq[q] < me ? 1 : 0;
+                        if (ahead == need_eq - 1) s_cut = me;
+                    }
+                    __syncthreads();
+                    pos_cut = s_cut;
+                } else {
                     int seen = 0;  // keys equal to thr in the chunks before
                     for (int base = 0; base < Pn && seen < need_eq; base += kLsChunk) {
                         const int jb = tid * PER, nvalid = min(kLsChunk, Pn - base) - jb;
@@ -1266,10 +1344,12 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
         }
         // (C) the kept positions in order, chunk by chunk, with their K/V rows; then the window
         int written = 0;
+        uint32_t key[PER];  // this chunk's keys; the next chunk's are loaded meanwhile
+        load_keys(keys, tid * PER, min(kLsChunk, Pn) - tid * PER, key);
         for (int base = 0; base < Pn; base += kLsChunk) {
             const int jb = tid * PER, nvalid = min(kLsChunk, Pn - base) - jb;
-            uint32_t key[PER];
-            load_keys(keys + base, jb, nvalid, key);
+            uint32_t nxt[PER];
+            next_keys(keys, base, Pn, jb, nxt);
             uint32_t taken = 0;
             int cnt = 0;
 #pragma unroll
@@ -1294,6 +1374,8 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
             emit_kept(p, u, list, tot, written, kv0, kv1);
             written += tot;
             __syncthreads();
+#pragma unroll
+            for (int i = 0; i < PER; ++i) key[i] = nxt[i];
         }
         if (written != k) {
             if (tid == 0) record_error(p.status, kDevBadIndex, 340 + unit);

@@ -104,3 +104,27 @@ def test_layers_call_equals_the_single_layer_calls():
         np.testing.assert_array_equal(res[l]["cu_keep_dev"], one["cu_keep_dev"])
         o = gu.run_oracle(wl, l, li, want_kv=False)
         gu.check_layer(wl, l, li, res[l], o)
+
+
+def test_equal_scores_keep_the_lowest_positions():
+    """Sequences whose keys are all zero give every candidate the same score (each window row
+    spreads its mass evenly), so the multi-layer selection keeps the lowest positions.  The
+    lengths take each of its tie paths: ties ranked by position in shared memory (168 equal
+    keys), ties found by a scan of the scratch keys (268 and 1468), and more keys sharing the
+    first digit than shared memory gathers (39968); the last sequence keeps random keys."""
+    wl = _wl(num_layers=1, seqlens=(200, 300, 1500, 40000, 2500), budget_mean=64,
+             budget_uniform=True)
+    cfg = ckv.Config.from_workload(wl)
+    li = wl.layer(0)
+    cu = wl.cu_seqlens()
+    for s in range(4):
+        li.k[cu[s]:cu[s + 1]] = 0
+    res = _run_layers(wl, cfg, [li], with_scores=True)
+    o = gu.run_oracle(wl, 0, li, want_kv=False)
+    gu.check_layer(wl, 0, li, res[0], o)
+    ck = o["cu_keep"]
+    for s in range(4):
+        P = int(cu[s + 1] - cu[s]) - wl.window
+        for g in range(wl.num_kv_heads):
+            np.testing.assert_array_equal(res[0]["idx"][g, ck[s]:ck[s] + 32], np.arange(32))
+            assert P > 32
