@@ -533,9 +533,10 @@ struct LayerJob {
 // split into m = ceil(tiles / c) items of balanced length, unit after unit (head batch major);
 // `units` ends with an entry holding the total.  c is kItemTiles, or more where a unit would
 // otherwise have more items than the launch has CTAs (the kernel's progress argument needs at
-// most G).  Short items let the faster SMs take more of the work and keep the tiles that pass
-// 2 re-reads few enough to stay in L2.
-constexpr int kItemTiles = 8;
+// most G).  Items are long enough that their fixed costs (taking the item, loading its query
+// rows, publishing its sums, computing the unit's lse) are paid rarely, and short enough that
+// the faster SMs take more of the work and that the tiles pass 2 re-reads stay in L2.
+constexpr int kItemTiles = 14;
 void plan_items(const std::vector<int>& tiles, int n_lb, int G, std::vector<LaunchUnit>& units) {
     units.clear();
     int max_tiles = 0;

@@ -24,8 +24,9 @@
 // publisher warp adds each s * 2^m in fp64 to the unit's accumulator with one atomic add and
 // counts the item's arrival on the unit's counter with a release (the wait for its adds to
 // land stays off pass 1's path).  A unit's lse per column is log2 of its accumulator once the
-// counter is complete: one read of N doubles, whatever the number of items.  fp64 holds 2^(+-1022), so a column's largest logit must lie within +-680 (natural
-// log units); beyond that the status word reports kDevRange.
+// counter is complete: one read of N doubles, whatever the number of items.  fp64 holds
+// 2^(+-1022), so a column's largest logit times log2 e must lie within +-990 (about +-686 in
+// natural log units); beyond that the status word reports kDevRange.
 //
 // One cooperative launch, one CTA per SM, 512 threads, warp-specialised:
 //   warp 0       the producer, one polling thread: takes the CTA's next item from the global
@@ -57,8 +58,9 @@ namespace ckv {
 
 namespace {
 
-constexpr int kP1Slots = 3;   // pass-1 ring (HBM)
-constexpr int kP2Slots = 2;   // pass-2 ring (L2)
+constexpr int kP1Slots = 2;   // pass-1 ring (HBM)
+constexpr int kP2Slots = 3;   // pass-2 ring (L2): pass 2 must outrun pass 1 after each exchange wait
+constexpr int kP1Prefetch = 0; // pass-1 tiles prefetched into L2 ahead of their load
 constexpr int kAcc = 4;       // TMEM accumulators per pass
 constexpr int kQBufs = 3;     // query-row buffers: pass 1 runs up to two items ahead of pass 2
 constexpr int kItemRing = 8;  // item indices posted by the producer (more than any role's lag)
@@ -332,6 +334,15 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
                     tma_load_3d(d + SL::kQHalf, qm, &q_full[qb], 64, h, row);
                 }
             };
+            // Tile t of an item into L2 ahead of its pass-1 load (the ring holds only kP1Slots
+            // tiles in flight; the prefetches add more without shared memory)
+            auto prefetch_tile = [&](const Item& I, int t) {
+                const int g = p.batch_group[I.batch];
+                const int tok = I.start + (I.tile0 + t) * kTileKeys;
+                const CUtensorMap* km = &p.tmap_k[I.layer];
+                tma_prefetch_l2_3d(km, 0, g, tok, pol1);
+                tma_prefetch_l2_3d(km, 64, g, tok, pol1);
+            };
             // it1: items taken (pass-1 cursor on the last one); it2: pass-2 cursor
             int it1 = 0, jt1 = 0, use1 = 0, it2 = 0, jt2 = 0, use2 = 0, have2 = -1;
             Item I1{}, I2{};
@@ -355,6 +366,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
                             load_q(I1, qb);
                             have1 = true;
                             jt1 = 0;
+                            for (int t = 0; t < kP1Prefetch && t < I1.ntiles; ++t) prefetch_tile(I1, t);
                         }
                         did = true;
                     }
@@ -369,6 +381,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
                         const CUtensorMap* km = &p.tmap_k[I1.layer];
                         tma_load_3d_hint(dst, km, &full1[s], 0, g, tok, pol1);
                         tma_load_3d_hint(dst + kHalfBytes, km, &full1[s], 64, g, tok, pol1);
+                        if (kP1Prefetch > 0 && jt1 + kP1Prefetch < I1.ntiles) prefetch_tile(I1, jt1 + kP1Prefetch);
                         ++use1;
                         did = true;
                         if (++jt1 == I1.ntiles) {
@@ -490,8 +503,8 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
     } else if (warp == 3) {
         // ------------------------------------------------------------ publisher
         // Per item: once both pass-1 warpgroups have left its column sums (pub_full), lane l
-        // adds columns l and l + 32 to the unit's fp64 accumulator, every lane fences its adds,
-        // and lane 0 releases the item's arrival on the unit's counter.
+        // adds columns l and l + 32 to the unit's fp64 accumulator, and lane 0 releases the
+        // item's arrival on the unit's counter after a warp barrier.
         bool ok = true;
         for (int it = 0;; ++it) {
             int gi = -1, good = 1;
@@ -518,7 +531,8 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
                     else atomicAdd(dst + c, scaled_sum(ms.x, ms.y));
                 }
             }
-            __threadfence();  // this lane's adds are performed before the release below
+            // the warp barrier orders every lane's adds before lane 0's release, and a release
+            // is cumulative: a thread that acquires the count sees the adds of every item counted
             __syncwarp();
             if (lane == 0) {
                 red_release_add(p.counters + I.unit, 1);

@@ -1052,6 +1052,116 @@ __global__ void __launch_bounds__(256) gather_kernel(const __grid_constant__ Gat
     *dst = __ldg(src);
 }
 
+// ------------------------------------------------------------------ vectorised stage
+// A stage of one score row for chunk positions base-4 .. base+n+3 (element e = position
+// base-4+e) in 16-byte groups: group c of the row sits at group c ^ ((c >> 3) & 3), an XOR of
+// its low two bits that keeps every group whole (so that it is copied by one 16-byte cp.async)
+// and makes the six 16-byte reads of a thread's 24 elements (below) hit distinct bank groups
+// in every quarter-warp.
+__device__ __forceinline__ int sidx_sw(int e) {
+    const int c = e >> 2;
+    return ((c ^ ((c >> 3) & 3)) << 2) | (e & 3);
+}
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+__device__ __forceinline__ void cp_async16(float* dst, const float* src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+
+// Issues the copies that stage score rows ra .. ra+nr-1 for the n positions from `base` (row i
+// at st + i*words, the layout above; zero outside [0, P)) and commits them as one group.  Every
+// row start (scores + r*T + t0) is 16-byte aligned and base is a multiple of 4 (checked by the
+// caller), so a group inside [0, P) is one 16-byte copy; the at most two groups that straddle
+// 0 or P are read element by element.
+template <int NT>
+__device__ __forceinline__ void stage_rows_issue16(float* st, int words, const float* scores, size_t T,
+                                                   int t0, int ra, int nr, int base, int n, int P) {
+    const int ng = (n + 8 + 3) >> 2;  // groups of the n positions and 4 on each side
+    for (int i = 0; i < nr; ++i) {
+        const float* row = scores + static_cast<size_t>(ra + i) * T + t0;
+        float* dst = st + i * words;
+        for (int g = threadIdx.x; g < ng; g += NT) {
+            const int u0 = base - 4 + 4 * g;  // position of the group's first element
+            float* d = dst + sidx_sw(4 * g);
+            if (u0 >= 0 && u0 + 4 <= P) {
+                cp_async16(d, row + u0);
+            } else {
+                float4 v;
+                v.x = (u0 >= 0 && u0 < P) ? __ldg(row + u0) : 0.f;
+                v.y = (u0 + 1 >= 0 && u0 + 1 < P) ? __ldg(row + u0 + 1) : 0.f;
+                v.z = (u0 + 2 >= 0 && u0 + 2 < P) ? __ldg(row + u0 + 2) : 0.f;
+                v.w = (u0 + 3 >= 0 && u0 + 3 < P) ? __ldg(row + u0 + 3) : 0.f;
+                *reinterpret_cast<float4*>(d) = v;
+            }
+        }
+    }
+    cp_async_commit();
+}
+
+// Pools the PER = 16 outputs of thread t (positions base+16t .. base+16t+15) from one row
+// staged by stage_rows_issue16: its 24 elements 16t .. 16t+23 in six 16-byte reads; output i
+// covers elements 16t+i+4-HALF .. 16t+i+4+HALF.  The same arithmetic, in the same order, as
+// pool_window.
+template <int HALF, int PER>
+__device__ __forceinline__ void pool_window16(const float* st, int t, int nvalid, bool is_max, float kf,
+                                              float (&acc)[PER]) {
+    static_assert(PER == 16 && HALF >= 0 && HALF <= 4, "window");
+    float w[24];
+#pragma unroll
+    for (int q = 0; q < 6; ++q) {
+        const float4 x = *reinterpret_cast<const float4*>(st + sidx_sw(16 * t + 4 * q));
+        w[4 * q] = x.x;
+        w[4 * q + 1] = x.y;
+        w[4 * q + 2] = x.z;
+        w[4 * q + 3] = x.w;
+    }
+    if (is_max) {
+        // maxima of three neighbours, shared by the windows that contain them (a maximum is
+        // exact in any order)
+        float m3[22];
+#pragma unroll
+        for (int j = 0; j < 22; ++j) m3[j] = fmax3(w[j], w[j + 1], w[j + 2]);
+#pragma unroll
+        for (int i = 0; i < PER; ++i) {
+            if (i < nvalid) {
+                constexpr int W = 2 * HALF + 1;
+                const int s0 = i + 4 - HALF;
+                float m;
+                if (W == 1) m = w[s0];
+                else if (W == 3) m = m3[s0];
+                else if (W == 5) m = fmax3(m3[s0], w[s0 + 3], w[s0 + 4]);
+                else if (W == 7) m = fmax3(m3[s0], m3[s0 + 3], w[s0 + 6]);
+                else m = fmax3(m3[s0], m3[s0 + 3], m3[s0 + 6]);
+                acc[i] += m;
+            }
+        }
+    } else {
+#pragma unroll
+        for (int i = 0; i < PER; ++i) {
+            if (i < nvalid) {
+                float m = w[i + 4 - HALF];
+#pragma unroll
+                for (int d = 1; d <= 2 * HALF; ++d) m += w[i + 4 - HALF + d];
+                acc[i] += m / kf;  // IEEE division, as in pool_kernel
+            }
+        }
+    }
+}
+
+template <int PER>
+__device__ __forceinline__ void pool_any16(const float* st, int t, int nvalid, int half, bool is_max,
+                                           float kf, float (&acc)[PER]) {
+    if (nvalid <= 0) return;
+    if (half == 3) pool_window16<3, PER>(st, t, nvalid, is_max, kf, acc);
+    else if (half == 2) pool_window16<2, PER>(st, t, nvalid, is_max, kf, acc);
+    else if (half == 1) pool_window16<1, PER>(st, t, nvalid, is_max, kf, acc);
+    else if (half == 0) pool_window16<0, PER>(st, t, nvalid, is_max, kf, acc);
+    else pool_window16<4, PER>(st, t, nvalid, is_max, kf, acc);
+}
+
 // ------------------------------------------------------------------ many layers at once
 // Selection of every (layer, sequence, selection) unit of a multi-layer call in one launch:
 // the CTAs take units from a global counter, and one CTA does a unit whole, streaming over its
@@ -1072,6 +1182,8 @@ constexpr int kLsChunk = kLsThreads * kLsPer;                    // 8192 positio
 constexpr int kLsStageFloats = kLsChunk + 2 * kMaxHalo;
 constexpr int kLsStageLoads = (kLsStageFloats + kLsThreads - 1) / kLsThreads;
 constexpr int kLsWords = 4 * stage_words(kLsStageFloats);        // four score rows at once
+constexpr int kLs16Words = kLsChunk + 32;                        // a row of the 16-byte stage
+constexpr int kLsList = kLsWords;                                // kept positions gathered at once
 constexpr int kLsSmem = kLsWords * 4;
 constexpr int kLsCand = 2048;   // keys sharing the k-th key's first digit gathered in shared memory
 constexpr int kLsTies = 256;    // keys equal to the k-th key ranked by position in shared memory
@@ -1167,9 +1279,18 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
         // chunk's rows are copied in while this chunk is pooled (two buffers of nr rows).
         const int half = p.pool_kernel >> 1;
         const int r0 = p.group_first[u.g], nr = p.group_first[u.g + 1] - r0;
-        const int words = stage_words(kLsChunk + 2 * half);
-        const bool piped = p.from_scores && p.head_order == 0 && 2 * nr * words + PER <= kLsWords;
-        if (piped)
+        // 16-byte staging when every row of the unit starts 16-byte aligned and the pooling
+        // window fits a thread's 24 staged elements; else 4-byte copies in the padded layout
+        bool aligned = true;
+        for (int i = 0; i < nr; ++i)
+            aligned = aligned && ((reinterpret_cast<uintptr_t>(p.scores + static_cast<size_t>(r0 + i) * p.T + u.t0) & 15u) == 0);
+        const bool v16 = p.from_scores && p.head_order == 0 && half <= 4 && aligned &&
+                         2 * nr * kLs16Words <= kLsWords;
+        const int words = v16 ? kLs16Words : stage_words(kLsChunk + 2 * half);
+        const bool piped = v16 || (p.from_scores && p.head_order == 0 && 2 * nr * words + PER <= kLsWords);
+        if (v16)
+            stage_rows_issue16<NT>(st, words, p.scores, p.T, u.t0, r0, nr, 0, min(kLsChunk, Pn), u.P);
+        else if (piped)
             stage_rows_issue<NT, kLsStageLoads>(st, words, p.scores, p.T, u.t0, r0, nr, 0, half,
                                                 min(kLsChunk, Pn), u.P);
         __syncthreads();
@@ -1180,9 +1301,13 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
             if (piped) {
                 const float* cur = st + (c & 1) * nr * words;
                 if (base + kLsChunk < Pn) {
-                    stage_rows_issue<NT, kLsStageLoads>(st + ((c + 1) & 1) * nr * words, words, p.scores,
-                                                        p.T, u.t0, r0, nr, base + kLsChunk, half,
-                                                        min(kLsChunk, Pn - base - kLsChunk), u.P);
+                    float* nxt_st = st + ((c + 1) & 1) * nr * words;
+                    const int nn = min(kLsChunk, Pn - base - kLsChunk);
+                    if (v16)
+                        stage_rows_issue16<NT>(nxt_st, words, p.scores, p.T, u.t0, r0, nr, base + kLsChunk, nn, u.P);
+                    else
+                        stage_rows_issue<NT, kLsStageLoads>(nxt_st, words, p.scores, p.T, u.t0, r0, nr,
+                                                            base + kLsChunk, half, nn, u.P);
                     cp_async_wait_group<1>();
                 } else {
                     cp_async_wait_group<0>();
@@ -1190,9 +1315,14 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
                 __syncthreads();
 #pragma unroll
                 for (int i = 0; i < PER; ++i) acc[i] = 0.f;
-                for (int i = 0; i < nr; ++i)
-                    pool_any<PER>(cur + i * words, jb, nvalid, half, p.pool_type == 0,
-                                  static_cast<float>(p.pool_kernel), acc);
+                for (int i = 0; i < nr; ++i) {
+                    if (v16)
+                        pool_any16<PER>(cur + i * words, tid, nvalid, half, p.pool_type == 0,
+                                        static_cast<float>(p.pool_kernel), acc);
+                    else
+                        pool_any<PER>(cur + i * words, jb, nvalid, half, p.pool_type == 0,
+                                      static_cast<float>(p.pool_kernel), acc);
+                }
             } else {
                 pooled_values<NT, PER, kLsStageLoads, kLsWords>(p, u, st, base, n, acc);
             }
@@ -1342,8 +1472,10 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
                 }
             }
         }
-        // (C) the kept positions in order, chunk by chunk, with their K/V rows; then the window
-        int written = 0;
+        // (C) the kept positions in order, chunk by chunk, gathered in the list (the stage is
+        // free now) and written out with their K/V rows when it is full and at the end, so that
+        // the rows' copies of many chunks share one round trip; then the window
+        int written = 0, lbase = 0, lcount = 0;  // list[0..lcount) are output rows lbase..
         uint32_t key[PER];  // this chunk's keys; the next chunk's are loaded meanwhile
         load_keys(keys, tid * PER, min(kLsChunk, Pn) - tid * PER, key);
         for (int base = 0; base < Pn; base += kLsChunk) {
@@ -1363,6 +1495,13 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
             int tot;
             int rk = block_excl_scan<NT>(cnt, scratch, &tot);
             if (written + tot > k) break;  // checked below
+            if (lcount + tot > kLsList) {  // block-uniform: write out the list first
+                emit_kept(p, u, list, lcount, lbase, kv0, kv1);
+                lbase += lcount;
+                lcount = 0;
+                __syncthreads();
+            }
+            rk += lcount;
 #pragma unroll
             for (int i = 0; i < PER; ++i) {
                 if ((taken >> i) & 1u) {
@@ -1370,20 +1509,26 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
                     ++rk;
                 }
             }
-            __syncthreads();
-            emit_kept(p, u, list, tot, written, kv0, kv1);
+            lcount += tot;
             written += tot;
-            __syncthreads();
 #pragma unroll
             for (int i = 0; i < PER; ++i) key[i] = nxt[i];
         }
         if (written != k) {
             if (tid == 0) record_error(p.status, kDevBadIndex, 340 + unit);
+            __syncthreads();  // every thread is done with the list before the next unit
             continue;
         }
-        for (int i = tid; i < p.w; i += NT) list[i] = Pn + i;
+        if (lcount + p.w > kLsList) {
+            __syncthreads();
+            emit_kept(p, u, list, lcount, lbase, kv0, kv1);
+            lbase += lcount;
+            lcount = 0;
+            __syncthreads();
+        }
+        for (int i = tid; i < p.w; i += NT) list[lcount + i] = Pn + i;
         __syncthreads();
-        emit_kept(p, u, list, p.w, k, kv0, kv1);
+        emit_kept(p, u, list, lcount + p.w, lbase, kv0, kv1);
         __syncthreads();
     }
 }
