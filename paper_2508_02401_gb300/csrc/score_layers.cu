@@ -60,7 +60,6 @@ namespace {
 
 constexpr int kP1Slots = 2;   // pass-1 ring (HBM)
 constexpr int kP2Slots = 3;   // pass-2 ring (L2): pass 2 must outrun pass 1 after each exchange wait
-constexpr int kP1Prefetch = 0; // pass-1 tiles prefetched into L2 ahead of their load
 constexpr int kAcc = 4;       // TMEM accumulators per pass
 constexpr int kQBufs = 3;     // query-row buffers: pass 1 runs up to two items ahead of pass 2
 constexpr int kItemRing = 8;  // item indices posted by the producer (more than any role's lag)
@@ -334,15 +333,6 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
                     tma_load_3d(d + SL::kQHalf, qm, &q_full[qb], 64, h, row);
                 }
             };
-            // Tile t of an item into L2 ahead of its pass-1 load (the ring holds only kP1Slots
-            // tiles in flight; the prefetches add more without shared memory)
-            auto prefetch_tile = [&](const Item& I, int t) {
-                const int g = p.batch_group[I.batch];
-                const int tok = I.start + (I.tile0 + t) * kTileKeys;
-                const CUtensorMap* km = &p.tmap_k[I.layer];
-                tma_prefetch_l2_3d(km, 0, g, tok, pol1);
-                tma_prefetch_l2_3d(km, 64, g, tok, pol1);
-            };
             // it1: items taken (pass-1 cursor on the last one); it2: pass-2 cursor
             int it1 = 0, jt1 = 0, use1 = 0, it2 = 0, jt2 = 0, use2 = 0, have2 = -1;
             Item I1{}, I2{};
@@ -366,7 +356,6 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
                             load_q(I1, qb);
                             have1 = true;
                             jt1 = 0;
-                            for (int t = 0; t < kP1Prefetch && t < I1.ntiles; ++t) prefetch_tile(I1, t);
                         }
                         did = true;
                     }
@@ -381,7 +370,6 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
                         const CUtensorMap* km = &p.tmap_k[I1.layer];
                         tma_load_3d_hint(dst, km, &full1[s], 0, g, tok, pol1);
                         tma_load_3d_hint(dst + kHalfBytes, km, &full1[s], 64, g, tok, pol1);
-                        if (kP1Prefetch > 0 && jt1 + kP1Prefetch < I1.ntiles) prefetch_tile(I1, jt1 + kP1Prefetch);
                         ++use1;
                         did = true;
                         if (++jt1 == I1.ntiles) {

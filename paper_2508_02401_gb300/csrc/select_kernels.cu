@@ -440,9 +440,10 @@ __device__ __forceinline__ void pooled_values(const SelectParams& p, const UnitG
 
 // Copies the K and V rows of sequence-local positions list[0..m) to output rows
 // out_row0 + 0..m-1 of KV head g: a warp per row (16 lanes for K, 16 for V), kRowsInFlight
-// rows in flight per warp.
+// rows in flight per warp (not inlined: the rows in flight then stay in registers whatever the
+// caller holds).
 constexpr int kRowsInFlight = 8;
-__device__ __forceinline__ void copy_rows(const SelectParams& p, const UnitGeo& u, int kv,
+__device__ __noinline__ void copy_rows(const SelectParams& p, const UnitGeo& u, int kv,
                                           const int* list, int m, int out_row0) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
     const int part = lane & 15;
@@ -1183,7 +1184,10 @@ constexpr int kLsStageFloats = kLsChunk + 2 * kMaxHalo;
 constexpr int kLsStageLoads = (kLsStageFloats + kLsThreads - 1) / kLsThreads;
 constexpr int kLsWords = 4 * stage_words(kLsStageFloats);        // four score rows at once
 constexpr int kLs16Words = kLsChunk + 32;                        // a row of the 16-byte stage
-constexpr int kLsList = kLsWords;                                // kept positions gathered at once
+constexpr int kKeyBufs = 3;                                      // key chunks in flight in (B), (C)
+constexpr int kKeyRingWords = kKeyBufs * kLsChunk;
+constexpr int kLsList = kLsWords - kKeyRingWords;                // kept positions gathered at once
+static_assert(kLsList >= kLsChunk, "a chunk's kept positions fit the list");
 constexpr int kLsSmem = kLsWords * 4;
 constexpr int kLsCand = 2048;   // keys sharing the k-th key's first digit gathered in shared memory
 constexpr int kLsTies = 256;    // keys equal to the k-th key ranked by position in shared memory
@@ -1191,9 +1195,10 @@ constexpr int kSelMaxLayers = 32;
 
 struct SelectLayersParams {
     SelectParams layer[kSelMaxLayers];
-    uint32_t* keys[kSelMaxLayers];   // per layer [n_vec, T]: the keys of the pooled scores
+    uint32_t* keys[kSelMaxLayers];   // per layer [n_vec, key_stride]: the keys of the pooled scores
     int* next_unit;                  // work counter, zero at launch
     int n_layers, units_per_layer;   // units_per_layer = S * n_vec
+    int key_stride;                  // select_key_stride(T, S)
 };
 
 // The keys at src[jb .. jb + kLsPer) (zero past nvalid); 16-byte loads when src is 16-byte
@@ -1214,14 +1219,40 @@ __device__ __forceinline__ void load_keys(const uint32_t* src, int jb, int nvali
     }
 }
 
-// The keys of a thread in the chunk after the one at `base` (zeros when there is none).
-__device__ __forceinline__ void next_keys(const uint32_t* keys, int base, int Pn, int jb, uint32_t (&key)[kLsPer]) {
-    const int nb = base + kLsChunk;
-    if (nb < Pn) {
-        load_keys(keys + nb, jb, min(kLsChunk, Pn - nb) - jb, key);
-    } else {
+// Issues the 16-byte copies of chunk c of a unit's keys (Pn of them, 16-byte aligned) into ring
+// buffer c % kKeyBufs, in the swizzled layout of the score stage, and commits them as one
+// group: an empty group past the last chunk, so that every wait counts the same groups.
+__device__ __forceinline__ void issue_key_chunk(uint32_t* ring, const uint32_t* keys, int c, int Pn) {
+    const int base = c * kLsChunk;
+    if (base < Pn) {
+        const int n = min(kLsChunk, Pn - base);
+        float* dst = reinterpret_cast<float*>(ring + (c % kKeyBufs) * kLsChunk);
+        const float* src = reinterpret_cast<const float*>(keys + base);
+        const int ng = (n + 3) >> 2;
+        for (int g = threadIdx.x; g < ng; g += kLsThreads) {
+            if (4 * g + 4 <= n) {
+                cp_async16(dst + sidx_sw(4 * g), src + 4 * g);
+            } else {
 #pragma unroll
-        for (int i = 0; i < kLsPer; ++i) key[i] = 0u;
+                for (int e = 0; e < 4; ++e)
+                    if (4 * g + e < n) dst[sidx_sw(4 * g + e)] = __ldcg(src + 4 * g + e);
+            }
+        }
+    }
+    cp_async_commit();
+}
+
+// Thread t's 16 keys (chunk positions 16t .. 16t+15) from a ring buffer: four 16-byte reads,
+// free of bank conflicts in the swizzled layout.  Keys past the chunk's end are stale; the
+// callers read only the first nvalid.
+__device__ __forceinline__ void ring_keys(const uint32_t* buf, uint32_t (&key)[kLsPer]) {
+#pragma unroll
+    for (int q = 0; q < kLsPer / 4; ++q) {
+        const uint4 x = *reinterpret_cast<const uint4*>(buf + sidx_sw(16 * threadIdx.x + 4 * q));
+        key[4 * q] = x.x;
+        key[4 * q + 1] = x.y;
+        key[4 * q + 2] = x.z;
+        key[4 * q + 3] = x.w;
     }
 }
 
@@ -1255,7 +1286,8 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
             if (u.s == 0) p.cu_keep[0] = 0;
         }
         float* pooled = p.write_pooled ? p.pooled + static_cast<size_t>(u.g) * p.T + u.t0 : nullptr;
-        int* list = reinterpret_cast<int*>(st);
+        int* list = reinterpret_cast<int*>(st) + kKeyRingWords;  // after the key ring
+        uint32_t* ring = reinterpret_cast<uint32_t*>(st);
         if (u.L <= p.budget) {  // kept whole; its pooled scores read as 0
             for (int e0 = 0; e0 < u.L; e0 += kLsChunk) {
                 const int m = min(kLsChunk, u.L - e0);
@@ -1270,7 +1302,10 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
             continue;
         }
         const int Pn = u.P, k = u.k;
-        uint32_t* keys = P.keys[li] + static_cast<size_t>(u.g) * p.T + u.t0;
+        // the unit's keys: sequence s's segment starts at its first token rounded up to a
+        // multiple of 4, plus 4 s, so that every segment is 16-byte aligned
+        uint32_t* keys = P.keys[li] + static_cast<size_t>(u.g) * P.key_stride + ((u.t0 + 3) & ~3) + 4 * u.s;
+        const bool kring = (reinterpret_cast<uintptr_t>(keys) & 15u) == 0;
         if (pooled)  // window positions are not candidates
             for (int j = Pn + tid; j < u.L; j += NT) pooled[j] = 0.f;
         // (A) pooled scores, keys and first-digit counts, chunk by chunk
@@ -1372,21 +1407,28 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
             if (in_smem) {
                 if (tid == 0) s_cnt = 0;
                 __syncthreads();
-                uint32_t key[PER];  // this chunk's keys; the next chunk's are loaded meanwhile
-                load_keys(keys, tid * PER, min(kLsChunk, Pn) - tid * PER, key);
-                for (int base = 0; base < Pn; base += kLsChunk) {
+                uint32_t key[PER];
+                if (kring)  // chunks through the shared-memory ring, two ahead
+                    for (int c = 0; c < kKeyBufs - 1; ++c) issue_key_chunk(ring, keys, c, Pn);
+                for (int base = 0, ch = 0; base < Pn; base += kLsChunk, ++ch) {
                     const int jb = tid * PER, nvalid = min(kLsChunk, Pn - base) - jb;
-                    uint32_t nxt[PER];
-                    next_keys(keys, base, Pn, jb, nxt);
+                    if (kring) {
+                        issue_key_chunk(ring, keys, ch + kKeyBufs - 1, Pn);
+                        cp_async_wait_group<kKeyBufs - 1>();
+                        __syncthreads();
+                        ring_keys(ring + (ch % kKeyBufs) * kLsChunk, key);
+                    } else {
+                        load_keys(keys + base, jb, nvalid, key);
+                    }
 #pragma unroll
                     for (int i = 0; i < PER; ++i)
                         if (i < nvalid && (key[i] >> kHistShift) == d1) {
                             const int c = atomicAdd(&s_cnt, 1);
                             if (c < kLsCand) cand[c] = make_uint2(key[i], base + jb + i);
                         }
-#pragma unroll
-                    for (int i = 0; i < PER; ++i) key[i] = nxt[i];
+                    if (kring) __syncthreads();  // the buffer is refilled by the next issue
                 }
+                cp_async_wait_group<0>();
             }
             // Two more digits (11 and 10 bits) of the k-th key, by counts of the keys that share
             // the digits so far: over the gathered candidates or over the scratch row.
@@ -1476,12 +1518,20 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
         // free now) and written out with their K/V rows when it is full and at the end, so that
         // the rows' copies of many chunks share one round trip; then the window
         int written = 0, lbase = 0, lcount = 0;  // list[0..lcount) are output rows lbase..
-        uint32_t key[PER];  // this chunk's keys; the next chunk's are loaded meanwhile
-        load_keys(keys, tid * PER, min(kLsChunk, Pn) - tid * PER, key);
-        for (int base = 0; base < Pn; base += kLsChunk) {
+        uint32_t key[PER];
+        __syncthreads();  // (B) is done with the ring
+        if (kring)  // chunks through the shared-memory ring, two ahead
+            for (int c = 0; c < kKeyBufs - 1; ++c) issue_key_chunk(ring, keys, c, Pn);
+        for (int base = 0, ch = 0; base < Pn; base += kLsChunk, ++ch) {
             const int jb = tid * PER, nvalid = min(kLsChunk, Pn - base) - jb;
-            uint32_t nxt[PER];
-            next_keys(keys, base, Pn, jb, nxt);
+            if (kring) {
+                issue_key_chunk(ring, keys, ch + kKeyBufs - 1, Pn);
+                cp_async_wait_group<kKeyBufs - 1>();
+                __syncthreads();
+                ring_keys(ring + (ch % kKeyBufs) * kLsChunk, key);
+            } else {
+                load_keys(keys + base, jb, nvalid, key);
+            }
             uint32_t taken = 0;
             int cnt = 0;
 #pragma unroll
@@ -1511,9 +1561,10 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
             }
             lcount += tot;
             written += tot;
-#pragma unroll
-            for (int i = 0; i < PER; ++i) key[i] = nxt[i];
+            // (the block scan above ordered every read of this chunk's ring buffer before the
+            // issue that refills it)
         }
+        cp_async_wait_group<0>();
         if (written != k) {
             if (tid == 0) record_error(p.status, kDevBadIndex, 340 + unit);
             __syncthreads();  // every thread is done with the list before the next unit
@@ -1661,9 +1712,12 @@ cudaError_t launch_gather(const GatherLaunch& L, cudaStream_t stream) {
 }
 
 // The selection of several layers in one launch (select_layers_kernel); Ls[i] as for
-// launch_select with from_scores = 1, and keys[i] a [n_vec, T] scratch per layer.  One launch per
+// launch_select with from_scores = 1, and keys[i] a [n_vec, select_key_stride(T, S)] scratch
+// per layer.  One launch per
 // kSelMaxLayers layers; `next_unit` (kSelMaxLayers-aligned count of ints) is the work counter
 // of each launch and is cleared first.
+int select_key_stride(int T, int S) { return (T + 4 * S + 3) & ~3; }
+
 cudaError_t launch_select_layers(const SelectLaunch* Ls, uint32_t* const* keys, int n_layers,
                                  int* next_unit, int grid, cudaStream_t stream) {
     static SelectLayersParams P;  // ~25 KB; calls are serialised by `mu`
@@ -1713,6 +1767,7 @@ cudaError_t launch_select_layers(const SelectLaunch* Ls, uint32_t* const* keys, 
         }
         P.n_layers = nl;
         P.units_per_layer = Ls[l0].S * Ls[l0].n_vec;
+        P.key_stride = select_key_stride(Ls[l0].T, Ls[l0].S);
         P.next_unit = next_unit;
         const int units = nl * P.units_per_layer;
         if (units == 0) continue;
