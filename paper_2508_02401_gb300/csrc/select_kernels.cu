@@ -251,9 +251,10 @@ __device__ __forceinline__ void find_digit(const int* hist, int r, int* scratch,
 
 // Adds a thread's run-aggregated counts of PER consecutive digits to a shared histogram:
 // consecutive keys of a thread are neighbouring positions and often share a digit, so one
-// atomic add per run of equal digits (a linear scan) instead of one per key.
+// atomic add per run of equal digits (a linear scan) instead of one per key.  Digits below
+// `lo` are not counted.
 template <int PER>
-__device__ __forceinline__ void add_runs(int* hist, const uint32_t (&bins)[PER], int nvalid) {
+__device__ __forceinline__ void add_runs(int* hist, const uint32_t (&bins)[PER], int nvalid, uint32_t lo = 0) {
     if (nvalid <= 0) return;
     uint32_t cur = bins[0];
     int len = 1;
@@ -263,13 +264,13 @@ __device__ __forceinline__ void add_runs(int* hist, const uint32_t (&bins)[PER],
             if (bins[i] == cur) {
                 ++len;
             } else {
-                atomicAdd(&hist[cur], len);
+                if (cur >= lo) atomicAdd(&hist[cur], len);
                 cur = bins[i];
                 len = 1;
             }
         }
     }
-    atomicAdd(&hist[cur], len);
+    if (cur >= lo) atomicAdd(&hist[cur], len);
 }
 
 // Stages the sum of score rows [ra, rb) at sequence positions base-half .. base+n+half-1
@@ -1329,6 +1330,7 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
             stage_rows_issue<NT, kLsStageLoads>(st, words, p.scores, p.T, u.t0, r0, nr, 0, half,
                                                 min(kLsChunk, Pn), u.P);
         __syncthreads();
+        uint32_t lo = 0;  // the lowest first digit counted (see below)
         for (int base = 0, c = 0; base < Pn; base += kLsChunk, ++c) {
             const int n = min(kLsChunk, Pn - base);
             const int jb = tid * PER, nvalid = n - jb;
@@ -1386,8 +1388,17 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
                         if (pooled) pooled[base + jb + i] = acc[i];
                     }
             }
-            add_runs<PER>(hist, bins, nvalid);
+            add_runs<PER>(hist, bins, nvalid, lo);
             if (piped) __syncthreads();  // every thread is done with this chunk's buffer
+            if (c == 0 && k > 0 && Pn > kLsChunk) {
+                // The k-th largest key of the first chunk bounds the k-th largest of the unit
+                // from below, so the later chunks count only digits at or above its digit: the
+                // counts the threshold search reads (at or above the final digit) stay exact,
+                // and the bulk of small scores costs no atomic.
+                __syncthreads();
+                find_digit<NT>(hist, k, scratch, &s_digit, &s_above);
+                lo = static_cast<uint32_t>(s_digit);  // 0 when the chunk holds fewer than k keys
+            }
         }
         __syncthreads();  // also orders the key stores before the reads below (same block)
         // (B) the k-th largest key thr, and the last position cut of a kept key equal to it
