@@ -249,23 +249,24 @@ __device__ __forceinline__ void find_digit(const int* hist, int r, int* scratch,
     __syncthreads();
 }
 
-// Adds a thread's run-aggregated counts of PER consecutive digits to a shared histogram:
-// consecutive keys of a thread are neighbouring positions and often share a digit, so one
-// atomic add per run of equal digits (a linear scan) instead of one per key.  Digits below
-// `lo` are not counted.
-template <int PER>
-__device__ __forceinline__ void add_runs(int* hist, const uint32_t (&bins)[PER], int nvalid, uint32_t lo = 0) {
+// Adds a thread's run-aggregated counts of PER consecutive digits (v[i] >> SHIFT) to a shared
+// histogram: consecutive keys of a thread are neighbouring positions and often share a digit,
+// so one atomic add per run of equal digits (a linear scan) instead of one per key.  Digits
+// below `lo` are not counted.
+template <int PER, int SHIFT = 0>
+__device__ __forceinline__ void add_runs(int* hist, const uint32_t (&v)[PER], int nvalid, uint32_t lo = 0) {
     if (nvalid <= 0) return;
-    uint32_t cur = bins[0];
+    uint32_t cur = v[0] >> SHIFT;
     int len = 1;
 #pragma unroll
     for (int i = 1; i < PER; ++i) {
         if (i < nvalid) {
-            if (bins[i] == cur) {
+            const uint32_t d = v[i] >> SHIFT;
+            if (d == cur) {
                 ++len;
             } else {
                 if (cur >= lo) atomicAdd(&hist[cur], len);
-                cur = bins[i];
+                cur = d;
                 len = 1;
             }
         }
@@ -1168,16 +1169,20 @@ __device__ __forceinline__ void pool_any16(const float* st, int t, int nvalid, i
 // Selection of every (layer, sequence, selection) unit of a multi-layer call in one launch:
 // the CTAs take units from a global counter, and one CTA does a unit whole, streaming over its
 // candidate positions in chunks of kLsChunk (so that no length is too long and little sits in
-// shared memory): (A) pools the chunk (the next chunk's score rows copied in meanwhile),
-// stores its order-preserving keys in a scratch row (and the pooled scores when asked) and
-// counts their first digits; the k-th largest key's digit follows from the counts; (B) refines
-// the threshold by two more digits (11 and 10 bits), counting over the keys that share the
-// digits so far: gathered into shared memory when at most kLsCand share the first digit, else
-// read again from the scratch row; the tie cutoff among keys equal to the threshold is their
-// rank by position, in shared memory when at most kLsTies were gathered, else by a
-// position-ordered scan of the scratch row; (C) writes the kept positions in order, a chunk at
-// a time (a block scan per chunk), copies their K/V rows, and appends the window.  The same
-// keys, ties and order as select_unit_kernel and the chunked kernels.
+// shared memory):
+//  (A) pools the chunk (the next chunk's score rows copied in meanwhile), counts the first
+//      digits of its order-preserving keys, and appends the keys that can still be kept, with
+//      their positions, to the unit's candidate list in a scratch row: once the chunks so far
+//      hold k keys, the first digit of their k-th largest bounds the unit's k-th largest from
+//      below, and keys under it are neither counted nor listed;
+//  (B) finds the k-th largest key from the counts (the first digit) and two more digits (11 and
+//      10 bits) counted over the candidates with the digits so far: gathered into shared memory
+//      when at most kLsCand share the first digit, else read from the list; the tie cutoff
+//      among keys equal to the threshold is their rank by position, in shared memory when at
+//      most kLsTies were gathered, else by a scan of the list (which is in position order);
+//  (C) writes the kept candidates' positions in order (a block scan per kLsChunk of the list)
+//      with their K/V rows, and appends the window.
+// The same keys, ties and order as select_unit_kernel and the chunked kernels.
 constexpr int kLsThreads = 512;
 constexpr int kLsPer = 16;
 constexpr int kLsChunk = kLsThreads * kLsPer;                    // 8192 positions
@@ -1185,9 +1190,7 @@ constexpr int kLsStageFloats = kLsChunk + 2 * kMaxHalo;
 constexpr int kLsStageLoads = (kLsStageFloats + kLsThreads - 1) / kLsThreads;
 constexpr int kLsWords = 4 * stage_words(kLsStageFloats);        // four score rows at once
 constexpr int kLs16Words = kLsChunk + 32;                        // a row of the 16-byte stage
-constexpr int kKeyBufs = 3;                                      // key chunks in flight in (B), (C)
-constexpr int kKeyRingWords = kKeyBufs * kLsChunk;
-constexpr int kLsList = kLsWords - kKeyRingWords;                // kept positions gathered at once
+constexpr int kLsList = kLsWords;                                // kept positions gathered at once
 static_assert(kLsList >= kLsChunk, "a chunk's kept positions fit the list");
 constexpr int kLsSmem = kLsWords * 4;
 constexpr int kLsCand = 2048;   // keys sharing the k-th key's first digit gathered in shared memory
@@ -1196,66 +1199,11 @@ constexpr int kSelMaxLayers = 32;
 
 struct SelectLayersParams {
     SelectParams layer[kSelMaxLayers];
-    uint32_t* keys[kSelMaxLayers];   // per layer [n_vec, key_stride]: the keys of the pooled scores
+    uint2* cands[kSelMaxLayers];     // per layer [n_vec, key_stride]: (key, position) candidates
     int* next_unit;                  // work counter, zero at launch
     int n_layers, units_per_layer;   // units_per_layer = S * n_vec
     int key_stride;                  // select_key_stride(T, S)
 };
-
-// The keys at src[jb .. jb + kLsPer) (zero past nvalid); 16-byte loads when src is 16-byte
-// aligned (jb is a multiple of kLsPer).
-__device__ __forceinline__ void load_keys(const uint32_t* src, int jb, int nvalid, uint32_t (&key)[kLsPer]) {
-    if (nvalid >= kLsPer && (reinterpret_cast<uintptr_t>(src) & 15u) == 0) {
-#pragma unroll
-        for (int q = 0; q < kLsPer / 4; ++q) {
-            const uint4 x = __ldcg(reinterpret_cast<const uint4*>(src + jb) + q);
-            key[4 * q] = x.x;
-            key[4 * q + 1] = x.y;
-            key[4 * q + 2] = x.z;
-            key[4 * q + 3] = x.w;
-        }
-    } else {
-#pragma unroll
-        for (int i = 0; i < kLsPer; ++i) key[i] = i < nvalid ? __ldcg(src + jb + i) : 0u;
-    }
-}
-
-// Issues the 16-byte copies of chunk c of a unit's keys (Pn of them, 16-byte aligned) into ring
-// buffer c % kKeyBufs, in the swizzled layout of the score stage, and commits them as one
-// group: an empty group past the last chunk, so that every wait counts the same groups.
-__device__ __forceinline__ void issue_key_chunk(uint32_t* ring, const uint32_t* keys, int c, int Pn) {
-    const int base = c * kLsChunk;
-    if (base < Pn) {
-        const int n = min(kLsChunk, Pn - base);
-        float* dst = reinterpret_cast<float*>(ring + (c % kKeyBufs) * kLsChunk);
-        const float* src = reinterpret_cast<const float*>(keys + base);
-        const int ng = (n + 3) >> 2;
-        for (int g = threadIdx.x; g < ng; g += kLsThreads) {
-            if (4 * g + 4 <= n) {
-                cp_async16(dst + sidx_sw(4 * g), src + 4 * g);
-            } else {
-#pragma unroll
-                for (int e = 0; e < 4; ++e)
-                    if (4 * g + e < n) dst[sidx_sw(4 * g + e)] = __ldcg(src + 4 * g + e);
-            }
-        }
-    }
-    cp_async_commit();
-}
-
-// Thread t's 16 keys (chunk positions 16t .. 16t+15) from a ring buffer: four 16-byte reads,
-// free of bank conflicts in the swizzled layout.  Keys past the chunk's end are stale; the
-// callers read only the first nvalid.
-__device__ __forceinline__ void ring_keys(const uint32_t* buf, uint32_t (&key)[kLsPer]) {
-#pragma unroll
-    for (int q = 0; q < kLsPer / 4; ++q) {
-        const uint4 x = *reinterpret_cast<const uint4*>(buf + sidx_sw(16 * threadIdx.x + 4 * q));
-        key[4 * q] = x.x;
-        key[4 * q + 1] = x.y;
-        key[4 * q + 2] = x.z;
-        key[4 * q + 3] = x.w;
-    }
-}
 
 __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __grid_constant__ SelectLayersParams P) {
     extern __shared__ __align__(16) float st[];  // pooling stage; the kept list of a chunk
@@ -1287,8 +1235,7 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
             if (u.s == 0) p.cu_keep[0] = 0;
         }
         float* pooled = p.write_pooled ? p.pooled + static_cast<size_t>(u.g) * p.T + u.t0 : nullptr;
-        int* list = reinterpret_cast<int*>(st) + kKeyRingWords;  // after the key ring
-        uint32_t* ring = reinterpret_cast<uint32_t*>(st);
+        int* list = reinterpret_cast<int*>(st);
         if (u.L <= p.budget) {  // kept whole; its pooled scores read as 0
             for (int e0 = 0; e0 < u.L; e0 += kLsChunk) {
                 const int m = min(kLsChunk, u.L - e0);
@@ -1303,10 +1250,11 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
             continue;
         }
         const int Pn = u.P, k = u.k;
-        // the unit's keys: sequence s's segment starts at its first token rounded up to a
-        // multiple of 4, plus 4 s, so that every segment is 16-byte aligned
-        uint32_t* keys = P.keys[li] + static_cast<size_t>(u.g) * P.key_stride + ((u.t0 + 3) & ~3) + 4 * u.s;
-        const bool kring = (reinterpret_cast<uintptr_t>(keys) & 15u) == 0;
+        // the unit's candidate list of (key, position) pairs: sequence s's segment of the
+        // scratch row starts at its first token rounded up to a multiple of 4, plus 4 s, so that
+        // every segment is 32-byte aligned and holds the sequence's P candidates at most
+        uint2* cands = P.cands[li] + static_cast<size_t>(u.g) * P.key_stride + ((u.t0 + 3) & ~3) + 4 * u.s;
+        int n_cand = 0;
         if (pooled)  // window positions are not candidates
             for (int j = Pn + tid; j < u.L; j += NT) pooled[j] = 0.f;
         // (A) pooled scores, keys and first-digit counts, chunk by chunk
@@ -1363,44 +1311,46 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
             } else {
                 pooled_values<NT, PER, kLsStageLoads, kLsWords>(p, u, st, base, n, acc);
             }
-            uint32_t key[PER], bins[PER];
+            uint32_t key[PER];  // first digit: key >> kHistShift
 #pragma unroll
-            for (int i = 0; i < PER; ++i) {
-                key[i] = rank_key(acc[i]);
-                bins[i] = key[i] >> kHistShift;
-            }
-            // 16-byte stores where the rows are 16-byte aligned (base + jb is a multiple of 16)
-            if (nvalid >= PER && (reinterpret_cast<uintptr_t>(keys) & 15u) == 0 &&
-                (!pooled || (reinterpret_cast<uintptr_t>(pooled) & 15u) == 0)) {
+            for (int i = 0; i < PER; ++i) key[i] = rank_key(acc[i]);
+            if (pooled) {  // 16-byte stores where the row is 16-byte aligned
+                if (nvalid >= PER && (reinterpret_cast<uintptr_t>(pooled) & 15u) == 0) {
 #pragma unroll
-                for (int q = 0; q < PER / 4; ++q) {
-                    reinterpret_cast<uint4*>(keys + base + jb)[q] =
-                        make_uint4(key[4 * q], key[4 * q + 1], key[4 * q + 2], key[4 * q + 3]);
-                    if (pooled)
+                    for (int q = 0; q < PER / 4; ++q)
                         reinterpret_cast<float4*>(pooled + base + jb)[q] =
                             make_float4(acc[4 * q], acc[4 * q + 1], acc[4 * q + 2], acc[4 * q + 3]);
-                }
-            } else {
+                } else {
 #pragma unroll
-                for (int i = 0; i < PER; ++i)
-                    if (i < nvalid) {
-                        keys[base + jb + i] = key[i];
-                        if (pooled) pooled[base + jb + i] = acc[i];
-                    }
+                    for (int i = 0; i < PER; ++i)
+                        if (i < nvalid) pooled[base + jb + i] = acc[i];
+                }
             }
-            add_runs<PER>(hist, bins, nvalid, lo);
-            if (piped) __syncthreads();  // every thread is done with this chunk's buffer
-            if (c == 0 && k > 0 && Pn > kLsChunk) {
-                // The k-th largest key of the first chunk bounds the k-th largest of the unit
-                // from below, so the later chunks count only digits at or above its digit: the
-                // counts the threshold search reads (at or above the final digit) stay exact,
-                // and the bulk of small scores costs no atomic.
+            add_runs<PER, kHistShift>(hist, key, nvalid, lo);
+            if (lo == 0 && k > 0) {
+                // The k-th largest key of the chunks so far bounds the unit's k-th largest from
+                // below: later chunks count only first digits at or above its digit (the counts
+                // that the threshold search reads stay exact, and the bulk of small scores costs
+                // no atomic), and only keys there can be kept.
                 __syncthreads();
                 find_digit<NT>(hist, k, scratch, &s_digit, &s_above);
-                lo = static_cast<uint32_t>(s_digit);  // 0 when the chunk holds fewer than k keys
+                lo = static_cast<uint32_t>(s_digit);  // 0 while fewer than k keys are counted
             }
+            if (k > 0) {  // the candidates, in position order: keys whose first digit is >= lo
+                int cnt = 0;
+#pragma unroll
+                for (int i = 0; i < PER; ++i) cnt += (i < nvalid && (key[i] >> kHistShift) >= lo) ? 1 : 0;
+                int tot;
+                int off = n_cand + block_excl_scan<NT>(cnt, scratch, &tot);
+#pragma unroll
+                for (int i = 0; i < PER; ++i)
+                    if (i < nvalid && (key[i] >> kHistShift) >= lo)
+                        cands[off++] = make_uint2(key[i], static_cast<uint32_t>(base + jb + i));
+                n_cand += tot;
+            }
+            if (piped) __syncthreads();  // every thread is done with this chunk's buffer
         }
-        __syncthreads();  // also orders the key stores before the reads below (same block)
+        __syncthreads();  // the candidates and counts are complete (same block)
         // (B) the k-th largest key thr, and the last position cut of a kept key equal to it
         // (k = 0 keeps only the window: no key is above 0xffffffff, no position at or below -1)
         uint32_t thr = 0xFFFFFFFFu;
@@ -1412,37 +1362,23 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
             int r = k - s_above, n_eq = hist[d1];
             const int n_first = n_eq;
             __syncthreads();
-            // The keys with the k-th key's first digit: gathered into shared memory when there
-            // are at most kLsCand of them (the usual case), else read again from the scratch row.
+            // The candidates with the k-th key's first digit: gathered into shared memory when
+            // there are at most kLsCand of them (the usual case), else read from the list.
             const bool in_smem = n_eq <= kLsCand;
             if (in_smem) {
                 if (tid == 0) s_cnt = 0;
                 __syncthreads();
-                uint32_t key[PER];
-                if (kring)  // chunks through the shared-memory ring, two ahead
-                    for (int c = 0; c < kKeyBufs - 1; ++c) issue_key_chunk(ring, keys, c, Pn);
-                for (int base = 0, ch = 0; base < Pn; base += kLsChunk, ++ch) {
-                    const int jb = tid * PER, nvalid = min(kLsChunk, Pn - base) - jb;
-                    if (kring) {
-                        issue_key_chunk(ring, keys, ch + kKeyBufs - 1, Pn);
-                        cp_async_wait_group<kKeyBufs - 1>();
-                        __syncthreads();
-                        ring_keys(ring + (ch % kKeyBufs) * kLsChunk, key);
-                    } else {
-                        load_keys(keys + base, jb, nvalid, key);
+                for (int c = tid; c < n_cand; c += NT) {
+                    const uint2 x = __ldcg(cands + c);
+                    if ((x.x >> kHistShift) == d1) {
+                        const int i = atomicAdd(&s_cnt, 1);
+                        if (i < kLsCand) cand[i] = x;
                     }
-#pragma unroll
-                    for (int i = 0; i < PER; ++i)
-                        if (i < nvalid && (key[i] >> kHistShift) == d1) {
-                            const int c = atomicAdd(&s_cnt, 1);
-                            if (c < kLsCand) cand[c] = make_uint2(key[i], base + jb + i);
-                        }
-                    if (kring) __syncthreads();  // the buffer is refilled by the next issue
                 }
-                cp_async_wait_group<0>();
+                __syncthreads();
             }
             // Two more digits (11 and 10 bits) of the k-th key, by counts of the keys that share
-            // the digits so far: over the gathered candidates or over the scratch row.
+            // the digits so far.
             uint32_t prefix = d1 << kHistShift, mask = 0x7FFu << kHistShift;
 #pragma unroll 1
             for (int level = 0; level < 2; ++level) {
@@ -1456,14 +1392,9 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
                         if ((kk & mask) == prefix) atomicAdd(&hist[(kk >> shift) & dmask], 1);
                     }
                 } else {
-                    for (int base = 0; base < Pn; base += kLsChunk) {
-                        const int jb = tid * PER, nvalid = min(kLsChunk, Pn - base) - jb;
-                        uint32_t key[PER];
-                        load_keys(keys + base, jb, nvalid, key);
-#pragma unroll
-                        for (int i = 0; i < PER; ++i)
-                            if (i < nvalid && (key[i] & mask) == prefix)
-                                atomicAdd(&hist[(key[i] >> shift) & dmask], 1);
+                    for (int c = tid; c < n_cand; c += NT) {
+                        const uint32_t kk = __ldcg(cands + c).x;
+                        if ((kk & mask) == prefix) atomicAdd(&hist[(kk >> shift) & dmask], 1);
                     }
                 }
                 __syncthreads();
@@ -1498,23 +1429,22 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
                     __syncthreads();
                     pos_cut = s_cut;
                 } else {
+                    // a scan of the list, which is in position order
                     int seen = 0;  // keys equal to thr in the chunks before
-                    for (int base = 0; base < Pn && seen < need_eq; base += kLsChunk) {
-                        const int jb = tid * PER, nvalid = min(kLsChunk, Pn - base) - jb;
-                        uint32_t key[PER];
-                        load_keys(keys + base, jb, nvalid, key);
+                    for (int b0 = 0; b0 < n_cand && seen < need_eq; b0 += kLsChunk) {
+                        const int jb = tid * PER, nvalid = min(kLsChunk, n_cand - b0) - jb;
                         int ne = 0;
 #pragma unroll
-                        for (int i = 0; i < PER; ++i) ne += (i < nvalid && key[i] == thr) ? 1 : 0;
+                        for (int i = 0; i < PER; ++i) ne += (i < nvalid && __ldcg(cands + b0 + jb + i).x == thr) ? 1 : 0;
                         int tot;
                         const int before = seen + block_excl_scan<NT>(ne, scratch, &tot);
                         if (before < need_eq && before + ne >= need_eq) {
                             int c = before;
 #pragma unroll
                             for (int i = 0; i < PER; ++i) {
-                                if (i < nvalid && key[i] == thr) {
-                                    ++c;
-                                    if (c == need_eq) s_cut = base + jb + i;
+                                if (i < nvalid) {
+                                    const uint2 x = __ldcg(cands + b0 + jb + i);
+                                    if (x.x == thr && ++c == need_eq) s_cut = static_cast<int>(x.y);
                                 }
                             }
                         }
@@ -1525,32 +1455,38 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
                 }
             }
         }
-        // (C) the kept positions in order, chunk by chunk, gathered in the list (the stage is
-        // free now) and written out with their K/V rows when it is full and at the end, so that
-        // the rows' copies of many chunks share one round trip; then the window
+        // (C) the kept positions in order: the candidates above the threshold, or equal to it
+        // and at or before the tie cutoff, a block scan per kLsChunk of the list; gathered in
+        // the stage (free now) and written out with their K/V rows when it is full and at the
+        // end, so that the rows' copies share one round trip; then the window
         int written = 0, lbase = 0, lcount = 0;  // list[0..lcount) are output rows lbase..
-        uint32_t key[PER];
-        __syncthreads();  // (B) is done with the ring
-        if (kring)  // chunks through the shared-memory ring, two ahead
-            for (int c = 0; c < kKeyBufs - 1; ++c) issue_key_chunk(ring, keys, c, Pn);
-        for (int base = 0, ch = 0; base < Pn; base += kLsChunk, ++ch) {
-            const int jb = tid * PER, nvalid = min(kLsChunk, Pn - base) - jb;
-            if (kring) {
-                issue_key_chunk(ring, keys, ch + kKeyBufs - 1, Pn);
-                cp_async_wait_group<kKeyBufs - 1>();
-                __syncthreads();
-                ring_keys(ring + (ch % kKeyBufs) * kLsChunk, key);
-            } else {
-                load_keys(keys + base, jb, nvalid, key);
-            }
+        for (int b0 = 0; b0 < n_cand && k > 0; b0 += kLsChunk) {
+            const int jb = tid * PER, nvalid = min(kLsChunk, n_cand - b0) - jb;
             uint32_t taken = 0;
-            int cnt = 0;
+            int cnt = 0, pos[PER];
 #pragma unroll
-            for (int i = 0; i < PER; ++i) {
-                const int j = base + jb + i;
-                if (i < nvalid && (key[i] > thr || (key[i] == thr && j <= pos_cut))) {
-                    taken |= 1u << i;
-                    ++cnt;
+            for (int q = 0; q < PER / 2; ++q) {
+                // 16-byte loads: the list is 32-byte aligned, b0 + jb a multiple of 16
+                uint4 x2 = make_uint4(0u, 0u, 0u, 0u);
+                if (2 * q < nvalid) {
+                    if (2 * q + 1 < nvalid) {
+                        x2 = __ldcg(reinterpret_cast<const uint4*>(cands + b0 + jb) + q);
+                    } else {
+                        const uint2 x = __ldcg(cands + b0 + jb + 2 * q);
+                        x2.x = x.x;
+                        x2.y = x.y;
+                    }
+                }
+                const uint32_t kx[2] = {x2.x, x2.z};
+                const int px[2] = {static_cast<int>(x2.y), static_cast<int>(x2.w)};
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    const int i = 2 * q + e;
+                    pos[i] = px[e];
+                    if (i < nvalid && (kx[e] > thr || (kx[e] == thr && px[e] <= pos_cut))) {
+                        taken |= 1u << i;
+                        ++cnt;
+                    }
                 }
             }
             int tot;
@@ -1566,16 +1502,13 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
 #pragma unroll
             for (int i = 0; i < PER; ++i) {
                 if ((taken >> i) & 1u) {
-                    list[rk] = base + jb + i;
+                    list[rk] = pos[i];
                     ++rk;
                 }
             }
             lcount += tot;
             written += tot;
-            // (the block scan above ordered every read of this chunk's ring buffer before the
-            // issue that refills it)
         }
-        cp_async_wait_group<0>();
         if (written != k) {
             if (tid == 0) record_error(p.status, kDevBadIndex, 340 + unit);
             __syncthreads();  // every thread is done with the list before the next unit
@@ -1723,8 +1656,8 @@ cudaError_t launch_gather(const GatherLaunch& L, cudaStream_t stream) {
 }
 
 // The selection of several layers in one launch (select_layers_kernel); Ls[i] as for
-// launch_select with from_scores = 1, and keys[i] a [n_vec, select_key_stride(T, S)] scratch
-// per layer.  One launch per
+// launch_select with from_scores = 1, and keys[i] a [n_vec, select_key_stride(T, S)] scratch of
+// 8-byte (key, position) slots per layer.  One launch per
 // kSelMaxLayers layers; `next_unit` (kSelMaxLayers-aligned count of ints) is the work counter
 // of each launch and is cleared first.
 int select_key_stride(int T, int S) { return (T + 4 * S + 3) & ~3; }
@@ -1774,7 +1707,7 @@ cudaError_t launch_select_layers(const SelectLaunch* Ls, uint32_t* const* keys, 
             p.write_pooled = L.write_pooled;
             p.cu_hash = L.cu_hash;
             for (int g = 0; g <= L.n_vec; ++g) p.group_first[g] = static_cast<int16_t>(L.group_first[g]);
-            P.keys[i] = keys[l0 + i];
+            P.cands[i] = reinterpret_cast<uint2*>(keys[l0 + i]);
         }
         P.n_layers = nl;
         P.units_per_layer = Ls[l0].S * Ls[l0].n_vec;
