@@ -33,12 +33,17 @@ UNIT = "prefix tokens/s per layer"
 WORKLOAD = "needle_l131072"
 HBM_FALLBACK_GBS = 6800.0
 
-# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) of one scoring launch (one layer)
-# per workload, from the ncu summaries under profiles/ ("+lse": bench.py --lse), keyed by the
-# sha256 of the scoring kernels' sources (SCORE_SOURCES); a changed kernel reports null until
-# it is captured again.  Figures that ncu printed in MB are rounded to 10 kB.
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) of the scoring kernel per layer, per
+# workload, from an ncu capture of a two-layer launch of the same kernel (bench.py --layers 2 on
+# the workload), halved; keyed by the sha256 of the scoring kernels' sources (SCORE_SOURCES), so
+# a changed kernel reports null until it is captured again.  Rounded to 10 kB.
 SCORE_SOURCES = ('score_layers.cu', 'score_resident.cu', 'score_lse.cu', 'score_common.cuh', 'ckv_device.cuh')
-SCORE_TRAFFIC = {}
+SCORE_TRAFFIC = {
+    "752bed29650d76be3e6146f6ad68f6c8786ca895c2ffe8c62734fe859d8e8b82": {
+        "needle_l131072": 385_810_000,
+        "ragged_qwen7b": 223_830_000,
+    },
+}
 # Sequences up to this many tokens are selected by one block per (sequence, KV head)
 # (one launch); longer ones by the chunked kernels (two launches).
 SELECT_UNIT_LEN = 16384
@@ -407,8 +412,9 @@ def run_ours(args):
     # per layer: the scoring kernel, then the selection (pool, top-k, compaction and gather)
     lens = list(wl.seqlens)
     sel_per_layer = (1 if min(lens) <= SELECT_UNIT_LEN else 0) + (2 if max(lens) > SELECT_UNIT_LEN else 0)
-    if multi:  # one scoring launch per 32 layers and per 512 sequences, then the selections
-        launches_per_step = -(-nl // 32) * -(-wl.num_seqs // 512) + sel_per_layer * nl
+    if multi:  # per 32 layers one scoring launch and one selection launch (the workloads here
+        # fit one launch's unit table; the selection's counter reset is a memset, not a kernel)
+        launches_per_step = 2 * -(-nl // 32)
     else:
         launches_per_step = (1 + sel_per_layer) * nl
 

@@ -155,17 +155,6 @@ __device__ __forceinline__ void tma_load_3d_hint(void* dst, const CUtensorMap* m
         : "memory");
 }
 
-// Prefetch of one box into L2 (no shared memory, no completion to wait for): a later load of
-// the same box then comes from L2.
-__device__ __forceinline__ void tma_prefetch_l2_3d(const CUtensorMap* map, int c0, int c1, int c2,
-                                                   uint64_t policy) {
-    asm volatile(
-        "cp.async.bulk.prefetch.tensor.3d.L2.global.tile.L2::cache_hint [%0, {%1, %2, %3}], %4;" ::"l"(
-            reinterpret_cast<uint64_t>(map)),
-        "r"(c0), "r"(c1), "r"(c2), "l"(policy)
-        : "memory");
-}
-
 // L2 policies: keep the lines (they are read again soon) / let them go first.
 __device__ __forceinline__ uint64_t l2_policy_evict_last() {
     uint64_t p;
