@@ -1162,8 +1162,8 @@ ckv_status prepare_layers(const ckv_config* cfg, int32_t n_layers, const ckv_lay
     for (int i = 0; i < n_layers; ++i) {
         lw->scores[i] = off;
         off = round_up(off + static_cast<size_t>(pls[i].n_sel) * *T * sizeof(float), kWsAlign);
-        lw->keys[i] = off;  // the selection's (key, position) candidates, [n_vec, key stride]
-        off = round_up(off + static_cast<size_t>(pls[i].n_vec) * select_key_stride(*T, b->num_seqs) *
+        lw->keys[i] = off;  // the selection's (key, position) candidates, [H_kv, key stride]
+        off = round_up(off + static_cast<size_t>(pls[i].Hkv) * select_key_stride(*T, b->num_seqs) *
                                  2 * sizeof(uint32_t), kWsAlign);
     }
     lw->total = off;

@@ -151,7 +151,7 @@ int select_unit_len();  // units up to this length take the one-block path
 cudaError_t launch_pool(const SelectLaunch& L, cudaStream_t stream);
 cudaError_t launch_select(const SelectLaunch& L, cudaStream_t stream);
 // The selections of several layers (one SelectLaunch each, pooling from their scores) in one
-// launch per 32 layers: keys[i] is a [n_vec, select_key_stride(T, S)] scratch of 8-byte slots
+// launch per 32 layers: keys[i] is a [H_kv, select_key_stride(T, S)] scratch of 8-byte slots
 // of layer i (each sequence's segment 32-byte aligned), next_unit a work counter (cleared by the
 // call).
 int select_key_stride(int T, int S);

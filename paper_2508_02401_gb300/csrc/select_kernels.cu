@@ -1225,16 +1225,20 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
         const int gu = s_unit;
         __syncthreads();
         if (gu >= n_units) break;
-        const int li = gu / P.units_per_layer, unit = gu % P.units_per_layer;
+        const int li = gu / P.units_per_layer, lu = gu % P.units_per_layer;
         const SelectParams& p = P.layer[li];
+        // One selection per layer (n_vec = 1) is made by H_kv units, each writing the positions
+        // and copying the rows of one KV head, so that the row copies spread over CTAs; every
+        // copy of the selection is the same (the same inputs and steps).
+        const int copies = p.n_vec == 1 ? p.Hkv : 1, cu = lu % copies, unit = lu / copies;
         UnitGeo u;
         if (!unit_geo(p, unit, u)) continue;
-        const int kv0 = p.n_vec == p.Hkv ? u.g : 0, kv1 = p.n_vec == p.Hkv ? u.g + 1 : p.Hkv;
-        if (u.g == 0 && tid == 0) {
+        const int kv0 = p.n_vec == p.Hkv ? u.g : cu, kv1 = kv0 + 1;
+        if (u.g == 0 && cu == 0 && tid == 0) {
             p.cu_keep[u.s + 1] = u.keep_off + u.n_keep;
             if (u.s == 0) p.cu_keep[0] = 0;
         }
-        float* pooled = p.write_pooled ? p.pooled + static_cast<size_t>(u.g) * p.T + u.t0 : nullptr;
+        float* pooled = p.write_pooled && cu == 0 ? p.pooled + static_cast<size_t>(u.g) * p.T + u.t0 : nullptr;
         int* list = reinterpret_cast<int*>(st);
         if (u.L <= p.budget) {  // kept whole; its pooled scores read as 0
             for (int e0 = 0; e0 < u.L; e0 += kLsChunk) {
@@ -1253,7 +1257,7 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
         // the unit's candidate list of (key, position) pairs: sequence s's segment of the
         // scratch row starts at its first token rounded up to a multiple of 4, plus 4 s, so that
         // every segment is 32-byte aligned and holds the sequence's P candidates at most
-        uint2* cands = P.cands[li] + static_cast<size_t>(u.g) * P.key_stride + ((u.t0 + 3) & ~3) + 4 * u.s;
+        uint2* cands = P.cands[li] + static_cast<size_t>(u.g * copies + cu) * P.key_stride + ((u.t0 + 3) & ~3) + 4 * u.s;
         int n_cand = 0;
         if (pooled)  // window positions are not candidates
             for (int j = Pn + tid; j < u.L; j += NT) pooled[j] = 0.f;
@@ -1656,7 +1660,7 @@ cudaError_t launch_gather(const GatherLaunch& L, cudaStream_t stream) {
 }
 
 // The selection of several layers in one launch (select_layers_kernel); Ls[i] as for
-// launch_select with from_scores = 1, and keys[i] a [n_vec, select_key_stride(T, S)] scratch of
+// launch_select with from_scores = 1, and keys[i] a [H_kv, select_key_stride(T, S)] scratch of
 // 8-byte (key, position) slots per layer.  One launch per
 // kSelMaxLayers layers; `next_unit` (kSelMaxLayers-aligned count of ints) is the work counter
 // of each launch and is cleared first.
@@ -1710,7 +1714,7 @@ cudaError_t launch_select_layers(const SelectLaunch* Ls, uint32_t* const* keys, 
             P.cands[i] = reinterpret_cast<uint2*>(keys[l0 + i]);
         }
         P.n_layers = nl;
-        P.units_per_layer = Ls[l0].S * Ls[l0].n_vec;
+        P.units_per_layer = Ls[l0].S * Ls[l0].n_vec * (Ls[l0].n_vec == 1 ? Ls[l0].Hkv : 1);
         P.key_stride = select_key_stride(Ls[l0].T, Ls[l0].S);
         P.next_unit = next_unit;
         const int units = nl * P.units_per_layer;

@@ -80,7 +80,9 @@ def _run_layers(wl, cfg, lis, with_scores):
     return res
 
 
-@pytest.mark.parametrize("max_ctas", [0, 5])
+# max_ctas: 0 = every SM, 5 = a capped grid (long items, many per CTA), 1 = one CTA (every unit
+# one item, the whole launch in one CTA's two passes)
+@pytest.mark.parametrize("max_ctas", [0, 5, 1])
 @pytest.mark.parametrize("case", range(len(CASES)))
 def test_layers_calls_match_the_oracle(case, max_ctas):
     wl = _wl(**CASES[case])

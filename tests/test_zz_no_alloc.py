@@ -4,7 +4,8 @@ Some callers have no device allocator to hand (an engine whose memory pool is ow
 elsewhere, or code that must not grow the device footprint after start-up), so this entry
 point takes no workspace and keeps its scratch in a fixed static device array.  The test
 calls it through the C ABI twice in a row and checks both results against the workspace
-entry point, within the score tolerance of the parity tests.  This file is collected last.
+entry point and against the fp64 oracle, within the score tolerance of the parity tests.  This
+file is collected last.
 """
 import ctypes as C
 
@@ -13,6 +14,7 @@ import pytest
 import torch
 
 import ckv_synth as cs
+import oracle
 import paper_2508_02401_gb300 as ckv
 from tests import gpu_util as gu
 
@@ -24,9 +26,10 @@ def _lib():
     if not torch.cuda.is_available():
         pytest.skip("needs a GPU")
     ckv.load()
+    oracle.build()
 
 
-def _static_against_workspace(wl, cfg):
+def _static_against_workspace(wl, cfg, check_oracle=True):
     li = wl.layer(0)
     batch = ckv.Batch(wl.cu_seqlens())
     q, k = gu.to_dev(li.q_win), gu.to_dev(li.k)
@@ -37,6 +40,7 @@ def _static_against_workspace(wl, cfg):
     ckv.ckv_score_window(cfg, 0, batch, q, k, ref, ws)
     assert ckv.ckv_read_device_status(ws) == (0, 0)
     ref = ref.cpu().numpy()
+    want = gu.run_oracle(wl, 0, li, want_kv=False)["scores"] if check_oracle else None
 
     lib = ckv.load()
     stream = torch.cuda.current_stream().cuda_stream
@@ -51,6 +55,8 @@ def _static_against_workspace(wl, cfg):
         assert status.tolist() == [0, 0]
         gout.check()
         gu.assert_close_rows(out.cpu().numpy(), ref)
+        if want is not None:  # and with the fp64 oracle, at the same tolerance
+            gu.assert_close_rows(out.cpu().numpy(), want)
 
 
 @pytest.mark.parametrize("path,max_ctas", [("auto", 0), ("reload", 3), ("resident", 0)])
