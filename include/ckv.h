@@ -250,9 +250,13 @@ CKV_API ckv_status ckv_score_windows(const ckv_config* cfg, int32_t n_layers,
                                      void* workspace, size_t workspace_bytes, ckv_stream stream);
 
 /* Steps 1-4 for several layers: for each io[i], what ckv_compress_layer(cfg, io[i].layer, ...)
- * writes.  The layers are scored as by ckv_score_windows (into the workspace), then each
- * layer's selection runs in order on the same stream.  Sequences with L_s at most every
- * layer's budget are copied whole without being scored. */
+ * writes.  The layers are scored as by ckv_score_windows (into the workspace), then every
+ * layer's selection runs in one launch (one per 32 layers) on the same stream, each (layer,
+ * sequence, selection) by one CTA that keeps a list of the keys that can still be kept in the
+ * workspace.  Sequences with L_s at most every layer's budget are copied whole without being
+ * scored.  The workspace (ckv_workspace_size_layers) holds, per layer, the scores [n_sel, T]
+ * fp32 and the selection's lists [H_kv, T + 4 S] of 8-byte entries, and per unit of the
+ * scoring launch N fp64 row sums and a counter. */
 CKV_API ckv_status ckv_compress_layers(const ckv_config* cfg, int32_t n_layers,
                                        const ckv_layer_io* io, const ckv_batch* batch,
                                        void* workspace, size_t workspace_bytes, ckv_stream stream);
