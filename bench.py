@@ -39,9 +39,9 @@ HBM_FALLBACK_GBS = 6800.0
 # a changed kernel reports null until it is captured again.  Rounded to 10 kB.
 SCORE_SOURCES = ('score_layers.cu', 'score_resident.cu', 'score_lse.cu', 'score_common.cuh', 'ckv_device.cuh')
 SCORE_TRAFFIC = {
-    "752bed29650d76be3e6146f6ad68f6c8786ca895c2ffe8c62734fe859d8e8b82": {
-        "needle_l131072": 385_810_000,
-        "ragged_qwen7b": 223_830_000,
+    "d43a4416edf56f3da424eefd7e9525afc76668f014115c0bd1ba6f2926be1e28": {
+        "needle_l131072": 362_390_000,
+        "ragged_qwen7b": 221_270_000,
     },
 }
 # Sequences up to this many tokens are selected by one block per (sequence, KV head)

@@ -33,9 +33,10 @@
 //                counter and posts it to the other roles (a ring of item indices in shared
 //                memory); per item, TMA loads of the window query rows into one of kQBufs
 //                buffers, then of its 128-key x 128-dim bf16 K tiles (two 128-byte-swizzled
-//                boxes of 64 dims) into the pass-1 ring (evict-last: pass 2 reads them again
-//                soon); the same tiles again into the pass-2 ring (evict-first) once the
-//                item's pass-1 loads are out;
+//                boxes of 64 dims) into the pass-1 ring (evict-last: pass 2 reads them again;
+//                evict-first for the first fifth of an item of a long unit, whose re-reads
+//                come too late for L2); the same tiles again into the pass-2 ring
+//                (evict-first) once the item's pass-1 loads are out;
 //   warp 1       allocates TMEM and issues the pass-1 tcgen05.mma (M = 128 keys, N = the
 //                window rows of a head batch, K = 128) into four pass-1 accumulators;
 //   warp 2       issues the pass-2 tcgen05.mma into four pass-2 accumulators;
@@ -62,6 +63,9 @@ constexpr int kP1Slots = 2;   // pass-1 ring (HBM)
 constexpr int kP2Slots = 3;   // pass-2 ring (L2): pass 2 must outrun pass 1 after each exchange wait
 constexpr int kAcc = 4;       // TMEM accumulators per pass
 constexpr int kQBufs = 3;     // query-row buffers: pass 1 runs up to two items ahead of pass 2
+// Units of more keys than this (16 MB of K, an eighth of L2) load the first fifth of each item's
+// tiles evict-first in pass 1: their re-reads come after most of L2 has turned over.
+constexpr int kLongUnitKeys = 65536;
 constexpr int kItemRing = 8;  // item indices posted by the producer (more than any role's lag)
 // Largest |log2| of an item's column maximum: an item's sum is then below 2^1000 (at most
 // 2^10 keys), and the sum of up to 2^20 items stays below fp64's 2^1024.
@@ -368,8 +372,11 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
                         const int g = p.batch_group[I1.batch];
                         const int tok = I1.start + (I1.tile0 + jt1) * kTileKeys;
                         const CUtensorMap* km = &p.tmap_k[I1.layer];
-                        tma_load_3d_hint(dst, km, &full1[s], 0, g, tok, pol1);
-                        tma_load_3d_hint(dst + kHalfBytes, km, &full1[s], 64, g, tok, pol1);
+                        // In a long unit pass 2 re-reads an item's first tiles too late for L2
+                        // anyway: loading them evict-first leaves L2 to the rest.
+                        const uint64_t polx = (I1.len > kLongUnitKeys && jt1 * 5 < I1.ntiles) ? pol2 : pol1;
+                        tma_load_3d_hint(dst, km, &full1[s], 0, g, tok, polx);
+                        tma_load_3d_hint(dst + kHalfBytes, km, &full1[s], 64, g, tok, polx);
                         ++use1;
                         did = true;
                         if (++jt1 == I1.ntiles) {
