@@ -218,6 +218,28 @@ __device__ __forceinline__ int block_excl_scan(int v, int* scratch, int* total) 
     return r;
 }
 
+// The same with one barrier: each warp's sum goes to buf[warp], then every warp adds up the
+// sums of the warps before it.  Consecutive calls must alternate between two buffers: a call's
+// barrier then orders every read of the buffer two calls back before it is written again.
+template <int NT>
+__device__ __forceinline__ int block_excl_scan1(int v, int* buf, int* total) {
+    constexpr int NW = NT / 32;
+    static_assert(NW <= 32, "warps");
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int incl = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+    }
+    if (lane == 31) buf[warp] = incl;
+    __syncthreads();
+    const int x = lane < NW ? buf[lane] : 0;
+    const int before = __reduce_add_sync(0xffffffffu, lane < warp ? x : 0);
+    *total = __reduce_add_sync(0xffffffffu, x);
+    return before + incl - v;
+}
+
 // The digit d of a kHistBins-bin histogram with count(bins above d) < r <= count(bins >= d),
 // r >= 1: *s_digit = d, *s_above = count(bins above d).  Thread 0 owns the highest bins.
 template <int NT>
@@ -1209,6 +1231,7 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
     extern __shared__ __align__(16) float st[];  // pooling stage; the kept list of a chunk
     __shared__ int hist[kHistBins];
     __shared__ int scratch[33];
+    __shared__ int wsum[2][kLsThreads / 32];  // the one-barrier scans' warp sums, alternating
     __shared__ int s_digit, s_above, s_cut, s_cnt, s_unit;
     __shared__ uint32_t s_thr;
     __shared__ uint2 cand[kLsCand];
@@ -1345,7 +1368,7 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
 #pragma unroll
                 for (int i = 0; i < PER; ++i) cnt += (i < nvalid && (key[i] >> kHistShift) >= lo) ? 1 : 0;
                 int tot;
-                int off = n_cand + block_excl_scan<NT>(cnt, scratch, &tot);
+                int off = n_cand + block_excl_scan1<NT>(cnt, wsum[c & 1], &tot);
 #pragma unroll
                 for (int i = 0; i < PER; ++i)
                     if (i < nvalid && (key[i] >> kHistShift) >= lo)
@@ -1494,7 +1517,7 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
                 }
             }
             int tot;
-            int rk = block_excl_scan<NT>(cnt, scratch, &tot);
+            int rk = block_excl_scan1<NT>(cnt, wsum[(b0 / kLsChunk) & 1], &tot);
             if (written + tot > k) break;  // checked below
             if (lcount + tot > kLsList) {  // block-uniform: write out the list first
                 emit_kept(p, u, list, lcount, lbase, kv0, kv1);

@@ -130,3 +130,31 @@ def test_equal_scores_keep_the_lowest_positions():
         for g in range(wl.num_kv_heads):
             np.testing.assert_array_equal(res[0]["idx"][g, ck[s]:ck[s] + 32], np.arange(32))
             assert P > 32
+
+
+def test_layers_call_with_interleaved_kv():
+    """K and V interleaved in one [T, 2, H_kv, 128] buffer per layer, through the multi-layer
+    call: the strides select each half, and the outputs equal those of the packed layout."""
+    wl = _wl(num_q_heads=32, num_kv_heads=8, seqlens=(2500, 700, 9000))
+    cfg = ckv.Config.from_workload(wl)
+    lis = [wl.layer(l) for l in range(wl.num_layers)]
+    packed = _run_layers(wl, cfg, lis, with_scores=False)
+    batch = ckv.Batch(wl.cu_seqlens())
+    ios, guards, keep = [], [], []
+    for l, li in enumerate(lis):
+        kv = torch.stack([gu.to_dev(li.k), gu.to_dev(li.v)], dim=1).contiguous()  # [T, 2, 8, 128]
+        keep.append(kv)
+        gidx, gck, gk, gv, _ = gu.guarded_outputs(cfg, l, batch)
+        ios.append(ckv.LayerIO(layer=l, q_win=gu.to_dev(li.q_win), k=kv[:, 0], v=kv[:, 1],
+                               idx=gidx.view, cu_keep_dev=gck.view, k_out=gk.view, v_out=gv.view,
+                               tok_stride=2 * 8 * 128, head_stride=128))
+        guards.append((gidx, gck, gk, gv))
+    ws = ckv.new_layers_workspace(cfg, ios, batch)
+    ckv.ckv_compress_layers(cfg, ios, batch, ws)
+    assert ckv.ckv_read_device_status(ws) == (0, 0)
+    for (gidx, gck, gk, gv), ref in zip(guards, packed):
+        for g_ in (gidx, gck, gk, gv):
+            g_.check()
+        np.testing.assert_array_equal(gidx.view.cpu().numpy(), ref["idx"])
+        np.testing.assert_array_equal(gu.to_host(gk.view), ref["k_out"])
+        np.testing.assert_array_equal(gu.to_host(gv.view), ref["v_out"])
