@@ -106,7 +106,8 @@ def _args():
                          "next layer's scoring need not wait")
     ap.add_argument("--lse", action="store_true",
                     help="the window rows' lse given (as a prefill attention kernel returns it): "
-                         "ckv_compress_layer_lse / ckv_score_window_lse, one pass over K")
+                         "ckv_compress_layers_lse (with --calls layer: ckv_compress_layer_lse), "
+                         "one pass over K")
     ap.add_argument("--max-ctas", type=int, default=0,
                     help="CTAs one call's scoring kernel may occupy (0: all SMs with --calls "
                          "layers; SMs / streams with --calls layer, so that one scoring kernel "
@@ -292,14 +293,16 @@ def run_ours(args):
 
     # One call for every layer of the step: ckv_compress_layers (the layers' scoring in one
     # persistent launch over all SMs, then the selections), with the window rows' lse computed.
-    multi = args.calls == "layers" and not args.lse and not args.split_select
+    multi = args.calls == "layers" and not args.split_select
     if multi:
         cap = args.max_ctas if args.max_ctas > 0 else 0
         cfg = ckv.Config.from_workload(wl, max_ctas=cap, score_path=path)
         nstreams = 1
         ios = [ckv.LayerIO(layer=l, q_win=d["q"], k=d["k"], v=d["v"], idx=d["idx"],
-                           cu_keep_dev=d["cu_keep_dev"], k_out=d["k_out"], v_out=d["v_out"])
+                           cu_keep_dev=d["cu_keep_dev"], k_out=d["k_out"], v_out=d["v_out"],
+                           lse=d.get("lse"))
                for l, d in enumerate(layers)]
+        compress_layers = ckv.ckv_compress_layers_lse if args.lse else ckv.ckv_compress_layers
         wss = [ckv.new_layers_workspace(cfg, ios, batch)]
         ws = wss[0]
 
@@ -339,7 +342,7 @@ def run_ours(args):
 
     def step():
         if multi:
-            ckv.ckv_compress_layers(cfg, ios, batch, ws, stream=stream)
+            compress_layers(cfg, ios, batch, ws, stream=stream)
         else:
             over_layers(compress, selections=args.split_select)
 
@@ -412,7 +415,9 @@ def run_ours(args):
     # per layer: the scoring kernel, then the selection (pool, top-k, compaction and gather)
     lens = list(wl.seqlens)
     sel_per_layer = (1 if min(lens) <= SELECT_UNIT_LEN else 0) + (2 if max(lens) > SELECT_UNIT_LEN else 0)
-    if multi:  # per 32 layers one scoring launch and one selection launch (the workloads here
+    if multi and args.lse:  # a single-pass scoring launch per layer, one selection launch per 32
+        launches_per_step = nl + -(-nl // 32)
+    elif multi:  # per 32 layers one scoring launch and one selection launch (the workloads here
         # fit one launch's unit table; the selection's counter reset is a memset, not a kernel)
         launches_per_step = 2 * -(-nl // 32)
     else:
@@ -451,7 +456,7 @@ def run_ours(args):
             ckv.ckv_score_window(cfg, l, batch, d["q"], d["k"], score_rows[l], w, stream=st)
 
     def score_all():
-        if multi:
+        if multi and not args.lse:
             ckv.ckv_score_windows(cfg, score_ios, batch, ws, stream=stream)
         else:
             over_layers(score_one)
@@ -487,7 +492,9 @@ def run_ours(args):
     for f in SCORE_SOURCES:
         digest.update(open(os.path.join(ROOT, "paper_2508_02401_gb300", "csrc", f), "rb").read())
     traffic = SCORE_TRAFFIC.get(digest.hexdigest(), {}).get(args.workload + ("+lse" if args.lse else ""))
-    kernel_desc = ("two-pass scoring kernel (ckv_score_windows): every layer of the step in one "
+    kernel_desc = ("single-pass scoring kernel (ckv_score_window_lse), one launch per layer on "
+                   f"{sms} CTAs; per layer" if multi and args.lse else
+                   "two-pass scoring kernel (ckv_score_windows): every layer of the step in one "
                    f"persistent launch on {cap or sms} CTAs; per layer" if multi else
                    "scoring kernel (ckv_score_window), per layer, layers overlapped on "
                    f"{nstreams} streams, {cap} CTAs per call")
@@ -537,10 +544,12 @@ def run_ours(args):
                         d["q"].copy_(hq[l], non_blocking=True)
                         d["k"].copy_(hk[l], non_blocking=True)
                         d["v"].copy_(hv[l], non_blocking=True)
+                        if args.lse:
+                            d["lse"].copy_(hl[l], non_blocking=True)
                 landed = torch.cuda.Event()
                 landed.record(cp)
                 stream.wait_event(landed)
-                ckv.ckv_compress_layers(cfg, ios[c0:c0 + E], batch, ws, stream=stream)
+                compress_layers(cfg, ios[c0:c0 + E], batch, ws, stream=stream)
                 done = torch.cuda.Event()
                 done.record(stream)
                 back.wait_event(done)
@@ -615,7 +624,8 @@ def run_ours(args):
                                 f"layers round-robin on {nstreams} streams, scoring capped at {cap} CTAs per call"),
                     "lse": ("window-row lse given (PyTorch logsumexp outside the timed region; "
                             "one pass over K)") if args.lse else "computed (two passes)",
-                    "calls": ("ckv_compress_layers over every layer of the step" if multi else
+                    "calls": (("ckv_compress_layers_lse" if args.lse else "ckv_compress_layers") +
+                              " over every layer of the step" if multi else
                               "ckv_score_window + ckv_select_compact, the selection on a stream "
                               "of its own" if args.split_select else "ckv_compress_layer per layer"),
                     "repetitions": len(reps_ms),

@@ -53,7 +53,7 @@
 extern "C" {
 #endif
 
-#define CKV_ABI_VERSION 5
+#define CKV_ABI_VERSION 6
 
 #if defined(__GNUC__)
 #define CKV_API __attribute__((visibility("default")))
@@ -217,8 +217,9 @@ CKV_API ckv_status ckv_select_compact(const ckv_config* cfg, int32_t layer, cons
                                       float* pooled_out, void* workspace, size_t workspace_bytes,
                                       ckv_stream stream);
 
-/* One layer of a multi-layer call (ckv_score_windows, ckv_compress_layers).  The layers of a
- * call share the config and the batch; each brings its own buffers. */
+/* One layer of a multi-layer call (ckv_score_windows, ckv_compress_layers,
+ * ckv_compress_layers_lse).  The layers of a call share the config and the batch; each brings
+ * its own buffers. */
 typedef struct ckv_layer_io {
     int32_t layer;                 /* index into the config's head_mask and budgets */
     const void* q_win;             /* [S, w, H_q, 128] */
@@ -232,6 +233,9 @@ typedef struct ckv_layer_io {
     void* k_out;
     void* v_out;
     float* pooled_out;             /* may be NULL */
+    const float* lse;              /* ckv_compress_layers_lse: the window rows' lse, as for
+                                      ckv_score_window_lse (fp32, natural log, [H_q][S*w]) */
+    int64_t lse_head_stride;       /* elements between heads; 0 = S*w */
 } ckv_layer_io;
 
 /* Workspace bytes for a multi-layer call over io[0..n_layers) (enough for either entry point). */
@@ -260,6 +264,17 @@ CKV_API ckv_status ckv_score_windows(const ckv_config* cfg, int32_t n_layers,
 CKV_API ckv_status ckv_compress_layers(const ckv_config* cfg, int32_t n_layers,
                                        const ckv_layer_io* io, const ckv_batch* batch,
                                        void* workspace, size_t workspace_bytes, ckv_stream stream);
+
+/* Steps 1-4 for several layers with every layer's window-row lse given (io[i].lse, NEXT #3 of
+ * the hot path: the lse a prefill attention kernel returns): for each io[i], what
+ * ckv_compress_layer_lse(cfg, io[i].layer, ...) writes.  Each layer is scored in one pass over K
+ * (one launch per layer, no exchange between CTAs), into the workspace, then every layer's
+ * selection runs in one launch as in ckv_compress_layers.  The same workspace
+ * (ckv_workspace_size_layers).  cfg->score_path is ignored. */
+CKV_API ckv_status ckv_compress_layers_lse(const ckv_config* cfg, int32_t n_layers,
+                                           const ckv_layer_io* io, const ckv_batch* batch,
+                                           void* workspace, size_t workspace_bytes,
+                                           ckv_stream stream);
 
 /* Steps 1-4 for one layer.  Sequences with L_s <= B_l are copied whole without being scored.
  * pooled_out may be NULL (then the pooled scores stay in the workspace). */

@@ -24,7 +24,7 @@ __all__ = [
     "SCORE_AUTO", "SCORE_RESIDENT", "SCORE_RELOAD", "ckv_score_window_lse",
     "ckv_compress_layer_lse", "ckv_semantic_retrieval_scores", "ckv_set_wait_limit_us",
     "new_workspace", "new_outputs", "LayerIO", "ckv_workspace_size_layers", "ckv_score_windows",
-    "ckv_compress_layers", "new_layers_workspace",
+    "ckv_compress_layers", "ckv_compress_layers_lse", "new_layers_workspace",
 ]
 
 POOL_MAX, POOL_AVG = 0, 1
@@ -62,7 +62,8 @@ class _LayerIO(C.Structure):
     _fields_ = [("layer", C.c_int32), ("q_win", C.c_void_p), ("k", C.c_void_p), ("v", C.c_void_p),
                 ("tok_stride", C.c_int64), ("head_stride", C.c_int64), ("scores", C.c_void_p),
                 ("idx", C.c_void_p), ("cu_keep_dev", C.c_void_p), ("k_out", C.c_void_p),
-                ("v_out", C.c_void_p), ("pooled_out", C.c_void_p)]
+                ("v_out", C.c_void_p), ("pooled_out", C.c_void_p), ("lse", C.c_void_p),
+                ("lse_head_stride", C.c_int64)]
 
 
 class _Batch(C.Structure):
@@ -107,6 +108,7 @@ def load():
         "ckv_workspace_size_layers": ([cfg, I32, P, bat, C.POINTER(SZ)], C.c_int),
         "ckv_score_windows": ([cfg, I32, P, bat, P, SZ, P], C.c_int),
         "ckv_compress_layers": ([cfg, I32, P, bat, P, SZ, P], C.c_int),
+        "ckv_compress_layers_lse": ([cfg, I32, P, bat, P, SZ, P], C.c_int),
     }
     for name, (args, res) in sigs.items():
         fn = getattr(lib, name)
@@ -357,6 +359,8 @@ class LayerIO:
     pooled_out: object = None
     tok_stride: int = 0
     head_stride: int = 0
+    lse: object = None          # ckv_compress_layers_lse: [H_q, S*w] fp32
+    lse_head_stride: int = 0
 
 
 def _layer_ios(ios):
@@ -365,7 +369,9 @@ def _layer_ios(ios):
         arr[i] = _LayerIO(x.layer, *(None if t is None else t.data_ptr() for t in (x.q_win, x.k, x.v)),
                           x.tok_stride, x.head_stride,
                           *(None if t is None else t.data_ptr()
-                            for t in (x.scores, x.idx, x.cu_keep_dev, x.k_out, x.v_out, x.pooled_out)))
+                            for t in (x.scores, x.idx, x.cu_keep_dev, x.k_out, x.v_out, x.pooled_out,
+                                      x.lse)),
+                          x.lse_head_stride)
     return arr
 
 
@@ -397,6 +403,15 @@ def ckv_compress_layers(cfg, ios, batch, workspace, stream=None):
     _check(load().ckv_compress_layers(cfg.ref, len(ios), arr, batch.ref, _ptr(workspace),
                                       workspace.numel() * workspace.element_size(), _stream(stream)),
            "ckv_compress_layers")
+
+
+def ckv_compress_layers_lse(cfg, ios, batch, workspace, stream=None):
+    """ckv_compress_layer_lse for every LayerIO of `ios` (each with its `lse`): one single-pass
+    scoring launch per layer, then the selections in one launch."""
+    arr = _layer_ios(ios)
+    _check(load().ckv_compress_layers_lse(cfg.ref, len(ios), arr, batch.ref, _ptr(workspace),
+                                          workspace.numel() * workspace.element_size(), _stream(stream)),
+           "ckv_compress_layers_lse")
 
 
 def ckv_read_device_status(workspace, stream=None, reset=True):

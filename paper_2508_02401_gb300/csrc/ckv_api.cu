@@ -1201,6 +1201,80 @@ ckv_status layer_jobs(const std::vector<Plan>& pls, const ckv_layer_io* io, int 
     return CKV_OK;
 }
 
+// ckv_compress_layers(_lse): the layers' scoring (one persistent two-pass launch, or with the
+// lse given one single-pass launch per layer) into the workspace, then every layer's selection
+// in one launch.
+ckv_status compress_layers_impl(const ckv_config* cfg, int32_t n_layers, const ckv_layer_io* io,
+                                const ckv_batch* batch, void* workspace, size_t workspace_bytes,
+                                ckv_stream stream, bool given_lse) {
+    static thread_local std::vector<Plan> pls;
+    static thread_local std::vector<LayerJob> jobs;
+    static thread_local std::vector<int64_t> tok, head;
+    LayersWs lw;
+    int T = 0;
+    ckv_status st;
+    if ((st = prepare_layers(cfg, n_layers, io, batch, pls, &T, &lw)) ||
+        (st = check_layers_ws(lw, workspace, workspace_bytes, true)))
+        return st;
+    uint8_t* w8 = static_cast<uint8_t*>(workspace);
+    if ((st = layer_jobs(pls, io, T, w8, lw, true, jobs, tok, head))) return st;
+    std::vector<int64_t> tks(n_layers, 0), lse_stride(n_layers, 0);
+    int min_budget = INT_MAX;
+    for (int i = 0; i < n_layers; ++i) {
+        if ((st = check_kv(io[i].v, "v", T)) ||
+            (st = check_select_outputs(batch, pls[i], io[i].idx, io[i].cu_keep_dev, io[i].k_out,
+                                       io[i].v_out, io[i].pooled_out, &tks[i])))
+            return st;
+        if (given_lse) {
+            if (!io[i].lse) return fail(CKV_ERR_INVALID_ARG, "io[%d].lse is NULL", i);
+            lse_stride[i] = io[i].lse_head_stride;
+            if ((st = check_lse(pls[i], batch, io[i].lse, &lse_stride[i]))) return st;
+        }
+        min_budget = std::min(min_budget, pls[i].budget);
+    }
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    // sequences that fit every layer's budget are kept whole by every selection
+    if (given_lse) {
+        for (int i = 0; i < n_layers; ++i)
+            if ((st = enqueue_score(pls[i], batch, T, jobs[i].q_win, jobs[i].k, tok[i], head[i],
+                                    jobs[i].scores, workspace, lw.sel, min_budget, s,
+                                    kMaxScoreItems, io[i].lse, lse_stride[i])))
+                return st;
+    } else if ((st = enqueue_layers(jobs, batch, T, w8 + lw.sums, reinterpret_cast<int*>(w8 + lw.counters),
+                                    reinterpret_cast<int*>(w8), min_budget, cfg->max_ctas, s))) {
+        return st;
+    }
+    // every layer's selection in one launch (one per 32 layers)
+    static thread_local std::vector<SelectLaunch> sls;
+    static thread_local std::vector<uint32_t*> keys;
+    sls.assign(n_layers, SelectLaunch{});
+    keys.assign(n_layers, nullptr);
+    for (int i = 0; i < n_layers; ++i) {
+        SelectLaunch& L = sls[i];
+        L = select_launch(pls[i], batch, T, static_cast<int>(tks[i]), pls[i].budget, cfg, workspace, &lw.sel);
+        L.scores = jobs[i].scores;
+        L.pooled = io[i].pooled_out;
+        L.write_pooled = io[i].pooled_out != nullptr;
+        L.from_scores = 1;
+        L.idx = io[i].idx;
+        L.cu_keep_dev = io[i].cu_keep_dev;
+        if (tks[i] > 0) {
+            L.k = io[i].k;
+            L.v = io[i].v;
+            L.tok_stride = tok[i];
+            L.head_stride = head[i];
+            L.k_out = io[i].k_out;
+            L.v_out = io[i].v_out;
+        }
+        keys[i] = reinterpret_cast<uint32_t*>(w8 + lw.keys[i]);
+    }
+    const int sms = device_sm_count();
+    if (sms <= 0) return cuda_fail(cudaGetLastError(), "querying the SM count");
+    const cudaError_t e = launch_select_layers(sls.data(), keys.data(), n_layers,
+                                               reinterpret_cast<int*>(w8 + lw.next_unit), sms, s);
+    return e == cudaSuccess ? CKV_OK : cuda_fail(e, "launching the multi-layer selection kernel");
+}
+
 }  // namespace
 
 extern "C" {
@@ -1239,60 +1313,13 @@ ckv_status ckv_score_windows(const ckv_config* cfg, int32_t n_layers, const ckv_
 ckv_status ckv_compress_layers(const ckv_config* cfg, int32_t n_layers, const ckv_layer_io* io,
                                const ckv_batch* batch, void* workspace, size_t workspace_bytes,
                                ckv_stream stream) {
-    static thread_local std::vector<Plan> pls;
-    static thread_local std::vector<LayerJob> jobs;
-    static thread_local std::vector<int64_t> tok, head;
-    LayersWs lw;
-    int T = 0;
-    ckv_status st;
-    if ((st = prepare_layers(cfg, n_layers, io, batch, pls, &T, &lw)) ||
-        (st = check_layers_ws(lw, workspace, workspace_bytes, true)))
-        return st;
-    uint8_t* w8 = static_cast<uint8_t*>(workspace);
-    if ((st = layer_jobs(pls, io, T, w8, lw, true, jobs, tok, head))) return st;
-    std::vector<int64_t> tks(n_layers, 0);
-    int min_budget = INT_MAX;
-    for (int i = 0; i < n_layers; ++i) {
-        if ((st = check_kv(io[i].v, "v", T)) ||
-            (st = check_select_outputs(batch, pls[i], io[i].idx, io[i].cu_keep_dev, io[i].k_out,
-                                       io[i].v_out, io[i].pooled_out, &tks[i])))
-            return st;
-        min_budget = std::min(min_budget, pls[i].budget);
-    }
-    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    // sequences that fit every layer's budget are kept whole by every selection
-    if ((st = enqueue_layers(jobs, batch, T, w8 + lw.sums, reinterpret_cast<int*>(w8 + lw.counters),
-                             reinterpret_cast<int*>(w8), min_budget, cfg->max_ctas, s)))
-        return st;
-    // every layer's selection in one launch (one per 32 layers)
-    static thread_local std::vector<SelectLaunch> sls;
-    static thread_local std::vector<uint32_t*> keys;
-    sls.assign(n_layers, SelectLaunch{});
-    keys.assign(n_layers, nullptr);
-    for (int i = 0; i < n_layers; ++i) {
-        SelectLaunch& L = sls[i];
-        L = select_launch(pls[i], batch, T, static_cast<int>(tks[i]), pls[i].budget, cfg, workspace, &lw.sel);
-        L.scores = jobs[i].scores;
-        L.pooled = io[i].pooled_out;
-        L.write_pooled = io[i].pooled_out != nullptr;
-        L.from_scores = 1;
-        L.idx = io[i].idx;
-        L.cu_keep_dev = io[i].cu_keep_dev;
-        if (tks[i] > 0) {
-            L.k = io[i].k;
-            L.v = io[i].v;
-            L.tok_stride = tok[i];
-            L.head_stride = head[i];
-            L.k_out = io[i].k_out;
-            L.v_out = io[i].v_out;
-        }
-        keys[i] = reinterpret_cast<uint32_t*>(w8 + lw.keys[i]);
-    }
-    const int sms = device_sm_count();
-    if (sms <= 0) return cuda_fail(cudaGetLastError(), "querying the SM count");
-    const cudaError_t e = launch_select_layers(sls.data(), keys.data(), n_layers,
-                                               reinterpret_cast<int*>(w8 + lw.next_unit), sms, s);
-    return e == cudaSuccess ? CKV_OK : cuda_fail(e, "launching the multi-layer selection kernel");
+    return compress_layers_impl(cfg, n_layers, io, batch, workspace, workspace_bytes, stream, false);
+}
+
+ckv_status ckv_compress_layers_lse(const ckv_config* cfg, int32_t n_layers, const ckv_layer_io* io,
+                                   const ckv_batch* batch, void* workspace, size_t workspace_bytes,
+                                   ckv_stream stream) {
+    return compress_layers_impl(cfg, n_layers, io, batch, workspace, workspace_bytes, stream, true);
 }
 
 ckv_status ckv_semantic_retrieval_scores(const ckv_config* cfg, int32_t layer, const ckv_batch* batch,

@@ -31,7 +31,7 @@ def test_header_declares_the_boundary():
     names = _declared()
     for n in ("ckv_score_window", "ckv_pool", "ckv_select_topk", "ckv_gather_compact",
               "ckv_compress_layer", "ckv_workspace_size", "ckv_keep_lengths", "ckv_score_windows",
-              "ckv_compress_layers", "ckv_workspace_size_layers",
+              "ckv_compress_layers", "ckv_compress_layers_lse", "ckv_workspace_size_layers",
               "ckv_read_device_status", "ckv_status_string"):
         assert n in names
 
@@ -48,7 +48,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 
 def test_version_and_status_strings(lib):
-    assert ckv.ckv_abi_version() == 5
+    assert ckv.ckv_abi_version() == 6
     assert ckv.ckv_status_string(0) == "CKV_OK"
     assert ckv.ckv_status_string(3) == "CKV_ERR_WORKSPACE"
 
@@ -223,6 +223,12 @@ def test_layers_argument_errors(lib):
     # the fused call needs room for every layer's scores; the scoring call does not
     need = ckv.ckv_workspace_size_layers(cfg, ios, b)
     assert lib.ckv_compress_layers(cfg.ref, 3, arr, b.ref, _P, need - 256, None) == 3
+    # the given-lse form needs every layer's lse, aligned, with a head stride of at least S*w
+    assert lib.ckv_compress_layers_lse(cfg.ref, 3, arr, b.ref, _P, 1 << 30, None) == 1   # no lse
+    bad = ckv._layer_ios(_ios(3, lse=_FakeT(_P + 2)))
+    assert lib.ckv_compress_layers_lse(cfg.ref, 3, bad, b.ref, _P, 1 << 30, None) == 1   # misaligned
+    bad = ckv._layer_ios(_ios(3, lse=_FakeT(_P), lse_head_stride=2 * 32 - 1))
+    assert lib.ckv_compress_layers_lse(cfg.ref, 3, bad, b.ref, _P, 1 << 30, None) == 1   # stride < S*w
 
 
 @pytest.mark.skipif(__import__("torch").cuda.is_available(), reason="CPU-only behaviour")
@@ -231,3 +237,5 @@ def test_valid_layers_call_without_a_gpu_reports_cuda_error(lib):
     arr = ckv._layer_ios(_ios(3))
     assert lib.ckv_score_windows(cfg.ref, 3, arr, b.ref, _P, 1 << 30, None) == 4
     assert lib.ckv_compress_layers(cfg.ref, 3, arr, b.ref, _P, 1 << 30, None) == 4
+    arr = ckv._layer_ios(_ios(3, lse=_FakeT(_P)))
+    assert lib.ckv_compress_layers_lse(cfg.ref, 3, arr, b.ref, _P, 1 << 30, None) == 4

@@ -177,3 +177,48 @@ def test_decode_attention_over_the_compacted_cache():
                 kept = [i for i, r in enumerate(rows) if int(r) in planted]
                 assert len(kept) == len(planted)
                 assert p_c[kept].sum() >= p_f[sorted(planted)].sum() * (1 - 1e-12)
+
+
+@pytest.mark.parametrize("case", [0, 1])
+def test_layers_call_with_given_lse(case):
+    """ckv_compress_layers_lse over several layers (one single-pass scoring launch per layer,
+    then every layer's selection in one launch) against the oracle's layer with the same lse,
+    layer by layer; canaries around every output.  Case 1: ragged lengths (some at most the
+    budget, one shorter than the window) and a padded lse head stride."""
+    if case == 0:
+        wl = _wl(num_layers=3, num_q_heads=32, num_kv_heads=8, seqlens=(6000, 900),
+                 budget_mean=200, outlier_channels=8)
+    else:
+        wl = _wl(num_layers=2, seqlens=(5, 31, 300, 2500, 40), budget_mean=64)
+    pad = 3 * case
+    cfg = ckv.Config.from_workload(wl)
+    batch = ckv.Batch(wl.cu_seqlens())
+    T = batch.total_tokens
+    ios, outs, refs = [], [], []
+    for l in range(wl.num_layers):
+        li = wl.layer(l)
+        lse64 = _oracle_lse(wl, li, pad)
+        refs.append((li, oracle.compress_layer(li.q_win, li.k, li.v, wl.cu_seqlens(), wl.head_mask()[l],
+                                               int(wl.budgets()[l]), wl.window, wl.pool_kernel,
+                                               0 if wl.pool_type == "max" else 1,
+                                               0 if wl.head_order == "pool_then_sum" else 1,
+                                               scope=oracle.SCOPE_KV_HEAD, lse=lse64)))
+        lse32 = torch.from_numpy(lse64.astype(np.float32)).cuda()
+        *gouts, cu_keep = gu.guarded_outputs(cfg, l, batch)
+        gpl = gu.Guarded((cfg.num_vectors, T), torch.float32, float("nan"))
+        ios.append(ckv.LayerIO(layer=l, q_win=gu.to_dev(li.q_win), k=gu.to_dev(li.k), v=gu.to_dev(li.v),
+                               idx=gouts[0].view, cu_keep_dev=gouts[1].view, k_out=gouts[2].view,
+                               v_out=gouts[3].view, pooled_out=gpl.view, lse=lse32,
+                               lse_head_stride=lse64.shape[1]))
+        outs.append((gouts, gpl, cu_keep))
+    ws = ckv.new_layers_workspace(cfg, ios, batch)
+    ckv.ckv_compress_layers_lse(cfg, ios, batch, ws)
+    code, detail = ckv.ckv_read_device_status(ws)
+    assert code == 0, (code, detail)
+    for l, ((gouts, gpl, cu_keep), (li, o)) in enumerate(zip(outs, refs)):
+        for g_ in [gpl, *gouts]:
+            g_.check()
+        idx, cu_keep_dev, k_out, v_out = (g_.view for g_ in gouts)
+        g = dict(cfg=cfg, cu_keep=cu_keep, pooled=gpl.view.cpu().numpy(), idx=idx.cpu().numpy(),
+                 cu_keep_dev=cu_keep_dev.cpu().numpy(), k_out=gu.to_host(k_out), v_out=gu.to_host(v_out))
+        gu.check_layer(wl, l, li, g, o)
