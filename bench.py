@@ -37,7 +37,8 @@ HBM_FALLBACK_GBS = 6800.0
 # workload, from an ncu capture of a two-layer launch of the same kernel (bench.py --layers 2 on
 # the workload), halved; keyed by the sha256 of the scoring kernels' sources (SCORE_SOURCES), so
 # a changed kernel reports null until it is captured again.  Rounded to 10 kB.
-SCORE_SOURCES = ('score_layers.cu', 'score_resident.cu', 'score_lse.cu', 'score_common.cuh', 'ckv_device.cuh')
+SCORE_SOURCES = ('score_layers.cu', 'score_layers.cuh', 'score_resident.cu', 'score_lse.cu', 'score_common.cuh',
+                 'ckv_device.cuh')
 SCORE_TRAFFIC = {
     "d43a4416edf56f3da424eefd7e9525afc76668f014115c0bd1ba6f2926be1e28": {
         "needle_l131072": 362_390_000,
@@ -415,10 +416,9 @@ def run_ours(args):
     # per layer: the scoring kernel, then the selection (pool, top-k, compaction and gather)
     lens = list(wl.seqlens)
     sel_per_layer = (1 if min(lens) <= SELECT_UNIT_LEN else 0) + (2 if max(lens) > SELECT_UNIT_LEN else 0)
-    if multi and args.lse:  # a single-pass scoring launch per layer, one selection launch per 32
-        launches_per_step = nl + -(-nl // 32)
-    elif multi:  # per 32 layers one scoring launch and one selection launch (the workloads here
-        # fit one launch's unit table; the selection's counter reset is a memset, not a kernel)
+    if multi:  # per 32 layers one scoring launch (two-pass, or single-pass with the lse given)
+        # and one selection launch (the workloads here fit one launch's unit table; the
+        # counter resets are memsets, not kernels)
         launches_per_step = 2 * -(-nl // 32)
     else:
         launches_per_step = (1 + sel_per_layer) * nl
@@ -456,13 +456,16 @@ def run_ours(args):
             ckv.ckv_score_window(cfg, l, batch, d["q"], d["k"], score_rows[l], w, stream=st)
 
     def score_all():
-        if multi and not args.lse:
+        if multi and args.lse:
+            ckv.ckv_score_windows_lse(cfg, score_ios, batch, ws, stream=stream)
+        elif multi:
             ckv.ckv_score_windows(cfg, score_ios, batch, ws, stream=stream)
         else:
             over_layers(score_one)
 
     if multi:
-        score_ios = [ckv.LayerIO(layer=l, q_win=d["q"], k=d["k"], scores=score_rows[l])
+        score_ios = [ckv.LayerIO(layer=l, q_win=d["q"], k=d["k"], scores=score_rows[l],
+                                 lse=d["lse"] if args.lse else None)
                      for l, d in enumerate(layers)]
 
     score_ms = stage(score_all)
@@ -492,8 +495,8 @@ def run_ours(args):
     for f in SCORE_SOURCES:
         digest.update(open(os.path.join(ROOT, "paper_2508_02401_gb300", "csrc", f), "rb").read())
     traffic = SCORE_TRAFFIC.get(digest.hexdigest(), {}).get(args.workload + ("+lse" if args.lse else ""))
-    kernel_desc = ("single-pass scoring kernel (ckv_score_window_lse), one launch per layer on "
-                   f"{sms} CTAs; per layer" if multi and args.lse else
+    kernel_desc = ("single-pass scoring kernel (ckv_score_windows_lse): every layer of the step "
+                   f"in one persistent launch on {cap or sms} CTAs; per layer" if multi and args.lse else
                    "two-pass scoring kernel (ckv_score_windows): every layer of the step in one "
                    f"persistent launch on {cap or sms} CTAs; per layer" if multi else
                    "scoring kernel (ckv_score_window), per layer, layers overlapped on "

@@ -53,7 +53,7 @@
 extern "C" {
 #endif
 
-#define CKV_ABI_VERSION 6
+#define CKV_ABI_VERSION 7
 
 #if defined(__GNUC__)
 #define CKV_API __attribute__((visibility("default")))
@@ -217,9 +217,8 @@ CKV_API ckv_status ckv_select_compact(const ckv_config* cfg, int32_t layer, cons
                                       float* pooled_out, void* workspace, size_t workspace_bytes,
                                       ckv_stream stream);
 
-/* One layer of a multi-layer call (ckv_score_windows, ckv_compress_layers,
- * ckv_compress_layers_lse).  The layers of a call share the config and the batch; each brings
- * its own buffers. */
+/* One layer of a multi-layer call (ckv_score_windows(_lse), ckv_compress_layers(_lse)).  The
+ * layers of a call share the config and the batch; each brings its own buffers. */
 typedef struct ckv_layer_io {
     int32_t layer;                 /* index into the config's head_mask and budgets */
     const void* q_win;             /* [S, w, H_q, 128] */
@@ -227,13 +226,13 @@ typedef struct ckv_layer_io {
     const void* v;                 /* ckv_compress_layers only; the same strides as k */
     int64_t tok_stride;            /* of k and v, in elements; 0 = packed */
     int64_t head_stride;
-    float* scores;                 /* ckv_score_windows: [n_sel, T] out, as ckv_score_window */
+    float* scores;                 /* ckv_score_windows(_lse): [n_sel, T] out, as ckv_score_window */
     int32_t* idx;                  /* ckv_compress_layers: outputs as for ckv_compress_layer */
     int32_t* cu_keep_dev;
     void* k_out;
     void* v_out;
     float* pooled_out;             /* may be NULL */
-    const float* lse;              /* ckv_compress_layers_lse: the window rows' lse, as for
+    const float* lse;              /* the _lse calls: the window rows' lse, as for
                                       ckv_score_window_lse (fp32, natural log, [H_q][S*w]) */
     int64_t lse_head_stride;       /* elements between heads; 0 = S*w */
 } ckv_layer_io;
@@ -253,6 +252,18 @@ CKV_API ckv_status ckv_score_windows(const ckv_config* cfg, int32_t n_layers,
                                      const ckv_layer_io* io, const ckv_batch* batch,
                                      void* workspace, size_t workspace_bytes, ckv_stream stream);
 
+/* Step 1 for several layers with every layer's window-row lse given (io[i].lse and
+ * io[i].lse_head_stride, as for ckv_score_window_lse): for each io[i], what
+ * ckv_score_window_lse(cfg, io[i].layer, ...) writes to io[i].scores.  Every layer's single
+ * pass over K runs in one persistent launch (one per 32 layers, and per 256 sequences); the CTAs
+ * take pieces of the (layer, head batch, sequence) units from a global counter, and no CTA
+ * waits for another.  CKV_ERR_INVALID_ARG for a NULL lse or a head stride below S*w; otherwise
+ * as ckv_score_windows. */
+CKV_API ckv_status ckv_score_windows_lse(const ckv_config* cfg, int32_t n_layers,
+                                         const ckv_layer_io* io, const ckv_batch* batch,
+                                         void* workspace, size_t workspace_bytes,
+                                         ckv_stream stream);
+
 /* Steps 1-4 for several layers: for each io[i], what ckv_compress_layer(cfg, io[i].layer, ...)
  * writes.  The layers are scored as by ckv_score_windows (into the workspace), then every
  * layer's selection runs in one launch (one per 32 layers) on the same stream, each (layer,
@@ -265,12 +276,12 @@ CKV_API ckv_status ckv_compress_layers(const ckv_config* cfg, int32_t n_layers,
                                        const ckv_layer_io* io, const ckv_batch* batch,
                                        void* workspace, size_t workspace_bytes, ckv_stream stream);
 
-/* Steps 1-4 for several layers with every layer's window-row lse given (io[i].lse, NEXT #3 of
- * the hot path: the lse a prefill attention kernel returns): for each io[i], what
- * ckv_compress_layer_lse(cfg, io[i].layer, ...) writes.  Each layer is scored in one pass over K
- * (one launch per layer, no exchange between CTAs), into the workspace, then every layer's
- * selection runs in one launch as in ckv_compress_layers.  The same workspace
- * (ckv_workspace_size_layers).  cfg->score_path is ignored. */
+/* Steps 1-4 for several layers with every layer's window-row lse given (io[i].lse: the lse a
+ * prefill attention kernel returns): for each io[i], what ckv_compress_layer_lse(cfg,
+ * io[i].layer, ...) writes.  The layers are scored as by ckv_score_windows_lse (one pass over
+ * K, into the workspace), then every layer's selection runs in one launch as in
+ * ckv_compress_layers.  The same workspace (ckv_workspace_size_layers).  cfg->score_path is
+ * ignored. */
 CKV_API ckv_status ckv_compress_layers_lse(const ckv_config* cfg, int32_t n_layers,
                                            const ckv_layer_io* io, const ckv_batch* batch,
                                            void* workspace, size_t workspace_bytes,

@@ -24,7 +24,7 @@ __all__ = [
     "SCORE_AUTO", "SCORE_RESIDENT", "SCORE_RELOAD", "ckv_score_window_lse",
     "ckv_compress_layer_lse", "ckv_semantic_retrieval_scores", "ckv_set_wait_limit_us",
     "new_workspace", "new_outputs", "LayerIO", "ckv_workspace_size_layers", "ckv_score_windows",
-    "ckv_compress_layers", "ckv_compress_layers_lse", "new_layers_workspace",
+    "ckv_compress_layers", "ckv_compress_layers_lse", "new_layers_workspace", "ckv_score_windows_lse",
 ]
 
 POOL_MAX, POOL_AVG = 0, 1
@@ -107,6 +107,7 @@ def load():
         "ckv_allocate_budgets": ([P, I32, I64, I32, I32, P], C.c_int),
         "ckv_workspace_size_layers": ([cfg, I32, P, bat, C.POINTER(SZ)], C.c_int),
         "ckv_score_windows": ([cfg, I32, P, bat, P, SZ, P], C.c_int),
+        "ckv_score_windows_lse": ([cfg, I32, P, bat, P, SZ, P], C.c_int),
         "ckv_compress_layers": ([cfg, I32, P, bat, P, SZ, P], C.c_int),
         "ckv_compress_layers_lse": ([cfg, I32, P, bat, P, SZ, P], C.c_int),
     }
@@ -359,7 +360,7 @@ class LayerIO:
     pooled_out: object = None
     tok_stride: int = 0
     head_stride: int = 0
-    lse: object = None          # ckv_compress_layers_lse: [H_q, S*w] fp32
+    lse: object = None          # the _lse calls: [H_q, S*w] fp32
     lse_head_stride: int = 0
 
 
@@ -397,6 +398,15 @@ def ckv_score_windows(cfg, ios, batch, workspace, stream=None):
            "ckv_score_windows")
 
 
+def ckv_score_windows_lse(cfg, ios, batch, workspace, stream=None):
+    """ckv_score_window_lse for every LayerIO of `ios` (their `scores`, each with its `lse`), in
+    one persistent single-pass launch."""
+    arr = _layer_ios(ios)
+    _check(load().ckv_score_windows_lse(cfg.ref, len(ios), arr, batch.ref, _ptr(workspace),
+                                        workspace.numel() * workspace.element_size(), _stream(stream)),
+           "ckv_score_windows_lse")
+
+
 def ckv_compress_layers(cfg, ios, batch, workspace, stream=None):
     """ckv_compress_layer for every LayerIO of `ios`: one scoring launch, then the selections."""
     arr = _layer_ios(ios)
@@ -407,7 +417,7 @@ def ckv_compress_layers(cfg, ios, batch, workspace, stream=None):
 
 def ckv_compress_layers_lse(cfg, ios, batch, workspace, stream=None):
     """ckv_compress_layer_lse for every LayerIO of `ios` (each with its `lse`): one single-pass
-    scoring launch per layer, then the selections in one launch."""
+    scoring launch over every layer, then the selections in one launch."""
     arr = _layer_ios(ios)
     _check(load().ckv_compress_layers_lse(cfg.ref, len(ios), arr, batch.ref, _ptr(workspace),
                                           workspace.numel() * workspace.element_size(), _stream(stream)),

@@ -527,6 +527,8 @@ struct LayerJob {
     const void* k;
     int64_t tok, head;
     float* scores;
+    const float* lse = nullptr;  // the window rows' lse: the single-pass kernel (all jobs or none)
+    int64_t lse_stride = 0;
 };
 
 // The items of one launch of the two-pass kernel: unit (lb, s), of tiles[s] key tiles, is
@@ -559,11 +561,12 @@ int launch_seq_chunk(int max_nb) {
     return std::max(1, std::min(kMaxLaunchSeqs, kMaxLaunchUnits / std::max(1, max_nb)));
 }
 
-// Enqueues the two-pass scoring of `jobs` (layers sharing the batch and the window): one
-// persistent launch per chunk of sequences (launch_seq_chunk) and per group of consecutive
-// layers whose tables fit the kernel's parameters.  Sequences of at most skip_le tokens are
-// skipped.  `sums`/`counters` hold the exchange of every unit of one launch (each launch
-// clears them first; launches are ordered on `stream`).
+// Enqueues the scoring of `jobs` (layers sharing the batch and the window) on the two-pass
+// kernel, or on the single-pass one where the jobs carry their lse: one persistent launch per
+// chunk of sequences (launch_seq_chunk) and per group of consecutive layers whose tables fit
+// the kernel's parameters.  Sequences of at most skip_le tokens are skipped.  `sums`/`counters`
+// hold the exchange of every unit of one launch and its item counter (each launch clears them
+// first; launches are ordered on `stream`).
 ckv_status enqueue_layers(const std::vector<LayerJob>& jobs, const ckv_batch* b, int T, void* sums,
                           int* counters, int* status, int skip_le, int max_ctas, cudaStream_t stream) {
     if (jobs.empty()) return CKV_OK;
@@ -624,6 +627,8 @@ ckv_status enqueue_layers(const std::vector<LayerJob>& jobs, const ckv_batch* b,
                 if ((st = make_k_map(&ly.tmap_k, J.k, J.pl->Hkv, T, J.tok, J.head))) return st;
                 if ((st = make_q_map(&ly.tmap_q, J.q_win, J.pl->Hq, S, w, w_pad))) return st;
                 ly.scores = J.scores;
+                ly.lse = J.lse;
+                ly.lse_stride = J.lse_stride;
                 const int sel_base = static_cast<int>(L.sel_heads.size());
                 for (int bt = 0; bt < J.pl->nb; ++bt) {
                     L.batch_layer.push_back(static_cast<int16_t>(j - j0));
@@ -649,6 +654,7 @@ ckv_status enqueue_layers(const std::vector<LayerJob>& jobs, const ckv_batch* b,
             L.grid = ctas;
             L.cu_hash = hash;
             L.softmax_scale = jobs[j0].pl->scale;
+            L.given_lse = jobs[j0].lse != nullptr;
             const cudaError_t e = launch_score_layers(L, stream);
             if (e != cudaSuccess) return cuda_fail(e, "launching the two-pass scoring kernel");
             j0 = j1;
@@ -1201,9 +1207,22 @@ ckv_status layer_jobs(const std::vector<Plan>& pls, const ckv_layer_io* io, int 
     return CKV_OK;
 }
 
-// ckv_compress_layers(_lse): the layers' scoring (one persistent two-pass launch, or with the
-// lse given one single-pass launch per layer) into the workspace, then every layer's selection
-// in one launch.
+// Each layer's given lse (io[i].lse, checked as for the one-layer call) into its scoring job.
+ckv_status layer_lse(const std::vector<Plan>& pls, const ckv_layer_io* io, const ckv_batch* b,
+                     std::vector<LayerJob>& jobs) {
+    ckv_status st;
+    for (size_t i = 0; i < jobs.size(); ++i) {
+        if (!io[i].lse) return fail(CKV_ERR_INVALID_ARG, "io[%zu].lse is NULL", i);
+        int64_t stride = io[i].lse_head_stride;
+        if ((st = check_lse(pls[i], b, io[i].lse, &stride))) return st;
+        jobs[i].lse = io[i].lse;
+        jobs[i].lse_stride = stride;
+    }
+    return CKV_OK;
+}
+
+// ckv_compress_layers(_lse): the layers' scoring (one persistent launch, two-pass or, with the
+// lse given, single-pass) into the workspace, then every layer's selection in one launch.
 ckv_status compress_layers_impl(const ckv_config* cfg, int32_t n_layers, const ckv_layer_io* io,
                                 const ckv_batch* batch, void* workspace, size_t workspace_bytes,
                                 ckv_stream stream, bool given_lse) {
@@ -1218,32 +1237,21 @@ ckv_status compress_layers_impl(const ckv_config* cfg, int32_t n_layers, const c
         return st;
     uint8_t* w8 = static_cast<uint8_t*>(workspace);
     if ((st = layer_jobs(pls, io, T, w8, lw, true, jobs, tok, head))) return st;
-    std::vector<int64_t> tks(n_layers, 0), lse_stride(n_layers, 0);
+    std::vector<int64_t> tks(n_layers, 0);
     int min_budget = INT_MAX;
     for (int i = 0; i < n_layers; ++i) {
         if ((st = check_kv(io[i].v, "v", T)) ||
             (st = check_select_outputs(batch, pls[i], io[i].idx, io[i].cu_keep_dev, io[i].k_out,
                                        io[i].v_out, io[i].pooled_out, &tks[i])))
             return st;
-        if (given_lse) {
-            if (!io[i].lse) return fail(CKV_ERR_INVALID_ARG, "io[%d].lse is NULL", i);
-            lse_stride[i] = io[i].lse_head_stride;
-            if ((st = check_lse(pls[i], batch, io[i].lse, &lse_stride[i]))) return st;
-        }
         min_budget = std::min(min_budget, pls[i].budget);
     }
+    if (given_lse && (st = layer_lse(pls, io, batch, jobs))) return st;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     // sequences that fit every layer's budget are kept whole by every selection
-    if (given_lse) {
-        for (int i = 0; i < n_layers; ++i)
-            if ((st = enqueue_score(pls[i], batch, T, jobs[i].q_win, jobs[i].k, tok[i], head[i],
-                                    jobs[i].scores, workspace, lw.sel, min_budget, s,
-                                    kMaxScoreItems, io[i].lse, lse_stride[i])))
-                return st;
-    } else if ((st = enqueue_layers(jobs, batch, T, w8 + lw.sums, reinterpret_cast<int*>(w8 + lw.counters),
-                                    reinterpret_cast<int*>(w8), min_budget, cfg->max_ctas, s))) {
+    if ((st = enqueue_layers(jobs, batch, T, w8 + lw.sums, reinterpret_cast<int*>(w8 + lw.counters),
+                             reinterpret_cast<int*>(w8), min_budget, cfg->max_ctas, s)))
         return st;
-    }
     // every layer's selection in one launch (one per 32 layers)
     static thread_local std::vector<SelectLaunch> sls;
     static thread_local std::vector<uint32_t*> keys;
@@ -1275,6 +1283,27 @@ ckv_status compress_layers_impl(const ckv_config* cfg, int32_t n_layers, const c
     return e == cudaSuccess ? CKV_OK : cuda_fail(e, "launching the multi-layer selection kernel");
 }
 
+// ckv_score_windows(_lse): every layer's scores into io[i].scores, in one persistent launch.
+ckv_status score_windows_impl(const ckv_config* cfg, int32_t n_layers, const ckv_layer_io* io,
+                              const ckv_batch* batch, void* workspace, size_t workspace_bytes,
+                              ckv_stream stream, bool given_lse) {
+    static thread_local std::vector<Plan> pls;
+    static thread_local std::vector<LayerJob> jobs;
+    static thread_local std::vector<int64_t> tok, head;
+    LayersWs lw;
+    int T = 0;
+    ckv_status st;
+    if ((st = prepare_layers(cfg, n_layers, io, batch, pls, &T, &lw)) ||
+        (st = check_layers_ws(lw, workspace, workspace_bytes, false)))
+        return st;
+    uint8_t* w8 = static_cast<uint8_t*>(workspace);
+    if ((st = layer_jobs(pls, io, T, w8, lw, false, jobs, tok, head))) return st;
+    if (given_lse && (st = layer_lse(pls, io, batch, jobs))) return st;
+    return enqueue_layers(jobs, batch, T, w8 + lw.sums, reinterpret_cast<int*>(w8 + lw.counters),
+                          reinterpret_cast<int*>(w8), -1, cfg->max_ctas,
+                          reinterpret_cast<cudaStream_t>(stream));
+}
+
 }  // namespace
 
 extern "C" {
@@ -1294,20 +1323,13 @@ ckv_status ckv_workspace_size_layers(const ckv_config* cfg, int32_t n_layers, co
 ckv_status ckv_score_windows(const ckv_config* cfg, int32_t n_layers, const ckv_layer_io* io,
                              const ckv_batch* batch, void* workspace, size_t workspace_bytes,
                              ckv_stream stream) {
-    static thread_local std::vector<Plan> pls;
-    static thread_local std::vector<LayerJob> jobs;
-    static thread_local std::vector<int64_t> tok, head;
-    LayersWs lw;
-    int T = 0;
-    ckv_status st;
-    if ((st = prepare_layers(cfg, n_layers, io, batch, pls, &T, &lw)) ||
-        (st = check_layers_ws(lw, workspace, workspace_bytes, false)))
-        return st;
-    uint8_t* w8 = static_cast<uint8_t*>(workspace);
-    if ((st = layer_jobs(pls, io, T, w8, lw, false, jobs, tok, head))) return st;
-    return enqueue_layers(jobs, batch, T, w8 + lw.sums, reinterpret_cast<int*>(w8 + lw.counters),
-                          reinterpret_cast<int*>(w8), -1, cfg->max_ctas,
-                          reinterpret_cast<cudaStream_t>(stream));
+    return score_windows_impl(cfg, n_layers, io, batch, workspace, workspace_bytes, stream, false);
+}
+
+ckv_status ckv_score_windows_lse(const ckv_config* cfg, int32_t n_layers, const ckv_layer_io* io,
+                                 const ckv_batch* batch, void* workspace, size_t workspace_bytes,
+                                 ckv_stream stream) {
+    return score_windows_impl(cfg, n_layers, io, batch, workspace, workspace_bytes, stream, true);
 }
 
 ckv_status ckv_compress_layers(const ckv_config* cfg, int32_t n_layers, const ckv_layer_io* io,

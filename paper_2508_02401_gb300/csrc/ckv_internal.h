@@ -94,6 +94,8 @@ struct LayersLayer {
     CUtensorMap tmap_k;
     CUtensorMap tmap_q;
     float* scores;       // [n_sel of the layer, T]
+    const float* lse;    // the window rows' lse, [H_q][lse_stride] (given_lse launches)
+    long long lse_stride;
 };
 struct LayersLaunch {
     std::vector<LayersLayer> layers;
@@ -110,6 +112,7 @@ struct LayersLaunch {
     int T, w, w_pad, n_cols, grid;
     uint32_t cu_hash;
     float softmax_scale;
+    bool given_lse;      // single pass with each layer's lse given (score_lse.cu)
 };
 cudaError_t launch_score_layers(const LayersLaunch& L, cudaStream_t stream);
 long long wait_limit_cycles();  // the current limit of a bounded wait, in SM clock cycles

@@ -49,7 +49,7 @@
 //                accumulator, then per key the sums of 2^(x - lse) over each head's rows.
 // Only the last tiles of a sequence (the window's own keys, the padding past its end) need a
 // per-column mask; the others take an unmasked path of packed fp32 pair instructions.
-#include "score_common.cuh"
+#include "score_layers.cuh"
 
 #include <string.h>
 
@@ -70,61 +70,6 @@ constexpr int kItemRing = 8;  // item indices posted by the producer (more than 
 // Largest |log2| of an item's column maximum: an item's sum is then below 2^1000 (at most
 // 2^10 keys), and the sum of up to 2^20 items stays below fp64's 2^1024.
 constexpr double kMaxLog2 = 990.0;
-
-struct alignas(128) LayersParams {
-    CUtensorMap tmap_k[kMaxLaunchLayers];  // K of each layer: {128, H_kv, T}, box {64, 1, 128}
-    CUtensorMap tmap_q[kMaxLaunchLayers];  // q_win of each layer: {128, H_q, S*w}, box {64, 1, W_PAD}
-    float* scores[kMaxLaunchLayers];       // [n_sel of the layer, T]
-    const int32_t* cu_seqlens;             // device [S+1] (checked against cu_hash)
-    double* sums;                          // [n_units][N]: per column, sum of 2^(x) over the unit
-    int* counters;                         // [n_units] arrivals, then the item counter; zero at launch
-    int* status;
-    int S, T, w, n_units, n_items, n_layers;
-    int seq0, S_all;                       // the launch's first sequence, sequences of the batch
-    uint32_t cu_hash;
-    float sl2;                             // softmax scale * log2(e)
-    long long wait_cycles;
-    int16_t batch_layer[kMaxLaunchBatches];   // layer (launch-local) of each flat head batch
-    int16_t batch_group[kMaxLaunchBatches];   // KV head
-    int16_t batch_first[kMaxLaunchBatches];   // score row (in its layer) of the batch's first head
-    int16_t batch_nheads[kMaxLaunchBatches];
-    int16_t batch_sel[kMaxLaunchBatches];     // index into sel_heads of the batch's first head
-    int16_t sel_heads[kMaxLaunchSel];         // query head of each head slot
-    int32_t seq_start[kMaxLaunchSeqs];        // of the launch's sequences seq0, seq0 + 1, ...
-    int32_t seq_len[kMaxLaunchSeqs];
-    LaunchUnit units[kMaxLaunchUnits + 1];    // units[n_units].item0 = n_items
-};
-static_assert(sizeof(LayersParams) <= 32000, "kernel parameters");
-
-struct Item {
-    int layer, batch, seq, unit, tile0, ntiles, start, len, nitems;
-};
-
-// Item i of the launch: the unit whose items hold i, and the (i - item0)-th of its m balanced
-// pieces of key tiles.
-__device__ __forceinline__ Item get_item(const LayersParams& p, int i) {
-    Item it;
-    int lo = 0, hi = p.n_units - 1;  // the last unit whose first item is at or before i
-    while (lo < hi) {
-        const int mid = (lo + hi + 1) >> 1;
-        if (p.units[mid].item0 <= i) lo = mid;
-        else hi = mid - 1;
-    }
-    const LaunchUnit U = p.units[lo];
-    const int m = p.units[lo + 1].item0 - U.item0;
-    const int k = i - U.item0;
-    it.unit = lo;
-    it.batch = U.lb;
-    it.layer = p.batch_layer[U.lb];
-    it.seq = U.seq;
-    it.start = p.seq_start[U.seq];
-    it.len = p.seq_len[U.seq];
-    it.nitems = m;
-    const int tiles = (it.len + kTileKeys - 1) / kTileKeys;
-    it.tile0 = k * tiles / m;
-    it.ntiles = (k + 1) * tiles / m - it.tile0;
-    return it;
-}
 
 template <int N>
 struct LayersSmem {
@@ -151,16 +96,6 @@ struct LayersSmem {
 };
 // dynamic + the kernel's static shared memory (under 6 KB) within the 227 KB a block may use
 static_assert(LayersSmem<64>::kDynamic + 6 * 1024 <= 232448, "shared memory, N = 64");
-
-// The index of the CTA's it-th item (-1 once its stream has ended), after the producer posted
-// it; false if the wait gave up.
-__device__ __forceinline__ bool wait_item(uint64_t* item_full, const int* items, int it, int* gi,
-                                          volatile int* abort, long long lim) {
-    const int k = it % kItemRing;
-    if (!mbar_wait(&item_full[k], (it / kItemRing) & 1, abort, lim)) return false;
-    *gi = items[k];
-    return true;
-}
 
 // End of a pass-1 item for one warpgroup of kCols columns: per column, the warp maximum by
 // redux and the sums rescaled to it, the warps' sums by recursive halving, then the four warps
@@ -451,7 +386,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
             bool ok = true;
             for (int it = 0; ok; ++it) {
                 int gi = -1;
-                if (!wait_item(item_full, items, it, &gi, abort, lim)) {
+                if (!wait_item<kItemRing>(item_full, items, it, &gi, abort, lim)) {
                     ok = false;
                     break;
                 }
@@ -503,7 +438,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
         bool ok = true;
         for (int it = 0;; ++it) {
             int gi = -1, good = 1;
-            if (lane == 0) good = wait_item(item_full, items, it, &gi, abort, lim) ? 1 : 0;
+            if (lane == 0) good = wait_item<kItemRing>(item_full, items, it, &gi, abort, lim) ? 1 : 0;
             gi = __shfl_sync(0xffffffffu, gi, 0);
             if (__shfl_sync(0xffffffffu, good, 0) == 0) {
                 ok = false;
@@ -554,7 +489,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
             bool ok = true;
             for (int it = 0; ok; ++it) {
                 int gi = -1;
-                if (!wait_item(item_full, items, it, &gi, abort, lim)) {
+                if (!wait_item<kItemRing>(item_full, items, it, &gi, abort, lim)) {
                     ok = false;
                     break;
                 }
@@ -634,7 +569,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_layers_kernel(const __grid_
         bool ok = true;
         for (int it = 0; ok; ++it) {
             int gi = -1, good = 1;
-            if (lane == 0) good = wait_item(item_full, items, it, &gi, abort, lim) ? 1 : 0;
+            if (lane == 0) good = wait_item<kItemRing>(item_full, items, it, &gi, abort, lim) ? 1 : 0;
             gi = __shfl_sync(0xffffffffu, gi, 0);
             if (__shfl_sync(0xffffffffu, good, 0) == 0) {
                 ok = false;
@@ -799,6 +734,8 @@ cudaError_t launch_score_layers(const LayersLaunch& L, cudaStream_t stream) {
         p.tmap_k[l] = L.layers[l].tmap_k;
         p.tmap_q[l] = L.layers[l].tmap_q;
         p.scores[l] = L.layers[l].scores;
+        p.lse[l] = L.layers[l].lse;
+        p.lse_stride[l] = L.layers[l].lse_stride;
     }
     p.cu_seqlens = L.cu_seqlens_dev;
     p.sums = L.sums;
@@ -829,11 +766,16 @@ cudaError_t launch_score_layers(const LayersLaunch& L, cudaStream_t stream) {
     }
     for (int u = 0; u <= nu; ++u) p.units[u] = L.units[u];
     if (p.n_items == 0) return cudaSuccess;
+    const int grid = std::min(L.grid, p.n_items);
+    if (L.given_lse) {  // one pass, no exchange: only the item counter
+        const cudaError_t e = cudaMemsetAsync(L.counters + nu, 0, sizeof(int), stream);
+        return e != cudaSuccess ? e : dispatch_lse_layers(p, L.n_cols, L.w_pad, grid, stream);
+    }
     // the exchange's accumulators, its arrival counters and the item counter start at zero
     cudaError_t e = cudaMemsetAsync(L.sums, 0, static_cast<size_t>(nu) * L.n_cols * sizeof(double), stream);
     if (e == cudaSuccess) e = cudaMemsetAsync(L.counters, 0, static_cast<size_t>(nu + 1) * sizeof(int), stream);
     if (e != cudaSuccess) return e;
-    return dispatch(p, L.n_cols, L.w_pad, std::min(L.grid, p.n_items), stream);
+    return dispatch(p, L.n_cols, L.w_pad, grid, stream);
 }
 
 }  // namespace ckv

@@ -32,6 +32,7 @@ def test_header_declares_the_boundary():
     for n in ("ckv_score_window", "ckv_pool", "ckv_select_topk", "ckv_gather_compact",
               "ckv_compress_layer", "ckv_workspace_size", "ckv_keep_lengths", "ckv_score_windows",
               "ckv_compress_layers", "ckv_compress_layers_lse", "ckv_workspace_size_layers",
+              "ckv_score_windows_lse",
               "ckv_read_device_status", "ckv_status_string"):
         assert n in names
 
@@ -48,7 +49,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 
 def test_version_and_status_strings(lib):
-    assert ckv.ckv_abi_version() == 6
+    assert ckv.ckv_abi_version() == 7
     assert ckv.ckv_status_string(0) == "CKV_OK"
     assert ckv.ckv_status_string(3) == "CKV_ERR_WORKSPACE"
 
@@ -229,6 +230,16 @@ def test_layers_argument_errors(lib):
     assert lib.ckv_compress_layers_lse(cfg.ref, 3, bad, b.ref, _P, 1 << 30, None) == 1   # misaligned
     bad = ckv._layer_ios(_ios(3, lse=_FakeT(_P), lse_head_stride=2 * 32 - 1))
     assert lib.ckv_compress_layers_lse(cfg.ref, 3, bad, b.ref, _P, 1 << 30, None) == 1   # stride < S*w
+    # the same checks in the scoring-only form
+    assert lib.ckv_score_windows_lse(cfg.ref, 3, arr, b.ref, _P, 1 << 30, None) == 1     # no lse
+    bad = ckv._layer_ios(_ios(3, lse=_FakeT(_P + 2)))
+    assert lib.ckv_score_windows_lse(cfg.ref, 3, bad, b.ref, _P, 1 << 30, None) == 1     # misaligned
+    bad = ckv._layer_ios(_ios(3, lse=_FakeT(_P), lse_head_stride=2 * 32 - 1))
+    assert lib.ckv_score_windows_lse(cfg.ref, 3, bad, b.ref, _P, 1 << 30, None) == 1     # stride < S*w
+    bad = ckv._layer_ios(_ios(2, lse=_FakeT(_P)) + _ios(1))
+    assert lib.ckv_score_windows_lse(cfg.ref, 3, bad, b.ref, _P, 1 << 30, None) == 1     # one missing
+    bad = ckv._layer_ios(_ios(3, lse=_FakeT(_P), scores=None))
+    assert lib.ckv_score_windows_lse(cfg.ref, 3, bad, b.ref, _P, 1 << 30, None) == 1     # no scores
 
 
 @pytest.mark.skipif(__import__("torch").cuda.is_available(), reason="CPU-only behaviour")
@@ -239,3 +250,4 @@ def test_valid_layers_call_without_a_gpu_reports_cuda_error(lib):
     assert lib.ckv_compress_layers(cfg.ref, 3, arr, b.ref, _P, 1 << 30, None) == 4
     arr = ckv._layer_ios(_ios(3, lse=_FakeT(_P)))
     assert lib.ckv_compress_layers_lse(cfg.ref, 3, arr, b.ref, _P, 1 << 30, None) == 4
+    assert lib.ckv_score_windows_lse(cfg.ref, 3, arr, b.ref, _P, 1 << 30, None) == 4

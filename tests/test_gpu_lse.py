@@ -179,19 +179,32 @@ def test_decode_attention_over_the_compacted_cache():
                 assert p_c[kept].sum() >= p_f[sorted(planted)].sum() * (1 - 1e-12)
 
 
-@pytest.mark.parametrize("case", [0, 1])
-def test_layers_call_with_given_lse(case):
-    """ckv_compress_layers_lse over several layers (one single-pass scoring launch per layer,
-    then every layer's selection in one launch) against the oracle's layer with the same lse,
-    layer by layer; canaries around every output.  Case 1: ragged lengths (some at most the
-    budget, one shorter than the window) and a padded lse head stride."""
-    if case == 0:
-        wl = _wl(num_layers=3, num_q_heads=32, num_kv_heads=8, seqlens=(6000, 900),
-                 budget_mean=200, outlier_channels=8)
-    else:
-        wl = _wl(num_layers=2, seqlens=(5, 31, 300, 2500, 40), budget_mean=64)
-    pad = 3 * case
-    cfg = ckv.Config.from_workload(wl)
+LAYERS_CASES = [
+    dict(num_layers=3, num_q_heads=32, num_kv_heads=8, seqlens=(6000, 900), budget_mean=200,
+         outlier_channels=8),
+    dict(num_layers=2, seqlens=(5, 31, 300, 2500, 40), budget_mean=64),
+    dict(num_layers=3, window=17, heads_per_group=3, num_q_heads=12, num_kv_heads=2,
+         seqlens=(900, 450), budget_uniform=False),
+    dict(num_layers=2, window=64, heads_per_group=2, seqlens=(1500, 700), budget_mean=100),
+    dict(num_layers=3, scope="layer", heads_per_layer=4, num_q_heads=32, num_kv_heads=8, window=8,
+         pool_kernel=5, pool_type="avg", seqlens=(4096, 333), budget_mean=128),
+]
+
+
+# max_ctas: 0 = every SM; 5 and 1 = a capped grid, where each CTA takes many items in turn
+# (the item ring wraps many times).
+@pytest.mark.parametrize("max_ctas", [0, 5, 1])
+@pytest.mark.parametrize("case", range(len(LAYERS_CASES)))
+def test_layers_call_with_given_lse(case, max_ctas):
+    """ckv_compress_layers_lse over several layers (every layer's single-pass scoring in one
+    launch, then every layer's selection in one launch), and ckv_score_windows_lse (the scoring
+    alone), against the oracle's layer with the same lse, layer by layer; canaries around every
+    output.  Case 1: ragged lengths (some at most the
+    budget, one shorter than the window) and a padded lse head stride; cases 2 and 3: 64-column
+    MMAs (three heads of 17 rows, two of 64); case 4: one selection per layer."""
+    wl = _wl(**LAYERS_CASES[case])
+    pad = 3 * (case % 2)
+    cfg = ckv.Config.from_workload(wl, max_ctas=max_ctas)
     batch = ckv.Batch(wl.cu_seqlens())
     T = batch.total_tokens
     ios, outs, refs = [], [], []
@@ -202,23 +215,30 @@ def test_layers_call_with_given_lse(case):
                                                int(wl.budgets()[l]), wl.window, wl.pool_kernel,
                                                0 if wl.pool_type == "max" else 1,
                                                0 if wl.head_order == "pool_then_sum" else 1,
-                                               scope=oracle.SCOPE_KV_HEAD, lse=lse64)))
+                                               scope=oracle.SCOPE_LAYER if wl.scope == "layer"
+                                               else oracle.SCOPE_KV_HEAD, lse=lse64)))
         lse32 = torch.from_numpy(lse64.astype(np.float32)).cuda()
         *gouts, cu_keep = gu.guarded_outputs(cfg, l, batch)
         gpl = gu.Guarded((cfg.num_vectors, T), torch.float32, float("nan"))
+        _, n_sel = ckv.ckv_keep_lengths(cfg, l, batch)
+        gsc = gu.Guarded((n_sel, T), torch.float32, float("nan"))
         ios.append(ckv.LayerIO(layer=l, q_win=gu.to_dev(li.q_win), k=gu.to_dev(li.k), v=gu.to_dev(li.v),
-                               idx=gouts[0].view, cu_keep_dev=gouts[1].view, k_out=gouts[2].view,
-                               v_out=gouts[3].view, pooled_out=gpl.view, lse=lse32,
+                               scores=gsc.view, idx=gouts[0].view, cu_keep_dev=gouts[1].view,
+                               k_out=gouts[2].view, v_out=gouts[3].view, pooled_out=gpl.view, lse=lse32,
                                lse_head_stride=lse64.shape[1]))
-        outs.append((gouts, gpl, cu_keep))
+        outs.append((gouts, gpl, gsc, cu_keep))
     ws = ckv.new_layers_workspace(cfg, ios, batch)
     ckv.ckv_compress_layers_lse(cfg, ios, batch, ws)
     code, detail = ckv.ckv_read_device_status(ws)
     assert code == 0, (code, detail)
-    for l, ((gouts, gpl, cu_keep), (li, o)) in enumerate(zip(outs, refs)):
-        for g_ in [gpl, *gouts]:
+    ckv.ckv_score_windows_lse(cfg, ios, batch, ws)  # the scoring alone, into io[i].scores
+    code, detail = ckv.ckv_read_device_status(ws)
+    assert code == 0, (code, detail)
+    for l, ((gouts, gpl, gsc, cu_keep), (li, o)) in enumerate(zip(outs, refs)):
+        for g_ in [gpl, gsc, *gouts]:
             g_.check()
         idx, cu_keep_dev, k_out, v_out = (g_.view for g_ in gouts)
-        g = dict(cfg=cfg, cu_keep=cu_keep, pooled=gpl.view.cpu().numpy(), idx=idx.cpu().numpy(),
-                 cu_keep_dev=cu_keep_dev.cpu().numpy(), k_out=gu.to_host(k_out), v_out=gu.to_host(v_out))
+        g = dict(cfg=cfg, cu_keep=cu_keep, scores=gsc.view.cpu().numpy(), pooled=gpl.view.cpu().numpy(),
+                 idx=idx.cpu().numpy(), cu_keep_dev=cu_keep_dev.cpu().numpy(), k_out=gu.to_host(k_out),
+                 v_out=gu.to_host(v_out))
         gu.check_layer(wl, l, li, g, o)
