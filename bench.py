@@ -40,9 +40,12 @@ HBM_FALLBACK_GBS = 6800.0
 SCORE_SOURCES = ('score_layers.cu', 'score_layers.cuh', 'score_resident.cu', 'score_lse.cu', 'score_common.cuh',
                  'ckv_device.cuh')
 SCORE_TRAFFIC = {
-    "d43a4416edf56f3da424eefd7e9525afc76668f014115c0bd1ba6f2926be1e28": {
-        "needle_l131072": 362_390_000,
-        "ragged_qwen7b": 221_270_000,
+    "5ad12ac092a0df5be55fdc9dc5b5c0bf3e276024a6e80def08d2a75911978807": {
+        "needle_l131072": 358_670_000,
+        "ragged_qwen7b": 222_220_000,
+        "needle_l131072+lse": 272_310_000,
+        "ragged_qwen7b+lse": 174_450_000,
+        "llama8b_l32768+lse": 69_110_000,
     },
 }
 # Sequences up to this many tokens are selected by one block per (sequence, KV head)
