@@ -1096,6 +1096,23 @@ __device__ __forceinline__ void cp_async16(float* dst, const float* src) {
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
 }
 
+// Asks L2 to fetch bytes [p, p + n) (16-byte aligned, n a multiple of 16): a hint that moves
+// nothing into the SM, so that a later copy of the same bytes finds them in L2.
+__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t n) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(n) : "memory");
+}
+
+// prefetch_l2 of positions [a, b) of a score row, clamped to [0, P) and trimmed to whole
+// 16-byte groups.
+__device__ __forceinline__ void prefetch_row_l2(const float* row, int a, int b, int P) {
+    a = max(a, 0);
+    b = min(b, P);
+    if (b <= a) return;
+    const uintptr_t s = (reinterpret_cast<uintptr_t>(row + a) + 15) & ~static_cast<uintptr_t>(15);
+    const uintptr_t e = reinterpret_cast<uintptr_t>(row + b) & ~static_cast<uintptr_t>(15);
+    if (e > s) prefetch_l2(reinterpret_cast<const void*>(s), static_cast<uint32_t>(e - s));
+}
+
 // Issues the copies that stage score rows ra .. ra+nr-1 for the n positions from `base` (row i
 // at st + i*words, the layout above; zero outside [0, P)) and commits them as one group.  Every
 // row start (scores + r*T + t0) is 16-byte aligned and base is a multiple of 4 (checked by the
@@ -1215,6 +1232,7 @@ constexpr int kLs16Words = kLsChunk + 32;                        // a row of the
 constexpr int kLsList = kLsWords;                                // kept positions gathered at once
 static_assert(kLsList >= kLsChunk, "a chunk's kept positions fit the list");
 constexpr int kLsSmem = kLsWords * 4;
+constexpr int kLsAhead = 2;     // score-row chunks asked into L2 ahead of the one being copied in
 constexpr int kLsCand = 2048;   // keys sharing the k-th key's first digit gathered in shared memory
 constexpr int kLsTies = 256;    // keys equal to the k-th key ranked by position in shared memory
 constexpr int kSelMaxLayers = 32;
@@ -1304,6 +1322,12 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
         else if (piped)
             stage_rows_issue<NT, kLsStageLoads>(st, words, p.scores, p.T, u.t0, r0, nr, 0, half,
                                                 min(kLsChunk, Pn), u.P);
+        // The chunks after the next are asked into L2 kLsAhead chunks ahead of their copy, so
+        // that the copies overlapped with pooling find them there.
+        const float* srow = p.scores + static_cast<size_t>(r0 + tid) * p.T + u.t0;
+        if (piped && tid < nr)
+            for (int d = 1; d <= kLsAhead; ++d)
+                prefetch_row_l2(srow, d * kLsChunk - 4, (d + 1) * kLsChunk + 4, Pn);
         __syncthreads();
         uint32_t lo = 0;  // the lowest first digit counted (see below)
         for (int base = 0, c = 0; base < Pn; base += kLsChunk, ++c) {
@@ -1320,6 +1344,10 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
                     else
                         stage_rows_issue<NT, kLsStageLoads>(nxt_st, words, p.scores, p.T, u.t0, r0, nr,
                                                             base + kLsChunk, half, nn, u.P);
+                    if (tid < nr) {
+                        const int a = base + (1 + kLsAhead) * kLsChunk;
+                        prefetch_row_l2(srow, a - 4, a + kLsChunk + 4, Pn);
+                    }
                     cp_async_wait_group<1>();
                 } else {
                     cp_async_wait_group<0>();
@@ -1705,8 +1733,13 @@ cudaError_t launch_select_layers(const SelectLaunch* Ls, uint32_t* const* keys, 
     for (int l0 = 0; l0 < n_layers; l0 += kSelMaxLayers) {
         const int nl = std::min(kSelMaxLayers, n_layers - l0);
         memset(&P, 0, sizeof P);
+        // The layers with the largest budgets (the longest gathers) first: the CTAs take units
+        // in order, so the last ones taken are the shortest.
+        int order[kSelMaxLayers];
+        for (int i = 0; i < nl; ++i) order[i] = l0 + i;
+        std::stable_sort(order, order + nl, [&](int a, int b) { return Ls[a].budget > Ls[b].budget; });
         for (int i = 0; i < nl; ++i) {
-            const SelectLaunch& L = Ls[l0 + i];
+            const SelectLaunch& L = Ls[order[i]];
             SelectParams& p = P.layer[i];
             p.scores = L.scores;
             p.pooled = L.pooled;
@@ -1734,7 +1767,7 @@ cudaError_t launch_select_layers(const SelectLaunch* Ls, uint32_t* const* keys, 
             p.write_pooled = L.write_pooled;
             p.cu_hash = L.cu_hash;
             for (int g = 0; g <= L.n_vec; ++g) p.group_first[g] = static_cast<int16_t>(L.group_first[g]);
-            P.cands[i] = reinterpret_cast<uint2*>(keys[l0 + i]);
+            P.cands[i] = reinterpret_cast<uint2*>(keys[order[i]]);
         }
         P.n_layers = nl;
         P.units_per_layer = Ls[l0].S * Ls[l0].n_vec * (Ls[l0].n_vec == 1 ? Ls[l0].Hkv : 1);
