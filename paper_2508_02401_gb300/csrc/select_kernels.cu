@@ -1209,11 +1209,12 @@ __device__ __forceinline__ void pool_any16(const float* st, int t, int nvalid, i
 // the CTAs take units from a global counter, and one CTA does a unit whole, streaming over its
 // candidate positions in chunks of kLsChunk (so that no length is too long and little sits in
 // shared memory):
-//  (A) pools the chunk (the next chunk's score rows copied in meanwhile), counts the first
-//      digits of its order-preserving keys, and appends the keys that can still be kept, with
-//      their positions, to the unit's candidate list in a scratch row: once the chunks so far
-//      hold k keys, the first digit of their k-th largest bounds the unit's k-th largest from
-//      below, and keys under it are neither counted nor listed;
+//  (A) pools the chunk (the next chunk's score rows copied in meanwhile) and appends the keys
+//      that can still be kept, with their positions, to the unit's candidate list in a scratch
+//      row: the first digits of the order-preserving keys are counted until the chunks so far
+//      hold k keys; the first digit of their k-th largest then bounds the unit's k-th largest
+//      from below, and later keys under it are not listed (the digits of later candidates are
+//      counted from the list before (B));
 //  (B) finds the k-th largest key from the counts (the first digit) and two more digits (11 and
 //      10 bits) counted over the candidates with the digits so far: gathered into shared memory
 //      when at most kLsCand share the first digit, else read from the list; the tie cutoff
@@ -1330,6 +1331,7 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
                 prefetch_row_l2(srow, d * kLsChunk - 4, (d + 1) * kLsChunk + 4, Pn);
         __syncthreads();
         uint32_t lo = 0;  // the lowest first digit counted (see below)
+        int n_hist = -1;  // candidates from n_hist on are not counted in hist (see below)
         for (int base = 0, c = 0; base < Pn; base += kLsChunk, ++c) {
             const int n = min(kLsChunk, Pn - base);
             const int jb = tid * PER, nvalid = n - jb;
@@ -1381,12 +1383,15 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
                         if (i < nvalid) pooled[base + jb + i] = acc[i];
                 }
             }
-            add_runs<PER, kHistShift>(hist, key, nvalid, lo);
+            // Once the bound is set, a chunk is not counted here: (B) adds the first digits of
+            // its candidates (its only keys that can be kept) from the list instead.
+            if (lo == 0) add_runs<PER, kHistShift>(hist, key, nvalid, lo);
+            else if (n_hist < 0) n_hist = n_cand;
             if (lo == 0 && k > 0) {
                 // The k-th largest key of the chunks so far bounds the unit's k-th largest from
-                // below: later chunks count only first digits at or above its digit (the counts
-                // that the threshold search reads stay exact, and the bulk of small scores costs
-                // no atomic), and only keys there can be kept.
+                // below: in later chunks only keys whose first digit is at or above its digit can
+                // be kept, and the counts at or above it, which the threshold search reads, stay
+                // exact when only those keys are counted.
                 __syncthreads();
                 find_digit<NT>(hist, k, scratch, &s_digit, &s_above);
                 lo = static_cast<uint32_t>(s_digit);  // 0 while fewer than k keys are counted
@@ -1412,6 +1417,10 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
         int pos_cut = -1;
         if (k > 0) {
             if (tid == 0) s_cut = INT_MAX;
+            if (n_hist >= 0) {  // the first digits of the candidates of the chunks not counted in (A)
+                for (int c = n_hist + tid; c < n_cand; c += NT) atomicAdd(&hist[__ldcg(cands + c).x >> kHistShift], 1);
+                __syncthreads();
+            }
             find_digit<NT>(hist, k, scratch, &s_digit, &s_above);
             const uint32_t d1 = static_cast<uint32_t>(s_digit);
             int r = k - s_above, n_eq = hist[d1];
