@@ -699,8 +699,8 @@ def _cpu_baseline(wl, host_layers, seconds):
     dt = time.perf_counter() - t0
     return {"value": round(done * wl.total_tokens / dt, 2), "unit": UNIT, "cores": cores,
             "kind": "oracle", "sample": f"{done} whole-layer calls (layers in order), {dt:.1f} s, "
-                                        f"OpenMP over (sequence, KV head) units on "
-                                        f"{oracle.threads(0)} host threads"}
+                                        f"OpenMP over (sequence, selection) units: {cores} of "
+                                        f"{oracle.threads(0)} host threads busy"}
 
 
 def run_reference(args):
@@ -744,8 +744,8 @@ def run_reference(args):
             "config": _workload_config(wl, world),
             "cpu_baseline": {"value": round(value, 2), "unit": UNIT, "cores": cores, "kind": "oracle",
                              "sample": f"one whole layer per step (layers 0..{n_distinct - 1} in turn), "
-                                       f"OpenMP over (sequence, KV head) units on "
-                                       f"{oracle.threads(0)} host threads"},
+                                       f"OpenMP over (sequence, selection) units: {cores} of "
+                                       f"{oracle.threads(0)} host threads busy"},
             "e2e": {"value": round(value, 2), "unit": UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
