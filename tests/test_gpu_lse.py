@@ -188,6 +188,12 @@ LAYERS_CASES = [
     dict(num_layers=2, window=64, heads_per_group=2, seqlens=(1500, 700), budget_mean=100),
     dict(num_layers=3, scope="layer", heads_per_layer=4, num_q_heads=32, num_kv_heads=8, window=8,
          pool_kernel=5, pool_type="avg", seqlens=(4096, 333), budget_mean=128),
+    # more layers than one launch takes (two scoring and two selection launches)
+    dict(num_layers=34, num_q_heads=4, num_kv_heads=2, heads_per_group=1, seqlens=(600, 130),
+         budget_mean=48),
+    # more sequences than one launch's tables hold (the scoring in chunks of sequences)
+    dict(num_layers=2, num_q_heads=2, num_kv_heads=1, heads_per_group=1, window=16,
+         seqlens=tuple(100 + (i * 37) % 90 for i in range(600)), budget_mean=48),
 ]
 
 
@@ -201,7 +207,8 @@ def test_layers_call_with_given_lse(case, max_ctas):
     alone), against the oracle's layer with the same lse, layer by layer; canaries around every
     output.  Case 1: ragged lengths (some at most the
     budget, one shorter than the window) and a padded lse head stride; cases 2 and 3: 64-column
-    MMAs (three heads of 17 rows, two of 64); case 4: one selection per layer."""
+    MMAs (three heads of 17 rows, two of 64); case 4: one selection per layer; cases 5 and 6:
+    more layers, or more sequences, than one launch takes."""
     wl = _wl(**LAYERS_CASES[case])
     pad = 3 * (case % 2)
     cfg = ckv.Config.from_workload(wl, max_ctas=max_ctas)
