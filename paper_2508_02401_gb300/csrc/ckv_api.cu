@@ -504,6 +504,23 @@ ckv_status make_k_map(CUtensorMap* map, const void* k, int Hkv, int T, int64_t t
     return CKV_OK;
 }
 
+// A [n_sel, T] fp32 score buffer as 16-float lines {16, score_map_lines}, a box of
+// kScoreMapBoxLines lines, 64-byte swizzled (the multi-layer selection's TMA stage).  The last
+// line may run up to 60 bytes past the buffer: its owner keeps 64 bytes of padding there.
+ckv_status make_score_map(CUtensorMap* map, const float* scores, int n_sel, int T) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return fail(CKV_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
+    const cuuint64_t dims[2] = {16, static_cast<cuuint64_t>(score_map_lines(n_sel, T))};
+    const cuuint64_t strides[1] = {64};
+    const cuuint32_t box[2] = {16, static_cast<cuuint32_t>(kScoreMapBoxLines)};
+    const cuuint32_t estr[2] = {1, 1};
+    const CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(scores), dims, strides,
+                          box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B,
+                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(CKV_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", static_cast<int>(r));
+    return CKV_OK;
+}
+
 }  // namespace
 
 int device_sm_count() {
@@ -1166,8 +1183,8 @@ ckv_status prepare_layers(const ckv_config* cfg, int32_t n_layers, const ckv_lay
     lw->scores.assign(n_layers, 0);
     lw->keys.assign(n_layers, 0);
     for (int i = 0; i < n_layers; ++i) {
-        lw->scores[i] = off;
-        off = round_up(off + static_cast<size_t>(pls[i].n_sel) * *T * sizeof(float), kWsAlign);
+        lw->scores[i] = off;  // 64 bytes of padding after: the last line of the scores' tensor map
+        off = round_up(off + static_cast<size_t>(pls[i].n_sel) * *T * sizeof(float) + 64, kWsAlign);
         lw->keys[i] = off;  // the selection's (key, position) candidates, [H_kv, key stride]
         off = round_up(off + static_cast<size_t>(pls[i].Hkv) * select_key_stride(*T, b->num_seqs) *
                                  2 * sizeof(uint32_t), kWsAlign);
@@ -1255,12 +1272,16 @@ ckv_status compress_layers_impl(const ckv_config* cfg, int32_t n_layers, const c
     // every layer's selection in one launch (one per 32 layers)
     static thread_local std::vector<SelectLaunch> sls;
     static thread_local std::vector<uint32_t*> keys;
+    static thread_local std::vector<CUtensorMap> maps;
     sls.assign(n_layers, SelectLaunch{});
     keys.assign(n_layers, nullptr);
+    maps.resize(n_layers);
     for (int i = 0; i < n_layers; ++i) {
         SelectLaunch& L = sls[i];
         L = select_launch(pls[i], batch, T, static_cast<int>(tks[i]), pls[i].budget, cfg, workspace, &lw.sel);
         L.scores = jobs[i].scores;
+        if ((st = make_score_map(&maps[i], jobs[i].scores, pls[i].n_sel, T))) return st;
+        L.score_map = &maps[i];
         L.pooled = io[i].pooled_out;
         L.write_pooled = io[i].pooled_out != nullptr;
         L.from_scores = 1;

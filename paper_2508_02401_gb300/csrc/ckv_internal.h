@@ -146,7 +146,14 @@ struct SelectLaunch {
     int64_t tok_stride, head_stride;
     void* k_out;
     void* v_out;
+    // The multi-layer selection: the scores viewed as 16-float lines (score_map_lines), with
+    // 64 bytes of readable padding after the last row; nullptr: no such view.
+    const CUtensorMap* score_map;
 };
+// Lines of 16 floats of a [n_sel, T] score buffer as the multi-layer selection's tensor map
+// views it: every element, the last line's tail running into the padding after the buffer.
+inline long long score_map_lines(int n_sel, int T) { return (static_cast<long long>(n_sel) * T + 15) / 16; }
+constexpr int kScoreMapBoxLines = 176;  // lines per TMA box of the score map
 int select_chunks(int max_len);
 size_t select_hist_ints();
 int select_chunk_positions();

@@ -1077,25 +1077,25 @@ __global__ void __launch_bounds__(256) gather_kernel(const __grid_constant__ Gat
     *dst = __ldg(src);
 }
 
-// ------------------------------------------------------------------ vectorised stage
-// A stage of one score row for chunk positions base-4 .. base+n+3 (element e = position
-// base-4+e) in 16-byte groups: group c of the row sits at group c ^ ((c >> 3) & 3), an XOR of
-// its low two bits that keeps every group whole (so that it is copied by one 16-byte cp.async)
-// and makes the six 16-byte reads of a thread's 24 elements (below) hit distinct bank groups
-// in every quarter-warp.
-__device__ __forceinline__ int sidx_sw(int e) {
-    const int c = e >> 2;
-    return ((c ^ ((c >> 3) & 3)) << 2) | (e & 3);
-}
+// ------------------------------------------------------------------ TMA stage
+// A stage row of one score row for one chunk, loaded by TMA from the score buffer viewed as
+// 16-float lines (64 bytes): kLsTmaBoxes boxes of kScoreMapBoxLines lines from the line holding
+// position base-4 on, so element e of the row sits at position base-4-d+e, d = the offset of
+// position base-4 in its line.  The TMA writes each 64-byte line with the 64-byte swizzle: the
+// 16-byte chunk bits 4-5 of a byte offset XOR its bits 7-8 (rows 1024-byte aligned).  For the
+// pooling's reads of 16 elements per thread that places the 16-byte reads of every
+// quarter-warp in distinct bank groups.
+constexpr int kLsTmaBoxes = 3;
+constexpr int kLsTmaRow = kLsTmaBoxes * kScoreMapBoxLines * 16;   // floats per stage row
+static_assert(kLsTmaRow >= 12 + 8192 + 8, "a chunk, its halo and the line offset fit a stage row");
+static_assert((kLsTmaRow * 4) % 1024 == 0 && (kScoreMapBoxLines * 64) % 1024 == 0, "1024-byte aligned boxes");
+__device__ __forceinline__ int sw64(int byte) { return byte ^ (((byte >> 7) & 3) << 4); }
+
 __device__ __forceinline__ float fmax3(float a, float b, float c) {
     float d;
     asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
     return d;
 }
-__device__ __forceinline__ void cp_async16(float* dst, const float* src) {
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
-}
-
 // Asks L2 to fetch bytes [p, p + n) (16-byte aligned, n a multiple of 16): a hint that moves
 // nothing into the SM, so that a later copy of the same bytes finds them in L2.
 __device__ __forceinline__ void prefetch_l2(const void* p, uint32_t n) {
@@ -1113,52 +1113,50 @@ __device__ __forceinline__ void prefetch_row_l2(const float* row, int a, int b, 
     if (e > s) prefetch_l2(reinterpret_cast<const void*>(s), static_cast<uint32_t>(e - s));
 }
 
-// Issues the copies that stage score rows ra .. ra+nr-1 for the n positions from `base` (row i
-// at st + i*words, the layout above; zero outside [0, P)) and commits them as one group.  Every
-// row start (scores + r*T + t0) is 16-byte aligned and base is a multiple of 4 (checked by the
-// caller), so a group inside [0, P) is one 16-byte copy; the at most two groups that straddle
-// 0 or P are read element by element.
-template <int NT>
-__device__ __forceinline__ void stage_rows_issue16(float* st, int words, const float* scores, size_t T,
-                                                   int t0, int ra, int nr, int base, int n, int P) {
-    const int ng = (n + 8 + 3) >> 2;  // groups of the n positions and 4 on each side
+// Issues, from one thread, the TMA loads that stage score rows ra .. ra+nr-1 of the chunk at
+// `base` (row i at st + i*words), completion on `bar`.  Earlier generic-proxy writes to the
+// stage (the previous unit's kept list) are ordered before the loads by the proxy fence.
+__device__ __forceinline__ void stage_rows_tma(float* st, int words, const CUtensorMap* map, uint64_t* bar,
+                                               size_t T, int t0, int ra, int nr, int base) {
+    fence_proxy_async_smem();
+    mbar_arrive_expect_tx(bar, static_cast<uint32_t>(nr * kLsTmaRow * 4));
     for (int i = 0; i < nr; ++i) {
-        const float* row = scores + static_cast<size_t>(ra + i) * T + t0;
-        float* dst = st + i * words;
-        for (int g = threadIdx.x; g < ng; g += NT) {
-            const int u0 = base - 4 + 4 * g;  // position of the group's first element
-            float* d = dst + sidx_sw(4 * g);
-            if (u0 >= 0 && u0 + 4 <= P) {
-                cp_async16(d, row + u0);
-            } else {
-                float4 v;
-                v.x = (u0 >= 0 && u0 < P) ? __ldg(row + u0) : 0.f;
-                v.y = (u0 + 1 >= 0 && u0 + 1 < P) ? __ldg(row + u0 + 1) : 0.f;
-                v.z = (u0 + 2 >= 0 && u0 + 2 < P) ? __ldg(row + u0 + 2) : 0.f;
-                v.w = (u0 + 3 >= 0 && u0 + 3 < P) ? __ldg(row + u0 + 3) : 0.f;
-                *reinterpret_cast<float4*>(d) = v;
-            }
-        }
+        const long long f = static_cast<long long>(ra + i) * static_cast<long long>(T) + t0 + base - 4;
+        const int line = f >= 0 ? static_cast<int>(f >> 4) : -1;  // f >= -4; line -1 reads zeros
+        for (int b = 0; b < kLsTmaBoxes; ++b)
+            tma_load_2d(st + i * words + b * kScoreMapBoxLines * 16, map, bar, 0, line + b * kScoreMapBoxLines);
     }
-    cp_async_commit();
 }
 
-// Pools the PER = 16 outputs of thread t (positions base+16t .. base+16t+15) from one row
-// staged by stage_rows_issue16: its 24 elements 16t .. 16t+23 in six 16-byte reads; output i
-// covers elements 16t+i+4-HALF .. 16t+i+4+HALF.  The same arithmetic, in the same order, as
-// pool_window.
+// The line offset d of row ra+i's chunk at `base` in its stage row (stage_rows_tma).
+__device__ __forceinline__ int stage_offset(size_t T, int t0, int r, int base) {
+    const long long f = static_cast<long long>(r) * static_cast<long long>(T) + t0 + base - 4;
+    return f >= 0 ? static_cast<int>(f & 15) : static_cast<int>(f + 16);
+}
+
+// Pools the PER = 16 outputs of thread t (positions base+16t .. base+16t+15) from one stage
+// row: its 24 elements d+16t .. d+16t+23 (positions base-4+16t ..) in six 16-byte reads
+// (d a multiple of 4), those outside [0, P) taken as zero; output i covers elements
+// 16t+i+4-HALF .. 16t+i+4+HALF.  The same arithmetic, in the same order, as pool_window.
 template <int HALF, int PER>
-__device__ __forceinline__ void pool_window16(const float* st, int t, int nvalid, bool is_max, float kf,
-                                              float (&acc)[PER]) {
+__device__ __forceinline__ void pool_window_tma(const float* row, int d, int t, int nvalid, bool is_max,
+                                                float kf, int pos0, int P, float (&acc)[PER]) {
     static_assert(PER == 16 && HALF >= 0 && HALF <= 4, "window");
     float w[24];
+    const char* rb = reinterpret_cast<const char*>(row);
 #pragma unroll
     for (int q = 0; q < 6; ++q) {
-        const float4 x = *reinterpret_cast<const float4*>(st + sidx_sw(16 * t + 4 * q));
+        const float4 x = *reinterpret_cast<const float4*>(rb + sw64(4 * (d + 16 * t + 4 * q)));
         w[4 * q] = x.x;
         w[4 * q + 1] = x.y;
         w[4 * q + 2] = x.z;
         w[4 * q + 3] = x.w;
+    }
+    const int p0 = pos0 + 16 * t;  // position of w[0]
+    if (p0 < 0 || p0 + 24 > P) {
+#pragma unroll
+        for (int j = 0; j < 24; ++j)
+            if (p0 + j < 0 || p0 + j >= P) w[j] = 0.f;
     }
     if (is_max) {
         // maxima of three neighbours, shared by the windows that contain them (a maximum is
@@ -1186,7 +1184,7 @@ __device__ __forceinline__ void pool_window16(const float* st, int t, int nvalid
             if (i < nvalid) {
                 float m = w[i + 4 - HALF];
 #pragma unroll
-                for (int d = 1; d <= 2 * HALF; ++d) m += w[i + 4 - HALF + d];
+                for (int dd = 1; dd <= 2 * HALF; ++dd) m += w[i + 4 - HALF + dd];
                 acc[i] += m / kf;  // IEEE division, as in pool_kernel
             }
         }
@@ -1194,14 +1192,14 @@ __device__ __forceinline__ void pool_window16(const float* st, int t, int nvalid
 }
 
 template <int PER>
-__device__ __forceinline__ void pool_any16(const float* st, int t, int nvalid, int half, bool is_max,
-                                           float kf, float (&acc)[PER]) {
+__device__ __forceinline__ void pool_any_tma(const float* row, int d, int t, int nvalid, int half, bool is_max,
+                                             float kf, int pos0, int P, float (&acc)[PER]) {
     if (nvalid <= 0) return;
-    if (half == 3) pool_window16<3, PER>(st, t, nvalid, is_max, kf, acc);
-    else if (half == 2) pool_window16<2, PER>(st, t, nvalid, is_max, kf, acc);
-    else if (half == 1) pool_window16<1, PER>(st, t, nvalid, is_max, kf, acc);
-    else if (half == 0) pool_window16<0, PER>(st, t, nvalid, is_max, kf, acc);
-    else pool_window16<4, PER>(st, t, nvalid, is_max, kf, acc);
+    if (half == 3) pool_window_tma<3, PER>(row, d, t, nvalid, is_max, kf, pos0, P, acc);
+    else if (half == 2) pool_window_tma<2, PER>(row, d, t, nvalid, is_max, kf, pos0, P, acc);
+    else if (half == 1) pool_window_tma<1, PER>(row, d, t, nvalid, is_max, kf, pos0, P, acc);
+    else if (half == 0) pool_window_tma<0, PER>(row, d, t, nvalid, is_max, kf, pos0, P, acc);
+    else pool_window_tma<4, PER>(row, d, t, nvalid, is_max, kf, pos0, P, acc);
 }
 
 // ------------------------------------------------------------------ many layers at once
@@ -1228,8 +1226,10 @@ constexpr int kLsPer = 16;
 constexpr int kLsChunk = kLsThreads * kLsPer;                    // 8192 positions
 constexpr int kLsStageFloats = kLsChunk + 2 * kMaxHalo;
 constexpr int kLsStageLoads = (kLsStageFloats + kLsThreads - 1) / kLsThreads;
-constexpr int kLsWords = 4 * stage_words(kLsStageFloats);        // four score rows at once
-constexpr int kLs16Words = kLsChunk + 32;                        // a row of the 16-byte stage
+// four score rows at once in the padded layout, or two buffers of two TMA stage rows (plus the
+// slack that aligns them to 1024 bytes)
+constexpr int kLsWords = 4 * stage_words(kLsStageFloats) > 4 * kLsTmaRow + 256 ? 4 * stage_words(kLsStageFloats)
+                                                                               : 4 * kLsTmaRow + 256;
 constexpr int kLsList = kLsWords;                                // kept positions gathered at once
 static_assert(kLsList >= kLsChunk, "a chunk's kept positions fit the list");
 constexpr int kLsSmem = kLsWords * 4;
@@ -1239,6 +1239,8 @@ constexpr int kLsTies = 256;    // keys equal to the k-th key ranked by position
 constexpr int kSelMaxLayers = 32;
 
 struct SelectLayersParams {
+    CUtensorMap score_map[kSelMaxLayers];  // each layer's scores as 16-float lines (map_mask)
+    uint32_t map_mask;                     // bit i: score_map[i] is set
     SelectParams layer[kSelMaxLayers];
     uint2* cands[kSelMaxLayers];     // per layer [n_vec, key_stride]: (key, position) candidates
     int* next_unit;                  // work counter, zero at launch
@@ -1254,8 +1256,18 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
     __shared__ int s_digit, s_above, s_cut, s_cnt, s_unit;
     __shared__ uint32_t s_thr;
     __shared__ uint2 cand[kLsCand];
+    __shared__ uint64_t tbar[2];  // TMA stage buffers: the loads of a chunk complete
+    __shared__ int s_abort;
     constexpr int NT = kLsThreads, PER = kLsPer;
     const int tid = threadIdx.x;
+    float* const sta = reinterpret_cast<float*>((reinterpret_cast<uintptr_t>(st) + 1023) & ~static_cast<uintptr_t>(1023));
+    uint32_t tph = 0;  // bit b: parity of the next completion of tbar[b]
+    if (tid == 0) {
+        mbar_init(&tbar[0], 1);
+        mbar_init(&tbar[1], 1);
+        s_abort = 0;
+        fence_mbar_init();
+    }
     if (blockIdx.x == 0 && tid == 0) {
         const SelectParams& p0 = P.layer[0];
         if (seqlens_hash(p0.cu_seqlens, p0.S) != p0.cu_hash) record_error(p0.status, kDevBadSeqlens, 240);
@@ -1263,6 +1275,7 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
     const int n_units = P.n_layers * P.units_per_layer;
     for (;;) {
         if (tid == 0) s_unit = atomicAdd(P.next_unit, 1);
+        fence_proxy_async_smem();  // this thread's writes to the stage before the unit's TMA loads
         __syncthreads();
         const int gu = s_unit;
         __syncthreads();
@@ -1309,18 +1322,19 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
         // chunk's rows are copied in while this chunk is pooled (two buffers of nr rows).
         const int half = p.pool_kernel >> 1;
         const int r0 = p.group_first[u.g], nr = p.group_first[u.g + 1] - r0;
-        // 16-byte staging when every row of the unit starts 16-byte aligned and the pooling
-        // window fits a thread's 24 staged elements; else 4-byte copies in the padded layout
+        // TMA staging when every row of the unit starts 16-byte aligned and the pooling window
+        // fits a thread's 24 staged elements; else 4-byte copies in the padded layout
         bool aligned = true;
         for (int i = 0; i < nr; ++i)
             aligned = aligned && ((reinterpret_cast<uintptr_t>(p.scores + static_cast<size_t>(r0 + i) * p.T + u.t0) & 15u) == 0);
-        const bool v16 = p.from_scores && p.head_order == 0 && half <= 4 && aligned &&
-                         2 * nr * kLs16Words <= kLsWords;
-        const int words = v16 ? kLs16Words : stage_words(kLsChunk + 2 * half);
-        const bool piped = v16 || (p.from_scores && p.head_order == 0 && 2 * nr * words + PER <= kLsWords);
-        if (v16)
-            stage_rows_issue16<NT>(st, words, p.scores, p.T, u.t0, r0, nr, 0, min(kLsChunk, Pn), u.P);
-        else if (piped)
+        const bool tma = ((P.map_mask >> li) & 1u) && p.from_scores && p.head_order == 0 && half <= 4 &&
+                         aligned && 2 * nr * kLsTmaRow + 256 <= kLsWords;
+        const int words = tma ? kLsTmaRow : stage_words(kLsChunk + 2 * half);
+        const bool piped = tma || (p.from_scores && p.head_order == 0 && 2 * nr * words + PER <= kLsWords);
+        float* const stg = tma ? sta : st;
+        if (tma) {
+            if (tid == 0) stage_rows_tma(stg, words, &P.score_map[li], &tbar[0], p.T, u.t0, r0, nr, 0);
+        } else if (piped)
             stage_rows_issue<NT, kLsStageLoads>(st, words, p.scores, p.T, u.t0, r0, nr, 0, half,
                                                 min(kLsChunk, Pn), u.P);
         // The chunks after the next are asked into L2 kLsAhead chunks ahead of their copy, so
@@ -1337,30 +1351,50 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
             const int jb = tid * PER, nvalid = n - jb;
             float acc[PER];
             if (piped) {
-                const float* cur = st + (c & 1) * nr * words;
-                if (base + kLsChunk < Pn) {
-                    float* nxt_st = st + ((c + 1) & 1) * nr * words;
+                const float* cur = stg + (c & 1) * nr * words;
+                const bool more = base + kLsChunk < Pn;
+                if (more) {
+                    float* nxt_st = stg + ((c + 1) & 1) * nr * words;
                     const int nn = min(kLsChunk, Pn - base - kLsChunk);
-                    if (v16)
-                        stage_rows_issue16<NT>(nxt_st, words, p.scores, p.T, u.t0, r0, nr, base + kLsChunk, nn, u.P);
-                    else
+                    if (tma) {
+                        if (tid == 0)
+                            stage_rows_tma(nxt_st, words, &P.score_map[li], &tbar[(c + 1) & 1], p.T, u.t0, r0, nr,
+                                           base + kLsChunk);
+                    } else {
                         stage_rows_issue<NT, kLsStageLoads>(nxt_st, words, p.scores, p.T, u.t0, r0, nr,
                                                             base + kLsChunk, half, nn, u.P);
+                    }
                     if (tid < nr) {
                         const int a = base + (1 + kLsAhead) * kLsChunk;
                         prefetch_row_l2(srow, a - 4, a + kLsChunk + 4, Pn);
                     }
-                    cp_async_wait_group<1>();
-                } else {
+                    if (!tma) cp_async_wait_group<1>();
+                } else if (!tma) {
                     cp_async_wait_group<0>();
                 }
-                __syncthreads();
+                if (tma) {  // this chunk's loads have landed (a bounded wait)
+                    const int b = c & 1;
+                    const bool ok = mbar_wait(&tbar[b], (tph >> b) & 1u, &s_abort);
+                    tph ^= 1u << b;
+                    if (__syncthreads_or(ok ? 0 : 1)) {
+                        // give up: report, let the loads still in flight land, leave
+                        if (tid == 0) {
+                            record_error(p.status, kDevTimeout, 250);
+                            volatile int never = 0;
+                            mbar_wait(&tbar[b], ((tph >> b) & 1u) ^ 1u, &never);
+                            if (more) mbar_wait(&tbar[b ^ 1], (tph >> (b ^ 1)) & 1u, &never);
+                        }
+                        return;
+                    }
+                } else {
+                    __syncthreads();
+                }
 #pragma unroll
                 for (int i = 0; i < PER; ++i) acc[i] = 0.f;
                 for (int i = 0; i < nr; ++i) {
-                    if (v16)
-                        pool_any16<PER>(cur + i * words, tid, nvalid, half, p.pool_type == 0,
-                                        static_cast<float>(p.pool_kernel), acc);
+                    if (tma)
+                        pool_any_tma<PER>(cur + i * words, stage_offset(p.T, u.t0, r0 + i, base), tid, nvalid, half,
+                                          p.pool_type == 0, static_cast<float>(p.pool_kernel), base - 4, Pn, acc);
                     else
                         pool_any<PER>(cur + i * words, jb, nvalid, half, p.pool_type == 0,
                                       static_cast<float>(p.pool_kernel), acc);
@@ -1777,6 +1811,10 @@ cudaError_t launch_select_layers(const SelectLaunch* Ls, uint32_t* const* keys, 
             p.cu_hash = L.cu_hash;
             for (int g = 0; g <= L.n_vec; ++g) p.group_first[g] = static_cast<int16_t>(L.group_first[g]);
             P.cands[i] = reinterpret_cast<uint2*>(keys[order[i]]);
+            if (L.score_map) {
+                P.score_map[i] = *L.score_map;
+                P.map_mask |= 1u << i;
+            }
         }
         P.n_layers = nl;
         P.units_per_layer = Ls[l0].S * Ls[l0].n_vec * (Ls[l0].n_vec == 1 ? Ls[l0].Hkv : 1);
