@@ -1087,7 +1087,7 @@ __global__ void __launch_bounds__(256) gather_kernel(const __grid_constant__ Gat
 // quarter-warp in distinct bank groups.
 constexpr int kLsTmaBoxes = 3;
 constexpr int kLsTmaRow = kLsTmaBoxes * kScoreMapBoxLines * 16;   // floats per stage row
-static_assert(kLsTmaRow >= 12 + 8192 + 8, "a chunk, its halo and the line offset fit a stage row");
+static_assert(kLsTmaRow >= 15 + 8192 + 8 + 3, "a chunk, its halo, the line offset and a shifted read fit a stage row");
 static_assert((kLsTmaRow * 4) % 1024 == 0 && (kScoreMapBoxLines * 64) % 1024 == 0, "1024-byte aligned boxes");
 __device__ __forceinline__ int sw64(int byte) { return byte ^ (((byte >> 7) & 3) << 4); }
 
@@ -1135,23 +1135,29 @@ __device__ __forceinline__ int stage_offset(size_t T, int t0, int r, int base) {
 }
 
 // Pools the PER = 16 outputs of thread t (positions base+16t .. base+16t+15) from one stage
-// row: its 24 elements d+16t .. d+16t+23 (positions base-4+16t ..) in six 16-byte reads
-// (d a multiple of 4), those outside [0, P) taken as zero; output i covers elements
-// 16t+i+4-HALF .. 16t+i+4+HALF.  The same arithmetic, in the same order, as pool_window.
-template <int HALF, int PER>
+// row: its 24 elements d+16t .. d+16t+23 (positions base-4+16t ..), d = 4a + SHIFT, in six
+// 16-byte reads from element 4a+16t on (seven when SHIFT > 0), those outside [0, P) taken as
+// zero; output i covers elements 16t+i+4-HALF .. 16t+i+4+HALF.  The same arithmetic, in the
+// same order, as pool_window.
+template <int HALF, int SHIFT, int PER>
 __device__ __forceinline__ void pool_window_tma(const float* row, int d, int t, int nvalid, bool is_max,
                                                 float kf, int pos0, int P, float (&acc)[PER]) {
-    static_assert(PER == 16 && HALF >= 0 && HALF <= 4, "window");
-    float w[24];
+    static_assert(PER == 16 && HALF >= 0 && HALF <= 4 && SHIFT >= 0 && SHIFT < 4, "window");
+    constexpr int kReads = SHIFT > 0 ? 7 : 6;
+    float r[4 * kReads];
     const char* rb = reinterpret_cast<const char*>(row);
+    const int e0 = (d & ~3) + 16 * t;
 #pragma unroll
-    for (int q = 0; q < 6; ++q) {
-        const float4 x = *reinterpret_cast<const float4*>(rb + sw64(4 * (d + 16 * t + 4 * q)));
-        w[4 * q] = x.x;
-        w[4 * q + 1] = x.y;
-        w[4 * q + 2] = x.z;
-        w[4 * q + 3] = x.w;
+    for (int q = 0; q < kReads; ++q) {
+        const float4 x = *reinterpret_cast<const float4*>(rb + sw64(4 * (e0 + 4 * q)));
+        r[4 * q] = x.x;
+        r[4 * q + 1] = x.y;
+        r[4 * q + 2] = x.z;
+        r[4 * q + 3] = x.w;
     }
+    float w[24];
+#pragma unroll
+    for (int j = 0; j < 24; ++j) w[j] = r[SHIFT + j];
     const int p0 = pos0 + 16 * t;  // position of w[0]
     if (p0 < 0 || p0 + 24 > P) {
 #pragma unroll
@@ -1191,15 +1197,25 @@ __device__ __forceinline__ void pool_window_tma(const float* row, int d, int t, 
     }
 }
 
+template <int HALF, int PER>
+__device__ __forceinline__ void pool_shift_tma(const float* row, int d, int t, int nvalid, bool is_max,
+                                               float kf, int pos0, int P, float (&acc)[PER]) {
+    const int shift = d & 3;  // the same for every thread of the block
+    if (shift == 0) pool_window_tma<HALF, 0, PER>(row, d, t, nvalid, is_max, kf, pos0, P, acc);
+    else if (shift == 1) pool_window_tma<HALF, 1, PER>(row, d, t, nvalid, is_max, kf, pos0, P, acc);
+    else if (shift == 2) pool_window_tma<HALF, 2, PER>(row, d, t, nvalid, is_max, kf, pos0, P, acc);
+    else pool_window_tma<HALF, 3, PER>(row, d, t, nvalid, is_max, kf, pos0, P, acc);
+}
+
 template <int PER>
 __device__ __forceinline__ void pool_any_tma(const float* row, int d, int t, int nvalid, int half, bool is_max,
                                              float kf, int pos0, int P, float (&acc)[PER]) {
     if (nvalid <= 0) return;
-    if (half == 3) pool_window_tma<3, PER>(row, d, t, nvalid, is_max, kf, pos0, P, acc);
-    else if (half == 2) pool_window_tma<2, PER>(row, d, t, nvalid, is_max, kf, pos0, P, acc);
-    else if (half == 1) pool_window_tma<1, PER>(row, d, t, nvalid, is_max, kf, pos0, P, acc);
-    else if (half == 0) pool_window_tma<0, PER>(row, d, t, nvalid, is_max, kf, pos0, P, acc);
-    else pool_window_tma<4, PER>(row, d, t, nvalid, is_max, kf, pos0, P, acc);
+    if (half == 3) pool_shift_tma<3, PER>(row, d, t, nvalid, is_max, kf, pos0, P, acc);
+    else if (half == 2) pool_shift_tma<2, PER>(row, d, t, nvalid, is_max, kf, pos0, P, acc);
+    else if (half == 1) pool_shift_tma<1, PER>(row, d, t, nvalid, is_max, kf, pos0, P, acc);
+    else if (half == 0) pool_shift_tma<0, PER>(row, d, t, nvalid, is_max, kf, pos0, P, acc);
+    else pool_shift_tma<4, PER>(row, d, t, nvalid, is_max, kf, pos0, P, acc);
 }
 
 // ------------------------------------------------------------------ many layers at once
@@ -1322,13 +1338,10 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
         // chunk's rows are copied in while this chunk is pooled (two buffers of nr rows).
         const int half = p.pool_kernel >> 1;
         const int r0 = p.group_first[u.g], nr = p.group_first[u.g + 1] - r0;
-        // TMA staging when every row of the unit starts 16-byte aligned and the pooling window
-        // fits a thread's 24 staged elements; else 4-byte copies in the padded layout
-        bool aligned = true;
-        for (int i = 0; i < nr; ++i)
-            aligned = aligned && ((reinterpret_cast<uintptr_t>(p.scores + static_cast<size_t>(r0 + i) * p.T + u.t0) & 15u) == 0);
+        // TMA staging when the pooling window fits a thread's 24 staged elements and two
+        // buffers of the unit's rows fit the stage; else 4-byte copies in the padded layout
         const bool tma = ((P.map_mask >> li) & 1u) && p.from_scores && p.head_order == 0 && half <= 4 &&
-                         aligned && 2 * nr * kLsTmaRow + 256 <= kLsWords;
+                         2 * nr * kLsTmaRow + 256 <= kLsWords;
         const int words = tma ? kLsTmaRow : stage_words(kLsChunk + 2 * half);
         const bool piped = tma || (p.from_scores && p.head_order == 0 && 2 * nr * words + PER <= kLsWords);
         float* const stg = tma ? sta : st;
