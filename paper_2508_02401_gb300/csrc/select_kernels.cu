@@ -1338,10 +1338,12 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
         // chunk's rows are copied in while this chunk is pooled (two buffers of nr rows).
         const int half = p.pool_kernel >> 1;
         const int r0 = p.group_first[u.g], nr = p.group_first[u.g + 1] - r0;
-        // TMA staging when the pooling window fits a thread's 24 staged elements and two
-        // buffers of the unit's rows fit the stage; else 4-byte copies in the padded layout
+        // TMA staging when the pooling window fits a thread's 24 staged elements and the unit's
+        // rows fit the stage, in two buffers (the next chunk loaded while this one is pooled)
+        // or else one; otherwise 4-byte copies in the padded layout
         const bool tma = ((P.map_mask >> li) & 1u) && p.from_scores && p.head_order == 0 && half <= 4 &&
-                         2 * nr * kLsTmaRow + 256 <= kLsWords;
+                         nr * kLsTmaRow + 256 <= kLsWords;
+        const int nb = tma && 2 * nr * kLsTmaRow + 256 > kLsWords ? 1 : 2;  // stage buffers
         const int words = tma ? kLsTmaRow : stage_words(kLsChunk + 2 * half);
         const bool piped = tma || (p.from_scores && p.head_order == 0 && 2 * nr * words + PER <= kLsWords);
         float* const stg = tma ? sta : st;
@@ -1364,9 +1366,13 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
             const int jb = tid * PER, nvalid = n - jb;
             float acc[PER];
             if (piped) {
-                const float* cur = stg + (c & 1) * nr * words;
+                const int bi = nb == 2 ? (c & 1) : 0;
+                const float* cur = stg + bi * nr * words;
                 const bool more = base + kLsChunk < Pn;
-                if (more) {
+                // one buffer: chunk c > 0 is loaded now, its buffer freed by the last chunk's barrier
+                if (nb == 1 && c > 0 && tid == 0)
+                    stage_rows_tma(stg, words, &P.score_map[li], &tbar[0], p.T, u.t0, r0, nr, base);
+                if (more && nb == 2) {
                     float* nxt_st = stg + ((c + 1) & 1) * nr * words;
                     const int nn = min(kLsChunk, Pn - base - kLsChunk);
                     if (tma) {
@@ -1377,16 +1383,16 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
                         stage_rows_issue<NT, kLsStageLoads>(nxt_st, words, p.scores, p.T, u.t0, r0, nr,
                                                             base + kLsChunk, half, nn, u.P);
                     }
-                    if (tid < nr) {
-                        const int a = base + (1 + kLsAhead) * kLsChunk;
-                        prefetch_row_l2(srow, a - 4, a + kLsChunk + 4, Pn);
-                    }
                     if (!tma) cp_async_wait_group<1>();
                 } else if (!tma) {
                     cp_async_wait_group<0>();
                 }
+                if (more && tid < nr) {
+                    const int a = base + (1 + kLsAhead) * kLsChunk;
+                    prefetch_row_l2(srow, a - 4, a + kLsChunk + 4, Pn);
+                }
                 if (tma) {  // this chunk's loads have landed (a bounded wait)
-                    const int b = c & 1;
+                    const int b = bi;
                     const bool ok = mbar_wait(&tbar[b], (tph >> b) & 1u, &s_abort);
                     tph ^= 1u << b;
                     if (__syncthreads_or(ok ? 0 : 1)) {
@@ -1395,7 +1401,7 @@ __global__ void __launch_bounds__(kLsThreads, 1) select_layers_kernel(const __gr
                             record_error(p.status, kDevTimeout, 250);
                             volatile int never = 0;
                             mbar_wait(&tbar[b], ((tph >> b) & 1u) ^ 1u, &never);
-                            if (more) mbar_wait(&tbar[b ^ 1], (tph >> (b ^ 1)) & 1u, &never);
+                            if (more && nb == 2) mbar_wait(&tbar[b ^ 1], (tph >> (b ^ 1)) & 1u, &never);
                         }
                         return;
                     }

@@ -44,6 +44,12 @@ CASES = [
          budget_mean=48),
     dict(num_layers=2, num_q_heads=2, num_kv_heads=1, heads_per_group=1, window=16,
          seqlens=tuple(100 + (i * 37) % 90 for i in range(600)), budget_mean=48),
+    # three or four score rows per selection over several 8192-position chunks: the selection
+    # stages them in one buffer
+    dict(num_layers=2, num_q_heads=12, num_kv_heads=2, heads_per_group=3, seqlens=(20000, 9001),
+         budget_mean=200),
+    dict(num_layers=2, scope="layer", heads_per_layer=4, num_q_heads=32, num_kv_heads=8, window=8,
+         pool_kernel=5, pool_type="avg", seqlens=(17000, 333), budget_mean=300),
 ]
 
 
