@@ -40,12 +40,13 @@ HBM_FALLBACK_GBS = 6800.0
 SCORE_SOURCES = ('score_layers.cu', 'score_layers.cuh', 'score_resident.cu', 'score_lse.cu', 'score_common.cuh',
                  'ckv_device.cuh')
 SCORE_TRAFFIC = {
-    "5ad12ac092a0df5be55fdc9dc5b5c0bf3e276024a6e80def08d2a75911978807": {
-        "needle_l131072": 358_670_000,
-        "ragged_qwen7b": 222_220_000,
+    "2420f73d42000877d15e1e55b8936cf6b89b5eaa3076715573ec3b7a0d634c9a": {
+        "needle_l131072": 362_430_000,
+        "llama8b_l32768": 73_830_000,
+        "ragged_qwen7b": 223_730_000,
         "needle_l131072+lse": 272_310_000,
-        "ragged_qwen7b+lse": 174_450_000,
-        "llama8b_l32768+lse": 69_110_000,
+        "llama8b_l32768+lse": 69_040_000,
+        "ragged_qwen7b+lse": 174_490_000,
     },
 }
 # Sequences up to this many tokens are selected by one block per (sequence, KV head)
