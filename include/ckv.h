@@ -270,8 +270,9 @@ CKV_API ckv_status ckv_score_windows_lse(const ckv_config* cfg, int32_t n_layers
  * sequence, selection) by one CTA that keeps a list of the keys that can still be kept in the
  * workspace.  Sequences with L_s at most every layer's budget are copied whole without being
  * scored.  The workspace (ckv_workspace_size_layers) holds, per layer, the scores [n_sel, T]
- * fp32 and the selection's lists [H_kv, T + 4 S] of 8-byte entries, and per unit of the
- * scoring launch N fp64 row sums and a counter. */
+ * fp32 (and 64 bytes after them, which the selection's TMA view of them may read) and the
+ * selection's lists [H_kv, T + 4 S] of 8-byte entries, and per unit of the scoring launch N
+ * fp64 row sums and a counter. */
 CKV_API ckv_status ckv_compress_layers(const ckv_config* cfg, int32_t n_layers,
                                        const ckv_layer_io* io, const ckv_batch* batch,
                                        void* workspace, size_t workspace_bytes, ckv_stream stream);
